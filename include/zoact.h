@@ -1,0 +1,215 @@
+/*
+ * zoact.h -- C ABI of libzoact, the GB300 (sm_103a) hot path of one ZO-Act step.
+ *
+ * ZO-Act (arXiv 2607.01125) fine-tunes a frozen model forward-only: every
+ * adapted linear layer keeps its weight W frozen and learns only a small
+ * coefficient matrix on a frozen activation basis (Section 3):
+ *
+ *     y = W x + (C + sigma * eps * Z)(U^T x),      sigma in {+1, -1}
+ *
+ * with U [d_in, r] the top-r right singular vectors of the layer's calibration
+ * activations (Algorithm 1), C [d_out, r] the coefficients (the paper's B,
+ * transposed; zero at initialisation) and Z [d_out, r] ~ N(0, I) a perturbation
+ * regenerated from a seed (never stored).  One ZO step (Algorithm 2, in
+ * two-sided form) runs the forward pass at +eps and -eps, forms
+ * a = (L+ - L-) / (2 eps) and updates C with Adam on g = a * Z.
+ *
+ * Conventions for every call:
+ *  - All tensor pointers are DEVICE pointers owned by the caller; the library
+ *    never frees caller memory and keeps no pointer after a call returns.
+ *  - Every call is asynchronous on the context's stream; none synchronises with
+ *    the host except zoact_get_device_status and zoact_destroy.
+ *  - Errors in arguments (shape, dtype, alignment, NULL) are found on the host
+ *    before any launch and returned as a negative status; nothing is launched
+ *    then.  Errors found on the device (non-finite loss, a bounded wait that
+ *    timed out) are recorded in the context's device status word.
+ *  - Row-major layouts throughout.  "Stacked" activations hold 2T rows: rows
+ *    [0, T) belong to sigma = +1 and rows [T, 2T) to sigma = -1.
+ *  - Z for a layer is a pure function of (seed, layer_id, query): element
+ *    e = i * r + j of Z is word (e & 3) of Philox4x32-10 with
+ *    key = (seed_lo, seed_hi) and counter = (e >> 2, layer_id, query_lo, query_hi),
+ *    turned into normals by Box-Muller on word pairs (w0, w1), (w2, w3) with
+ *    u1 = ((w_a >> 8) + 1) 2^-24, u2 = (w_b >> 8) 2^-24, z_a = sqrt(-2 ln u1) cos(2 pi u2),
+ *    z_b = sqrt(-2 ln u1) sin(2 pi u2).  The forward pass and the optimizer step
+ *    must be given the same (seed, query) to see the same Z.
+ */
+#ifndef ZOACT_H_
+#define ZOACT_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ---- */
+#define ZOACT_OK               0
+#define ZOACT_ERR_INVALID_ARG (-1)  /* bad shape, dtype, NULL or misaligned pointer */
+#define ZOACT_ERR_UNSUPPORTED (-2)  /* valid request this build does not implement */
+#define ZOACT_ERR_CUDA        (-3)  /* a CUDA runtime call failed */
+#define ZOACT_ERR_NONFINITE   (-4)  /* device: a loss or the estimator scalar was NaN/Inf */
+#define ZOACT_ERR_TIMEOUT     (-5)  /* device: a bounded wait in a kernel gave up */
+#define ZOACT_ERR_NOMEM       (-6)  /* the context could not allocate its scratch */
+
+/* ---- storage types ---- */
+#define ZOACT_DT_FP32       0
+#define ZOACT_DT_BF16       1
+#define ZOACT_DT_FP16       2
+#define ZOACT_DT_INT4_G128  3  /* weights only: see zoact_layer.W */
+
+/* ---- activations fused into the pair-forward epilogue ---- */
+#define ZOACT_ACT_NONE  0
+#define ZOACT_ACT_RELU  1
+#define ZOACT_ACT_GELU  2  /* exact: 0.5 x (1 + erf(x / sqrt 2)) */
+
+typedef struct zoact_ctx zoact_ctx;
+
+/* One adapted linear layer (Section 3: W_eff = W + V_r B).  All pointers are
+ * caller-owned device memory that must stay valid until the work using them
+ * has run on the stream.                                                     */
+typedef struct zoact_layer {
+  int32_t d_in;        /* input width  (the paper's m) */
+  int32_t d_out;       /* output width (the paper's n) */
+  int32_t r;           /* basis rank, 1 <= r <= 32 in this build */
+  int32_t wtype;       /* ZOACT_DT_* of W */
+  const void* W;       /* frozen weight [d_out, d_in] row-major.  INT4_G128:
+                          [d_out, d_in/2] bytes, element k in byte k/2, low nibble
+                          for even k, 4-bit two's complement q in [-8, 7]      */
+  const void* w_scales;/* INT4_G128 only: [d_out, d_in/128] fp16 scales, w = q*s;
+                          NULL otherwise                                        */
+  const float* U;      /* frozen basis [d_in, r] fp32 (the paper's V_r)        */
+  const float* C;      /* coefficients [d_out, r] fp32 (the paper's B^T)       */
+  uint32_t layer_id;   /* Philox stream id of this layer's Z; unique per layer */
+} zoact_layer;
+
+/* A block of coefficients inside the flat C/m/v arenas given to the
+ * optimizer: elements [offset, offset + d_out*r) hold one layer's [d_out, r]. */
+typedef struct zoact_coeff_block {
+  int64_t offset;      /* element offset into the arenas; multiple of 4 */
+  int32_t d_out;
+  int32_t r;
+  uint32_t layer_id;
+  uint32_t reserved;
+} zoact_coeff_block;
+
+/* Create a context on CUDA device `device` that launches on `stream`
+ * (a cudaStream_t; NULL = the legacy default stream).  The context owns only
+ * scratch (projection buffer, reduction partials, basis workspace, the device
+ * status word); it allocates device memory here and may grow its scratch on
+ * later calls.  Returns ZOACT_OK and sets *out, or a negative status.          */
+int zoact_create(zoact_ctx** out, int device, void* stream);
+
+/* Destroy a context: synchronises its stream, frees its scratch.  NULL is a no-op. */
+int zoact_destroy(zoact_ctx* ctx);
+
+/* Change the stream later launches go to (cudaStream_t).                       */
+int zoact_set_stream(zoact_ctx* ctx, void* stream);
+
+/* Human-readable text of a status code (static storage).                       */
+const char* zoact_status_string(int status);
+
+/* Synchronise the stream and read the device status word (ZOACT_OK or the
+ * first device-side error recorded since the last reset).  reset != 0 clears it. */
+int zoact_get_device_status(zoact_ctx* ctx, int* status, int reset);
+
+/* Number of SMs of the context's device (host query, no launch).               */
+int zoact_device_sm_count(zoact_ctx* ctx, int* sm_count);
+
+/* Number of kernels this context has launched since it was created (a host
+ * counter, incremented at every launch; no synchronisation).                   */
+int zoact_get_launch_count(zoact_ctx* ctx, int64_t* count);
+
+/* ---- Z: the perturbation generator (Section 3, Z ~ N(0, I)) ----
+ * Writes the first n elements of the (seed, layer_id, query) stream:
+ * z_out[e] (fp32 normal) and, if words_out != NULL, the raw Philox word of
+ * element e.  The pair forward and the optimizer use the same device function. */
+int zoact_philox_normals(zoact_ctx* ctx, uint64_t seed, uint32_t layer_id, uint64_t query,
+                         int64_t n, float* z_out, uint32_t* words_out);
+
+/* ---- the low-rank projection p = U^T x (Section 3: the factor X V_r) ----
+ * X [rows, d_in] of xdtype (FP32/BF16/FP16), U [d_in, r] fp32 -> P [rows, r] fp32.
+ * d_in % 8 == 0 for BF16/FP16, % 4 for FP32.                                    */
+int zoact_lowrank_proj(zoact_ctx* ctx, const void* X, int xdtype, int64_t rows, int32_t d_in,
+                       const float* U, int32_t r, float* P);
+
+/* ---- the pair forward (Section 3, perturbed forward pass; Algorithm 2) ----
+ * Y = the stacked outputs y(+1), y(-1) of one adapted linear:
+ *   input_shared == 0: X is [2T, d_in] stacked; row t of Y uses sigma(t).
+ *   input_shared == 1: X is [T, d_in], the same input for both signs; W x is
+ *                      computed once per row and Y rows t and T + t are written.
+ * X has xdtype == the weight's compute type (FP32 for FP32 weights; BF16 for
+ * BF16 and INT4_G128; FP16 for FP16).  Y [2T, d_out] of ydtype (same as xdtype,
+ * or FP32).  `act` (ZOACT_ACT_*) is applied to y before it is stored.
+ * P: optional [rows(X), r] fp32 projection U^T x computed earlier (e.g. by
+ * zoact_lowrank_proj, or shared by layers with the same input and basis); when
+ * NULL the call computes it into context scratch first.
+ * Requirements: d_in % 8 == 0 (BF16/FP16), d_in % 128 == 0 (INT4), d_out % 8 == 0,
+ * 16-byte aligned X, W, Y.                                                       */
+int zoact_pair_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype,
+                       int64_t T, int input_shared, const float* P, float eps, uint64_t seed,
+                       uint64_t query, int act, void* Y, int ydtype);
+
+/* ---- SiLU-gated pair forward (the Llama MLP gate/up pair) ----
+ * H = silu(y_gate) * y_up for both signs, with y_gate, y_up the pair forwards of
+ * `gate` and `up` on the same X (same d_in, d_out, r and wtype).  H [2T, d_out]
+ * of ydtype.  Gate and up keep their own U, C and layer_id (P_gate / P_up may be
+ * the same pointer when the bases are equal; NULL computes them).               */
+int zoact_pair_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up,
+                             const void* X, int xdtype, int64_t T, int input_shared,
+                             const float* P_gate, const float* P_up, float eps, uint64_t seed,
+                             uint64_t query, void* H, int ydtype);
+
+/* ---- the loss pair (Section 3 estimator, two-sided; Algorithm 2) ----
+ * Y [2T, n] stacked outputs of ydtype; target [T, n] of ydtype, or NULL for the
+ * mean square loss.  Writes out[0] = L+ = mean((y+ - t)^2), out[1] = L-,
+ * out[2] = D = L+ - L- (formed as mean((y+ - y-)(y+ + y- - 2t)), without
+ * cancellation), out[3] = a = D / (2 eps), all fp64, to DEVICE memory out[4].
+ * A non-finite result sets ZOACT_ERR_NONFINITE in the device status word.       */
+int zoact_loss_pair(zoact_ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T,
+                    int64_t n, float eps, double* out);
+
+/* ---- ZO-Adam (Section 3: Adam on g = a * Z; Appendix B: weight decay 0) ----
+ * Updates the flat fp32 arenas C, m, v (n_total elements) in place for every
+ * block: g = a * Z(seed, layer_id, query) with a = loss_out[3] (device fp64),
+ *   m = b1 m + (1-b1) g;  v = b2 v + (1-b2) g^2;
+ *   C -= lr * (m / (1 - b1^step)) / (sqrt(v / (1 - b2^step)) + adam_eps).
+ * step is 1-based.  If a is not finite nothing is updated and the device status
+ * word gets ZOACT_ERR_NONFINITE.  blocks is a HOST array of n_blocks entries.    */
+int zoact_adam_step(zoact_ctx* ctx, float* C, float* m, float* v, int64_t n_total,
+                    const zoact_coeff_block* blocks, int32_t n_blocks, const double* loss_out,
+                    float lr, float beta1, float beta2, float adam_eps, int64_t step,
+                    uint64_t seed, uint64_t query);
+
+/* ---- ZO-SGD (Table 1, "ZO-Act Full SGD"): C -= lr * a * Z, same layout. ---- */
+int zoact_sgd_step(zoact_ctx* ctx, float* C, int64_t n_total, const zoact_coeff_block* blocks,
+                   int32_t n_blocks, const double* loss_out, float lr, uint64_t seed,
+                   uint64_t query);
+
+/* ---- the one-shot basis (Algorithm 1) ----
+ * U_out [d_in, r] fp32 = the top-r right singular vectors of the calibration
+ * activations X_cal [n_tok, d_in] (xdtype FP32/BF16/FP16), i.e. the top-r
+ * eigenvectors of G = X^T X (uncentred), by randomised subspace iteration:
+ * k = r + oversample columns, Omega from the Z generator with (seed, 0, 0)
+ * (element i*k + j), Q0 = orth(Omega), Q <- orth(G Q) n_iter times, then
+ * Rayleigh-Ritz.  Columns in descending eigenvalue order, each flipped so its
+ * largest-magnitude entry is positive.  Optional evals_out [k] fp32 (device)
+ * receives the Ritz values.  Requires k <= 64 and k <= d_in; uses d_in^2 * 4
+ * bytes of context scratch.                                                    */
+int zoact_basis_init(zoact_ctx* ctx, const void* X_cal, int xdtype, int64_t n_tok, int32_t d_in,
+                     int32_t r, int32_t oversample, int32_t n_iter, uint64_t seed, float* U_out,
+                     float* evals_out);
+
+/* ---- glue ops of the synthetic graphs (row-wise; activations of one dtype) ----
+ * zoact_rms_norm:  Y = X / sqrt(mean(X^2, row) + eps), no gain.                  */
+int zoact_rms_norm(zoact_ctx* ctx, const void* X, int dtype, int64_t rows, int32_t n, float eps,
+                   void* Y);
+/* zoact_mix_rms: Y = rms_norm(q + rep(k) + rep(v)) with q [rows, n], k and v
+ * [rows, n / n_rep]; rep repeats each head_dim-wide kv head for n_rep
+ * consecutive query heads (n_rep = 1: plain sum).                              */
+int zoact_mix_rms(zoact_ctx* ctx, const void* q, const void* k, const void* v, int dtype,
+                  int64_t rows, int32_t n, int32_t n_rep, int32_t head_dim, float eps, void* Y);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ZOACT_H_ */

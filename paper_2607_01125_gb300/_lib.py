@@ -1,0 +1,240 @@
+"""ctypes binding of libzoact (include/zoact.h): argument marshalling only.
+
+Every function below has the name of the C entry point it calls and passes
+torch tensors as raw device pointers; no step of the ZO-Act path runs in
+Python.  Loading fails loudly when the library has not been built: there is no
+CPU fallback.
+"""
+import ctypes
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libzoact.so")
+
+ZOACT_OK = 0
+ZOACT_ERR_INVALID_ARG = -1
+ZOACT_ERR_UNSUPPORTED = -2
+ZOACT_ERR_CUDA = -3
+ZOACT_ERR_NONFINITE = -4
+ZOACT_ERR_TIMEOUT = -5
+ZOACT_ERR_NOMEM = -6
+
+DT_FP32, DT_BF16, DT_FP16, DT_INT4_G128 = 0, 1, 2, 3
+ACT_NONE, ACT_RELU, ACT_GELU = 0, 1, 2
+
+TORCH_DT = {torch.float32: DT_FP32, torch.bfloat16: DT_BF16, torch.float16: DT_FP16}
+
+# every entry point include/zoact.h declares
+EXPORTS = [
+    "zoact_create", "zoact_destroy", "zoact_set_stream", "zoact_status_string", "zoact_get_device_status",
+    "zoact_device_sm_count", "zoact_get_launch_count", "zoact_philox_normals", "zoact_lowrank_proj", "zoact_pair_forward",
+    "zoact_pair_forward_gated", "zoact_loss_pair", "zoact_adam_step", "zoact_sgd_step", "zoact_basis_init",
+    "zoact_rms_norm", "zoact_mix_rms",
+]
+
+
+class ZoactError(RuntimeError):
+    def __init__(self, fn, status):
+        self.status = status
+        super().__init__(f"{fn} failed: {status} ({status_string(status)})")
+
+
+class zoact_layer(ctypes.Structure):
+    _fields_ = [("d_in", ctypes.c_int32), ("d_out", ctypes.c_int32), ("r", ctypes.c_int32),
+                ("wtype", ctypes.c_int32), ("W", ctypes.c_void_p), ("w_scales", ctypes.c_void_p),
+                ("U", ctypes.c_void_p), ("C", ctypes.c_void_p), ("layer_id", ctypes.c_uint32)]
+
+
+class zoact_coeff_block(ctypes.Structure):
+    _fields_ = [("offset", ctypes.c_int64), ("d_out", ctypes.c_int32), ("r", ctypes.c_int32),
+                ("layer_id", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+
+
+_lib = None
+
+
+def load():
+    """Load libzoact.so (built in-tree by __graft_entry__.build())."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"libzoact.so is not built ({LIB_PATH}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, I32, I64, U32, U64, F32 = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32,
+                                  ctypes.c_uint64, ctypes.c_float)
+    sig = {
+        "zoact_create": [ctypes.POINTER(ctypes.c_void_p), I32, P],
+        "zoact_destroy": [P],
+        "zoact_set_stream": [P, P],
+        "zoact_get_device_status": [P, ctypes.POINTER(ctypes.c_int), I32],
+        "zoact_device_sm_count": [P, ctypes.POINTER(ctypes.c_int)],
+        "zoact_get_launch_count": [P, ctypes.POINTER(ctypes.c_int64)],
+        "zoact_philox_normals": [P, U64, U32, U64, I64, P, P],
+        "zoact_lowrank_proj": [P, P, I32, I64, I32, P, I32, P],
+        "zoact_pair_forward": [P, ctypes.POINTER(zoact_layer), P, I32, I64, I32, P, F32, U64, U64, I32, P, I32],
+        "zoact_pair_forward_gated": [P, ctypes.POINTER(zoact_layer), ctypes.POINTER(zoact_layer), P, I32, I64, I32,
+                                     P, P, F32, U64, U64, P, I32],
+        "zoact_loss_pair": [P, P, I32, P, I64, I64, F32, P],
+        "zoact_adam_step": [P, P, P, P, I64, ctypes.POINTER(zoact_coeff_block), I32, P, F32, F32, F32, F32, I64,
+                            U64, U64],
+        "zoact_sgd_step": [P, P, I64, ctypes.POINTER(zoact_coeff_block), I32, P, F32, U64, U64],
+        "zoact_basis_init": [P, P, I32, I64, I32, I32, I32, I32, U64, P, P],
+        "zoact_rms_norm": [P, P, I32, I64, I32, F32, P],
+        "zoact_mix_rms": [P, P, P, P, I32, I64, I32, I32, I32, F32, P],
+    }
+    for name, argtypes in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = argtypes
+        fn.restype = ctypes.c_int
+    lib.zoact_status_string.argtypes = [ctypes.c_int]
+    lib.zoact_status_string.restype = ctypes.c_char_p
+    _lib = lib
+    return lib
+
+
+def status_string(status):
+    return load().zoact_status_string(int(status)).decode()
+
+
+def _check(name, status):
+    if status != ZOACT_OK:
+        raise ZoactError(name, status)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _dt(t):
+    return TORCH_DT[t.dtype]
+
+
+class Context:
+    """A libzoact context bound to one CUDA device; launches on torch's current stream."""
+
+    def __init__(self, device=0):
+        lib = load()
+        self.device = int(device)
+        h = ctypes.c_void_p()
+        with torch.cuda.device(self.device):
+            stream = torch.cuda.current_stream().cuda_stream
+        _check("zoact_create", lib.zoact_create(ctypes.byref(h), self.device, ctypes.c_void_p(stream)))
+        self.handle = h
+
+    def sync_stream(self):
+        """Point the context at torch's current stream on its device."""
+        with torch.cuda.device(self.device):
+            s = torch.cuda.current_stream().cuda_stream
+        load().zoact_set_stream(self.handle, ctypes.c_void_p(s))
+
+    def sm_count(self):
+        v = ctypes.c_int()
+        _check("zoact_device_sm_count", load().zoact_device_sm_count(self.handle, ctypes.byref(v)))
+        return v.value
+
+    def launch_count(self):
+        v = ctypes.c_int64()
+        _check("zoact_get_launch_count", load().zoact_get_launch_count(self.handle, ctypes.byref(v)))
+        return v.value
+
+    def device_status(self, reset=True):
+        v = ctypes.c_int()
+        _check("zoact_get_device_status", load().zoact_get_device_status(self.handle, ctypes.byref(v), int(reset)))
+        return v.value
+
+    def close(self):
+        if getattr(self, "handle", None):
+            load().zoact_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def make_layer(W, U, C, layer_id, w_scales=None, wtype=None, d_in=None):
+    """A zoact_layer for torch tensors W [d_out, d_in] (or INT4 packed), U [d_in, r] fp32, C [d_out, r] fp32."""
+    if wtype is None:
+        wtype = _dt(W)
+    d_out = W.shape[0]
+    if d_in is None:
+        d_in = W.shape[1] * (2 if wtype == DT_INT4_G128 else 1)
+    L = zoact_layer(d_in=int(d_in), d_out=int(d_out), r=int(U.shape[1]), wtype=int(wtype),
+                    W=W.data_ptr(), w_scales=(w_scales.data_ptr() if w_scales is not None else None),
+                    U=U.data_ptr(), C=C.data_ptr(), layer_id=int(layer_id))
+    L._keep = (W, U, C, w_scales)
+    return L
+
+
+def zoact_philox_normals(ctx, seed, layer_id, query, n, z_out, words_out=None):
+    _check("zoact_philox_normals", load().zoact_philox_normals(ctx.handle, seed, layer_id, query, n, _ptr(z_out),
+                                                                _ptr(words_out)))
+
+
+def zoact_lowrank_proj(ctx, X, U, P):
+    rows, d_in = X.shape
+    _check("zoact_lowrank_proj", load().zoact_lowrank_proj(ctx.handle, _ptr(X), _dt(X), rows, d_in, _ptr(U),
+                                                            U.shape[1], _ptr(P)))
+
+
+def zoact_pair_forward(ctx, layer, X, T, input_shared, eps, seed, query, Y, P=None, act=ACT_NONE):
+    _check("zoact_pair_forward", load().zoact_pair_forward(ctx.handle, ctypes.byref(layer), _ptr(X), _dt(X), int(T),
+                                                            int(input_shared), _ptr(P), float(eps), int(seed),
+                                                            int(query), int(act), _ptr(Y), _dt(Y)))
+
+
+def zoact_pair_forward_gated(ctx, gate, up, X, T, input_shared, eps, seed, query, H, P_gate=None, P_up=None):
+    _check("zoact_pair_forward_gated", load().zoact_pair_forward_gated(
+        ctx.handle, ctypes.byref(gate), ctypes.byref(up), _ptr(X), _dt(X), int(T), int(input_shared), _ptr(P_gate),
+        _ptr(P_up), float(eps), int(seed), int(query), _ptr(H), _dt(H)))
+
+
+def zoact_loss_pair(ctx, Y, T, eps, out, target=None):
+    n = Y.shape[1]
+    _check("zoact_loss_pair", load().zoact_loss_pair(ctx.handle, _ptr(Y), _dt(Y), _ptr(target), int(T), int(n),
+                                                      float(eps), _ptr(out)))
+
+
+def _blocks(blocks):
+    arr = (zoact_coeff_block * max(1, len(blocks)))()
+    for i, (offset, d_out, r, layer_id) in enumerate(blocks):
+        arr[i] = zoact_coeff_block(offset=int(offset), d_out=int(d_out), r=int(r), layer_id=int(layer_id))
+    return arr
+
+
+def zoact_adam_step(ctx, C, m, v, blocks, loss_out, lr, beta1, beta2, adam_eps, step, seed, query):
+    """blocks: list of (offset, d_out, r, layer_id) into the flat arenas C, m, v."""
+    arr = _blocks(blocks)
+    _check("zoact_adam_step", load().zoact_adam_step(ctx.handle, _ptr(C), _ptr(m), _ptr(v), C.numel(), arr,
+                                                      len(blocks), _ptr(loss_out), float(lr), float(beta1),
+                                                      float(beta2), float(adam_eps), int(step), int(seed),
+                                                      int(query)))
+
+
+def zoact_sgd_step(ctx, C, blocks, loss_out, lr, seed, query):
+    arr = _blocks(blocks)
+    _check("zoact_sgd_step", load().zoact_sgd_step(ctx.handle, _ptr(C), C.numel(), arr, len(blocks),
+                                                    _ptr(loss_out), float(lr), int(seed), int(query)))
+
+
+def zoact_basis_init(ctx, X_cal, r, U_out, oversample=8, n_iter=8, seed=0, evals_out=None):
+    n_tok, d_in = X_cal.shape
+    _check("zoact_basis_init", load().zoact_basis_init(ctx.handle, _ptr(X_cal), _dt(X_cal), n_tok, d_in, int(r),
+                                                        int(oversample), int(n_iter), int(seed), _ptr(U_out),
+                                                        _ptr(evals_out)))
+
+
+def zoact_rms_norm(ctx, X, Y, eps=1e-5):
+    rows, n = X.shape
+    _check("zoact_rms_norm", load().zoact_rms_norm(ctx.handle, _ptr(X), _dt(X), rows, n, float(eps), _ptr(Y)))
+
+
+def zoact_mix_rms(ctx, q, k, v, Y, n_rep, head_dim, eps=1e-5):
+    rows, n = q.shape
+    _check("zoact_mix_rms", load().zoact_mix_rms(ctx.handle, _ptr(q), _ptr(k), _ptr(v), _dt(q), rows, n,
+                                                  int(n_rep), int(head_dim), float(eps), _ptr(Y)))

@@ -1,0 +1,322 @@
+// The C ABI of libzoact (declared in include/zoact.h): context, scratch,
+// argument validation and dispatch to the kernels.  No compute happens on the
+// host; every entry point only checks its arguments and enqueues kernels.
+#include <cstdio>
+#include <cstdlib>
+#include <new>
+
+#include "internal.h"
+
+namespace zoact {
+
+int cuda_fail(cudaError_t e, const char* what) {
+  if (std::getenv("ZOACT_DEBUG")) std::fprintf(stderr, "libzoact: %s failed: %s\n", what, cudaGetErrorString(e));
+  return e == cudaErrorMemoryAllocation ? ZOACT_ERR_NOMEM : ZOACT_ERR_CUDA;
+}
+
+void* scratch(Ctx* ctx, ScratchSlot slot, size_t bytes) {
+  if (bytes == 0) bytes = 256;
+  if (ctx->slot_bytes[slot] >= bytes) return ctx->slot_ptr[slot];
+  if (ctx->slot_ptr[slot]) {
+    // queued kernels may still use the old buffer
+    if (cudaStreamSynchronize(ctx->stream) != cudaSuccess) return nullptr;
+    cudaFree(ctx->slot_ptr[slot]);
+    ctx->slot_ptr[slot] = nullptr;
+    ctx->slot_bytes[slot] = 0;
+  }
+  const size_t want = (bytes + 4095) / 4096 * 4096;
+  void* p = nullptr;
+  if (cudaMalloc(&p, want) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  ctx->slot_ptr[slot] = p;
+  ctx->slot_bytes[slot] = want;
+  return p;
+}
+
+}  // namespace zoact
+
+using namespace zoact;
+
+namespace {
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+int set_device(zoact_ctx* ctx) {
+  int cur = -1;
+  if (cudaGetDevice(&cur) != cudaSuccess) return ZOACT_ERR_CUDA;
+  if (cur != ctx->device && cudaSetDevice(ctx->device) != cudaSuccess) return ZOACT_ERR_CUDA;
+  return ZOACT_OK;
+}
+
+#define ZOACT_ENTER(ctx)                  \
+  do {                                    \
+    if (!(ctx)) return ZOACT_ERR_INVALID_ARG; \
+    const int s_ = set_device(ctx);       \
+    if (s_) return s_;                    \
+  } while (0)
+
+bool valid_act_dtype(int dt) { return dt == ZOACT_DT_FP32 || dt == ZOACT_DT_BF16 || dt == ZOACT_DT_FP16; }
+
+int check_layer(const zoact_layer* L) {
+  if (!L || !L->W || !L->U || !L->C) return ZOACT_ERR_INVALID_ARG;
+  if (L->d_in <= 0 || L->d_out <= 0 || L->r <= 0) return ZOACT_ERR_INVALID_ARG;
+  if (L->r > 32) return ZOACT_ERR_UNSUPPORTED;
+  if ((int64_t)L->d_out * L->r >= (int64_t)1 << 34) return ZOACT_ERR_INVALID_ARG;
+  if (L->wtype == ZOACT_DT_INT4_G128) return ZOACT_ERR_UNSUPPORTED;
+  if (!valid_act_dtype(L->wtype)) return ZOACT_ERR_INVALID_ARG;
+  return ZOACT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int zoact_create(zoact_ctx** out, int device, void* stream) {
+  if (!out) return ZOACT_ERR_INVALID_ARG;
+  *out = nullptr;
+  int n = 0;
+  if (cudaGetDeviceCount(&n) != cudaSuccess || device < 0 || device >= n) {
+    cudaGetLastError();
+    return ZOACT_ERR_INVALID_ARG;
+  }
+  zoact_ctx* ctx = new (std::nothrow) zoact_ctx();
+  if (!ctx) return ZOACT_ERR_NOMEM;
+  ctx->device = device;
+  ctx->stream = static_cast<cudaStream_t>(stream);
+  int st = set_device(ctx);
+  if (st) { delete ctx; return st; }
+  if (cudaDeviceGetAttribute(&ctx->sm_count, cudaDevAttrMultiProcessorCount, device) != cudaSuccess) {
+    delete ctx;
+    return ZOACT_ERR_CUDA;
+  }
+  if (cudaMalloc(&ctx->d_status, 256) != cudaSuccess || cudaMalloc(&ctx->d_tickets, 256) != cudaSuccess ||
+      cudaMemsetAsync(ctx->d_status, 0, 256, ctx->stream) != cudaSuccess ||
+      cudaMemsetAsync(ctx->d_tickets, 0, 256, ctx->stream) != cudaSuccess ||
+      cudaStreamSynchronize(ctx->stream) != cudaSuccess) {
+    cudaGetLastError();
+    if (ctx->d_status) cudaFree(ctx->d_status);
+    if (ctx->d_tickets) cudaFree(ctx->d_tickets);
+    delete ctx;
+    return ZOACT_ERR_NOMEM;
+  }
+  *out = ctx;
+  return ZOACT_OK;
+}
+
+int zoact_destroy(zoact_ctx* ctx) {
+  if (!ctx) return ZOACT_OK;
+  set_device(ctx);
+  cudaStreamSynchronize(ctx->stream);
+  for (int s = 0; s < SLOT_COUNT; ++s)
+    if (ctx->slot_ptr[s]) cudaFree(ctx->slot_ptr[s]);
+  cudaFree(ctx->d_status);
+  cudaFree(ctx->d_tickets);
+  delete ctx;
+  return ZOACT_OK;
+}
+
+int zoact_set_stream(zoact_ctx* ctx, void* stream) {
+  if (!ctx) return ZOACT_ERR_INVALID_ARG;
+  ctx->stream = static_cast<cudaStream_t>(stream);
+  return ZOACT_OK;
+}
+
+const char* zoact_status_string(int status) {
+  switch (status) {
+    case ZOACT_OK: return "ok";
+    case ZOACT_ERR_INVALID_ARG: return "invalid argument";
+    case ZOACT_ERR_UNSUPPORTED: return "unsupported by this build";
+    case ZOACT_ERR_CUDA: return "CUDA runtime error";
+    case ZOACT_ERR_NONFINITE: return "non-finite loss or estimator";
+    case ZOACT_ERR_TIMEOUT: return "bounded device wait timed out";
+    case ZOACT_ERR_NOMEM: return "out of device memory";
+    default: return "unknown status";
+  }
+}
+
+int zoact_get_device_status(zoact_ctx* ctx, int* status, int reset) {
+  ZOACT_ENTER(ctx);
+  if (!status) return ZOACT_ERR_INVALID_ARG;
+  ZOACT_CUDA_TRY(cudaStreamSynchronize(ctx->stream));
+  int v = 0;
+  ZOACT_CUDA_TRY(cudaMemcpy(&v, ctx->d_status, sizeof(int), cudaMemcpyDeviceToHost));
+  *status = v;
+  if (reset) {
+    ZOACT_CUDA_TRY(cudaMemsetAsync(ctx->d_status, 0, sizeof(int), ctx->stream));
+    ZOACT_CUDA_TRY(cudaStreamSynchronize(ctx->stream));
+  }
+  return ZOACT_OK;
+}
+
+int zoact_device_sm_count(zoact_ctx* ctx, int* sm_count) {
+  if (!ctx || !sm_count) return ZOACT_ERR_INVALID_ARG;
+  *sm_count = ctx->sm_count;
+  return ZOACT_OK;
+}
+
+int zoact_get_launch_count(zoact_ctx* ctx, int64_t* count) {
+  if (!ctx || !count) return ZOACT_ERR_INVALID_ARG;
+  *count = ctx->n_launch;
+  return ZOACT_OK;
+}
+
+int zoact_philox_normals(zoact_ctx* ctx, uint64_t seed, uint32_t layer_id, uint64_t query, int64_t n, float* z_out,
+                         uint32_t* words_out) {
+  ZOACT_ENTER(ctx);
+  if (n < 0 || (n > 0 && !z_out)) return ZOACT_ERR_INVALID_ARG;
+  if (n > ((int64_t)1 << 34)) return ZOACT_ERR_INVALID_ARG;
+  return launch_philox_normals(ctx, seed, layer_id, query, n, z_out, words_out);
+}
+
+int zoact_lowrank_proj(zoact_ctx* ctx, const void* X, int xdtype, int64_t rows, int32_t d_in, const float* U,
+                       int32_t r, float* P) {
+  ZOACT_ENTER(ctx);
+  if (rows < 0 || d_in <= 0 || r <= 0 || !valid_act_dtype(xdtype)) return ZOACT_ERR_INVALID_ARG;
+  if (r > 32) return ZOACT_ERR_UNSUPPORTED;
+  if (rows == 0) return ZOACT_OK;
+  if (!X || !U || !P || !aligned16(X)) return ZOACT_ERR_INVALID_ARG;
+  if (d_in % (xdtype == ZOACT_DT_FP32 ? 4 : 8) != 0) return ZOACT_ERR_INVALID_ARG;
+  return launch_lowrank_proj(ctx, X, xdtype, rows, d_in, U, r, P);
+}
+
+static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* L2, const void* X, int xdtype,
+                       int64_t T, int input_shared, const float* P, const float* P2, float eps, uint64_t seed,
+                       uint64_t query, int act, void* Y, int ydtype) {
+  int st = check_layer(L);
+  if (st) return st;
+  if (L2) {
+    st = check_layer(L2);
+    if (st) return st;
+    if (L2->d_in != L->d_in || L2->d_out != L->d_out || L2->r != L->r || L2->wtype != L->wtype)
+      return ZOACT_ERR_INVALID_ARG;
+  }
+  if (T < 0 || !valid_act_dtype(xdtype) || !valid_act_dtype(ydtype)) return ZOACT_ERR_INVALID_ARG;
+  if (act < ZOACT_ACT_NONE || act > ZOACT_ACT_GELU) return ZOACT_ERR_INVALID_ARG;
+  if (T == 0) return ZOACT_OK;
+  if (!X || !Y) return ZOACT_ERR_INVALID_ARG;
+  if (xdtype != L->wtype) return ZOACT_ERR_INVALID_ARG;
+  if (!aligned16(X) || !aligned16(Y) || !aligned16(L->W) || (L2 && !aligned16(L2->W))) return ZOACT_ERR_INVALID_ARG;
+  if (L->d_in % (xdtype == ZOACT_DT_FP32 ? 4 : 8) != 0) return ZOACT_ERR_INVALID_ARG;
+  if (L->d_out % 8 != 0) return ZOACT_ERR_INVALID_ARG;
+  const int64_t rows = input_shared ? T : 2 * T;
+  // projection(s) U^T x, unless the caller passed them
+  if (!P) {
+    float* p = static_cast<float*>(scratch(ctx, SLOT_P0, (size_t)rows * L->r * sizeof(float)));
+    if (!p) return ZOACT_ERR_NOMEM;
+    st = launch_lowrank_proj(ctx, X, xdtype, rows, L->d_in, L->U, L->r, p);
+    if (st) return st;
+    P = p;
+  }
+  if (L2 && !P2) {
+    float* p = static_cast<float*>(scratch(ctx, SLOT_P1, (size_t)rows * L2->r * sizeof(float)));
+    if (!p) return ZOACT_ERR_NOMEM;
+    st = launch_lowrank_proj(ctx, X, xdtype, rows, L2->d_in, L2->U, L2->r, p);
+    if (st) return st;
+    P2 = p;
+  }
+  PairArgs a{};
+  a.X = X; a.W = L->W; a.w_scales = L->w_scales; a.P = P; a.C = L->C; a.Y = Y;
+  a.rows = rows; a.T = T; a.d_in = L->d_in; a.d_out = L->d_out; a.r = L->r;
+  a.shared = input_shared ? 1 : 0; a.act = act;
+  a.xdtype = xdtype; a.wtype = L->wtype; a.ydtype = ydtype;
+  a.eps = eps; a.seed = seed; a.query = query; a.layer_id = L->layer_id;
+  if (L2) { a.W2 = L2->W; a.P2 = P2; a.C2 = L2->C; a.layer_id2 = L2->layer_id; }
+  if (xdtype == ZOACT_DT_FP32) return launch_pair_simt(ctx, a);
+  return launch_pair_tc(ctx, a);
+}
+
+int zoact_pair_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype, int64_t T,
+                       int input_shared, const float* P, float eps, uint64_t seed, uint64_t query, int act, void* Y,
+                       int ydtype) {
+  ZOACT_ENTER(ctx);
+  return pair_common(ctx, layer, nullptr, X, xdtype, T, input_shared, P, nullptr, eps, seed, query, act, Y, ydtype);
+}
+
+int zoact_pair_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up, const void* X,
+                             int xdtype, int64_t T, int input_shared, const float* P_gate, const float* P_up,
+                             float eps, uint64_t seed, uint64_t query, void* H, int ydtype) {
+  ZOACT_ENTER(ctx);
+  if (!gate || !up) return ZOACT_ERR_INVALID_ARG;
+  if (xdtype == ZOACT_DT_FP32) return ZOACT_ERR_UNSUPPORTED;
+  return pair_common(ctx, gate, up, X, xdtype, T, input_shared, P_gate, P_up, eps, seed, query, ZOACT_ACT_NONE, H,
+                     ydtype);
+}
+
+int zoact_loss_pair(zoact_ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T, int64_t n, float eps,
+                    double* out) {
+  ZOACT_ENTER(ctx);
+  if (!Y || !out || T <= 0 || n <= 0 || !valid_act_dtype(ydtype)) return ZOACT_ERR_INVALID_ARG;
+  if (!(eps > 0.0f)) return ZOACT_ERR_INVALID_ARG;
+  const int max_blocks = loss_pair_max_blocks(ctx);
+  double* partials = static_cast<double*>(scratch(ctx, SLOT_PARTIALS, (size_t)max_blocks * 3 * sizeof(double)));
+  if (!partials) return ZOACT_ERR_NOMEM;
+  return launch_loss_pair(ctx, Y, ydtype, target, T, n, eps, out, partials, max_blocks);
+}
+
+static int check_blocks(const float* C, int64_t n_total, const zoact_coeff_block* blocks, int32_t n_blocks) {
+  if (!C || n_total < 0 || n_blocks < 0 || (n_blocks > 0 && !blocks)) return ZOACT_ERR_INVALID_ARG;
+  if (!aligned16(C)) return ZOACT_ERR_INVALID_ARG;
+  int64_t prev_end = 0;
+  for (int i = 0; i < n_blocks; ++i) {
+    const zoact_coeff_block& b = blocks[i];
+    if (b.offset < prev_end || b.offset % 4 != 0 || b.d_out <= 0 || b.r <= 0) return ZOACT_ERR_INVALID_ARG;
+    const int64_t end = b.offset + (int64_t)b.d_out * b.r;
+    if (end > n_total || (int64_t)b.d_out * b.r >= (int64_t)1 << 34) return ZOACT_ERR_INVALID_ARG;
+    prev_end = end;
+  }
+  return ZOACT_OK;
+}
+
+int zoact_adam_step(zoact_ctx* ctx, float* C, float* m, float* v, int64_t n_total, const zoact_coeff_block* blocks,
+                    int32_t n_blocks, const double* loss_out, float lr, float beta1, float beta2, float adam_eps,
+                    int64_t step, uint64_t seed, uint64_t query) {
+  ZOACT_ENTER(ctx);
+  int st = check_blocks(C, n_total, blocks, n_blocks);
+  if (st) return st;
+  if (!m || !v || !loss_out || step < 1 || !aligned16(m) || !aligned16(v)) return ZOACT_ERR_INVALID_ARG;
+  if (!(beta1 >= 0.f && beta1 < 1.f && beta2 >= 0.f && beta2 < 1.f)) return ZOACT_ERR_INVALID_ARG;
+  return launch_adam(ctx, C, m, v, blocks, n_blocks, loss_out, lr, beta1, beta2, adam_eps, step, seed, query, 0);
+}
+
+int zoact_sgd_step(zoact_ctx* ctx, float* C, int64_t n_total, const zoact_coeff_block* blocks, int32_t n_blocks,
+                   const double* loss_out, float lr, uint64_t seed, uint64_t query) {
+  ZOACT_ENTER(ctx);
+  int st = check_blocks(C, n_total, blocks, n_blocks);
+  if (st) return st;
+  if (!loss_out) return ZOACT_ERR_INVALID_ARG;
+  return launch_adam(ctx, C, nullptr, nullptr, blocks, n_blocks, loss_out, lr, 0.f, 0.f, 0.f, 1, seed, query, 1);
+}
+
+int zoact_basis_init(zoact_ctx* ctx, const void* X_cal, int xdtype, int64_t n_tok, int32_t d_in, int32_t r,
+                     int32_t oversample, int32_t n_iter, uint64_t seed, float* U_out, float* evals_out) {
+  ZOACT_ENTER(ctx);
+  if (!X_cal || !U_out || n_tok <= 0 || d_in <= 0 || r <= 0 || oversample < 0 || n_iter < 0 ||
+      !valid_act_dtype(xdtype))
+    return ZOACT_ERR_INVALID_ARG;
+  if (r > d_in) return ZOACT_ERR_INVALID_ARG;
+  if (xdtype != ZOACT_DT_FP32 && (d_in % 8 != 0 || !aligned16(X_cal))) return ZOACT_ERR_INVALID_ARG;
+  if (n_tok > INT32_MAX) return ZOACT_ERR_UNSUPPORTED;
+  return run_basis_init(ctx, X_cal, xdtype, n_tok, d_in, r, oversample, n_iter, seed, U_out, evals_out);
+}
+
+int zoact_rms_norm(zoact_ctx* ctx, const void* X, int dtype, int64_t rows, int32_t n, float eps, void* Y) {
+  ZOACT_ENTER(ctx);
+  if (rows < 0 || n <= 0 || !valid_act_dtype(dtype)) return ZOACT_ERR_INVALID_ARG;
+  if (rows > 0 && (!X || !Y)) return ZOACT_ERR_INVALID_ARG;
+  if (rows > 0x7fffffff) return ZOACT_ERR_UNSUPPORTED;
+  return launch_rms_norm(ctx, X, dtype, rows, n, eps, Y);
+}
+
+int zoact_mix_rms(zoact_ctx* ctx, const void* q, const void* k, const void* v, int dtype, int64_t rows, int32_t n,
+                  int32_t n_rep, int32_t head_dim, float eps, void* Y) {
+  ZOACT_ENTER(ctx);
+  if (rows < 0 || n <= 0 || n_rep <= 0 || head_dim <= 0 || !valid_act_dtype(dtype)) return ZOACT_ERR_INVALID_ARG;
+  if (n % (n_rep * head_dim) != 0) return ZOACT_ERR_INVALID_ARG;
+  if (rows > 0 && (!q || !k || !v || !Y)) return ZOACT_ERR_INVALID_ARG;
+  if (rows > 0x7fffffff) return ZOACT_ERR_UNSUPPORTED;
+  return launch_mix_rms(ctx, q, k, v, dtype, rows, n, n_rep, head_dim, eps, Y);
+}
+
+}  // extern "C"

@@ -1,0 +1,127 @@
+// Internal declarations shared by the libzoact translation units.
+#pragma once
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cstdint>
+#include <cstddef>
+
+#include "../../include/zoact.h"
+
+#define ZOACT_CUDA_TRY(expr)                                  \
+  do {                                                        \
+    cudaError_t e_ = (expr);                                  \
+    if (e_ != cudaSuccess) return zoact::cuda_fail(e_, #expr); \
+  } while (0)
+
+#define ZOACT_CHECK_LAUNCH() ZOACT_CUDA_TRY(cudaGetLastError())
+
+namespace zoact {
+
+// Scratch slots owned by a context.  Each slot grows on demand; growing
+// synchronises the stream first so no queued kernel still uses the old buffer.
+enum ScratchSlot {
+  SLOT_P0 = 0,       // projection U^T x of the current call
+  SLOT_P1,           // second projection (gated pair forward)
+  SLOT_SPLITK,       // split-K partials of the projection
+  SLOT_PARTIALS,     // per-block partial sums of grid reductions
+  SLOT_BASIS,        // Gram matrix and subspace-iteration workspace
+  SLOT_BASIS_X,      // transposed calibration activations
+  SLOT_COUNT
+};
+
+struct Ctx {
+  int device = 0;
+  cudaStream_t stream = nullptr;
+  int sm_count = 0;
+  int64_t n_launch = 0;              // kernels launched through this context (host counter)
+  int* d_status = nullptr;            // device status word (first error wins)
+  unsigned int* d_tickets = nullptr;  // grid-reduction tickets, reset by their last block
+  void* slot_ptr[SLOT_COUNT] = {};
+  size_t slot_bytes[SLOT_COUNT] = {};
+};
+
+int cuda_fail(cudaError_t e, const char* what);
+// Returns a device pointer of at least `bytes` for the slot, or nullptr on failure.
+void* scratch(Ctx* ctx, ScratchSlot slot, size_t bytes);
+
+// Device-side error recording: keeps the first non-zero code.
+__device__ __forceinline__ void record_error(int* status, int code) {
+  if (status) atomicCAS(status, 0, code);
+}
+
+// ---- dtype helpers ----
+template <typename T> __device__ __forceinline__ float to_f32(T v);
+template <> __device__ __forceinline__ float to_f32<float>(float v) { return v; }
+template <> __device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+template <> __device__ __forceinline__ float to_f32<__half>(__half v) { return __half2float(v); }
+
+template <typename T> __device__ __forceinline__ T from_f32(float v);
+template <> __device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+template <> __device__ __forceinline__ __half from_f32<__half>(float v) { return __float2half_rn(v); }
+
+__device__ __forceinline__ float apply_act(float y, int act) {
+  if (act == ZOACT_ACT_RELU) return fmaxf(y, 0.0f);
+  if (act == ZOACT_ACT_GELU) return 0.5f * y * (1.0f + erff(y * 0.70710678118654752f));
+  return y;
+}
+
+__device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
+
+inline size_t dtype_size(int dt) {
+  return dt == ZOACT_DT_FP32 ? 4 : 2;
+}
+
+// ---- launchers (return ZOACT_* status) ----
+int launch_philox_normals(Ctx* ctx, uint64_t seed, uint32_t layer_id, uint64_t query, int64_t n,
+                          float* z, uint32_t* words);
+int launch_lowrank_proj(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const float* U,
+                        int r, float* P);
+
+struct PairArgs {
+  const void* X;        // [rows, d_in]
+  const void* W;        // [d_out, d_in] (or INT4 packed)
+  const void* w_scales;
+  const float* P;       // [rows, r]
+  const float* C;       // [d_out, r]
+  void* Y;              // [2T, d_out]
+  int64_t rows;         // rows of X (T if shared else 2T)
+  int64_t T;
+  int d_in, d_out, r;
+  int shared;
+  int act;
+  int xdtype, wtype, ydtype;
+  float eps;
+  uint64_t seed, query;
+  uint32_t layer_id;
+  // gated mode (second layer: up); W2 == nullptr for the plain pair forward
+  const void* W2;
+  const float* P2;
+  const float* C2;
+  uint32_t layer_id2;
+};
+int launch_pair_simt(Ctx* ctx, const PairArgs& a);
+int launch_pair_tc(Ctx* ctx, const PairArgs& a);
+// Plain product D[M, N] (fp32) = A[M, K] * B[N, K]^T with 16-bit A, B (K-major), on tcgen05.
+int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int M, int N, int K,
+                          float* D);
+
+int launch_loss_pair(Ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T, int64_t n,
+                     float eps, double* out, double* partials, int max_blocks);
+int loss_pair_max_blocks(Ctx* ctx);
+
+int launch_adam(Ctx* ctx, float* C, float* m, float* v, const zoact_coeff_block* blocks, int n_blocks,
+                const double* loss_out, float lr, float b1, float b2, float adam_eps, int64_t step,
+                uint64_t seed, uint64_t query, int sgd);
+
+int launch_rms_norm(Ctx* ctx, const void* X, int dtype, int64_t rows, int n, float eps, void* Y);
+int launch_mix_rms(Ctx* ctx, const void* q, const void* k, const void* v, int dtype, int64_t rows,
+                   int n, int n_rep, int head_dim, float eps, void* Y);
+
+int run_basis_init(Ctx* ctx, const void* X, int xdtype, int64_t n_tok, int d_in, int r, int oversample,
+                   int n_iter, uint64_t seed, float* U_out, float* evals_out);
+
+}  // namespace zoact
+
+struct zoact_ctx : public zoact::Ctx {};

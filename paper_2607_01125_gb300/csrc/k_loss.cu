@@ -1,0 +1,145 @@
+// Loss pair and estimator scalar (Section 3 estimator in two-sided form; Algorithm 2):
+//   L+ = mean((y+ - t)^2),  L- = mean((y- - t)^2),
+//   D  = mean((y+ - y-)(y+ + y- - 2t))   (= L+ - L-, without cancellation),
+//   a  = D / (2 eps).
+// One pass over the stacked outputs (HBM-bound).  Each thread reads 16-byte
+// vectors of y+, y- and t, sums a vector's terms in fp32 and adds the vector sum
+// to fp64 accumulators; warps reduce by shuffles, blocks write fp64 partials to
+// scratch, and the last block to finish (an atomic ticket) adds the partials in
+// block order, so the result is deterministic.  The ticket is reset by that
+// block, leaving the scratch ready for the next call.
+#include "internal.h"
+
+namespace zoact {
+namespace {
+
+constexpr int LOSS_THREADS = 256;
+
+template <typename TY>
+__device__ __forceinline__ void load8(const TY* p, float* out) {
+  const uint4 raw = *reinterpret_cast<const uint4*>(p);
+  const TY* e = reinterpret_cast<const TY*>(&raw);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) out[i] = to_f32<TY>(e[i]);
+}
+template <>
+__device__ __forceinline__ void load8<float>(const float* p, float* out) {
+  const float4 a = *reinterpret_cast<const float4*>(p);
+  const float4 b = *reinterpret_cast<const float4*>(p + 4);
+  out[0] = a.x; out[1] = a.y; out[2] = a.z; out[3] = a.w;
+  out[4] = b.x; out[5] = b.y; out[6] = b.z; out[7] = b.w;
+}
+
+__device__ __forceinline__ double warp_sum(double v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+template <typename TY>
+__global__ void __launch_bounds__(LOSS_THREADS)
+loss_pair_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t count, int vec_ok, float eps,
+                 double* __restrict__ out, double* __restrict__ partials, unsigned int* __restrict__ ticket,
+                 int* __restrict__ status) {
+  const TY* yp = Y;
+  const TY* ym = Y + count;
+  double ap = 0.0, am = 0.0, ad = 0.0;
+  // 16-byte vectors need y+, y- and t 16-byte aligned (host checks the bases;
+  // y- = y+ + count is aligned when count % 8 == 0)
+  const int64_t n_vec = vec_ok ? count / 8 : 0;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < n_vec; v += stride) {
+    float p[8], m[8], t[8];
+    load8<TY>(yp + 8 * v, p);
+    load8<TY>(ym + 8 * v, m);
+    if (tgt) {
+      load8<TY>(tgt + 8 * v, t);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) t[i] = 0.f;
+    }
+    float sp = 0.f, sm = 0.f, sd = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float dp = p[i] - t[i], dm = m[i] - t[i];
+      sp = fmaf(dp, dp, sp);
+      sm = fmaf(dm, dm, sm);
+      sd = fmaf(p[i] - m[i], dp + dm, sd);
+    }
+    ap += sp; am += sm; ad += sd;
+  }
+  // scalar remainder (everything when the vector path is off)
+  for (int64_t i = 8 * n_vec + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < count; i += stride) {
+    const float tv = tgt ? to_f32<TY>(tgt[i]) : 0.f;
+    const float dp = to_f32<TY>(yp[i]) - tv, dm = to_f32<TY>(ym[i]) - tv;
+    ap += (double)(dp * dp); am += (double)(dm * dm);
+    ad += (double)((to_f32<TY>(yp[i]) - to_f32<TY>(ym[i])) * (dp + dm));
+  }
+  __shared__ double red[3][LOSS_THREADS / 32];
+  __shared__ bool is_last;
+  ap = warp_sum(ap); am = warp_sum(am); ad = warp_sum(ad);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0) { red[0][warp] = ap; red[1][warp] = am; red[2][warp] = ad; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s0 = 0.0, s1 = 0.0, s2 = 0.0;
+    for (int w = 0; w < LOSS_THREADS / 32; ++w) { s0 += red[0][w]; s1 += red[1][w]; s2 += red[2][w]; }
+    partials[3 * blockIdx.x + 0] = s0;
+    partials[3 * blockIdx.x + 1] = s1;
+    partials[3 * blockIdx.x + 2] = s2;
+    __threadfence();
+    const unsigned int prev = atomicAdd(ticket, 1u);
+    is_last = (prev == gridDim.x - 1);
+  }
+  __syncthreads();
+  if (is_last && threadIdx.x == 0) {
+    __threadfence();
+    double s0 = 0.0, s1 = 0.0, s2 = 0.0;
+    const volatile double* pv = partials;
+    for (unsigned int b = 0; b < gridDim.x; ++b) { s0 += pv[3 * b]; s1 += pv[3 * b + 1]; s2 += pv[3 * b + 2]; }
+    const double inv = 1.0 / (double)count;
+    const double Lp = s0 * inv, Lm = s1 * inv, D = s2 * inv;
+    const double a = D / (2.0 * (double)eps);
+    out[0] = Lp; out[1] = Lm; out[2] = D; out[3] = a;
+    if (!isfinite(Lp) || !isfinite(Lm) || !isfinite(a)) record_error(status, ZOACT_ERR_NONFINITE);
+    *ticket = 0u;
+  }
+}
+
+template <typename TY>
+int loss_dispatch(Ctx* ctx, const TY* Y, const TY* tgt, int64_t count, float eps, double* out,
+                  double* partials, int max_blocks, unsigned int* ticket) {
+  const int vec_ok = (count % 8 == 0) && ((uintptr_t)Y % 16 == 0) && ((uintptr_t)tgt % 16 == 0);
+  int64_t blocks = ((vec_ok ? count / 8 : count) + LOSS_THREADS - 1) / LOSS_THREADS;
+  if (blocks < 1) blocks = 1;
+  if (blocks > max_blocks) blocks = max_blocks;
+  loss_pair_kernel<TY><<<(unsigned)blocks, LOSS_THREADS, 0, ctx->stream>>>(Y, tgt, count, vec_ok, eps, out,
+                                                                           partials, ticket, ctx->d_status); ++ctx->n_launch;
+  ZOACT_CHECK_LAUNCH();
+  return ZOACT_OK;
+}
+
+}  // namespace
+
+int loss_pair_max_blocks(Ctx* ctx) { return 2 * ctx->sm_count; }
+
+int launch_loss_pair(Ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T, int64_t n, float eps,
+                     double* out, double* partials, int max_blocks) {
+  const int64_t count = T * n;
+  unsigned int* ticket = ctx->d_tickets;
+  switch (ydtype) {
+    case ZOACT_DT_FP32:
+      return loss_dispatch(ctx, static_cast<const float*>(Y), static_cast<const float*>(target), count, eps, out,
+                           partials, max_blocks, ticket);
+    case ZOACT_DT_BF16:
+      return loss_dispatch(ctx, static_cast<const __nv_bfloat16*>(Y), static_cast<const __nv_bfloat16*>(target),
+                           count, eps, out, partials, max_blocks, ticket);
+    case ZOACT_DT_FP16:
+      return loss_dispatch(ctx, static_cast<const __half*>(Y), static_cast<const __half*>(target), count, eps, out,
+                           partials, max_blocks, ticket);
+    default:
+      return ZOACT_ERR_INVALID_ARG;
+  }
+}
+
+}  // namespace zoact

@@ -1,0 +1,111 @@
+// Host side of the tensor-core pair forward: tensor-map encoding, argument
+// checks and dispatch to the per-dtype instantiations of pair_tc_kernel.
+#include <mutex>
+
+#include "pair_tc_kernel.cuh"
+
+namespace zoact {
+
+namespace pairtc {
+int dispatch_bf16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const CUtensorMap& b,
+                  const CUtensorMap& b2, const Params& p);
+int dispatch_fp16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const CUtensorMap& b,
+                  const CUtensorMap& b2, const Params& p);
+}  // namespace pairtc
+
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+int rank_template(int r) { return r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32; }
+
+}  // namespace
+
+int encode_tmap_2d_16bit(CUtensorMap* map, const void* base, int dtype, int64_t rows, int64_t cols, int box_rows) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return ZOACT_ERR_CUDA;
+  const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  const cuuint32_t box[2] = {64u, (cuuint32_t)box_rows};
+  const cuuint32_t estr[2] = {1u, 1u};
+  const CUtensorMapDataType dt =
+      dtype == ZOACT_DT_FP16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  const CUresult res = fn(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return res == CUDA_SUCCESS ? ZOACT_OK : ZOACT_ERR_INVALID_ARG;
+}
+
+int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
+  using namespace pairtc;
+  if (a.xdtype != ZOACT_DT_BF16 && a.xdtype != ZOACT_DT_FP16) return ZOACT_ERR_UNSUPPORTED;
+  if (a.wtype != a.xdtype) return ZOACT_ERR_UNSUPPORTED;
+  if (a.ydtype != a.xdtype && a.ydtype != ZOACT_DT_FP32) return ZOACT_ERR_UNSUPPORTED;
+  const bool gated = a.W2 != nullptr;
+  const int rt = rank_template(a.r);
+  if (gated && rt > 16) return ZOACT_ERR_UNSUPPORTED;
+  if (a.rows <= 0) return ZOACT_OK;
+  CUtensorMap ma, mb, mb2;
+  int st = encode_tmap_2d_16bit(&ma, a.X, a.xdtype, a.rows, a.d_in, BM);
+  if (st) return st;
+  st = encode_tmap_2d_16bit(&mb, a.W, a.wtype, a.d_out, a.d_in, gated ? BN / 2 : BN);
+  if (st) return st;
+  if (gated) {
+    st = encode_tmap_2d_16bit(&mb2, a.W2, a.wtype, a.d_out, a.d_in, BN / 2);
+    if (st) return st;
+  } else {
+    mb2 = mb;
+  }
+  Params p{};
+  p.P = a.P; p.C = a.C; p.P2 = a.P2; p.C2 = a.C2; p.Y = a.Y;
+  p.rows = a.rows; p.T = a.T; p.d_in = a.d_in; p.d_out = a.d_out; p.r = a.r;
+  p.shared = a.shared; p.act = a.act; p.eps = a.eps; p.seed = a.seed; p.query = a.query;
+  p.layer_id = a.layer_id; p.layer_id2 = a.layer_id2;
+  p.num_m = (int)((a.rows + BM - 1) / BM);
+  p.num_n = gated ? (a.d_out + BN / 2 - 1) / (BN / 2) : (a.d_out + BN - 1) / BN;
+  p.num_k = (a.d_in + BK - 1) / BK;
+  p.num_tiles = p.num_m * p.num_n;
+  p.ldy = a.d_out;
+  p.status = ctx->d_status;
+  const int mode = gated ? MODE_GATED : MODE_PAIR;
+  return a.xdtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p)
+                                   : dispatch_fp16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p);
+}
+
+int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int M, int N, int K, float* D) {
+  using namespace pairtc;
+  if (M <= 0 || N <= 0) return ZOACT_OK;
+  CUtensorMap ma, mb;
+  int st = encode_tmap_2d_16bit(&ma, A, dtype, M, K, BM);
+  if (st) return st;
+  st = encode_tmap_2d_16bit(&mb, B, dtype, N, K, BN);
+  if (st) return st;
+  Params p{};
+  p.Y = D;
+  p.rows = M; p.T = M; p.d_in = K; p.d_out = N; p.r = 0;
+  p.num_m = (M + BM - 1) / BM;
+  p.num_n = (N + BN - 1) / BN;
+  p.num_k = (K + BK - 1) / BK;
+  p.num_tiles = p.num_m * p.num_n;
+  p.ldy = N;
+  p.status = ctx->d_status;
+  return dtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, MODE_PLAIN, 4, ZOACT_DT_FP32, ma, mb, mb, p)
+                                : dispatch_fp16(ctx, MODE_PLAIN, 4, ZOACT_DT_FP32, ma, mb, mb, p);
+}
+
+}  // namespace zoact

@@ -1,0 +1,419 @@
+// Pair forward on the 5th-generation tensor cores (Section 3, the perturbed
+// forward pass; Algorithm 2 evaluates it at +eps and -eps):
+//
+//   Y[t, n] = act( sum_k X[t, k] W[n, k] + sum_j (C[n, j] + sigma(t) eps Z[n, j]) P[t, j] )
+//
+// with P = X U (computed before), Z regenerated from Philox inside the epilogue.
+// The + and - perturbations are stacked along the token axis, so every W tile
+// is fetched once for both signs; when both signs share the input (the first
+// layer, or gate/up of an MLP) the product is computed once and each
+// accumulator row is written twice.
+//
+// Structure (one persistent CTA per SM, 192 threads):
+//   warp 0      TMA producer: X and W tiles (128x64 and 256x64, bf16/fp16,
+//               128-byte swizzle) into a 4-stage shared-memory ring;
+//   warp 1      MMA issuer: tcgen05.mma 128x256x16 into a TMEM accumulator,
+//               two accumulators (512 TMEM columns) so the epilogue of one
+//               tile overlaps the main loop of the next;
+//   warps 2-5   epilogue: per tile, build the C and Z columns of the tile in
+//               shared memory, then tcgen05.ld the accumulator 16 columns at
+//               a time, add the low-rank term in fp32, apply the activation
+//               and store.
+// Gated mode (SiLU MLP gate/up): the 256-row W tile is 128 rows of W_gate and
+// the same 128 rows of W_up; the epilogue writes silu(gate) * up for 128 columns.
+// Plain mode (no P): the accumulator is stored as fp32 (used for X^T X).
+#pragma once
+#include "internal.h"
+#include "philox.cuh"
+#include "tc_common.cuh"
+
+namespace zoact {
+namespace pairtc {
+
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;
+constexpr int B_BYTES = BN * BK * 2;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int TABLE_FLOATS = 4096;  // per table (C or Z): slots * RT
+constexpr int NUM_THREADS = 192;
+constexpr int EPI_THREADS = 128;
+constexpr int TMEM_COLS = 512;
+constexpr int SMEM_BYTES = 1024 /*align slack*/ + STAGES * STAGE_BYTES + 2 * TABLE_FLOATS * 4 + 256;
+constexpr int GROUP_M = 8;
+
+enum Mode { MODE_PAIR = 0, MODE_GATED = 1, MODE_PLAIN = 2 };
+
+struct Params {
+  const float* P;
+  const float* C;
+  const float* P2;   // gated: up
+  const float* C2;
+  void* Y;
+  int64_t rows;      // rows of X
+  int64_t T;
+  int d_in, d_out, r;
+  int shared;
+  int act;
+  float eps;
+  uint64_t seed, query;
+  uint32_t layer_id, layer_id2;
+  int num_m, num_n, num_k, num_tiles;
+  int64_t ldy;       // plain mode: row stride of D
+  int* status;
+};
+
+struct SharedState {
+  uint64_t full[STAGES];
+  uint64_t empty[STAGES];
+  uint64_t tmem_full[2];
+  uint64_t tmem_empty[2];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort_flag;
+  int epi_ok;
+};
+
+__device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& m_blk, int& n_blk) {
+  const int per_group = GROUP_M * num_n;
+  const int group = tile / per_group;
+  const int first_m = group * GROUP_M;
+  const int gm = min(GROUP_M, num_m - first_m);
+  const int in_group = tile - group * per_group;
+  m_blk = first_m + in_group % gm;
+  n_blk = in_group / gm;
+}
+
+// Fill table slots [slot0, slot0 + ncols) with C and Z of output columns
+// [col0, col0 + ncols) of one layer; columns >= d_out get zeros.  RT >= r is
+// the padded rank of the table rows.
+template <int RT>
+__device__ __forceinline__ void build_table(float* Ct, float* Zt, const float* __restrict__ Cg, uint32_t layer_id,
+                                            int col0, int ncols, int slot0, int d_out, int r, uint64_t seed,
+                                            uint64_t query, int tid) {
+  // elements of the layer's [d_out, r] Z in the column range: e in [col0*r, (col0+ncols)*r)
+  const int valid_cols = max(0, min(ncols, d_out - col0));
+  const int64_t e_begin = (int64_t)col0 * r;
+  const int64_t e_end = e_begin + (int64_t)valid_cols * r;
+  // zero the padded / out-of-range slots first
+  for (int i = tid; i < ncols * RT; i += EPI_THREADS) {
+    const int c = i / RT, j = i % RT;
+    if (c >= valid_cols || j >= r) {
+      Ct[(slot0 + c) * RT + j] = 0.f;
+      Zt[(slot0 + c) * RT + j] = 0.f;
+    }
+  }
+  const int64_t g_begin = e_begin >> 2, g_end = (e_end + 3) >> 2;
+  for (int64_t g = g_begin + tid; g < g_end; g += EPI_THREADS) {
+    const float4 z = z_normals4(seed, layer_id, query, (uint64_t)g);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int64_t e = 4 * g + i;
+      if (e >= e_begin && e < e_end) {
+        const int64_t le = e - e_begin;
+        const int c = (int)(le / r), j = (int)(le % r);
+        Zt[(slot0 + c) * RT + j] = z_select(z, i);
+        Ct[(slot0 + c) * RT + j] = Cg[e];
+      }
+    }
+  }
+}
+
+template <int RT>
+__device__ __forceinline__ void lowrank(const float* Ct, const float* Zt, int slot, const float* p, float& sC,
+                                        float& sZ) {
+  const float4* c4 = reinterpret_cast<const float4*>(Ct + slot * RT);
+  const float4* z4 = reinterpret_cast<const float4*>(Zt + slot * RT);
+  float a = 0.f, b = 0.f;
+#pragma unroll
+  for (int q = 0; q < RT / 4; ++q) {
+    const float4 cv = c4[q];
+    const float4 zv = z4[q];
+    a = fmaf(cv.x, p[4 * q + 0], a); a = fmaf(cv.y, p[4 * q + 1], a);
+    a = fmaf(cv.z, p[4 * q + 2], a); a = fmaf(cv.w, p[4 * q + 3], a);
+    b = fmaf(zv.x, p[4 * q + 0], b); b = fmaf(zv.y, p[4 * q + 1], b);
+    b = fmaf(zv.z, p[4 * q + 2], b); b = fmaf(zv.w, p[4 * q + 3], b);
+  }
+  sC = a;
+  sZ = b;
+}
+
+// The epilogue's wait for a finished accumulator, taken by one thread and
+// shared through a named barrier so that all 128 epilogue threads leave (or
+// continue) together even if the wait gives up.
+__device__ __forceinline__ bool epi_wait_full(SharedState* ss, int buf, uint32_t parity, volatile int* abort_flag,
+                                              int* status, int etid) {
+  if (etid == 0) ss->epi_ok = tc::mbar_wait(tc::smem_u32(&ss->tmem_full[buf]), parity, abort_flag, status) ? 1 : 0;
+  tc::named_bar_sync(2, EPI_THREADS);
+  tc::tc_fence_after();
+  const bool ok = *reinterpret_cast<volatile int*>(&ss->epi_ok) != 0;
+  tc::named_bar_sync(2, EPI_THREADS);   // everyone has read epi_ok before thread 0 may rewrite it
+  return ok;
+}
+
+template <typename TO>
+__device__ __forceinline__ void store16(TO* dst, const float* v, int n_valid) {
+  if (n_valid >= 16) {
+    alignas(16) TO o[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) o[i] = from_f32<TO>(v[i]);
+    uint4* d4 = reinterpret_cast<uint4*>(dst);
+    const uint4* s4 = reinterpret_cast<const uint4*>(o);
+#pragma unroll
+    for (int i = 0; i < (int)(16 * sizeof(TO) / 16); ++i) d4[i] = s4[i];
+  } else {
+    for (int i = 0; i < n_valid; ++i) dst[i] = from_f32<TO>(v[i]);
+  }
+}
+
+template <typename TO, int RT, int MODE, int AB_BF16>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+               const __grid_constant__ CUtensorMap tmB2, const Params prm) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  float* Ct = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);
+  float* Zt = Ct + TABLE_FLOATS;
+  SharedState* ss = reinterpret_cast<SharedState*>(Zt + TABLE_FLOATS);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  volatile int* abort_flag = &ss->abort_flag;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      tc::mbar_init(tc::smem_u32(&ss->full[s]), 1);
+      tc::mbar_init(tc::smem_u32(&ss->empty[s]), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      tc::mbar_init(tc::smem_u32(&ss->tmem_full[b]), 1);
+      tc::mbar_init(tc::smem_u32(&ss->tmem_empty[b]), EPI_THREADS);
+    }
+    tc::mbar_init(tc::smem_u32(&ss->drain), 1);
+    ss->abort_flag = 0;
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&tmA);
+    tc::prefetch_tmap(&tmB);
+    if (MODE == MODE_GATED) tc::prefetch_tmap(&tmB2);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc(tc::smem_u32(&ss->tmem_base), TMEM_COLS);
+    tc::tmem_relinquish();
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem_base = ss->tmem_base;
+
+  const int num_m = prm.num_m, num_n = prm.num_n, num_k = prm.num_k;
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued_mask = 0, issued_parity = 0;   // per stage: a load in flight, and its full-phase parity
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < prm.num_tiles && ok; tile += gridDim.x) {
+        int m_blk, n_blk;
+        tile_coords(tile, num_m, num_n, m_blk, n_blk);
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
+          const uint32_t full = tc::smem_u32(&ss->full[stage]);
+          tc::mbar_arrive_expect_tx(full, STAGE_BYTES);
+          const uint32_t sa = tc::smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t sb = sa + A_BYTES;
+          tc::tma_load_2d(sa, &tmA, kb * BK, m_blk * BM, full);
+          if (MODE == MODE_GATED) {
+            tc::tma_load_2d(sb, &tmB, kb * BK, n_blk * (BN / 2), full);
+            tc::tma_load_2d(sb + B_BYTES / 2, &tmB2, kb * BK, n_blk * (BN / 2), full);
+          } else {
+            tc::tma_load_2d(sb, &tmB, kb * BK, n_blk * BN, full);
+          }
+          issued_mask |= 1u << stage;
+          issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      if (!ok) {
+        // wind down: wait (bounded) for our own copies still in flight
+        for (int s = 0; s < STAGES; ++s)
+          if (issued_mask & (1u << s))
+            tc::mbar_wait_drain(tc::smem_u32(&ss->full[s]), (issued_parity >> s) & 1u, 100000000ull);
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      constexpr uint32_t IDESC = tc::idesc_f16(BM, BN, AB_BF16);
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      int local = 0;
+      bool issued_any = false;
+      for (int tile = blockIdx.x; tile < prm.num_tiles && ok; tile += gridDim.x, ++local) {
+        const int buf = local & 1;
+        const uint32_t acc_phase = (local >> 1) & 1;
+        if (!tc::mbar_wait(tc::smem_u32(&ss->tmem_empty[buf]), acc_phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
+        tc::tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!tc::mbar_wait(tc::smem_u32(&ss->full[stage]), phase, abort_flag, prm.status)) { ok = false; break; }
+          tc::tc_fence_after();
+          const uint32_t sa = tc::smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t sb = sa + A_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            const uint64_t ad = tc::sdesc_k_sw128(sa + k * 32);
+            const uint64_t bd = tc::sdesc_k_sw128(sb + k * 32);
+            tc::mma_f16(d_tmem, ad, bd, IDESC, (kb | k) != 0 ? 1u : 0u);
+          }
+          tc::mma_commit(tc::smem_u32(&ss->empty[stage]));   // frees the stage when these MMAs finish
+          issued_any = true;
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        tc::mma_commit(tc::smem_u32(&ss->tmem_full[buf]));   // accumulator ready for the epilogue
+      }
+      if (issued_any) {
+        // all MMAs issued by this thread complete before TMEM is released
+        tc::mma_commit(tc::smem_u32(&ss->drain));
+        tc::mbar_wait_drain(tc::smem_u32(&ss->drain), 0, 100000000ull);
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5) ----------------
+    const int etid = threadIdx.x - 64;              // 0..127
+    const int quad = warp & 3;                      // TMEM lane quadrant this warp may access
+    const int row_in_tile = quad * 32 + lane;
+    const int r = prm.r;
+    int local = 0;
+    for (int tile = blockIdx.x; tile < prm.num_tiles; tile += gridDim.x, ++local) {
+      int m_blk, n_blk;
+      tile_coords(tile, num_m, num_n, m_blk, n_blk);
+      const int buf = local & 1;
+      const uint32_t acc_phase = (local >> 1) & 1;
+      const int64_t m = (int64_t)m_blk * BM + row_in_tile;
+      const bool row_ok = m < prm.rows;
+      const uint32_t t_row = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * BN);
+
+      if (MODE == MODE_PLAIN) {
+        if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) break;
+        float* D = static_cast<float*>(prm.Y);
+        for (int c0 = 0; c0 < BN; c0 += 16) {
+          float v[16];
+          tc::tmem_ld16(t_row + (uint32_t)c0, v);
+          const int n = n_blk * BN + c0;
+          if (row_ok && n < prm.d_out) {
+            float* dst = D + m * prm.ldy + n;
+            const int nv = min(16, prm.d_out - n);
+            if (nv == 16 && (prm.ldy % 4) == 0) {
+#pragma unroll
+              for (int i = 0; i < 4; ++i)
+                reinterpret_cast<float4*>(dst)[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+            } else {
+              for (int i = 0; i < nv; ++i) dst[i] = v[i];
+            }
+          }
+        }
+        tc::tc_fence_before();
+        tc::mbar_arrive(tc::smem_u32(&ss->tmem_empty[buf]));
+        continue;
+      }
+
+      // ---- pair / gated epilogue ----
+      // table chunks: slots per chunk such that slots * RT <= TABLE_FLOATS
+      constexpr int CHUNK = (TABLE_FLOATS / RT) < BN ? (TABLE_FLOATS / RT) : BN;
+      static_assert(MODE != MODE_GATED || CHUNK == BN, "gated mode keeps the whole tile's table");
+      float p[RT], p2[RT];
+#pragma unroll
+      for (int j = 0; j < RT; ++j) {
+        p[j] = (row_ok && j < r) ? prm.P[m * r + j] : 0.f;
+        p2[j] = (MODE == MODE_GATED && row_ok && j < r) ? prm.P2[m * r + j] : 0.f;
+      }
+      bool ok = true;
+      for (int s0 = 0; s0 < BN && ok; s0 += CHUNK) {
+        tc::named_bar_sync(1, EPI_THREADS);          // previous chunk's readers are done
+        if (MODE == MODE_GATED) {
+          build_table<RT>(Ct, Zt, prm.C, prm.layer_id, n_blk * (BN / 2), BN / 2, 0, prm.d_out, r, prm.seed,
+                          prm.query, etid);
+          build_table<RT>(Ct, Zt, prm.C2, prm.layer_id2, n_blk * (BN / 2), BN / 2, BN / 2, prm.d_out, r,
+                          prm.seed, prm.query, etid);
+        } else {
+          build_table<RT>(Ct, Zt, prm.C, prm.layer_id, n_blk * BN + s0, CHUNK, 0, prm.d_out, r, prm.seed,
+                          prm.query, etid);
+        }
+        tc::named_bar_sync(1, EPI_THREADS);
+        if (s0 == 0) {
+          if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) { ok = false; break; }
+        }
+        if (MODE == MODE_GATED) {
+          TO* Y = static_cast<TO*>(prm.Y);
+          for (int c0 = 0; c0 < BN / 2; c0 += 16) {
+            float g[16], u[16];
+            tc::tmem_ld16(t_row + (uint32_t)c0, g);
+            tc::tmem_ld16(t_row + (uint32_t)(BN / 2 + c0), u);
+            const int n = n_blk * (BN / 2) + c0;
+            if (!row_ok || n >= prm.d_out) continue;
+            float hp[16], hm[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              float gC, gZ, uC, uZ;
+              lowrank<RT>(Ct, Zt, c0 + i, p, gC, gZ);
+              lowrank<RT>(Ct, Zt, BN / 2 + c0 + i, p2, uC, uZ);
+              const float gb = g[i] + gC, ub = u[i] + uC;
+              if (prm.shared) {
+                hp[i] = silu_f(gb + prm.eps * gZ) * (ub + prm.eps * uZ);
+                hm[i] = silu_f(gb - prm.eps * gZ) * (ub - prm.eps * uZ);
+              } else {
+                const float se = m < prm.T ? prm.eps : -prm.eps;
+                hp[i] = silu_f(gb + se * gZ) * (ub + se * uZ);
+              }
+            }
+            const int nv = min(16, prm.d_out - n);
+            store16<TO>(Y + m * prm.d_out + n, hp, nv);
+            if (prm.shared) store16<TO>(Y + (prm.T + m) * prm.d_out + n, hm, nv);
+          }
+        } else {
+          TO* Y = static_cast<TO*>(prm.Y);
+          for (int c0 = s0; c0 < s0 + CHUNK; c0 += 16) {
+            float acc[16];
+            tc::tmem_ld16(t_row + (uint32_t)c0, acc);
+            const int n = n_blk * BN + c0;
+            if (!row_ok || n >= prm.d_out) continue;
+            float yp[16], ym[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              float sC, sZ;
+              lowrank<RT>(Ct, Zt, c0 - s0 + i, p, sC, sZ);
+              const float base = acc[i] + sC;
+              if (prm.shared) {
+                yp[i] = apply_act(base + prm.eps * sZ, prm.act);
+                ym[i] = apply_act(base - prm.eps * sZ, prm.act);
+              } else {
+                const float se = m < prm.T ? prm.eps : -prm.eps;
+                yp[i] = apply_act(base + se * sZ, prm.act);
+              }
+            }
+            const int nv = min(16, prm.d_out - n);
+            store16<TO>(Y + m * prm.d_out + n, yp, nv);
+            if (prm.shared) store16<TO>(Y + (prm.T + m) * prm.d_out + n, ym, nv);
+          }
+        }
+      }
+      if (!ok) break;
+      tc::tc_fence_before();
+      tc::mbar_arrive(tc::smem_u32(&ss->tmem_empty[buf]));
+    }
+  }
+
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tc_fence_after();
+    tc::tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+}  // namespace pairtc
+}  // namespace zoact

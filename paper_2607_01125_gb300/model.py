@@ -1,0 +1,158 @@
+"""ZO steps of the synthetic workloads, chained from libzoact C-ABI calls.
+
+One ZO step (Algorithm 2 with one two-sided query) is
+
+    for every adapted linear, in graph order:  zoact_pair_forward (+ glue ops)
+    zoact_loss_pair   -> L+, L-, D, a  (device memory)
+    zoact_adam_step   -> C, m, v updated with g = a * Z over all layers
+
+with no host synchronisation.  This module only allocates buffers and issues
+the calls; every arithmetic step runs in libzoact's kernels.
+
+Graph wiring (names follow synth.Workload):
+  toy        h = GELU(l1 x) (shared input, GELU fused in the epilogue); y = l2 h
+  llama_mlp  h = silu(gate x) * up x  (one gated call, shared input); y = down h
+  llama/opt  per decoder layer on input h:
+               a = rms(h); q, k, v = Q a, K a, V a
+               o = O rms(q + rep(k) + rep(v));  b = rms(o)
+               llama: h' = down rms(silu(gate b) * up b)
+               opt:   h' = fc2 rms(relu(fc1 b))
+             the first layer's q, k, v see the same input for both signs.
+"""
+import torch
+
+from . import _lib as Z
+
+_TORCH = {"fp32": torch.float32, "bf16": torch.bfloat16, "fp16": torch.float16}
+
+
+class AdaptedLinear:
+    def __init__(self, name, W, U, layer_id, offset, r, w_scales=None, wtype=None, d_in=None):
+        self.name = name
+        self.W = W
+        self.U = U
+        self.w_scales = w_scales
+        self.layer_id = int(layer_id)
+        self.offset = int(offset)
+        self.r = int(r)
+        self.wtype = Z.TORCH_DT[W.dtype] if wtype is None else wtype
+        self.d_out = W.shape[0]
+        self.d_in = int(d_in) if d_in is not None else W.shape[1]
+        self.layer = None
+
+    def bind(self, C):
+        view = C[self.offset:self.offset + self.d_out * self.r]
+        self.layer = Z.make_layer(self.W, self.U, view, self.layer_id, w_scales=self.w_scales, wtype=self.wtype,
+                                  d_in=self.d_in)
+
+
+class ZOStep:
+    """Holds frozen weights/bases, the coefficient arenas and activation buffers."""
+
+    def __init__(self, ctx, kind, linears, T, act_dtype, eps=1e-3, lr=1e-4, beta1=0.9, beta2=0.999,
+                 adam_eps=1e-8, n_heads=32, n_kv_heads=8, head_dim=128):
+        self.ctx = ctx
+        self.kind = kind
+        self.T = int(T)
+        self.dtype = _TORCH[act_dtype] if isinstance(act_dtype, str) else act_dtype
+        self.eps, self.lr, self.beta1, self.beta2, self.adam_eps = eps, lr, beta1, beta2, adam_eps
+        self.n_rep = n_heads // n_kv_heads if kind == "llama" else 1
+        self.head_dim = head_dim
+        self.linears = linears                      # list of AdaptedLinear, forward order
+        self.by_name = {l.name: l for l in linears}
+        dev = linears[0].W.device
+        n = max(l.offset + l.d_out * l.r for l in linears)
+        n = (n + 3) // 4 * 4
+        self.C = torch.zeros(n, dtype=torch.float32, device=dev)
+        self.m = torch.zeros_like(self.C)
+        self.v = torch.zeros_like(self.C)
+        for l in linears:
+            l.bind(self.C)
+        self.blocks = [(l.offset, l.d_out, l.r, l.layer_id) for l in linears]
+        self.loss_out = torch.zeros(4, dtype=torch.float64, device=dev)
+        self._bufs = {}
+        self.device = dev
+
+    # ---- buffers ----
+    def buf(self, key, rows, cols):
+        t = self._bufs.get(key)
+        if t is None or t.shape != (rows, cols):
+            t = torch.empty(rows, cols, dtype=self.dtype, device=self.device)
+            self._bufs[key] = t
+        return t
+
+    def pair(self, name, X, shared, seed, query, out_key, act=Z.ACT_NONE):
+        l = self.by_name[name]
+        Y = self.buf(out_key, 2 * self.T, l.d_out)
+        Z.zoact_pair_forward(self.ctx, l.layer, X, self.T, shared, self.eps, seed, query, Y, act=act)
+        return Y
+
+    # ---- forward graphs ----
+    def forward(self, x, seed, query):
+        T = self.T
+        if self.kind == "toy":
+            h = self.pair("l1", x, True, seed, query, "h", act=Z.ACT_GELU)
+            return self.pair("l2", h, False, seed, query, "y")
+        if self.kind == "llama_mlp":
+            g, u = self.by_name["gate"], self.by_name["up"]
+            H = self.buf("h", 2 * T, g.d_out)
+            Z.zoact_pair_forward_gated(self.ctx, g.layer, u.layer, x, T, True, self.eps, seed, query, H)
+            return self.pair("down", H, False, seed, query, "y")
+        return self._stack(x, seed, query)
+
+    def _stack(self, x, seed, query):
+        T = self.T
+        n_dec = len(self.linears) // (7 if self.kind == "llama" else 6)
+        h = x
+        shared = True
+        for L in range(n_dec):
+            rows = T if shared else 2 * T
+            a = self.buf(f"a{rows}", rows, h.shape[1])
+            Z.zoact_rms_norm(self.ctx, h, a)
+            q = self.pair(f"{L}.q", a, shared, seed, query, "q")
+            k = self.pair(f"{L}.k", a, shared, seed, query, "k")
+            v = self.pair(f"{L}.v", a, shared, seed, query, "v")
+            shared = False
+            mix = self.buf("mix", 2 * T, q.shape[1])
+            Z.zoact_mix_rms(self.ctx, q, k, v, mix, self.n_rep if self.kind == "llama" else 1, self.head_dim)
+            o = self.pair(f"{L}.o", mix, False, seed, query, "o")
+            b = self.buf("b", 2 * T, o.shape[1])
+            Z.zoact_rms_norm(self.ctx, o, b)
+            if self.kind == "llama":
+                g, u = self.by_name[f"{L}.gate"], self.by_name[f"{L}.up"]
+                H = self.buf("hmlp", 2 * T, g.d_out)
+                Z.zoact_pair_forward_gated(self.ctx, g.layer, u.layer, b, T, False, self.eps, seed, query, H)
+                Hn = self.buf("hmlp_n", 2 * T, g.d_out)
+                Z.zoact_rms_norm(self.ctx, H, Hn)
+                h = self.pair(f"{L}.down", Hn, False, seed, query, "h" if L % 2 == 0 else "h2")
+            else:
+                f = self.pair(f"{L}.fc1", b, False, seed, query, "f", act=Z.ACT_RELU)
+                fn = self.buf("f_n", 2 * T, f.shape[1])
+                Z.zoact_rms_norm(self.ctx, f, fn)
+                h = self.pair(f"{L}.fc2", fn, False, seed, query, "h" if L % 2 == 0 else "h2")
+        return h
+
+    # ---- loss and update ----
+    def loss(self, Y, target):
+        Z.zoact_loss_pair(self.ctx, Y, self.T, self.eps, self.loss_out, target=target)
+        return self.loss_out
+
+    def update(self, step, seed, query, lr=None):
+        Z.zoact_adam_step(self.ctx, self.C, self.m, self.v, self.blocks, self.loss_out,
+                          self.lr if lr is None else lr, self.beta1, self.beta2, self.adam_eps, step, seed, query)
+
+    def step(self, x, target, step, seed, query, lr=None):
+        """One ZO step: pair forwards, loss pair, Adam.  Returns the device loss tensor [L+, L-, D, a]."""
+        Y = self.forward(x, seed, query)
+        self.loss(Y, target)
+        self.update(step, seed, query, lr)
+        return self.loss_out
+
+
+def coefficient_offsets(specs, r):
+    """Offsets (multiples of 4) of each layer's [d_out, r] block in the flat arena."""
+    offs, cur = [], 0
+    for s in specs:
+        offs.append(cur)
+        cur += (s.d_out * r + 3) // 4 * 4
+    return offs

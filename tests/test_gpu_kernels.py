@@ -1,0 +1,277 @@
+"""GPU parity of each libzoact kernel against the CPU oracle, through the C ABI.
+
+Inputs come from synth (seeded); both sides read the same stored values.
+Tolerances (written per test):
+  * Philox words and index bookkeeping: bit-exact.
+  * fp32 normals: |dz| <= 1e-6 (1 + |z|)  (fp32 logf/sqrtf/sincospif vs fp64 libm).
+  * fp32 arithmetic paths: <= 1e-4 of the output scale, and a per-element bound
+    from the fp32 accumulation error (c * eps32 * sum |terms|).
+  * 16-bit outputs: the bf16/fp16 rounding of the output (2^-8 / 2^-11 relative)
+    on top of the fp32 bound; the bar is 2e-2 relative.
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2607_01125_gb300 as zo
+from oracle import philox, layers, loss as oloss, optim, basis, graphs
+from synth import normal, lowrank_activations
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    c = zo.Context(0)
+    yield c
+    assert c.device_status() == 0
+    c.close()
+
+
+def np64(t):
+    return t.detach().double().cpu().numpy()
+
+
+# ---------------- Z ----------------
+@pytest.mark.parametrize("seed,layer,query,n", [(0, 0, 0, 4096), (0xDEADBEEF12345678, 77, (3 << 32) | 5, 1001),
+                                                (1, 2**32 - 1, 2**64 - 1, 13)])
+def test_philox_bit_exact_and_normals(ctx, seed, layer, query, n):
+    z = torch.empty(n, dtype=torch.float32, device=DEV)
+    w = torch.empty(n, dtype=torch.int32, device=DEV)
+    zo.zoact_philox_normals(ctx, seed, layer, query, n, z, w)
+    torch.cuda.synchronize()
+    words = w.cpu().numpy().view(np.uint32).astype(np.uint64)
+    assert np.array_equal(words, philox.stream_words(seed, layer, query, n))
+    zr = philox.normals(seed, layer, query, n)
+    zg = np64(z)
+    assert np.all(np.abs(zg - zr) <= 1e-6 * (1.0 + np.abs(zr)))
+
+
+# ---------------- projection ----------------
+@pytest.mark.parametrize("rows,d_in,r,dt", [(300, 1000, 16, torch.bfloat16), (64, 256, 8, torch.float32),
+                                            (1000, 4096, 32, torch.float16), (7, 40, 3, torch.bfloat16),
+                                            (2048, 14336, 16, torch.bfloat16)])
+def test_lowrank_proj(ctx, rows, d_in, r, dt):
+    X = normal((rows, d_in), 1, DEV, dtype=dt)
+    U = normal((d_in, r), 2, DEV) / np.sqrt(d_in)
+    P = torch.empty(rows, r, dtype=torch.float32, device=DEV)
+    zo.zoact_lowrank_proj(ctx, X, U, P)
+    torch.cuda.synchronize()
+    Xn, Un = np64(X), np64(U)
+    ref = Xn @ Un
+    bound = 4 * d_in ** 0.5 * 2.0 ** -24 * (np.abs(Xn) @ np.abs(Un)) + 1e-30
+    assert np.all(np.abs(np64(P) - ref) <= bound + 1e-6 * np.abs(ref))
+
+
+# ---------------- pair forward ----------------
+def _pair_case(d_in, d_out, r, T, shared, dt, eps, c_scale, seed=0):
+    X = normal(((T if shared else 2 * T), d_in), seed + 1, DEV, dtype=dt)
+    W = normal((d_out, d_in), seed + 2, DEV, std=d_in ** -0.5, dtype=dt)
+    U = normal((d_in, r), seed + 3, DEV) / np.sqrt(d_in)
+    C = normal((d_out * r,), seed + 4, DEV, std=c_scale)
+    return X, W, U, C
+
+
+def _oracle_pair(X, W, U, C, eps, T, shared, seed, layer_id, query, d_out, r):
+    Zm = philox.perturbation(seed, layer_id, query, d_out, r)
+    Y = layers.pair_forward(np64(W), np64(U), np64(C).reshape(d_out, r), Zm, np64(X), eps, T, shared)
+    Xn, Wn, Un = np64(X), np64(W), np64(U)
+    if shared:
+        Xn = np.concatenate([Xn, Xn])
+    absb = np.abs(Xn) @ np.abs(Wn).T + (np.abs(Xn @ Un)) @ (np.abs(np64(C).reshape(d_out, r)) + abs(eps) * np.abs(Zm)).T
+    return Y, absb
+
+
+@pytest.mark.parametrize("d_in,d_out,r,T,shared,dt", [
+    (256, 256, 8, 64, True, torch.float32),
+    (256, 200, 8, 37, False, torch.float32),
+    (1000, 520, 16, 200, False, torch.bfloat16),     # 4 M tiles (ragged), 3 N tiles (ragged), ragged K
+    (1024, 768, 16, 96, True, torch.bfloat16),       # shared input: 1 M tile, both signs written
+    (512, 264, 4, 130, False, torch.float16),        # stacked rows cross a tile with both signs
+    (4096, 1024, 32, 128, False, torch.bfloat16),    # rank 32: epilogue table in two chunks
+    (320, 128, 1, 20, True, torch.bfloat16),         # rank 1
+])
+def test_pair_forward_fp32_out(ctx, d_in, d_out, r, T, shared, dt):
+    # eps = 0.5 and |C| ~ 0.3 make the low-rank term visible at fp32 precision
+    eps, seed, query, layer_id = 0.5, 11, 7, 5
+    X, W, U, C = _pair_case(d_in, d_out, r, T, shared, dt, eps, 0.3)
+    Y = torch.empty(2 * T, d_out, dtype=torch.float32, device=DEV)
+    L = zo.make_layer(W, U, C, layer_id)
+    zo.zoact_pair_forward(ctx, L, X, T, shared, eps, seed, query, Y)
+    torch.cuda.synchronize()
+    ref, absb = _oracle_pair(X, W, U, C, eps, T, shared, seed, layer_id, query, d_out, r)
+    err = np.abs(np64(Y) - ref)
+    assert np.all(err <= 8 * np.sqrt(d_in) * 2.0 ** -24 * absb + 1e-6), err.max()
+    assert err.max() <= 1e-4 * np.abs(ref).max()
+
+
+@pytest.mark.parametrize("d_in,d_out,r,T,shared,dt,act", [
+    (1000, 520, 16, 200, False, torch.bfloat16, zo.ACT_NONE),
+    (1024, 768, 8, 96, True, torch.bfloat16, zo.ACT_RELU),
+    (512, 264, 16, 130, False, torch.float16, zo.ACT_GELU),
+    (256, 256, 8, 64, True, torch.float32, zo.ACT_GELU),
+])
+def test_pair_forward_16bit_out_and_acts(ctx, d_in, d_out, r, T, shared, dt, act):
+    eps, seed, query, layer_id = 1e-3, 3, 1, 9
+    X, W, U, C = _pair_case(d_in, d_out, r, T, shared, dt, eps, 0.05)
+    Y = torch.empty(2 * T, d_out, dtype=dt, device=DEV)
+    L = zo.make_layer(W, U, C, layer_id)
+    zo.zoact_pair_forward(ctx, L, X, T, shared, eps, seed, query, Y, act=act)
+    torch.cuda.synchronize()
+    ref, absb = _oracle_pair(X, W, U, C, eps, T, shared, seed, layer_id, query, d_out, r)
+    ref = {zo.ACT_NONE: lambda y: y, zo.ACT_RELU: layers.relu, zo.ACT_GELU: layers.gelu_erf}[act](ref)
+    rel = {torch.bfloat16: 2.0 ** -8, torch.float16: 2.0 ** -11, torch.float32: 2.0 ** -23}[dt]
+    err = np.abs(np64(Y) - ref)
+    assert np.all(err <= rel * np.abs(ref) + 8 * np.sqrt(d_in) * 2.0 ** -24 * absb + 1e-6)
+    assert err.max() <= 2e-2 * np.abs(ref).max()
+
+
+def test_pair_difference_isolates_the_perturbation(ctx):
+    # y+ - y- = 2 eps Z p exactly in the definition; fp32 output keeps it visible at eps = 1e-3
+    d_in, d_out, r, T = 768, 512, 16, 64
+    eps, seed, query, lid = 1e-3, 5, 2, 3
+    X, W, U, C = _pair_case(d_in, d_out, r, T, True, torch.bfloat16, eps, 0.1)
+    Y = torch.empty(2 * T, d_out, dtype=torch.float32, device=DEV)
+    zo.zoact_pair_forward(ctx, zo.make_layer(W, U, C, lid), X, T, True, eps, seed, query, Y)
+    torch.cuda.synchronize()
+    Yn = np64(Y)
+    Zm = philox.perturbation(seed, lid, query, d_out, r)
+    ref = 2 * eps * (np64(X) @ np64(U)) @ Zm.T
+    # the accumulator is common to both halves, so the difference carries only epilogue rounding
+    assert np.abs((Yn[:T] - Yn[T:]) - ref).max() <= 1e-6 * np.abs(Yn).max()
+
+
+@pytest.mark.parametrize("T,shared,dt", [(96, True, torch.bfloat16), (70, False, torch.bfloat16)])
+def test_pair_forward_gated(ctx, T, shared, dt):
+    d_in, d_out, r = 512, 400, 16
+    eps, seed, query = 0.25, 8, 4
+    X = normal(((T if shared else 2 * T), d_in), 21, DEV, dtype=dt)
+    Wg = normal((d_out, d_in), 22, DEV, std=d_in ** -0.5, dtype=dt)
+    Wu = normal((d_out, d_in), 23, DEV, std=d_in ** -0.5, dtype=dt)
+    Ug = normal((d_in, r), 24, DEV) / np.sqrt(d_in)
+    Uu = normal((d_in, r), 25, DEV) / np.sqrt(d_in)
+    Cg = normal((d_out * r,), 26, DEV, std=0.2)
+    Cu = normal((d_out * r,), 27, DEV, std=0.2)
+    H = torch.empty(2 * T, d_out, dtype=torch.float32, device=DEV)
+    zo.zoact_pair_forward_gated(ctx, zo.make_layer(Wg, Ug, Cg, 0), zo.make_layer(Wu, Uu, Cu, 1), X, T, shared,
+                                eps, seed, query, H)
+    torch.cuda.synchronize()
+    g, _ = _oracle_pair(X, Wg, Ug, Cg, eps, T, shared, seed, 0, query, d_out, r)
+    u, _ = _oracle_pair(X, Wu, Uu, Cu, eps, T, shared, seed, 1, query, d_out, r)
+    ref = layers.silu(g) * u
+    assert np.abs(np64(H) - ref).max() <= 1e-4 * np.abs(ref).max()
+
+
+# ---------------- loss ----------------
+@pytest.mark.parametrize("T,n,dt,with_target", [(64, 256, torch.float32, True), (2048, 4096, torch.bfloat16, True),
+                                                (33, 7, torch.bfloat16, False), (300, 1000, torch.float16, True)])
+def test_loss_pair(ctx, T, n, dt, with_target):
+    Y = normal((2 * T, n), 31, DEV, dtype=dt)
+    Y[T:] = (Y[:T].float() + 1e-2 * normal((T, n), 32, DEV)).to(dt)   # close pair: D << L
+    tgt = normal((T, n), 33, DEV, dtype=dt) if with_target else None
+    out = torch.zeros(4, dtype=torch.float64, device=DEV)
+    zo.zoact_loss_pair(ctx, Y, T, 1e-3, out, target=tgt)
+    torch.cuda.synchronize()
+    Lp, Lm, D, a = oloss.loss_pair(np64(Y), T, None if tgt is None else np64(tgt), 1e-3)
+    o = out.cpu().numpy()
+    assert o[0] == pytest.approx(Lp, rel=1e-5) and o[1] == pytest.approx(Lm, rel=1e-5)
+    assert o[2] == pytest.approx(D, rel=1e-4, abs=1e-7 * Lp)
+    assert o[3] == pytest.approx(a, rel=1e-4, abs=1e-7 * Lp / 2e-3)
+    assert np.sign(o[3]) == np.sign(a)
+
+
+# ---------------- Adam / SGD ----------------
+def test_adam_step_over_blocks(ctx):
+    specs = [(0, 256, 8, 0), (2048, 100, 3, 7), (2352, 14336, 16, 2)]     # (offset, d_out, r, layer_id)
+    n = 2352 + 14336 * 16
+    C = normal((n,), 41, DEV, std=0.1)
+    m = normal((n,), 42, DEV, std=0.01)
+    v = normal((n,), 43, DEV, std=0.01).abs()
+    C0, m0, v0 = np64(C), np64(m), np64(v)
+    out = torch.tensor([1.0, 0.5, 0.5, 0.73], dtype=torch.float64, device=DEV)
+    seed, query, step, lr = 99, 12, 3, 1e-3
+    zo.zoact_adam_step(ctx, C, m, v, specs, out, lr, 0.9, 0.999, 1e-8, step, seed, query)
+    torch.cuda.synchronize()
+    Cr, mr, vr = C0.copy(), m0.copy(), v0.copy()
+    # the ABI carries lr, betas and eps as fp32: the oracle reads those stored values
+    f32 = lambda x: float(np.float32(x))
+    for off, d_out, r, lid in specs:
+        sl = slice(off, off + d_out * r)
+        g = optim.zo_gradient(0.73, philox.perturbation(seed, lid, query, d_out, r).reshape(-1))
+        Cr[sl], mr[sl], vr[sl] = optim.adam_step(C0[sl], m0[sl], v0[sl], g, f32(lr), f32(0.9), f32(0.999),
+                                                 f32(1e-8), step)
+    np.testing.assert_allclose(np64(m), mr, rtol=1e-5, atol=1e-7)
+    np.testing.assert_allclose(np64(v), vr, rtol=1e-5, atol=1e-9)
+    np.testing.assert_allclose(np64(C), Cr, rtol=1e-4, atol=1e-6 * lr)
+    # elements between blocks (2348 .. 2351) are untouched
+    np.testing.assert_array_equal(np64(C)[2348:2352], C0[2348:2352])
+    np.testing.assert_array_equal(np64(m)[2348:2352], m0[2348:2352])
+
+
+def test_sgd_and_nonfinite_guard(ctx):
+    specs = [(0, 64, 4, 5)]
+    C = normal((256,), 51, DEV)
+    C0 = np64(C)
+    out = torch.tensor([0, 0, 0, -2.0], dtype=torch.float64, device=DEV)
+    zo.zoact_sgd_step(ctx, C, specs, out, 0.01, 3, 4)
+    torch.cuda.synchronize()
+    ref = optim.sgd_step(C0, optim.zo_gradient(-2.0, philox.perturbation(3, 5, 4, 64, 4).reshape(-1)),
+                         float(np.float32(0.01)))
+    np.testing.assert_allclose(np64(C), ref, rtol=1e-6, atol=1e-7)
+    # a NaN estimator leaves C alone and raises the device status
+    before = C.clone()
+    out[3] = float("nan")
+    zo.zoact_sgd_step(ctx, C, specs, out, 0.01, 3, 5)
+    assert ctx.device_status(reset=True) == zo._lib.ZOACT_ERR_NONFINITE
+    assert torch.equal(C, before)
+
+
+# ---------------- glue ----------------
+def test_rms_norm_and_mix(ctx):
+    rows, n = 37, 4096
+    X = normal((rows, n), 61, DEV, dtype=torch.bfloat16)
+    Y = torch.empty_like(X)
+    zo.zoact_rms_norm(ctx, X, Y)
+    q = normal((rows, n), 62, DEV, dtype=torch.bfloat16)
+    k = normal((rows, 1024), 63, DEV, dtype=torch.bfloat16)
+    v = normal((rows, 1024), 64, DEV, dtype=torch.bfloat16)
+    M = torch.empty_like(q)
+    zo.zoact_mix_rms(ctx, q, k, v, M, 4, 128)
+    torch.cuda.synchronize()
+    ref = layers.rms_norm(np64(X))
+    assert np.all(np.abs(np64(Y) - ref) <= 2.0 ** -8 * np.abs(ref) + 1e-5)
+    mix = np64(q) + layers.repeat_kv(np64(k), 8, 4, 128) + layers.repeat_kv(np64(v), 8, 4, 128)
+    ref = layers.rms_norm(mix)
+    assert np.all(np.abs(np64(M) - ref) <= 2.0 ** -8 * np.abs(ref) + 1e-5)
+
+
+# ---------------- basis ----------------
+def test_basis_fp32_matches_oracle_iteration_and_eigenspace(ctx):
+    n, d, r, p, iters, seed = 512, 256, 8, 8, 8, 17
+    X, _ = lowrank_activations(n, d, 16, 0.1, 71, DEV, dtype=torch.float32, unit_rms=False, noise_is_energy=False)
+    U = torch.empty(d, r, dtype=torch.float32, device=DEV)
+    ev = torch.empty(r + p, dtype=torch.float32, device=DEV)
+    zo.zoact_basis_init(ctx, X, r, U, oversample=p, n_iter=iters, seed=seed, evals_out=ev)
+    torch.cuda.synchronize()
+    Xn = np64(X)
+    Ui, theta = basis.subspace_iteration(basis.gram(Xn), r, p, iters, seed)
+    Ue, evals = basis.top_r_basis(Xn, r)
+    Ug = np64(U)
+    np.testing.assert_allclose(Ug.T @ Ug, np.eye(r), atol=1e-5)
+    assert basis.subspace_overlap(Ug, Ue) >= 1 - 1e-6
+    np.testing.assert_allclose(Ug, Ui, atol=1e-4)
+    np.testing.assert_allclose(np64(ev)[:r], evals[:r], rtol=1e-4)
+
+
+def test_basis_bf16_tensor_core_gram(ctx):
+    n, d, r = 1000, 1024, 16
+    X, _ = lowrank_activations(n, d, 32, 0.05, 72, DEV, dtype=torch.bfloat16)
+    U = torch.empty(d, r, dtype=torch.float32, device=DEV)
+    zo.zoact_basis_init(ctx, X, r, U, oversample=16, n_iter=10, seed=1)
+    torch.cuda.synchronize()
+    Ue, evals = basis.top_r_basis(np64(X), r)
+    gap = (evals[r - 1] - evals[r]) / evals[0]
+    ov = basis.subspace_overlap(np64(U), Ue)
+    # Davis-Kahan: sin(theta) <~ ||E|| / gap, with E the fp32 Gram error (~1e-6 relative)
+    assert ov >= 1 - (1e-5 / gap) ** 2 - 1e-6, (ov, gap)
