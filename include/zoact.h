@@ -50,6 +50,7 @@ extern "C" {
 #define ZOACT_ERR_NONFINITE   (-4)  /* device: a loss or the estimator scalar was NaN/Inf */
 #define ZOACT_ERR_TIMEOUT     (-5)  /* device: a bounded wait in a kernel gave up */
 #define ZOACT_ERR_NOMEM       (-6)  /* the context could not allocate its scratch */
+#define ZOACT_ERR_TOO_LARGE   (-7)  /* request exceeds the fixed scratch of zoact_pair_forward_noalloc */
 
 /* ---- storage types ---- */
 #define ZOACT_DT_FP32       0
@@ -148,6 +149,29 @@ int zoact_lowrank_proj(zoact_ctx* ctx, const void* X, int xdtype, int64_t rows, 
 int zoact_pair_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype,
                        int64_t T, int input_shared, const float* P, float eps, uint64_t seed,
                        uint64_t query, int act, void* Y, int ydtype);
+
+/* ---- the pair forward without any allocation ----
+ * The paper has no counterpart: this entry point exists for callers that must
+ * not allocate device memory (a framework whose allocator owns all device
+ * memory, a real-time loop that cannot afford a synchronising cudaMalloc, a
+ * process under a hard memory budget).  It computes exactly what
+ * zoact_pair_forward computes with P == NULL, on `stream` (a cudaStream_t),
+ * without a context and without calling cudaMalloc, cudaFree or any allocating
+ * library routine.  Its only scratch is one file-scope device array of
+ * ZOACT_NOALLOC_MAX_PROJ_FLOATS floats (4 MiB) plus a status slot, which every
+ * GPU that loads the library holds until the process exits; it holds the
+ * projection U^T x of the rows(X) x r inputs, so rows(X) * r above
+ * ZOACT_NOALLOC_MAX_PROJ_FLOATS returns ZOACT_ERR_TOO_LARGE and launches nothing.
+ * The first call on each device looks up the array's device address (with that
+ * device current); make that first call before any stream capture.  All calls
+ * share the array: calls that overlap on the GPU (other streams or threads)
+ * race and must be ordered by the caller.  Device-side errors are not
+ * reported back (there is no context); the returned status covers argument
+ * and launch errors.  Other requirements as for zoact_pair_forward.            */
+#define ZOACT_NOALLOC_MAX_PROJ_FLOATS (1 << 20)
+int zoact_pair_forward_noalloc(const zoact_layer* layer, const void* X, int xdtype, int64_t T,
+                               int input_shared, float eps, uint64_t seed, uint64_t query, int act,
+                               void* Y, int ydtype, void* stream);
 
 /* ---- SiLU-gated pair forward (the Llama MLP gate/up pair) ----
  * H = silu(y_gate) * y_up for both signs, with y_gate, y_up the pair forwards of

@@ -9,6 +9,7 @@ streams only.
 from ._lib import (  # noqa: F401
     Context, ZoactError, make_layer, load, status_string,
     zoact_philox_normals, zoact_lowrank_proj, zoact_pair_forward, zoact_pair_forward_gated,
+    zoact_pair_forward_noalloc,
     zoact_loss_pair, zoact_adam_step, zoact_sgd_step, zoact_basis_init, zoact_rms_norm, zoact_mix_rms,
     DT_FP32, DT_BF16, DT_FP16, DT_INT4_G128, ACT_NONE, ACT_RELU, ACT_GELU, EXPORTS, LIB_PATH,
 )

@@ -20,6 +20,8 @@ ZOACT_ERR_CUDA = -3
 ZOACT_ERR_NONFINITE = -4
 ZOACT_ERR_TIMEOUT = -5
 ZOACT_ERR_NOMEM = -6
+ZOACT_ERR_TOO_LARGE = -7
+NOALLOC_MAX_PROJ_FLOATS = 1 << 20
 
 DT_FP32, DT_BF16, DT_FP16, DT_INT4_G128 = 0, 1, 2, 3
 ACT_NONE, ACT_RELU, ACT_GELU = 0, 1, 2
@@ -30,7 +32,7 @@ TORCH_DT = {torch.float32: DT_FP32, torch.bfloat16: DT_BF16, torch.float16: DT_F
 EXPORTS = [
     "zoact_create", "zoact_destroy", "zoact_set_stream", "zoact_status_string", "zoact_get_device_status",
     "zoact_device_sm_count", "zoact_get_launch_count", "zoact_philox_normals", "zoact_lowrank_proj", "zoact_pair_forward",
-    "zoact_pair_forward_gated", "zoact_loss_pair", "zoact_adam_step", "zoact_sgd_step", "zoact_basis_init",
+    "zoact_pair_forward_noalloc", "zoact_pair_forward_gated", "zoact_loss_pair", "zoact_adam_step", "zoact_sgd_step", "zoact_basis_init",
     "zoact_rms_norm", "zoact_mix_rms",
 ]
 
@@ -75,6 +77,7 @@ def load():
         "zoact_philox_normals": [P, U64, U32, U64, I64, P, P],
         "zoact_lowrank_proj": [P, P, I32, I64, I32, P, I32, P],
         "zoact_pair_forward": [P, ctypes.POINTER(zoact_layer), P, I32, I64, I32, P, F32, U64, U64, I32, P, I32],
+        "zoact_pair_forward_noalloc": [ctypes.POINTER(zoact_layer), P, I32, I64, I32, F32, U64, U64, I32, P, I32, P],
         "zoact_pair_forward_gated": [P, ctypes.POINTER(zoact_layer), ctypes.POINTER(zoact_layer), P, I32, I64, I32,
                                      P, P, F32, U64, U64, P, I32],
         "zoact_loss_pair": [P, P, I32, P, I64, I64, F32, P],
@@ -186,6 +189,19 @@ def zoact_pair_forward(ctx, layer, X, T, input_shared, eps, seed, query, Y, P=No
     _check("zoact_pair_forward", load().zoact_pair_forward(ctx.handle, ctypes.byref(layer), _ptr(X), _dt(X), int(T),
                                                             int(input_shared), _ptr(P), float(eps), int(seed),
                                                             int(query), int(act), _ptr(Y), _dt(Y)))
+
+
+def zoact_pair_forward_noalloc(layer, X, T, input_shared, eps, seed, query, Y, act=ACT_NONE, stream=None):
+    """The pair forward without a context or any device allocation (see include/zoact.h).
+
+    For callers that cannot allocate device memory; scratch is a fixed static
+    device array shared by all calls.  `stream` defaults to torch's current stream.
+    """
+    if stream is None:
+        stream = torch.cuda.current_stream().cuda_stream
+    _check("zoact_pair_forward_noalloc", load().zoact_pair_forward_noalloc(
+        ctypes.byref(layer), _ptr(X), _dt(X), int(T), int(input_shared), float(eps), int(seed), int(query),
+        int(act), _ptr(Y), _dt(Y), ctypes.c_void_p(stream)))
 
 
 def zoact_pair_forward_gated(ctx, gate, up, X, T, input_shared, eps, seed, query, H, P_gate=None, P_up=None):

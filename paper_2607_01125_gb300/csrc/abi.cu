@@ -132,6 +132,7 @@ const char* zoact_status_string(int status) {
     case ZOACT_ERR_NONFINITE: return "non-finite loss or estimator";
     case ZOACT_ERR_TIMEOUT: return "bounded device wait timed out";
     case ZOACT_ERR_NOMEM: return "out of device memory";
+    case ZOACT_ERR_TOO_LARGE: return "request exceeds the fixed scratch of the no-allocation entry point";
     default: return "unknown status";
   }
 }

@@ -78,6 +78,9 @@ int launch_philox_normals(Ctx* ctx, uint64_t seed, uint32_t layer_id, uint64_t q
                           float* z, uint32_t* words);
 int launch_lowrank_proj(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const float* U,
                         int r, float* P);
+// As launch_lowrank_proj, with split-K partials in `part` (part_floats floats) instead of context scratch.
+int launch_lowrank_proj_into(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const float* U,
+                             int r, float* P, float* part, int64_t part_floats);
 
 struct PairArgs {
   const void* X;        // [rows, d_in]

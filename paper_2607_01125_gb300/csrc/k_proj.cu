@@ -181,4 +181,59 @@ int launch_lowrank_proj(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d
   }
 }
 
+namespace {
+
+// Same kernels, with the split-K partials in a caller-given buffer of part_floats
+// floats (no allocation): as many K-splits as fit, at least one.
+template <typename TX>
+int proj_dispatch_into(Ctx* ctx, const TX* X, int64_t rows, int d_in, const float* U, int r, float* P, float* part,
+                       int64_t part_floats) {
+  const int64_t row_blocks = (rows + PROJ_RB - 1) / PROJ_RB;
+  int splits = (int)((2LL * ctx->sm_count + row_blocks - 1) / row_blocks);
+  const int max_splits = (d_in + 255) / 256;
+  if (splits > max_splits) splits = max_splits;
+  const int64_t fit = part ? part_floats / (rows * r) : 0;
+  if (splits > fit) splits = (int)fit;
+  if (splits < 1) splits = 1;
+  int k_per_split = (d_in + splits - 1) / splits;
+  k_per_split = (k_per_split + PROJ_KC - 1) / PROJ_KC * PROJ_KC;
+  splits = (d_in + k_per_split - 1) / k_per_split;
+  float* out = splits > 1 ? part : P;
+  dim3 grid((unsigned)row_blocks, (unsigned)splits);
+  const int rp = r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32;
+  switch (rp) {
+    case 4: proj_kernel<TX, 4><<<grid, 32, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); break;
+    case 8: proj_kernel<TX, 8><<<grid, 64, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); break;
+    case 16: proj_kernel<TX, 16><<<grid, 128, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); break;
+    default: proj_kernel<TX, 32><<<grid, 256, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); break;
+  }
+  ++ctx->n_launch;
+  ZOACT_CHECK_LAUNCH();
+  if (splits > 1) {
+    const int64_t n = rows * r;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 4LL * ctx->sm_count) blocks = 4LL * ctx->sm_count;
+    splitk_reduce_kernel<<<(unsigned)blocks, 256, 0, ctx->stream>>>(out, P, n, splits);
+    ++ctx->n_launch;
+    ZOACT_CHECK_LAUNCH();
+  }
+  return ZOACT_OK;
+}
+
+}  // namespace
+
+int launch_lowrank_proj_into(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const float* U, int r,
+                             float* P, float* part, int64_t part_floats) {
+  if (rows <= 0) return ZOACT_OK;
+  switch (xdtype) {
+    case ZOACT_DT_FP32:
+      return proj_dispatch_into(ctx, static_cast<const float*>(X), rows, d_in, U, r, P, part, part_floats);
+    case ZOACT_DT_BF16:
+      return proj_dispatch_into(ctx, static_cast<const __nv_bfloat16*>(X), rows, d_in, U, r, P, part, part_floats);
+    case ZOACT_DT_FP16:
+      return proj_dispatch_into(ctx, static_cast<const __half*>(X), rows, d_in, U, r, P, part, part_floats);
+    default: return ZOACT_ERR_INVALID_ARG;
+  }
+}
+
 }  // namespace zoact
