@@ -81,6 +81,8 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   p.num_k = (a.d_in + BK - 1) / BK;
   p.num_tiles = p.num_m * p.num_n;
   p.ldy = a.d_out;
+  auto al16 = [](const void* q) { return q == nullptr || ((uintptr_t)q & 15u) == 0; };
+  p.vec_ok = al16(a.C) && al16(a.C2) && al16(a.P) && al16(a.P2);
   p.status = ctx->d_status;
   const int mode = gated ? MODE_GATED : MODE_PAIR;
   return a.xdtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p)
@@ -103,6 +105,7 @@ int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int
   p.num_k = (K + BK - 1) / BK;
   p.num_tiles = p.num_m * p.num_n;
   p.ldy = N;
+  p.vec_ok = (N % 4) == 0 && ((uintptr_t)D & 15u) == 0;
   p.status = ctx->d_status;
   return dtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, MODE_PLAIN, 4, ZOACT_DT_FP32, ma, mb, mb, p)
                                 : dispatch_fp16(ctx, MODE_PLAIN, 4, ZOACT_DT_FP32, ma, mb, mb, p);

@@ -9,16 +9,19 @@
 // layer, or gate/up of an MLP) the product is computed once and each
 // accumulator row is written twice.
 //
-// Structure (one persistent CTA per SM, 192 threads):
+// Structure (one persistent CTA per SM, 320 threads):
 //   warp 0      TMA producer: X and W tiles (128x64 and 256x64, bf16/fp16,
 //               128-byte swizzle) into a 4-stage shared-memory ring;
 //   warp 1      MMA issuer: tcgen05.mma 128x256x16 into a TMEM accumulator,
 //               two accumulators (512 TMEM columns) so the epilogue of one
 //               tile overlaps the main loop of the next;
-//   warps 2-5   epilogue: per tile, build the C and Z columns of the tile in
-//               shared memory, then tcgen05.ld the accumulator 16 columns at
-//               a time, add the low-rank term in fp32, apply the activation
-//               and store.
+//   warps 2-9   epilogue, two warpgroups: warp w reads TMEM lanes
+//               32*(w%4) .. +31 (its rows) and warpgroup h the h-th half of
+//               the tile's columns.  Per tile they build the C and Z columns of
+//               the tile in shared memory (Z from Philox), tcgen05.ld the
+//               accumulator 16 columns at a time, add the low-rank term in
+//               fp32 (32 independent accumulators per 16 columns), apply the
+//               activation and store from registers.
 // Gated mode (SiLU MLP gate/up): the 256-row W tile is 128 rows of W_gate and
 // the same 128 rows of W_up; the epilogue writes silu(gate) * up for 128 columns.
 // Plain mode (no P): the accumulator is stored as fp32 (used for X^T X).
@@ -35,8 +38,9 @@ constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TABLE_FLOATS = 4096;  // per table (C or Z): slots * RT
-constexpr int NUM_THREADS = 192;
-constexpr int EPI_THREADS = 128;
+constexpr int EPI_WARPS = 8;
+constexpr int EPI_THREADS = 32 * EPI_WARPS;
+constexpr int NUM_THREADS = 64 + EPI_THREADS;
 constexpr int TMEM_COLS = 512;
 constexpr int SMEM_BYTES = 1024 /*align slack*/ + STAGES * STAGE_BYTES + 2 * TABLE_FLOATS * 4 + 256;
 constexpr int GROUP_M = 8;
@@ -59,6 +63,7 @@ struct Params {
   uint32_t layer_id, layer_id2;
   int num_m, num_n, num_k, num_tiles;
   int64_t ldy;       // plain mode: row stride of D
+  int vec_ok;        // C, C2, P, P2 and ldy allow 16-byte vector access
   int* status;
 };
 
@@ -84,17 +89,32 @@ __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int&
 }
 
 // Fill table slots [slot0, slot0 + ncols) with C and Z of output columns
-// [col0, col0 + ncols) of one layer; columns >= d_out get zeros.  RT >= r is
-// the padded rank of the table rows.
+// [col0, col0 + ncols) of one layer; columns >= d_out and the padded ranks
+// j >= r get zeros.  Rows of the tables are RT floats (RT >= r, RT % 4 == 0).
 template <int RT>
 __device__ __forceinline__ void build_table(float* Ct, float* Zt, const float* __restrict__ Cg, uint32_t layer_id,
                                             int col0, int ncols, int slot0, int d_out, int r, uint64_t seed,
-                                            uint64_t query, int tid) {
-  // elements of the layer's [d_out, r] Z in the column range: e in [col0*r, (col0+ncols)*r)
+                                            uint64_t query, int tid, bool vec_ok) {
   const int valid_cols = max(0, min(ncols, d_out - col0));
-  const int64_t e_begin = (int64_t)col0 * r;
+  const int64_t e_begin = (int64_t)col0 * r;            // element range of the layer's [d_out, r] C and Z
   const int64_t e_end = e_begin + (int64_t)valid_cols * r;
-  // zero the padded / out-of-range slots first
+  if (r == RT && vec_ok) {
+    // rows of the table are the rows of C and Z: one group of 4 lands in one slot row
+    const int n_groups = ncols * RT / 4;
+    float4* C4 = reinterpret_cast<float4*>(Ct + slot0 * RT);
+    float4* Z4 = reinterpret_cast<float4*>(Zt + slot0 * RT);
+    for (int g = tid; g < n_groups; g += EPI_THREADS) {
+      const int64_t e = e_begin + 4 * (int64_t)g;
+      float4 c = make_float4(0.f, 0.f, 0.f, 0.f), z = c;
+      if (e < e_end) {
+        c = *reinterpret_cast<const float4*>(Cg + e);
+        z = z_normals4(seed, layer_id, query, (uint64_t)(e >> 2));
+      }
+      C4[g] = c;
+      Z4[g] = z;
+    }
+    return;
+  }
   for (int i = tid; i < ncols * RT; i += EPI_THREADS) {
     const int c = i / RT, j = i % RT;
     if (c >= valid_cols || j >= r) {
@@ -118,27 +138,65 @@ __device__ __forceinline__ void build_table(float* Ct, float* Zt, const float* _
   }
 }
 
+// Low-rank sums of 16 consecutive table slots for one token row:
+//   sC[i] = sum_j Ct[slot0+i][j] p[j],   sZ[i] = sum_j Zt[slot0+i][j] p[j].
 template <int RT>
-__device__ __forceinline__ void lowrank(const float* Ct, const float* Zt, int slot, const float* p, float& sC,
-                                        float& sZ) {
-  const float4* c4 = reinterpret_cast<const float4*>(Ct + slot * RT);
-  const float4* z4 = reinterpret_cast<const float4*>(Zt + slot * RT);
-  float a = 0.f, b = 0.f;
+__device__ __forceinline__ void lowrank16(const float* Ct, const float* Zt, int slot0, const float* p, float* sC,
+                                          float* sZ) {
+#pragma unroll
+  for (int i = 0; i < 16; ++i) { sC[i] = 0.f; sZ[i] = 0.f; }
+  const float4* c4 = reinterpret_cast<const float4*>(Ct + slot0 * RT);
+  const float4* z4 = reinterpret_cast<const float4*>(Zt + slot0 * RT);
 #pragma unroll
   for (int q = 0; q < RT / 4; ++q) {
-    const float4 cv = c4[q];
-    const float4 zv = z4[q];
-    a = fmaf(cv.x, p[4 * q + 0], a); a = fmaf(cv.y, p[4 * q + 1], a);
-    a = fmaf(cv.z, p[4 * q + 2], a); a = fmaf(cv.w, p[4 * q + 3], a);
-    b = fmaf(zv.x, p[4 * q + 0], b); b = fmaf(zv.y, p[4 * q + 1], b);
-    b = fmaf(zv.z, p[4 * q + 2], b); b = fmaf(zv.w, p[4 * q + 3], b);
+    const float p0 = p[4 * q], p1 = p[4 * q + 1], p2 = p[4 * q + 2], p3 = p[4 * q + 3];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const float4 c = c4[i * (RT / 4) + q];
+      const float4 z = z4[i * (RT / 4) + q];
+      sC[i] = fmaf(c.x, p0, fmaf(c.y, p1, fmaf(c.z, p2, fmaf(c.w, p3, sC[i]))));
+      sZ[i] = fmaf(z.x, p0, fmaf(z.y, p1, fmaf(z.z, p2, fmaf(z.w, p3, sZ[i]))));
+    }
   }
-  sC = a;
-  sZ = b;
+}
+
+__device__ __forceinline__ float silu_fast(float x) { return __fdividef(x, 1.0f + __expf(-x)); }
+
+__device__ __forceinline__ uint32_t pack2(float a, float b, __nv_bfloat16*) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+__device__ __forceinline__ uint32_t pack2(float a, float b, __half*) {
+  __half2 h = __floats2half2_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Store 16 consecutive outputs from registers (16-byte vectors when all 16 are
+// valid and the destination is 16-byte aligned).
+template <typename TO>
+__device__ __forceinline__ void store16(TO* dst, const float* v, int n_valid, bool vec_ok = true) {
+  if (n_valid >= 16 && vec_ok) {
+    if constexpr (sizeof(TO) == 4) {
+      float4* d4 = reinterpret_cast<float4*>(dst);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) d4[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+    } else {
+      uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+      for (int i = 0; i < 2; ++i)
+        d4[i] = make_uint4(pack2(v[8 * i], v[8 * i + 1], (TO*)nullptr), pack2(v[8 * i + 2], v[8 * i + 3], (TO*)nullptr),
+                           pack2(v[8 * i + 4], v[8 * i + 5], (TO*)nullptr),
+                           pack2(v[8 * i + 6], v[8 * i + 7], (TO*)nullptr));
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (i < n_valid) dst[i] = from_f32<TO>(v[i]);
+  }
 }
 
 // The epilogue's wait for a finished accumulator, taken by one thread and
-// shared through a named barrier so that all 128 epilogue threads leave (or
+// shared through a named barrier so that all epilogue threads leave (or
 // continue) together even if the wait gives up.
 __device__ __forceinline__ bool epi_wait_full(SharedState* ss, int buf, uint32_t parity, volatile int* abort_flag,
                                               int* status, int etid) {
@@ -150,18 +208,19 @@ __device__ __forceinline__ bool epi_wait_full(SharedState* ss, int buf, uint32_t
   return ok;
 }
 
-template <typename TO>
-__device__ __forceinline__ void store16(TO* dst, const float* v, int n_valid) {
-  if (n_valid >= 16) {
-    alignas(16) TO o[16];
+template <int RT>
+__device__ __forceinline__ void load_p(float* p, const float* __restrict__ P, int64_t m, int r, bool row_ok,
+                                       bool vec_ok) {
+  if (row_ok && r == RT && vec_ok) {
+    const float4* src = reinterpret_cast<const float4*>(P + m * r);
 #pragma unroll
-    for (int i = 0; i < 16; ++i) o[i] = from_f32<TO>(v[i]);
-    uint4* d4 = reinterpret_cast<uint4*>(dst);
-    const uint4* s4 = reinterpret_cast<const uint4*>(o);
-#pragma unroll
-    for (int i = 0; i < (int)(16 * sizeof(TO) / 16); ++i) d4[i] = s4[i];
+    for (int q = 0; q < RT / 4; ++q) {
+      const float4 v = src[q];
+      p[4 * q] = v.x; p[4 * q + 1] = v.y; p[4 * q + 2] = v.z; p[4 * q + 3] = v.w;
+    }
   } else {
-    for (int i = 0; i < n_valid; ++i) dst[i] = from_f32<TO>(v[i]);
+#pragma unroll
+    for (int j = 0; j < RT; ++j) p[j] = (row_ok && j < r) ? P[m * r + j] : 0.f;
   }
 }
 
@@ -281,8 +340,9 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     }
   } else {
-    // ---------------- epilogue (warps 2..5) ----------------
-    const int etid = threadIdx.x - 64;              // 0..127
+    // ---------------- epilogue (warps 2..9) ----------------
+    const int etid = threadIdx.x - 64;              // 0..255
+    const int half = etid >> 7;                     // which half of the tile's columns
     const int quad = warp & 3;                      // TMEM lane quadrant this warp may access
     const int row_in_tile = quad * 32 + lane;
     const int r = prm.r;
@@ -299,20 +359,12 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       if (MODE == MODE_PLAIN) {
         if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) break;
         float* D = static_cast<float*>(prm.Y);
-        for (int c0 = 0; c0 < BN; c0 += 16) {
+        for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 16) {
           float v[16];
           tc::tmem_ld16(t_row + (uint32_t)c0, v);
           const int n = n_blk * BN + c0;
           if (row_ok && n < prm.d_out) {
-            float* dst = D + m * prm.ldy + n;
-            const int nv = min(16, prm.d_out - n);
-            if (nv == 16 && (prm.ldy % 4) == 0) {
-#pragma unroll
-              for (int i = 0; i < 4; ++i)
-                reinterpret_cast<float4*>(dst)[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-            } else {
-              for (int i = 0; i < nv; ++i) dst[i] = v[i];
-            }
+            store16<float>(D + m * prm.ldy + n, v, min(16, prm.d_out - n), prm.vec_ok != 0);
           }
         }
         tc::tc_fence_before();
@@ -325,78 +377,85 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       constexpr int CHUNK = (TABLE_FLOATS / RT) < BN ? (TABLE_FLOATS / RT) : BN;
       static_assert(MODE != MODE_GATED || CHUNK == BN, "gated mode keeps the whole tile's table");
       float p[RT], p2[RT];
-#pragma unroll
-      for (int j = 0; j < RT; ++j) {
-        p[j] = (row_ok && j < r) ? prm.P[m * r + j] : 0.f;
-        p2[j] = (MODE == MODE_GATED && row_ok && j < r) ? prm.P2[m * r + j] : 0.f;
-      }
+      const bool vec = prm.vec_ok != 0;
+      load_p<RT>(p, prm.P, m, r, row_ok, vec);
+      if (MODE == MODE_GATED) load_p<RT>(p2, prm.P2, m, r, row_ok, vec);
+      const float sgn_eps = m < prm.T ? prm.eps : -prm.eps;   // stacked rows: sign of the half
+      TO* Y = static_cast<TO*>(prm.Y);
       bool ok = true;
       for (int s0 = 0; s0 < BN && ok; s0 += CHUNK) {
         tc::named_bar_sync(1, EPI_THREADS);          // previous chunk's readers are done
         if (MODE == MODE_GATED) {
           build_table<RT>(Ct, Zt, prm.C, prm.layer_id, n_blk * (BN / 2), BN / 2, 0, prm.d_out, r, prm.seed,
-                          prm.query, etid);
+                          prm.query, etid, vec);
           build_table<RT>(Ct, Zt, prm.C2, prm.layer_id2, n_blk * (BN / 2), BN / 2, BN / 2, prm.d_out, r,
-                          prm.seed, prm.query, etid);
+                          prm.seed, prm.query, etid, vec);
         } else {
           build_table<RT>(Ct, Zt, prm.C, prm.layer_id, n_blk * BN + s0, CHUNK, 0, prm.d_out, r, prm.seed,
-                          prm.query, etid);
+                          prm.query, etid, vec);
         }
         tc::named_bar_sync(1, EPI_THREADS);
         if (s0 == 0) {
           if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) { ok = false; break; }
         }
         if (MODE == MODE_GATED) {
-          TO* Y = static_cast<TO*>(prm.Y);
-          for (int c0 = 0; c0 < BN / 2; c0 += 16) {
+          for (int c0 = half * (BN / 4); c0 < (half + 1) * (BN / 4); c0 += 16) {
             float g[16], u[16];
             tc::tmem_ld16(t_row + (uint32_t)c0, g);
             tc::tmem_ld16(t_row + (uint32_t)(BN / 2 + c0), u);
             const int n = n_blk * (BN / 2) + c0;
             if (!row_ok || n >= prm.d_out) continue;
-            float hp[16], hm[16];
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              float gC, gZ, uC, uZ;
-              lowrank<RT>(Ct, Zt, c0 + i, p, gC, gZ);
-              lowrank<RT>(Ct, Zt, BN / 2 + c0 + i, p2, uC, uZ);
-              const float gb = g[i] + gC, ub = u[i] + uC;
-              if (prm.shared) {
-                hp[i] = silu_f(gb + prm.eps * gZ) * (ub + prm.eps * uZ);
-                hm[i] = silu_f(gb - prm.eps * gZ) * (ub - prm.eps * uZ);
-              } else {
-                const float se = m < prm.T ? prm.eps : -prm.eps;
-                hp[i] = silu_f(gb + se * gZ) * (ub + se * uZ);
-              }
-            }
             const int nv = min(16, prm.d_out - n);
-            store16<TO>(Y + m * prm.d_out + n, hp, nv);
-            if (prm.shared) store16<TO>(Y + (prm.T + m) * prm.d_out + n, hm, nv);
+            float gC[16], gZ[16];
+            lowrank16<RT>(Ct, Zt, c0, p, gC, gZ);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) g[i] += gC[i];      // g = W_g x + C_g p
+            float uC[16], uZ[16];
+            lowrank16<RT>(Ct, Zt, BN / 2 + c0, p2, uC, uZ);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) u[i] += uC[i];
+            if (prm.shared) {
+              float hp[16], hm[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                hp[i] = silu_fast(fmaf(prm.eps, gZ[i], g[i])) * fmaf(prm.eps, uZ[i], u[i]);
+                hm[i] = silu_fast(fmaf(-prm.eps, gZ[i], g[i])) * fmaf(-prm.eps, uZ[i], u[i]);
+              }
+              store16<TO>(Y + m * prm.d_out + n, hp, nv);
+              store16<TO>(Y + (prm.T + m) * prm.d_out + n, hm, nv);
+            } else {
+              float h[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i) h[i] = silu_fast(fmaf(sgn_eps, gZ[i], g[i])) * fmaf(sgn_eps, uZ[i], u[i]);
+              store16<TO>(Y + m * prm.d_out + n, h, nv);
+            }
           }
         } else {
-          TO* Y = static_cast<TO*>(prm.Y);
-          for (int c0 = s0; c0 < s0 + CHUNK; c0 += 16) {
+          const int cbeg = s0 + half * (CHUNK / 2);
+          for (int c0 = cbeg; c0 < cbeg + CHUNK / 2; c0 += 16) {
             float acc[16];
             tc::tmem_ld16(t_row + (uint32_t)c0, acc);
             const int n = n_blk * BN + c0;
             if (!row_ok || n >= prm.d_out) continue;
-            float yp[16], ym[16];
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              float sC, sZ;
-              lowrank<RT>(Ct, Zt, c0 - s0 + i, p, sC, sZ);
-              const float base = acc[i] + sC;
-              if (prm.shared) {
-                yp[i] = apply_act(base + prm.eps * sZ, prm.act);
-                ym[i] = apply_act(base - prm.eps * sZ, prm.act);
-              } else {
-                const float se = m < prm.T ? prm.eps : -prm.eps;
-                yp[i] = apply_act(base + se * sZ, prm.act);
-              }
-            }
             const int nv = min(16, prm.d_out - n);
-            store16<TO>(Y + m * prm.d_out + n, yp, nv);
-            if (prm.shared) store16<TO>(Y + (prm.T + m) * prm.d_out + n, ym, nv);
+            float sC[16], sZ[16];
+            lowrank16<RT>(Ct, Zt, c0 - s0, p, sC, sZ);
+            if (prm.shared) {
+              float yp[16], ym[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                const float base = acc[i] + sC[i];
+                yp[i] = apply_act(fmaf(prm.eps, sZ[i], base), prm.act);
+                ym[i] = apply_act(fmaf(-prm.eps, sZ[i], base), prm.act);
+              }
+              store16<TO>(Y + m * prm.d_out + n, yp, nv);
+              store16<TO>(Y + (prm.T + m) * prm.d_out + n, ym, nv);
+            } else {
+              float y[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i) y[i] = apply_act(fmaf(sgn_eps, sZ[i], acc[i] + sC[i]), prm.act);
+              store16<TO>(Y + m * prm.d_out + n, y, nv);
+            }
           }
         }
       }
