@@ -27,6 +27,7 @@ enum ScratchSlot {
   SLOT_PARTIALS,     // per-block partial sums of grid reductions
   SLOT_BASIS,        // Gram matrix and subspace-iteration workspace
   SLOT_BASIS_X,      // transposed calibration activations
+  SLOT_UT,           // 16-bit split copy of the basis for the tensor-core projection
   SLOT_COUNT
 };
 
@@ -78,6 +79,9 @@ int launch_philox_normals(Ctx* ctx, uint64_t seed, uint32_t layer_id, uint64_t q
                           float* z, uint32_t* words);
 int launch_lowrank_proj(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const float* U,
                         int r, float* P);
+// Tensor-core projection for 16-bit X (U split into three 16-bit terms).
+int launch_lowrank_proj_tc(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const float* U, int r,
+                           float* P);
 // As launch_lowrank_proj, with split-K partials in `part` (part_floats floats) instead of context scratch.
 int launch_lowrank_proj_into(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const float* U,
                              int r, float* P, float* part, int64_t part_floats);

@@ -15,12 +15,23 @@ namespace {
 
 constexpr int LOSS_THREADS = 256;
 
+__device__ __forceinline__ void unpack2(uint32_t w, float* out, const __nv_bfloat16*) {
+  out[0] = __uint_as_float(w << 16);
+  out[1] = __uint_as_float(w & 0xffff0000u);
+}
+__device__ __forceinline__ void unpack2(uint32_t w, float* out, const __half*) {
+  const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w));
+  out[0] = f.x;
+  out[1] = f.y;
+}
+
 template <typename TY>
 __device__ __forceinline__ void load8(const TY* p, float* out) {
-  const uint4 raw = *reinterpret_cast<const uint4*>(p);
-  const TY* e = reinterpret_cast<const TY*>(&raw);
-#pragma unroll
-  for (int i = 0; i < 8; ++i) out[i] = to_f32<TY>(e[i]);
+  const uint4 raw = __ldg(reinterpret_cast<const uint4*>(p));
+  unpack2(raw.x, out + 0, p);
+  unpack2(raw.y, out + 2, p);
+  unpack2(raw.z, out + 4, p);
+  unpack2(raw.w, out + 6, p);
 }
 template <>
 __device__ __forceinline__ void load8<float>(const float* p, float* out) {
@@ -48,7 +59,31 @@ loss_pair_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t c
   // y- = y+ + count is aligned when count % 8 == 0)
   const int64_t n_vec = vec_ok ? count / 8 : 0;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < n_vec; v += stride) {
+  int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  // four vectors per round with all twelve 16-byte loads issued before any use
+  for (; v + 3 * stride < n_vec; v += 4 * stride) {
+    float p[4][8], m[4][8], t[4][8];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      load8<TY>(yp + 8 * (v + u * stride), p[u]);
+      load8<TY>(ym + 8 * (v + u * stride), m[u]);
+      if (tgt) load8<TY>(tgt + 8 * (v + u * stride), t[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      float sp = 0.f, sm = 0.f, sd = 0.f;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float tv = tgt ? t[u][i] : 0.f;
+        const float dp = p[u][i] - tv, dm = m[u][i] - tv;
+        sp = fmaf(dp, dp, sp);
+        sm = fmaf(dm, dm, sm);
+        sd = fmaf(p[u][i] - m[u][i], dp + dm, sd);
+      }
+      ap += sp; am += sm; ad += sd;
+    }
+  }
+  for (; v < n_vec; v += stride) {
     float p[8], m[8], t[8];
     load8<TY>(yp + 8 * v, p);
     load8<TY>(ym + 8 * v, m);
@@ -121,7 +156,7 @@ int loss_dispatch(Ctx* ctx, const TY* Y, const TY* tgt, int64_t count, float eps
 
 }  // namespace
 
-int loss_pair_max_blocks(Ctx* ctx) { return 2 * ctx->sm_count; }
+int loss_pair_max_blocks(Ctx* ctx) { return 4 * ctx->sm_count; }
 
 int launch_loss_pair(Ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T, int64_t n, float eps,
                      double* out, double* partials, int max_blocks) {

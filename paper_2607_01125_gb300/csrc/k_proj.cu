@@ -175,8 +175,8 @@ int launch_lowrank_proj(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d
   if (rows <= 0) return ZOACT_OK;
   switch (xdtype) {
     case ZOACT_DT_FP32: return proj_dispatch(ctx, static_cast<const float*>(X), rows, d_in, U, r, P);
-    case ZOACT_DT_BF16: return proj_dispatch(ctx, static_cast<const __nv_bfloat16*>(X), rows, d_in, U, r, P);
-    case ZOACT_DT_FP16: return proj_dispatch(ctx, static_cast<const __half*>(X), rows, d_in, U, r, P);
+    case ZOACT_DT_BF16:
+    case ZOACT_DT_FP16: return launch_lowrank_proj_tc(ctx, X, xdtype, rows, d_in, U, r, P);
     default: return ZOACT_ERR_INVALID_ARG;
   }
 }
