@@ -178,9 +178,8 @@ class MLPRunner:
             self.events.append((e0, e1, e2, e3))
         s.loss(self.Y, target)
         if self.world > 1:
-            import torch.distributed as dist
-            dist.all_reduce(s.loss_out)          # L+, L-, D and a are means over equal token counts
-            s.loss_out.div_(self.world)
+            from paper_2607_01125_gb300.dp import allreduce_loss
+            allreduce_loss(s.loss_out)           # L+, L-, D and a are means over equal token counts
         s.update(t, seed, t)
         return s.loss_out
 

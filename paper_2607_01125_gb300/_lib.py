@@ -108,7 +108,12 @@ def _check(name, status):
 
 
 def _ptr(t):
-    return None if t is None else ctypes.c_void_p(t.data_ptr())
+    """Device address of a row-major tensor (the ABI's layout); other layouts are refused."""
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("libzoact takes row-major (contiguous) tensors")
+    return ctypes.c_void_p(t.data_ptr())
 
 
 def _dt(t):
@@ -162,6 +167,9 @@ class Context:
 
 def make_layer(W, U, C, layer_id, w_scales=None, wtype=None, d_in=None):
     """A zoact_layer for torch tensors W [d_out, d_in] (or INT4 packed), U [d_in, r] fp32, C [d_out, r] fp32."""
+    for t in (W, U, C, w_scales):
+        if t is not None and not t.is_contiguous():
+            raise ValueError("libzoact takes row-major (contiguous) tensors")
     if wtype is None:
         wtype = _dt(W)
     d_out = W.shape[0]

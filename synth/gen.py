@@ -65,7 +65,7 @@ def decaying_spectrum_activations(n_tok, d, rank, noise, seed, device="cpu", dty
     B = orthonormal rows (QR of a Gaussian), then unit RMS per token.
     """
     g = _gen(seed, device)
-    B = torch.linalg.qr(torch.randn(d, rank, generator=g, device=device))[0].T  # [rank, d]
+    B = torch.linalg.qr(torch.randn(d, rank, generator=g, device=device))[0].T.contiguous()  # [rank, d]
     s = 1.0 / torch.arange(1, rank + 1, device=device, dtype=torch.float32)
     A = torch.randn(n_tok, rank, generator=g, device=device) * s * math.sqrt(d)
     x = A @ B + noise * torch.randn(n_tok, d, generator=g, device=device)
@@ -98,4 +98,5 @@ def quantize_int4_g128(W):
 def random_orthonormal(d, r, seed, device="cpu"):
     """A [d, r] matrix with orthonormal columns (QR of a Gaussian)."""
     g = _gen(seed, device)
-    return torch.linalg.qr(torch.randn(d, r, generator=g, device=device, dtype=torch.float64))[0].float()
+    q = torch.linalg.qr(torch.randn(d, r, generator=g, device=device, dtype=torch.float64))[0]
+    return q.float().contiguous()

@@ -1,0 +1,84 @@
+"""Data-parallel ZO step across 2 CPU ranks (gloo): the scalar exchange of dp.allreduce_loss.
+
+Each rank evaluates the oracle's loss pair on its own token shard; after the
+all-reduce every rank holds the loss pair of the whole batch, and the Adam
+updates the ranks then apply independently are identical to the single-process
+update on the concatenated batch.
+"""
+import os
+import socket
+
+import numpy as np
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+from oracle import layers, loss as oloss, optim, philox
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _problem():
+    rng = np.random.default_rng(0)
+    d_in, d_out, r, T = 48, 40, 4, 24
+    W = rng.standard_normal((d_out, d_in)) / np.sqrt(d_in)
+    U = np.linalg.qr(rng.standard_normal((d_in, r)))[0]
+    C = 0.1 * rng.standard_normal((d_out, r))
+    X = rng.standard_normal((2 * T, d_in))      # the whole batch: two shards of T tokens
+    tgt = rng.standard_normal((2 * T, d_out))
+    return W, U, C, X, tgt, T
+
+
+def _rank_step(rank, world, W, U, C, X, tgt, T, eps=1e-3, seed=9, query=1):
+    Z = philox.perturbation(seed, 3, query, *C.shape)
+    xs, ts = X[rank * T:(rank + 1) * T], tgt[rank * T:(rank + 1) * T]
+    Y = layers.pair_forward(W, U, C, Z, xs, eps, T, True)
+    out = torch.tensor(oloss.loss_pair(Y, T, ts, eps), dtype=torch.float64)
+    return out, Z
+
+
+def _worker(rank, world, port, q):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    from paper_2607_01125_gb300.dp import allreduce_loss
+    W, U, C, X, tgt, T = _problem()
+    out, Z = _rank_step(rank, world, W, U, C, X, tgt, T)
+    allreduce_loss(out)
+    a = float(out[3])
+    Cn, _, _ = optim.adam_step(C, 0, 0, optim.zo_gradient(a, Z), 1e-3, 0.9, 0.999, 1e-8, 1)
+    gathered = [torch.zeros(Cn.size, dtype=torch.float64) for _ in range(world)]
+    dist.all_gather(gathered, torch.from_numpy(Cn.reshape(-1).copy()))
+    q.put((rank, out.numpy().tolist(), [g.numpy() for g in gathered]))
+    dist.destroy_process_group()
+
+
+def test_two_rank_scalar_exchange_matches_single_process():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    results = [q.get(timeout=120) for _ in procs]
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    W, U, C, X, tgt, T = _problem()
+    Z = philox.perturbation(9, 3, 1, *C.shape)
+    # single process on the concatenated batch (both halves see the same x per shard: shared input)
+    Yfull = np.concatenate([layers.pair_forward(W, U, C, Z, X[i * T:(i + 1) * T], 1e-3, T, True) for i in range(2)])
+    yp = np.concatenate([Yfull[:T], Yfull[2 * T:3 * T]])
+    ym = np.concatenate([Yfull[T:2 * T], Yfull[3 * T:]])
+    ref = oloss.loss_pair(np.concatenate([yp, ym]), 2 * T, tgt, 1e-3)
+    Cref, _, _ = optim.adam_step(C, 0, 0, optim.zo_gradient(ref[3], Z), 1e-3, 0.9, 0.999, 1e-8, 1)
+    for rank, out, gathered in results:
+        np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-15)
+        for g in gathered:                           # every rank holds the same C, equal to the reference
+            np.testing.assert_allclose(g, Cref.reshape(-1), rtol=0, atol=1e-15)
