@@ -127,13 +127,30 @@ loss_pair_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t c
     is_last = (prev == gridDim.x - 1);
   }
   __syncthreads();
-  if (is_last && threadIdx.x == 0) {
-    __threadfence();
-    double s0 = 0.0, s1 = 0.0, s2 = 0.0;
-    const volatile double* pv = partials;
-    for (unsigned int b = 0; b < gridDim.x; ++b) { s0 += pv[3 * b]; s1 += pv[3 * b + 1]; s2 += pv[3 * b + 2]; }
+  if (!is_last) return;
+  // the last block adds the partials: thread t takes blocks t, t + 256, ... in order, then a fixed
+  // shared-memory tree combines the threads, so the result does not depend on scheduling
+  __threadfence();
+  double s0 = 0.0, s1 = 0.0, s2 = 0.0;
+  for (unsigned int b = threadIdx.x; b < gridDim.x; b += LOSS_THREADS) {
+    s0 += __ldcg(partials + 3 * b);
+    s1 += __ldcg(partials + 3 * b + 1);
+    s2 += __ldcg(partials + 3 * b + 2);
+  }
+  __shared__ double tree[3][LOSS_THREADS];
+  tree[0][threadIdx.x] = s0; tree[1][threadIdx.x] = s1; tree[2][threadIdx.x] = s2;
+  __syncthreads();
+  for (int h = LOSS_THREADS / 2; h > 0; h >>= 1) {
+    if (threadIdx.x < h) {
+      tree[0][threadIdx.x] += tree[0][threadIdx.x + h];
+      tree[1][threadIdx.x] += tree[1][threadIdx.x + h];
+      tree[2][threadIdx.x] += tree[2][threadIdx.x + h];
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
     const double inv = 1.0 / (double)count;
-    const double Lp = s0 * inv, Lm = s1 * inv, D = s2 * inv;
+    const double Lp = tree[0][0] * inv, Lm = tree[1][0] * inv, D = tree[2][0] * inv;
     const double a = D / (2.0 * (double)eps);
     out[0] = Lp; out[1] = Lm; out[2] = D; out[3] = a;
     if (!isfinite(Lp) || !isfinite(Lm) || !isfinite(a)) record_error(status, ZOACT_ERR_NONFINITE);
