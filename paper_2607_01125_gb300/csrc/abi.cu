@@ -64,7 +64,10 @@ int check_layer(const zoact_layer* L) {
   if (L->d_in <= 0 || L->d_out <= 0 || L->r <= 0) return ZOACT_ERR_INVALID_ARG;
   if (L->r > 32) return ZOACT_ERR_UNSUPPORTED;
   if ((int64_t)L->d_out * L->r >= (int64_t)1 << 34) return ZOACT_ERR_INVALID_ARG;
-  if (L->wtype == ZOACT_DT_INT4_G128) return ZOACT_ERR_UNSUPPORTED;
+  if (L->wtype == ZOACT_DT_INT4_G128) {
+    if (!L->w_scales || L->d_in % 128 != 0 || ((uintptr_t)L->W & 15u) != 0) return ZOACT_ERR_INVALID_ARG;
+    return ZOACT_OK;
+  }
   if (!valid_act_dtype(L->wtype)) return ZOACT_ERR_INVALID_ARG;
   return ZOACT_OK;
 }
@@ -197,7 +200,7 @@ static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* 
   if (act < ZOACT_ACT_NONE || act > ZOACT_ACT_GELU) return ZOACT_ERR_INVALID_ARG;
   if (T == 0) return ZOACT_OK;
   if (!X || !Y) return ZOACT_ERR_INVALID_ARG;
-  if (xdtype != L->wtype) return ZOACT_ERR_INVALID_ARG;
+  if (L->wtype == ZOACT_DT_INT4_G128 ? xdtype != ZOACT_DT_BF16 : xdtype != L->wtype) return ZOACT_ERR_INVALID_ARG;
   if (!aligned16(X) || !aligned16(Y) || !aligned16(L->W) || (L2 && !aligned16(L2->W))) return ZOACT_ERR_INVALID_ARG;
   if (L->d_in % (xdtype == ZOACT_DT_FP32 ? 4 : 8) != 0) return ZOACT_ERR_INVALID_ARG;
   if (L->d_out % 8 != 0) return ZOACT_ERR_INVALID_ARG;
@@ -223,7 +226,7 @@ static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* 
   a.shared = input_shared ? 1 : 0; a.act = act;
   a.xdtype = xdtype; a.wtype = L->wtype; a.ydtype = ydtype;
   a.eps = eps; a.seed = seed; a.query = query; a.layer_id = L->layer_id;
-  if (L2) { a.W2 = L2->W; a.P2 = P2; a.C2 = L2->C; a.layer_id2 = L2->layer_id; }
+  if (L2) { a.W2 = L2->W; a.w_scales2 = L2->w_scales; a.P2 = P2; a.C2 = L2->C; a.layer_id2 = L2->layer_id; }
   if (xdtype == ZOACT_DT_FP32) return launch_pair_simt(ctx, a);
   return launch_pair_tc(ctx, a);
 }

@@ -104,6 +104,7 @@ struct PairArgs {
   uint32_t layer_id;
   // gated mode (second layer: up); W2 == nullptr for the plain pair forward
   const void* W2;
+  const void* w_scales2;
   const float* P2;
   const float* C2;
   uint32_t layer_id2;

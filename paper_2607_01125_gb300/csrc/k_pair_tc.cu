@@ -11,6 +11,7 @@ int dispatch_bf16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, 
                   const CUtensorMap& b2, const Params& p);
 int dispatch_fp16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const CUtensorMap& b,
                   const CUtensorMap& b2, const Params& p);
+int dispatch_w4(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const Params& p);
 }  // namespace pairtc
 
 namespace {
@@ -54,7 +55,8 @@ int encode_tmap_2d_16bit(CUtensorMap* map, const void* base, int dtype, int64_t 
 int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   using namespace pairtc;
   if (a.xdtype != ZOACT_DT_BF16 && a.xdtype != ZOACT_DT_FP16) return ZOACT_ERR_UNSUPPORTED;
-  if (a.wtype != a.xdtype) return ZOACT_ERR_UNSUPPORTED;
+  const bool w4 = a.wtype == ZOACT_DT_INT4_G128;
+  if (w4 ? a.xdtype != ZOACT_DT_BF16 : a.wtype != a.xdtype) return ZOACT_ERR_UNSUPPORTED;
   if (a.ydtype != a.xdtype && a.ydtype != ZOACT_DT_FP32) return ZOACT_ERR_UNSUPPORTED;
   const bool gated = a.W2 != nullptr;
   const int rt = rank_template(a.r);
@@ -63,9 +65,13 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   CUtensorMap ma, mb, mb2;
   int st = encode_tmap_2d_16bit(&ma, a.X, a.xdtype, a.rows, a.d_in, BM);
   if (st) return st;
-  st = encode_tmap_2d_16bit(&mb, a.W, a.wtype, a.d_out, a.d_in, gated ? BN / 2 : BN);
-  if (st) return st;
-  if (gated) {
+  if (w4) {
+    mb = mb2 = ma;                       // W arrives through the dequantising warps, not TMA
+  } else {
+    st = encode_tmap_2d_16bit(&mb, a.W, a.wtype, a.d_out, a.d_in, gated ? BN / 2 : BN);
+    if (st) return st;
+  }
+  if (gated && !w4) {
     st = encode_tmap_2d_16bit(&mb2, a.W2, a.wtype, a.d_out, a.d_in, BN / 2);
     if (st) return st;
   } else {
@@ -85,6 +91,13 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   p.vec_ok = al16(a.C) && al16(a.C2) && al16(a.P) && al16(a.P2);
   p.status = ctx->d_status;
   const int mode = gated ? MODE_GATED : MODE_PAIR;
+  if (w4) {
+    p.Wq = static_cast<const uint8_t*>(a.W);
+    p.Ws = static_cast<const __half*>(a.w_scales);
+    p.Wq2 = static_cast<const uint8_t*>(a.W2);
+    p.Ws2 = static_cast<const __half*>(a.w_scales2);
+    return dispatch_w4(ctx, mode, rt, a.ydtype, ma, p);
+  }
   return a.xdtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p)
                                    : dispatch_fp16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p);
 }

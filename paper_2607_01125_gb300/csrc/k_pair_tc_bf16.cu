@@ -6,10 +6,10 @@ namespace pairtc {
 
 template <typename TO, int RT, int MODE>
 static int launch_one(Ctx* ctx, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& b2, const Params& p) {
-  auto kern = pair_tc_kernel<TO, RT, MODE, 1>;
+  auto kern = pair_tc_kernel<TO, RT, MODE, 1, false>;
   ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
   const int grid = p.num_tiles < ctx->sm_count ? p.num_tiles : ctx->sm_count;
-  kern<<<grid, NUM_THREADS, SMEM_BYTES, ctx->stream>>>(a, b, b2, p); ++ctx->n_launch;
+  kern<<<grid, num_threads(false), SMEM_BYTES, ctx->stream>>>(a, b, b2, p); ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
 }

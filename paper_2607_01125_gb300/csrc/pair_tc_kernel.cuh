@@ -25,6 +25,17 @@
 // Gated mode (SiLU MLP gate/up): the 256-row W tile is 128 rows of W_gate and
 // the same 128 rows of W_up; the epilogue writes silu(gate) * up for 128 columns.
 // Plain mode (no P): the accumulator is stored as fp32 (used for X^T X).
+//
+// INT4 weights (W4): the frozen W is symmetric INT4 in groups of 128 along d_in
+// with fp16 scales.  Four more warps (448 threads in all) dequantise it: per
+// K-block each thread loads 2 rows x 32 packed bytes and their scales with
+// plain global loads (prefetched one K-block ahead), turns every nibble q into
+// bf16 q * s (magic-number conversion 0x4300 | (q ^ 8) = 128 + q + 8, minus
+// 136, times the scale, in bf16x2 arithmetic) and writes the 128-byte-swizzled
+// bf16 tile straight into the MMA's shared-memory stage, then fences the
+// async proxy and arrives on the stage's barrier.  Only X comes by TMA.  With
+// 14 warps the registers per thread drop to 128, so the epilogue works on
+// 8-column chunks.
 #pragma once
 #include "internal.h"
 #include "philox.cuh"
@@ -40,7 +51,9 @@ constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TABLE_FLOATS = 4096;  // per table (C or Z): slots * RT
 constexpr int EPI_WARPS = 8;
 constexpr int EPI_THREADS = 32 * EPI_WARPS;
-constexpr int NUM_THREADS = 64 + EPI_THREADS;
+constexpr int DQ_THREADS = 128;                     // INT4 dequantisation warps
+__host__ __device__ constexpr int num_threads(bool w4) { return 64 + EPI_THREADS + (w4 ? DQ_THREADS : 0); }
+__host__ __device__ constexpr int epi_base(bool w4) { return 64 + (w4 ? DQ_THREADS : 0); }
 constexpr int TMEM_COLS = 512;
 constexpr int SMEM_BYTES = 1024 /*align slack*/ + STAGES * STAGE_BYTES + 2 * TABLE_FLOATS * 4 + 256;
 constexpr int GROUP_M = 8;
@@ -64,6 +77,11 @@ struct Params {
   int num_m, num_n, num_k, num_tiles;
   int64_t ldy;       // plain mode: row stride of D
   int vec_ok;        // C, C2, P, P2 and ldy allow 16-byte vector access
+  // INT4 weights: packed [d_out, d_in/2] bytes and fp16 scales [d_out, d_in/128]
+  const uint8_t* Wq;
+  const __half* Ws;
+  const uint8_t* Wq2;
+  const __half* Ws2;
   int* status;
 };
 
@@ -138,20 +156,20 @@ __device__ __forceinline__ void build_table(float* Ct, float* Zt, const float* _
   }
 }
 
-// Low-rank sums of 16 consecutive table slots for one token row:
+// Low-rank sums of CW consecutive table slots for one token row:
 //   sC[i] = sum_j Ct[slot0+i][j] p[j],   sZ[i] = sum_j Zt[slot0+i][j] p[j].
-template <int RT>
-__device__ __forceinline__ void lowrank16(const float* Ct, const float* Zt, int slot0, const float* p, float* sC,
-                                          float* sZ) {
+template <int RT, int CW>
+__device__ __forceinline__ void lowrankN(const float* Ct, const float* Zt, int slot0, const float* p, float* sC,
+                                         float* sZ) {
 #pragma unroll
-  for (int i = 0; i < 16; ++i) { sC[i] = 0.f; sZ[i] = 0.f; }
+  for (int i = 0; i < CW; ++i) { sC[i] = 0.f; sZ[i] = 0.f; }
   const float4* c4 = reinterpret_cast<const float4*>(Ct + slot0 * RT);
   const float4* z4 = reinterpret_cast<const float4*>(Zt + slot0 * RT);
 #pragma unroll
   for (int q = 0; q < RT / 4; ++q) {
     const float p0 = p[4 * q], p1 = p[4 * q + 1], p2 = p[4 * q + 2], p3 = p[4 * q + 3];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
+    for (int i = 0; i < CW; ++i) {
       const float4 c = c4[i * (RT / 4) + q];
       const float4 z = z4[i * (RT / 4) + q];
       sC[i] = fmaf(c.x, p0, fmaf(c.y, p1, fmaf(c.z, p2, fmaf(c.w, p3, sC[i]))));
@@ -171,28 +189,93 @@ __device__ __forceinline__ uint32_t pack2(float a, float b, __half*) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-// Store 16 consecutive outputs from registers (16-byte vectors when all 16 are
-// valid and the destination is 16-byte aligned).
-template <typename TO>
-__device__ __forceinline__ void store16(TO* dst, const float* v, int n_valid, bool vec_ok = true) {
-  if (n_valid >= 16 && vec_ok) {
+// Store CW (8 or 16) consecutive outputs from registers (16-byte vectors when
+// all are valid and the destination is 16-byte aligned).
+template <typename TO, int CW>
+__device__ __forceinline__ void storeN(TO* dst, const float* v, int n_valid, bool vec_ok = true) {
+  if (n_valid >= CW && vec_ok) {
     if constexpr (sizeof(TO) == 4) {
       float4* d4 = reinterpret_cast<float4*>(dst);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) d4[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+      for (int i = 0; i < CW / 4; ++i) d4[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
     } else {
       uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
-      for (int i = 0; i < 2; ++i)
+      for (int i = 0; i < CW / 8; ++i)
         d4[i] = make_uint4(pack2(v[8 * i], v[8 * i + 1], (TO*)nullptr), pack2(v[8 * i + 2], v[8 * i + 3], (TO*)nullptr),
                            pack2(v[8 * i + 4], v[8 * i + 5], (TO*)nullptr),
                            pack2(v[8 * i + 6], v[8 * i + 7], (TO*)nullptr));
     }
   } else {
 #pragma unroll
-    for (int i = 0; i < 16; ++i)
+    for (int i = 0; i < CW; ++i)
       if (i < n_valid) dst[i] = from_f32<TO>(v[i]);
   }
+}
+
+template <int CW>
+__device__ __forceinline__ void tmem_ldN(uint32_t taddr, float* v) {
+  if constexpr (CW == 16) tc::tmem_ld16(taddr, v);
+  else tc::tmem_ld8(taddr, v);
+}
+
+// ---- INT4 dequantisation into a 128-byte-swizzled bf16 B tile ----
+// 8 nibbles (elements k..k+7, low nibble first) scaled by s -> 8 bf16 (16 bytes).
+__device__ __forceinline__ uint4 dequant8(uint32_t w, __nv_bfloat162 s2) {
+  const uint32_t x = w ^ 0x88888888u;                 // nibble q -> q + 8 in [0, 15]
+  const __nv_bfloat162 c136 = __floats2bfloat162_rn(136.0f, 136.0f);
+  uint32_t out[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t lo = (x >> (8 * i)) & 0xFu, hi = (x >> (8 * i + 4)) & 0xFu;
+    uint32_t v = 0x43004300u | lo | (hi << 16);       // bf16 pair (128 + q + 8)
+    __nv_bfloat162 h = *reinterpret_cast<__nv_bfloat162*>(&v);
+    h = __hmul2(__hsub2(h, c136), s2);                // q exactly, then q * s rounded to bf16
+    out[i] = *reinterpret_cast<uint32_t*>(&h);
+  }
+  return make_uint4(out[0], out[1], out[2], out[3]);
+}
+
+// Row `row` (0..255) of the B tile of K-block kb: source row, packed bytes and scale.
+struct DqRow {
+  uint4 q0, q1;       // 32 packed bytes = 64 elements
+  __half s;
+  bool valid;
+};
+
+template <int MODE>
+__device__ __forceinline__ DqRow dq_load(const Params& prm, int n_blk, int row, int kb) {
+  DqRow d;
+  const uint8_t* Wq = prm.Wq;
+  const __half* Ws = prm.Ws;
+  int n;
+  if (MODE == MODE_GATED) {
+    n = n_blk * (BN / 2) + (row & (BN / 2 - 1));
+    if (row >= BN / 2) { Wq = prm.Wq2; Ws = prm.Ws2; }
+  } else {
+    n = n_blk * BN + row;
+  }
+  d.valid = n < prm.d_out;
+  if (d.valid) {
+    const uint4* src = reinterpret_cast<const uint4*>(Wq + (int64_t)n * (prm.d_in / 2) + kb * (BK / 2));
+    d.q0 = __ldg(src);
+    d.q1 = __ldg(src + 1);
+    d.s = Ws[(int64_t)n * (prm.d_in / 128) + (kb * BK) / 128];
+  } else {
+    d.q0 = d.q1 = make_uint4(0x88888888u, 0x88888888u, 0x88888888u, 0x88888888u);   // q = 0
+    d.s = __float2half_rn(0.f);
+  }
+  return d;
+}
+
+__device__ __forceinline__ void dq_store(uint8_t* btile, int row, const DqRow& d) {
+  const __nv_bfloat16 sb = __float2bfloat16_rn(__half2float(d.s));
+  const __nv_bfloat162 s2 = __halves2bfloat162(sb, sb);
+  uint8_t* rowp = btile + row * 128;
+  const uint32_t w[8] = {d.q0.x, d.q0.y, d.q0.z, d.q0.w, d.q1.x, d.q1.y, d.q1.z, d.q1.w};
+#pragma unroll
+  for (int c = 0; c < 8; ++c)
+    *reinterpret_cast<uint4*>(rowp + ((c ^ (row & 7)) << 4)) = dequant8(w[c], s2);
 }
 
 // The epilogue's wait for a finished accumulator, taken by one thread and
@@ -224,10 +307,11 @@ __device__ __forceinline__ void load_p(float* p, const float* __restrict__ P, in
   }
 }
 
-template <typename TO, int RT, int MODE, int AB_BF16>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+template <typename TO, int RT, int MODE, int AB_BF16, bool W4>
+__global__ void __launch_bounds__(num_threads(W4), 1)
 pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                const __grid_constant__ CUtensorMap tmB2, const Params prm) {
+  constexpr int CW = W4 ? 8 : 16;                   // epilogue chunk width (columns per tcgen05.ld)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   float* Ct = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);
@@ -240,7 +324,8 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
-      tc::mbar_init(tc::smem_u32(&ss->full[s]), 1);
+      // full: the producer's expect_tx arrival, plus one arrival per dequantising thread (INT4)
+      tc::mbar_init(tc::smem_u32(&ss->full[s]), W4 ? 1 + DQ_THREADS : 1);
       tc::mbar_init(tc::smem_u32(&ss->empty[s]), 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -251,8 +336,8 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     ss->abort_flag = 0;
     tc::fence_mbar_init();
     tc::prefetch_tmap(&tmA);
-    tc::prefetch_tmap(&tmB);
-    if (MODE == MODE_GATED) tc::prefetch_tmap(&tmB2);
+    if (!W4) tc::prefetch_tmap(&tmB);
+    if (!W4 && MODE == MODE_GATED) tc::prefetch_tmap(&tmB2);
   }
   if (warp == 1) {
     tc::tmem_alloc(tc::smem_u32(&ss->tmem_base), TMEM_COLS);
@@ -278,11 +363,13 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         for (int kb = 0; kb < num_k; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
           const uint32_t full = tc::smem_u32(&ss->full[stage]);
-          tc::mbar_arrive_expect_tx(full, STAGE_BYTES);
+          tc::mbar_arrive_expect_tx(full, W4 ? A_BYTES : STAGE_BYTES);
           const uint32_t sa = tc::smem_u32(smem + stage * STAGE_BYTES);
           const uint32_t sb = sa + A_BYTES;
           tc::tma_load_2d(sa, &tmA, kb * BK, m_blk * BM, full);
-          if (MODE == MODE_GATED) {
+          if (W4) {
+            // B arrives from the dequantising warps
+          } else if (MODE == MODE_GATED) {
             tc::tma_load_2d(sb, &tmB, kb * BK, n_blk * (BN / 2), full);
             tc::tma_load_2d(sb + B_BYTES / 2, &tmB2, kb * BK, n_blk * (BN / 2), full);
           } else {
@@ -339,9 +426,47 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         tc::mbar_wait_drain(tc::smem_u32(&ss->drain), 0, 100000000ull);
       }
     }
+  } else if (W4 && warp < 2 + DQ_THREADS / 32) {
+    // ---------------- INT4 dequantisation (warps 2..5) ----------------
+    const int dtid = threadIdx.x - 64;             // 0..127: rows 2*dtid and 2*dtid + 1 of each B tile
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    bool have = false;
+    DqRow cur0, cur1;
+    // walk the same (tile, K-block) sequence as the producer, one K-block of loads ahead
+    int tile = blockIdx.x, kb = 0;
+    if (tile < prm.num_tiles) {
+      int m_blk, n_blk;
+      tile_coords(tile, num_m, num_n, m_blk, n_blk);
+      cur0 = dq_load<MODE>(prm, n_blk, 2 * dtid, 0);
+      cur1 = dq_load<MODE>(prm, n_blk, 2 * dtid + 1, 0);
+      have = true;
+    }
+    while (have && ok) {
+      // next K-block's loads first
+      int nt = tile, nkb = kb + 1;
+      if (nkb == num_k) { nkb = 0; nt += gridDim.x; }
+      DqRow nxt0, nxt1;
+      const bool more = nt < prm.num_tiles;
+      if (more) {
+        int m_blk, n_blk;
+        tile_coords(nt, num_m, num_n, m_blk, n_blk);
+        nxt0 = dq_load<MODE>(prm, n_blk, 2 * dtid, nkb);
+        nxt1 = dq_load<MODE>(prm, n_blk, 2 * dtid + 1, nkb);
+      }
+      if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
+      uint8_t* btile = smem + stage * STAGE_BYTES + A_BYTES;
+      dq_store(btile, 2 * dtid, cur0);
+      dq_store(btile, 2 * dtid + 1, cur1);
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // generic writes -> tensor-core reads
+      tc::mbar_arrive(tc::smem_u32(&ss->full[stage]));
+      if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+      tile = nt; kb = nkb; cur0 = nxt0; cur1 = nxt1; have = more;
+    }
   } else {
-    // ---------------- epilogue (warps 2..9) ----------------
-    const int etid = threadIdx.x - 64;              // 0..255
+    // ---------------- epilogue (8 warps) ----------------
+    const int etid = threadIdx.x - epi_base(W4);    // 0..255
     const int half = etid >> 7;                     // which half of the tile's columns
     const int quad = warp & 3;                      // TMEM lane quadrant this warp may access
     const int row_in_tile = quad * 32 + lane;
@@ -359,12 +484,12 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       if (MODE == MODE_PLAIN) {
         if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) break;
         float* D = static_cast<float*>(prm.Y);
-        for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += 16) {
-          float v[16];
-          tc::tmem_ld16(t_row + (uint32_t)c0, v);
+        for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += CW) {
+          float v[CW];
+          tmem_ldN<CW>(t_row + (uint32_t)c0, v);
           const int n = n_blk * BN + c0;
           if (row_ok && n < prm.d_out) {
-            store16<float>(D + m * prm.ldy + n, v, min(16, prm.d_out - n), prm.vec_ok != 0);
+            storeN<float, CW>(D + m * prm.ldy + n, v, min(CW, prm.d_out - n), prm.vec_ok != 0);
           }
         }
         tc::tc_fence_before();
@@ -399,62 +524,62 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) { ok = false; break; }
         }
         if (MODE == MODE_GATED) {
-          for (int c0 = half * (BN / 4); c0 < (half + 1) * (BN / 4); c0 += 16) {
-            float g[16], u[16];
-            tc::tmem_ld16(t_row + (uint32_t)c0, g);
-            tc::tmem_ld16(t_row + (uint32_t)(BN / 2 + c0), u);
+          for (int c0 = half * (BN / 4); c0 < (half + 1) * (BN / 4); c0 += CW) {
+            float g[CW], u[CW];
+            tmem_ldN<CW>(t_row + (uint32_t)c0, g);
+            tmem_ldN<CW>(t_row + (uint32_t)(BN / 2 + c0), u);
             const int n = n_blk * (BN / 2) + c0;
             if (!row_ok || n >= prm.d_out) continue;
-            const int nv = min(16, prm.d_out - n);
-            float gC[16], gZ[16];
-            lowrank16<RT>(Ct, Zt, c0, p, gC, gZ);
+            const int nv = min(CW, prm.d_out - n);
+            float gC[CW], gZ[CW];
+            lowrankN<RT, CW>(Ct, Zt, c0, p, gC, gZ);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) g[i] += gC[i];      // g = W_g x + C_g p
-            float uC[16], uZ[16];
-            lowrank16<RT>(Ct, Zt, BN / 2 + c0, p2, uC, uZ);
+            for (int i = 0; i < CW; ++i) g[i] += gC[i];      // g = W_g x + C_g p
+            float uC[CW], uZ[CW];
+            lowrankN<RT, CW>(Ct, Zt, BN / 2 + c0, p2, uC, uZ);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) u[i] += uC[i];
+            for (int i = 0; i < CW; ++i) u[i] += uC[i];
             if (prm.shared) {
-              float hp[16], hm[16];
+              float hp[CW], hm[CW];
 #pragma unroll
-              for (int i = 0; i < 16; ++i) {
+              for (int i = 0; i < CW; ++i) {
                 hp[i] = silu_fast(fmaf(prm.eps, gZ[i], g[i])) * fmaf(prm.eps, uZ[i], u[i]);
                 hm[i] = silu_fast(fmaf(-prm.eps, gZ[i], g[i])) * fmaf(-prm.eps, uZ[i], u[i]);
               }
-              store16<TO>(Y + m * prm.d_out + n, hp, nv);
-              store16<TO>(Y + (prm.T + m) * prm.d_out + n, hm, nv);
+              storeN<TO, CW>(Y + m * prm.d_out + n, hp, nv);
+              storeN<TO, CW>(Y + (prm.T + m) * prm.d_out + n, hm, nv);
             } else {
-              float h[16];
+              float h[CW];
 #pragma unroll
-              for (int i = 0; i < 16; ++i) h[i] = silu_fast(fmaf(sgn_eps, gZ[i], g[i])) * fmaf(sgn_eps, uZ[i], u[i]);
-              store16<TO>(Y + m * prm.d_out + n, h, nv);
+              for (int i = 0; i < CW; ++i) h[i] = silu_fast(fmaf(sgn_eps, gZ[i], g[i])) * fmaf(sgn_eps, uZ[i], u[i]);
+              storeN<TO, CW>(Y + m * prm.d_out + n, h, nv);
             }
           }
         } else {
           const int cbeg = s0 + half * (CHUNK / 2);
-          for (int c0 = cbeg; c0 < cbeg + CHUNK / 2; c0 += 16) {
-            float acc[16];
-            tc::tmem_ld16(t_row + (uint32_t)c0, acc);
+          for (int c0 = cbeg; c0 < cbeg + CHUNK / 2; c0 += CW) {
+            float acc[CW];
+            tmem_ldN<CW>(t_row + (uint32_t)c0, acc);
             const int n = n_blk * BN + c0;
             if (!row_ok || n >= prm.d_out) continue;
-            const int nv = min(16, prm.d_out - n);
-            float sC[16], sZ[16];
-            lowrank16<RT>(Ct, Zt, c0 - s0, p, sC, sZ);
+            const int nv = min(CW, prm.d_out - n);
+            float sC[CW], sZ[CW];
+            lowrankN<RT, CW>(Ct, Zt, c0 - s0, p, sC, sZ);
             if (prm.shared) {
-              float yp[16], ym[16];
+              float yp[CW], ym[CW];
 #pragma unroll
-              for (int i = 0; i < 16; ++i) {
+              for (int i = 0; i < CW; ++i) {
                 const float base = acc[i] + sC[i];
                 yp[i] = apply_act(fmaf(prm.eps, sZ[i], base), prm.act);
                 ym[i] = apply_act(fmaf(-prm.eps, sZ[i], base), prm.act);
               }
-              store16<TO>(Y + m * prm.d_out + n, yp, nv);
-              store16<TO>(Y + (prm.T + m) * prm.d_out + n, ym, nv);
+              storeN<TO, CW>(Y + m * prm.d_out + n, yp, nv);
+              storeN<TO, CW>(Y + (prm.T + m) * prm.d_out + n, ym, nv);
             } else {
-              float y[16];
+              float y[CW];
 #pragma unroll
-              for (int i = 0; i < 16; ++i) y[i] = apply_act(fmaf(sgn_eps, sZ[i], acc[i] + sC[i]), prm.act);
-              store16<TO>(Y + m * prm.d_out + n, y, nv);
+              for (int i = 0; i < CW; ++i) y[i] = apply_act(fmaf(sgn_eps, sZ[i], acc[i] + sC[i]), prm.act);
+              storeN<TO, CW>(Y + m * prm.d_out + n, y, nv);
             }
           }
         }

@@ -15,7 +15,7 @@ import torch
 
 import paper_2607_01125_gb300 as zo
 from oracle import philox, layers, loss as oloss, optim, basis, graphs
-from synth import normal, lowrank_activations
+from synth import normal, lowrank_activations, quantize_int4_g128
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
@@ -161,6 +161,56 @@ def test_pair_forward_gated(ctx, T, shared, dt):
     u, _ = _oracle_pair(X, Wu, Uu, Cu, eps, T, shared, seed, 1, query, d_out, r)
     ref = layers.silu(g) * u
     assert np.abs(np64(H) - ref).max() <= 1e-4 * np.abs(ref).max()
+
+
+# ---------------- INT4 weights ----------------
+def _int4_layer(d_in, d_out, r, seed, lid):
+    Wf = normal((d_out, d_in), seed, DEV, std=0.02)
+    packed, scales = quantize_int4_g128(Wf)
+    U = normal((d_in, r), seed + 1, DEV) / np.sqrt(d_in)
+    C = normal((d_out * r,), seed + 2, DEV, std=0.3)
+    L = zo.make_layer(packed, U, C, lid, w_scales=scales, wtype=zo.DT_INT4_G128, d_in=d_in)
+    Wd = layers.dequant_int4_g128(packed.cpu().numpy(), scales.float().cpu().numpy(), d_in)
+    return L, Wd, U, C
+
+
+@pytest.mark.parametrize("d_in,d_out,r,T,shared", [(1024, 520, 16, 200, False), (512, 256, 32, 64, True),
+                                                   (4096, 1024, 16, 130, False)])
+def test_pair_forward_int4(ctx, d_in, d_out, r, T, shared):
+    # the kernel rounds every dequantised weight q * s to bf16 (scale via bf16): |dw| <= 2^-8 |w|
+    eps, seed, query, lid = 0.5, 13, 2, 6
+    L, Wd, U, C = _int4_layer(d_in, d_out, r, 40, lid)
+    X = normal(((T if shared else 2 * T), d_in), 41, DEV, dtype=torch.bfloat16)
+    Y = torch.empty(2 * T, d_out, dtype=torch.float32, device=DEV)
+    zo.zoact_pair_forward(ctx, L, X, T, shared, eps, seed, query, Y)
+    torch.cuda.synchronize()
+    Zm = philox.perturbation(seed, lid, query, d_out, r)
+    Xn = np64(X)
+    ref = layers.pair_forward(Wd, np64(U), np64(C).reshape(d_out, r), Zm, Xn, eps, T, shared)
+    Xs = np.concatenate([Xn, Xn]) if shared else Xn
+    absw = np.abs(Xs) @ np.abs(Wd).T
+    absl = np.abs(Xs @ np64(U)) @ (np.abs(np64(C).reshape(d_out, r)) + eps * np.abs(Zm)).T
+    err = np.abs(np64(Y) - ref)
+    assert np.all(err <= 2.0 ** -8 * absw + 8 * np.sqrt(d_in) * 2.0 ** -24 * (absw + absl) + 1e-6), err.max()
+    assert err.max() <= 2e-2 * np.abs(ref).max()
+
+
+def test_pair_forward_gated_int4(ctx):
+    d_in, d_out, r, T = 1024, 384, 16, 96
+    eps, seed, query = 0.25, 3, 5
+    Lg, Wg, Ug, Cg = _int4_layer(d_in, d_out, r, 50, 0)
+    Lu, Wu, Uu, Cu = _int4_layer(d_in, d_out, r, 60, 1)
+    X = normal((T, d_in), 61, DEV, dtype=torch.bfloat16)
+    H = torch.empty(2 * T, d_out, dtype=torch.bfloat16, device=DEV)
+    zo.zoact_pair_forward_gated(ctx, Lg, Lu, X, T, True, eps, seed, query, H)
+    torch.cuda.synchronize()
+    g = layers.pair_forward(Wg, np64(Ug), np64(Cg).reshape(d_out, r), philox.perturbation(seed, 0, query, d_out, r),
+                            np64(X), eps, T, True)
+    u = layers.pair_forward(Wu, np64(Uu), np64(Cu).reshape(d_out, r), philox.perturbation(seed, 1, query, d_out, r),
+                            np64(X), eps, T, True)
+    ref = layers.silu(g) * u
+    assert np.abs(np64(H) - ref).max() <= 2e-2 * np.abs(ref).max()
+    assert np.mean(np.abs(np64(H) - ref)) <= 5e-3 * np.mean(np.abs(ref))
 
 
 # ---------------- loss ----------------

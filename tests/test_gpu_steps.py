@@ -21,7 +21,8 @@ import torch
 import paper_2607_01125_gb300 as zo
 from paper_2607_01125_gb300.model import AdaptedLinear, ZOStep, coefficient_offsets
 from oracle import basis, graphs, loss as oloss, optim, philox
-from synth import workload, normal, lowrank_activations, random_orthonormal, tensor_seed
+from synth import workload, normal, lowrank_activations, random_orthonormal, tensor_seed, quantize_int4_g128
+from oracle import layers as olayers
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
@@ -38,15 +39,24 @@ def _build(w, c_std=0.01):
     specs = w.linears()
     offs = coefficient_offsets(specs, w.r)
     lins, ora = [], {}
+    Wfp64 = {}
     for s, off in zip(specs, offs):
-        W = normal((s.d_out, s.d_in), tensor_seed(w, "W", s.name), DEV, std=w.weight_std, dtype=dt)
         U = random_orthonormal(s.d_in, w.r, tensor_seed(w, "U", s.name), DEV)
-        lins.append(AdaptedLinear(s.name, W, U, s.layer_id, off, w.r))
+        if w.wtype == "int4_g128":
+            Wf = normal((s.d_out, s.d_in), tensor_seed(w, "W", s.name), DEV, std=w.weight_std)
+            packed, scales = quantize_int4_g128(Wf)
+            lins.append(AdaptedLinear(s.name, packed, U, s.layer_id, off, w.r, w_scales=scales,
+                                      wtype=zo.DT_INT4_G128, d_in=s.d_in))
+            Wfp64[s.name] = olayers.dequant_int4_g128(packed.cpu().numpy(), scales.float().cpu().numpy(), s.d_in)
+        else:
+            W = normal((s.d_out, s.d_in), tensor_seed(w, "W", s.name), DEV, std=w.weight_std, dtype=dt)
+            lins.append(AdaptedLinear(s.name, W, U, s.layer_id, off, w.r))
     step = ZOStep(zo.Context(0), w.kind, lins, w.T, w.act_dtype, eps=w.eps, lr=w.lr)
     step.C.copy_(normal(tuple(step.C.shape), tensor_seed(w, "C0"), DEV, std=c_std))
     for l in lins:
         C = n64(step.C[l.offset:l.offset + l.d_out * w.r]).reshape(l.d_out, w.r)
-        ora[l.name] = dict(W=n64(l.W), U=n64(l.U), C=C, layer_id=l.layer_id)
+        Wo = Wfp64[l.name] if l.name in Wfp64 else n64(l.W)
+        ora[l.name] = dict(W=Wo, U=n64(l.U), C=C, layer_id=l.layer_id)
     return step, ora
 
 
@@ -94,7 +104,8 @@ def test_llama_mlp_step_full_width():
     step.ctx.close()
 
 
-@pytest.mark.parametrize("name,n_dec,T", [("llama_stack_bf16", 2, 64), ("opt_stack_fp16", 2, 48)])
+@pytest.mark.parametrize("name,n_dec,T", [("llama_stack_bf16", 2, 64), ("opt_stack_fp16", 2, 48),
+                                          ("llama_stack_int4", 1, 64)])
 def test_stack_step(name, n_dec, T):
     w = workload(name, T=T, n_decoder=n_dec)
     step, ora = _build(w)
