@@ -1,26 +1,27 @@
 #!/usr/bin/env python
 """ZO-step throughput of the ZO-Act hot path on GB300.
 
-Workload (default): the Llama-3-8B MLP block in bf16 -- gate/up 4096 -> 14336
-on a shared input, SiLU gate, down 14336 -> 4096 -- r = 16, T = 2048 tokens per
+Default workload: the Llama-3-8B MLP block in bf16 -- gate/up 4096 -> 14336 on
+a shared input, SiLU gate, down 14336 -> 4096 -- r = 16, T = 2048 tokens per
 perturbation (4096 stacked rows for the +/- pair), MSE to N(0,1) targets,
-eps = 1e-3, Adam on all coefficients.  Synthetic data: rank-64 Gaussian signal
-plus 5% noise, unit RMS per token; W ~ N(0, 0.02); bases from a 2048-token
-calibration batch (Algorithm 1, on the device, before timing).
+eps = 1e-3, Adam on all coefficients.  Other workloads (--workload):
+llama_stack_bf16 (224 linears, T = 16 x 256), llama_stack_int4 (same, INT4 g128
+weights), opt_stack_fp16 (240 linears, r = 32).  Synthetic data: rank-64
+Gaussian signal plus 5% noise, unit RMS per token; W ~ N(0, 0.02).  The bases
+come from Algorithm 1 on the device before timing: one calibration forward pass
+of the base model, then zoact_basis_init on every layer's input.
 
-One step = zoact_lowrank_proj + zoact_pair_forward_gated (gate/up) +
-zoact_lowrank_proj + zoact_pair_forward (down) + zoact_loss_pair +
+One step = per adapted linear zoact_lowrank_proj + zoact_pair_forward (gate/up:
+zoact_pair_forward_gated) with the glue ops, then zoact_loss_pair and
 zoact_adam_step, all on one stream, no host synchronisation.
 
-value = training tokens/s = world_size * T / step time (device time, CUDA
-events around exactly --steps steps, max over ranks).  The weights (352 MB) are
-larger than L2 (129 MB), so every step streams them from HBM.
-`--impl reference` times the CPU oracle (numpy fp64) on a bounded sample of the
-same workload instead.
+value = training tokens/s = world_size * T / step time (CUDA events around
+exactly --steps steps, max over ranks).  The frozen weights are larger than L2
+(129 MB), so every step reads them from HBM.  `--impl reference` times the CPU
+oracle (numpy fp64) on a bounded sample of the default workload instead.
 """
 import argparse
 import json
-import math
 import os
 import statistics
 import subprocess
@@ -32,10 +33,8 @@ sys.path.insert(0, ROOT)
 
 METRIC = "ZO-step tokens/s per adapted-linear stack; % of HBM or tensor-pipe roofline"
 UNIT = "tokens/s"
-T_TOKENS = 2048
-D_MODEL, D_FF, RANK = 4096, 14336, 16
-N_CAL = 2048
-EPS = 1e-3
+DEFAULT_WORKLOAD = "llama_mlp_bf16"
+N_CAL = {"llama_mlp_bf16": 2048, "llama_stack_bf16": 512, "llama_stack_int4": 512, "opt_stack_fp16": 4096}
 LR = 1e-4
 
 
@@ -112,76 +111,57 @@ def dist_setup():
     return world, rank, local
 
 
-def build_mlp(ctx, dev, rank, seed=0):
-    """Weights, bases and the ZOStep of the Llama MLP block (inputs per rank for weak scaling)."""
+def build(ctx, dev, rank, name, tokens=None):
+    """Weights, bases (Algorithm 1 on the device) and the ZOStep of a workload.
+
+    Returns (step, x, target, basis_seconds, workload).  Weights are the same on every
+    rank; the calibration and training tokens and the targets are drawn per rank.
+    """
     import torch
     import paper_2607_01125_gb300 as zo
-    from paper_2607_01125_gb300.model import AdaptedLinear, ZOStep
-    from synth import workload, normal, lowrank_activations, tensor_seed
-    w = workload("llama_mlp_bf16", seed=seed)
-    x_all, _ = lowrank_activations(N_CAL + T_TOKENS, D_MODEL, 64, 0.05, tensor_seed(w, "x", rank), dev)
-    X_cal, x = x_all[:N_CAL].contiguous(), x_all[N_CAL:].contiguous()
-    target = normal((T_TOKENS, D_MODEL), tensor_seed(w, "target", rank), dev, dtype=torch.bfloat16)
-    Wg = normal((D_FF, D_MODEL), tensor_seed(w, "W", "gate"), dev, std=w.weight_std, dtype=torch.bfloat16)
-    Wu = normal((D_FF, D_MODEL), tensor_seed(w, "W", "up"), dev, std=w.weight_std, dtype=torch.bfloat16)
-    Wd = normal((D_MODEL, D_FF), tensor_seed(w, "W", "down"), dev, std=w.weight_std, dtype=torch.bfloat16)
-    # Algorithm 1: one calibration pass of the base model, bases of each layer's input
-    U_x = torch.empty(D_MODEL, RANK, device=dev)
-    zo.zoact_basis_init(ctx, X_cal, RANK, U_x, oversample=16, n_iter=8, seed=tensor_seed(w, "basis", "x"))
-    C0 = torch.zeros(D_FF * RANK, device=dev)
-    Hc = torch.empty(2 * N_CAL, D_FF, dtype=torch.bfloat16, device=dev)
-    zo.zoact_pair_forward_gated(ctx, zo.make_layer(Wg, U_x, C0, 0), zo.make_layer(Wu, U_x, C0, 1), X_cal, N_CAL,
-                                True, 0.0, 0, 0, Hc)
-    U_h = torch.empty(D_FF, RANK, device=dev)
-    zo.zoact_basis_init(ctx, Hc[:N_CAL].contiguous(), RANK, U_h, oversample=16, n_iter=8,
-                        seed=tensor_seed(w, "basis", "h"))
-    del Hc
-    lins = [AdaptedLinear("gate", Wg, U_x, 0, 0, RANK), AdaptedLinear("up", Wu, U_x, 1, D_FF * RANK, RANK),
-            AdaptedLinear("down", Wd, U_h, 2, 2 * D_FF * RANK, RANK)]
-    step = ZOStep(ctx, "llama_mlp", lins, T_TOKENS, "bf16", eps=EPS, lr=LR)
-    return step, x, target
+    from paper_2607_01125_gb300.model import AdaptedLinear, ZOStep, coefficient_offsets, calibrate_bases
+    from synth import workload, normal, lowrank_activations, quantize_int4_g128, tensor_seed
+    w = workload(name) if tokens is None else workload(name, T=tokens)
+    dt = {"bf16": torch.bfloat16, "fp16": torch.float16}[w.act_dtype]
+    specs = w.linears()
+    offs = coefficient_offsets(specs, w.r)
+    lins = []
+    for s, off in zip(specs, offs):
+        U = torch.zeros(s.d_in, w.r, device=dev)
+        if w.wtype == "int4_g128":
+            Wf = normal((s.d_out, s.d_in), tensor_seed(w, "W", s.name), dev, std=w.weight_std)
+            packed, scales = quantize_int4_g128(Wf)
+            del Wf
+            lins.append(AdaptedLinear(s.name, packed, U, s.layer_id, off, w.r, w_scales=scales,
+                                      wtype=zo.DT_INT4_G128, d_in=s.d_in))
+        else:
+            W = normal((s.d_out, s.d_in), tensor_seed(w, "W", s.name), dev, std=w.weight_std, dtype=dt)
+            lins.append(AdaptedLinear(s.name, W, U, s.layer_id, off, w.r))
+    n_cal = N_CAL[name]
+    x_all, _ = lowrank_activations(n_cal + w.T, w.d_model, 64, 0.05, tensor_seed(w, "x", rank), dev, dtype=dt)
+    x_cal, x = x_all[:n_cal].contiguous(), x_all[n_cal:].contiguous()
+    del x_all
+    target = normal((w.T, w.d_model), tensor_seed(w, "target", rank), dev, dtype=dt) if w.kind == "llama_mlp" else None
+    # Algorithm 1: calibration forward pass of the base model, one basis per layer input
+    step_cal = ZOStep(ctx, w.kind, lins, n_cal, w.act_dtype, eps=w.eps)
+    torch.cuda.synchronize()
+    t0 = time.time()
+    calibrate_bases(ctx, step_cal, x_cal, w.r, oversample=16, n_iter=8, seed=tensor_seed(w, "basis"))
+    torch.cuda.synchronize()
+    basis_s = time.time() - t0
+    del step_cal
+    step = ZOStep(ctx, w.kind, lins, w.T, w.act_dtype, eps=w.eps, lr=LR)
+    return step, x, target, basis_s, w
 
 
-class MLPRunner:
-    """One ZO step of the MLP block with the tensor-core launches bracketed by CUDA events."""
-
-    def __init__(self, step, world):
-        import torch
-        import paper_2607_01125_gb300 as zo
-        self.zo, self.torch = zo, torch
-        self.s = step
-        self.world = world
-        T = step.T
-        dev = step.device
-        self.P_x = torch.empty(T, RANK, device=dev)
-        self.P_h = torch.empty(2 * T, RANK, device=dev)
-        self.H = torch.empty(2 * T, D_FF, dtype=torch.bfloat16, device=dev)
-        self.Y = torch.empty(2 * T, D_MODEL, dtype=torch.bfloat16, device=dev)
-        self.events = []
-
-    def run(self, x, target, t, seed, instrument):
-        zo, torch, s = self.zo, self.torch, self.s
-        g, u, d = s.by_name["gate"], s.by_name["up"], s.by_name["down"]
-        zo.zoact_lowrank_proj(s.ctx, x, g.U, self.P_x)                 # gate and up share U (same input)
-        if instrument:
-            e0 = torch.cuda.Event(enable_timing=True); e0.record()
-        zo.zoact_pair_forward_gated(s.ctx, g.layer, u.layer, x, s.T, True, s.eps, seed, t, self.H,
-                                    P_gate=self.P_x, P_up=self.P_x)
-        if instrument:
-            e1 = torch.cuda.Event(enable_timing=True); e1.record()
-        zo.zoact_lowrank_proj(s.ctx, self.H, d.U, self.P_h)
-        if instrument:
-            e2 = torch.cuda.Event(enable_timing=True); e2.record()
-        zo.zoact_pair_forward(s.ctx, d.layer, self.H, s.T, False, s.eps, seed, t, self.Y, P=self.P_h)
-        if instrument:
-            e3 = torch.cuda.Event(enable_timing=True); e3.record()
-            self.events.append((e0, e1, e2, e3))
-        s.loss(self.Y, target)
-        if self.world > 1:
-            from paper_2607_01125_gb300.dp import allreduce_loss
-            allreduce_loss(s.loss_out)           # L+, L-, D and a are means over equal token counts
-        s.update(t, seed, t)
-        return s.loss_out
+def run_step(step, x, target, t, seed, world):
+    Y = step.forward(x, seed, t)
+    step.loss(Y, target)
+    if world > 1:
+        from paper_2607_01125_gb300.dp import allreduce_loss
+        allreduce_loss(step.loss_out)            # L+, L-, D and a are means over equal token counts
+    step.update(t, seed, t)
+    return step.loss_out
 
 
 def run_ours(args):
@@ -194,54 +174,56 @@ def run_ours(args):
     dev = f"cuda:{local}"
     torch.cuda.set_device(local)
     ctx = zo.Context(local)
-    step, x, target = build_mlp(ctx, dev, rank)
-    runner = MLPRunner(step, world)
+    step, x, target, basis_s, w = build(ctx, dev, rank, args.workload, args.tokens)
     seed = 1234
 
     def barrier():
         if world > 1:
             dist.barrier()
 
-    # warm-up (untimed), then a ~2 s soak so clocks are at their loaded steady state
     t = 1
     for _ in range(args.warmup):
-        runner.run(x, target, t, seed, False); t += 1
+        run_step(step, x, target, t, seed, world); t += 1
     sampler = ClockSampler(local)
     sampler.start()
     torch.cuda.synchronize()
-    soak_end = time.time() + args.soak
+    soak_end = time.time() + args.soak       # untimed steps so the clocks reach their loaded state
     while time.time() < soak_end:
-        for _ in range(20):
-            runner.run(x, target, t, seed, False); t += 1
+        run_step(step, x, target, t, seed, world); t += 1
         torch.cuda.synchronize()
 
     # ---- timed region: exactly args.steps steps ----
     n0 = ctx.launch_count()
+    step.timer = []
     barrier(); torch.cuda.synchronize()
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.nvtx.range_push("timed")          # profilers select the timed steps by this range
     start.record()
     for _ in range(args.steps):
-        runner.run(x, target, t, seed, True); t += 1
+        run_step(step, x, target, t, seed, world); t += 1
     end.record()
     torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize(); barrier()
     launches = ctx.launch_count() - n0
     ms = start.elapsed_time(end) / args.steps
-    gemm_ms = [(a.elapsed_time(b), c.elapsed_time(d)) for a, b, c, d in runner.events]
+    gemm_ms = sum(a.elapsed_time(b) for a, b, _ in step.timer)
+    gemm_flops = sum(f for _, _, f in step.timer)
+    step.timer = None
 
     # ---- end to end through the public API with host buffers ----
     x_h = x.cpu().pin_memory()
-    t_h = target.cpu().pin_memory()
+    t_h = target.cpu().pin_memory() if target is not None else None
     out_h = torch.empty(4, dtype=torch.float64).pin_memory()
-    x_d, t_d = torch.empty_like(x), torch.empty_like(target)
+    x_d = torch.empty_like(x)
+    t_d = torch.empty_like(target) if target is not None else None
     barrier(); torch.cuda.synchronize()
     e_s, e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e_s.record()
     for _ in range(args.steps):
         x_d.copy_(x_h, non_blocking=True)
-        t_d.copy_(t_h, non_blocking=True)
-        out = runner.run(x_d, t_d, t, seed, False); t += 1
+        if t_d is not None:
+            t_d.copy_(t_h, non_blocking=True)
+        out = run_step(step, x_d, t_d, t, seed, world); t += 1
         out_h.copy_(out, non_blocking=True)
     e_e.record()
     torch.cuda.synchronize(); barrier()
@@ -256,56 +238,47 @@ def run_ours(args):
     if rank != 0:
         return
     hbm, tf_burst, tf_sust, peak_kind = _peaks()
-    T = T_TOKENS
-    flops_gated = 2.0 * T * D_MODEL * (2 * D_FF)          # gate + up on T shared rows
-    flops_down = 2.0 * (2 * T) * D_FF * D_MODEL            # down on 2T stacked rows
-    tg = statistics.mean(a for a, _ in gemm_ms)
-    td = statistics.mean(b for _, b in gemm_ms)
-    achieved = (flops_gated + flops_down) / ((tg + td) * 1e-3) / 1e12
+    # a step of about a millisecond times its kernels as bursts; the stacks' ~100 ms steps use the sustained peak
+    long_step = ms > 20.0
+    peak = tf_sust if long_step else tf_burst
+    achieved = gemm_flops / (gemm_ms * 1e-3) / 1e12
+    T = w.T
+    h2d = x.numel() * x.element_size() + (target.numel() * target.element_size() if target is not None else 0)
     line = {
         "metric": METRIC, "value": world * T / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": "llama_mlp_bf16", "tokens_per_perturbation": T, "stacked_rows": 2 * T,
-                   "d_model": D_MODEL, "d_ff": D_FF, "r": RANK, "eps": EPS, "estimator": "two-sided, q=1",
-                   "l2": "inputs larger than L2 (352 MB of frozen weights streamed per step)",
+        "scaling": "weak", "vs_baseline": None, "dtype": "int4-bf16" if w.wtype == "int4_g128" else w.act_dtype,
+        "data": "synthetic",
+        "config": {"workload": w.name, "tokens_per_perturbation": T, "stacked_rows": 2 * T, "r": w.r, "eps": w.eps,
+                   "adapted_linears": len(w.linears()), "estimator": "two-sided, q=1",
+                   "l2": "inputs larger than L2 (frozen weights streamed from HBM every step)",
                    "parallelism": f"dp{world}" if world > 1 else "single"},
         "evaluated_tokens_per_s": world * 2 * T / (ms * 1e-3),
         "zo_steps_per_s": 1e3 / ms,
-        "kernel_ms": {"pair_forward_gated": tg, "pair_forward_down": td},
-        "roofline": {"bound": "tensor", "achieved": achieved, "peak": tf_burst, "unit": "TFLOP/s",
-                     "frac": achieved / tf_burst, "peak_kind": f"bf16 dense burst, {peak_kind}",
-                     "kernel": "pair_tc_kernel (gated gate/up + down)",
+        "pair_forward_ms_per_step": gemm_ms / args.steps,
+        "basis_init_s": basis_s,
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak,
+                     "peak_kind": f"bf16 dense {'sustained' if long_step else 'burst'}, {peak_kind}",
+                     "kernel": "pair_tc_kernel (every pair-forward launch of the step)",
+                     "algorithmic_flops_per_step": gemm_flops / args.steps,
                      "traffic": None},
-        "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": UNIT,
-                "h2d_bytes_per_step": x.numel() * 2 + target.numel() * 2, "d2h_bytes_per_step": 32},
+        "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": 32},
         "gpu_launches": launches,
         "clocks": clocks,
         "device_status": status,
     }
-    if world == 1 and not args.no_cpu_baseline:
+    if world == 1 and not args.no_cpu_baseline and args.workload == DEFAULT_WORKLOAD:
         line["cpu_baseline"] = cpu_baseline(step, budget_s=args.cpu_budget)
     print(json.dumps(line))
-
-
-def _oracle_sample_step(step, n_tok, seed):
-    """Everything the oracle needs for one ZO step on n_tok tokens (fp64 numpy), prepared outside the timing."""
-    import numpy as np
-    from synth import lowrank_activations, normal, random_orthonormal
-    n64 = lambda t: t.detach().double().cpu().numpy()
-    g, u, d = step.by_name["gate"], step.by_name["up"], step.by_name["down"]
-    lay = [dict(W=n64(l.W), U=random_orthonormal(l.d_in, RANK, 90 + i).double().numpy(),
-                C=np.zeros((l.d_out, RANK)), layer_id=l.layer_id) for i, l in enumerate((g, u, d))]
-    x, _ = lowrank_activations(n_tok, D_MODEL, 64, 0.05, seed, "cpu")
-    tgt = normal((n_tok, D_MODEL), seed + 1, "cpu", dtype=__import__("torch").bfloat16)
-    return lay, x.double().numpy(), tgt.double().numpy()
 
 
 def _oracle_step(lay, x, tgt, seed, query, t):
     import numpy as np
     from oracle import graphs, loss as oloss, optim, philox
-    Y = graphs.llama_mlp_forward(lay, x, EPS, seed, query, store="bf16")
-    _, _, _, a = oloss.loss_pair(Y, x.shape[0], tgt, EPS)
+    Y = graphs.llama_mlp_forward(lay, x, 1e-3, seed, query, store="bf16")
+    _, _, _, a = oloss.loss_pair(Y, x.shape[0], tgt, 1e-3)
     for l in lay:
         gz = optim.zo_gradient(a, philox.perturbation(seed, l["layer_id"], query, *l["C"].shape))
         l.setdefault("m", np.zeros_like(l["C"]))
@@ -313,10 +286,22 @@ def _oracle_step(lay, x, tgt, seed, query, t):
         l["C"], l["m"], l["v"] = optim.adam_step(l["C"], l["m"], l["v"], gz, LR, 0.9, 0.999, 1e-8, t)
 
 
-def cpu_baseline(step, budget_s=20.0, n_tok=None):
+def _oracle_mlp(weights, n_tok):
+    """The oracle's inputs for ZO steps of the MLP block on n_tok tokens (fp64), outside any timing."""
+    import numpy as np
+    import torch
+    from synth import lowrank_activations, normal, random_orthonormal
+    lay = [dict(W=W, U=random_orthonormal(W.shape[1], 16, 90 + i).double().numpy(),
+                C=np.zeros((W.shape[0], 16)), layer_id=i) for i, W in enumerate(weights)]
+    x, _ = lowrank_activations(n_tok, 4096, 64, 0.05, 77, "cpu")
+    tgt = normal((n_tok, 4096), 78, "cpu", dtype=torch.bfloat16)
+    return lay, x.double().numpy(), tgt.double().numpy()
+
+
+def cpu_baseline(step, budget_s=20.0, n_tok=256):
     """The oracle (as it stands) on the host cores: ZO steps of the same block on a token sample."""
-    n_tok = n_tok or 256
-    lay, x, tgt = _oracle_sample_step(step, n_tok, 77)
+    n64 = lambda t: t.detach().double().cpu().numpy()
+    lay, x, tgt = _oracle_mlp([n64(step.by_name[n].W) for n in ("gate", "up", "down")], n_tok)
     t0 = time.time()
     _oracle_step(lay, x, tgt, 5, 0, 1)
     one = time.time() - t0
@@ -337,20 +322,14 @@ def run_reference(args):
     if rank != 0:
         return
     import torch
-    import numpy as np
-    from synth import workload, normal, tensor_seed, lowrank_activations, random_orthonormal
-    w = workload("llama_mlp_bf16")
+    from synth import workload, normal, tensor_seed
+    w = workload(DEFAULT_WORKLOAD)
     n_tok = args.ref_tokens
-    # weights drawn on the CPU with the same shapes (the reference arm never touches the GPU)
-    shapes = [("gate", D_FF, D_MODEL), ("up", D_FF, D_MODEL), ("down", D_MODEL, D_FF)]
-    lay = []
-    for i, (nm, do, di) in enumerate(shapes):
-        Wt = normal((do, di), tensor_seed(w, "W", nm), "cpu", std=w.weight_std, dtype=torch.bfloat16)
-        lay.append(dict(W=Wt.double().numpy(), U=random_orthonormal(di, RANK, 90 + i).double().numpy(),
-                        C=np.zeros((do, RANK)), layer_id=i))
-    x, _ = lowrank_activations(n_tok, D_MODEL, 64, 0.05, 77, "cpu")
-    x = x.double().numpy()
-    tgt = normal((n_tok, D_MODEL), 78, "cpu", dtype=torch.bfloat16).double().numpy()
+    # the weights drawn on the CPU with the same shapes (the reference arm never touches the GPU)
+    weights = [normal((do, di), tensor_seed(w, "W", nm), "cpu", std=w.weight_std,
+                      dtype=torch.bfloat16).double().numpy()
+               for nm, do, di in (("gate", 14336, 4096), ("up", 14336, 4096), ("down", 4096, 14336))]
+    lay, x, tgt = _oracle_mlp(weights, n_tok)
     t = 1
     for _ in range(args.warmup):
         _oracle_step(lay, x, tgt, 5, t, t); t += 1
@@ -364,8 +343,7 @@ def run_reference(args):
         "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f64", "data": "synthetic", "impl": "reference",
-        "config": {"workload": "llama_mlp_bf16", "tokens_per_perturbation": n_tok, "d_model": D_MODEL,
-                   "d_ff": D_FF, "r": RANK, "eps": EPS},
+        "config": {"workload": DEFAULT_WORKLOAD, "tokens_per_perturbation": n_tok, "r": 16, "eps": 1e-3},
         "cpu_baseline": {"value": v, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample},
         "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
@@ -377,6 +355,9 @@ def main():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
+                    choices=["llama_mlp_bf16", "llama_stack_bf16", "llama_stack_int4", "opt_stack_fp16"])
+    ap.add_argument("--tokens", type=int, default=None, help="tokens per perturbation (default: the workload's)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--soak", type=float, default=2.0,
                     help="seconds of untimed steps before the timed region (clocks reach their loaded state)")

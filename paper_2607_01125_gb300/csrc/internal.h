@@ -28,6 +28,8 @@ enum ScratchSlot {
   SLOT_BASIS,        // Gram matrix and subspace-iteration workspace
   SLOT_BASIS_X,      // transposed calibration activations
   SLOT_UT,           // 16-bit split copy of the basis for the tensor-core projection
+  SLOT_WDQ0,         // bf16 copy of an INT4 weight (staged INT4 pair forward)
+  SLOT_WDQ1,         // second copy (gated up weight)
   SLOT_COUNT
 };
 
@@ -110,6 +112,10 @@ struct PairArgs {
   uint32_t layer_id2;
 };
 int launch_pair_simt(Ctx* ctx, const PairArgs& a);
+// INT4 g128 weight [d_out, d_in/2] + fp16 scales -> bf16 [d_out, d_in].
+int launch_dequant_int4(Ctx* ctx, const void* Wq, const void* Ws, void* Wb, int64_t d_out, int d_in);
+// Row count from which the INT4 pair forward expands W to bf16 first instead of dequantising per M-tile.
+constexpr int64_t INT4_STAGED_MIN_ROWS = 1024;
 int launch_pair_tc(Ctx* ctx, const PairArgs& a);
 // Plain product D[M, N] (fp32) = A[M, K] * B[N, K]^T with 16-bit A, B (K-major), on tcgen05.
 int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int M, int N, int K,

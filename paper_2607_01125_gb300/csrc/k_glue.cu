@@ -1,6 +1,8 @@
 // Glue ops of the synthetic graphs: per-row RMS normalisation (no gain) and the
-// attention-free mixer rms(q + rep(k) + rep(v)).  One block per row; the row is
-// read twice (sum of squares, then scale), the second time from L1/L2.
+// attention-free mixer rms(q + rep(k) + rep(v)).  One block per row.  When the
+// row is a whole number of 16-byte vectors (and fits), each thread keeps its
+// vectors in registers, so the row is read once and written once; otherwise a
+// two-pass kernel reads it twice (the second time from L1/L2).
 #include "internal.h"
 
 namespace zoact {
@@ -62,28 +64,168 @@ mix_rms_kernel(const T* __restrict__ Q, const T* __restrict__ K, const T* __rest
   for (int i = threadIdx.x; i < n; i += GLUE_THREADS) y[i] = from_f32<T>(mix_at(q, k, v, i, n_rep, head_dim) * inv);
 }
 
+// ---- single-pass versions: VPT 16-byte vectors per thread held in registers ----
+template <typename T>
+struct Vec {
+  static constexpr int N = 16 / sizeof(T);           // elements per 16-byte vector
+};
+
+template <typename T>
+__device__ __forceinline__ void vec_to_f32(const uint4& u, float* f) {
+  const T* e = reinterpret_cast<const T*>(&u);
+#pragma unroll
+  for (int i = 0; i < Vec<T>::N; ++i) f[i] = to_f32<T>(e[i]);
+}
+
+template <typename T>
+__device__ __forceinline__ uint4 f32_to_vec(const float* f) {
+  uint4 u;
+  T* e = reinterpret_cast<T*>(&u);
+#pragma unroll
+  for (int i = 0; i < Vec<T>::N; ++i) e[i] = from_f32<T>(f[i]);
+  return u;
+}
+
+template <typename T, int VPT>
+__global__ void __launch_bounds__(GLUE_THREADS)
+rms_norm_reg_kernel(const T* __restrict__ X, T* __restrict__ Y, int n, float eps) {
+  constexpr int E = Vec<T>::N;
+  __shared__ float red[GLUE_THREADS / 32];
+  const int64_t row = blockIdx.x;
+  const uint4* x = reinterpret_cast<const uint4*>(X + row * n);
+  const int nv = n / E;
+  float v[VPT][E];
+  float ss = 0.f;
+#pragma unroll
+  for (int j = 0; j < VPT; ++j) {
+    const int idx = threadIdx.x + j * GLUE_THREADS;
+    if (idx < nv) {
+      vec_to_f32<T>(__ldg(x + idx), v[j]);
+#pragma unroll
+      for (int i = 0; i < E; ++i) ss = fmaf(v[j][i], v[j][i], ss);
+    }
+  }
+  const float inv = rsqrtf(block_sum(ss, red) / (float)n + eps);
+  uint4* y = reinterpret_cast<uint4*>(Y + row * n);
+#pragma unroll
+  for (int j = 0; j < VPT; ++j) {
+    const int idx = threadIdx.x + j * GLUE_THREADS;
+    if (idx < nv) {
+#pragma unroll
+      for (int i = 0; i < E; ++i) v[j][i] *= inv;
+      y[idx] = f32_to_vec<T>(v[j]);
+    }
+  }
+}
+
+template <typename T, int VPT>
+__global__ void __launch_bounds__(GLUE_THREADS)
+mix_rms_reg_kernel(const T* __restrict__ Q, const T* __restrict__ K, const T* __restrict__ V, T* __restrict__ Y,
+                   int n, int n_rep, int head_dim, float eps) {
+  constexpr int E = Vec<T>::N;
+  __shared__ float red[GLUE_THREADS / 32];
+  const int64_t row = blockIdx.x;
+  const int nk = n / n_rep;
+  const uint4* q = reinterpret_cast<const uint4*>(Q + row * n);
+  const T* k = K + row * nk;
+  const T* v = V + row * nk;
+  const int nv = n / E;
+  float m[VPT][E];
+  float ss = 0.f;
+#pragma unroll
+  for (int j = 0; j < VPT; ++j) {
+    const int idx = threadIdx.x + j * GLUE_THREADS;
+    if (idx < nv) {
+      const int i0 = idx * E;                            // head_dim % E == 0: one kv head per vector
+      const int kv = (i0 / head_dim) / n_rep * head_dim + (i0 % head_dim);
+      float a[E], b[E];
+      vec_to_f32<T>(__ldg(q + idx), m[j]);
+      vec_to_f32<T>(__ldg(reinterpret_cast<const uint4*>(k + kv)), a);
+      vec_to_f32<T>(__ldg(reinterpret_cast<const uint4*>(v + kv)), b);
+#pragma unroll
+      for (int i = 0; i < E; ++i) {
+        m[j][i] = m[j][i] + a[i] + b[i];
+        ss = fmaf(m[j][i], m[j][i], ss);
+      }
+    }
+  }
+  const float inv = rsqrtf(block_sum(ss, red) / (float)n + eps);
+  uint4* y = reinterpret_cast<uint4*>(Y + row * n);
+#pragma unroll
+  for (int j = 0; j < VPT; ++j) {
+    const int idx = threadIdx.x + j * GLUE_THREADS;
+    if (idx < nv) {
+#pragma unroll
+      for (int i = 0; i < E; ++i) m[j][i] *= inv;
+      y[idx] = f32_to_vec<T>(m[j]);
+    }
+  }
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+// vectors per thread for a row of n elements, or 0 when the register path does not apply
+template <typename T>
+int reg_vpt(int n) {
+  constexpr int E = Vec<T>::N;
+  if (n % E != 0) return 0;
+  const int vecs = n / E;
+  const int vpt = (vecs + GLUE_THREADS - 1) / GLUE_THREADS;
+  if (vpt <= 2) return 2;
+  if (vpt <= 4) return 4;
+  if (vpt <= 8) return 8;
+  if (vpt <= 12) return 12;
+  return 0;
+}
+
+template <typename T>
+int rms_dispatch(Ctx* ctx, const T* X, T* Y, int64_t rows, int n, float eps) {
+  const int vpt = (aligned16(X) && aligned16(Y)) ? reg_vpt<T>(n) : 0;
+  switch (vpt) {
+    case 2: rms_norm_reg_kernel<T, 2><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(X, Y, n, eps); break;
+    case 4: rms_norm_reg_kernel<T, 4><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(X, Y, n, eps); break;
+    case 8: rms_norm_reg_kernel<T, 8><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(X, Y, n, eps); break;
+    case 12: rms_norm_reg_kernel<T, 12><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(X, Y, n, eps); break;
+    default: rms_norm_kernel<T><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(X, Y, n, eps); break;
+  }
+  ++ctx->n_launch;
+  ZOACT_CHECK_LAUNCH();
+  return ZOACT_OK;
+}
+
+template <typename T>
+int mix_dispatch(Ctx* ctx, const T* q, const T* k, const T* v, T* Y, int64_t rows, int n, int n_rep, int head_dim,
+                 float eps) {
+  constexpr int E = Vec<T>::N;
+  const bool ok = aligned16(q) && aligned16(k) && aligned16(v) && aligned16(Y) && head_dim % E == 0 &&
+                  (n / n_rep) % E == 0;
+  const int vpt = ok ? reg_vpt<T>(n) : 0;
+  switch (vpt) {
+    case 2: mix_rms_reg_kernel<T, 2><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(q, k, v, Y, n, n_rep, head_dim, eps); break;
+    case 4: mix_rms_reg_kernel<T, 4><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(q, k, v, Y, n, n_rep, head_dim, eps); break;
+    case 8: mix_rms_reg_kernel<T, 8><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(q, k, v, Y, n, n_rep, head_dim, eps); break;
+    case 12: mix_rms_reg_kernel<T, 12><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(q, k, v, Y, n, n_rep, head_dim, eps); break;
+    default: mix_rms_kernel<T><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(q, k, v, Y, n, n_rep, head_dim, eps); break;
+  }
+  ++ctx->n_launch;
+  ZOACT_CHECK_LAUNCH();
+  return ZOACT_OK;
+}
+
 }  // namespace
 
 int launch_rms_norm(Ctx* ctx, const void* X, int dtype, int64_t rows, int n, float eps, void* Y) {
   if (rows <= 0) return ZOACT_OK;
   switch (dtype) {
     case ZOACT_DT_FP32:
-      rms_norm_kernel<float><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(
-          static_cast<const float*>(X), static_cast<float*>(Y), n, eps); ++ctx->n_launch;
-      break;
+      return rms_dispatch(ctx, static_cast<const float*>(X), static_cast<float*>(Y), rows, n, eps);
     case ZOACT_DT_BF16:
-      rms_norm_kernel<__nv_bfloat16><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(
-          static_cast<const __nv_bfloat16*>(X), static_cast<__nv_bfloat16*>(Y), n, eps); ++ctx->n_launch;
-      break;
+      return rms_dispatch(ctx, static_cast<const __nv_bfloat16*>(X), static_cast<__nv_bfloat16*>(Y), rows, n, eps);
     case ZOACT_DT_FP16:
-      rms_norm_kernel<__half><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(
-          static_cast<const __half*>(X), static_cast<__half*>(Y), n, eps); ++ctx->n_launch;
-      break;
+      return rms_dispatch(ctx, static_cast<const __half*>(X), static_cast<__half*>(Y), rows, n, eps);
     default:
       return ZOACT_ERR_INVALID_ARG;
   }
-  ZOACT_CHECK_LAUNCH();
-  return ZOACT_OK;
 }
 
 int launch_mix_rms(Ctx* ctx, const void* q, const void* k, const void* v, int dtype, int64_t rows, int n, int n_rep,
@@ -91,25 +233,18 @@ int launch_mix_rms(Ctx* ctx, const void* q, const void* k, const void* v, int dt
   if (rows <= 0) return ZOACT_OK;
   switch (dtype) {
     case ZOACT_DT_FP32:
-      mix_rms_kernel<float><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(
-          static_cast<const float*>(q), static_cast<const float*>(k), static_cast<const float*>(v),
-          static_cast<float*>(Y), n, n_rep, head_dim, eps); ++ctx->n_launch;
-      break;
+      return mix_dispatch(ctx, static_cast<const float*>(q), static_cast<const float*>(k),
+                          static_cast<const float*>(v), static_cast<float*>(Y), rows, n, n_rep, head_dim, eps);
     case ZOACT_DT_BF16:
-      mix_rms_kernel<__nv_bfloat16><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(
-          static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k),
-          static_cast<const __nv_bfloat16*>(v), static_cast<__nv_bfloat16*>(Y), n, n_rep, head_dim, eps); ++ctx->n_launch;
-      break;
+      return mix_dispatch(ctx, static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k),
+                          static_cast<const __nv_bfloat16*>(v), static_cast<__nv_bfloat16*>(Y), rows, n, n_rep,
+                          head_dim, eps);
     case ZOACT_DT_FP16:
-      mix_rms_kernel<__half><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(
-          static_cast<const __half*>(q), static_cast<const __half*>(k), static_cast<const __half*>(v),
-          static_cast<__half*>(Y), n, n_rep, head_dim, eps); ++ctx->n_launch;
-      break;
+      return mix_dispatch(ctx, static_cast<const __half*>(q), static_cast<const __half*>(k),
+                          static_cast<const __half*>(v), static_cast<__half*>(Y), rows, n, n_rep, head_dim, eps);
     default:
       return ZOACT_ERR_INVALID_ARG;
   }
-  ZOACT_CHECK_LAUNCH();
-  return ZOACT_OK;
 }
 
 }  // namespace zoact

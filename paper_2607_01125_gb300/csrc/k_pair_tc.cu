@@ -54,6 +54,27 @@ int encode_tmap_2d_16bit(CUtensorMap* map, const void* base, int dtype, int64_t 
 
 int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   using namespace pairtc;
+  if (a.wtype == ZOACT_DT_INT4_G128 && a.rows >= INT4_STAGED_MIN_ROWS) {
+    // staged INT4: expand W (and W2) to bf16 in context scratch, then the bf16 kernel
+    const size_t bytes = (size_t)a.d_out * a.d_in * 2;
+    void* wb = scratch(ctx, SLOT_WDQ0, bytes);
+    if (!wb) return ZOACT_ERR_NOMEM;
+    int st = launch_dequant_int4(ctx, a.W, a.w_scales, wb, a.d_out, a.d_in);
+    if (st) return st;
+    PairArgs b = a;
+    b.W = wb;
+    b.w_scales = nullptr;
+    b.wtype = ZOACT_DT_BF16;
+    if (a.W2) {
+      void* wb2 = scratch(ctx, SLOT_WDQ1, bytes);
+      if (!wb2) return ZOACT_ERR_NOMEM;
+      st = launch_dequant_int4(ctx, a.W2, a.w_scales2, wb2, a.d_out, a.d_in);
+      if (st) return st;
+      b.W2 = wb2;
+      b.w_scales2 = nullptr;
+    }
+    return launch_pair_tc(ctx, b);
+  }
   if (a.xdtype != ZOACT_DT_BF16 && a.xdtype != ZOACT_DT_FP16) return ZOACT_ERR_UNSUPPORTED;
   const bool w4 = a.wtype == ZOACT_DT_INT4_G128;
   if (w4 ? a.xdtype != ZOACT_DT_BF16 : a.wtype != a.xdtype) return ZOACT_ERR_UNSUPPORTED;

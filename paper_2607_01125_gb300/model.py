@@ -2,12 +2,14 @@
 
 One ZO step (Algorithm 2 with one two-sided query) is
 
-    for every adapted linear, in graph order:  zoact_pair_forward (+ glue ops)
+    for every adapted linear, in graph order:  zoact_lowrank_proj + zoact_pair_forward (+ glue)
     zoact_loss_pair   -> L+, L-, D, a  (device memory)
     zoact_adam_step   -> C, m, v updated with g = a * Z over all layers
 
 with no host synchronisation.  This module only allocates buffers and issues
-the calls; every arithmetic step runs in libzoact's kernels.
+the calls; every arithmetic step runs in libzoact's kernels.  Layers that read
+the same input with the same basis (q/k/v, gate/up after a calibration pass)
+share one projection P = X U.
 
 Graph wiring (names follow synth.Workload):
   toy        h = GELU(l1 x) (shared input, GELU fused in the epilogue); y = l2 h
@@ -18,6 +20,11 @@ Graph wiring (names follow synth.Workload):
                llama: h' = down rms(silu(gate b) * up b)
                opt:   h' = fc2 rms(relu(fc1 b))
              the first layer's q, k, v see the same input for both signs.
+
+Hooks: `capture(name, X)` is called with each linear's input (the + half)
+before its pair forward -- Algorithm 1's calibration pass uses it to take the
+bases; `timer`, when a list, receives (start event, end event, flops) around
+every tensor-core pair-forward launch.
 """
 import torch
 
@@ -71,32 +78,89 @@ class ZOStep:
         self.blocks = [(l.offset, l.d_out, l.r, l.layer_id) for l in linears]
         self.loss_out = torch.zeros(4, dtype=torch.float64, device=dev)
         self._bufs = {}
+        self._pcache = {}
         self.device = dev
+        self.capture = None
+        self.timer = None
 
     # ---- buffers ----
-    def buf(self, key, rows, cols):
+    def buf(self, key, rows, cols, dtype=None):
+        dtype = self.dtype if dtype is None else dtype
         t = self._bufs.get(key)
-        if t is None or t.shape != (rows, cols):
-            t = torch.empty(rows, cols, dtype=self.dtype, device=self.device)
+        if t is None or t.shape != (rows, cols) or t.dtype != dtype:
+            t = torch.empty(rows, cols, dtype=dtype, device=self.device)
             self._bufs[key] = t
         return t
 
+    def _wrote(self, t):
+        """A buffer was rewritten: projections of it are stale."""
+        for slot in [s for s, (key, _) in self._pcache.items() if key[0] == t.data_ptr()]:
+            del self._pcache[slot]
+
+    def _proj(self, lin, X, slot):
+        key = (X.data_ptr(), X.shape[0], lin.U.data_ptr())
+        hit = self._pcache.get(slot)
+        if hit is not None and hit[0] == key:
+            return hit[1]
+        for s, (k, P) in self._pcache.items():      # same input and basis already projected
+            if k == key:
+                self._pcache[slot] = (key, P)
+                return P
+        P = self.buf(f"P{slot}", X.shape[0], lin.r, torch.float32)
+        Z.zoact_lowrank_proj(self.ctx, X, lin.U, P)
+        self._pcache[slot] = (key, P)
+        return P
+
+    def _timed(self, fn, flops):
+        if self.timer is None:
+            fn()
+            return
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        fn()
+        e1.record()
+        self.timer.append((e0, e1, flops))
+
     def pair(self, name, X, shared, seed, query, out_key, act=Z.ACT_NONE):
         l = self.by_name[name]
+        if self.capture is not None:
+            self.capture(name, X[:self.T])
+        P = self._proj(l, X, 0)
         Y = self.buf(out_key, 2 * self.T, l.d_out)
-        Z.zoact_pair_forward(self.ctx, l.layer, X, self.T, shared, self.eps, seed, query, Y, act=act)
+        flops = 2.0 * X.shape[0] * l.d_in * l.d_out
+        self._timed(lambda: Z.zoact_pair_forward(self.ctx, l.layer, X, self.T, shared, self.eps, seed, query, Y,
+                                                 P=P, act=act), flops)
+        self._wrote(Y)
+        return Y
+
+    def gated(self, gname, uname, X, shared, seed, query, out_key):
+        g, u = self.by_name[gname], self.by_name[uname]
+        if self.capture is not None:
+            self.capture(gname, X[:self.T])
+            self.capture(uname, X[:self.T])
+        Pg = self._proj(g, X, 0)
+        Pu = self._proj(u, X, 1)
+        H = self.buf(out_key, 2 * self.T, g.d_out)
+        flops = 2.0 * X.shape[0] * g.d_in * g.d_out * 2
+        self._timed(lambda: Z.zoact_pair_forward_gated(self.ctx, g.layer, u.layer, X, self.T, shared, self.eps, seed,
+                                                       query, H, P_gate=Pg, P_up=Pu), flops)
+        self._wrote(H)
+        return H
+
+    def _glue_rms(self, X, key):
+        Y = self.buf(key, X.shape[0], X.shape[1])
+        Z.zoact_rms_norm(self.ctx, X, Y)
+        self._wrote(Y)
         return Y
 
     # ---- forward graphs ----
     def forward(self, x, seed, query):
-        T = self.T
+        self._pcache = {}
         if self.kind == "toy":
             h = self.pair("l1", x, True, seed, query, "h", act=Z.ACT_GELU)
             return self.pair("l2", h, False, seed, query, "y")
         if self.kind == "llama_mlp":
-            g, u = self.by_name["gate"], self.by_name["up"]
-            H = self.buf("h", 2 * T, g.d_out)
-            Z.zoact_pair_forward_gated(self.ctx, g.layer, u.layer, x, T, True, self.eps, seed, query, H)
+            H = self.gated("gate", "up", x, True, seed, query, "h")
             return self.pair("down", H, False, seed, query, "y")
         return self._stack(x, seed, query)
 
@@ -107,28 +171,23 @@ class ZOStep:
         shared = True
         for L in range(n_dec):
             rows = T if shared else 2 * T
-            a = self.buf(f"a{rows}", rows, h.shape[1])
-            Z.zoact_rms_norm(self.ctx, h, a)
+            a = self._glue_rms(h, f"a{rows}")
             q = self.pair(f"{L}.q", a, shared, seed, query, "q")
             k = self.pair(f"{L}.k", a, shared, seed, query, "k")
             v = self.pair(f"{L}.v", a, shared, seed, query, "v")
             shared = False
             mix = self.buf("mix", 2 * T, q.shape[1])
             Z.zoact_mix_rms(self.ctx, q, k, v, mix, self.n_rep if self.kind == "llama" else 1, self.head_dim)
+            self._wrote(mix)
             o = self.pair(f"{L}.o", mix, False, seed, query, "o")
-            b = self.buf("b", 2 * T, o.shape[1])
-            Z.zoact_rms_norm(self.ctx, o, b)
+            b = self._glue_rms(o, "b")
             if self.kind == "llama":
-                g, u = self.by_name[f"{L}.gate"], self.by_name[f"{L}.up"]
-                H = self.buf("hmlp", 2 * T, g.d_out)
-                Z.zoact_pair_forward_gated(self.ctx, g.layer, u.layer, b, T, False, self.eps, seed, query, H)
-                Hn = self.buf("hmlp_n", 2 * T, g.d_out)
-                Z.zoact_rms_norm(self.ctx, H, Hn)
+                H = self.gated(f"{L}.gate", f"{L}.up", b, False, seed, query, "hmlp")
+                Hn = self._glue_rms(H, "hmlp_n")
                 h = self.pair(f"{L}.down", Hn, False, seed, query, "h" if L % 2 == 0 else "h2")
             else:
                 f = self.pair(f"{L}.fc1", b, False, seed, query, "f", act=Z.ACT_RELU)
-                fn = self.buf("f_n", 2 * T, f.shape[1])
-                Z.zoact_rms_norm(self.ctx, f, fn)
+                fn = self._glue_rms(f, "f_n")
                 h = self.pair(f"{L}.fc2", fn, False, seed, query, "h" if L % 2 == 0 else "h2")
         return h
 
@@ -156,3 +215,32 @@ def coefficient_offsets(specs, r):
         offs.append(cur)
         cur += (s.d_out * r + 3) // 4 * 4
     return offs
+
+
+def calibrate_bases(ctx, step_cal, x_cal, r, oversample=16, n_iter=8, seed=0):
+    """Algorithm 1: one calibration forward pass of the base model (C = 0, eps = 0) on x_cal,
+    and each layer's basis U = top-r right singular vectors of its input, written in place.
+
+    step_cal is a ZOStep over the same AdaptedLinear objects with T = len(x_cal); layers whose
+    inputs are the same tensor (q/k/v, gate/up) share one basis computation.
+    """
+    last = {}
+
+    def cap(name, X):
+        # consecutive layers on the same input tensor (q/k/v, gate/up) share the basis
+        lin = step_cal.by_name[name]
+        key = (X.data_ptr(), X.shape[0])
+        if last.get("key") == key:
+            lin.U.copy_(last["U"])
+            return
+        Z.zoact_basis_init(ctx, X.contiguous(), r, lin.U, oversample=oversample, n_iter=n_iter,
+                           seed=seed + lin.layer_id)
+        last["key"], last["U"] = key, lin.U
+
+    step_cal.capture = cap
+    step_cal.C.zero_()
+    eps = step_cal.eps
+    step_cal.eps = 0.0
+    step_cal.forward(x_cal, 0, 0)
+    step_cal.eps = eps
+    step_cal.capture = None

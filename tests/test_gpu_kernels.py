@@ -195,8 +195,22 @@ def test_pair_forward_int4(ctx, d_in, d_out, r, T, shared):
     assert err.max() <= 2e-2 * np.abs(ref).max()
 
 
+@pytest.mark.parametrize("d_in,d_out,r,T,shared", [(1024, 520, 16, 600, False), (4096, 768, 8, 1100, True)])
+def test_pair_forward_int4_staged(ctx, d_in, d_out, r, T, shared):
+    # >= 1024 token rows: W is first expanded to bf16 (fp32 product q * s, one rounding), then the bf16 kernel
+    test_pair_forward_int4(ctx, d_in, d_out, r, T, shared)
+
+
 def test_pair_forward_gated_int4(ctx):
-    d_in, d_out, r, T = 1024, 384, 16, 96
+    _gated_int4(ctx, 96)
+
+
+def test_pair_forward_gated_int4_staged(ctx):
+    _gated_int4(ctx, 1024)
+
+
+def _gated_int4(ctx, T):
+    d_in, d_out, r = 1024, 384, 16
     eps, seed, query = 0.25, 3, 5
     Lg, Wg, Ug, Cg = _int4_layer(d_in, d_out, r, 50, 0)
     Lu, Wu, Uu, Cu = _int4_layer(d_in, d_out, r, 60, 1)
@@ -278,6 +292,19 @@ def test_sgd_and_nonfinite_guard(ctx):
 
 
 # ---------------- glue ----------------
+@pytest.mark.parametrize("n,dt", [(4096, torch.bfloat16), (5120, torch.float16), (14336, torch.bfloat16),
+                                  (20480, torch.float16), (100, torch.bfloat16), (256, torch.float32)])
+def test_rms_norm_widths(ctx, n, dt):
+    rows = 19
+    X = normal((rows, n), 65, DEV, dtype=dt)
+    Y = torch.empty_like(X)
+    zo.zoact_rms_norm(ctx, X, Y)
+    torch.cuda.synchronize()
+    ref = layers.rms_norm(np64(X))
+    rel = {torch.bfloat16: 2.0 ** -8, torch.float16: 2.0 ** -11, torch.float32: 2.0 ** -22}[dt]
+    assert np.all(np.abs(np64(Y) - ref) <= rel * np.abs(ref) + 1e-5)
+
+
 def test_rms_norm_and_mix(ctx):
     rows, n = 37, 4096
     X = normal((rows, n), 61, DEV, dtype=torch.bfloat16)
