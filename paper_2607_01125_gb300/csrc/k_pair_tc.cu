@@ -1,5 +1,7 @@
 // Host side of the tensor-core pair forward: tensor-map encoding, argument
 // checks and dispatch to the per-dtype instantiations of pair_tc_kernel.
+#include <cstdlib>
+#include <cstring>
 #include <mutex>
 
 #include "pair_tc_kernel.cuh"
@@ -12,6 +14,10 @@ int dispatch_bf16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, 
 int dispatch_fp16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const CUtensorMap& b,
                   const CUtensorMap& b2, const Params& p);
 int dispatch_w4(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const Params& p);
+int dispatch2_bf16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const CUtensorMap& b,
+                   const CUtensorMap& b2, const Params& p);
+int dispatch2_fp16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const CUtensorMap& b,
+                   const CUtensorMap& b2, const Params& p);
 }  // namespace pairtc
 
 namespace {
@@ -34,6 +40,27 @@ EncodeTiledFn get_encode_fn() {
 }
 
 int rank_template(int r) { return r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32; }
+
+// N-tile width for a rows x n output on sm_count persistent CTAs: the width whose
+// tiles fill the last wave best (useful outputs / (waves * SMs * tile size)); ties
+// go to the wider tile, which reuses each A tile for more columns.  Widths below
+// 192 measured slower per FLOP than the wave model predicts, so they are not tried.
+int choose_bn(int64_t rows, int64_t n, int sm_count, int bm = pairtc::BM) {
+  static const int cand[] = {256, 224, 192};
+  const int64_t num_m = (rows + bm - 1) / bm;
+  int best = 256;
+  double best_eff = -1.0;
+  for (int bn : cand) {
+    const int64_t tiles = num_m * ((n + bn - 1) / bn);
+    const int64_t waves = (tiles + sm_count - 1) / sm_count;
+    const double eff = (double)rows * (double)n / ((double)waves * sm_count * bm * bn);
+    if (eff > best_eff * 1.01) {
+      best_eff = eff;
+      best = bn;
+    }
+  }
+  return best;
+}
 
 }  // namespace
 
@@ -88,8 +115,15 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   if (st) return st;
   if (w4) {
     mb = mb2 = ma;                       // W arrives through the dequantising warps, not TMA
-  } else {
-    st = encode_tmap_2d_16bit(&mb, a.W, a.wtype, a.d_out, a.d_in, gated ? BN / 2 : BN);
+  }
+  // CTA pairs (256-row tiles) once there are enough rows to fill them; INT4 in-kernel dequant stays on one CTA
+  const char* sel = std::getenv("ZOACT_PAIR_KERNEL");
+  const bool two = !w4 && a.rows >= 2 * BM && !(sel && std::strcmp(sel, "1cta") == 0);
+  const int bn = (gated || w4) ? BN
+                               : (two ? choose_bn(a.rows, a.d_out, ctx->sm_count / 2, 2 * BM)
+                                      : choose_bn(a.rows, a.d_out, ctx->sm_count));
+  if (!w4) {
+    st = encode_tmap_2d_16bit(&mb, a.W, a.wtype, a.d_out, a.d_in, gated ? BN / 2 : (two ? bn / 2 : bn));
     if (st) return st;
   }
   if (gated && !w4) {
@@ -104,8 +138,10 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   p.shared = a.shared; p.act = a.act; p.eps = a.eps; p.seed = a.seed; p.query = a.query;
   p.layer_id = a.layer_id; p.layer_id2 = a.layer_id2;
   p.num_m = (int)((a.rows + BM - 1) / BM);
-  p.num_n = gated ? (a.d_out + BN / 2 - 1) / (BN / 2) : (a.d_out + BN - 1) / BN;
+  p.bn = bn;
+  p.num_n = gated ? (a.d_out + BN / 2 - 1) / (BN / 2) : (a.d_out + bn - 1) / bn;
   p.num_k = (a.d_in + BK - 1) / BK;
+  if (two) p.num_m = (int)((a.rows + 2 * BM - 1) / (2 * BM));
   p.num_tiles = p.num_m * p.num_n;
   p.ldy = a.d_out;
   auto al16 = [](const void* q) { return q == nullptr || ((uintptr_t)q & 15u) == 0; };
@@ -119,6 +155,9 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     p.Ws2 = static_cast<const __half*>(a.w_scales2);
     return dispatch_w4(ctx, mode, rt, a.ydtype, ma, p);
   }
+  if (two)
+    return a.xdtype == ZOACT_DT_BF16 ? dispatch2_bf16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p)
+                                     : dispatch2_fp16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p);
   return a.xdtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p)
                                    : dispatch_fp16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p);
 }
@@ -127,15 +166,17 @@ int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int
   using namespace pairtc;
   if (M <= 0 || N <= 0) return ZOACT_OK;
   CUtensorMap ma, mb;
+  const int bn = choose_bn(M, N, ctx->sm_count);
   int st = encode_tmap_2d_16bit(&ma, A, dtype, M, K, BM);
   if (st) return st;
-  st = encode_tmap_2d_16bit(&mb, B, dtype, N, K, BN);
+  st = encode_tmap_2d_16bit(&mb, B, dtype, N, K, bn);
   if (st) return st;
   Params p{};
   p.Y = D;
   p.rows = M; p.T = M; p.d_in = K; p.d_out = N; p.r = 0;
+  p.bn = bn;
   p.num_m = (M + BM - 1) / BM;
-  p.num_n = (N + BN - 1) / BN;
+  p.num_n = (N + bn - 1) / bn;
   p.num_k = (K + BK - 1) / BK;
   p.num_tiles = p.num_m * p.num_n;
   p.ldy = N;

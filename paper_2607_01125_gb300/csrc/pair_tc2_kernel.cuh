@@ -1,0 +1,261 @@
+// Pair forward on CTA pairs (tcgen05 cta_group::2): the same computation as
+// pair_tc_kernel (Section 3, the perturbed forward pass stacked over both
+// signs), with 256-row tiles split across the two SMs of a cluster.
+//
+// Each CTA loads its 128 rows of X and half of the tile's W rows (bn / 2) into
+// its own shared memory; the leader CTA issues tcgen05.mma.cta_group::2
+// 256 x bn x 16, which reads the operands of both CTAs and accumulates rows
+// 0..127 in the leader's TMEM and rows 128..255 in the peer's.  Per SM this
+// moves half the W bytes of the one-CTA kernel for the same FLOPs, so the ring
+// holds 6 stages of 32 KB.  Barriers: each producer arrives (with its byte
+// count) on the leader's stage barrier and its TMA completes there; the
+// leader's commits are multicast to both CTAs' stage-free and
+// accumulator-ready barriers; each CTA's epilogue signals the leader's
+// accumulator-free barrier once all of its threads have read the tile.
+// Gated mode: the leader's half of B is W_gate, the peer's W_up, so the
+// accumulator columns are [gate | up] as in the one-CTA kernel.
+#pragma once
+#include "pair_tc_kernel.cuh"
+
+namespace zoact {
+namespace pairtc {
+
+constexpr int STAGES2 = 6;
+constexpr int B_HALF_BYTES = (BN / 2) * BK * 2;
+constexpr int STAGE2_BYTES = A_BYTES + B_HALF_BYTES;
+constexpr int SMEM2_BYTES = 1024 + STAGES2 * STAGE2_BYTES + 2 * TABLE_FLOATS * 4 + 256;
+constexpr int BM2 = 2 * BM;
+
+struct SharedState2 {
+  uint64_t full[STAGES2];
+  uint64_t empty[STAGES2];
+  uint64_t tmem_full[2];
+  uint64_t tmem_empty[2];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort_flag;
+  int epi_ok;
+};
+
+namespace tc2 {
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_to(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+// Arrivals on a barrier of (possibly) the other CTA, with the default (CTA-scope
+// release) semantics: a cluster-scope release here would order the arrival
+// after this thread's outstanding bulk copies and serialise the copy ring.
+__device__ __forceinline__ void arrive_expect_tx_cluster(uint32_t bar_cluster, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cluster.b64 _, [%0], %1;" ::"r"(bar_cluster), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void arrive_cluster(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+// TMA tile load into this CTA's shared memory whose completion is signalled on
+// a barrier of the leader CTA of the pair.
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int32_t x, int32_t y,
+                                                 uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
+      "[%4];" ::"r"(dst),
+      "l"(map), "r"(x), "r"(y), "r"(bar_cluster)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_alloc2(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish2() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc2(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void mma2_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on the barrier at this offset in both CTAs of the pair once the
+// issuing thread's MMAs have completed.
+__device__ __forceinline__ void commit2_both(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+      "h"((uint16_t)3)
+      : "memory");
+}
+__device__ __forceinline__ void commit2_own(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+}  // namespace tc2
+
+template <typename TO, int RT, int MODE, int AB_BF16>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(num_threads(false), 1)
+pair_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                const __grid_constant__ CUtensorMap tmB2, const Params prm) {
+  constexpr int CW = 16;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  float* Ct = reinterpret_cast<float*>(smem + STAGES2 * STAGE2_BYTES);
+  float* Zt = Ct + TABLE_FLOATS;
+  SharedState2* ss = reinterpret_cast<SharedState2*>(Zt + TABLE_FLOATS);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = tc2::cluster_rank();
+  const bool leader = rank == 0;
+  volatile int* abort_flag = &ss->abort_flag;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES2; ++s) {
+      tc::mbar_init(tc::smem_u32(&ss->full[s]), 2);     // one producer arrival from each CTA (leader's copy is used)
+      tc::mbar_init(tc::smem_u32(&ss->empty[s]), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      tc::mbar_init(tc::smem_u32(&ss->tmem_full[b]), 1);
+      tc::mbar_init(tc::smem_u32(&ss->tmem_empty[b]), 2);   // one arrival per CTA (leader's copy is used)
+    }
+    tc::mbar_init(tc::smem_u32(&ss->drain), 1);
+    ss->abort_flag = 0;
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&tmA);
+    tc::prefetch_tmap(&tmB);
+    if (MODE == MODE_GATED) tc::prefetch_tmap(&tmB2);
+  }
+  if (warp == 1) {
+    tc2::tmem_alloc2(tc::smem_u32(&ss->tmem_base), TMEM_COLS);
+    tc2::tmem_relinquish2();
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  tc2::cluster_sync();                    // both CTAs' barriers exist before any remote arrival
+  tc::tc_fence_after();
+  const uint32_t tmem_base = ss->tmem_base;
+
+  const int num_m = prm.num_m, num_n = prm.num_n, num_k = prm.num_k;
+  const int bn = MODE == MODE_GATED ? BN : prm.bn;
+  const int bh = bn / 2;                  // W rows per CTA
+  const uint32_t stage_tx = A_BYTES + bh * BK * 2;
+  const int cluster_id = blockIdx.x >> 1, n_clusters = gridDim.x >> 1;
+
+  if (warp == 0) {
+    // ---------------- TMA producer (both CTAs) ----------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int tile = cluster_id; tile < prm.num_tiles && ok; tile += n_clusters) {
+        int m_blk, n_blk;
+        tile_coords(tile, num_m, num_n, m_blk, n_blk);
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
+          const uint32_t full_leader = tc2::map_to(tc::smem_u32(&ss->full[stage]), 0);
+          tc2::arrive_expect_tx_cluster(full_leader, stage_tx);
+          const uint32_t sa = tc::smem_u32(smem + stage * STAGE2_BYTES);
+          const uint32_t sb = sa + A_BYTES;
+          tc2::tma_load_2d_pair(sa, &tmA, kb * BK, m_blk * BM2 + (int)rank * BM, full_leader);
+          if (MODE == MODE_GATED)
+            tc2::tma_load_2d_pair(sb, leader ? &tmB : &tmB2, kb * BK, n_blk * (BN / 2), full_leader);
+          else
+            tc2::tma_load_2d_pair(sb, &tmB, kb * BK, n_blk * bn + (int)rank * bh, full_leader);
+          if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
+        }
+      }
+      if (!ok) {
+        // our copies complete on the leader's barriers; give them time to land before the CTA winds down
+        const uint64_t t0 = tc::global_timer_ns();
+        while (tc::global_timer_ns() - t0 < 2000000ull) {
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer (leader CTA) ----------------
+    if (lane == 0 && leader) {
+      const uint32_t idesc = tc::idesc_f16(BM2, bn, AB_BF16);
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      int local = 0;
+      bool issued_any = false;
+      for (int tile = cluster_id; tile < prm.num_tiles && ok; tile += n_clusters, ++local) {
+        const int buf = local & 1;
+        const uint32_t acc_phase = (local >> 1) & 1;
+        if (!tc::mbar_wait(tc::smem_u32(&ss->tmem_empty[buf]), acc_phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
+        tc::tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!tc::mbar_wait(tc::smem_u32(&ss->full[stage]), phase, abort_flag, prm.status)) { ok = false; break; }
+          tc::tc_fence_after();
+          const uint32_t sa = tc::smem_u32(smem + stage * STAGE2_BYTES);
+          const uint32_t sb = sa + A_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            tc2::mma2_f16(d_tmem, tc::sdesc_k_sw128(sa + k * 32), tc::sdesc_k_sw128(sb + k * 32), idesc,
+                          (kb | k) != 0 ? 1u : 0u);
+          tc2::commit2_both(tc::smem_u32(&ss->empty[stage]));    // frees the stage in both CTAs
+          issued_any = true;
+          if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        tc2::commit2_both(tc::smem_u32(&ss->tmem_full[buf]));   // accumulator ready in both CTAs
+      }
+      if (issued_any) {
+        tc2::commit2_own(tc::smem_u32(&ss->drain));
+        tc::mbar_wait_drain(tc::smem_u32(&ss->drain), 0, 100000000ull);
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..9, both CTAs) ----------------
+    const int etid = threadIdx.x - epi_base(false);
+    const int half = etid >> 7;
+    const int quad = warp & 3;
+    const int row_in_tile = quad * 32 + lane;
+    const uint32_t tmem_empty_leader0 = tc2::map_to(tc::smem_u32(&ss->tmem_empty[0]), 0);
+    const uint32_t tmem_empty_leader1 = tc2::map_to(tc::smem_u32(&ss->tmem_empty[1]), 0);
+    int local = 0;
+    for (int tile = cluster_id; tile < prm.num_tiles; tile += n_clusters, ++local) {
+      int m_blk, n_blk;
+      tile_coords(tile, num_m, num_n, m_blk, n_blk);
+      const int buf = local & 1;
+      const uint32_t acc_phase = (local >> 1) & 1;
+      const int64_t m = (int64_t)m_blk * BM2 + (int64_t)rank * BM + row_in_tile;
+      const bool row_ok = m < prm.rows;
+      const uint32_t t_row = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * BN);
+      const bool ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, Ct, Zt, etid, half, m, row_ok, n_blk, bn, buf,
+                                                      acc_phase, t_row, abort_flag);
+      if (!ok) break;
+      tc::tc_fence_before();
+      tc::named_bar_sync(3, EPI_THREADS);        // every epilogue thread of this CTA has read the tile
+      if (etid == 0) tc2::arrive_cluster(buf ? tmem_empty_leader1 : tmem_empty_leader0);
+    }
+  }
+
+  tc::tc_fence_before();
+  __syncthreads();
+  tc2::cluster_sync();                    // the peer's MMAs and copies are done before TMEM and smem go away
+  if (warp == 1) {
+    __syncwarp();
+    tc::tc_fence_after();
+    tc2::tmem_dealloc2(tmem_base, TMEM_COLS);
+  }
+}
+
+}  // namespace pairtc
+}  // namespace zoact

@@ -77,6 +77,7 @@ struct Params {
   int num_m, num_n, num_k, num_tiles;
   int64_t ldy;       // plain mode: row stride of D
   int vec_ok;        // C, C2, P, P2 and ldy allow 16-byte vector access
+  int bn;            // N-tile width of pair / plain tiles (multiple of 32, <= BN); gated tiles use BN
   // INT4 weights: packed [d_out, d_in/2] bytes and fp16 scales [d_out, d_in/128]
   const uint8_t* Wq;
   const __half* Ws;
@@ -281,7 +282,8 @@ __device__ __forceinline__ void dq_store(uint8_t* btile, int row, const DqRow& d
 // The epilogue's wait for a finished accumulator, taken by one thread and
 // shared through a named barrier so that all epilogue threads leave (or
 // continue) together even if the wait gives up.
-__device__ __forceinline__ bool epi_wait_full(SharedState* ss, int buf, uint32_t parity, volatile int* abort_flag,
+template <typename SS>
+__device__ __forceinline__ bool epi_wait_full(SS* ss, int buf, uint32_t parity, volatile int* abort_flag,
                                               int* status, int etid) {
   if (etid == 0) ss->epi_ok = tc::mbar_wait(tc::smem_u32(&ss->tmem_full[buf]), parity, abort_flag, status) ? 1 : 0;
   tc::named_bar_sync(2, EPI_THREADS);
@@ -305,6 +307,106 @@ __device__ __forceinline__ void load_p(float* p, const float* __restrict__ P, in
 #pragma unroll
     for (int j = 0; j < RT; ++j) p[j] = (row_ok && j < r) ? P[m * r + j] : 0.f;
   }
+}
+
+// Pair / gated epilogue of one accumulator tile for this CTA's 128 rows (row m
+// of thread (quad, lane)): builds the tile's C and Z tables, waits for the
+// accumulator, adds the low-rank term, applies the activation or the SiLU gate
+// and stores.  Returns false when the wait gave up.
+template <typename TO, int RT, int MODE, int CW, typename SS>
+__device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* Ct, float* Zt, int etid,
+                                              int half, int64_t m, bool row_ok, int n_blk, int bn, int buf,
+                                              uint32_t acc_phase, uint32_t t_row, volatile int* abort_flag) {
+  const int r = prm.r;
+  // ---- pair / gated epilogue ----
+  // table chunks: slots per chunk such that slots * RT <= TABLE_FLOATS
+  constexpr int CHUNK = (TABLE_FLOATS / RT) < BN ? (TABLE_FLOATS / RT) : BN;
+  static_assert(MODE != MODE_GATED || CHUNK == BN, "gated mode keeps the whole tile's table");
+  float p[RT], p2[RT];
+  const bool vec = prm.vec_ok != 0;
+  load_p<RT>(p, prm.P, m, r, row_ok, vec);
+  if (MODE == MODE_GATED) load_p<RT>(p2, prm.P2, m, r, row_ok, vec);
+  const float sgn_eps = m < prm.T ? prm.eps : -prm.eps;   // stacked rows: sign of the half
+  TO* Y = static_cast<TO*>(prm.Y);
+  bool ok = true;
+  for (int s0 = 0; s0 < bn && ok; s0 += CHUNK) {
+    const int cwid = min(CHUNK, bn - s0);        // slots in this chunk (a multiple of 32)
+    tc::named_bar_sync(1, EPI_THREADS);          // previous chunk's readers are done
+    if (MODE == MODE_GATED) {
+      build_table<RT>(Ct, Zt, prm.C, prm.layer_id, n_blk * (BN / 2), BN / 2, 0, prm.d_out, r, prm.seed,
+                      prm.query, etid, vec);
+      build_table<RT>(Ct, Zt, prm.C2, prm.layer_id2, n_blk * (BN / 2), BN / 2, BN / 2, prm.d_out, r,
+                      prm.seed, prm.query, etid, vec);
+    } else {
+      build_table<RT>(Ct, Zt, prm.C, prm.layer_id, n_blk * bn + s0, cwid, 0, prm.d_out, r, prm.seed,
+                      prm.query, etid, vec);
+    }
+    tc::named_bar_sync(1, EPI_THREADS);
+    if (s0 == 0) {
+      if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) { ok = false; break; }
+    }
+    if (MODE == MODE_GATED) {
+      for (int c0 = half * (BN / 4); c0 < (half + 1) * (BN / 4); c0 += CW) {
+        float g[CW], u[CW];
+        tmem_ldN<CW>(t_row + (uint32_t)c0, g);
+        tmem_ldN<CW>(t_row + (uint32_t)(BN / 2 + c0), u);
+        const int n = n_blk * (BN / 2) + c0;
+        if (!row_ok || n >= prm.d_out) continue;
+        const int nv = min(CW, prm.d_out - n);
+        float gC[CW], gZ[CW];
+        lowrankN<RT, CW>(Ct, Zt, c0, p, gC, gZ);
+#pragma unroll
+        for (int i = 0; i < CW; ++i) g[i] += gC[i];      // g = W_g x + C_g p
+        float uC[CW], uZ[CW];
+        lowrankN<RT, CW>(Ct, Zt, BN / 2 + c0, p2, uC, uZ);
+#pragma unroll
+        for (int i = 0; i < CW; ++i) u[i] += uC[i];
+        if (prm.shared) {
+          float hp[CW], hm[CW];
+#pragma unroll
+          for (int i = 0; i < CW; ++i) {
+            hp[i] = silu_fast(fmaf(prm.eps, gZ[i], g[i])) * fmaf(prm.eps, uZ[i], u[i]);
+            hm[i] = silu_fast(fmaf(-prm.eps, gZ[i], g[i])) * fmaf(-prm.eps, uZ[i], u[i]);
+          }
+          storeN<TO, CW>(Y + m * prm.d_out + n, hp, nv);
+          storeN<TO, CW>(Y + (prm.T + m) * prm.d_out + n, hm, nv);
+        } else {
+          float h[CW];
+#pragma unroll
+          for (int i = 0; i < CW; ++i) h[i] = silu_fast(fmaf(sgn_eps, gZ[i], g[i])) * fmaf(sgn_eps, uZ[i], u[i]);
+          storeN<TO, CW>(Y + m * prm.d_out + n, h, nv);
+        }
+      }
+    } else {
+      const int cbeg = s0 + half * (cwid / 2);
+      for (int c0 = cbeg; c0 < cbeg + cwid / 2; c0 += CW) {
+        float acc[CW];
+        tmem_ldN<CW>(t_row + (uint32_t)c0, acc);
+        const int n = n_blk * bn + c0;
+        if (!row_ok || n >= prm.d_out) continue;
+        const int nv = min(CW, prm.d_out - n);
+        float sC[CW], sZ[CW];
+        lowrankN<RT, CW>(Ct, Zt, c0 - s0, p, sC, sZ);
+        if (prm.shared) {
+          float yp[CW], ym[CW];
+#pragma unroll
+          for (int i = 0; i < CW; ++i) {
+            const float base = acc[i] + sC[i];
+            yp[i] = apply_act(fmaf(prm.eps, sZ[i], base), prm.act);
+            ym[i] = apply_act(fmaf(-prm.eps, sZ[i], base), prm.act);
+          }
+          storeN<TO, CW>(Y + m * prm.d_out + n, yp, nv);
+          storeN<TO, CW>(Y + (prm.T + m) * prm.d_out + n, ym, nv);
+        } else {
+          float y[CW];
+#pragma unroll
+          for (int i = 0; i < CW; ++i) y[i] = apply_act(fmaf(sgn_eps, sZ[i], acc[i] + sC[i]), prm.act);
+          storeN<TO, CW>(Y + m * prm.d_out + n, y, nv);
+        }
+      }
+    }
+  }
+  return ok;
 }
 
 template <typename TO, int RT, int MODE, int AB_BF16, bool W4>
@@ -349,6 +451,7 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const uint32_t tmem_base = ss->tmem_base;
 
   const int num_m = prm.num_m, num_n = prm.num_n, num_k = prm.num_k;
+  const int bn = MODE == MODE_GATED ? BN : prm.bn;  // this launch's N-tile width
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
@@ -363,7 +466,7 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         for (int kb = 0; kb < num_k; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
           const uint32_t full = tc::smem_u32(&ss->full[stage]);
-          tc::mbar_arrive_expect_tx(full, W4 ? A_BYTES : STAGE_BYTES);
+          tc::mbar_arrive_expect_tx(full, W4 ? A_BYTES : (MODE == MODE_GATED ? STAGE_BYTES : A_BYTES + bn * BK * 2));
           const uint32_t sa = tc::smem_u32(smem + stage * STAGE_BYTES);
           const uint32_t sb = sa + A_BYTES;
           tc::tma_load_2d(sa, &tmA, kb * BK, m_blk * BM, full);
@@ -373,7 +476,7 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             tc::tma_load_2d(sb, &tmB, kb * BK, n_blk * (BN / 2), full);
             tc::tma_load_2d(sb + B_BYTES / 2, &tmB2, kb * BK, n_blk * (BN / 2), full);
           } else {
-            tc::tma_load_2d(sb, &tmB, kb * BK, n_blk * BN, full);
+            tc::tma_load_2d(sb, &tmB, kb * BK, n_blk * bn, full);
           }
           issued_mask |= 1u << stage;
           issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
@@ -390,7 +493,7 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   } else if (warp == 1) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
-      constexpr uint32_t IDESC = tc::idesc_f16(BM, BN, AB_BF16);
+      const uint32_t IDESC = tc::idesc_f16(BM, bn, AB_BF16);
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
@@ -484,10 +587,10 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       if (MODE == MODE_PLAIN) {
         if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) break;
         float* D = static_cast<float*>(prm.Y);
-        for (int c0 = half * (BN / 2); c0 < (half + 1) * (BN / 2); c0 += CW) {
+        for (int c0 = half * (bn / 2); c0 < (half + 1) * (bn / 2); c0 += CW) {
           float v[CW];
           tmem_ldN<CW>(t_row + (uint32_t)c0, v);
-          const int n = n_blk * BN + c0;
+          const int n = n_blk * bn + c0;
           if (row_ok && n < prm.d_out) {
             storeN<float, CW>(D + m * prm.ldy + n, v, min(CW, prm.d_out - n), prm.vec_ok != 0);
           }
@@ -497,93 +600,8 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         continue;
       }
 
-      // ---- pair / gated epilogue ----
-      // table chunks: slots per chunk such that slots * RT <= TABLE_FLOATS
-      constexpr int CHUNK = (TABLE_FLOATS / RT) < BN ? (TABLE_FLOATS / RT) : BN;
-      static_assert(MODE != MODE_GATED || CHUNK == BN, "gated mode keeps the whole tile's table");
-      float p[RT], p2[RT];
-      const bool vec = prm.vec_ok != 0;
-      load_p<RT>(p, prm.P, m, r, row_ok, vec);
-      if (MODE == MODE_GATED) load_p<RT>(p2, prm.P2, m, r, row_ok, vec);
-      const float sgn_eps = m < prm.T ? prm.eps : -prm.eps;   // stacked rows: sign of the half
-      TO* Y = static_cast<TO*>(prm.Y);
-      bool ok = true;
-      for (int s0 = 0; s0 < BN && ok; s0 += CHUNK) {
-        tc::named_bar_sync(1, EPI_THREADS);          // previous chunk's readers are done
-        if (MODE == MODE_GATED) {
-          build_table<RT>(Ct, Zt, prm.C, prm.layer_id, n_blk * (BN / 2), BN / 2, 0, prm.d_out, r, prm.seed,
-                          prm.query, etid, vec);
-          build_table<RT>(Ct, Zt, prm.C2, prm.layer_id2, n_blk * (BN / 2), BN / 2, BN / 2, prm.d_out, r,
-                          prm.seed, prm.query, etid, vec);
-        } else {
-          build_table<RT>(Ct, Zt, prm.C, prm.layer_id, n_blk * BN + s0, CHUNK, 0, prm.d_out, r, prm.seed,
-                          prm.query, etid, vec);
-        }
-        tc::named_bar_sync(1, EPI_THREADS);
-        if (s0 == 0) {
-          if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) { ok = false; break; }
-        }
-        if (MODE == MODE_GATED) {
-          for (int c0 = half * (BN / 4); c0 < (half + 1) * (BN / 4); c0 += CW) {
-            float g[CW], u[CW];
-            tmem_ldN<CW>(t_row + (uint32_t)c0, g);
-            tmem_ldN<CW>(t_row + (uint32_t)(BN / 2 + c0), u);
-            const int n = n_blk * (BN / 2) + c0;
-            if (!row_ok || n >= prm.d_out) continue;
-            const int nv = min(CW, prm.d_out - n);
-            float gC[CW], gZ[CW];
-            lowrankN<RT, CW>(Ct, Zt, c0, p, gC, gZ);
-#pragma unroll
-            for (int i = 0; i < CW; ++i) g[i] += gC[i];      // g = W_g x + C_g p
-            float uC[CW], uZ[CW];
-            lowrankN<RT, CW>(Ct, Zt, BN / 2 + c0, p2, uC, uZ);
-#pragma unroll
-            for (int i = 0; i < CW; ++i) u[i] += uC[i];
-            if (prm.shared) {
-              float hp[CW], hm[CW];
-#pragma unroll
-              for (int i = 0; i < CW; ++i) {
-                hp[i] = silu_fast(fmaf(prm.eps, gZ[i], g[i])) * fmaf(prm.eps, uZ[i], u[i]);
-                hm[i] = silu_fast(fmaf(-prm.eps, gZ[i], g[i])) * fmaf(-prm.eps, uZ[i], u[i]);
-              }
-              storeN<TO, CW>(Y + m * prm.d_out + n, hp, nv);
-              storeN<TO, CW>(Y + (prm.T + m) * prm.d_out + n, hm, nv);
-            } else {
-              float h[CW];
-#pragma unroll
-              for (int i = 0; i < CW; ++i) h[i] = silu_fast(fmaf(sgn_eps, gZ[i], g[i])) * fmaf(sgn_eps, uZ[i], u[i]);
-              storeN<TO, CW>(Y + m * prm.d_out + n, h, nv);
-            }
-          }
-        } else {
-          const int cbeg = s0 + half * (CHUNK / 2);
-          for (int c0 = cbeg; c0 < cbeg + CHUNK / 2; c0 += CW) {
-            float acc[CW];
-            tmem_ldN<CW>(t_row + (uint32_t)c0, acc);
-            const int n = n_blk * BN + c0;
-            if (!row_ok || n >= prm.d_out) continue;
-            const int nv = min(CW, prm.d_out - n);
-            float sC[CW], sZ[CW];
-            lowrankN<RT, CW>(Ct, Zt, c0 - s0, p, sC, sZ);
-            if (prm.shared) {
-              float yp[CW], ym[CW];
-#pragma unroll
-              for (int i = 0; i < CW; ++i) {
-                const float base = acc[i] + sC[i];
-                yp[i] = apply_act(fmaf(prm.eps, sZ[i], base), prm.act);
-                ym[i] = apply_act(fmaf(-prm.eps, sZ[i], base), prm.act);
-              }
-              storeN<TO, CW>(Y + m * prm.d_out + n, yp, nv);
-              storeN<TO, CW>(Y + (prm.T + m) * prm.d_out + n, ym, nv);
-            } else {
-              float y[CW];
-#pragma unroll
-              for (int i = 0; i < CW; ++i) y[i] = apply_act(fmaf(sgn_eps, sZ[i], acc[i] + sC[i]), prm.act);
-              storeN<TO, CW>(Y + m * prm.d_out + n, y, nv);
-            }
-          }
-        }
-      }
+      const bool ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, Ct, Zt, etid, half, m, row_ok, n_blk, bn, buf,
+                                                      acc_phase, t_row, abort_flag);
       if (!ok) break;
       tc::tc_fence_before();
       tc::mbar_arrive(tc::smem_u32(&ss->tmem_empty[buf]));

@@ -127,6 +127,52 @@ def test_pair_forward_16bit_out_and_acts(ctx, d_in, d_out, r, T, shared, dt, act
     assert err.max() <= 2e-2 * np.abs(ref).max()
 
 
+@pytest.mark.parametrize("which", ["down", "gated"])
+def test_pair_forward_full_size_sampled(ctx, which):
+    # the bench's launches at full size (Llama-3-8B MLP block, T = 2048, r = 16, bf16 out); the oracle
+    # computes 96 sampled token rows (from both halves) over every output column
+    T, r, eps, seed, query = 2048, 16, 1e-3, 77, 9
+    rng = np.random.default_rng(5)
+    if which == "down":
+        d_in, d_out = 14336, 4096
+        X, W, U, C = _pair_case(d_in, d_out, r, T, False, torch.bfloat16, eps, 0.05, seed=20)
+        Y = torch.empty(2 * T, d_out, dtype=torch.bfloat16, device=DEV)
+        zo.zoact_pair_forward(ctx, zo.make_layer(W, U, C, 2), X, T, False, eps, seed, query, Y)
+        torch.cuda.synchronize()
+        rows = np.sort(rng.choice(2 * T, 96, replace=False))
+        Xs, Wn, Un = np64(X)[rows], np64(W), np64(U)
+        Zm = philox.perturbation(seed, 2, query, d_out, r)
+        sig = np.where(rows < T, 1.0, -1.0)[:, None]
+        Cn = np64(C).reshape(d_out, r)
+        ref = Xs @ Wn.T + ((Xs @ Un) @ Cn.T) + sig * eps * ((Xs @ Un) @ Zm.T)
+        got = np64(Y)[rows]
+    else:
+        d_in, d_out = 4096, 14336
+        X = normal((T, d_in), 31, DEV, dtype=torch.bfloat16)
+        Wg = normal((d_out, d_in), 32, DEV, std=0.02, dtype=torch.bfloat16)
+        Wu = normal((d_out, d_in), 33, DEV, std=0.02, dtype=torch.bfloat16)
+        U = normal((d_in, r), 34, DEV) / np.sqrt(d_in)
+        Cg = normal((d_out * r,), 35, DEV, std=0.05)
+        Cu = normal((d_out * r,), 36, DEV, std=0.05)
+        H = torch.empty(2 * T, d_out, dtype=torch.bfloat16, device=DEV)
+        zo.zoact_pair_forward_gated(ctx, zo.make_layer(Wg, U, Cg, 0), zo.make_layer(Wu, U, Cu, 1), X, T, True,
+                                    eps, seed, query, H)
+        torch.cuda.synchronize()
+        tok = np.sort(rng.choice(T, 48, replace=False))
+        Xs, Un = np64(X)[tok], np64(U)
+        P = Xs @ Un
+        out = []
+        for sgn in (1.0, -1.0):
+            g = Xs @ np64(Wg).T + P @ (np64(Cg).reshape(d_out, r) + sgn * eps * philox.perturbation(seed, 0, query, d_out, r)).T
+            u = Xs @ np64(Wu).T + P @ (np64(Cu).reshape(d_out, r) + sgn * eps * philox.perturbation(seed, 1, query, d_out, r)).T
+            out.append(layers.silu(g) * u)
+        ref = np.concatenate(out)
+        got = np.concatenate([np64(H)[tok], np64(H)[T + tok]])
+    err = np.abs(got - ref)
+    assert err.max() <= 2e-2 * np.abs(ref).max()
+    assert np.all(err <= 2.0 ** -7 * np.abs(ref) + 2e-3 * np.abs(ref).max())
+
+
 def test_pair_difference_isolates_the_perturbation(ctx):
     # y+ - y- = 2 eps Z p exactly in the definition; fp32 output keeps it visible at eps = 1e-3
     d_in, d_out, r, T = 768, 512, 16, 64
@@ -142,7 +188,8 @@ def test_pair_difference_isolates_the_perturbation(ctx):
     assert np.abs((Yn[:T] - Yn[T:]) - ref).max() <= 1e-6 * np.abs(Yn).max()
 
 
-@pytest.mark.parametrize("T,shared,dt", [(96, True, torch.bfloat16), (70, False, torch.bfloat16)])
+@pytest.mark.parametrize("T,shared,dt", [(96, True, torch.bfloat16), (70, False, torch.bfloat16),
+                                         (300, True, torch.bfloat16), (200, False, torch.float16)])
 def test_pair_forward_gated(ctx, T, shared, dt):
     d_in, d_out, r = 512, 400, 16
     eps, seed, query = 0.25, 8, 4
