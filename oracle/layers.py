@@ -48,6 +48,38 @@ def pair_forward(W, U, C, Z, X, eps, T, input_shared):
     return np.concatenate([Y_plus, Y_minus], axis=0)
 
 
+def multi_forward(W, U, C, Zs, coefs, X, T, input_shared):
+    """Forward of one adapted linear at several coefficient points, stacked by blocks.
+
+    Algorithm 2 evaluates the loss at W_eff = W + V_r B (the unperturbed pass)
+    and at W + V_r (B + mu Z^(j)) for j = 1..q (Section 3).  Block b of the
+    stacked output is the layer evaluated at C + coefs[b] * Zs[b]:
+
+        Y_b = X_b W^T + (X_b U)(C + coefs[b] Z_b)^T
+
+    Zs[b] may be None where coefs[b] == 0 (no perturbation is drawn there).
+    X: [n_blocks * T, d_in] (block b in rows [bT, (b+1)T)), or [T, d_in] when
+    input_shared (every block sees the same x).  Returns Y [n_blocks * T, d_out].
+    The two-sided pair is the case coefs = (eps, -eps) with the same Z twice.
+    """
+    W = np.asarray(W, np.float64)
+    U = np.asarray(U, np.float64)
+    C = np.asarray(C, np.float64)
+    X = np.asarray(X, np.float64)
+    nb = len(coefs)
+    assert len(Zs) == nb
+    assert X.shape[0] == (T if input_shared else nb * T)
+    out = []
+    for b in range(nb):
+        Xb = X if input_shared else X[b * T:(b + 1) * T]
+        if coefs[b] == 0.0:
+            Cb = C
+        else:
+            Cb = C + coefs[b] * np.asarray(Zs[b], np.float64)
+        out.append(Xb @ W.T + (Xb @ U) @ Cb.T)
+    return np.concatenate(out, axis=0)
+
+
 def dequant_int4_g128(packed, scales, d_in):
     """Frozen INT4 weight -> fp64, group size 128 along d_in (test infrastructure only).
 

@@ -38,3 +38,13 @@ def sgd_step(C, g, lr):
 def zo_gradient(a, Z):
     """g_hat = a * Z (Section 3 estimator with one query)."""
     return float(a) * np.asarray(Z, np.float64)
+
+
+def zo_gradient_queries(a, Zs):
+    """g_hat = (1/q) sum_j a_j Z^(j)  (Algorithm 2, averaged over q queries)."""
+    q = len(a)
+    assert q == len(Zs) and q > 0
+    g = np.zeros_like(np.asarray(Zs[0], np.float64))
+    for aj, Zj in zip(a, Zs):
+        g = g + float(aj) * np.asarray(Zj, np.float64)
+    return g / q
