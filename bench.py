@@ -111,7 +111,7 @@ def dist_setup():
     return world, rank, local
 
 
-def build(ctx, dev, rank, name, tokens=None):
+def build(ctx, dev, rank, name, tokens=None, n_queries=None):
     """Weights, bases (Algorithm 1 on the device) and the ZOStep of a workload.
 
     Returns (step, x, target, basis_seconds, workload).  Weights are the same on every
@@ -150,7 +150,7 @@ def build(ctx, dev, rank, name, tokens=None):
     torch.cuda.synchronize()
     basis_s = time.time() - t0
     del step_cal
-    step = ZOStep(ctx, w.kind, lins, w.T, w.act_dtype, eps=w.eps, lr=LR)
+    step = ZOStep(ctx, w.kind, lins, w.T, w.act_dtype, eps=w.eps, lr=LR, n_queries=n_queries)
     return step, x, target, basis_s, w
 
 
@@ -159,7 +159,7 @@ def run_step(step, x, target, t, seed, world):
     step.loss(Y, target)
     if world > 1:
         from paper_2607_01125_gb300.dp import allreduce_loss
-        allreduce_loss(step.loss_out)            # L+, L-, D and a are means over equal token counts
+        allreduce_loss(step.loss_out)            # losses and a's are means over equal token counts
     step.update(t, seed, t)
     return step.loss_out
 
@@ -174,7 +174,7 @@ def run_ours(args):
     dev = f"cuda:{local}"
     torch.cuda.set_device(local)
     ctx = zo.Context(local)
-    step, x, target, basis_s, w = build(ctx, dev, rank, args.workload, args.tokens)
+    step, x, target, basis_s, w = build(ctx, dev, rank, args.workload, args.tokens, args.queries)
     seed = 1234
 
     def barrier():
@@ -213,7 +213,7 @@ def run_ours(args):
     # ---- end to end through the public API with host buffers ----
     x_h = x.cpu().pin_memory()
     t_h = target.cpu().pin_memory() if target is not None else None
-    out_h = torch.empty(4, dtype=torch.float64).pin_memory()
+    out_h = torch.empty(step.loss_out.numel(), dtype=torch.float64).pin_memory()
     x_d = torch.empty_like(x)
     t_d = torch.empty_like(target) if target is not None else None
     barrier(); torch.cuda.synchronize()
@@ -249,27 +249,28 @@ def run_ours(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int4-bf16" if w.wtype == "int4_g128" else w.act_dtype,
         "data": "synthetic",
-        "config": {"workload": w.name, "tokens_per_perturbation": T, "stacked_rows": 2 * T, "r": w.r, "eps": w.eps,
-                   "adapted_linears": len(w.linears()), "estimator": "two-sided, q=1",
+        "config": {"workload": w.name, "tokens_per_perturbation": T, "stacked_rows": step.nb * T, "r": w.r,
+                   "eps": w.eps, "adapted_linears": len(w.linears()),
+                   "estimator": "two-sided, q=1" if args.queries is None else f"one-sided, q={args.queries}",
                    "l2": "inputs larger than L2 (frozen weights streamed from HBM every step)",
                    "parallelism": f"dp{world}" if world > 1 else "single"},
-        "evaluated_tokens_per_s": world * 2 * T / (ms * 1e-3),
+        "evaluated_tokens_per_s": world * step.nb * T / (ms * 1e-3),
         "zo_steps_per_s": 1e3 / ms,
         "pair_forward_ms_per_step": gemm_ms / args.steps,
         "basis_init_s": basis_s,
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak,
                      "peak_kind": f"bf16 dense {'sustained' if long_step else 'burst'}, {peak_kind}",
-                     "kernel": "pair_tc_kernel (every pair-forward launch of the step)",
+                     "kernel": "pair_tc2_kernel / pair_tc_kernel (every pair-forward launch of the step)",
                      "algorithmic_flops_per_step": gemm_flops / args.steps,
                      "traffic": None},
         "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": 32},
+                "d2h_bytes_per_step": 8 * step.loss_out.numel()},
         "gpu_launches": launches,
         "clocks": clocks,
         "device_status": status,
     }
-    if world == 1 and not args.no_cpu_baseline and args.workload == DEFAULT_WORKLOAD:
+    if world == 1 and not args.no_cpu_baseline and args.workload == DEFAULT_WORKLOAD and args.queries is None:
         line["cpu_baseline"] = cpu_baseline(step, budget_s=args.cpu_budget)
     print(json.dumps(line))
 
@@ -358,6 +359,8 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
                     choices=["llama_mlp_bf16", "llama_stack_bf16", "llama_stack_int4", "opt_stack_fp16"])
     ap.add_argument("--tokens", type=int, default=None, help="tokens per perturbation (default: the workload's)")
+    ap.add_argument("--queries", type=int, default=None,
+                    help="one-sided estimator with this many queries (Algorithm 2); default: two-sided pair")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--soak", type=float, default=2.0,
                     help="seconds of untimed steps before the timed region (clocks reach their loaded state)")

@@ -173,6 +173,42 @@ int zoact_pair_forward_noalloc(const zoact_layer* layer, const void* X, int xdty
                                int input_shared, float eps, uint64_t seed, uint64_t query, int act,
                                void* Y, int ydtype, void* stream);
 
+/* ---- evaluation blocks: the forward pass at several coefficient points ----
+ * Algorithm 2 evaluates each mini-batch at the unperturbed C (loss L) and at
+ * C + mu Z^(j) for q independent perturbations (losses L^(j,+)).  A
+ * zoact_eval_blocks lists n_blocks such points; a stacked activation then holds
+ * n_blocks * T rows, rows [b T, (b + 1) T) evaluated at
+ *     C + coef[b] * Z(seed, layer_id, query[b]).
+ * coef[b] == 0 draws no Z (query[b] is ignored).  The paper's estimator with q
+ * queries is n_blocks = q + 1, coef = {0, mu, ..., mu}, query = {-, q_1, ..., q_q};
+ * the two-sided pair of zoact_pair_forward is n_blocks = 2, coef = {eps, -eps},
+ * query = {q, q}.  Passed by HOST pointer; read during the call only.          */
+#define ZOACT_MAX_EVAL_BLOCKS 17
+typedef struct zoact_eval_blocks {
+  int32_t n_blocks;                          /* 1 .. ZOACT_MAX_EVAL_BLOCKS */
+  int32_t reserved;                          /* 0 */
+  float coef[ZOACT_MAX_EVAL_BLOCKS];         /* finite */
+  uint64_t query[ZOACT_MAX_EVAL_BLOCKS];
+} zoact_eval_blocks;
+
+/* ---- the multi-point forward (Algorithm 2: the unperturbed pass and the q
+ * forward-perturbed passes of one adapted linear in one launch) ----
+ * As zoact_pair_forward with the two signs replaced by the blocks of `blocks`:
+ *   input_shared == 0: X is [n_blocks T, d_in]; row t of Y uses block t / T.
+ *   input_shared == 1: X is [T, d_in]; W x is computed once per row and Y rows
+ *                      b T + t are written for every block b.
+ * Y is [n_blocks T, d_out].  Other arguments and requirements as for
+ * zoact_pair_forward.                                                          */
+int zoact_multi_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype,
+                        int64_t T, int input_shared, const float* P, const zoact_eval_blocks* blocks,
+                        uint64_t seed, int act, void* Y, int ydtype);
+
+/* ---- SiLU-gated multi-point forward: H = silu(y_gate) * y_up per block ---- */
+int zoact_multi_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up,
+                              const void* X, int xdtype, int64_t T, int input_shared,
+                              const float* P_gate, const float* P_up, const zoact_eval_blocks* blocks,
+                              uint64_t seed, void* H, int ydtype);
+
 /* ---- SiLU-gated pair forward (the Llama MLP gate/up pair) ----
  * H = silu(y_gate) * y_up for both signs, with y_gate, y_up the pair forwards of
  * `gate` and `up` on the same X (same d_in, d_out, r and wtype).  H [2T, d_out]
@@ -192,6 +228,17 @@ int zoact_pair_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoac
 int zoact_loss_pair(zoact_ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T,
                     int64_t n, float eps, double* out);
 
+/* ---- the losses of a multi-point evaluation (Algorithm 2, one-sided) ----
+ * Y [n_blocks T, n] of ydtype, block 0 the unperturbed pass; target [T, n] or
+ * NULL (mean square).  Writes to DEVICE memory out[2 n_blocks - 1] (fp64):
+ *   out[b]                = L_b = mean((y_b - t)^2),            b = 0 .. n_blocks-1
+ *   out[n_blocks + j - 1] = a_j = (L_j - L_0) / mu,             j = 1 .. n_blocks-1
+ * with L_j - L_0 formed as mean((y_j - y_0)(y_j + y_0 - 2t)), without
+ * cancellation.  n_blocks >= 2, mu > 0.  A non-finite result sets
+ * ZOACT_ERR_NONFINITE in the device status word.                               */
+int zoact_loss_multi(zoact_ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T,
+                     int64_t n, int32_t n_blocks, float mu, double* out);
+
 /* ---- ZO-Adam (Section 3: Adam on g = a * Z; Appendix B: weight decay 0) ----
  * Updates the flat fp32 arenas C, m, v (n_total elements) in place for every
  * block: g = a * Z(seed, layer_id, query) with a = loss_out[3] (device fp64),
@@ -208,6 +255,20 @@ int zoact_adam_step(zoact_ctx* ctx, float* C, float* m, float* v, int64_t n_tota
 int zoact_sgd_step(zoact_ctx* ctx, float* C, int64_t n_total, const zoact_coeff_block* blocks,
                    int32_t n_blocks, const double* loss_out, float lr, uint64_t seed,
                    uint64_t query);
+
+/* ---- ZO-Adam / ZO-SGD on the q-query average (Algorithm 2) ----
+ * As zoact_adam_step / zoact_sgd_step with
+ *   g = (1/q) sum_j a[j] * Z(seed, layer_id, queries[j]),   j = 0 .. q-1,
+ * a: DEVICE fp64 [q] (e.g. zoact_loss_multi's out + n_blocks), queries: HOST
+ * array of q ids, 1 <= q <= ZOACT_MAX_EVAL_BLOCKS - 1.  If any a[j] is not
+ * finite nothing is updated and the device status word gets ZOACT_ERR_NONFINITE. */
+int zoact_adam_step_multi(zoact_ctx* ctx, float* C, float* m, float* v, int64_t n_total,
+                          const zoact_coeff_block* blocks, int32_t n_blocks, const double* a, int32_t q,
+                          const uint64_t* queries, float lr, float beta1, float beta2, float adam_eps,
+                          int64_t step, uint64_t seed);
+int zoact_sgd_step_multi(zoact_ctx* ctx, float* C, int64_t n_total, const zoact_coeff_block* blocks,
+                         int32_t n_blocks, const double* a, int32_t q, const uint64_t* queries, float lr,
+                         uint64_t seed);
 
 /* ---- the one-shot basis (Algorithm 1) ----
  * U_out [d_in, r] fp32 = the top-r right singular vectors of the calibration

@@ -22,6 +22,7 @@ ZOACT_ERR_TIMEOUT = -5
 ZOACT_ERR_NOMEM = -6
 ZOACT_ERR_TOO_LARGE = -7
 NOALLOC_MAX_PROJ_FLOATS = 1 << 20
+MAX_EVAL_BLOCKS = 17
 
 DT_FP32, DT_BF16, DT_FP16, DT_INT4_G128 = 0, 1, 2, 3
 ACT_NONE, ACT_RELU, ACT_GELU = 0, 1, 2
@@ -33,7 +34,8 @@ EXPORTS = [
     "zoact_create", "zoact_destroy", "zoact_set_stream", "zoact_status_string", "zoact_get_device_status",
     "zoact_device_sm_count", "zoact_get_launch_count", "zoact_philox_normals", "zoact_lowrank_proj", "zoact_pair_forward",
     "zoact_pair_forward_noalloc", "zoact_pair_forward_gated", "zoact_loss_pair", "zoact_adam_step", "zoact_sgd_step", "zoact_basis_init",
-    "zoact_rms_norm", "zoact_mix_rms",
+    "zoact_rms_norm", "zoact_mix_rms", "zoact_multi_forward", "zoact_multi_forward_gated", "zoact_loss_multi",
+    "zoact_adam_step_multi", "zoact_sgd_step_multi",
 ]
 
 
@@ -52,6 +54,27 @@ class zoact_layer(ctypes.Structure):
 class zoact_coeff_block(ctypes.Structure):
     _fields_ = [("offset", ctypes.c_int64), ("d_out", ctypes.c_int32), ("r", ctypes.c_int32),
                 ("layer_id", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+
+
+class zoact_eval_blocks(ctypes.Structure):
+    _fields_ = [("n_blocks", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("coef", ctypes.c_float * MAX_EVAL_BLOCKS), ("query", ctypes.c_uint64 * MAX_EVAL_BLOCKS)]
+
+
+def eval_blocks(points):
+    """A zoact_eval_blocks from a list of (coef, query) pairs (block order = row-block order)."""
+    if not 1 <= len(points) <= MAX_EVAL_BLOCKS:
+        raise ValueError(f"1 .. {MAX_EVAL_BLOCKS} evaluation blocks")
+    b = zoact_eval_blocks(n_blocks=len(points))
+    for i, (c, q) in enumerate(points):
+        b.coef[i] = float(c)
+        b.query[i] = int(q)
+    return b
+
+
+def one_sided_blocks(mu, queries):
+    """Algorithm 2's evaluation points: the unperturbed pass, then C + mu Z^(j) for each query."""
+    return [(0.0, 0)] + [(float(mu), int(q)) for q in queries]
 
 
 _lib = None
@@ -87,6 +110,15 @@ def load():
         "zoact_basis_init": [P, P, I32, I64, I32, I32, I32, I32, U64, P, P],
         "zoact_rms_norm": [P, P, I32, I64, I32, F32, P],
         "zoact_mix_rms": [P, P, P, P, I32, I64, I32, I32, I32, F32, P],
+        "zoact_multi_forward": [P, ctypes.POINTER(zoact_layer), P, I32, I64, I32, P, ctypes.POINTER(zoact_eval_blocks),
+                                U64, I32, P, I32],
+        "zoact_multi_forward_gated": [P, ctypes.POINTER(zoact_layer), ctypes.POINTER(zoact_layer), P, I32, I64, I32,
+                                      P, P, ctypes.POINTER(zoact_eval_blocks), U64, P, I32],
+        "zoact_loss_multi": [P, P, I32, P, I64, I64, I32, F32, P],
+        "zoact_adam_step_multi": [P, P, P, P, I64, ctypes.POINTER(zoact_coeff_block), I32, P, I32,
+                                  ctypes.POINTER(ctypes.c_uint64), F32, F32, F32, F32, I64, U64],
+        "zoact_sgd_step_multi": [P, P, I64, ctypes.POINTER(zoact_coeff_block), I32, P, I32,
+                                 ctypes.POINTER(ctypes.c_uint64), F32, U64],
     }
     for name, argtypes in sig.items():
         fn = getattr(lib, name)
@@ -262,3 +294,47 @@ def zoact_mix_rms(ctx, q, k, v, Y, n_rep, head_dim, eps=1e-5):
     rows, n = q.shape
     _check("zoact_mix_rms", load().zoact_mix_rms(ctx.handle, _ptr(q), _ptr(k), _ptr(v), _dt(q), rows, n,
                                                   int(n_rep), int(head_dim), float(eps), _ptr(Y)))
+
+
+def zoact_multi_forward(ctx, layer, X, T, input_shared, points, seed, Y, P=None, act=ACT_NONE):
+    """points: list of (coef, query); Y has len(points) * T rows."""
+    b = eval_blocks(points)
+    _check("zoact_multi_forward", load().zoact_multi_forward(ctx.handle, ctypes.byref(layer), _ptr(X), _dt(X), int(T),
+                                                              int(input_shared), _ptr(P), ctypes.byref(b), int(seed),
+                                                              int(act), _ptr(Y), _dt(Y)))
+
+
+def zoact_multi_forward_gated(ctx, gate, up, X, T, input_shared, points, seed, H, P_gate=None, P_up=None):
+    b = eval_blocks(points)
+    _check("zoact_multi_forward_gated", load().zoact_multi_forward_gated(
+        ctx.handle, ctypes.byref(gate), ctypes.byref(up), _ptr(X), _dt(X), int(T), int(input_shared), _ptr(P_gate),
+        _ptr(P_up), ctypes.byref(b), int(seed), _ptr(H), _dt(H)))
+
+
+def zoact_loss_multi(ctx, Y, T, n_blocks, mu, out, target=None):
+    """out: device fp64 [2 n_blocks - 1] = [L_0 .. L_{nb-1}, a_1 .. a_q]."""
+    n = Y.shape[1]
+    _check("zoact_loss_multi", load().zoact_loss_multi(ctx.handle, _ptr(Y), _dt(Y), _ptr(target), int(T), int(n),
+                                                        int(n_blocks), float(mu), _ptr(out)))
+
+
+def _queries(queries):
+    arr = (ctypes.c_uint64 * max(1, len(queries)))()
+    for i, q in enumerate(queries):
+        arr[i] = int(q)
+    return arr
+
+
+def zoact_adam_step_multi(ctx, C, m, v, blocks, a, queries, lr, beta1, beta2, adam_eps, step, seed):
+    """a: device fp64 tensor of len(queries) estimator scalars (e.g. a slice of zoact_loss_multi's out)."""
+    arr = _blocks(blocks)
+    _check("zoact_adam_step_multi", load().zoact_adam_step_multi(
+        ctx.handle, _ptr(C), _ptr(m), _ptr(v), C.numel(), arr, len(blocks), _ptr(a), len(queries),
+        _queries(queries), float(lr), float(beta1), float(beta2), float(adam_eps), int(step), int(seed)))
+
+
+def zoact_sgd_step_multi(ctx, C, blocks, a, queries, lr, seed):
+    arr = _blocks(blocks)
+    _check("zoact_sgd_step_multi", load().zoact_sgd_step_multi(ctx.handle, _ptr(C), C.numel(), arr, len(blocks),
+                                                                _ptr(a), len(queries), _queries(queries), float(lr),
+                                                                int(seed)))

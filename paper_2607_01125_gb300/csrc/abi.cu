@@ -185,9 +185,26 @@ int zoact_lowrank_proj(zoact_ctx* ctx, const void* X, int xdtype, int64_t rows, 
   return launch_lowrank_proj(ctx, X, xdtype, rows, d_in, U, r, P);
 }
 
+static int check_eval_blocks(const zoact_eval_blocks* b) {
+  if (!b || b->n_blocks < 1 || b->n_blocks > ZOACT_MAX_EVAL_BLOCKS) return ZOACT_ERR_INVALID_ARG;
+  for (int i = 0; i < b->n_blocks; ++i)
+    if (!(b->coef[i] == b->coef[i]) || b->coef[i] > 3.0e38f || b->coef[i] < -3.0e38f) return ZOACT_ERR_INVALID_ARG;
+  return ZOACT_OK;
+}
+
+static zoact_eval_blocks pair_blocks(float eps, uint64_t query) {
+  zoact_eval_blocks b{};
+  b.n_blocks = 2;
+  b.coef[0] = eps;
+  b.coef[1] = -eps;
+  b.query[0] = b.query[1] = query;
+  return b;
+}
+
 static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* L2, const void* X, int xdtype,
-                       int64_t T, int input_shared, const float* P, const float* P2, float eps, uint64_t seed,
-                       uint64_t query, int act, void* Y, int ydtype) {
+                       int64_t T, int input_shared, const float* P, const float* P2, const zoact_eval_blocks* blk,
+                       uint64_t seed, int act, void* Y, int ydtype) {
+  if (check_eval_blocks(blk)) return ZOACT_ERR_INVALID_ARG;
   int st = check_layer(L);
   if (st) return st;
   if (L2) {
@@ -204,7 +221,8 @@ static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* 
   if (!aligned16(X) || !aligned16(Y) || !aligned16(L->W) || (L2 && !aligned16(L2->W))) return ZOACT_ERR_INVALID_ARG;
   if (L->d_in % (xdtype == ZOACT_DT_FP32 ? 4 : 8) != 0) return ZOACT_ERR_INVALID_ARG;
   if (L->d_out % 8 != 0) return ZOACT_ERR_INVALID_ARG;
-  const int64_t rows = input_shared ? T : 2 * T;
+  if (T > ((int64_t)1 << 40) / blk->n_blocks) return ZOACT_ERR_INVALID_ARG;
+  const int64_t rows = input_shared ? T : blk->n_blocks * T;
   // projection(s) U^T x, unless the caller passed them
   if (!P) {
     float* p = static_cast<float*>(scratch(ctx, SLOT_P0, (size_t)rows * L->r * sizeof(float)));
@@ -225,7 +243,9 @@ static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* 
   a.rows = rows; a.T = T; a.d_in = L->d_in; a.d_out = L->d_out; a.r = L->r;
   a.shared = input_shared ? 1 : 0; a.act = act;
   a.xdtype = xdtype; a.wtype = L->wtype; a.ydtype = ydtype;
-  a.eps = eps; a.seed = seed; a.query = query; a.layer_id = L->layer_id;
+  a.nb = blk->n_blocks;
+  for (int b = 0; b < blk->n_blocks; ++b) { a.coef[b] = blk->coef[b]; a.qry[b] = blk->query[b]; }
+  a.seed = seed; a.layer_id = L->layer_id;
   if (L2) { a.W2 = L2->W; a.w_scales2 = L2->w_scales; a.P2 = P2; a.C2 = L2->C; a.layer_id2 = L2->layer_id; }
   if (xdtype == ZOACT_DT_FP32) return launch_pair_simt(ctx, a);
   return launch_pair_tc(ctx, a);
@@ -235,7 +255,25 @@ int zoact_pair_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X, 
                        int input_shared, const float* P, float eps, uint64_t seed, uint64_t query, int act, void* Y,
                        int ydtype) {
   ZOACT_ENTER(ctx);
-  return pair_common(ctx, layer, nullptr, X, xdtype, T, input_shared, P, nullptr, eps, seed, query, act, Y, ydtype);
+  const zoact_eval_blocks b = pair_blocks(eps, query);
+  return pair_common(ctx, layer, nullptr, X, xdtype, T, input_shared, P, nullptr, &b, seed, act, Y, ydtype);
+}
+
+int zoact_multi_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype, int64_t T,
+                        int input_shared, const float* P, const zoact_eval_blocks* blocks, uint64_t seed, int act,
+                        void* Y, int ydtype) {
+  ZOACT_ENTER(ctx);
+  return pair_common(ctx, layer, nullptr, X, xdtype, T, input_shared, P, nullptr, blocks, seed, act, Y, ydtype);
+}
+
+int zoact_multi_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up, const void* X,
+                              int xdtype, int64_t T, int input_shared, const float* P_gate, const float* P_up,
+                              const zoact_eval_blocks* blocks, uint64_t seed, void* H, int ydtype) {
+  ZOACT_ENTER(ctx);
+  if (!gate || !up) return ZOACT_ERR_INVALID_ARG;
+  if (xdtype == ZOACT_DT_FP32) return ZOACT_ERR_UNSUPPORTED;
+  return pair_common(ctx, gate, up, X, xdtype, T, input_shared, P_gate, P_up, blocks, seed, ZOACT_ACT_NONE, H,
+                     ydtype);
 }
 
 int zoact_pair_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up, const void* X,
@@ -244,8 +282,8 @@ int zoact_pair_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoac
   ZOACT_ENTER(ctx);
   if (!gate || !up) return ZOACT_ERR_INVALID_ARG;
   if (xdtype == ZOACT_DT_FP32) return ZOACT_ERR_UNSUPPORTED;
-  return pair_common(ctx, gate, up, X, xdtype, T, input_shared, P_gate, P_up, eps, seed, query, ZOACT_ACT_NONE, H,
-                     ydtype);
+  const zoact_eval_blocks b = pair_blocks(eps, query);
+  return pair_common(ctx, gate, up, X, xdtype, T, input_shared, P_gate, P_up, &b, seed, ZOACT_ACT_NONE, H, ydtype);
 }
 
 int zoact_loss_pair(zoact_ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T, int64_t n, float eps,
@@ -257,6 +295,19 @@ int zoact_loss_pair(zoact_ctx* ctx, const void* Y, int ydtype, const void* targe
   double* partials = static_cast<double*>(scratch(ctx, SLOT_PARTIALS, (size_t)max_blocks * 3 * sizeof(double)));
   if (!partials) return ZOACT_ERR_NOMEM;
   return launch_loss_pair(ctx, Y, ydtype, target, T, n, eps, out, partials, max_blocks);
+}
+
+int zoact_loss_multi(zoact_ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T, int64_t n,
+                     int32_t n_blocks, float mu, double* out) {
+  ZOACT_ENTER(ctx);
+  if (!Y || !out || T <= 0 || n <= 0 || !valid_act_dtype(ydtype)) return ZOACT_ERR_INVALID_ARG;
+  if (n_blocks < 2 || n_blocks > ZOACT_MAX_EVAL_BLOCKS || !(mu > 0.0f)) return ZOACT_ERR_INVALID_ARG;
+  if (T * n > ((int64_t)1 << 40) / n_blocks) return ZOACT_ERR_INVALID_ARG;
+  const int max_blocks = loss_pair_max_blocks(ctx);
+  double* partials =
+      static_cast<double*>(scratch(ctx, SLOT_PARTIALS, (size_t)max_blocks * 2 * n_blocks * sizeof(double)));
+  if (!partials) return ZOACT_ERR_NOMEM;
+  return launch_loss_multi(ctx, Y, ydtype, target, T, n, n_blocks, mu, out, partials, max_blocks);
 }
 
 static int check_blocks(const float* C, int64_t n_total, const zoact_coeff_block* blocks, int32_t n_blocks) {
@@ -281,7 +332,31 @@ int zoact_adam_step(zoact_ctx* ctx, float* C, float* m, float* v, int64_t n_tota
   if (st) return st;
   if (!m || !v || !loss_out || step < 1 || !aligned16(m) || !aligned16(v)) return ZOACT_ERR_INVALID_ARG;
   if (!(beta1 >= 0.f && beta1 < 1.f && beta2 >= 0.f && beta2 < 1.f)) return ZOACT_ERR_INVALID_ARG;
-  return launch_adam(ctx, C, m, v, blocks, n_blocks, loss_out, lr, beta1, beta2, adam_eps, step, seed, query, 0);
+  return launch_adam(ctx, C, m, v, blocks, n_blocks, loss_out + 3, 1, &query, lr, beta1, beta2, adam_eps, step, seed,
+                     0);
+}
+
+int zoact_adam_step_multi(zoact_ctx* ctx, float* C, float* m, float* v, int64_t n_total,
+                          const zoact_coeff_block* blocks, int32_t n_blocks, const double* a, int32_t q,
+                          const uint64_t* queries, float lr, float beta1, float beta2, float adam_eps, int64_t step,
+                          uint64_t seed) {
+  ZOACT_ENTER(ctx);
+  int st = check_blocks(C, n_total, blocks, n_blocks);
+  if (st) return st;
+  if (!m || !v || !a || !queries || step < 1 || !aligned16(m) || !aligned16(v)) return ZOACT_ERR_INVALID_ARG;
+  if (q < 1 || q > ZOACT_MAX_EVAL_BLOCKS - 1) return ZOACT_ERR_INVALID_ARG;
+  if (!(beta1 >= 0.f && beta1 < 1.f && beta2 >= 0.f && beta2 < 1.f)) return ZOACT_ERR_INVALID_ARG;
+  return launch_adam(ctx, C, m, v, blocks, n_blocks, a, q, queries, lr, beta1, beta2, adam_eps, step, seed, 0);
+}
+
+int zoact_sgd_step_multi(zoact_ctx* ctx, float* C, int64_t n_total, const zoact_coeff_block* blocks,
+                         int32_t n_blocks, const double* a, int32_t q, const uint64_t* queries, float lr,
+                         uint64_t seed) {
+  ZOACT_ENTER(ctx);
+  int st = check_blocks(C, n_total, blocks, n_blocks);
+  if (st) return st;
+  if (!a || !queries || q < 1 || q > ZOACT_MAX_EVAL_BLOCKS - 1) return ZOACT_ERR_INVALID_ARG;
+  return launch_adam(ctx, C, nullptr, nullptr, blocks, n_blocks, a, q, queries, lr, 0.f, 0.f, 0.f, 1, seed, 1);
 }
 
 int zoact_sgd_step(zoact_ctx* ctx, float* C, int64_t n_total, const zoact_coeff_block* blocks, int32_t n_blocks,
@@ -290,7 +365,8 @@ int zoact_sgd_step(zoact_ctx* ctx, float* C, int64_t n_total, const zoact_coeff_
   int st = check_blocks(C, n_total, blocks, n_blocks);
   if (st) return st;
   if (!loss_out) return ZOACT_ERR_INVALID_ARG;
-  return launch_adam(ctx, C, nullptr, nullptr, blocks, n_blocks, loss_out, lr, 0.f, 0.f, 0.f, 1, seed, query, 1);
+  return launch_adam(ctx, C, nullptr, nullptr, blocks, n_blocks, loss_out + 3, 1, &query, lr, 0.f, 0.f, 0.f, 1, seed,
+                     1);
 }
 
 int zoact_basis_init(zoact_ctx* ctx, const void* X_cal, int xdtype, int64_t n_tok, int32_t d_in, int32_t r,

@@ -94,15 +94,18 @@ struct PairArgs {
   const void* w_scales;
   const float* P;       // [rows, r]
   const float* C;       // [d_out, r]
-  void* Y;              // [2T, d_out]
-  int64_t rows;         // rows of X (T if shared else 2T)
+  void* Y;              // [nb T, d_out]
+  int64_t rows;         // rows of X (T if shared else nb T)
   int64_t T;
   int d_in, d_out, r;
   int shared;
   int act;
   int xdtype, wtype, ydtype;
-  float eps;
-  uint64_t seed, query;
+  // evaluation blocks: rows [b T, (b+1) T) of Y at C + coef[b] Z(seed, layer_id, qry[b])
+  int nb;
+  float coef[ZOACT_MAX_EVAL_BLOCKS];
+  uint64_t qry[ZOACT_MAX_EVAL_BLOCKS];
+  uint64_t seed;
   uint32_t layer_id;
   // gated mode (second layer: up); W2 == nullptr for the plain pair forward
   const void* W2;
@@ -111,6 +114,13 @@ struct PairArgs {
   const float* C2;
   uint32_t layer_id2;
 };
+// The two-sided pair as evaluation blocks: {+eps, -eps} with the same query.
+inline void set_pair_blocks(PairArgs& a, float eps, uint64_t query) {
+  a.nb = 2;
+  a.coef[0] = eps;
+  a.coef[1] = -eps;
+  a.qry[0] = a.qry[1] = query;
+}
 int launch_pair_simt(Ctx* ctx, const PairArgs& a);
 // INT4 g128 weight [d_out, d_in/2] + fp16 scales -> bf16 [d_out, d_in].
 int launch_dequant_int4(Ctx* ctx, const void* Wq, const void* Ws, void* Wb, int64_t d_out, int d_in);
@@ -125,9 +135,13 @@ int launch_loss_pair(Ctx* ctx, const void* Y, int ydtype, const void* target, in
                      float eps, double* out, double* partials, int max_blocks);
 int loss_pair_max_blocks(Ctx* ctx);
 
+int launch_loss_multi(Ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T, int64_t n, int nb,
+                      float mu, double* out, double* partials, int max_blocks);
+
+// g = (1/q) sum_j a[j] Z(seed, layer_id, queries[j]) (q = 1: the two-sided a * Z).
 int launch_adam(Ctx* ctx, float* C, float* m, float* v, const zoact_coeff_block* blocks, int n_blocks,
-                const double* loss_out, float lr, float b1, float b2, float adam_eps, int64_t step,
-                uint64_t seed, uint64_t query, int sgd);
+                const double* a, int q, const uint64_t* queries, float lr, float b1, float b2, float adam_eps,
+                int64_t step, uint64_t seed, int sgd);
 
 int launch_rms_norm(Ctx* ctx, const void* X, int dtype, int64_t rows, int n, float eps, void* Y);
 int launch_mix_rms(Ctx* ctx, const void* q, const void* k, const void* v, int dtype, int64_t rows,

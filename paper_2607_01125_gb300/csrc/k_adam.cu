@@ -1,7 +1,8 @@
 // ZO-Adam and ZO-SGD over the flat coefficient arenas (Section 3: Adam on the
 // estimated coefficient gradient; Table 1 "Full SGD"; Appendix B: weight decay 0).
 //
-//   g = a * Z(seed, layer_id, query)          (Z regenerated, never stored)
+//   g = (1/q) sum_j a_j Z(seed, layer_id, query_j)   (Z regenerated, never stored;
+//                                                      q = 1, a = a_pair: the two-sided g = a Z)
 //   m = b1 m + (1 - b1) g ;  v = b2 v + (1 - b2) g^2
 //   C -= (lr / (1 - b1^t)) * m / (sqrt(v) / sqrt(1 - b2^t) + adam_eps)
 //
@@ -10,7 +11,8 @@
 // normals, and C, m, v move as 16-byte vectors.  The layer table (offsets,
 // layer ids) travels in the kernel parameters; a group finds its layer by binary
 // search.  a is read from device memory (the loss kernel's output), so a whole
-// ZO step runs without a host synchronisation.
+// ZO step runs without a host synchronisation.  With q queries every group
+// draws q Philox groups (one per query) and sums a_j z_j in query order.
 #include "internal.h"
 #include "philox.cuh"
 
@@ -20,6 +22,10 @@ namespace zoact {
 namespace {
 
 constexpr int ADAM_TABLE = 256;  // layers per launch
+
+struct QueryList {
+  uint64_t q[ZOACT_MAX_EVAL_BLOCKS];
+};
 
 struct AdamTable {
   int64_t begin[ADAM_TABLE];
@@ -40,23 +46,42 @@ __device__ __forceinline__ int find_block(const AdamTable& t, int64_t e) {
 template <bool SGD>
 __global__ void __launch_bounds__(256)
 zo_update_kernel(float* __restrict__ C, float* __restrict__ m, float* __restrict__ v, const __grid_constant__ AdamTable tab,
-                 int64_t g_begin, int64_t g_end, const double* __restrict__ loss_out, float lr, float b1, float b2,
-                 float adam_eps, float step_size, float inv_sqrt_bc2, uint64_t seed, uint64_t query,
-                 int* __restrict__ status) {
-  const double a_d = loss_out[3];
-  if (!isfinite(a_d)) {
+                 int64_t g_begin, int64_t g_end, const double* __restrict__ a_dev, int nq,
+                 const __grid_constant__ QueryList qs, float lr, float b1, float b2, float adam_eps, float step_size,
+                 float inv_sqrt_bc2, uint64_t seed, int* __restrict__ status) {
+  float a[ZOACT_MAX_EVAL_BLOCKS];
+  bool finite = true;
+#pragma unroll
+  for (int j = 0; j < ZOACT_MAX_EVAL_BLOCKS; ++j) {
+    const double aj = j < nq ? a_dev[j] : 0.0;
+    finite = finite && isfinite(aj);
+    a[j] = (float)aj;
+  }
+  if (!finite) {
     if (blockIdx.x == 0 && threadIdx.x == 0) record_error(status, ZOACT_ERR_NONFINITE);
     return;
   }
-  const float a = (float)a_d;
+  const float inv_q = 1.0f / (float)nq;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t g = g_begin + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; g < g_end; g += stride) {
     const int64_t e = 4 * g;
     const int b = find_block(tab, e);
     if (e >= tab.end[b]) continue;                       // gap between blocks
     const int64_t local = e - tab.begin[b];              // element index inside the layer's [d_out, r]
-    const float4 z = z_normals4(seed, tab.layer_id[b], query, (uint64_t)(local >> 2));
-    const float gz[4] = {a * z.x, a * z.y, a * z.z, a * z.w};
+    float gz[4];
+    {
+      const float4 z = z_normals4(seed, tab.layer_id[b], qs.q[0], (uint64_t)(local >> 2));
+      gz[0] = a[0] * z.x; gz[1] = a[0] * z.y; gz[2] = a[0] * z.z; gz[3] = a[0] * z.w;
+    }
+    if (nq > 1) {
+      for (int j = 1; j < nq; ++j) {
+        const float4 z = z_normals4(seed, tab.layer_id[b], qs.q[j], (uint64_t)(local >> 2));
+        gz[0] = fmaf(a[j], z.x, gz[0]); gz[1] = fmaf(a[j], z.y, gz[1]);
+        gz[2] = fmaf(a[j], z.z, gz[2]); gz[3] = fmaf(a[j], z.w, gz[3]);
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) gz[i] *= inv_q;
+    }
     const bool full = e + 4 <= tab.end[b];
     if (SGD) {
       if (full) {
@@ -102,8 +127,11 @@ zo_update_kernel(float* __restrict__ C, float* __restrict__ m, float* __restrict
 }  // namespace
 
 int launch_adam(Ctx* ctx, float* C, float* m, float* v, const zoact_coeff_block* blocks, int n_blocks,
-                const double* loss_out, float lr, float b1, float b2, float adam_eps, int64_t step, uint64_t seed,
-                uint64_t query, int sgd) {
+                const double* a, int q, const uint64_t* queries, float lr, float b1, float b2, float adam_eps,
+                int64_t step, uint64_t seed, int sgd) {
+  if (q < 1 || q > ZOACT_MAX_EVAL_BLOCKS) return ZOACT_ERR_INVALID_ARG;
+  QueryList qs{};
+  for (int j = 0; j < q; ++j) qs.q[j] = queries[j];
   const double bc1 = 1.0 - std::pow((double)b1, (double)step);
   const double bc2 = 1.0 - std::pow((double)b2, (double)step);
   const float step_size = sgd ? 0.f : (float)((double)lr / bc1);
@@ -126,12 +154,12 @@ int launch_adam(Ctx* ctx, float* C, float* m, float* v, const zoact_coeff_block*
     const int64_t cap = (int64_t)ctx->sm_count * 8;
     if (nb > cap) nb = cap;
     if (sgd) {
-      zo_update_kernel<true><<<(unsigned)nb, 256, 0, ctx->stream>>>(C, m, v, tab, g_begin, g_end, loss_out, lr, b1, b2,
-                                                                    adam_eps, step_size, inv_sqrt_bc2, seed, query,
+      zo_update_kernel<true><<<(unsigned)nb, 256, 0, ctx->stream>>>(C, m, v, tab, g_begin, g_end, a, q, qs, lr, b1,
+                                                                    b2, adam_eps, step_size, inv_sqrt_bc2, seed,
                                                                     ctx->d_status);
     } else {
-      zo_update_kernel<false><<<(unsigned)nb, 256, 0, ctx->stream>>>(C, m, v, tab, g_begin, g_end, loss_out, lr, b1, b2,
-                                                                     adam_eps, step_size, inv_sqrt_bc2, seed, query,
+      zo_update_kernel<false><<<(unsigned)nb, 256, 0, ctx->stream>>>(C, m, v, tab, g_begin, g_end, a, q, qs, lr, b1,
+                                                                     b2, adam_eps, step_size, inv_sqrt_bc2, seed,
                                                                      ctx->d_status);
     }
     ++ctx->n_launch;

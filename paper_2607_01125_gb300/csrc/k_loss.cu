@@ -171,9 +171,151 @@ int loss_dispatch(Ctx* ctx, const TY* Y, const TY* tgt, int64_t count, float eps
   return ZOACT_OK;
 }
 
+// Losses of a multi-point evaluation (Algorithm 2, one-sided, q queries):
+//   L_b = mean((y_b - t)^2) for every block b,
+//   D_j = mean((y_j - y_0)(y_j + y_0 - 2t)) (= L_j - L_0),  a_j = D_j / mu.
+// blockIdx.y is the block b; each CTA reads y_b, y_0 and t over its share of
+// the elements (y_0 and t are re-read once per block, from L2 when they fit).
+// Partials [nb][gridDim.x][2] are added in a fixed order by the last CTA.
+template <typename TY>
+__global__ void __launch_bounds__(LOSS_THREADS)
+loss_multi_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t count, int vec_ok, int nb, float mu,
+                  double* __restrict__ out, double* __restrict__ partials, unsigned int* __restrict__ ticket,
+                  int* __restrict__ status) {
+  const int b = blockIdx.y;
+  const TY* yb = Y + (int64_t)b * count;
+  const TY* y0 = Y;
+  double as = 0.0, ad = 0.0;
+  const int64_t n_vec = vec_ok ? count / 8 : 0;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t first = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  for (int64_t v = first; v < n_vec; v += stride) {
+    float y[8], z[8], t[8];
+    load8<TY>(yb + 8 * v, y);
+    if (b > 0) {
+      load8<TY>(y0 + 8 * v, z);
+    }
+    if (tgt) {
+      load8<TY>(tgt + 8 * v, t);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) t[i] = 0.f;
+    }
+    float ss = 0.f, sd = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float dy = y[i] - t[i];
+      ss = fmaf(dy, dy, ss);
+      if (b > 0) sd = fmaf(y[i] - z[i], dy + (z[i] - t[i]), sd);
+    }
+    as += ss; ad += sd;
+  }
+  for (int64_t i = 8 * n_vec + first; i < count; i += stride) {
+    const float tv = tgt ? to_f32<TY>(tgt[i]) : 0.f;
+    const float yv = to_f32<TY>(yb[i]);
+    const float dy = yv - tv;
+    as += (double)(dy * dy);
+    if (b > 0) {
+      const float zv = to_f32<TY>(y0[i]);
+      ad += (double)((yv - zv) * (dy + (zv - tv)));
+    }
+  }
+  __shared__ double red[2][LOSS_THREADS / 32];
+  __shared__ bool is_last;
+  as = warp_sum(as); ad = warp_sum(ad);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0) { red[0][warp] = as; red[1][warp] = ad; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double s0 = 0.0, s1 = 0.0;
+    for (int w = 0; w < LOSS_THREADS / 32; ++w) { s0 += red[0][w]; s1 += red[1][w]; }
+    double* pb = partials + 2 * ((int64_t)b * gridDim.x + blockIdx.x);
+    pb[0] = s0;
+    pb[1] = s1;
+    __threadfence();
+    const unsigned int prev = atomicAdd(ticket, 1u);
+    is_last = (prev == gridDim.x * gridDim.y - 1);
+  }
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  __shared__ double tree[2][LOSS_THREADS];
+  const double inv = 1.0 / (double)count;
+  bool finite = true;
+  for (int bb = 0; bb < nb; ++bb) {
+    double s0 = 0.0, s1 = 0.0;
+    for (unsigned int x = threadIdx.x; x < gridDim.x; x += LOSS_THREADS) {
+      const double* pb = partials + 2 * ((int64_t)bb * gridDim.x + x);
+      s0 += __ldcg(pb);
+      s1 += __ldcg(pb + 1);
+    }
+    tree[0][threadIdx.x] = s0; tree[1][threadIdx.x] = s1;
+    __syncthreads();
+    for (int h = LOSS_THREADS / 2; h > 0; h >>= 1) {
+      if (threadIdx.x < h) {
+        tree[0][threadIdx.x] += tree[0][threadIdx.x + h];
+        tree[1][threadIdx.x] += tree[1][threadIdx.x + h];
+      }
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+      const double L = tree[0][0] * inv;
+      out[bb] = L;
+      finite = finite && isfinite(L);
+      if (bb > 0) {
+        const double a = tree[1][0] * inv / (double)mu;
+        out[nb + bb - 1] = a;
+        finite = finite && isfinite(a);
+      }
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    if (!finite) record_error(status, ZOACT_ERR_NONFINITE);
+    *ticket = 0u;
+  }
+}
+
+template <typename TY>
+int loss_multi_dispatch(Ctx* ctx, const TY* Y, const TY* tgt, int64_t count, int nb, float mu, double* out,
+                        double* partials, int max_blocks, unsigned int* ticket) {
+  const int vec_ok = (count % 8 == 0) && ((uintptr_t)Y % 16 == 0) && ((uintptr_t)tgt % 16 == 0);
+  int64_t bx = ((vec_ok ? count / 8 : count) + LOSS_THREADS - 1) / LOSS_THREADS;
+  if (bx < 1) bx = 1;
+  int64_t cap = max_blocks / nb;
+  if (cap < 1) cap = 1;
+  if (bx > cap) bx = cap;
+  dim3 grid((unsigned)bx, (unsigned)nb);
+  loss_multi_kernel<TY><<<grid, LOSS_THREADS, 0, ctx->stream>>>(Y, tgt, count, vec_ok, nb, mu, out, partials, ticket,
+                                                               ctx->d_status);
+  ++ctx->n_launch;
+  ZOACT_CHECK_LAUNCH();
+  return ZOACT_OK;
+}
+
 }  // namespace
 
 int loss_pair_max_blocks(Ctx* ctx) { return 4 * ctx->sm_count; }
+
+int launch_loss_multi(Ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T, int64_t n, int nb, float mu,
+                      double* out, double* partials, int max_blocks) {
+  const int64_t count = T * n;
+  unsigned int* ticket = ctx->d_tickets;
+  switch (ydtype) {
+    case ZOACT_DT_FP32:
+      return loss_multi_dispatch(ctx, static_cast<const float*>(Y), static_cast<const float*>(target), count, nb, mu,
+                                 out, partials, max_blocks, ticket);
+    case ZOACT_DT_BF16:
+      return loss_multi_dispatch(ctx, static_cast<const __nv_bfloat16*>(Y),
+                                 static_cast<const __nv_bfloat16*>(target), count, nb, mu, out, partials, max_blocks,
+                                 ticket);
+    case ZOACT_DT_FP16:
+      return loss_multi_dispatch(ctx, static_cast<const __half*>(Y), static_cast<const __half*>(target), count, nb,
+                                 mu, out, partials, max_blocks, ticket);
+    default:
+      return ZOACT_ERR_INVALID_ARG;
+  }
+}
 
 int launch_loss_pair(Ctx* ctx, const void* Y, int ydtype, const void* target, int64_t T, int64_t n, float eps,
                      double* out, double* partials, int max_blocks) {

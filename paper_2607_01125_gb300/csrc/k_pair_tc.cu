@@ -135,7 +135,12 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   Params p{};
   p.P = a.P; p.C = a.C; p.P2 = a.P2; p.C2 = a.C2; p.Y = a.Y;
   p.rows = a.rows; p.T = a.T; p.d_in = a.d_in; p.d_out = a.d_out; p.r = a.r;
-  p.shared = a.shared; p.act = a.act; p.eps = a.eps; p.seed = a.seed; p.query = a.query;
+  p.shared = a.shared; p.act = a.act; p.seed = a.seed;
+  p.nb = a.nb;
+  for (int b = 0; b < ZOACT_MAX_EVAL_BLOCKS; ++b) {
+    p.coef[b] = b < a.nb ? a.coef[b] : 0.f;
+    p.qry[b] = b < a.nb ? a.qry[b] : 0;
+  }
   p.layer_id = a.layer_id; p.layer_id2 = a.layer_id2;
   p.num_m = (int)((a.rows + BM - 1) / BM);
   p.bn = bn;

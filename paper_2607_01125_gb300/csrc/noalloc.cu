@@ -102,6 +102,7 @@ extern "C" int zoact_pair_forward_noalloc(const zoact_layer* L, const void* X, i
   a.rows = rows; a.T = T; a.d_in = L->d_in; a.d_out = L->d_out; a.r = L->r;
   a.shared = input_shared ? 1 : 0; a.act = act;
   a.xdtype = xdtype; a.wtype = L->wtype; a.ydtype = ydtype;
-  a.eps = eps; a.seed = seed; a.query = query; a.layer_id = L->layer_id;
+  set_pair_blocks(a, eps, query);
+  a.seed = seed; a.layer_id = L->layer_id;
   return xdtype == ZOACT_DT_FP32 ? launch_pair_simt(&c, a) : launch_pair_tc(&c, a);
 }

@@ -23,7 +23,7 @@ namespace pairtc {
 constexpr int STAGES2 = 6;
 constexpr int B_HALF_BYTES = (BN / 2) * BK * 2;
 constexpr int STAGE2_BYTES = A_BYTES + B_HALF_BYTES;
-constexpr int SMEM2_BYTES = 1024 + STAGES2 * STAGE2_BYTES + 2 * TABLE_FLOATS * 4 + 256;
+constexpr int SMEM2_BYTES = 1024 + STAGES2 * STAGE2_BYTES + TBL_FLOATS * 4 + 256;
 constexpr int BM2 = 2 * BM;
 
 struct SharedState2 {
@@ -36,6 +36,8 @@ struct SharedState2 {
   int abort_flag;
   int epi_ok;
 };
+static_assert(sizeof(SharedState2) <= 256, "barrier block outgrew its shared-memory slot");
+static_assert(SMEM2_BYTES <= 232448, "dynamic shared memory above the 227 KB a CTA may use");
 
 namespace tc2 {
 
@@ -113,9 +115,8 @@ pair_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
   constexpr int CW = 16;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  float* Ct = reinterpret_cast<float*>(smem + STAGES2 * STAGE2_BYTES);
-  float* Zt = Ct + TABLE_FLOATS;
-  SharedState2* ss = reinterpret_cast<SharedState2*>(Zt + TABLE_FLOATS);
+  float* tbl = reinterpret_cast<float*>(smem + STAGES2 * STAGE2_BYTES);
+  SharedState2* ss = reinterpret_cast<SharedState2*>(tbl + TBL_FLOATS);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -238,7 +239,9 @@ pair_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
       const int64_t m = (int64_t)m_blk * BM2 + (int64_t)rank * BM + row_in_tile;
       const bool row_ok = m < prm.rows;
       const uint32_t t_row = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * BN);
-      const bool ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, Ct, Zt, etid, half, m, row_ok, n_blk, bn, buf,
+      const bool ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, tbl, etid, half,
+                                                      (int64_t)m_blk * BM2 + (int64_t)rank * BM, m, row_ok,
+                                                      n_blk, bn, buf,
                                                       acc_phase, t_row, abort_flag);
       if (!ok) break;
       tc::tc_fence_before();

@@ -1,13 +1,15 @@
 // Pair forward on the 5th-generation tensor cores (Section 3, the perturbed
 // forward pass; Algorithm 2 evaluates it at +eps and -eps):
 //
-//   Y[t, n] = act( sum_k X[t, k] W[n, k] + sum_j (C[n, j] + sigma(t) eps Z[n, j]) P[t, j] )
+//   Y[t, n] = act( sum_k X[t, k] W[n, k] + sum_j (C[n, j] + c_b Z_b[n, j]) P[t, j] )
 //
-// with P = X U (computed before), Z regenerated from Philox inside the epilogue.
-// The + and - perturbations are stacked along the token axis, so every W tile
-// is fetched once for both signs; when both signs share the input (the first
-// layer, or gate/up of an MLP) the product is computed once and each
-// accumulator row is written twice.
+// with P = X U (computed before) and Z_b regenerated from Philox inside the
+// epilogue.  The evaluation points b (the two signs +eps / -eps of the pair,
+// or Algorithm 2's unperturbed pass and its q forward-perturbed passes) are
+// stacked along the token axis in blocks of T rows, so every W tile is fetched
+// once for all of them; when all blocks share the input (the first layer, or
+// gate/up of an MLP) the product is computed once and each accumulator row is
+// written once per block.
 //
 // Structure (one persistent CTA per SM, 320 threads):
 //   warp 0      TMA producer: X and W tiles (128x64 and 256x64, bf16/fp16,
@@ -17,11 +19,12 @@
 //               tile overlaps the main loop of the next;
 //   warps 2-9   epilogue, two warpgroups: warp w reads TMEM lanes
 //               32*(w%4) .. +31 (its rows) and warpgroup h the h-th half of
-//               the tile's columns.  Per tile they build the C and Z columns of
-//               the tile in shared memory (Z from Philox), tcgen05.ld the
-//               accumulator 16 columns at a time, add the low-rank term in
-//               fp32 (32 independent accumulators per 16 columns), apply the
-//               activation and store from registers.
+//               the tile's columns.  Per tile and block they build the table
+//               C + c_b Z_b of the tile's columns in shared memory (Z from
+//               Philox; two blocks per pass), tcgen05.ld the accumulator 16
+//               columns at a time, add the low-rank term with packed fp32x2
+//               FMAs (column pairs), apply the activation and store from
+//               registers.
 // Gated mode (SiLU MLP gate/up): the 256-row W tile is 128 rows of W_gate and
 // the same 128 rows of W_up; the epilogue writes silu(gate) * up for 128 columns.
 // Plain mode (no P): the accumulator is stored as fp32 (used for X^T X).
@@ -48,15 +51,24 @@ constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int TABLE_FLOATS = 4096;  // per table (C or Z): slots * RT
+// Epilogue tables: C + c_b Z_b for the tile's columns, one [RT][slots + 4]
+// table per evaluation block of a pass (two blocks per pass; gated mode keeps
+// gate and up tables, four in all).  The 4-float row padding spreads the
+// table writes over the banks and keeps rows 16-byte aligned.
+constexpr int TBL_FLOATS = 8448;
+constexpr int TPAD = 4;
+__host__ __device__ constexpr int pair_slots(int rt) {
+  return (2 * rt * (BN + TPAD) <= TBL_FLOATS) ? BN : (2 * rt * (BN / 2 + TPAD) <= TBL_FLOATS ? BN / 2 : BN / 4);
+}
 constexpr int EPI_WARPS = 8;
 constexpr int EPI_THREADS = 32 * EPI_WARPS;
 constexpr int DQ_THREADS = 128;                     // INT4 dequantisation warps
 __host__ __device__ constexpr int num_threads(bool w4) { return 64 + EPI_THREADS + (w4 ? DQ_THREADS : 0); }
 __host__ __device__ constexpr int epi_base(bool w4) { return 64 + (w4 ? DQ_THREADS : 0); }
 constexpr int TMEM_COLS = 512;
-constexpr int SMEM_BYTES = 1024 /*align slack*/ + STAGES * STAGE_BYTES + 2 * TABLE_FLOATS * 4 + 256;
+constexpr int SMEM_BYTES = 1024 /*align slack*/ + STAGES * STAGE_BYTES + TBL_FLOATS * 4 + 256;
 constexpr int GROUP_M = 8;
+static_assert(SMEM_BYTES <= 232448, "dynamic shared memory above the 227 KB a CTA may use");
 
 enum Mode { MODE_PAIR = 0, MODE_GATED = 1, MODE_PLAIN = 2 };
 
@@ -71,8 +83,10 @@ struct Params {
   int d_in, d_out, r;
   int shared;
   int act;
-  float eps;
-  uint64_t seed, query;
+  int nb;                                   // evaluation blocks (rows [b T, (b+1) T) of Y)
+  float coef[ZOACT_MAX_EVAL_BLOCKS];
+  uint64_t qry[ZOACT_MAX_EVAL_BLOCKS];
+  uint64_t seed;
   uint32_t layer_id, layer_id2;
   int num_m, num_n, num_k, num_tiles;
   int64_t ldy;       // plain mode: row stride of D
@@ -96,6 +110,7 @@ struct SharedState {
   int abort_flag;
   int epi_ok;
 };
+static_assert(sizeof(SharedState) <= 256, "barrier block outgrew its shared-memory slot");
 
 __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& m_blk, int& n_blk) {
   const int per_group = GROUP_M * num_n;
@@ -107,76 +122,102 @@ __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int&
   n_blk = in_group / gm;
 }
 
-// Fill table slots [slot0, slot0 + ncols) with C and Z of output columns
-// [col0, col0 + ncols) of one layer; columns >= d_out and the padded ranks
-// j >= r get zeros.  Rows of the tables are RT floats (RT >= r, RT % 4 == 0).
+// Fill the tables of one layer for output columns [col0, col0 + ncols) at two
+// evaluation points (tb1 may be null):
+//   tb0[j * stride + s] = C[col0 + s][j] + c0 Z(q0)[col0 + s][j]   (tb1: c1, q1)
+// zero where col0 + s >= d_out or j >= r.  A point with coefficient 0 draws no
+// Z; when both points use the same query (the two signs of the pair) Z is drawn
+// once.
 template <int RT>
-__device__ __forceinline__ void build_table(float* Ct, float* Zt, const float* __restrict__ Cg, uint32_t layer_id,
-                                            int col0, int ncols, int slot0, int d_out, int r, uint64_t seed,
-                                            uint64_t query, int tid, bool vec_ok) {
+__device__ __forceinline__ void build_tables(float* tb0, float* tb1, int stride, const float* __restrict__ Cg,
+                                             uint32_t layer_id, int col0, int ncols, int d_out, int r,
+                                             uint64_t seed, float c0, uint64_t q0, float c1, uint64_t q1, int tid,
+                                             bool vec_ok) {
   const int valid_cols = max(0, min(ncols, d_out - col0));
-  const int64_t e_begin = (int64_t)col0 * r;            // element range of the layer's [d_out, r] C and Z
-  const int64_t e_end = e_begin + (int64_t)valid_cols * r;
+  const bool z0_on = c0 != 0.f, z1_on = tb1 != nullptr && c1 != 0.f;
+  const bool z1_same = z1_on && z0_on && q1 == q0;
   if (r == RT && vec_ok) {
-    // rows of the table are the rows of C and Z: one group of 4 lands in one slot row
-    const int n_groups = ncols * RT / 4;
-    float4* C4 = reinterpret_cast<float4*>(Ct + slot0 * RT);
-    float4* Z4 = reinterpret_cast<float4*>(Zt + slot0 * RT);
+    // one thread per 4 consecutive ranks of one column: one float4 of C, one Philox group
+    constexpr int GPC = RT / 4;                          // groups per column
+    const int n_groups = ncols * GPC;
     for (int g = tid; g < n_groups; g += EPI_THREADS) {
-      const int64_t e = e_begin + 4 * (int64_t)g;
-      float4 c = make_float4(0.f, 0.f, 0.f, 0.f), z = c;
-      if (e < e_end) {
+      const int s = g / GPC, jg = g % GPC;
+      float4 c = make_float4(0.f, 0.f, 0.f, 0.f), z0 = c, z1 = c;
+      if (s < valid_cols) {
+        const int64_t e = (int64_t)(col0 + s) * RT + 4 * jg;
         c = *reinterpret_cast<const float4*>(Cg + e);
-        z = z_normals4(seed, layer_id, query, (uint64_t)(e >> 2));
+        if (z0_on) z0 = z_normals4(seed, layer_id, q0, (uint64_t)(e >> 2));
+        if (z1_on) z1 = z1_same ? z0 : z_normals4(seed, layer_id, q1, (uint64_t)(e >> 2));
       }
-      C4[g] = c;
-      Z4[g] = z;
+      float* d0 = tb0 + (4 * jg) * stride + s;
+      d0[0] = fmaf(c0, z0.x, c.x);
+      d0[stride] = fmaf(c0, z0.y, c.y);
+      d0[2 * stride] = fmaf(c0, z0.z, c.z);
+      d0[3 * stride] = fmaf(c0, z0.w, c.w);
+      if (tb1) {
+        float* d1 = tb1 + (4 * jg) * stride + s;
+        d1[0] = fmaf(c1, z1.x, c.x);
+        d1[stride] = fmaf(c1, z1.y, c.y);
+        d1[2 * stride] = fmaf(c1, z1.z, c.z);
+        d1[3 * stride] = fmaf(c1, z1.w, c.w);
+      }
     }
     return;
   }
+  // general ranks / unaligned C: one element per iteration
   for (int i = tid; i < ncols * RT; i += EPI_THREADS) {
-    const int c = i / RT, j = i % RT;
-    if (c >= valid_cols || j >= r) {
-      Ct[(slot0 + c) * RT + j] = 0.f;
-      Zt[(slot0 + c) * RT + j] = 0.f;
+    const int s = i / RT, j = i % RT;
+    float v0 = 0.f, v1 = 0.f;
+    if (s < valid_cols && j < r) {
+      const int64_t e = (int64_t)(col0 + s) * r + j;
+      const float c = Cg[e];
+      const uint64_t grp = (uint64_t)(e >> 2);
+      const int w = (int)(e & 3);
+      const float z0 = z0_on ? z_select(z_normals4(seed, layer_id, q0, grp), w) : 0.f;
+      const float z1 = z1_on ? (z1_same ? z0 : z_select(z_normals4(seed, layer_id, q1, grp), w)) : 0.f;
+      v0 = fmaf(c0, z0, c);
+      v1 = fmaf(c1, z1, c);
     }
-  }
-  const int64_t g_begin = e_begin >> 2, g_end = (e_end + 3) >> 2;
-  for (int64_t g = g_begin + tid; g < g_end; g += EPI_THREADS) {
-    const float4 z = z_normals4(seed, layer_id, query, (uint64_t)g);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int64_t e = 4 * g + i;
-      if (e >= e_begin && e < e_end) {
-        const int64_t le = e - e_begin;
-        const int c = (int)(le / r), j = (int)(le % r);
-        Zt[(slot0 + c) * RT + j] = z_select(z, i);
-        Ct[(slot0 + c) * RT + j] = Cg[e];
-      }
-    }
+    tb0[j * stride + s] = v0;
+    if (tb1) tb1[j * stride + s] = v1;
   }
 }
 
-// Low-rank sums of CW consecutive table slots for one token row:
-//   sC[i] = sum_j Ct[slot0+i][j] p[j],   sZ[i] = sum_j Zt[slot0+i][j] p[j].
+// d = a * b + c on two fp32 lanes at once (one packed FMA; each lane rounds
+// like fmaf).
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\t"
+      "mov.b64 rb, {%4, %5};\n\t"
+      "mov.b64 rc, {%6, %7};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\t"
+      "mov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+
+// Low-rank sums of CW consecutive table columns for one token row:
+//   s[i] = sum_j tb[j * stride + c + i] p[j]     (j ascending).
 template <int RT, int CW>
-__device__ __forceinline__ void lowrankN(const float* Ct, const float* Zt, int slot0, const float* p, float* sC,
-                                         float* sZ) {
+__device__ __forceinline__ void lowrank_t(const float* tb, int stride, int c, const float* p, float* s) {
+  float2 acc[CW / 2];
 #pragma unroll
-  for (int i = 0; i < CW; ++i) { sC[i] = 0.f; sZ[i] = 0.f; }
-  const float4* c4 = reinterpret_cast<const float4*>(Ct + slot0 * RT);
-  const float4* z4 = reinterpret_cast<const float4*>(Zt + slot0 * RT);
+  for (int i = 0; i < CW / 2; ++i) acc[i] = make_float2(0.f, 0.f);
 #pragma unroll
-  for (int q = 0; q < RT / 4; ++q) {
-    const float p0 = p[4 * q], p1 = p[4 * q + 1], p2 = p[4 * q + 2], p3 = p[4 * q + 3];
+  for (int j = 0; j < RT; ++j) {
+    const float4* t4 = reinterpret_cast<const float4*>(tb + j * stride + c);
+    const float2 pj = make_float2(p[j], p[j]);
 #pragma unroll
-    for (int i = 0; i < CW; ++i) {
-      const float4 c = c4[i * (RT / 4) + q];
-      const float4 z = z4[i * (RT / 4) + q];
-      sC[i] = fmaf(c.x, p0, fmaf(c.y, p1, fmaf(c.z, p2, fmaf(c.w, p3, sC[i]))));
-      sZ[i] = fmaf(z.x, p0, fmaf(z.y, p1, fmaf(z.z, p2, fmaf(z.w, p3, sZ[i]))));
+    for (int q = 0; q < CW / 4; ++q) {
+      const float4 v = t4[q];
+      acc[2 * q] = ffma2(make_float2(v.x, v.y), pj, acc[2 * q]);
+      acc[2 * q + 1] = ffma2(make_float2(v.z, v.w), pj, acc[2 * q + 1]);
     }
   }
+#pragma unroll
+  for (int i = 0; i < CW / 2; ++i) { s[2 * i] = acc[i].x; s[2 * i + 1] = acc[i].y; }
 }
 
 __device__ __forceinline__ float silu_fast(float x) { return __fdividef(x, 1.0f + __expf(-x)); }
@@ -309,104 +350,102 @@ __device__ __forceinline__ void load_p(float* p, const float* __restrict__ P, in
   }
 }
 
-// Pair / gated epilogue of one accumulator tile for this CTA's 128 rows (row m
-// of thread (quad, lane)): builds the tile's C and Z tables, waits for the
-// accumulator, adds the low-rank term, applies the activation or the SiLU gate
-// and stores.  Returns false when the wait gave up.
+// Pair / gated epilogue of one accumulator tile for this CTA's 128 rows
+// [row0, row0 + 128) (row m of thread (quad, lane)).  Column chunk by column
+// chunk, and two evaluation blocks per pass, it builds the tables C + c_b Z_b,
+// waits for the accumulator (first pass), adds the low-rank term, applies the
+// activation or the SiLU gate and stores.  Stacked rows use the block they
+// belong to; shared rows are written once per block.  Returns false when the
+// wait gave up.
 template <typename TO, int RT, int MODE, int CW, typename SS>
-__device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* Ct, float* Zt, int etid,
-                                              int half, int64_t m, bool row_ok, int n_blk, int bn, int buf,
+__device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* tbl, int etid, int half,
+                                              int64_t row0, int64_t m, bool row_ok, int n_blk, int bn, int buf,
                                               uint32_t acc_phase, uint32_t t_row, volatile int* abort_flag) {
+  constexpr bool GATED = MODE == MODE_GATED;
+  constexpr int SLOTS = GATED ? BN / 2 : pair_slots(RT);   // table columns per chunk
+  constexpr int STRIDE = SLOTS + TPAD;
+  constexpr int TSZ = RT * STRIDE;                         // floats per table
+  static_assert((GATED ? 4 : 2) * TSZ <= TBL_FLOATS, "epilogue tables exceed their shared-memory region");
   const int r = prm.r;
-  // ---- pair / gated epilogue ----
-  // table chunks: slots per chunk such that slots * RT <= TABLE_FLOATS
-  constexpr int CHUNK = (TABLE_FLOATS / RT) < BN ? (TABLE_FLOATS / RT) : BN;
-  static_assert(MODE != MODE_GATED || CHUNK == BN, "gated mode keeps the whole tile's table");
+  const int64_t T = prm.T;
   float p[RT], p2[RT];
   const bool vec = prm.vec_ok != 0;
   load_p<RT>(p, prm.P, m, r, row_ok, vec);
-  if (MODE == MODE_GATED) load_p<RT>(p2, prm.P2, m, r, row_ok, vec);
-  const float sgn_eps = m < prm.T ? prm.eps : -prm.eps;   // stacked rows: sign of the half
+  if (GATED) load_p<RT>(p2, prm.P2, m, r, row_ok, vec);
+  // evaluation blocks this CTA's rows touch
+  int b_first = 0, b_last = prm.nb - 1;
+  if (!prm.shared) {
+    const int64_t last_row = min(row0 + BM, prm.rows) - 1;
+    b_first = (int)(row0 / T);
+    b_last = (int)(last_row / T);
+  }
+  if (b_last < b_first)    // no valid row in this CTA's part of the tile: only release the accumulator
+    return epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid);
+  const int my_b = (!prm.shared && row_ok) ? (int)(m / T) : -1;
   TO* Y = static_cast<TO*>(prm.Y);
-  bool ok = true;
-  for (int s0 = 0; s0 < bn && ok; s0 += CHUNK) {
-    const int cwid = min(CHUNK, bn - s0);        // slots in this chunk (a multiple of 32)
-    tc::named_bar_sync(1, EPI_THREADS);          // previous chunk's readers are done
-    if (MODE == MODE_GATED) {
-      build_table<RT>(Ct, Zt, prm.C, prm.layer_id, n_blk * (BN / 2), BN / 2, 0, prm.d_out, r, prm.seed,
-                      prm.query, etid, vec);
-      build_table<RT>(Ct, Zt, prm.C2, prm.layer_id2, n_blk * (BN / 2), BN / 2, BN / 2, prm.d_out, r,
-                      prm.seed, prm.query, etid, vec);
-    } else {
-      build_table<RT>(Ct, Zt, prm.C, prm.layer_id, n_blk * bn + s0, cwid, 0, prm.d_out, r, prm.seed,
-                      prm.query, etid, vec);
-    }
-    tc::named_bar_sync(1, EPI_THREADS);
-    if (s0 == 0) {
-      if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) { ok = false; break; }
-    }
-    if (MODE == MODE_GATED) {
-      for (int c0 = half * (BN / 4); c0 < (half + 1) * (BN / 4); c0 += CW) {
-        float g[CW], u[CW];
-        tmem_ldN<CW>(t_row + (uint32_t)c0, g);
-        tmem_ldN<CW>(t_row + (uint32_t)(BN / 2 + c0), u);
-        const int n = n_blk * (BN / 2) + c0;
-        if (!row_ok || n >= prm.d_out) continue;
-        const int nv = min(CW, prm.d_out - n);
-        float gC[CW], gZ[CW];
-        lowrankN<RT, CW>(Ct, Zt, c0, p, gC, gZ);
-#pragma unroll
-        for (int i = 0; i < CW; ++i) g[i] += gC[i];      // g = W_g x + C_g p
-        float uC[CW], uZ[CW];
-        lowrankN<RT, CW>(Ct, Zt, BN / 2 + c0, p2, uC, uZ);
-#pragma unroll
-        for (int i = 0; i < CW; ++i) u[i] += uC[i];
-        if (prm.shared) {
-          float hp[CW], hm[CW];
-#pragma unroll
-          for (int i = 0; i < CW; ++i) {
-            hp[i] = silu_fast(fmaf(prm.eps, gZ[i], g[i])) * fmaf(prm.eps, uZ[i], u[i]);
-            hm[i] = silu_fast(fmaf(-prm.eps, gZ[i], g[i])) * fmaf(-prm.eps, uZ[i], u[i]);
-          }
-          storeN<TO, CW>(Y + m * prm.d_out + n, hp, nv);
-          storeN<TO, CW>(Y + (prm.T + m) * prm.d_out + n, hm, nv);
-        } else {
-          float h[CW];
-#pragma unroll
-          for (int i = 0; i < CW; ++i) h[i] = silu_fast(fmaf(sgn_eps, gZ[i], g[i])) * fmaf(sgn_eps, uZ[i], u[i]);
-          storeN<TO, CW>(Y + m * prm.d_out + n, h, nv);
-        }
+  const int ncol_tile = GATED ? BN / 2 : bn;               // output columns of this tile
+  bool waited = false;
+  for (int s0 = 0; s0 < ncol_tile; s0 += SLOTS) {
+    const int cwid = min(SLOTS, ncol_tile - s0);          // a multiple of 32
+    const int col0 = n_blk * ncol_tile + s0;
+    for (int bp = b_first; bp <= b_last; bp += 2) {
+      const bool two = bp + 1 <= b_last;
+      const int b1 = two ? bp + 1 : bp;
+      tc::named_bar_sync(1, EPI_THREADS);                 // previous pass's readers are done
+      build_tables<RT>(tbl, two ? tbl + TSZ : nullptr, STRIDE, prm.C, prm.layer_id, col0, cwid, prm.d_out, r,
+                       prm.seed, prm.coef[bp], prm.qry[bp], prm.coef[b1], prm.qry[b1], etid, vec);
+      if (GATED)
+        build_tables<RT>(tbl + 2 * TSZ, two ? tbl + 3 * TSZ : nullptr, STRIDE, prm.C2, prm.layer_id2, col0, cwid, prm.d_out, r,
+                         prm.seed, prm.coef[bp], prm.qry[bp], prm.coef[b1], prm.qry[b1], etid, vec);
+      tc::named_bar_sync(1, EPI_THREADS);
+      if (!waited) {
+        if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
+        waited = true;
       }
-    } else {
+      const int sel = my_b - bp;                          // stacked: my table in this pass
+      const bool active = prm.shared ? row_ok : (sel == 0 || (sel == 1 && two));
+      if (!prm.shared && !__any_sync(0xffffffffu, active)) continue;   // no row of this warp in the pass
+      const int nt = prm.shared ? (two ? 2 : 1) : 1;
       const int cbeg = s0 + half * (cwid / 2);
       for (int c0 = cbeg; c0 < cbeg + cwid / 2; c0 += CW) {
-        float acc[CW];
-        tmem_ldN<CW>(t_row + (uint32_t)c0, acc);
-        const int n = n_blk * bn + c0;
-        if (!row_ok || n >= prm.d_out) continue;
+        const int n = n_blk * ncol_tile + c0;
+        if (n >= prm.d_out) break;                        // uniform: same columns for the whole warp
         const int nv = min(CW, prm.d_out - n);
-        float sC[CW], sZ[CW];
-        lowrankN<RT, CW>(Ct, Zt, c0 - s0, p, sC, sZ);
-        if (prm.shared) {
-          float yp[CW], ym[CW];
+        if (GATED) {
+          float g[CW], u[CW];
+          tmem_ldN<CW>(t_row + (uint32_t)c0, g);
+          tmem_ldN<CW>(t_row + (uint32_t)(BN / 2 + c0), u);
+          if (active) {
+            for (int t = 0; t < nt; ++t) {
+              const int ts = prm.shared ? t : sel;
+              float sg[CW], su[CW], h[CW];
+              lowrank_t<RT, CW>(tbl + ts * TSZ, STRIDE, c0 - s0, p, sg);
+              lowrank_t<RT, CW>(tbl + (2 + ts) * TSZ, STRIDE, c0 - s0, p2, su);
 #pragma unroll
-          for (int i = 0; i < CW; ++i) {
-            const float base = acc[i] + sC[i];
-            yp[i] = apply_act(fmaf(prm.eps, sZ[i], base), prm.act);
-            ym[i] = apply_act(fmaf(-prm.eps, sZ[i], base), prm.act);
+              for (int i = 0; i < CW; ++i) h[i] = silu_fast(g[i] + sg[i]) * (u[i] + su[i]);
+              const int64_t row = prm.shared ? (int64_t)(bp + t) * T + m : m;
+              storeN<TO, CW>(Y + row * prm.d_out + n, h, nv);
+            }
           }
-          storeN<TO, CW>(Y + m * prm.d_out + n, yp, nv);
-          storeN<TO, CW>(Y + (prm.T + m) * prm.d_out + n, ym, nv);
         } else {
-          float y[CW];
+          float acc[CW];
+          tmem_ldN<CW>(t_row + (uint32_t)c0, acc);
+          if (active) {
+            for (int t = 0; t < nt; ++t) {
+              const int ts = prm.shared ? t : sel;
+              float sl[CW], y[CW];
+              lowrank_t<RT, CW>(tbl + ts * TSZ, STRIDE, c0 - s0, p, sl);
 #pragma unroll
-          for (int i = 0; i < CW; ++i) y[i] = apply_act(fmaf(sgn_eps, sZ[i], acc[i] + sC[i]), prm.act);
-          storeN<TO, CW>(Y + m * prm.d_out + n, y, nv);
+              for (int i = 0; i < CW; ++i) y[i] = apply_act(acc[i] + sl[i], prm.act);
+              const int64_t row = prm.shared ? (int64_t)(bp + t) * T + m : m;
+              storeN<TO, CW>(Y + row * prm.d_out + n, y, nv);
+            }
+          }
         }
       }
     }
   }
-  return ok;
+  return true;
 }
 
 template <typename TO, int RT, int MODE, int AB_BF16, bool W4>
@@ -416,9 +455,8 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   constexpr int CW = W4 ? 8 : 16;                   // epilogue chunk width (columns per tcgen05.ld)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  float* Ct = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);
-  float* Zt = Ct + TABLE_FLOATS;
-  SharedState* ss = reinterpret_cast<SharedState*>(Zt + TABLE_FLOATS);
+  float* tbl = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);
+  SharedState* ss = reinterpret_cast<SharedState*>(tbl + TBL_FLOATS);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -600,7 +638,8 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         continue;
       }
 
-      const bool ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, Ct, Zt, etid, half, m, row_ok, n_blk, bn, buf,
+      const bool ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, tbl, etid, half, (int64_t)m_blk * BM, m, row_ok,
+                                                      n_blk, bn, buf,
                                                       acc_phase, t_row, abort_flag);
       if (!ok) break;
       tc::tc_fence_before();

@@ -6,6 +6,12 @@ One ZO step (Algorithm 2 with one two-sided query) is
     zoact_loss_pair   -> L+, L-, D, a  (device memory)
     zoact_adam_step   -> C, m, v updated with g = a * Z over all layers
 
+With ``n_queries = q`` the step is the paper's own one-sided form: every
+linear is evaluated at q + 1 points in one launch (zoact_multi_forward: the
+unperturbed C, then C + mu Z^(j) with mu = eps), zoact_loss_multi gives
+L_0..L_q and a_j = (L_j - L_0) / mu, and zoact_adam_step_multi updates C with
+g = (1/q) sum_j a_j Z^(j).
+
 with no host synchronisation.  This module only allocates buffers and issues
 the calls; every arithmetic step runs in libzoact's kernels.  Layers that read
 the same input with the same basis (q/k/v, gate/up after a calibration pass)
@@ -57,7 +63,7 @@ class ZOStep:
     """Holds frozen weights/bases, the coefficient arenas and activation buffers."""
 
     def __init__(self, ctx, kind, linears, T, act_dtype, eps=1e-3, lr=1e-4, beta1=0.9, beta2=0.999,
-                 adam_eps=1e-8, n_heads=32, n_kv_heads=8, head_dim=128):
+                 adam_eps=1e-8, n_heads=32, n_kv_heads=8, head_dim=128, n_queries=None):
         self.ctx = ctx
         self.kind = kind
         self.T = int(T)
@@ -76,7 +82,9 @@ class ZOStep:
         for l in linears:
             l.bind(self.C)
         self.blocks = [(l.offset, l.d_out, l.r, l.layer_id) for l in linears]
-        self.loss_out = torch.zeros(4, dtype=torch.float64, device=dev)
+        self.n_queries = n_queries                  # None: two-sided pair; q: one-sided with q queries
+        self.nb = 2 if n_queries is None else int(n_queries) + 1
+        self.loss_out = torch.zeros(4 if n_queries is None else 2 * self.nb - 1, dtype=torch.float64, device=dev)
         self._bufs = {}
         self._pcache = {}
         self.device = dev
@@ -121,15 +129,27 @@ class ZOStep:
         e1.record()
         self.timer.append((e0, e1, flops))
 
+    def query_ids(self, query):
+        """The q Philox query ids of one one-sided step."""
+        return [int(query) * self.n_queries + j for j in range(self.n_queries)]
+
+    def points(self, query):
+        return Z.one_sided_blocks(self.eps, self.query_ids(query))
+
     def pair(self, name, X, shared, seed, query, out_key, act=Z.ACT_NONE):
         l = self.by_name[name]
         if self.capture is not None:
             self.capture(name, X[:self.T])
         P = self._proj(l, X, 0)
-        Y = self.buf(out_key, 2 * self.T, l.d_out)
+        Y = self.buf(out_key, self.nb * self.T, l.d_out)
         flops = 2.0 * X.shape[0] * l.d_in * l.d_out
-        self._timed(lambda: Z.zoact_pair_forward(self.ctx, l.layer, X, self.T, shared, self.eps, seed, query, Y,
-                                                 P=P, act=act), flops)
+        if self.n_queries is None:
+            fn = lambda: Z.zoact_pair_forward(self.ctx, l.layer, X, self.T, shared, self.eps, seed, query, Y, P=P,
+                                              act=act)
+        else:
+            fn = lambda: Z.zoact_multi_forward(self.ctx, l.layer, X, self.T, shared, self.points(query), seed, Y,
+                                               P=P, act=act)
+        self._timed(fn, flops)
         self._wrote(Y)
         return Y
 
@@ -140,10 +160,15 @@ class ZOStep:
             self.capture(uname, X[:self.T])
         Pg = self._proj(g, X, 0)
         Pu = self._proj(u, X, 1)
-        H = self.buf(out_key, 2 * self.T, g.d_out)
+        H = self.buf(out_key, self.nb * self.T, g.d_out)
         flops = 2.0 * X.shape[0] * g.d_in * g.d_out * 2
-        self._timed(lambda: Z.zoact_pair_forward_gated(self.ctx, g.layer, u.layer, X, self.T, shared, self.eps, seed,
-                                                       query, H, P_gate=Pg, P_up=Pu), flops)
+        if self.n_queries is None:
+            fn = lambda: Z.zoact_pair_forward_gated(self.ctx, g.layer, u.layer, X, self.T, shared, self.eps, seed,
+                                                    query, H, P_gate=Pg, P_up=Pu)
+        else:
+            fn = lambda: Z.zoact_multi_forward_gated(self.ctx, g.layer, u.layer, X, self.T, shared,
+                                                     self.points(query), seed, H, P_gate=Pg, P_up=Pu)
+        self._timed(fn, flops)
         self._wrote(H)
         return H
 
@@ -170,13 +195,13 @@ class ZOStep:
         h = x
         shared = True
         for L in range(n_dec):
-            rows = T if shared else 2 * T
+            rows = T if shared else self.nb * T
             a = self._glue_rms(h, f"a{rows}")
             q = self.pair(f"{L}.q", a, shared, seed, query, "q")
             k = self.pair(f"{L}.k", a, shared, seed, query, "k")
             v = self.pair(f"{L}.v", a, shared, seed, query, "v")
             shared = False
-            mix = self.buf("mix", 2 * T, q.shape[1])
+            mix = self.buf("mix", self.nb * T, q.shape[1])
             Z.zoact_mix_rms(self.ctx, q, k, v, mix, self.n_rep if self.kind == "llama" else 1, self.head_dim)
             self._wrote(mix)
             o = self.pair(f"{L}.o", mix, False, seed, query, "o")
@@ -193,12 +218,21 @@ class ZOStep:
 
     # ---- loss and update ----
     def loss(self, Y, target):
-        Z.zoact_loss_pair(self.ctx, Y, self.T, self.eps, self.loss_out, target=target)
+        """Two-sided: [L+, L-, D, a].  One-sided: [L_0 .. L_q, a_1 .. a_q]."""
+        if self.n_queries is None:
+            Z.zoact_loss_pair(self.ctx, Y, self.T, self.eps, self.loss_out, target=target)
+        else:
+            Z.zoact_loss_multi(self.ctx, Y, self.T, self.nb, self.eps, self.loss_out, target=target)
         return self.loss_out
 
     def update(self, step, seed, query, lr=None):
-        Z.zoact_adam_step(self.ctx, self.C, self.m, self.v, self.blocks, self.loss_out,
-                          self.lr if lr is None else lr, self.beta1, self.beta2, self.adam_eps, step, seed, query)
+        lr = self.lr if lr is None else lr
+        if self.n_queries is None:
+            Z.zoact_adam_step(self.ctx, self.C, self.m, self.v, self.blocks, self.loss_out, lr, self.beta1,
+                              self.beta2, self.adam_eps, step, seed, query)
+        else:
+            Z.zoact_adam_step_multi(self.ctx, self.C, self.m, self.v, self.blocks, self.loss_out[self.nb:],
+                                    self.query_ids(query), lr, self.beta1, self.beta2, self.adam_eps, step, seed)
 
     def step(self, x, target, step, seed, query, lr=None):
         """One ZO step: pair forwards, loss pair, Adam.  Returns the device loss tensor [L+, L-, D, a]."""
