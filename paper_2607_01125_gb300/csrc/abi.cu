@@ -17,6 +17,7 @@ int cuda_fail(cudaError_t e, const char* what) {
 void* scratch(Ctx* ctx, ScratchSlot slot, size_t bytes) {
   if (bytes == 0) bytes = 256;
   if (ctx->slot_bytes[slot] >= bytes) return ctx->slot_ptr[slot];
+  if (!ctx->may_allocate) return nullptr;
   if (ctx->slot_ptr[slot]) {
     // queued kernels may still use the old buffer
     if (cudaStreamSynchronize(ctx->stream) != cudaSuccess) return nullptr;

@@ -30,6 +30,8 @@ enum ScratchSlot {
   SLOT_UT,           // 16-bit split copy of the basis for the tensor-core projection
   SLOT_WDQ0,         // bf16 copy of an INT4 weight (staged INT4 pair forward)
   SLOT_WDQ1,         // second copy (gated up weight)
+  SLOT_AUG_A,        // 16-bit split of the projection P (extra K columns of the tensor-core pair forward)
+  SLOT_AUG_B,        // 16-bit split of C (+ c_b Z_b) for those K columns (gate and up)
   SLOT_COUNT
 };
 
@@ -38,6 +40,7 @@ struct Ctx {
   cudaStream_t stream = nullptr;
   int sm_count = 0;
   int64_t n_launch = 0;              // kernels launched through this context (host counter)
+  bool may_allocate = true;          // false: no scratch may be allocated (kernels that need none only)
   int* d_status = nullptr;            // device status word (first error wins)
   unsigned int* d_tickets = nullptr;  // grid-reduction tickets, reset by their last block
   void* slot_ptr[SLOT_COUNT] = {};
@@ -128,6 +131,18 @@ int launch_dequant_int4(Ctx* ctx, const void* Wq, const void* Ws, void* Wb, int6
 constexpr int64_t INT4_STAGED_MIN_ROWS = 1024;
 int launch_pair_tc(Ctx* ctx, const PairArgs& a);
 // Plain product D[M, N] (fp32) = A[M, K] * B[N, K]^T with 16-bit A, B (K-major), on tcgen05.
+// Low-rank term of the tensor-core pair forward (see k_aug.cu):
+//   LOWRANK_EPILOGUE  (C + c_b Z_b) p summed in the epilogue (fp32 tables)
+//   LOWRANK_C_ON_TC   C p as extra K columns of the MMA, c_b Z_b p in the epilogue
+//   LOWRANK_ALL_ON_TC (C + c_b Z_b) p as extra K columns (stacked rows whose tiles lie in one block)
+enum LowrankMode { LOWRANK_EPILOGUE = 0, LOWRANK_C_ON_TC = 1, LOWRANK_ALL_ON_TC = 2 };
+// Extra K columns per layer for rank r: the three 16-bit products P_hi T_hi, P_hi T_lo, P_lo T_hi
+// padded to whole 64-column K-blocks.
+inline int aug_cols(int r) { return (3 * r + 63) / 64 * 64; }
+// Writes A_aug [rows, ka_tot] and B_aug / B_aug2 [nbB * d_out, ka_tot] (bf16) for one pair forward.
+// distinct: gate and up have their own projections (A_aug holds both, B_aug zero-pads the other half).
+int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct, void* A_aug, void* B_aug,
+                    void* B_aug2);
 int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int M, int N, int K,
                           float* D);
 

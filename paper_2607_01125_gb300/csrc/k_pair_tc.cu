@@ -9,15 +9,11 @@
 namespace zoact {
 
 namespace pairtc {
-int dispatch_bf16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const CUtensorMap& b,
-                  const CUtensorMap& b2, const Params& p);
-int dispatch_fp16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const CUtensorMap& b,
-                  const CUtensorMap& b2, const Params& p);
+int dispatch_bf16(Ctx* ctx, int mode, int rt, int ydtype, const TmaSet& tm, const Params& p);
+int dispatch_fp16(Ctx* ctx, int mode, int rt, int ydtype, const TmaSet& tm, const Params& p);
 int dispatch_w4(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const Params& p);
-int dispatch2_bf16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const CUtensorMap& b,
-                   const CUtensorMap& b2, const Params& p);
-int dispatch2_fp16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const CUtensorMap& b,
-                   const CUtensorMap& b2, const Params& p);
+int dispatch2_bf16(Ctx* ctx, int mode, int rt, int ydtype, const TmaSet& tm, const Params& p);
+int dispatch2_fp16(Ctx* ctx, int mode, int rt, int ydtype, const TmaSet& tm, const Params& p);
 }  // namespace pairtc
 
 namespace {
@@ -110,27 +106,61 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   const int rt = rank_template(a.r);
   if (gated && rt > 16) return ZOACT_ERR_UNSUPPORTED;
   if (a.rows <= 0) return ZOACT_OK;
-  CUtensorMap ma, mb, mb2;
-  int st = encode_tmap_2d_16bit(&ma, a.X, a.xdtype, a.rows, a.d_in, BM);
+  TmaSet tm;
+  int st = encode_tmap_2d_16bit(&tm.a, a.X, a.xdtype, a.rows, a.d_in, BM);
   if (st) return st;
-  if (w4) {
-    mb = mb2 = ma;                       // W arrives through the dequantising warps, not TMA
-  }
   // CTA pairs (256-row tiles) once there are enough rows to fill them; INT4 in-kernel dequant stays on one CTA
   const char* sel = std::getenv("ZOACT_PAIR_KERNEL");
   const bool two = !w4 && a.rows >= 2 * BM && !(sel && std::strcmp(sel, "1cta") == 0);
   const int bn = (gated || w4) ? BN
                                : (two ? choose_bn(a.rows, a.d_out, ctx->sm_count / 2, 2 * BM)
                                       : choose_bn(a.rows, a.d_out, ctx->sm_count));
-  if (!w4) {
-    st = encode_tmap_2d_16bit(&mb, a.W, a.wtype, a.d_out, a.d_in, gated ? BN / 2 : (two ? bn / 2 : bn));
-    if (st) return st;
-  }
-  if (gated && !w4) {
-    st = encode_tmap_2d_16bit(&mb2, a.W2, a.wtype, a.d_out, a.d_in, BN / 2);
-    if (st) return st;
+  const int b_box = gated ? BN / 2 : (two ? bn / 2 : bn);
+  if (w4) {
+    tm.b = tm.b2 = tm.a;                 // W arrives through the dequantising warps, not TMA
   } else {
-    mb2 = mb;
+    st = encode_tmap_2d_16bit(&tm.b, a.W, a.wtype, a.d_out, a.d_in, b_box);
+    if (st) return st;
+    if (gated) {
+      st = encode_tmap_2d_16bit(&tm.b2, a.W2, a.wtype, a.d_out, a.d_in, BN / 2);
+      if (st) return st;
+    } else {
+      tm.b2 = tm.b;
+    }
+  }
+  // low-rank term: on the tensor cores where the context may hold the split operands
+  const char* lsel = std::getenv("ZOACT_LOWRANK");
+  int lmode = LOWRANK_EPILOGUE;
+  if (!w4 && ctx->may_allocate && !(lsel && std::strcmp(lsel, "epilogue") == 0)) {
+    const int64_t tile_rows = two ? 2 * BM : BM;
+    lmode = (!a.shared && a.T % tile_rows == 0) ? LOWRANK_ALL_ON_TC : LOWRANK_C_ON_TC;
+  }
+  const int ka = aug_cols(a.r);
+  const bool distinct = gated && a.P2 != a.P;
+  const int ka_tot = distinct ? 2 * ka : ka;
+  tm.aa = tm.a; tm.ba = tm.b; tm.ba2 = tm.b2;
+  int64_t aug_block_rows = 0;
+  if (lmode != LOWRANK_EPILOGUE) {
+    const int64_t nbB = lmode == LOWRANK_ALL_ON_TC ? a.nb : 1;
+    const size_t a_bytes = (size_t)a.rows * ka_tot * 2;
+    const size_t b_bytes = (size_t)nbB * a.d_out * ka_tot * 2;
+    uint8_t* abuf = static_cast<uint8_t*>(scratch(ctx, SLOT_AUG_A, a_bytes));
+    uint8_t* bbuf = static_cast<uint8_t*>(scratch(ctx, SLOT_AUG_B, (gated ? 2 : 1) * b_bytes));
+    if (!abuf || !bbuf) return ZOACT_ERR_NOMEM;
+    uint8_t* bbuf2 = gated ? bbuf + b_bytes : nullptr;
+    st = launch_aug_prep(ctx, a, lmode, ka, distinct ? 1 : 0, abuf, bbuf, bbuf2);
+    if (st) return st;
+    st = encode_tmap_2d_16bit(&tm.aa, abuf, ZOACT_DT_BF16, a.rows, ka_tot, BM);
+    if (st) return st;
+    st = encode_tmap_2d_16bit(&tm.ba, bbuf, ZOACT_DT_BF16, nbB * a.d_out, ka_tot, b_box);
+    if (st) return st;
+    if (gated) {
+      st = encode_tmap_2d_16bit(&tm.ba2, bbuf2, ZOACT_DT_BF16, nbB * a.d_out, ka_tot, b_box);
+      if (st) return st;
+    } else {
+      tm.ba2 = tm.ba;
+    }
+    aug_block_rows = a.d_out;
   }
   Params p{};
   p.P = a.P; p.C = a.C; p.P2 = a.P2; p.C2 = a.C2; p.Y = a.Y;
@@ -149,6 +179,9 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   if (two) p.num_m = (int)((a.rows + 2 * BM - 1) / (2 * BM));
   p.num_tiles = p.num_m * p.num_n;
   p.ldy = a.d_out;
+  p.aug_mode = lmode;
+  p.aug_kb = lmode == LOWRANK_EPILOGUE ? 0 : ka_tot / BK;
+  p.aug_block_rows = aug_block_rows;
   auto al16 = [](const void* q) { return q == nullptr || ((uintptr_t)q & 15u) == 0; };
   p.vec_ok = al16(a.C) && al16(a.C2) && al16(a.P) && al16(a.P2);
   p.status = ctx->d_status;
@@ -158,24 +191,26 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     p.Ws = static_cast<const __half*>(a.w_scales);
     p.Wq2 = static_cast<const uint8_t*>(a.W2);
     p.Ws2 = static_cast<const __half*>(a.w_scales2);
-    return dispatch_w4(ctx, mode, rt, a.ydtype, ma, p);
+    return dispatch_w4(ctx, mode, rt, a.ydtype, tm.a, p);
   }
   if (two)
-    return a.xdtype == ZOACT_DT_BF16 ? dispatch2_bf16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p)
-                                     : dispatch2_fp16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p);
-  return a.xdtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p)
-                                   : dispatch_fp16(ctx, mode, rt, a.ydtype, ma, mb, mb2, p);
+    return a.xdtype == ZOACT_DT_BF16 ? dispatch2_bf16(ctx, mode, rt, a.ydtype, tm, p)
+                                     : dispatch2_fp16(ctx, mode, rt, a.ydtype, tm, p);
+  return a.xdtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, mode, rt, a.ydtype, tm, p)
+                                   : dispatch_fp16(ctx, mode, rt, a.ydtype, tm, p);
 }
 
 int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int M, int N, int K, float* D) {
   using namespace pairtc;
   if (M <= 0 || N <= 0) return ZOACT_OK;
-  CUtensorMap ma, mb;
+  TmaSet tm;
   const int bn = choose_bn(M, N, ctx->sm_count);
-  int st = encode_tmap_2d_16bit(&ma, A, dtype, M, K, BM);
+  int st = encode_tmap_2d_16bit(&tm.a, A, dtype, M, K, BM);
   if (st) return st;
-  st = encode_tmap_2d_16bit(&mb, B, dtype, N, K, bn);
+  st = encode_tmap_2d_16bit(&tm.b, B, dtype, N, K, bn);
   if (st) return st;
+  tm.b2 = tm.ba = tm.ba2 = tm.b;
+  tm.aa = tm.a;
   Params p{};
   p.Y = D;
   p.rows = M; p.T = M; p.d_in = K; p.d_out = N; p.r = 0;
@@ -187,8 +222,8 @@ int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int
   p.ldy = N;
   p.vec_ok = (N % 4) == 0 && ((uintptr_t)D & 15u) == 0;
   p.status = ctx->d_status;
-  return dtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, MODE_PLAIN, 4, ZOACT_DT_FP32, ma, mb, mb, p)
-                                : dispatch_fp16(ctx, MODE_PLAIN, 4, ZOACT_DT_FP32, ma, mb, mb, p);
+  return dtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, MODE_PLAIN, 4, ZOACT_DT_FP32, tm, p)
+                                : dispatch_fp16(ctx, MODE_PLAIN, 4, ZOACT_DT_FP32, tm, p);
 }
 
 }  // namespace zoact

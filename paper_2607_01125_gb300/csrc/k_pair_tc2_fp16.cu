@@ -4,42 +4,39 @@
 namespace zoact {
 namespace pairtc {
 
-// ---- CTA-pair kernel ----
 template <typename TO, int RT, int MODE>
-static int launch_two(Ctx* ctx, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& b2, const Params& p) {
+static int launch_two(Ctx* ctx, const TmaSet& tm, const Params& p) {
   auto kern = pair_tc2_kernel<TO, RT, MODE, 0>;
   ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES));
   const int clusters = p.num_tiles < ctx->sm_count / 2 ? p.num_tiles : ctx->sm_count / 2;
-  kern<<<2 * clusters, num_threads(false), SMEM2_BYTES, ctx->stream>>>(a, b, b2, p);
+  kern<<<2 * clusters, num_threads(false), SMEM2_BYTES, ctx->stream>>>(tm, p);
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
 }
 
 template <typename TO>
-static int by_rank_two(Ctx* ctx, int mode, int rt, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& b2,
-                       const Params& p) {
+static int by_rank_two(Ctx* ctx, int mode, int rt, const TmaSet& tm, const Params& p) {
   if (mode == MODE_GATED) {
     switch (rt) {
-      case 4: return launch_two<TO, 4, MODE_GATED>(ctx, a, b, b2, p);
-      case 8: return launch_two<TO, 8, MODE_GATED>(ctx, a, b, b2, p);
-      case 16: return launch_two<TO, 16, MODE_GATED>(ctx, a, b, b2, p);
+      case 4: return launch_two<TO, 4, MODE_GATED>(ctx, tm, p);
+      case 8: return launch_two<TO, 8, MODE_GATED>(ctx, tm, p);
+      case 16: return launch_two<TO, 16, MODE_GATED>(ctx, tm, p);
       default: return ZOACT_ERR_UNSUPPORTED;
     }
   }
   switch (rt) {
-    case 4: return launch_two<TO, 4, MODE_PAIR>(ctx, a, b, b2, p);
-    case 8: return launch_two<TO, 8, MODE_PAIR>(ctx, a, b, b2, p);
-    case 16: return launch_two<TO, 16, MODE_PAIR>(ctx, a, b, b2, p);
-    case 32: return launch_two<TO, 32, MODE_PAIR>(ctx, a, b, b2, p);
+    case 4: return launch_two<TO, 4, MODE_PAIR>(ctx, tm, p);
+    case 8: return launch_two<TO, 8, MODE_PAIR>(ctx, tm, p);
+    case 16: return launch_two<TO, 16, MODE_PAIR>(ctx, tm, p);
+    case 32: return launch_two<TO, 32, MODE_PAIR>(ctx, tm, p);
     default: return ZOACT_ERR_UNSUPPORTED;
   }
 }
 
-int dispatch2_fp16(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const CUtensorMap& b,
-                   const CUtensorMap& b2, const Params& p) {
-  if (ydtype == ZOACT_DT_FP32) return by_rank_two<float>(ctx, mode, rt, a, b, b2, p);
-  return by_rank_two<__half>(ctx, mode, rt, a, b, b2, p);
+int dispatch2_fp16(Ctx* ctx, int mode, int rt, int ydtype, const TmaSet& tm, const Params& p) {
+  if (ydtype == ZOACT_DT_FP32) return by_rank_two<float>(ctx, mode, rt, tm, p);
+  return by_rank_two<__half>(ctx, mode, rt, tm, p);
 }
 
 }  // namespace pairtc

@@ -9,7 +9,9 @@ static int launch_one(Ctx* ctx, const CUtensorMap& a, const Params& p) {
   auto kern = pair_tc_kernel<TO, RT, MODE, 1, true>;
   ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
   const int grid = p.num_tiles < ctx->sm_count ? p.num_tiles : ctx->sm_count;
-  kern<<<grid, num_threads(true), SMEM_BYTES, ctx->stream>>>(a, a, a, p);
+  TmaSet tm;
+  tm.a = tm.b = tm.b2 = tm.aa = tm.ba = tm.ba2 = a;   // only X comes by TMA
+  kern<<<grid, num_threads(true), SMEM_BYTES, ctx->stream>>>(tm, p);
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;

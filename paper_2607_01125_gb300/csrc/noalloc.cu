@@ -90,6 +90,7 @@ extern "C" int zoact_pair_forward_noalloc(const zoact_layer* L, const void* X, i
   c.stream = static_cast<cudaStream_t>(stream);
   c.d_status = reinterpret_cast<int*>(base + NOALLOC_FLOATS);
   c.d_tickets = nullptr;
+  c.may_allocate = false;
   ZOACT_CUDA_TRY(cudaMemsetAsync(c.d_status, 0, sizeof(int), c.stream));
 
   float* P = base;

@@ -110,9 +110,8 @@ __device__ __forceinline__ void commit2_own(uint32_t bar) {
 
 template <typename TO, int RT, int MODE, int AB_BF16>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(num_threads(false), 1)
-pair_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                const __grid_constant__ CUtensorMap tmB2, const Params prm) {
-  constexpr int CW = 16;
+pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
+  constexpr int CW = MODE == MODE_GATED ? 8 : 16;   // epilogue chunk width (gated: two accumulators)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   float* tbl = reinterpret_cast<float*>(smem + STAGES2 * STAGE2_BYTES);
@@ -136,9 +135,14 @@ pair_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
     tc::mbar_init(tc::smem_u32(&ss->drain), 1);
     ss->abort_flag = 0;
     tc::fence_mbar_init();
-    tc::prefetch_tmap(&tmA);
-    tc::prefetch_tmap(&tmB);
-    if (MODE == MODE_GATED) tc::prefetch_tmap(&tmB2);
+    tc::prefetch_tmap(&tm.a);
+    tc::prefetch_tmap(&tm.b);
+    if (MODE == MODE_GATED) tc::prefetch_tmap(&tm.b2);
+    if (prm.aug_kb > 0) {
+      tc::prefetch_tmap(&tm.aa);
+      tc::prefetch_tmap(&tm.ba);
+      if (MODE == MODE_GATED) tc::prefetch_tmap(&tm.ba2);
+    }
   }
   if (warp == 1) {
     tc2::tmem_alloc2(tc::smem_u32(&ss->tmem_base), TMEM_COLS);
@@ -151,6 +155,7 @@ pair_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
   const uint32_t tmem_base = ss->tmem_base;
 
   const int num_m = prm.num_m, num_n = prm.num_n, num_k = prm.num_k;
+  const int total_k = num_k + prm.aug_kb;   // main K-blocks, then the low-rank ones
   const int bn = MODE == MODE_GATED ? BN : prm.bn;
   const int bh = bn / 2;                  // W rows per CTA
   const uint32_t stage_tx = A_BYTES + bh * BK * 2;
@@ -165,17 +170,24 @@ pair_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
       for (int tile = cluster_id; tile < prm.num_tiles && ok; tile += n_clusters) {
         int m_blk, n_blk;
         tile_coords(tile, num_m, num_n, m_blk, n_blk);
-        for (int kb = 0; kb < num_k; ++kb) {
+        // low-rank K-blocks read the table of the tile's evaluation block (whole term on the tensor cores)
+        const int aug_row0 = prm.aug_mode == LOWRANK_ALL_ON_TC
+                                 ? (int)(((int64_t)m_blk * BM2 / prm.T) * prm.aug_block_rows) : 0;
+        for (int kb = 0; kb < total_k; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
           const uint32_t full_leader = tc2::map_to(tc::smem_u32(&ss->full[stage]), 0);
           tc2::arrive_expect_tx_cluster(full_leader, stage_tx);
           const uint32_t sa = tc::smem_u32(smem + stage * STAGE2_BYTES);
           const uint32_t sb = sa + A_BYTES;
-          tc2::tma_load_2d_pair(sa, &tmA, kb * BK, m_blk * BM2 + (int)rank * BM, full_leader);
+          const bool aug = kb >= num_k;
+          const int kx = (aug ? kb - num_k : kb) * BK;
+          const int yb = aug ? aug_row0 : 0;
+          tc2::tma_load_2d_pair(sa, aug ? &tm.aa : &tm.a, kx, m_blk * BM2 + (int)rank * BM, full_leader);
           if (MODE == MODE_GATED)
-            tc2::tma_load_2d_pair(sb, leader ? &tmB : &tmB2, kb * BK, n_blk * (BN / 2), full_leader);
+            tc2::tma_load_2d_pair(sb, aug ? (leader ? &tm.ba : &tm.ba2) : (leader ? &tm.b : &tm.b2), kx,
+                                  yb + n_blk * (BN / 2), full_leader);
           else
-            tc2::tma_load_2d_pair(sb, &tmB, kb * BK, n_blk * bn + (int)rank * bh, full_leader);
+            tc2::tma_load_2d_pair(sb, aug ? &tm.ba : &tm.b, kx, yb + n_blk * bn + (int)rank * bh, full_leader);
           if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
         }
       }
@@ -189,7 +201,8 @@ pair_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
   } else if (warp == 1) {
     // ---------------- MMA issuer (leader CTA) ----------------
     if (lane == 0 && leader) {
-      const uint32_t idesc = tc::idesc_f16(BM2, bn, AB_BF16);
+      const uint32_t idesc_main = tc::idesc_f16(BM2, bn, AB_BF16);
+      const uint32_t idesc_aug = tc::idesc_f16(BM2, bn, 1);   // low-rank K-blocks are bf16
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
@@ -201,11 +214,12 @@ pair_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__
         if (!tc::mbar_wait(tc::smem_u32(&ss->tmem_empty[buf]), acc_phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
         tc::tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
-        for (int kb = 0; kb < num_k; ++kb) {
+        for (int kb = 0; kb < total_k; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->full[stage]), phase, abort_flag, prm.status)) { ok = false; break; }
           tc::tc_fence_after();
           const uint32_t sa = tc::smem_u32(smem + stage * STAGE2_BYTES);
           const uint32_t sb = sa + A_BYTES;
+          const uint32_t idesc = kb < num_k ? idesc_main : idesc_aug;
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             tc2::mma2_f16(d_tmem, tc::sdesc_k_sw128(sa + k * 32), tc::sdesc_k_sw128(sb + k * 32), idesc,

@@ -29,6 +29,14 @@
 // the same 128 rows of W_up; the epilogue writes silu(gate) * up for 128 columns.
 // Plain mode (no P): the accumulator is stored as fp32 (used for X^T X).
 //
+// Low-rank term on the tensor cores (Params::aug_mode, operands from
+// k_aug.cu): after a tile's d_in / 64 K-blocks the producer loads aug_kb more,
+// from A_aug (16-bit split of P) and B_aug (16-bit split of C, or of C + c_b Z_b
+// for the tile's block), and the MMA adds them as bf16 products.  With the whole
+// term there (stacked rows whose tiles lie in one block) the epilogue only
+// converts and stores; with C p there the epilogue adds c_b Z_b p from Z tables,
+// once for both signs of a shared-input pair (y+- = acc +- eps Z p).
+//
 // INT4 weights (W4): the frozen W is symmetric INT4 in groups of 128 along d_in
 // with fp16 scales.  Four more warps (448 threads in all) dequantise it: per
 // K-block each thread loads 2 rows x 32 packed bytes and their scales with
@@ -72,6 +80,12 @@ static_assert(SMEM_BYTES <= 232448, "dynamic shared memory above the 227 KB a CT
 
 enum Mode { MODE_PAIR = 0, MODE_GATED = 1, MODE_PLAIN = 2 };
 
+// Tensor maps of one launch: X, W (gate), W up, and the low-rank K columns
+// A_aug, B_aug, B_aug up (unused ones are copies of a valid map).
+struct TmaSet {
+  CUtensorMap a, b, b2, aa, ba, ba2;
+};
+
 struct Params {
   const float* P;
   const float* C;
@@ -89,6 +103,9 @@ struct Params {
   uint64_t seed;
   uint32_t layer_id, layer_id2;
   int num_m, num_n, num_k, num_tiles;
+  int aug_mode;      // LowrankMode
+  int aug_kb;        // extra K-blocks per tile from A_aug / B_aug (0 with LOWRANK_EPILOGUE)
+  int64_t aug_block_rows;   // rows of one block's table in B_aug (LOWRANK_ALL_ON_TC)
   int64_t ldy;       // plain mode: row stride of D
   int vec_ok;        // C, C2, P, P2 and ldy allow 16-byte vector access
   int bn;            // N-tile width of pair / plain tiles (multiple of 32, <= BN); gated tiles use BN
@@ -125,9 +142,9 @@ __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int&
 // Fill the tables of one layer for output columns [col0, col0 + ncols) at two
 // evaluation points (tb1 may be null):
 //   tb0[j * stride + s] = C[col0 + s][j] + c0 Z(q0)[col0 + s][j]   (tb1: c1, q1)
-// zero where col0 + s >= d_out or j >= r.  A point with coefficient 0 draws no
-// Z; when both points use the same query (the two signs of the pair) Z is drawn
-// once.
+// (without the C term when Cg is null), zero where col0 + s >= d_out or j >= r.
+// A point with coefficient 0 draws no Z; when both points use the same query
+// (the two signs of the pair) Z is drawn once.
 template <int RT>
 __device__ __forceinline__ void build_tables(float* tb0, float* tb1, int stride, const float* __restrict__ Cg,
                                              uint32_t layer_id, int col0, int ncols, int d_out, int r,
@@ -145,7 +162,7 @@ __device__ __forceinline__ void build_tables(float* tb0, float* tb1, int stride,
       float4 c = make_float4(0.f, 0.f, 0.f, 0.f), z0 = c, z1 = c;
       if (s < valid_cols) {
         const int64_t e = (int64_t)(col0 + s) * RT + 4 * jg;
-        c = *reinterpret_cast<const float4*>(Cg + e);
+        if (Cg) c = *reinterpret_cast<const float4*>(Cg + e);
         if (z0_on) z0 = z_normals4(seed, layer_id, q0, (uint64_t)(e >> 2));
         if (z1_on) z1 = z1_same ? z0 : z_normals4(seed, layer_id, q1, (uint64_t)(e >> 2));
       }
@@ -170,7 +187,7 @@ __device__ __forceinline__ void build_tables(float* tb0, float* tb1, int stride,
     float v0 = 0.f, v1 = 0.f;
     if (s < valid_cols && j < r) {
       const int64_t e = (int64_t)(col0 + s) * r + j;
-      const float c = Cg[e];
+      const float c = Cg ? Cg[e] : 0.f;
       const uint64_t grp = (uint64_t)(e >> 2);
       const int w = (int)(e & 3);
       const float z0 = z0_on ? z_select(z_normals4(seed, layer_id, q0, grp), w) : 0.f;
@@ -205,6 +222,7 @@ __device__ __forceinline__ void lowrank_t(const float* tb, int stride, int c, co
   float2 acc[CW / 2];
 #pragma unroll
   for (int i = 0; i < CW / 2; ++i) acc[i] = make_float2(0.f, 0.f);
+  asm volatile("" ::: "memory");     // keep the table loads of one call together (register pressure)
 #pragma unroll
   for (int j = 0; j < RT; ++j) {
     const float4* t4 = reinterpret_cast<const float4*>(tb + j * stride + c);
@@ -352,11 +370,14 @@ __device__ __forceinline__ void load_p(float* p, const float* __restrict__ P, in
 
 // Pair / gated epilogue of one accumulator tile for this CTA's 128 rows
 // [row0, row0 + 128) (row m of thread (quad, lane)).  Column chunk by column
-// chunk, and two evaluation blocks per pass, it builds the tables C + c_b Z_b,
-// waits for the accumulator (first pass), adds the low-rank term, applies the
-// activation or the SiLU gate and stores.  Stacked rows use the block they
-// belong to; shared rows are written once per block.  Returns false when the
-// wait gave up.
+// chunk, and two evaluation blocks per pass, it builds the tables of the
+// low-rank terms the MMA did not add (C + c_b Z_b, or c_b Z_b when C p came
+// from the tensor cores), waits for the accumulator (first pass), adds them,
+// applies the activation or the SiLU gate and stores.  Stacked rows use the
+// block they belong to; shared rows are written once per block, and a pass
+// over the two signs of one query (coefficients +c, -c) builds one Z table and
+// forms acc +- c Z p.  With the whole term on the tensor cores it only converts
+// and stores.  Returns false when the wait gave up.
 template <typename TO, int RT, int MODE, int CW, typename SS>
 __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* tbl, int etid, int half,
                                               int64_t row0, int64_t m, bool row_ok, int n_blk, int bn, int buf,
@@ -368,6 +389,34 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
   static_assert((GATED ? 4 : 2) * TSZ <= TBL_FLOATS, "epilogue tables exceed their shared-memory region");
   const int r = prm.r;
   const int64_t T = prm.T;
+  TO* Y = static_cast<TO*>(prm.Y);
+  const int ncol_tile = GATED ? BN / 2 : bn;               // output columns of this tile
+  if (prm.aug_mode == LOWRANK_ALL_ON_TC) {
+    // stacked rows, the whole low-rank term in the accumulator
+    if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
+    const int cbeg = half * (ncol_tile / 2);
+    for (int c0 = cbeg; c0 < cbeg + ncol_tile / 2; c0 += CW) {
+      const int n = n_blk * ncol_tile + c0;
+      if (n >= prm.d_out) break;
+      const int nv = min(CW, prm.d_out - n);
+      if (GATED) {
+        float g[CW], u[CW], h[CW];
+        tmem_ldN<CW>(t_row + (uint32_t)c0, g);
+        tmem_ldN<CW>(t_row + (uint32_t)(BN / 2 + c0), u);
+#pragma unroll
+        for (int i = 0; i < CW; ++i) h[i] = silu_fast(g[i]) * u[i];
+        if (row_ok) storeN<TO, CW>(Y + m * prm.d_out + n, h, nv);
+      } else {
+        float acc[CW];
+        tmem_ldN<CW>(t_row + (uint32_t)c0, acc);
+#pragma unroll
+        for (int i = 0; i < CW; ++i) acc[i] = apply_act(acc[i], prm.act);
+        if (row_ok) storeN<TO, CW>(Y + m * prm.d_out + n, acc, nv);
+      }
+    }
+    return true;
+  }
+  const bool c_in_acc = prm.aug_mode == LOWRANK_C_ON_TC;
   float p[RT], p2[RT];
   const bool vec = prm.vec_ok != 0;
   load_p<RT>(p, prm.P, m, r, row_ok, vec);
@@ -382,8 +431,8 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
   if (b_last < b_first)    // no valid row in this CTA's part of the tile: only release the accumulator
     return epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid);
   const int my_b = (!prm.shared && row_ok) ? (int)(m / T) : -1;
-  TO* Y = static_cast<TO*>(prm.Y);
-  const int ncol_tile = GATED ? BN / 2 : bn;               // output columns of this tile
+  const float* Cg = c_in_acc ? nullptr : prm.C;
+  const float* Cg2 = c_in_acc ? nullptr : prm.C2;
   bool waited = false;
   for (int s0 = 0; s0 < ncol_tile; s0 += SLOTS) {
     const int cwid = min(SLOTS, ncol_tile - s0);          // a multiple of 32
@@ -391,18 +440,35 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
     for (int bp = b_first; bp <= b_last; bp += 2) {
       const bool two = bp + 1 <= b_last;
       const int b1 = two ? bp + 1 : bp;
+      // the two signs of one query on a shared input: one table Z, outputs acc +- c Z p
+      const bool mirror = c_in_acc && prm.shared && two && prm.qry[b1] == prm.qry[bp] &&
+                          prm.coef[b1] == -prm.coef[bp] && prm.coef[bp] != 0.f;
+      // a block needs a table unless its term is already in the accumulator (C p there, c_b = 0)
+      const bool need0 = !c_in_acc || prm.coef[bp] != 0.f;
+      const bool need1 = two && !mirror && (!c_in_acc || prm.coef[b1] != 0.f);
+      const float tc0 = mirror ? 1.f : prm.coef[bp];
       tc::named_bar_sync(1, EPI_THREADS);                 // previous pass's readers are done
-      build_tables<RT>(tbl, two ? tbl + TSZ : nullptr, STRIDE, prm.C, prm.layer_id, col0, cwid, prm.d_out, r,
-                       prm.seed, prm.coef[bp], prm.qry[bp], prm.coef[b1], prm.qry[b1], etid, vec);
-      if (GATED)
-        build_tables<RT>(tbl + 2 * TSZ, two ? tbl + 3 * TSZ : nullptr, STRIDE, prm.C2, prm.layer_id2, col0, cwid, prm.d_out, r,
-                         prm.seed, prm.coef[bp], prm.qry[bp], prm.coef[b1], prm.qry[b1], etid, vec);
+      if (need0 || need1) {
+        // table slot 0 holds block bp (or block b1 alone when bp needs none)
+        float* t0 = tbl;
+        float* t1 = (need0 && need1) ? tbl + TSZ : nullptr;
+        const float c0v = need0 ? tc0 : prm.coef[b1];
+        const uint64_t q0v = need0 ? prm.qry[bp] : prm.qry[b1];
+        build_tables<RT>(t0, t1, STRIDE, Cg, prm.layer_id, col0, cwid, prm.d_out, r, prm.seed, c0v, q0v,
+                         prm.coef[b1], prm.qry[b1], etid, vec);
+        if (GATED)
+          build_tables<RT>(t0 + 2 * TSZ, t1 ? t1 + 2 * TSZ : nullptr, STRIDE, Cg2, prm.layer_id2, col0, cwid,
+                           prm.d_out, r, prm.seed, c0v, q0v, prm.coef[b1], prm.qry[b1], etid, vec);
+      }
       tc::named_bar_sync(1, EPI_THREADS);
       if (!waited) {
         if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
         waited = true;
       }
-      const int sel = my_b - bp;                          // stacked: my table in this pass
+      // table index of block bp + t (-1: no term to add)
+      const int tix0 = need0 ? 0 : -1;
+      const int tix1 = need1 ? (need0 ? 1 : 0) : -1;
+      const int sel = my_b - bp;                          // stacked: my block in this pass
       const bool active = prm.shared ? row_ok : (sel == 0 || (sel == 1 && two));
       if (!prm.shared && !__any_sync(0xffffffffu, active)) continue;   // no row of this warp in the pass
       const int nt = prm.shared ? (two ? 2 : 1) : 1;
@@ -416,29 +482,71 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
           tmem_ldN<CW>(t_row + (uint32_t)c0, g);
           tmem_ldN<CW>(t_row + (uint32_t)(BN / 2 + c0), u);
           if (active) {
-            for (int t = 0; t < nt; ++t) {
-              const int ts = prm.shared ? t : sel;
-              float sg[CW], su[CW], h[CW];
-              lowrank_t<RT, CW>(tbl + ts * TSZ, STRIDE, c0 - s0, p, sg);
-              lowrank_t<RT, CW>(tbl + (2 + ts) * TSZ, STRIDE, c0 - s0, p2, su);
+            if (mirror) {
+              float sg[CW], su[CW];
+              lowrank_t<RT, CW>(tbl, STRIDE, c0 - s0, p, sg);
+              lowrank_t<RT, CW>(tbl + 2 * TSZ, STRIDE, c0 - s0, p2, su);
+              const float cz = prm.coef[bp];
 #pragma unroll
-              for (int i = 0; i < CW; ++i) h[i] = silu_fast(g[i] + sg[i]) * (u[i] + su[i]);
-              const int64_t row = prm.shared ? (int64_t)(bp + t) * T + m : m;
-              storeN<TO, CW>(Y + row * prm.d_out + n, h, nv);
+              for (int i = 0; i < CW; ++i) {       // in place: sg <- h(+c), su <- h(-c)
+                const float hp = silu_fast(fmaf(cz, sg[i], g[i])) * fmaf(cz, su[i], u[i]);
+                const float hm = silu_fast(fmaf(-cz, sg[i], g[i])) * fmaf(-cz, su[i], u[i]);
+                sg[i] = hp;
+                su[i] = hm;
+              }
+              storeN<TO, CW>(Y + ((int64_t)bp * T + m) * prm.d_out + n, sg, nv);
+              storeN<TO, CW>(Y + ((int64_t)b1 * T + m) * prm.d_out + n, su, nv);
+            } else {
+#pragma unroll 1
+              for (int t = 0; t < nt; ++t) {
+                const int tix = (prm.shared ? t : sel) == 0 ? tix0 : tix1;
+                float hg[CW], hu[CW];
+                if (tix >= 0) {
+                  lowrank_t<RT, CW>(tbl + tix * TSZ, STRIDE, c0 - s0, p, hg);
+#pragma unroll
+                  for (int i = 0; i < CW; ++i) hg[i] += g[i];
+                  lowrank_t<RT, CW>(tbl + (2 + tix) * TSZ, STRIDE, c0 - s0, p2, hu);
+#pragma unroll
+                  for (int i = 0; i < CW; ++i) hu[i] = silu_fast(hg[i]) * (hu[i] + u[i]);
+                } else {
+#pragma unroll
+                  for (int i = 0; i < CW; ++i) hu[i] = silu_fast(g[i]) * u[i];
+                }
+                const int64_t row = prm.shared ? (int64_t)(bp + t) * T + m : m;
+                storeN<TO, CW>(Y + row * prm.d_out + n, hu, nv);
+              }
             }
           }
         } else {
           float acc[CW];
           tmem_ldN<CW>(t_row + (uint32_t)c0, acc);
           if (active) {
-            for (int t = 0; t < nt; ++t) {
-              const int ts = prm.shared ? t : sel;
+            if (mirror) {
               float sl[CW], y[CW];
-              lowrank_t<RT, CW>(tbl + ts * TSZ, STRIDE, c0 - s0, p, sl);
+              lowrank_t<RT, CW>(tbl, STRIDE, c0 - s0, p, sl);
+              const float cz = prm.coef[bp];
 #pragma unroll
-              for (int i = 0; i < CW; ++i) y[i] = apply_act(acc[i] + sl[i], prm.act);
-              const int64_t row = prm.shared ? (int64_t)(bp + t) * T + m : m;
-              storeN<TO, CW>(Y + row * prm.d_out + n, y, nv);
+              for (int i = 0; i < CW; ++i) y[i] = apply_act(fmaf(cz, sl[i], acc[i]), prm.act);
+              storeN<TO, CW>(Y + ((int64_t)bp * T + m) * prm.d_out + n, y, nv);
+#pragma unroll
+              for (int i = 0; i < CW; ++i) y[i] = apply_act(fmaf(-cz, sl[i], acc[i]), prm.act);
+              storeN<TO, CW>(Y + ((int64_t)b1 * T + m) * prm.d_out + n, y, nv);
+            } else {
+#pragma unroll 1
+              for (int t = 0; t < nt; ++t) {
+                const int tix = (prm.shared ? t : sel) == 0 ? tix0 : tix1;
+                float sl[CW], y[CW];
+                if (tix >= 0) {
+                  lowrank_t<RT, CW>(tbl + tix * TSZ, STRIDE, c0 - s0, p, sl);
+                } else {
+#pragma unroll
+                  for (int i = 0; i < CW; ++i) sl[i] = 0.f;
+                }
+#pragma unroll
+                for (int i = 0; i < CW; ++i) y[i] = apply_act(acc[i] + sl[i], prm.act);
+                const int64_t row = prm.shared ? (int64_t)(bp + t) * T + m : m;
+                storeN<TO, CW>(Y + row * prm.d_out + n, y, nv);
+              }
             }
           }
         }
@@ -450,9 +558,10 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
 
 template <typename TO, int RT, int MODE, int AB_BF16, bool W4>
 __global__ void __launch_bounds__(num_threads(W4), 1)
-pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-               const __grid_constant__ CUtensorMap tmB2, const Params prm) {
-  constexpr int CW = W4 ? 8 : 16;                   // epilogue chunk width (columns per tcgen05.ld)
+pair_tc_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
+  // epilogue chunk width (columns per tcgen05.ld): 8 where the registers are scarce (INT4's 14 warps,
+  // the gated pair's two accumulators and two projections)
+  constexpr int CW = (W4 || MODE == MODE_GATED) ? 8 : 16;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   float* tbl = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES);
@@ -475,9 +584,14 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     tc::mbar_init(tc::smem_u32(&ss->drain), 1);
     ss->abort_flag = 0;
     tc::fence_mbar_init();
-    tc::prefetch_tmap(&tmA);
-    if (!W4) tc::prefetch_tmap(&tmB);
-    if (!W4 && MODE == MODE_GATED) tc::prefetch_tmap(&tmB2);
+    tc::prefetch_tmap(&tm.a);
+    if (!W4) tc::prefetch_tmap(&tm.b);
+    if (!W4 && MODE == MODE_GATED) tc::prefetch_tmap(&tm.b2);
+    if (prm.aug_kb > 0) {
+      tc::prefetch_tmap(&tm.aa);
+      tc::prefetch_tmap(&tm.ba);
+      if (MODE == MODE_GATED) tc::prefetch_tmap(&tm.ba2);
+    }
   }
   if (warp == 1) {
     tc::tmem_alloc(tc::smem_u32(&ss->tmem_base), TMEM_COLS);
@@ -489,6 +603,7 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const uint32_t tmem_base = ss->tmem_base;
 
   const int num_m = prm.num_m, num_n = prm.num_n, num_k = prm.num_k;
+  const int total_k = num_k + (W4 ? 0 : prm.aug_kb);   // main K-blocks, then the low-rank ones
   const int bn = MODE == MODE_GATED ? BN : prm.bn;  // this launch's N-tile width
 
   if (warp == 0) {
@@ -501,20 +616,26 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       for (int tile = blockIdx.x; tile < prm.num_tiles && ok; tile += gridDim.x) {
         int m_blk, n_blk;
         tile_coords(tile, num_m, num_n, m_blk, n_blk);
-        for (int kb = 0; kb < num_k; ++kb) {
+        // low-rank K-blocks read the table of the tile's evaluation block (whole term on the tensor cores)
+        const int aug_row0 = prm.aug_mode == LOWRANK_ALL_ON_TC
+                                 ? (int)(((int64_t)m_blk * BM / prm.T) * prm.aug_block_rows) : 0;
+        for (int kb = 0; kb < total_k; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
           const uint32_t full = tc::smem_u32(&ss->full[stage]);
           tc::mbar_arrive_expect_tx(full, W4 ? A_BYTES : (MODE == MODE_GATED ? STAGE_BYTES : A_BYTES + bn * BK * 2));
           const uint32_t sa = tc::smem_u32(smem + stage * STAGE_BYTES);
           const uint32_t sb = sa + A_BYTES;
-          tc::tma_load_2d(sa, &tmA, kb * BK, m_blk * BM, full);
+          const bool aug = kb >= num_k;
+          const int kx = (aug ? kb - num_k : kb) * BK;
+          const int yb = aug ? aug_row0 : 0;
+          tc::tma_load_2d(sa, aug ? &tm.aa : &tm.a, kx, m_blk * BM, full);
           if (W4) {
             // B arrives from the dequantising warps
           } else if (MODE == MODE_GATED) {
-            tc::tma_load_2d(sb, &tmB, kb * BK, n_blk * (BN / 2), full);
-            tc::tma_load_2d(sb + B_BYTES / 2, &tmB2, kb * BK, n_blk * (BN / 2), full);
+            tc::tma_load_2d(sb, aug ? &tm.ba : &tm.b, kx, yb + n_blk * (BN / 2), full);
+            tc::tma_load_2d(sb + B_BYTES / 2, aug ? &tm.ba2 : &tm.b2, kx, yb + n_blk * (BN / 2), full);
           } else {
-            tc::tma_load_2d(sb, &tmB, kb * BK, n_blk * bn, full);
+            tc::tma_load_2d(sb, aug ? &tm.ba : &tm.b, kx, yb + n_blk * bn, full);
           }
           issued_mask |= 1u << stage;
           issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
@@ -532,6 +653,7 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       const uint32_t IDESC = tc::idesc_f16(BM, bn, AB_BF16);
+      const uint32_t IDESC_AUG = tc::idesc_f16(BM, bn, 1);   // low-rank K-blocks are bf16
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
@@ -543,16 +665,17 @@ pair_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         if (!tc::mbar_wait(tc::smem_u32(&ss->tmem_empty[buf]), acc_phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
         tc::tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
-        for (int kb = 0; kb < num_k; ++kb) {
+        for (int kb = 0; kb < total_k; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->full[stage]), phase, abort_flag, prm.status)) { ok = false; break; }
           tc::tc_fence_after();
           const uint32_t sa = tc::smem_u32(smem + stage * STAGE_BYTES);
           const uint32_t sb = sa + A_BYTES;
+          const uint32_t idesc = kb < num_k ? IDESC : IDESC_AUG;
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             const uint64_t ad = tc::sdesc_k_sw128(sa + k * 32);
             const uint64_t bd = tc::sdesc_k_sw128(sb + k * 32);
-            tc::mma_f16(d_tmem, ad, bd, IDESC, (kb | k) != 0 ? 1u : 0u);
+            tc::mma_f16(d_tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
           }
           tc::mma_commit(tc::smem_u32(&ss->empty[stage]));   // frees the stage when these MMAs finish
           issued_any = true;

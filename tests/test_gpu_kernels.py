@@ -5,7 +5,10 @@ Tolerances (written per test):
   * Philox words and index bookkeeping: bit-exact.
   * fp32 normals: |dz| <= 1e-6 (1 + |z|)  (fp32 logf/sqrtf/sincospif vs fp64 libm).
   * fp32 arithmetic paths: <= 1e-4 of the output scale, and a per-element bound
-    from the fp32 accumulation error (c * eps32 * sum |terms|).
+    from the fp32 accumulation error (c * eps32 * sum |terms|).  Where the
+    low-rank term runs on the tensor cores as three bf16 products of 16-bit
+    splits, it carries at most 2^-15 sum_j |P_j| |T_j| more (the dropped
+    P_lo T_lo and the rounding of the lo parts); the bound adds 2^-14 of it.
   * 16-bit outputs: the bf16/fp16 rounding of the output (2^-8 / 2^-11 relative)
     on top of the fp32 bound; the bar is 2e-2 relative.
 """
@@ -79,8 +82,14 @@ def _oracle_pair(X, W, U, C, eps, T, shared, seed, layer_id, query, d_out, r):
     Xn, Wn, Un = np64(X), np64(W), np64(U)
     if shared:
         Xn = np.concatenate([Xn, Xn])
-    absb = np.abs(Xn) @ np.abs(Wn).T + (np.abs(Xn @ Un)) @ (np.abs(np64(C).reshape(d_out, r)) + abs(eps) * np.abs(Zm)).T
-    return Y, absb
+    lrabs = (np.abs(Xn @ Un)) @ (np.abs(np64(C).reshape(d_out, r)) + abs(eps) * np.abs(Zm)).T
+    absb = np.abs(Xn) @ np.abs(Wn).T + lrabs
+    return Y, absb, lrabs
+
+
+def _bound(d_in, absb, lrabs):
+    """fp32 accumulation bound plus the 16-bit split of the low-rank term."""
+    return 8 * np.sqrt(d_in) * 2.0 ** -24 * absb + 2.0 ** -14 * lrabs + 1e-6
 
 
 @pytest.mark.parametrize("d_in,d_out,r,T,shared,dt", [
@@ -100,10 +109,49 @@ def test_pair_forward_fp32_out(ctx, d_in, d_out, r, T, shared, dt):
     L = zo.make_layer(W, U, C, layer_id)
     zo.zoact_pair_forward(ctx, L, X, T, shared, eps, seed, query, Y)
     torch.cuda.synchronize()
-    ref, absb = _oracle_pair(X, W, U, C, eps, T, shared, seed, layer_id, query, d_out, r)
+    ref, absb, lrabs = _oracle_pair(X, W, U, C, eps, T, shared, seed, layer_id, query, d_out, r)
     err = np.abs(np64(Y) - ref)
-    assert np.all(err <= 8 * np.sqrt(d_in) * 2.0 ** -24 * absb + 1e-6), err.max()
+    assert np.all(err <= _bound(d_in, absb, lrabs)), err.max()
     assert err.max() <= 1e-4 * np.abs(ref).max()
+
+
+@pytest.mark.parametrize("T,shared,lowrank,kernel", [
+    (256, False, "auto", "auto"),        # stacked, tiles inside one block: whole low-rank term on the tensor cores
+    (256, False, "epilogue", "auto"),    # the same in fp32 epilogue tables
+    (200, False, "auto", "auto"),        # stacked, tiles across the sign boundary: C p on the tensor cores
+    (300, True, "auto", "auto"),         # shared input: C p on the tensor cores, +-eps Z p in the epilogue
+    (300, True, "epilogue", "auto"),
+    (128, False, "auto", "1cta"),        # one-CTA kernel with the whole term on the tensor cores
+    (100, False, "auto", "1cta"),
+])
+@pytest.mark.parametrize("gated", [False, True])
+def test_pair_forward_lowrank_modes(ctx, monkeypatch, T, shared, lowrank, kernel, gated):
+    # every placement of the low-rank term gives the oracle's output within the fp32 bound
+    if lowrank != "auto":
+        monkeypatch.setenv("ZOACT_LOWRANK", lowrank)
+    if kernel != "auto":
+        monkeypatch.setenv("ZOACT_PAIR_KERNEL", kernel)
+    d_in, d_out, r, eps, seed, query = 1024, 392, 16, 0.5, 19, 6
+    X, W, U, C = _pair_case(d_in, d_out, r, T, shared, torch.bfloat16, eps, 0.3, seed=60)
+    Y = torch.empty(2 * T, d_out, dtype=torch.float32, device=DEV)
+    if gated:
+        W2 = normal((d_out, d_in), 70, DEV, std=d_in ** -0.5, dtype=torch.bfloat16)
+        U2 = normal((d_in, r), 71, DEV) / np.sqrt(d_in)
+        C2 = normal((d_out * r,), 72, DEV, std=0.3)
+        zo.zoact_pair_forward_gated(ctx, zo.make_layer(W, U, C, 3), zo.make_layer(W2, U2, C2, 4), X, T, shared,
+                                    eps, seed, query, Y)
+        torch.cuda.synchronize()
+        g, _, _ = _oracle_pair(X, W, U, C, eps, T, shared, seed, 3, query, d_out, r)
+        u, _, _ = _oracle_pair(X, W2, U2, C2, eps, T, shared, seed, 4, query, d_out, r)
+        ref = layers.silu(g) * u
+        assert np.abs(np64(Y) - ref).max() <= 1e-4 * np.abs(ref).max()
+    else:
+        zo.zoact_pair_forward(ctx, zo.make_layer(W, U, C, 3), X, T, shared, eps, seed, query, Y)
+        torch.cuda.synchronize()
+        ref, absb, lrabs = _oracle_pair(X, W, U, C, eps, T, shared, seed, 3, query, d_out, r)
+        err = np.abs(np64(Y) - ref)
+        assert np.all(err <= _bound(d_in, absb, lrabs)), err.max()
+        assert err.max() <= 1e-4 * np.abs(ref).max()
 
 
 @pytest.mark.parametrize("d_in,d_out,r,T,shared,dt,act", [
@@ -119,11 +167,11 @@ def test_pair_forward_16bit_out_and_acts(ctx, d_in, d_out, r, T, shared, dt, act
     L = zo.make_layer(W, U, C, layer_id)
     zo.zoact_pair_forward(ctx, L, X, T, shared, eps, seed, query, Y, act=act)
     torch.cuda.synchronize()
-    ref, absb = _oracle_pair(X, W, U, C, eps, T, shared, seed, layer_id, query, d_out, r)
+    ref, absb, lrabs = _oracle_pair(X, W, U, C, eps, T, shared, seed, layer_id, query, d_out, r)
     ref = {zo.ACT_NONE: lambda y: y, zo.ACT_RELU: layers.relu, zo.ACT_GELU: layers.gelu_erf}[act](ref)
     rel = {torch.bfloat16: 2.0 ** -8, torch.float16: 2.0 ** -11, torch.float32: 2.0 ** -23}[dt]
     err = np.abs(np64(Y) - ref)
-    assert np.all(err <= rel * np.abs(ref) + 8 * np.sqrt(d_in) * 2.0 ** -24 * absb + 1e-6)
+    assert np.all(err <= rel * np.abs(ref) + _bound(d_in, absb, lrabs))
     assert err.max() <= 2e-2 * np.abs(ref).max()
 
 
@@ -204,8 +252,8 @@ def test_pair_forward_gated(ctx, T, shared, dt):
     zo.zoact_pair_forward_gated(ctx, zo.make_layer(Wg, Ug, Cg, 0), zo.make_layer(Wu, Uu, Cu, 1), X, T, shared,
                                 eps, seed, query, H)
     torch.cuda.synchronize()
-    g, _ = _oracle_pair(X, Wg, Ug, Cg, eps, T, shared, seed, 0, query, d_out, r)
-    u, _ = _oracle_pair(X, Wu, Uu, Cu, eps, T, shared, seed, 1, query, d_out, r)
+    g, _, _ = _oracle_pair(X, Wg, Ug, Cg, eps, T, shared, seed, 0, query, d_out, r)
+    u, _, _ = _oracle_pair(X, Wu, Uu, Cu, eps, T, shared, seed, 1, query, d_out, r)
     ref = layers.silu(g) * u
     assert np.abs(np64(H) - ref).max() <= 1e-4 * np.abs(ref).max()
 
@@ -238,7 +286,7 @@ def test_pair_forward_int4(ctx, d_in, d_out, r, T, shared):
     absw = np.abs(Xs) @ np.abs(Wd).T
     absl = np.abs(Xs @ np64(U)) @ (np.abs(np64(C).reshape(d_out, r)) + eps * np.abs(Zm)).T
     err = np.abs(np64(Y) - ref)
-    assert np.all(err <= 2.0 ** -8 * absw + 8 * np.sqrt(d_in) * 2.0 ** -24 * (absw + absl) + 1e-6), err.max()
+    assert np.all(err <= 2.0 ** -8 * absw + _bound(d_in, absw + absl, absl)), err.max()
     assert err.max() <= 2e-2 * np.abs(ref).max()
 
 
