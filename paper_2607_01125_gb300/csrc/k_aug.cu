@@ -27,77 +27,79 @@ struct AugBlocks {
   uint64_t qry[ZOACT_MAX_EVAL_BLOCKS];
 };
 
-// part index of K column k of one layer's aug columns: 0 -> hi, 1 -> hi (A) / lo (B), 2 -> lo (A) / hi (B)
+// v = hi + lo (+ what bf16 cannot hold): hi = bf16(v), lo = bf16(v - hi); v - hi is exact in fp32.
 __device__ __forceinline__ void split16(float v, __nv_bfloat16& hi, __nv_bfloat16& lo) {
   hi = __float2bfloat16_rn(v);
   lo = __float2bfloat16_rn(v - __bfloat162float(hi));
 }
 
-__device__ __forceinline__ __nv_bfloat16 a_part(float v, int part) {
-  __nv_bfloat16 hi, lo;
-  split16(v, hi, lo);
-  return part == 2 ? lo : hi;
-}
-__device__ __forceinline__ __nv_bfloat16 b_part(float v, int part) {
-  __nv_bfloat16 hi, lo;
-  split16(v, hi, lo);
-  return part == 1 ? lo : hi;
+__device__ __forceinline__ uint32_t pack_bf16x2(__nv_bfloat16 a, __nv_bfloat16 b) {
+  return (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(b) << 16);
 }
 
-// One thread writes 8 consecutive bf16 of one aug row (a 16-byte store).
-// Work items: [0, nA) rows of A_aug, then [nA, nA + nB) rows of B_aug, then B_aug2.
+// One warp per output row: rows [0, nA) of A_aug, then the nB rows of B_aug
+// (block b, column n), then those of B_aug2.  Lane j < r holds the row's source
+// value j (and of the second projection, distinct gated A rows only); the warp
+// writes the row as bf16 pairs, each lane fetching its K columns' source values
+// by shuffle and splitting them into hi/lo.
 __global__ void __launch_bounds__(256)
 aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const float* __restrict__ C,
                 const float* __restrict__ C2, __nv_bfloat16* __restrict__ A, __nv_bfloat16* __restrict__ B,
                 __nv_bfloat16* __restrict__ B2, int64_t rows, int d_out, int r, int ka, int distinct, int full,
                 int nb, const __grid_constant__ AugBlocks blk, uint64_t seed, uint32_t lid, uint32_t lid2) {
+  const int lane = threadIdx.x & 31;
   const int ka_tot = distinct ? 2 * ka : ka;
-  const int cpr = ka_tot / 8;                         // 16-byte chunks per row
-  const int64_t nA = rows * cpr;
   const int nbB = full ? nb : 1;
-  const int64_t nB = (int64_t)nbB * d_out * cpr;
+  const int64_t nA = rows;
+  const int64_t nB = (int64_t)nbB * d_out;
   const int64_t total = nA + (B2 ? 2 * nB : nB);
-  for (int64_t it = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; it < total; it += (int64_t)gridDim.x * blockDim.x) {
-    alignas(16) __nv_bfloat16 out[8];
-    if (it < nA) {
-      const int64_t t = it / cpr;
-      const int k0 = (int)(it % cpr) * 8;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int k = k0 + i;
-        const int half = k / ka, kk = k % ka;          // half 1: the up projection (distinct only)
-        const int part = kk / r, j = kk % r;
-        const float* src = half ? P2 : P;
-        out[i] = part < 3 ? a_part(src[t * r + j], part) : __float2bfloat16_rn(0.f);
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; w < total; w += nwarps) {
+    const bool is_a = w < nA;
+    float v0 = 0.f, v1 = 0.f;                       // this lane's source value (v1: second half, distinct A)
+    bool up = false;
+    int64_t orow;
+    if (is_a) {
+      orow = w;
+      if (lane < r) {
+        v0 = P[w * r + lane];
+        if (distinct) v1 = P2[w * r + lane];
       }
-      *reinterpret_cast<uint4*>(A + t * ka_tot + k0) = *reinterpret_cast<const uint4*>(out);
     } else {
-      const int64_t ib = it - nA;
-      const bool up = ib >= nB;
-      const int64_t jb = up ? ib - nB : ib;
-      const int64_t row = jb / cpr;                     // b * d_out + n
-      const int k0 = (int)(jb % cpr) * 8;
-      const int b = (int)(row / d_out), n = (int)(row % d_out);
-      const float* Cs = up ? C2 : C;
-      const uint32_t layer = up ? lid2 : lid;
-      const float cb = full ? blk.coef[b] : 0.f;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int k = k0 + i;
-        const int half = k / ka, kk = k % ka;
-        const int part = kk / r, j = kk % r;
-        // distinct projections: gate rows use the first half, up rows the second
-        const bool live = part < 3 && (!distinct || half == (up ? 1 : 0));
-        float v = 0.f;
-        if (live) {
-          const int64_t e = (int64_t)n * r + j;
-          v = Cs[e];
-          if (cb != 0.f) v = fmaf(cb, z_select(z_normals4(seed, layer, blk.qry[b], (uint64_t)(e >> 2)), (int)(e & 3)), v);
-        }
-        out[i] = live ? b_part(v, part) : __float2bfloat16_rn(0.f);
+      const int64_t ib = w - nA;
+      up = ib >= nB;
+      orow = up ? ib - nB : ib;                      // b * d_out + n
+      const int b = (int)(orow / d_out), n = (int)(orow - (int64_t)b * d_out);
+      if (lane < r) {
+        const int64_t e = (int64_t)n * r + lane;
+        v0 = (up ? C2 : C)[e];
+        const float cb = full ? blk.coef[b] : 0.f;
+        if (cb != 0.f)
+          v0 = fmaf(cb, z_select(z_normals4(seed, up ? lid2 : lid, blk.qry[b], (uint64_t)(e >> 2)), (int)(e & 3)), v0);
       }
-      __nv_bfloat16* dst = up ? B2 : B;
-      *reinterpret_cast<uint4*>(dst + row * ka_tot + k0) = *reinterpret_cast<const uint4*>(out);
+    }
+    __nv_bfloat16* dst = is_a ? A : (up ? B2 : B);
+    uint32_t* drow = reinterpret_cast<uint32_t*>(dst + orow * ka_tot);
+    for (int wd = lane; wd < ka_tot / 2; wd += 32) {
+      __nv_bfloat16 o[2];
+#pragma unroll
+      for (int e2 = 0; e2 < 2; ++e2) {
+        const int k = 2 * wd + e2;
+        const int half = k >= ka ? 1 : 0, kk = k - half * ka;
+        const int part = kk / r, j = kk - part * r;
+        // A: [hi | hi | lo], B: [hi | lo | hi]
+        const bool want_lo = is_a ? part == 2 : part == 1;
+        const bool second = is_a && half == 1;       // distinct A: the up projection's parts
+        // every lane fetches its column's source value and splits it itself
+        const float a0 = __shfl_sync(0xffffffffu, v0, j & 31);
+        const float a1 = __shfl_sync(0xffffffffu, v1, j & 31);
+        __nv_bfloat16 hi, lo;
+        split16(second ? a1 : a0, hi, lo);
+        // distinct gated B: gate rows fill the first half, up rows the second
+        const bool live = part < 3 && (is_a || !distinct || half == (up ? 1 : 0));
+        o[e2] = live ? (want_lo ? lo : hi) : __float2bfloat16_rn(0.f);
+      }
+      drow[wd] = pack_bf16x2(o[0], o[1]);
     }
   }
 }
@@ -110,10 +112,10 @@ int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct,
   for (int b = 0; b < a.nb; ++b) { blk.coef[b] = a.coef[b]; blk.qry[b] = a.qry[b]; }
   const int full = mode == LOWRANK_ALL_ON_TC;
   const int ka_tot = distinct ? 2 * ka : ka;
-  const int64_t cpr = ka_tot / 8;
+  (void)ka_tot;
   const int64_t nbB = full ? a.nb : 1;
-  const int64_t total = a.rows * cpr + (B_aug2 ? 2 : 1) * nbB * a.d_out * cpr;
-  int64_t grid = (total + 255) / 256;
+  const int64_t total_rows = a.rows + (B_aug2 ? 2 : 1) * nbB * a.d_out;   // one warp per row, 8 per block
+  int64_t grid = (total_rows + 7) / 8;
   const int64_t cap = (int64_t)ctx->sm_count * 16;
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;

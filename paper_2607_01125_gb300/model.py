@@ -256,16 +256,18 @@ def calibrate_bases(ctx, step_cal, x_cal, r, oversample=16, n_iter=8, seed=0):
     and each layer's basis U = top-r right singular vectors of its input, written in place.
 
     step_cal is a ZOStep over the same AdaptedLinear objects with T = len(x_cal); layers whose
-    inputs are the same tensor (q/k/v, gate/up) share one basis computation.
+    inputs are the same tensor (q/k/v, gate/up) have the same basis by definition: they get one
+    basis computation and share its tensor, so later steps project their common input once (and a
+    gated pair sees one projection).  ZOSteps built after this call bind the shared tensors.
     """
     last = {}
 
     def cap(name, X):
-        # consecutive layers on the same input tensor (q/k/v, gate/up) share the basis
         lin = step_cal.by_name[name]
         key = (X.data_ptr(), X.shape[0])
         if last.get("key") == key:
-            lin.U.copy_(last["U"])
+            lin.U = last["U"]
+            lin.bind(step_cal.C)
             return
         Z.zoact_basis_init(ctx, X.contiguous(), r, lin.U, oversample=oversample, n_iter=n_iter,
                            seed=seed + lin.layer_id)
