@@ -32,6 +32,7 @@ enum ScratchSlot {
   SLOT_WDQ1,         // second copy (gated up weight)
   SLOT_AUG_A,        // 16-bit split of the projection P (extra K columns of the tensor-core pair forward)
   SLOT_AUG_B,        // 16-bit split of C (+ c_b Z_b) for those K columns (gate and up)
+  SLOT_AUG_Z,        // Z of each query, transposed, for the epilogue (C on the tensor cores)
   SLOT_COUNT
 };
 
@@ -141,8 +142,9 @@ enum LowrankMode { LOWRANK_EPILOGUE = 0, LOWRANK_C_ON_TC = 1, LOWRANK_ALL_ON_TC 
 inline int aug_cols(int r) { return (3 * r + 63) / 64 * 64; }
 // Writes A_aug [rows, ka_tot] and B_aug / B_aug2 [nbB * d_out, ka_tot] (bf16) for one pair forward.
 // distinct: gate and up have their own projections (A_aug holds both, B_aug zero-pads the other half).
+// Zt / Zt2 (optional): Z of the nzq queries zq, transposed, [nzq][r][d_out] fp32 each.
 int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct, void* A_aug, void* B_aug,
-                    void* B_aug2);
+                    void* B_aug2, float* Zt, float* Zt2, const uint64_t* zq, int nzq);
 int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int M, int N, int K,
                           float* D);
 

@@ -14,7 +14,10 @@
 // holds both ([gate parts | up parts]) and each B_aug zero-fills the other half.
 // B_aug holds one table per evaluation block when the whole term goes to the
 // tensor cores (LOWRANK_ALL_ON_TC: T = C + c_b Z_b, Z_b from the same Philox
-// stream as every other kernel), and the single table T = C otherwise.
+// stream as every other kernel), and the single table T = C otherwise.  With C
+// on the tensor cores the epilogue still adds c_b Z_b p: for it this kernel
+// also writes Z of every distinct query transposed, Zt[q][j][n] (fp32), so the
+// pair kernel copies its tile's columns instead of regenerating them per tile.
 // Purely memory-bound and small (rows x r and d_out x r inputs).
 #include "internal.h"
 #include "philox.cuh"
@@ -25,6 +28,8 @@ namespace {
 struct AugBlocks {
   float coef[ZOACT_MAX_EVAL_BLOCKS];
   uint64_t qry[ZOACT_MAX_EVAL_BLOCKS];
+  uint64_t zq[ZOACT_MAX_EVAL_BLOCKS];   // distinct queries whose Z is written transposed
+  int nzq;
 };
 
 // v = hi + lo (+ what bf16 cannot hold): hi = bf16(v), lo = bf16(v - hi); v - hi is exact in fp32.
@@ -46,7 +51,8 @@ __global__ void __launch_bounds__(256)
 aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const float* __restrict__ C,
                 const float* __restrict__ C2, __nv_bfloat16* __restrict__ A, __nv_bfloat16* __restrict__ B,
                 __nv_bfloat16* __restrict__ B2, int64_t rows, int d_out, int r, int ka, int distinct, int full,
-                int nb, const __grid_constant__ AugBlocks blk, uint64_t seed, uint32_t lid, uint32_t lid2) {
+                int nb, const __grid_constant__ AugBlocks blk, uint64_t seed, uint32_t lid, uint32_t lid2,
+                float* __restrict__ Zt, float* __restrict__ Zt2) {
   const int lane = threadIdx.x & 31;
   const int ka_tot = distinct ? 2 * ka : ka;
   const int nbB = full ? nb : 1;
@@ -102,14 +108,42 @@ aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const
       drow[wd] = pack_bf16x2(o[0], o[1]);
     }
   }
+  // transposed Z tables: Zt[q][j][n] for each distinct query (gate, then up); one thread per
+  // (matrix, query, group of 4 ranks, column n), columns fastest so that the stores coalesce
+  if (Zt && blk.nzq > 0) {
+    const int groups = (r + 3) / 4;
+    const int n_mat = Zt2 ? 2 : 1;
+    const int64_t items = (int64_t)n_mat * blk.nzq * groups * d_out;
+    for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < items;
+         it += (int64_t)gridDim.x * blockDim.x) {
+      const int n = (int)(it % d_out);
+      int64_t rest = it / d_out;
+      const int jg = (int)(rest % groups);
+      rest /= groups;
+      const int qi = (int)(rest % blk.nzq);
+      const int mat = (int)(rest / blk.nzq);
+      float* dst = (mat ? Zt2 : Zt) + (int64_t)qi * r * d_out;
+      const uint32_t layer = mat ? lid2 : lid;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int j = 4 * jg + i;
+        if (j < r) {
+          const int64_t e = (int64_t)n * r + j;
+          dst[(int64_t)j * d_out + n] = z_select(z_normals4(seed, layer, blk.zq[qi], (uint64_t)(e >> 2)), (int)(e & 3));
+        }
+      }
+    }
+  }
 }
 
 }  // namespace
 
 int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct, void* A_aug, void* B_aug,
-                    void* B_aug2) {
+                    void* B_aug2, float* Zt, float* Zt2, const uint64_t* zq, int nzq) {
   AugBlocks blk{};
   for (int b = 0; b < a.nb; ++b) { blk.coef[b] = a.coef[b]; blk.qry[b] = a.qry[b]; }
+  for (int i = 0; i < nzq; ++i) blk.zq[i] = zq[i];
+  blk.nzq = Zt ? nzq : 0;
   const int full = mode == LOWRANK_ALL_ON_TC;
   const int ka_tot = distinct ? 2 * ka : ka;
   (void)ka_tot;
@@ -122,7 +156,7 @@ int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct,
   aug_prep_kernel<<<(unsigned)grid, 256, 0, ctx->stream>>>(
       a.P, distinct ? a.P2 : nullptr, a.C, a.C2, static_cast<__nv_bfloat16*>(A_aug),
       static_cast<__nv_bfloat16*>(B_aug), static_cast<__nv_bfloat16*>(B_aug2), a.rows, a.d_out, a.r, ka, distinct,
-      full, a.nb, blk, a.seed, a.layer_id, a.layer_id2);
+      full, a.nb, blk, a.seed, a.layer_id, a.layer_id2, Zt, Zt2);
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;

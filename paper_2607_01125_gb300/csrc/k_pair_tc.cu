@@ -140,6 +140,22 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   const int ka_tot = distinct ? 2 * ka : ka;
   tm.aa = tm.a; tm.ba = tm.b; tm.ba2 = tm.b2;
   int64_t aug_block_rows = 0;
+  // C on the tensor cores: the distinct queries of the perturbed blocks, each one transposed Z table
+  uint64_t zq_list[ZOACT_MAX_EVAL_BLOCKS];
+  int zq_of[ZOACT_MAX_EVAL_BLOCKS];
+  int nzq = 0;
+  for (int b = 0; b < a.nb; ++b) {
+    zq_of[b] = -1;
+    if (lmode != LOWRANK_C_ON_TC || a.coef[b] == 0.f) continue;
+    for (int i = 0; i < nzq; ++i)
+      if (zq_list[i] == a.qry[b]) zq_of[b] = i;
+    if (zq_of[b] < 0) {
+      zq_list[nzq] = a.qry[b];
+      zq_of[b] = nzq++;
+    }
+  }
+  float* zt = nullptr;
+  float* zt2 = nullptr;
   if (lmode != LOWRANK_EPILOGUE) {
     const int64_t nbB = lmode == LOWRANK_ALL_ON_TC ? a.nb : 1;
     const size_t a_bytes = (size_t)a.rows * ka_tot * 2;
@@ -148,7 +164,13 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     uint8_t* bbuf = static_cast<uint8_t*>(scratch(ctx, SLOT_AUG_B, (gated ? 2 : 1) * b_bytes));
     if (!abuf || !bbuf) return ZOACT_ERR_NOMEM;
     uint8_t* bbuf2 = gated ? bbuf + b_bytes : nullptr;
-    st = launch_aug_prep(ctx, a, lmode, ka, distinct ? 1 : 0, abuf, bbuf, bbuf2);
+    if (nzq > 0) {
+      const size_t z_floats = (size_t)nzq * a.r * a.d_out;
+      zt = static_cast<float*>(scratch(ctx, SLOT_AUG_Z, (gated ? 2 : 1) * z_floats * sizeof(float)));
+      if (!zt) return ZOACT_ERR_NOMEM;
+      zt2 = gated ? zt + z_floats : nullptr;
+    }
+    st = launch_aug_prep(ctx, a, lmode, ka, distinct ? 1 : 0, abuf, bbuf, bbuf2, zt, zt2, zq_list, nzq);
     if (st) return st;
     st = encode_tmap_2d_16bit(&tm.aa, abuf, ZOACT_DT_BF16, a.rows, ka_tot, BM);
     if (st) return st;
@@ -182,6 +204,10 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   p.aug_mode = lmode;
   p.aug_kb = lmode == LOWRANK_EPILOGUE ? 0 : ka_tot / BK;
   p.aug_block_rows = aug_block_rows;
+  p.Zt = zt;
+  p.Zt2 = zt2;
+  p.zt_qstride = (int64_t)a.r * a.d_out;
+  for (int b = 0; b < ZOACT_MAX_EVAL_BLOCKS; ++b) p.zq[b] = b < a.nb ? zq_of[b] : -1;
   auto al16 = [](const void* q) { return q == nullptr || ((uintptr_t)q & 15u) == 0; };
   p.vec_ok = al16(a.C) && al16(a.C2) && al16(a.P) && al16(a.P2);
   p.status = ctx->d_status;

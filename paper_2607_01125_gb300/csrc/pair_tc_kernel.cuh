@@ -106,6 +106,11 @@ struct Params {
   int aug_mode;      // LowrankMode
   int aug_kb;        // extra K-blocks per tile from A_aug / B_aug (0 with LOWRANK_EPILOGUE)
   int64_t aug_block_rows;   // rows of one block's table in B_aug (LOWRANK_ALL_ON_TC)
+  // LOWRANK_C_ON_TC: Z of each distinct query, transposed [q][r][d_out] (gate / up), and the table of each block
+  const float* Zt;
+  const float* Zt2;
+  int64_t zt_qstride;       // floats per query table (r * d_out)
+  int zq[ZOACT_MAX_EVAL_BLOCKS];   // block b's table in Zt (-1: coefficient 0)
   int64_t ldy;       // plain mode: row stride of D
   int vec_ok;        // C, C2, P, P2 and ldy allow 16-byte vector access
   int bn;            // N-tile width of pair / plain tiles (multiple of 32, <= BN); gated tiles use BN
@@ -197,6 +202,31 @@ __device__ __forceinline__ void build_tables(float* tb0, float* tb1, int stride,
     }
     tb0[j * stride + s] = v0;
     if (tb1) tb1[j * stride + s] = v1;
+  }
+}
+
+// The same tables from precomputed transposed Z (Zq0 / Zq1: a query's [r][d_out]
+// table, Zq1 may equal Zq0): tb[j * stride + s] = c Z[j][col0 + s].  One thread
+// per 4 consecutive columns of one rank: coalesced 16-byte loads (d_out % 8 == 0).
+template <int RT>
+__device__ __forceinline__ void build_tables_z(float* tb0, float* tb1, int stride, const float* __restrict__ Zq0,
+                                               const float* __restrict__ Zq1, float c0, float c1, int col0,
+                                               int ncols, int d_out, int r, int tid) {
+  const int per_row = ncols / 4;
+  for (int it = tid; it < RT * per_row; it += EPI_THREADS) {
+    const int j = it / per_row, s = 4 * (it - j * per_row);
+    const int col = col0 + s;
+    float4 v0 = make_float4(0.f, 0.f, 0.f, 0.f), v1 = v0;
+    if (j < r && col < d_out) {
+      const float4 z0 = *reinterpret_cast<const float4*>(Zq0 + (int64_t)j * d_out + col);
+      v0 = make_float4(c0 * z0.x, c0 * z0.y, c0 * z0.z, c0 * z0.w);
+      if (tb1) {
+        const float4 z1 = Zq1 == Zq0 ? z0 : *reinterpret_cast<const float4*>(Zq1 + (int64_t)j * d_out + col);
+        v1 = make_float4(c1 * z1.x, c1 * z1.y, c1 * z1.z, c1 * z1.w);
+      }
+    }
+    *reinterpret_cast<float4*>(tb0 + j * stride + s) = v0;
+    if (tb1) *reinterpret_cast<float4*>(tb1 + j * stride + s) = v1;
   }
 }
 
@@ -453,12 +483,23 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
         float* t0 = tbl;
         float* t1 = (need0 && need1) ? tbl + TSZ : nullptr;
         const float c0v = need0 ? tc0 : prm.coef[b1];
-        const uint64_t q0v = need0 ? prm.qry[bp] : prm.qry[b1];
-        build_tables<RT>(t0, t1, STRIDE, Cg, prm.layer_id, col0, cwid, prm.d_out, r, prm.seed, c0v, q0v,
-                         prm.coef[b1], prm.qry[b1], etid, vec);
-        if (GATED)
-          build_tables<RT>(t0 + 2 * TSZ, t1 ? t1 + 2 * TSZ : nullptr, STRIDE, Cg2, prm.layer_id2, col0, cwid,
-                           prm.d_out, r, prm.seed, c0v, q0v, prm.coef[b1], prm.qry[b1], etid, vec);
+        if (c_in_acc) {
+          // c_b Z_b from the transposed Z tables
+          const int z0 = need0 ? prm.zq[bp] : prm.zq[b1];
+          const int z1 = prm.zq[b1] >= 0 ? prm.zq[b1] : z0;
+          build_tables_z<RT>(t0, t1, STRIDE, prm.Zt + z0 * prm.zt_qstride, prm.Zt + z1 * prm.zt_qstride, c0v,
+                             prm.coef[b1], col0, cwid, prm.d_out, r, etid);
+          if (GATED)
+            build_tables_z<RT>(t0 + 2 * TSZ, t1 ? t1 + 2 * TSZ : nullptr, STRIDE, prm.Zt2 + z0 * prm.zt_qstride,
+                               prm.Zt2 + z1 * prm.zt_qstride, c0v, prm.coef[b1], col0, cwid, prm.d_out, r, etid);
+        } else {
+          const uint64_t q0v = need0 ? prm.qry[bp] : prm.qry[b1];
+          build_tables<RT>(t0, t1, STRIDE, Cg, prm.layer_id, col0, cwid, prm.d_out, r, prm.seed, c0v, q0v,
+                           prm.coef[b1], prm.qry[b1], etid, vec);
+          if (GATED)
+            build_tables<RT>(t0 + 2 * TSZ, t1 ? t1 + 2 * TSZ : nullptr, STRIDE, Cg2, prm.layer_id2, col0, cwid,
+                             prm.d_out, r, prm.seed, c0v, q0v, prm.coef[b1], prm.qry[b1], etid, vec);
+        }
       }
       tc::named_bar_sync(1, EPI_THREADS);
       if (!waited) {
