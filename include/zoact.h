@@ -133,6 +133,22 @@ int zoact_philox_normals(zoact_ctx* ctx, uint64_t seed, uint32_t layer_id, uint6
 int zoact_lowrank_proj(zoact_ctx* ctx, const void* X, int xdtype, int64_t rows, int32_t d_in,
                        const float* U, int32_t r, float* P);
 
+/* ---- the frozen basis in the projection's tensor-core operand form ----
+ * Algorithm 1 freezes U; the tensor-core projection multiplies 16-bit X by U
+ * split into three 16-bit terms (U = U0 + U1 + U2, each the rounding of what
+ * the previous terms left), which keeps the product at fp32 accuracy.
+ * zoact_basis_prepare writes that operand once (U_tc: zoact_basis_prepared_bytes
+ * bytes of device memory, 16-byte aligned, caller-owned; xdtype BF16 or FP16 is
+ * the dtype of the X it will multiply; d_in % 8 == 0) so that
+ * zoact_lowrank_proj_prepared computes P = X U from it without re-splitting U.
+ * U_tc must be prepared again if U changes.  zoact_basis_prepared_bytes returns -1
+ * for unsupported sizes (r > 32).                                               */
+int64_t zoact_basis_prepared_bytes(int32_t d_in, int32_t r);
+int zoact_basis_prepare(zoact_ctx* ctx, const float* U, int32_t d_in, int32_t r, int32_t xdtype,
+                        void* U_tc);
+int zoact_lowrank_proj_prepared(zoact_ctx* ctx, const void* X, int xdtype, int64_t rows, int32_t d_in,
+                                const void* U_tc, int32_t r, float* P);
+
 /* ---- the pair forward (Section 3, perturbed forward pass; Algorithm 2) ----
  * Y = the stacked outputs y(+1), y(-1) of one adapted linear:
  *   input_shared == 0: X is [2T, d_in] stacked; row t of Y uses sigma(t).

@@ -13,5 +13,6 @@ from ._lib import (  # noqa: F401
     zoact_loss_pair, zoact_adam_step, zoact_sgd_step, zoact_basis_init, zoact_rms_norm, zoact_mix_rms,
     zoact_multi_forward, zoact_multi_forward_gated, zoact_loss_multi, zoact_adam_step_multi, zoact_sgd_step_multi,
     eval_blocks, one_sided_blocks, MAX_EVAL_BLOCKS,
+    zoact_basis_prepared_bytes, zoact_basis_prepare, zoact_lowrank_proj_prepared,
     DT_FP32, DT_BF16, DT_FP16, DT_INT4_G128, ACT_NONE, ACT_RELU, ACT_GELU, EXPORTS, LIB_PATH,
 )

@@ -35,7 +35,8 @@ EXPORTS = [
     "zoact_device_sm_count", "zoact_get_launch_count", "zoact_philox_normals", "zoact_lowrank_proj", "zoact_pair_forward",
     "zoact_pair_forward_noalloc", "zoact_pair_forward_gated", "zoact_loss_pair", "zoact_adam_step", "zoact_sgd_step", "zoact_basis_init",
     "zoact_rms_norm", "zoact_mix_rms", "zoact_multi_forward", "zoact_multi_forward_gated", "zoact_loss_multi",
-    "zoact_adam_step_multi", "zoact_sgd_step_multi",
+    "zoact_adam_step_multi", "zoact_sgd_step_multi", "zoact_basis_prepared_bytes", "zoact_basis_prepare",
+    "zoact_lowrank_proj_prepared",
 ]
 
 
@@ -110,6 +111,8 @@ def load():
         "zoact_basis_init": [P, P, I32, I64, I32, I32, I32, I32, U64, P, P],
         "zoact_rms_norm": [P, P, I32, I64, I32, F32, P],
         "zoact_mix_rms": [P, P, P, P, I32, I64, I32, I32, I32, F32, P],
+        "zoact_basis_prepare": [P, P, I32, I32, I32, P],
+        "zoact_lowrank_proj_prepared": [P, P, I32, I64, I32, P, I32, P],
         "zoact_multi_forward": [P, ctypes.POINTER(zoact_layer), P, I32, I64, I32, P, ctypes.POINTER(zoact_eval_blocks),
                                 U64, I32, P, I32],
         "zoact_multi_forward_gated": [P, ctypes.POINTER(zoact_layer), ctypes.POINTER(zoact_layer), P, I32, I64, I32,
@@ -124,6 +127,8 @@ def load():
         fn = getattr(lib, name)
         fn.argtypes = argtypes
         fn.restype = ctypes.c_int
+    lib.zoact_basis_prepared_bytes.argtypes = [I32, I32]
+    lib.zoact_basis_prepared_bytes.restype = ctypes.c_int64
     lib.zoact_status_string.argtypes = [ctypes.c_int]
     lib.zoact_status_string.restype = ctypes.c_char_p
     _lib = lib
@@ -338,3 +343,19 @@ def zoact_sgd_step_multi(ctx, C, blocks, a, queries, lr, seed):
     _check("zoact_sgd_step_multi", load().zoact_sgd_step_multi(ctx.handle, _ptr(C), C.numel(), arr, len(blocks),
                                                                 _ptr(a), len(queries), _queries(queries), float(lr),
                                                                 int(seed)))
+
+
+def zoact_basis_prepared_bytes(d_in, r):
+    return int(load().zoact_basis_prepared_bytes(int(d_in), int(r)))
+
+
+def zoact_basis_prepare(ctx, U, xdtype, U_tc):
+    """U [d_in, r] fp32 -> U_tc (uint8 device tensor of zoact_basis_prepared_bytes bytes) for X of xdtype."""
+    d_in, r = U.shape
+    _check("zoact_basis_prepare", load().zoact_basis_prepare(ctx.handle, _ptr(U), d_in, r, int(xdtype), _ptr(U_tc)))
+
+
+def zoact_lowrank_proj_prepared(ctx, X, U_tc, r, P):
+    rows, d_in = X.shape
+    _check("zoact_lowrank_proj_prepared", load().zoact_lowrank_proj_prepared(ctx.handle, _ptr(X), _dt(X), rows, d_in,
+                                                                              _ptr(U_tc), int(r), _ptr(P)))

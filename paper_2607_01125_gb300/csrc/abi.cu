@@ -36,6 +36,19 @@ void* scratch(Ctx* ctx, ScratchSlot slot, size_t bytes) {
   return p;
 }
 
+void* scratch_zeroed(Ctx* ctx, ScratchSlot slot, size_t bytes) {
+  const void* before = ctx->slot_ptr[slot];
+  const size_t had = ctx->slot_bytes[slot];
+  void* p = scratch(ctx, slot, bytes);
+  if (p && (p != before || ctx->slot_bytes[slot] != had)) {
+    if (cudaMemsetAsync(p, 0, ctx->slot_bytes[slot], ctx->stream) != cudaSuccess) {
+      cudaGetLastError();
+      return nullptr;
+    }
+  }
+  return p;
+}
+
 }  // namespace zoact
 
 using namespace zoact;
@@ -200,6 +213,31 @@ static zoact_eval_blocks pair_blocks(float eps, uint64_t query) {
   b.coef[1] = -eps;
   b.query[0] = b.query[1] = query;
   return b;
+}
+
+int64_t zoact_basis_prepared_bytes(int32_t d_in, int32_t r) {
+  if (d_in <= 0 || r <= 0 || r > 32) return -1;
+  return (int64_t)basis_tc_rows(r) * d_in * 2;
+}
+
+int zoact_basis_prepare(zoact_ctx* ctx, const float* U, int32_t d_in, int32_t r, int32_t xdtype, void* U_tc) {
+  ZOACT_ENTER(ctx);
+  if (!U || !U_tc || d_in <= 0 || r <= 0) return ZOACT_ERR_INVALID_ARG;
+  if (r > 32) return ZOACT_ERR_UNSUPPORTED;
+  if (xdtype != ZOACT_DT_BF16 && xdtype != ZOACT_DT_FP16) return ZOACT_ERR_INVALID_ARG;
+  if (d_in % 8 != 0 || !aligned16(U_tc)) return ZOACT_ERR_INVALID_ARG;
+  return launch_basis_prepare(ctx, U, d_in, r, xdtype, U_tc);
+}
+
+int zoact_lowrank_proj_prepared(zoact_ctx* ctx, const void* X, int xdtype, int64_t rows, int32_t d_in,
+                                const void* U_tc, int32_t r, float* P) {
+  ZOACT_ENTER(ctx);
+  if (rows < 0 || d_in <= 0 || r <= 0) return ZOACT_ERR_INVALID_ARG;
+  if (r > 32) return ZOACT_ERR_UNSUPPORTED;
+  if (xdtype != ZOACT_DT_BF16 && xdtype != ZOACT_DT_FP16) return ZOACT_ERR_INVALID_ARG;
+  if (rows == 0) return ZOACT_OK;
+  if (!X || !U_tc || !P || !aligned16(X) || !aligned16(U_tc) || d_in % 8 != 0) return ZOACT_ERR_INVALID_ARG;
+  return launch_lowrank_proj_tc_prepared(ctx, X, xdtype, rows, d_in, U_tc, r, P);
 }
 
 static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* L2, const void* X, int xdtype,

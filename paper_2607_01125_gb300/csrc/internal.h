@@ -33,6 +33,7 @@ enum ScratchSlot {
   SLOT_AUG_A,        // 16-bit split of the projection P (extra K columns of the tensor-core pair forward)
   SLOT_AUG_B,        // 16-bit split of C (+ c_b Z_b) for those K columns (gate and up)
   SLOT_AUG_Z,        // Z of each query, transposed, for the epilogue (C on the tensor cores)
+  SLOT_PROJ_TICKETS, // split-K tickets of the tensor-core projection (zero between calls)
   SLOT_COUNT
 };
 
@@ -51,6 +52,8 @@ struct Ctx {
 int cuda_fail(cudaError_t e, const char* what);
 // Returns a device pointer of at least `bytes` for the slot, or nullptr on failure.
 void* scratch(Ctx* ctx, ScratchSlot slot, size_t bytes);
+// As scratch(), and a newly allocated buffer is zero-filled (on the context's stream).
+void* scratch_zeroed(Ctx* ctx, ScratchSlot slot, size_t bytes);
 
 // Device-side error recording: keeps the first non-zero code.
 __device__ __forceinline__ void record_error(int* status, int code) {
@@ -88,6 +91,12 @@ int launch_lowrank_proj(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d
 // Tensor-core projection for 16-bit X (U split into three 16-bit terms).
 int launch_lowrank_proj_tc(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const float* U, int r,
                            float* P);
+// The basis in the tensor-core projection's operand form: [basis_tc_rows(r), d_in] 16-bit (xdtype),
+// rows [0, RT) / [RT, 2RT) / [2RT, 3RT) the three 16-bit terms of U^T (RT = r rounded up to 4, 8, 16, 32).
+int basis_tc_rows(int r);
+int launch_basis_prepare(Ctx* ctx, const float* U, int d_in, int r, int xdtype, void* Ut);
+int launch_lowrank_proj_tc_prepared(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const void* Ut,
+                                    int r, float* P);
 // As launch_lowrank_proj, with split-K partials in `part` (part_floats floats) instead of context scratch.
 int launch_lowrank_proj_into(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const float* U,
                              int r, float* P, float* part, int64_t part_floats);

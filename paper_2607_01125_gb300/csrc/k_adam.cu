@@ -49,18 +49,13 @@ zo_update_kernel(float* __restrict__ C, float* __restrict__ m, float* __restrict
                  int64_t g_begin, int64_t g_end, const double* __restrict__ a_dev, int nq,
                  const __grid_constant__ QueryList qs, float lr, float b1, float b2, float adam_eps, float step_size,
                  float inv_sqrt_bc2, uint64_t seed, int* __restrict__ status) {
-  float a[ZOACT_MAX_EVAL_BLOCKS];
   bool finite = true;
-#pragma unroll
-  for (int j = 0; j < ZOACT_MAX_EVAL_BLOCKS; ++j) {
-    const double aj = j < nq ? a_dev[j] : 0.0;
-    finite = finite && isfinite(aj);
-    a[j] = (float)aj;
-  }
+  for (int j = 0; j < nq; ++j) finite = finite && isfinite(a_dev[j]);
   if (!finite) {
     if (blockIdx.x == 0 && threadIdx.x == 0) record_error(status, ZOACT_ERR_NONFINITE);
     return;
   }
+  const float a0 = (float)a_dev[0];
   const float inv_q = 1.0f / (float)nq;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t g = g_begin + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; g < g_end; g += stride) {
@@ -71,13 +66,14 @@ zo_update_kernel(float* __restrict__ C, float* __restrict__ m, float* __restrict
     float gz[4];
     {
       const float4 z = z_normals4(seed, tab.layer_id[b], qs.q[0], (uint64_t)(local >> 2));
-      gz[0] = a[0] * z.x; gz[1] = a[0] * z.y; gz[2] = a[0] * z.z; gz[3] = a[0] * z.w;
+      gz[0] = a0 * z.x; gz[1] = a0 * z.y; gz[2] = a0 * z.z; gz[3] = a0 * z.w;
     }
     if (nq > 1) {
       for (int j = 1; j < nq; ++j) {
+        const float aj = (float)a_dev[j];
         const float4 z = z_normals4(seed, tab.layer_id[b], qs.q[j], (uint64_t)(local >> 2));
-        gz[0] = fmaf(a[j], z.x, gz[0]); gz[1] = fmaf(a[j], z.y, gz[1]);
-        gz[2] = fmaf(a[j], z.z, gz[2]); gz[3] = fmaf(a[j], z.w, gz[3]);
+        gz[0] = fmaf(aj, z.x, gz[0]); gz[1] = fmaf(aj, z.y, gz[1]);
+        gz[2] = fmaf(aj, z.z, gz[2]); gz[3] = fmaf(aj, z.w, gz[3]);
       }
 #pragma unroll
       for (int i = 0; i < 4; ++i) gz[i] *= inv_q;

@@ -3,10 +3,13 @@
 //   D  = mean((y+ - y-)(y+ + y- - 2t))   (= L+ - L-, without cancellation),
 //   a  = D / (2 eps).
 // One pass over the stacked outputs (HBM-bound).  Each thread reads 16-byte
-// vectors of y+, y- and t, sums a vector's terms in fp32 and adds the vector sum
-// to fp64 accumulators; warps reduce by shuffles, blocks write fp64 partials to
-// scratch, and the last block to finish (an atomic ticket) adds the partials in
-// block order, so the result is deterministic.  The ticket is reset by that
+// vectors of y+, y- and t (kept as raw words until used; 64 registers, four
+// 256-thread blocks per SM), sums a round of two vectors' terms (16 per
+// accumulator) in fp32 and adds the round's sum to fp64 accumulators (fp64 adds
+// are scarce on this part: one per 16 terms keeps them off the critical path);
+// warps reduce by shuffles, blocks write fp64 partials to scratch, and the last
+// block to finish (an atomic ticket) adds the partials in block order, so the
+// result is deterministic.  The ticket is reset by that
 // block, leaving the scratch ready for the next call.
 #include "internal.h"
 
@@ -23,6 +26,37 @@ __device__ __forceinline__ void unpack2(uint32_t w, float* out, const __half*) {
   const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w));
   out[0] = f.x;
   out[1] = f.y;
+}
+
+// 8 consecutive elements as raw 16-byte words (unpacked only when used, so a
+// round of loads in flight costs 4 registers per 8 elements of 16-bit data)
+template <typename TY> struct Raw8 { uint4 w; };
+template <> struct Raw8<float> { float4 a, b; };
+
+template <typename TY>
+__device__ __forceinline__ Raw8<TY> ld8(const TY* p) {
+  Raw8<TY> r;
+  r.w = __ldg(reinterpret_cast<const uint4*>(p));
+  return r;
+}
+template <>
+__device__ __forceinline__ Raw8<float> ld8<float>(const float* p) {
+  Raw8<float> r;
+  r.a = __ldg(reinterpret_cast<const float4*>(p));
+  r.b = __ldg(reinterpret_cast<const float4*>(p + 4));
+  return r;
+}
+template <typename TY>
+__device__ __forceinline__ void unpack8(const Raw8<TY>& r, float* out) {
+  unpack2(r.w.x, out + 0, (const TY*)nullptr);
+  unpack2(r.w.y, out + 2, (const TY*)nullptr);
+  unpack2(r.w.z, out + 4, (const TY*)nullptr);
+  unpack2(r.w.w, out + 6, (const TY*)nullptr);
+}
+template <>
+__device__ __forceinline__ void unpack8<float>(const Raw8<float>& r, float* out) {
+  out[0] = r.a.x; out[1] = r.a.y; out[2] = r.a.z; out[3] = r.a.w;
+  out[4] = r.b.x; out[5] = r.b.y; out[6] = r.b.z; out[7] = r.b.w;
 }
 
 template <typename TY>
@@ -48,7 +82,7 @@ __device__ __forceinline__ double warp_sum(double v) {
 }
 
 template <typename TY>
-__global__ void __launch_bounds__(LOSS_THREADS)
+__global__ void __launch_bounds__(LOSS_THREADS, 4)
 loss_pair_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t count, int vec_ok, float eps,
                  double* __restrict__ out, double* __restrict__ partials, unsigned int* __restrict__ ticket,
                  int* __restrict__ status) {
@@ -61,27 +95,36 @@ loss_pair_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t c
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   // four vectors per round with all twelve 16-byte loads issued before any use
-  for (; v + 3 * stride < n_vec; v += 4 * stride) {
-    float p[4][8], m[4][8], t[4][8];
+  constexpr int R = sizeof(TY) == 4 ? 1 : 2;   // vectors per round (fp32 words take twice the registers)
+  for (; v + (R - 1) * stride < n_vec; v += R * stride) {
+    Raw8<TY> rp[R], rm[R], rt[R];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      load8<TY>(yp + 8 * (v + u * stride), p[u]);
-      load8<TY>(ym + 8 * (v + u * stride), m[u]);
-      if (tgt) load8<TY>(tgt + 8 * (v + u * stride), t[u]);
+    for (int u = 0; u < R; ++u) {
+      rp[u] = ld8<TY>(yp + 8 * (v + u * stride));
+      rm[u] = ld8<TY>(ym + 8 * (v + u * stride));
+      if (tgt) rt[u] = ld8<TY>(tgt + 8 * (v + u * stride));
     }
+    float sp = 0.f, sm = 0.f, sd = 0.f;
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      float sp = 0.f, sm = 0.f, sd = 0.f;
+    for (int u = 0; u < R; ++u) {
+      float p[8], m[8], t[8];
+      unpack8<TY>(rp[u], p);
+      unpack8<TY>(rm[u], m);
+      if (tgt) {
+        unpack8<TY>(rt[u], t);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) t[i] = 0.f;
+      }
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
-        const float tv = tgt ? t[u][i] : 0.f;
-        const float dp = p[u][i] - tv, dm = m[u][i] - tv;
+        const float dp = p[i] - t[i], dm = m[i] - t[i];
         sp = fmaf(dp, dp, sp);
         sm = fmaf(dm, dm, sm);
-        sd = fmaf(p[u][i] - m[u][i], dp + dm, sd);
+        sd = fmaf(p[i] - m[i], dp + dm, sd);
       }
-      ap += sp; am += sm; ad += sd;
     }
+    ap += sp; am += sm; ad += sd;
   }
   for (; v < n_vec; v += stride) {
     float p[8], m[8], t[8];
@@ -178,7 +221,7 @@ int loss_dispatch(Ctx* ctx, const TY* Y, const TY* tgt, int64_t count, float eps
 // the elements (y_0 and t are re-read once per block, from L2 when they fit).
 // Partials [nb][gridDim.x][2] are added in a fixed order by the last CTA.
 template <typename TY>
-__global__ void __launch_bounds__(LOSS_THREADS)
+__global__ void __launch_bounds__(LOSS_THREADS, 4)
 loss_multi_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t count, int vec_ok, int nb, float mu,
                   double* __restrict__ out, double* __restrict__ partials, unsigned int* __restrict__ ticket,
                   int* __restrict__ status) {
@@ -189,12 +232,42 @@ loss_multi_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t 
   const int64_t n_vec = vec_ok ? count / 8 : 0;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int64_t first = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  for (int64_t v = first; v < n_vec; v += stride) {
+  // rounds of two vectors, all loads issued first; one fp64 add per accumulator per round
+  int64_t v = first;
+  constexpr int R = sizeof(TY) == 4 ? 1 : 2;   // vectors per round (fp32 words take twice the registers)
+  for (; v + (R - 1) * stride < n_vec; v += R * stride) {
+    Raw8<TY> ry[R], rz[R], rt[R];
+#pragma unroll
+    for (int u = 0; u < R; ++u) {
+      ry[u] = ld8<TY>(yb + 8 * (v + u * stride));
+      if (b > 0) rz[u] = ld8<TY>(y0 + 8 * (v + u * stride));
+      if (tgt) rt[u] = ld8<TY>(tgt + 8 * (v + u * stride));
+    }
+    float ss = 0.f, sd = 0.f;
+#pragma unroll
+    for (int u = 0; u < R; ++u) {
+      float y[8], z[8], t[8];
+      unpack8<TY>(ry[u], y);
+      if (b > 0) unpack8<TY>(rz[u], z);
+      if (tgt) {
+        unpack8<TY>(rt[u], t);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) t[i] = 0.f;
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float dy = y[i] - t[i];
+        ss = fmaf(dy, dy, ss);
+        if (b > 0) sd = fmaf(y[i] - z[i], dy + (z[i] - t[i]), sd);
+      }
+    }
+    as += ss; ad += sd;
+  }
+  for (; v < n_vec; v += stride) {
     float y[8], z[8], t[8];
     load8<TY>(yb + 8 * v, y);
-    if (b > 0) {
-      load8<TY>(y0 + 8 * v, z);
-    }
+    if (b > 0) load8<TY>(y0 + 8 * v, z);
     if (tgt) {
       load8<TY>(tgt + 8 * v, t);
     } else {

@@ -11,7 +11,8 @@
 // products into TMEM; the epilogue adds them.
 //
 // Grid: (row blocks of 128, K-splits).  Per CTA: warp 0 streams X tiles
-// (128 x 64) and Ut tiles (NB x 64) through an 8-stage TMA ring, warp 1 issues
+// (128 x 64) and Ut tiles (NB x 64) through a 4-stage TMA ring (two CTAs per
+// SM; the grid is one wave of them), warp 1 issues
 // the MMAs, then all four warps read the accumulator (one row per thread) and
 // write the split's partial [rows, r] (or P itself without split).
 #include "internal.h"
@@ -20,7 +21,7 @@
 namespace zoact {
 namespace {
 
-constexpr int PBM = 128, PBK = 64, PSTAGES = 8;
+constexpr int PBM = 128, PBK = 64, PSTAGES = 4;
 constexpr int P_A_BYTES = PBM * PBK * 2;
 
 template <int NB>
@@ -202,26 +203,43 @@ int dispatch(Ctx* ctx, int rt, const CUtensorMap& mx, const CUtensorMap& mu, flo
 
 }  // namespace
 
+int basis_tc_rows(int r) {
+  const int rt = r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32;
+  return 3 * rt <= 16 ? 16 : (3 * rt <= 32 ? 32 : (3 * rt <= 48 ? 48 : 96));
+}
+
+int launch_basis_prepare(Ctx* ctx, const float* U, int d_in, int r, int xdtype, void* Ut) {
+  const int rt = r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32;
+  const int nb = basis_tc_rows(r);
+  const int64_t n = (int64_t)nb * d_in;
+  int64_t blocks = (n + 255) / 256;
+  if (blocks > 8LL * ctx->sm_count) blocks = 8LL * ctx->sm_count;
+  if (xdtype == ZOACT_DT_BF16)
+    split_u_kernel<__nv_bfloat16><<<(unsigned)blocks, 256, 0, ctx->stream>>>(U, static_cast<__nv_bfloat16*>(Ut), d_in,
+                                                                             r, rt, nb);
+  else
+    split_u_kernel<__half><<<(unsigned)blocks, 256, 0, ctx->stream>>>(U, static_cast<__half*>(Ut), d_in, r, rt, nb);
+  ++ctx->n_launch;
+  ZOACT_CHECK_LAUNCH();
+  return ZOACT_OK;
+}
+
 int launch_lowrank_proj_tc(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const float* U, int r,
                            float* P) {
   if (rows <= 0) return ZOACT_OK;
-  const int rt = r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32;
-  const int nb = rt == 4 ? 16 : rt == 8 ? 32 : rt == 16 ? 48 : 96;
   // Ut: the split basis, [nb, d_in] 16-bit, rebuilt on every call (U is small)
-  void* Ut = scratch(ctx, SLOT_UT, (size_t)nb * d_in * 2);
+  void* Ut = scratch(ctx, SLOT_UT, (size_t)basis_tc_rows(r) * d_in * 2);
   if (!Ut) return ZOACT_ERR_NOMEM;
-  {
-    const int64_t n = (int64_t)nb * d_in;
-    int64_t blocks = (n + 255) / 256;
-    if (blocks > 8LL * ctx->sm_count) blocks = 8LL * ctx->sm_count;
-    if (xdtype == ZOACT_DT_BF16)
-      split_u_kernel<__nv_bfloat16><<<(unsigned)blocks, 256, 0, ctx->stream>>>(U, static_cast<__nv_bfloat16*>(Ut),
-                                                                               d_in, r, rt, nb);
-    else
-      split_u_kernel<__half><<<(unsigned)blocks, 256, 0, ctx->stream>>>(U, static_cast<__half*>(Ut), d_in, r, rt, nb);
-    ++ctx->n_launch;
-    ZOACT_CHECK_LAUNCH();
-  }
+  const int st = launch_basis_prepare(ctx, U, d_in, r, xdtype, Ut);
+  if (st) return st;
+  return launch_lowrank_proj_tc_prepared(ctx, X, xdtype, rows, d_in, Ut, r, P);
+}
+
+int launch_lowrank_proj_tc_prepared(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const void* Ut,
+                                    int r, float* P) {
+  if (rows <= 0) return ZOACT_OK;
+  const int rt = r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32;
+  const int nb = basis_tc_rows(r);
   CUtensorMap mx, mu;
   int st = encode_tmap_2d_16bit(&mx, X, xdtype, rows, d_in, PBM);
   if (st) return st;
@@ -229,9 +247,9 @@ int launch_lowrank_proj_tc(Ctx* ctx, const void* X, int xdtype, int64_t rows, in
   if (st) return st;
   const int num_kb = (d_in + PBK - 1) / PBK;
   const int64_t row_blocks = (rows + PBM - 1) / PBM;
-  // K-splits so the grid covers every SM about twice, at least 4 K-blocks per split
-  int splits = (int)((2LL * ctx->sm_count + row_blocks - 1) / row_blocks);
-  if (splits > num_kb / 4) splits = num_kb / 4;
+  // K-splits so the grid is one wave of two CTAs per SM, at least 2 K-blocks per split
+  int splits = (int)((2LL * ctx->sm_count) / row_blocks);
+  if (splits > num_kb / 2) splits = num_kb / 2;
   if (splits < 1) splits = 1;
   const int kbps = (num_kb + splits - 1) / splits;
   splits = (num_kb + kbps - 1) / kbps;

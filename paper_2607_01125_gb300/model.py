@@ -90,6 +90,22 @@ class ZOStep:
         self.device = dev
         self.capture = None
         self.timer = None
+        self._utc = {}
+        self.prepare_bases()
+
+    def prepare_bases(self):
+        """The frozen bases in the tensor-core projection's operand form, once per distinct U
+        (16-bit activations only).  Call again after changing a U in place."""
+        self._utc = {}
+        if self.dtype not in (torch.bfloat16, torch.float16):
+            return
+        for l in self.linears:
+            key = l.U.data_ptr()
+            if key in self._utc or l.r > 32:
+                continue
+            t = torch.empty(Z.zoact_basis_prepared_bytes(l.d_in, l.r), dtype=torch.uint8, device=self.device)
+            Z.zoact_basis_prepare(self.ctx, l.U, Z.TORCH_DT[self.dtype], t)
+            self._utc[key] = t
 
     # ---- buffers ----
     def buf(self, key, rows, cols, dtype=None):
@@ -115,7 +131,11 @@ class ZOStep:
                 self._pcache[slot] = (key, P)
                 return P
         P = self.buf(f"P{slot}", X.shape[0], lin.r, torch.float32)
-        Z.zoact_lowrank_proj(self.ctx, X, lin.U, P)
+        utc = self._utc.get(lin.U.data_ptr())
+        if utc is not None and X.dtype == self.dtype:
+            Z.zoact_lowrank_proj_prepared(self.ctx, X, utc, lin.r, P)
+        else:
+            Z.zoact_lowrank_proj(self.ctx, X, lin.U, P)
         self._pcache[slot] = (key, P)
         return P
 
