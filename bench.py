@@ -38,6 +38,11 @@ N_CAL = {"llama_mlp_bf16": 2048, "llama_stack_bf16": 512, "llama_stack_int4": 51
 LR = 1e-4
 
 
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one step's pair launches, from one ncu
+# capture of the current kernels at the default sizes; workloads without such a capture report null.
+PAIR_TRAFFIC_BYTES = {"llama_mlp_bf16": 900.9e6}
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -263,7 +268,9 @@ def run_ours(args):
                      "peak_kind": f"bf16 dense {'sustained' if long_step else 'burst'}, {peak_kind}",
                      "kernel": "pair_tc2_kernel / pair_tc_kernel (every pair-forward launch of the step)",
                      "algorithmic_flops_per_step": gemm_flops / args.steps,
-                     "traffic": None},
+                     "traffic": (PAIR_TRAFFIC_BYTES.get(w.name)
+                                 if args.tokens is None and args.queries is None else None),
+                     "traffic_unit": "bytes per step (both pair launches)"},
         "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": 8 * step.loss_out.numel()},
         "gpu_launches": launches,
