@@ -142,3 +142,14 @@ def subspace_overlap(U1, U2):
     U1 = np.asarray(U1, np.float64)
     U2 = np.asarray(U2, np.float64)
     return float(np.sum((U1.T @ U2) ** 2) / U1.shape[1])
+
+
+def gradient_energy(U, G):
+    """Gradient-energy capture of Section 5.3: the share of a weight gradient's energy inside the basis,
+    ||U^T G||_F^2 / ||G||_F^2, with U [d_in, r] orthonormal and G [d_in, n] (the gradient of W in the
+    paper's [d_in, d_out] orientation).  Returns (||U^T G||_F^2, ||G||_F^2, ratio)."""
+    U = np.asarray(U, np.float64)
+    G = np.asarray(G, np.float64)
+    num = float(np.sum((U.T @ G) ** 2))
+    den = float(np.sum(G * G))
+    return num, den, num / den

@@ -103,3 +103,24 @@ def test_overlap_metric_section53():
     assert basis.subspace_overlap(I[:, :2], I[:, :2]) == 1.0
     assert basis.subspace_overlap(I[:, :2], I[:, 2:4]) == 0.0
     assert basis.subspace_overlap(I[:, :2], I[:, 1:3]) == 0.5
+
+
+def test_gradient_energy_pins():
+    # Section 5.3 energy capture ||U^T G||^2 / ||G||^2: 1 inside the span, 0 orthogonal to it, the sum of the
+    # squared coordinates in between, and 1 for a complete orthonormal basis
+    rng = np.random.default_rng(12)
+    d, r, n = 40, 6, 9
+    Q = np.linalg.qr(rng.standard_normal((d, d)))[0]
+    U, Uperp = Q[:, :r], Q[:, r:]
+    A = rng.standard_normal((r, n))
+    B = rng.standard_normal((d - r, n))
+    assert basis.gradient_energy(U, U @ A)[2] == pytest.approx(1.0, abs=1e-13)
+    assert basis.gradient_energy(U, Uperp @ B)[2] == pytest.approx(0.0, abs=1e-13)
+    G = U @ A + Uperp @ B
+    num, den, ratio = basis.gradient_energy(U, G)
+    assert num == pytest.approx(np.sum(A ** 2), rel=1e-12)
+    assert den == pytest.approx(np.sum(A ** 2) + np.sum(B ** 2), rel=1e-12)
+    assert basis.gradient_energy(Q, G)[2] == pytest.approx(1.0, abs=1e-13)
+    # overlap of the same pair of subspaces equals the energy of U2 (as a gradient) in U1, divided by r
+    U2 = np.linalg.qr(rng.standard_normal((d, r)))[0]
+    assert basis.subspace_overlap(U, U2) == pytest.approx(basis.gradient_energy(U, U2)[0] / r, rel=1e-12)
