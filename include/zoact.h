@@ -300,6 +300,20 @@ int zoact_basis_init(zoact_ctx* ctx, const void* X_cal, int xdtype, int64_t n_to
                      int32_t r, int32_t oversample, int32_t n_iter, uint64_t seed, float* U_out,
                      float* evals_out);
 
+/* ---- subspace diagnostics (Section 5.3) ----
+ * zoact_subspace_overlap: out[0] = ||U_a^T U_b||_F^2, out[1] = ||U_b||_F^2,
+ *   out[2] = ||U_a^T U_b||_F^2 / r_a  (the basis-stability metric; 1 for the same
+ *   subspace, 0 for orthogonal ones).  U_a [d, r_a], U_b [d, r_b] fp32 row-major.
+ * zoact_gradient_energy: out[0] = ||U^T G||_F^2, out[1] = ||G||_F^2, out[2] = their
+ *   ratio (the share of a weight gradient's energy inside the basis; 0 when G = 0).
+ *   U [d_in, r] fp32, G [d_in, n] row-major of gdtype (FP32/BF16/FP16), i.e. the
+ *   gradient of W in the paper's [d_in, d_out] orientation.
+ * out: DEVICE fp64 [3].  1 <= r, r_a, r_b <= 256.  Deterministic; two launches each.  */
+int zoact_subspace_overlap(zoact_ctx* ctx, const float* U_a, const float* U_b, int32_t d, int32_t r_a,
+                           int32_t r_b, double* out);
+int zoact_gradient_energy(zoact_ctx* ctx, const float* U, int32_t d_in, int32_t r, const void* G, int gdtype,
+                          int64_t n, double* out);
+
 /* ---- glue ops of the synthetic graphs (row-wise; activations of one dtype) ----
  * zoact_rms_norm:  Y = X / sqrt(mean(X^2, row) + eps), no gain.                  */
 int zoact_rms_norm(zoact_ctx* ctx, const void* X, int dtype, int64_t rows, int32_t n, float eps,

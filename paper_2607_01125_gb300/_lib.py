@@ -36,7 +36,7 @@ EXPORTS = [
     "zoact_pair_forward_noalloc", "zoact_pair_forward_gated", "zoact_loss_pair", "zoact_adam_step", "zoact_sgd_step", "zoact_basis_init",
     "zoact_rms_norm", "zoact_mix_rms", "zoact_multi_forward", "zoact_multi_forward_gated", "zoact_loss_multi",
     "zoact_adam_step_multi", "zoact_sgd_step_multi", "zoact_basis_prepared_bytes", "zoact_basis_prepare",
-    "zoact_lowrank_proj_prepared",
+    "zoact_lowrank_proj_prepared", "zoact_subspace_overlap", "zoact_gradient_energy",
 ]
 
 
@@ -113,6 +113,8 @@ def load():
         "zoact_mix_rms": [P, P, P, P, I32, I64, I32, I32, I32, F32, P],
         "zoact_basis_prepare": [P, P, I32, I32, I32, P],
         "zoact_lowrank_proj_prepared": [P, P, I32, I64, I32, P, I32, P],
+        "zoact_subspace_overlap": [P, P, P, I32, I32, I32, P],
+        "zoact_gradient_energy": [P, P, I32, I32, P, I32, I64, P],
         "zoact_multi_forward": [P, ctypes.POINTER(zoact_layer), P, I32, I64, I32, P, ctypes.POINTER(zoact_eval_blocks),
                                 U64, I32, P, I32],
         "zoact_multi_forward_gated": [P, ctypes.POINTER(zoact_layer), ctypes.POINTER(zoact_layer), P, I32, I64, I32,
@@ -359,3 +361,17 @@ def zoact_lowrank_proj_prepared(ctx, X, U_tc, r, P):
     rows, d_in = X.shape
     _check("zoact_lowrank_proj_prepared", load().zoact_lowrank_proj_prepared(ctx.handle, _ptr(X), _dt(X), rows, d_in,
                                                                               _ptr(U_tc), int(r), _ptr(P)))
+
+
+def zoact_subspace_overlap(ctx, U_a, U_b, out):
+    """out: device fp64 [3] = [||U_a^T U_b||^2, ||U_b||^2, ||U_a^T U_b||^2 / r_a]."""
+    d, ra = U_a.shape
+    _check("zoact_subspace_overlap", load().zoact_subspace_overlap(ctx.handle, _ptr(U_a), _ptr(U_b), d, ra,
+                                                                    U_b.shape[1], _ptr(out)))
+
+
+def zoact_gradient_energy(ctx, U, G, out):
+    """out: device fp64 [3] = [||U^T G||^2, ||G||^2, ratio]; G [d_in, n]."""
+    d_in, r = U.shape
+    _check("zoact_gradient_energy", load().zoact_gradient_energy(ctx.handle, _ptr(U), d_in, r, _ptr(G), _dt(G),
+                                                                  G.shape[1], _ptr(out)))

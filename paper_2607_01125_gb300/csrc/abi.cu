@@ -420,6 +420,22 @@ int zoact_basis_init(zoact_ctx* ctx, const void* X_cal, int xdtype, int64_t n_to
   return run_basis_init(ctx, X_cal, xdtype, n_tok, d_in, r, oversample, n_iter, seed, U_out, evals_out);
 }
 
+int zoact_subspace_overlap(zoact_ctx* ctx, const float* U_a, const float* U_b, int32_t d, int32_t r_a, int32_t r_b,
+                           double* out) {
+  ZOACT_ENTER(ctx);
+  if (!U_a || !U_b || !out || d <= 0 || r_a <= 0 || r_b <= 0) return ZOACT_ERR_INVALID_ARG;
+  if (r_a > 256 || r_b > 256) return ZOACT_ERR_UNSUPPORTED;
+  return launch_subspace_overlap(ctx, U_a, U_b, d, r_a, r_b, out);
+}
+
+int zoact_gradient_energy(zoact_ctx* ctx, const float* U, int32_t d_in, int32_t r, const void* G, int gdtype, int64_t n,
+                          double* out) {
+  ZOACT_ENTER(ctx);
+  if (!U || !G || !out || d_in <= 0 || r <= 0 || n <= 0 || !valid_act_dtype(gdtype)) return ZOACT_ERR_INVALID_ARG;
+  if (r > 256) return ZOACT_ERR_UNSUPPORTED;
+  return launch_gradient_energy(ctx, U, d_in, r, G, gdtype, n, out);
+}
+
 int zoact_rms_norm(zoact_ctx* ctx, const void* X, int dtype, int64_t rows, int32_t n, float eps, void* Y) {
   ZOACT_ENTER(ctx);
   if (rows < 0 || n <= 0 || !valid_act_dtype(dtype)) return ZOACT_ERR_INVALID_ARG;

@@ -34,6 +34,7 @@ enum ScratchSlot {
   SLOT_AUG_B,        // 16-bit split of C (+ c_b Z_b) for those K columns (gate and up)
   SLOT_AUG_Z,        // Z of each query, transposed, for the epilogue (C on the tensor cores)
   SLOT_PROJ_TICKETS, // split-K tickets of the tensor-core projection (zero between calls)
+  SLOT_DIAG,         // partial products of the subspace diagnostics
   SLOT_COUNT
 };
 
@@ -172,6 +173,12 @@ int launch_adam(Ctx* ctx, float* C, float* m, float* v, const zoact_coeff_block*
 int launch_rms_norm(Ctx* ctx, const void* X, int dtype, int64_t rows, int n, float eps, void* Y);
 int launch_mix_rms(Ctx* ctx, const void* q, const void* k, const void* v, int dtype, int64_t rows,
                    int n, int n_rep, int head_dim, float eps, void* Y);
+
+// Section 5.3 diagnostics (k_diag.cu): out[0] = ||Ua^T Ub||_F^2, out[2] = out[0] / ra;
+// energy: out[0] = ||U^T G||_F^2, out[1] = ||G||_F^2, out[2] = their ratio.  out: device fp64 [3].
+int launch_subspace_overlap(Ctx* ctx, const float* Ua, const float* Ub, int d, int ra, int rb, double* out);
+int launch_gradient_energy(Ctx* ctx, const float* U, int d_in, int r, const void* G, int gdtype, int64_t n,
+                           double* out);
 
 int run_basis_init(Ctx* ctx, const void* X, int xdtype, int64_t n_tok, int d_in, int r, int oversample,
                    int n_iter, uint64_t seed, float* U_out, float* evals_out);
