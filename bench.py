@@ -159,6 +159,37 @@ def build(ctx, dev, rank, name, tokens=None, n_queries=None):
     return step, x, target, basis_s, w
 
 
+def time_diagnostics(ctx, step, dev, reps=20):
+    """Section 5.3 diagnostics on the first layer's basis: gradient-energy capture of a synthetic bf16
+    gradient shaped like that layer's weight ([d_in, d_out]) and the overlap of the basis with a rotated copy.
+    HBM-bound on G; reported with its achieved GB/s."""
+    import torch
+    import paper_2607_01125_gb300 as zo
+    from synth import normal
+    lin = step.linears[0]
+    G = normal((lin.d_in, lin.d_out), 99, dev, dtype=torch.bfloat16)
+    U2 = torch.linalg.qr(lin.U + 0.1 * normal(tuple(lin.U.shape), 98, dev))[0].contiguous()
+    out = torch.zeros(3, dtype=torch.float64, device=dev)
+    res = {}
+    for name, fn, nbytes in (("gradient_energy", lambda: zo.zoact_gradient_energy(ctx, lin.U, G, out),
+                              G.numel() * G.element_size()),
+                             ("subspace_overlap", lambda: zo.zoact_subspace_overlap(ctx, lin.U, U2, out),
+                              2 * lin.U.numel() * 4)):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        res[name] = {"ms": ms, "GB/s": nbytes / (ms * 1e-3) / 1e9, "value": float(out[2]),
+                     "shape": [lin.d_in, lin.d_out if name == "gradient_energy" else lin.r]}
+    return res
+
+
 def run_step(step, x, target, t, seed, world):
     Y = step.forward(x, seed, t)
     step.loss(Y, target)
@@ -277,6 +308,8 @@ def run_ours(args):
         "clocks": clocks,
         "device_status": status,
     }
+    if args.diag:
+        line["diag"] = time_diagnostics(ctx, step, dev)
     if world == 1 and not args.no_cpu_baseline and args.workload == DEFAULT_WORKLOAD and args.queries is None:
         line["cpu_baseline"] = cpu_baseline(step, budget_s=args.cpu_budget)
     print(json.dumps(line))
@@ -368,6 +401,7 @@ def main():
     ap.add_argument("--tokens", type=int, default=None, help="tokens per perturbation (default: the workload's)")
     ap.add_argument("--queries", type=int, default=None,
                     help="one-sided estimator with this many queries (Algorithm 2); default: two-sided pair")
+    ap.add_argument("--diag", action="store_true", help="also time the Section 5.3 subspace diagnostics")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--soak", type=float, default=2.0,
                     help="seconds of untimed steps before the timed region (clocks reach their loaded state)")

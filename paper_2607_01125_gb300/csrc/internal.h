@@ -145,7 +145,8 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a);
 // Low-rank term of the tensor-core pair forward (see k_aug.cu):
 //   LOWRANK_EPILOGUE  (C + c_b Z_b) p summed in the epilogue (fp32 tables)
 //   LOWRANK_C_ON_TC   C p as extra K columns of the MMA, c_b Z_b p in the epilogue
-//   LOWRANK_ALL_ON_TC (C + c_b Z_b) p as extra K columns (stacked rows whose tiles lie in one block)
+//   LOWRANK_ALL_ON_TC (C + c_b Z_b) p as extra K columns (stacked rows): one K slot when every tile lies in
+//                     one evaluation block, two slots (block parity) when tiles straddle two blocks
 enum LowrankMode { LOWRANK_EPILOGUE = 0, LOWRANK_C_ON_TC = 1, LOWRANK_ALL_ON_TC = 2 };
 // Extra K columns per layer for rank r: the three 16-bit products P_hi T_hi, P_hi T_lo, P_lo T_hi
 // padded to whole 64-column K-blocks.
@@ -153,8 +154,9 @@ inline int aug_cols(int r) { return (3 * r + 63) / 64 * 64; }
 // Writes A_aug [rows, ka_tot] and B_aug / B_aug2 [nbB * d_out, ka_tot] (bf16) for one pair forward.
 // distinct: gate and up have their own projections (A_aug holds both, B_aug zero-pads the other half).
 // Zt / Zt2 (optional): Z of the nzq queries zq, transposed, [nzq][r][d_out] fp32 each.
-int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct, void* A_aug, void* B_aug,
-                    void* B_aug2, float* Zt, float* Zt2, const uint64_t* zq, int nzq);
+// slots (LOWRANK_ALL_ON_TC): 2 puts row t's parts in K slot (block(t) & 1) of an A_aug row of 2 ka columns.
+int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct, int slots, void* A_aug,
+                    void* B_aug, void* B_aug2, float* Zt, float* Zt2, const uint64_t* zq, int nzq);
 int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int M, int N, int K,
                           float* D);
 

@@ -14,7 +14,9 @@
 // holds both ([gate parts | up parts]) and each B_aug zero-fills the other half.
 // B_aug holds one table per evaluation block when the whole term goes to the
 // tensor cores (LOWRANK_ALL_ON_TC: T = C + c_b Z_b, Z_b from the same Philox
-// stream as every other kernel), and the single table T = C otherwise.  With C
+// stream as every other kernel; when a tile's rows straddle two blocks, A_aug
+// has two K slots and row t fills slot block(t) & 1, so each slot meets the
+// table of the block of its parity), and the single table T = C otherwise.  With C
 // on the tensor cores the epilogue still adds c_b Z_b p: for it this kernel
 // also writes Z of every distinct query transposed, Zt[q][j][n] (fp32), so the
 // pair kernel copies its tile's columns instead of regenerating them per tile.
@@ -43,18 +45,23 @@ __device__ __forceinline__ uint32_t pack_bf16x2(__nv_bfloat16 a, __nv_bfloat16 b
 }
 
 // One warp per output row: rows [0, nA) of A_aug, then the nB rows of B_aug
-// (block b, column n), then those of B_aug2.  Lane j < r holds the row's source
-// value j (and of the second projection, distinct gated A rows only); the warp
-// writes the row as bf16 pairs, each lane fetching its K columns' source values
-// by shuffle and splitting them into hi/lo.
+// (block b, column n), then those of B_aug2.  The warp stages the row's r source
+// values (and those of the second projection, distinct gated A rows only) in its
+// slice of shared memory, then writes the row as bf16 pairs, each lane splitting
+// its K columns' source values into hi/lo.  r <= 256.
 __global__ void __launch_bounds__(256)
 aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const float* __restrict__ C,
                 const float* __restrict__ C2, __nv_bfloat16* __restrict__ A, __nv_bfloat16* __restrict__ B,
                 __nv_bfloat16* __restrict__ B2, int64_t rows, int d_out, int r, int ka, int distinct, int full,
                 int nb, const __grid_constant__ AugBlocks blk, uint64_t seed, uint32_t lid, uint32_t lid2,
-                float* __restrict__ Zt, float* __restrict__ Zt2) {
+                float* __restrict__ Zt, float* __restrict__ Zt2, int slots, int64_t T) {
+  __shared__ float stage[8][2][256];
   const int lane = threadIdx.x & 31;
-  const int ka_tot = distinct ? 2 * ka : ka;
+  float* s0 = stage[threadIdx.x >> 5][0];
+  float* s1 = stage[threadIdx.x >> 5][1];
+  const int ka_row = distinct ? 2 * ka : ka;          // columns of one slot
+  const int ka_tot_a = slots * ka_row;                // A_aug row width
+  const int ka_tot = ka_row;                          // B_aug row width
   const int nbB = full ? nb : 1;
   const int64_t nA = rows;
   const int64_t nB = (int64_t)nbB * d_out;
@@ -62,47 +69,49 @@ aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   for (int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; w < total; w += nwarps) {
     const bool is_a = w < nA;
-    float v0 = 0.f, v1 = 0.f;                       // this lane's source value (v1: second half, distinct A)
     bool up = false;
     int64_t orow;
+    __syncwarp();                                    // the previous row's readers are done with the stage
     if (is_a) {
       orow = w;
-      if (lane < r) {
-        v0 = P[w * r + lane];
-        if (distinct) v1 = P2[w * r + lane];
+      for (int j = lane; j < r; j += 32) {
+        s0[j] = P[w * r + j];
+        if (distinct) s1[j] = P2[w * r + j];
       }
     } else {
       const int64_t ib = w - nA;
       up = ib >= nB;
       orow = up ? ib - nB : ib;                      // b * d_out + n
       const int b = (int)(orow / d_out), n = (int)(orow - (int64_t)b * d_out);
-      if (lane < r) {
-        const int64_t e = (int64_t)n * r + lane;
-        v0 = (up ? C2 : C)[e];
-        const float cb = full ? blk.coef[b] : 0.f;
+      const float cb = full ? blk.coef[b] : 0.f;
+      for (int j = lane; j < r; j += 32) {
+        const int64_t e = (int64_t)n * r + j;
+        float v = (up ? C2 : C)[e];
         if (cb != 0.f)
-          v0 = fmaf(cb, z_select(z_normals4(seed, up ? lid2 : lid, blk.qry[b], (uint64_t)(e >> 2)), (int)(e & 3)), v0);
+          v = fmaf(cb, z_select(z_normals4(seed, up ? lid2 : lid, blk.qry[b], (uint64_t)(e >> 2)), (int)(e & 3)), v);
+        s0[j] = v;
       }
     }
+    __syncwarp();
     __nv_bfloat16* dst = is_a ? A : (up ? B2 : B);
-    uint32_t* drow = reinterpret_cast<uint32_t*>(dst + orow * ka_tot);
-    for (int wd = lane; wd < ka_tot / 2; wd += 32) {
+    const int row_w = is_a ? ka_tot_a : ka_tot;
+    const int my_slot = (is_a && slots == 2) ? (int)((orow / T) & 1) : 0;
+    uint32_t* drow = reinterpret_cast<uint32_t*>(dst + orow * row_w);
+    for (int wd = lane; wd < row_w / 2; wd += 32) {
       __nv_bfloat16 o[2];
 #pragma unroll
       for (int e2 = 0; e2 < 2; ++e2) {
-        const int k = 2 * wd + e2;
+        const int slot = (2 * wd + e2) / ka_row;
+        const int k = 2 * wd + e2 - slot * ka_row;
         const int half = k >= ka ? 1 : 0, kk = k - half * ka;
         const int part = kk / r, j = kk - part * r;
         // A: [hi | hi | lo], B: [hi | lo | hi]
         const bool want_lo = is_a ? part == 2 : part == 1;
         const bool second = is_a && half == 1;       // distinct A: the up projection's parts
-        // every lane fetches its column's source value and splits it itself
-        const float a0 = __shfl_sync(0xffffffffu, v0, j & 31);
-        const float a1 = __shfl_sync(0xffffffffu, v1, j & 31);
-        __nv_bfloat16 hi, lo;
-        split16(second ? a1 : a0, hi, lo);
         // distinct gated B: gate rows fill the first half, up rows the second
-        const bool live = part < 3 && (is_a || !distinct || half == (up ? 1 : 0));
+        const bool live = part < 3 && slot == my_slot && (is_a || !distinct || half == (up ? 1 : 0));
+        __nv_bfloat16 hi = __float2bfloat16_rn(0.f), lo = hi;
+        if (live) split16(second ? s1[j] : s0[j], hi, lo);
         o[e2] = live ? (want_lo ? lo : hi) : __float2bfloat16_rn(0.f);
       }
       drow[wd] = pack_bf16x2(o[0], o[1]);
@@ -138,8 +147,8 @@ aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const
 
 }  // namespace
 
-int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct, void* A_aug, void* B_aug,
-                    void* B_aug2, float* Zt, float* Zt2, const uint64_t* zq, int nzq) {
+int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct, int slots, void* A_aug,
+                    void* B_aug, void* B_aug2, float* Zt, float* Zt2, const uint64_t* zq, int nzq) {
   AugBlocks blk{};
   for (int b = 0; b < a.nb; ++b) { blk.coef[b] = a.coef[b]; blk.qry[b] = a.qry[b]; }
   for (int i = 0; i < nzq; ++i) blk.zq[i] = zq[i];
@@ -156,7 +165,7 @@ int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct,
   aug_prep_kernel<<<(unsigned)grid, 256, 0, ctx->stream>>>(
       a.P, distinct ? a.P2 : nullptr, a.C, a.C2, static_cast<__nv_bfloat16*>(A_aug),
       static_cast<__nv_bfloat16*>(B_aug), static_cast<__nv_bfloat16*>(B_aug2), a.rows, a.d_out, a.r, ka, distinct,
-      full, a.nb, blk, a.seed, a.layer_id, a.layer_id2, Zt, Zt2);
+      full, a.nb, blk, a.seed, a.layer_id, a.layer_id2, Zt, Zt2, slots, a.T);
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;

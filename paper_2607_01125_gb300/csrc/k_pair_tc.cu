@@ -131,12 +131,21 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   // low-rank term: on the tensor cores where the context may hold the split operands
   const char* lsel = std::getenv("ZOACT_LOWRANK");
   int lmode = LOWRANK_EPILOGUE;
+  const bool distinct = gated && a.P2 != a.P;
+  int slots = 1;
   if (!w4 && ctx->may_allocate && !(lsel && std::strcmp(lsel, "epilogue") == 0)) {
+    // stacked rows: the whole term on the tensor cores when every tile lies in one block (one K slot) or
+    // straddles at most two (two K slots by block parity); shared inputs keep +-Z p in the epilogue
     const int64_t tile_rows = two ? 2 * BM : BM;
-    lmode = (!a.shared && a.T % tile_rows == 0) ? LOWRANK_ALL_ON_TC : LOWRANK_C_ON_TC;
+    lmode = LOWRANK_C_ON_TC;
+    if (!a.shared && a.T % tile_rows == 0) {
+      lmode = LOWRANK_ALL_ON_TC;
+    } else if (!a.shared && a.T >= tile_rows && !distinct) {
+      lmode = LOWRANK_ALL_ON_TC;
+      slots = 2;
+    }
   }
   const int ka = aug_cols(a.r);
-  const bool distinct = gated && a.P2 != a.P;
   const int ka_tot = distinct ? 2 * ka : ka;
   tm.aa = tm.a; tm.ba = tm.b; tm.ba2 = tm.b2;
   int64_t aug_block_rows = 0;
@@ -158,7 +167,7 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   float* zt2 = nullptr;
   if (lmode != LOWRANK_EPILOGUE) {
     const int64_t nbB = lmode == LOWRANK_ALL_ON_TC ? a.nb : 1;
-    const size_t a_bytes = (size_t)a.rows * ka_tot * 2;
+    const size_t a_bytes = (size_t)a.rows * slots * ka_tot * 2;
     const size_t b_bytes = (size_t)nbB * a.d_out * ka_tot * 2;
     uint8_t* abuf = static_cast<uint8_t*>(scratch(ctx, SLOT_AUG_A, a_bytes));
     uint8_t* bbuf = static_cast<uint8_t*>(scratch(ctx, SLOT_AUG_B, (gated ? 2 : 1) * b_bytes));
@@ -170,9 +179,9 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
       if (!zt) return ZOACT_ERR_NOMEM;
       zt2 = gated ? zt + z_floats : nullptr;
     }
-    st = launch_aug_prep(ctx, a, lmode, ka, distinct ? 1 : 0, abuf, bbuf, bbuf2, zt, zt2, zq_list, nzq);
+    st = launch_aug_prep(ctx, a, lmode, ka, distinct ? 1 : 0, slots, abuf, bbuf, bbuf2, zt, zt2, zq_list, nzq);
     if (st) return st;
-    st = encode_tmap_2d_16bit(&tm.aa, abuf, ZOACT_DT_BF16, a.rows, ka_tot, BM);
+    st = encode_tmap_2d_16bit(&tm.aa, abuf, ZOACT_DT_BF16, a.rows, (int64_t)slots * ka_tot, BM);
     if (st) return st;
     st = encode_tmap_2d_16bit(&tm.ba, bbuf, ZOACT_DT_BF16, nbB * a.d_out, ka_tot, b_box);
     if (st) return st;
@@ -202,7 +211,9 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   p.num_tiles = p.num_m * p.num_n;
   p.ldy = a.d_out;
   p.aug_mode = lmode;
-  p.aug_kb = lmode == LOWRANK_EPILOGUE ? 0 : ka_tot / BK;
+  p.aug_kb = lmode == LOWRANK_EPILOGUE ? 0 : slots * ka_tot / BK;
+  p.aug_kb_slot = ka_tot / BK;
+  p.aug_slots = slots;
   p.aug_block_rows = aug_block_rows;
   p.Zt = zt;
   p.Zt2 = zt2;

@@ -170,9 +170,6 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       for (int tile = cluster_id; tile < prm.num_tiles && ok; tile += n_clusters) {
         int m_blk, n_blk;
         tile_coords(tile, num_m, num_n, m_blk, n_blk);
-        // low-rank K-blocks read the table of the tile's evaluation block (whole term on the tensor cores)
-        const int aug_row0 = prm.aug_mode == LOWRANK_ALL_ON_TC
-                                 ? (int)(((int64_t)m_blk * BM2 / prm.T) * prm.aug_block_rows) : 0;
         for (int kb = 0; kb < total_k; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
           const uint32_t full_leader = tc2::map_to(tc::smem_u32(&ss->full[stage]), 0);
@@ -180,14 +177,14 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
           const uint32_t sa = tc::smem_u32(smem + stage * STAGE2_BYTES);
           const uint32_t sb = sa + A_BYTES;
           const bool aug = kb >= num_k;
-          const int kx = (aug ? kb - num_k : kb) * BK;
-          const int yb = aug ? aug_row0 : 0;
+          int kx = kb * BK, kxb = kb * BK, yb = 0;
+          if (aug) aug_coords(prm, (int64_t)m_blk * BM2, BM2, kb - num_k, kx, kxb, yb);
           tc2::tma_load_2d_pair(sa, aug ? &tm.aa : &tm.a, kx, m_blk * BM2 + (int)rank * BM, full_leader);
           if (MODE == MODE_GATED)
-            tc2::tma_load_2d_pair(sb, aug ? (leader ? &tm.ba : &tm.ba2) : (leader ? &tm.b : &tm.b2), kx,
+            tc2::tma_load_2d_pair(sb, aug ? (leader ? &tm.ba : &tm.ba2) : (leader ? &tm.b : &tm.b2), kxb,
                                   yb + n_blk * (BN / 2), full_leader);
           else
-            tc2::tma_load_2d_pair(sb, aug ? &tm.ba : &tm.b, kx, yb + n_blk * bn + (int)rank * bh, full_leader);
+            tc2::tma_load_2d_pair(sb, aug ? &tm.ba : &tm.b, kxb, yb + n_blk * bn + (int)rank * bh, full_leader);
           if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
         }
       }

@@ -56,6 +56,7 @@ namespace zoact {
 namespace pairtc {
 
 constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int BK_AUG = BK;   // K columns per low-rank K-block
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
@@ -105,6 +106,8 @@ struct Params {
   int num_m, num_n, num_k, num_tiles;
   int aug_mode;      // LowrankMode
   int aug_kb;        // extra K-blocks per tile from A_aug / B_aug (0 with LOWRANK_EPILOGUE)
+  int aug_kb_slot;   // K-blocks of one slot (B_aug row width / 64)
+  int aug_slots;     // LOWRANK_ALL_ON_TC: 1, or 2 when tiles straddle two evaluation blocks
   int64_t aug_block_rows;   // rows of one block's table in B_aug (LOWRANK_ALL_ON_TC)
   // LOWRANK_C_ON_TC: Z of each distinct query, transposed [q][r][d_out] (gate / up), and the table of each block
   const float* Zt;
@@ -133,6 +136,23 @@ struct SharedState {
   int epi_ok;
 };
 static_assert(sizeof(SharedState) <= 256, "barrier block outgrew its shared-memory slot");
+
+// TMA coordinates of low-rank K-block `ka` (0 .. aug_kb) of a tile whose rows start at tile_row0:
+// x in A_aug (slots side by side), x in B_aug (one slot wide), and the first B_aug row of the table the
+// slot meets -- the tile's block (one slot), or the tile's block of the slot's parity (two slots).
+__device__ __forceinline__ void aug_coords(const Params& prm, int64_t tile_row0, int tile_rows, int ka, int& kx_a,
+                                           int& kx_b, int& y_b) {
+  const int slot = ka / prm.aug_kb_slot;
+  kx_a = ka * BK_AUG;
+  kx_b = (ka - slot * prm.aug_kb_slot) * BK_AUG;
+  y_b = 0;
+  if (prm.aug_mode == LOWRANK_ALL_ON_TC) {
+    const int b_lo = (int)(tile_row0 / prm.T);
+    const int b_hi = (int)((min(tile_row0 + tile_rows, prm.rows) - 1) / prm.T);
+    const int blk = prm.aug_slots == 1 ? b_lo : (((b_lo & 1) == slot) ? b_lo : min(b_lo + 1, b_hi));
+    y_b = (int)(blk * prm.aug_block_rows);
+  }
+}
 
 __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& m_blk, int& n_blk) {
   const int per_group = GROUP_M * num_n;
@@ -657,9 +677,6 @@ pair_tc_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       for (int tile = blockIdx.x; tile < prm.num_tiles && ok; tile += gridDim.x) {
         int m_blk, n_blk;
         tile_coords(tile, num_m, num_n, m_blk, n_blk);
-        // low-rank K-blocks read the table of the tile's evaluation block (whole term on the tensor cores)
-        const int aug_row0 = prm.aug_mode == LOWRANK_ALL_ON_TC
-                                 ? (int)(((int64_t)m_blk * BM / prm.T) * prm.aug_block_rows) : 0;
         for (int kb = 0; kb < total_k; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
           const uint32_t full = tc::smem_u32(&ss->full[stage]);
@@ -667,16 +684,16 @@ pair_tc_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
           const uint32_t sa = tc::smem_u32(smem + stage * STAGE_BYTES);
           const uint32_t sb = sa + A_BYTES;
           const bool aug = kb >= num_k;
-          const int kx = (aug ? kb - num_k : kb) * BK;
-          const int yb = aug ? aug_row0 : 0;
+          int kx = kb * BK, kxb = kb * BK, yb = 0;
+          if (aug) aug_coords(prm, (int64_t)m_blk * BM, BM, kb - num_k, kx, kxb, yb);
           tc::tma_load_2d(sa, aug ? &tm.aa : &tm.a, kx, m_blk * BM, full);
           if (W4) {
             // B arrives from the dequantising warps
           } else if (MODE == MODE_GATED) {
-            tc::tma_load_2d(sb, aug ? &tm.ba : &tm.b, kx, yb + n_blk * (BN / 2), full);
-            tc::tma_load_2d(sb + B_BYTES / 2, aug ? &tm.ba2 : &tm.b2, kx, yb + n_blk * (BN / 2), full);
+            tc::tma_load_2d(sb, aug ? &tm.ba : &tm.b, kxb, yb + n_blk * (BN / 2), full);
+            tc::tma_load_2d(sb + B_BYTES / 2, aug ? &tm.ba2 : &tm.b2, kxb, yb + n_blk * (BN / 2), full);
           } else {
-            tc::tma_load_2d(sb, aug ? &tm.ba : &tm.b, kx, yb + n_blk * bn, full);
+            tc::tma_load_2d(sb, aug ? &tm.ba : &tm.b, kxb, yb + n_blk * bn, full);
           }
           issued_mask |= 1u << stage;
           issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);

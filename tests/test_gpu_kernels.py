@@ -118,11 +118,13 @@ def test_pair_forward_fp32_out(ctx, d_in, d_out, r, T, shared, dt):
 @pytest.mark.parametrize("T,shared,lowrank,kernel", [
     (256, False, "auto", "auto"),        # stacked, tiles inside one block: whole low-rank term on the tensor cores
     (256, False, "epilogue", "auto"),    # the same in fp32 epilogue tables
-    (200, False, "auto", "auto"),        # stacked, tiles across the sign boundary: C p on the tensor cores
+    (200, False, "auto", "auto"),        # stacked, T below the tile height: C p on the tensor cores
+    (300, False, "auto", "auto"),        # stacked, tiles across the sign boundary: two K slots by block parity
     (300, True, "auto", "auto"),         # shared input: C p on the tensor cores, +-eps Z p in the epilogue
     (300, True, "epilogue", "auto"),
     (128, False, "auto", "1cta"),        # one-CTA kernel with the whole term on the tensor cores
     (100, False, "auto", "1cta"),
+    (200, False, "auto", "1cta"),        # one-CTA tiles across the sign boundary: two K slots
 ])
 @pytest.mark.parametrize("gated", [False, True])
 def test_pair_forward_lowrank_modes(ctx, monkeypatch, T, shared, lowrank, kernel, gated):

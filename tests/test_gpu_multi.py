@@ -62,6 +62,7 @@ def _oracle(Wn, Un, Cn, Xn, points, T, shared, seed, lid):
     (768, 512, 16, 300, 9, True, torch.bfloat16),     # shared: 9 outputs per accumulator row, 5 passes
     (512, 264, 8, 40, 3, False, torch.float16),       # 120 rows: one-CTA tiles
     (1024, 520, 16, 256, 9, False, torch.bfloat16),   # tiles inside one block: whole term on the tensor cores
+    (1024, 520, 16, 300, 9, False, torch.bfloat16),   # tiles across two blocks: two K slots by block parity
     (4096, 1024, 32, 160, 5, False, torch.bfloat16),  # rank 32: two table chunks per tile
     (256, 200, 8, 37, 4, False, torch.float32),       # fp32 weights: CUDA-core kernel
     (256, 256, 8, 64, 6, True, torch.float32),
