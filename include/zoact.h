@@ -71,7 +71,8 @@ typedef struct zoact_ctx zoact_ctx;
 typedef struct zoact_layer {
   int32_t d_in;        /* input width  (the paper's m) */
   int32_t d_out;       /* output width (the paper's n) */
-  int32_t r;           /* basis rank, 1 <= r <= 32 in this build */
+  int32_t r;           /* basis rank, 1 <= r <= 256 (above 32 with 16-bit activations only when
+                          the pair forward may use context scratch; see zoact_pair_forward) */
   int32_t wtype;       /* ZOACT_DT_* of W */
   const void* W;       /* frozen weight [d_out, d_in] row-major.  INT4_G128:
                           [d_out, d_in/2] bytes, element k in byte k/2, low nibble
@@ -128,7 +129,7 @@ int zoact_philox_normals(zoact_ctx* ctx, uint64_t seed, uint32_t layer_id, uint6
                          int64_t n, float* z_out, uint32_t* words_out);
 
 /* ---- the low-rank projection p = U^T x (Section 3: the factor X V_r) ----
- * X [rows, d_in] of xdtype (FP32/BF16/FP16), U [d_in, r] fp32 -> P [rows, r] fp32.
+ * X [rows, d_in] of xdtype (FP32/BF16/FP16), U [d_in, r] fp32 -> P [rows, r] fp32, r <= 256.
  * d_in % 8 == 0 for BF16/FP16, % 4 for FP32.                                    */
 int zoact_lowrank_proj(zoact_ctx* ctx, const void* X, int xdtype, int64_t rows, int32_t d_in,
                        const float* U, int32_t r, float* P);
@@ -142,7 +143,7 @@ int zoact_lowrank_proj(zoact_ctx* ctx, const void* X, int xdtype, int64_t rows, 
  * the dtype of the X it will multiply; d_in % 8 == 0) so that
  * zoact_lowrank_proj_prepared computes P = X U from it without re-splitting U.
  * U_tc must be prepared again if U changes.  zoact_basis_prepared_bytes returns -1
- * for unsupported sizes (r > 32).                                               */
+ * for unsupported sizes (r > 256).                                              */
 int64_t zoact_basis_prepared_bytes(int32_t d_in, int32_t r);
 int zoact_basis_prepare(zoact_ctx* ctx, const float* U, int32_t d_in, int32_t r, int32_t xdtype,
                         void* U_tc);
@@ -161,7 +162,9 @@ int zoact_lowrank_proj_prepared(zoact_ctx* ctx, const void* X, int xdtype, int64
  * zoact_lowrank_proj, or shared by layers with the same input and basis); when
  * NULL the call computes it into context scratch first.
  * Requirements: d_in % 8 == 0 (BF16/FP16), d_in % 128 == 0 (INT4), d_out % 8 == 0,
- * 16-byte aligned X, W, Y.                                                       */
+ * 16-byte aligned X, W, Y.  Ranks above 32 (16-bit X) add the whole low-rank term on
+ * the tensor cores, which needs stacked rows: a shared input is first copied once
+ * per sign into context scratch.                                                 */
 int zoact_pair_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype,
                        int64_t T, int input_shared, const float* P, float eps, uint64_t seed,
                        uint64_t query, int act, void* Y, int ydtype);

@@ -76,7 +76,7 @@ bool valid_act_dtype(int dt) { return dt == ZOACT_DT_FP32 || dt == ZOACT_DT_BF16
 int check_layer(const zoact_layer* L) {
   if (!L || !L->W || !L->U || !L->C) return ZOACT_ERR_INVALID_ARG;
   if (L->d_in <= 0 || L->d_out <= 0 || L->r <= 0) return ZOACT_ERR_INVALID_ARG;
-  if (L->r > 32) return ZOACT_ERR_UNSUPPORTED;
+  if (L->r > 256) return ZOACT_ERR_UNSUPPORTED;
   if ((int64_t)L->d_out * L->r >= (int64_t)1 << 34) return ZOACT_ERR_INVALID_ARG;
   if (L->wtype == ZOACT_DT_INT4_G128) {
     if (!L->w_scales || L->d_in % 128 != 0 || ((uintptr_t)L->W & 15u) != 0) return ZOACT_ERR_INVALID_ARG;
@@ -192,7 +192,7 @@ int zoact_lowrank_proj(zoact_ctx* ctx, const void* X, int xdtype, int64_t rows, 
                        int32_t r, float* P) {
   ZOACT_ENTER(ctx);
   if (rows < 0 || d_in <= 0 || r <= 0 || !valid_act_dtype(xdtype)) return ZOACT_ERR_INVALID_ARG;
-  if (r > 32) return ZOACT_ERR_UNSUPPORTED;
+  if (r > 256) return ZOACT_ERR_UNSUPPORTED;
   if (rows == 0) return ZOACT_OK;
   if (!X || !U || !P || !aligned16(X)) return ZOACT_ERR_INVALID_ARG;
   if (d_in % (xdtype == ZOACT_DT_FP32 ? 4 : 8) != 0) return ZOACT_ERR_INVALID_ARG;
@@ -216,14 +216,14 @@ static zoact_eval_blocks pair_blocks(float eps, uint64_t query) {
 }
 
 int64_t zoact_basis_prepared_bytes(int32_t d_in, int32_t r) {
-  if (d_in <= 0 || r <= 0 || r > 32) return -1;
+  if (d_in <= 0 || r <= 0 || r > 256) return -1;
   return (int64_t)basis_tc_rows(r) * d_in * 2;
 }
 
 int zoact_basis_prepare(zoact_ctx* ctx, const float* U, int32_t d_in, int32_t r, int32_t xdtype, void* U_tc) {
   ZOACT_ENTER(ctx);
   if (!U || !U_tc || d_in <= 0 || r <= 0) return ZOACT_ERR_INVALID_ARG;
-  if (r > 32) return ZOACT_ERR_UNSUPPORTED;
+  if (r > 256) return ZOACT_ERR_UNSUPPORTED;
   if (xdtype != ZOACT_DT_BF16 && xdtype != ZOACT_DT_FP16) return ZOACT_ERR_INVALID_ARG;
   if (d_in % 8 != 0 || !aligned16(U_tc)) return ZOACT_ERR_INVALID_ARG;
   return launch_basis_prepare(ctx, U, d_in, r, xdtype, U_tc);
@@ -233,7 +233,7 @@ int zoact_lowrank_proj_prepared(zoact_ctx* ctx, const void* X, int xdtype, int64
                                 const void* U_tc, int32_t r, float* P) {
   ZOACT_ENTER(ctx);
   if (rows < 0 || d_in <= 0 || r <= 0) return ZOACT_ERR_INVALID_ARG;
-  if (r > 32) return ZOACT_ERR_UNSUPPORTED;
+  if (r > 256) return ZOACT_ERR_UNSUPPORTED;
   if (xdtype != ZOACT_DT_BF16 && xdtype != ZOACT_DT_FP16) return ZOACT_ERR_INVALID_ARG;
   if (rows == 0) return ZOACT_OK;
   if (!X || !U_tc || !P || !aligned16(X) || !aligned16(U_tc) || d_in % 8 != 0) return ZOACT_ERR_INVALID_ARG;

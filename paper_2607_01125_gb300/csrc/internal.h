@@ -35,6 +35,7 @@ enum ScratchSlot {
   SLOT_AUG_Z,        // Z of each query, transposed, for the epilogue (C on the tensor cores)
   SLOT_PROJ_TICKETS, // split-K tickets of the tensor-core projection (zero between calls)
   SLOT_DIAG,         // partial products of the subspace diagnostics
+  SLOT_STACKED_X,    // a shared input and its projection copied once per evaluation block (ranks above 32)
   SLOT_COUNT
 };
 
@@ -154,7 +155,7 @@ inline int aug_cols(int r) { return (3 * r + 63) / 64 * 64; }
 // Writes A_aug [rows, ka_tot] and B_aug / B_aug2 [nbB * d_out, ka_tot] (bf16) for one pair forward.
 // distinct: gate and up have their own projections (A_aug holds both, B_aug zero-pads the other half).
 // Zt / Zt2 (optional): Z of the nzq queries zq, transposed, [nzq][r][d_out] fp32 each.
-// slots (LOWRANK_ALL_ON_TC): 2 puts row t's parts in K slot (block(t) & 1) of an A_aug row of 2 ka columns.
+// slots (LOWRANK_ALL_ON_TC): S > 1 puts row t's parts in K slot block(t) mod S of an A_aug row of S ka columns.
 int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct, int slots, void* A_aug,
                     void* B_aug, void* B_aug2, float* Zt, float* Zt2, const uint64_t* zq, int nzq);
 int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int M, int N, int K,

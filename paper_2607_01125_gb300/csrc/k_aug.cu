@@ -14,9 +14,9 @@
 // holds both ([gate parts | up parts]) and each B_aug zero-fills the other half.
 // B_aug holds one table per evaluation block when the whole term goes to the
 // tensor cores (LOWRANK_ALL_ON_TC: T = C + c_b Z_b, Z_b from the same Philox
-// stream as every other kernel; when a tile's rows straddle two blocks, A_aug
-// has two K slots and row t fills slot block(t) & 1, so each slot meets the
-// table of the block of its parity), and the single table T = C otherwise.  With C
+// stream as every other kernel; when a tile's rows span up to S blocks, A_aug
+// has S K slots and row t fills slot block(t) mod S, so each slot meets the
+// table of the tile's block congruent to it), and the single table T = C otherwise.  With C
 // on the tensor cores the epilogue still adds c_b Z_b p: for it this kernel
 // also writes Z of every distinct query transposed, Zt[q][j][n] (fp32), so the
 // pair kernel copies its tile's columns instead of regenerating them per tile.
@@ -95,7 +95,7 @@ aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const
     __syncwarp();
     __nv_bfloat16* dst = is_a ? A : (up ? B2 : B);
     const int row_w = is_a ? ka_tot_a : ka_tot;
-    const int my_slot = (is_a && slots == 2) ? (int)((orow / T) & 1) : 0;
+    const int my_slot = (is_a && slots > 1) ? (int)((orow / T) % slots) : 0;
     uint32_t* drow = reinterpret_cast<uint32_t*>(dst + orow * row_w);
     for (int wd = lane; wd < row_w / 2; wd += 32) {
       __nv_bfloat16 o[2];

@@ -6,9 +6,9 @@
 // graph), which are latency-bound.  64x64 output tile per 256-thread block,
 // 4x4 register tile per thread, K staged through shared memory in chunks of 16.
 // The epilogue builds the table C + c_b Z_b of the tile's columns in shared
-// memory for one block at a time (Z from the shared Philox generator) and adds
-// the low-rank term in fp32: stacked rows use their own block, shared rows are
-// written once per block.
+// memory for one block and 32 ranks at a time (Z from the shared Philox
+// generator) and adds the low-rank term in fp32: stacked rows use their own
+// block, shared rows are written once per block.
 #include "internal.h"
 #include "philox.cuh"
 
@@ -17,7 +17,7 @@ namespace {
 
 constexpr int SB = 64;   // tile rows and cols
 constexpr int SK = 16;   // K chunk
-constexpr int SR = 32;   // max rank
+constexpr int SR = 32;   // ranks per epilogue table chunk
 
 struct EvalBlocks {
   int nb;
@@ -69,40 +69,42 @@ pair_simt_kernel(const float* __restrict__ X, const float* __restrict__ W, const
     b_first = (int)(m0 / T);
     b_last = (int)(last / T);
   }
-  const int64_t e0 = (int64_t)n0 * r;  // multiple of 4 (n0 is a multiple of 64)
   const int n_cols = min(SB, d_out - n0);
-  const int n_elem = n_cols * r;
   for (int b = b_first; b <= b_last; ++b) {
-    // ---- table C + c_b Z_b for the tile's columns, [col][j] ----
     const float cb = blk.coef[b];
-    __syncthreads();
-    for (int g = tid; g < (n_elem + 3) / 4; g += 256) {
-      const float4 z = cb != 0.f ? z_normals4(seed, layer_id, blk.qry[b], (uint64_t)((e0 >> 2) + g))
-                                 : make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
+    float sl[4][4] = {};
+    // the low-rank term in chunks of SR ranks: table C + c_b Z_b of the tile's columns, [col][j]
+    for (int jc = 0; jc < r; jc += SR) {
+      const int rc = min(SR, r - jc);
+      __syncthreads();
+      for (int idx = tid; idx < n_cols * rc; idx += 256) {
+        const int c = idx / rc, j = jc + idx % rc;
+        const int64_t e = (int64_t)(n0 + c) * r + j;
+        const float z = cb != 0.f ? z_select(z_normals4(seed, layer_id, blk.qry[b], (uint64_t)(e >> 2)), (int)(e & 3))
+                                  : 0.f;
+        Tt[c * SR + (j - jc)] = fmaf(cb, z, Cg[e]);
+      }
+      __syncthreads();
       for (int i = 0; i < 4; ++i) {
-        const int idx = 4 * g + i;
-        if (idx < n_elem) Tt[idx] = fmaf(cb, z_select(z, i), Cg[e0 + idx]);
+        const int64_t m = m0 + ty * 4 + i;
+        if (m >= rows || (!shared_in && m / T != b)) continue;
+        for (int jj = 0; jj < rc; ++jj) {
+          const float pj = P[m * r + jc + jj];
+#pragma unroll
+          for (int jc4 = 0; jc4 < 4; ++jc4) {
+            const int c = tx * 4 + jc4;
+            if (c < n_cols) sl[i][jc4] = fmaf(Tt[c * SR + jj], pj, sl[i][jc4]);
+          }
+        }
       }
     }
-    __syncthreads();
     for (int i = 0; i < 4; ++i) {
       const int64_t m = m0 + ty * 4 + i;
-      if (m >= rows) continue;
-      if (!shared_in && m / T != b) continue;
-      float p[SR];
-#pragma unroll
-      for (int j = 0; j < SR; ++j) p[j] = j < r ? P[m * r + j] : 0.f;
+      if (m >= rows || (!shared_in && m / T != b)) continue;
       const int64_t row = shared_in ? (int64_t)b * T + m : m;
-      for (int jc = 0; jc < 4; ++jc) {
-        const int c = tx * 4 + jc;
-        const int n = n0 + c;
-        if (n >= d_out) continue;
-        float sl = 0.f;
-#pragma unroll
-        for (int j = 0; j < SR; ++j)
-          if (j < r) sl = fmaf(Tt[c * r + j], p[j], sl);
-        Y[row * d_out + n] = apply_act(acc[i][jc] + sl, act);
+      for (int jc4 = 0; jc4 < 4; ++jc4) {
+        const int n = n0 + tx * 4 + jc4;
+        if (n < d_out) Y[row * d_out + n] = apply_act(acc[i][jc4] + sl[i][jc4], act);
       }
     }
   }
@@ -113,7 +115,7 @@ pair_simt_kernel(const float* __restrict__ X, const float* __restrict__ W, const
 int launch_pair_simt(Ctx* ctx, const PairArgs& a) {
   if (a.xdtype != ZOACT_DT_FP32 || a.wtype != ZOACT_DT_FP32 || a.ydtype != ZOACT_DT_FP32)
     return ZOACT_ERR_UNSUPPORTED;
-  if (a.r > SR || a.W2) return ZOACT_ERR_UNSUPPORTED;
+  if (a.W2) return ZOACT_ERR_UNSUPPORTED;
   EvalBlocks blk{};
   blk.nb = a.nb;
   for (int b = 0; b < a.nb; ++b) { blk.coef[b] = a.coef[b]; blk.qry[b] = a.qry[b]; }

@@ -77,7 +77,35 @@ int encode_tmap_2d_16bit(CUtensorMap* map, const void* base, int dtype, int64_t 
 
 int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   using namespace pairtc;
-  if (a.wtype == ZOACT_DT_INT4_G128 && a.rows >= INT4_STAGED_MIN_ROWS) {
+  // ranks above 32 have no epilogue tables: the low-rank term must ride the MMA, which needs stacked rows
+  const bool big_r = a.r > 32;
+  if (big_r && !ctx->may_allocate) return ZOACT_ERR_UNSUPPORTED;
+  if (big_r && a.shared) {
+    // a shared input is copied once per evaluation block (and its projection with it), then run stacked
+    const size_t x_bytes = (size_t)a.T * a.d_in * dtype_size(a.xdtype);
+    const size_t p_bytes = (size_t)a.T * a.r * sizeof(float);
+    const int np = a.W2 && a.P2 != a.P ? 2 : 1;
+    uint8_t* buf = static_cast<uint8_t*>(scratch(ctx, SLOT_STACKED_X, a.nb * (x_bytes + np * p_bytes) + 1024));
+    if (!buf) return ZOACT_ERR_NOMEM;
+    uint8_t* xs = buf;
+    float* ps = reinterpret_cast<float*>(buf + (a.nb * x_bytes + 255) / 256 * 256);
+    float* ps2 = np == 2 ? ps + (size_t)a.nb * a.T * a.r : ps;
+    for (int b = 0; b < a.nb; ++b) {
+      ZOACT_CUDA_TRY(cudaMemcpyAsync(xs + b * x_bytes, a.X, x_bytes, cudaMemcpyDeviceToDevice, ctx->stream));
+      ZOACT_CUDA_TRY(cudaMemcpyAsync(ps + (size_t)b * a.T * a.r, a.P, p_bytes, cudaMemcpyDeviceToDevice, ctx->stream));
+      if (np == 2)
+        ZOACT_CUDA_TRY(cudaMemcpyAsync(ps2 + (size_t)b * a.T * a.r, a.P2, p_bytes, cudaMemcpyDeviceToDevice,
+                                       ctx->stream));
+    }
+    PairArgs b = a;
+    b.X = xs;
+    b.P = ps;
+    b.P2 = a.W2 ? ps2 : nullptr;
+    b.shared = 0;
+    b.rows = (int64_t)a.nb * a.T;
+    return launch_pair_tc(ctx, b);
+  }
+  if (a.wtype == ZOACT_DT_INT4_G128 && (a.rows >= INT4_STAGED_MIN_ROWS || big_r)) {
     // staged INT4: expand W (and W2) to bf16 in context scratch, then the bf16 kernel
     const size_t bytes = (size_t)a.d_out * a.d_in * 2;
     void* wb = scratch(ctx, SLOT_WDQ0, bytes);
@@ -103,7 +131,8 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   if (w4 ? a.xdtype != ZOACT_DT_BF16 : a.wtype != a.xdtype) return ZOACT_ERR_UNSUPPORTED;
   if (a.ydtype != a.xdtype && a.ydtype != ZOACT_DT_FP32) return ZOACT_ERR_UNSUPPORTED;
   const bool gated = a.W2 != nullptr;
-  const int rt = rank_template(a.r);
+  // epilogue-table rank template; above 32 ranks (whole term on the tensor cores) the tables are unused
+  const int rt = big_r ? (gated ? 16 : 32) : rank_template(a.r);
   if (gated && rt > 16) return ZOACT_ERR_UNSUPPORTED;
   if (a.rows <= 0) return ZOACT_OK;
   TmaSet tm;
@@ -133,18 +162,21 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   int lmode = LOWRANK_EPILOGUE;
   const bool distinct = gated && a.P2 != a.P;
   int slots = 1;
-  if (!w4 && ctx->may_allocate && !(lsel && std::strcmp(lsel, "epilogue") == 0)) {
-    // stacked rows: the whole term on the tensor cores when every tile lies in one block (one K slot) or
-    // straddles at most two (two K slots by block parity); shared inputs keep +-Z p in the epilogue
+  if (!w4 && ctx->may_allocate && (big_r || !(lsel && std::strcmp(lsel, "epilogue") == 0))) {
+    // stacked rows: the whole term on the tensor cores -- one K slot when every tile lies in one evaluation
+    // block, else S slots (block index mod S) with S the most blocks a tile can span; shared inputs keep
+    // +-Z p in the epilogue (C p on the tensor cores)
     const int64_t tile_rows = two ? 2 * BM : BM;
     lmode = LOWRANK_C_ON_TC;
-    if (!a.shared && a.T % tile_rows == 0) {
+    if (!a.shared) {
       lmode = LOWRANK_ALL_ON_TC;
-    } else if (!a.shared && a.T >= tile_rows && !distinct) {
-      lmode = LOWRANK_ALL_ON_TC;
-      slots = 2;
+      if (a.T % tile_rows != 0) {
+        const int64_t span = (tile_rows - 1) / a.T + 2;
+        slots = (int)(span < a.nb ? span : a.nb);
+      }
     }
   }
+  if (big_r && lmode != LOWRANK_ALL_ON_TC) return ZOACT_ERR_UNSUPPORTED;
   const int ka = aug_cols(a.r);
   const int ka_tot = distinct ? 2 * ka : ka;
   tm.aa = tm.a; tm.ba = tm.b; tm.ba2 = tm.b2;

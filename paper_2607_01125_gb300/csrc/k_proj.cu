@@ -68,10 +68,11 @@ __device__ __forceinline__ void load_x_chunk<__half>(float (*Xs)[PROJ_KC + 1], c
 }
 
 // RPAD: basis columns padded to a power of two >= 4; blockDim = 32 * RPAD / 4.
+// r columns of U (row stride ldu) -> out rows of stride ld_out (split s at out + s * rows * ld_out).
 template <typename TX, int RPAD>
 __global__ void __launch_bounds__(8 * RPAD)
 proj_kernel(const TX* __restrict__ X, const float* __restrict__ U, float* __restrict__ out, int64_t rows,
-            int d_in, int r, int k_per_split) {
+            int d_in, int r, int k_per_split, int ldu, int ld_out) {
   constexpr int NCG = RPAD / 4;        // column groups
   constexpr int NT = 32 * NCG;         // threads
   __shared__ float Xs[PROJ_RB][PROJ_KC + 1];
@@ -95,7 +96,7 @@ proj_kernel(const TX* __restrict__ X, const float* __restrict__ U, float* __rest
     for (int v = tid; v < PROJ_KC * RPAD; v += NT) {
       const int kk = v / RPAD, j = v % RPAD;
       const int k = k0 + kk;
-      Us[kk][j] = (k < k_end && j < r) ? U[(int64_t)k * r + j] : 0.f;
+      Us[kk][j] = (k < k_end && j < r) ? U[(int64_t)k * ldu + j] : 0.f;
     }
     __syncthreads();
 #pragma unroll 8
@@ -111,7 +112,7 @@ proj_kernel(const TX* __restrict__ X, const float* __restrict__ U, float* __rest
       }
     }
   }
-  float* dst = out + (int64_t)split * rows * r;
+  float* dst = out + (int64_t)split * rows * ld_out;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const int64_t row = row0 + rg * 4 + i;
@@ -119,17 +120,19 @@ proj_kernel(const TX* __restrict__ X, const float* __restrict__ U, float* __rest
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
       const int j = cg * 4 + c;
-      if (j < r) dst[row * r + j] = acc[i][c];
+      if (j < r) dst[row * ld_out + j] = acc[i][c];
     }
   }
 }
 
+// P[t, j0 + j] (row stride ldp) = sum over splits of part[split][t][j], j < rg, in split order.
 __global__ void splitk_reduce_kernel(const float* __restrict__ part, float* __restrict__ P, int64_t n,
-                                     int splits) {
+                                     int splits, int rg, int ldp, int j0) {
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
     float s = 0.f;
     for (int k = 0; k < splits; ++k) s += part[(int64_t)k * n + i];
-    P[i] = s;
+    const int64_t t = i / rg;
+    P[t * ldp + j0 + (i - t * rg)] = s;
   }
 }
 
@@ -144,26 +147,35 @@ int proj_dispatch(Ctx* ctx, const TX* X, int64_t rows, int d_in, const float* U,
   int k_per_split = (d_in + splits - 1) / splits;
   k_per_split = (k_per_split + PROJ_KC - 1) / PROJ_KC * PROJ_KC;
   splits = (d_in + k_per_split - 1) / k_per_split;
-  float* out = P;
-  if (splits > 1) {
-    out = static_cast<float*>(scratch(ctx, SLOT_SPLITK, (size_t)splits * rows * r * sizeof(float)));
-    if (!out) return ZOACT_ERR_NOMEM;
-  }
   dim3 grid((unsigned)row_blocks, (unsigned)splits);
-  int rp = r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32;
-  switch (rp) {
-    case 4: proj_kernel<TX, 4><<<grid, 32, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); ++ctx->n_launch; break;
-    case 8: proj_kernel<TX, 8><<<grid, 64, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); ++ctx->n_launch; break;
-    case 16: proj_kernel<TX, 16><<<grid, 128, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); ++ctx->n_launch; break;
-    default: proj_kernel<TX, 32><<<grid, 256, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); ++ctx->n_launch; break;
-  }
-  ZOACT_CHECK_LAUNCH();
-  if (splits > 1) {
-    const int64_t n = rows * r;
-    int64_t blocks = (n + 255) / 256;
-    if (blocks > 4LL * ctx->sm_count) blocks = 4LL * ctx->sm_count;
-    splitk_reduce_kernel<<<(unsigned)blocks, 256, 0, ctx->stream>>>(out, P, n, splits); ++ctx->n_launch;
+  // groups of up to 32 basis columns, one launch each
+  for (int j0 = 0; j0 < r; j0 += 32) {
+    const int rg = r - j0 < 32 ? r - j0 : 32;
+    float* out = P + j0;
+    int ld_out = r;
+    if (splits > 1) {
+      out = static_cast<float*>(scratch(ctx, SLOT_SPLITK, (size_t)splits * rows * rg * sizeof(float)));
+      if (!out) return ZOACT_ERR_NOMEM;
+      ld_out = rg;
+    }
+    const float* Ug = U + j0;
+    const int rp = rg <= 4 ? 4 : rg <= 8 ? 8 : rg <= 16 ? 16 : 32;
+    switch (rp) {
+      case 4: proj_kernel<TX, 4><<<grid, 32, 0, ctx->stream>>>(X, Ug, out, rows, d_in, rg, k_per_split, r, ld_out); break;
+      case 8: proj_kernel<TX, 8><<<grid, 64, 0, ctx->stream>>>(X, Ug, out, rows, d_in, rg, k_per_split, r, ld_out); break;
+      case 16: proj_kernel<TX, 16><<<grid, 128, 0, ctx->stream>>>(X, Ug, out, rows, d_in, rg, k_per_split, r, ld_out); break;
+      default: proj_kernel<TX, 32><<<grid, 256, 0, ctx->stream>>>(X, Ug, out, rows, d_in, rg, k_per_split, r, ld_out); break;
+    }
+    ++ctx->n_launch;
     ZOACT_CHECK_LAUNCH();
+    if (splits > 1) {
+      const int64_t n = rows * rg;
+      int64_t blocks = (n + 255) / 256;
+      if (blocks > 4LL * ctx->sm_count) blocks = 4LL * ctx->sm_count;
+      splitk_reduce_kernel<<<(unsigned)blocks, 256, 0, ctx->stream>>>(out, P, n, splits, rg, r, j0);
+      ++ctx->n_launch;
+      ZOACT_CHECK_LAUNCH();
+    }
   }
   return ZOACT_OK;
 }
@@ -202,10 +214,10 @@ int proj_dispatch_into(Ctx* ctx, const TX* X, int64_t rows, int d_in, const floa
   dim3 grid((unsigned)row_blocks, (unsigned)splits);
   const int rp = r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32;
   switch (rp) {
-    case 4: proj_kernel<TX, 4><<<grid, 32, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); break;
-    case 8: proj_kernel<TX, 8><<<grid, 64, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); break;
-    case 16: proj_kernel<TX, 16><<<grid, 128, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); break;
-    default: proj_kernel<TX, 32><<<grid, 256, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split); break;
+    case 4: proj_kernel<TX, 4><<<grid, 32, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split, r, r); break;
+    case 8: proj_kernel<TX, 8><<<grid, 64, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split, r, r); break;
+    case 16: proj_kernel<TX, 16><<<grid, 128, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split, r, r); break;
+    default: proj_kernel<TX, 32><<<grid, 256, 0, ctx->stream>>>(X, U, out, rows, d_in, r, k_per_split, r, r); break;
   }
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
@@ -213,7 +225,7 @@ int proj_dispatch_into(Ctx* ctx, const TX* X, int64_t rows, int d_in, const floa
     const int64_t n = rows * r;
     int64_t blocks = (n + 255) / 256;
     if (blocks > 4LL * ctx->sm_count) blocks = 4LL * ctx->sm_count;
-    splitk_reduce_kernel<<<(unsigned)blocks, 256, 0, ctx->stream>>>(out, P, n, splits);
+    splitk_reduce_kernel<<<(unsigned)blocks, 256, 0, ctx->stream>>>(out, P, n, splits, r, r, 0);
     ++ctx->n_launch;
     ZOACT_CHECK_LAUNCH();
   }

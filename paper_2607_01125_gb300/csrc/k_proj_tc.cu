@@ -38,14 +38,17 @@ struct ProjShared {
   int ok;
 };
 
-// Ut rows: [0, RT) = U0^T, [RT, 2RT) = U1^T, [2RT, 3RT) = U2^T, rest zero.
+// Ut: groups of RT ranks (one group for r <= 32; groups of 64 above), each NB rows:
+// [0, RT) = U0^T, [RT, 2RT) = U1^T, [2RT, 3RT) = U2^T of the group's ranks, rest zero.
 template <typename T16>
-__global__ void split_u_kernel(const float* __restrict__ U, T16* __restrict__ Ut, int d_in, int r, int RT, int NB) {
-  const int64_t n = (int64_t)NB * d_in;
+__global__ void split_u_kernel(const float* __restrict__ U, T16* __restrict__ Ut, int d_in, int r, int RT, int NB,
+                               int groups) {
+  const int64_t n = (int64_t)groups * NB * d_in;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-    const int row = (int)(i / d_in);
+    const int row_all = (int)(i / d_in);
     const int k = (int)(i % d_in);
-    const int term = row / RT, j = row % RT;
+    const int g = row_all / NB, row = row_all % NB;
+    const int term = row / RT, j = g * RT + row % RT;
     float v = 0.f;
     if (term < 3 && j < r) {
       float rest = U[(int64_t)k * r + j];
@@ -62,9 +65,9 @@ __global__ void split_u_kernel(const float* __restrict__ U, T16* __restrict__ Ut
 template <int NB, int RT, int AB_BF16>
 __global__ void __launch_bounds__(128, 1)
 proj_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmU, float* __restrict__ out,
-               int64_t rows, int r, int kb_per_split, int num_kb, int* status) {
+               int64_t rows, int r, int ld_out, int kb_per_split, int num_kb, int* status) {
   constexpr int STAGE = p_stage_bytes<NB>();
-  constexpr uint32_t TCOLS = NB <= 32 ? 32 : (NB <= 64 ? 64 : 128);
+  constexpr uint32_t TCOLS = NB <= 32 ? 32 : (NB <= 64 ? 64 : (NB <= 128 ? 128 : 256));
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   ProjShared* ss = reinterpret_cast<ProjShared*>(smem + PSTAGES * STAGE);
@@ -148,19 +151,42 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ 
   tc::tc_fence_after();
   const bool ok = *reinterpret_cast<volatile int*>(&ss->ok) != 0 && kb1 > kb0;
   const int64_t m = m0 + threadIdx.x;
-  float acc[NB];
-  if (ok) {
+  // r valid ranks of this launch; split partials are [splits][rows][r], direct output rows have stride ld_out
+  float* dst = out + (int64_t)blockIdx.y * rows * ld_out + m * ld_out;
+  const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+  if constexpr (RT <= 8) {
+    float acc[NB];
+    if (ok) {
 #pragma unroll
-    for (int c = 0; c < NB; c += 16) tc::tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c, acc + c);
+      for (int c = 0; c < NB; c += 16) tc::tmem_ld16(lane_base + (uint32_t)c, acc + c);
+    } else {
+#pragma unroll
+      for (int c = 0; c < NB; ++c) acc[c] = 0.f;
+    }
+    if (m < rows) {
+#pragma unroll
+      for (int j = 0; j < RT; ++j)
+        if (j < r) dst[j] = (acc[j] + acc[RT + j]) + acc[2 * RT + j];
+    }
   } else {
+    // 16 ranks at a time: their three terms are columns j, RT + j, 2 RT + j
+#pragma unroll 1
+    for (int jc = 0; jc < RT; jc += 16) {
+      float t0[16], t1[16], t2[16];
+      if (ok) {
+        tc::tmem_ld16(lane_base + (uint32_t)jc, t0);
+        tc::tmem_ld16(lane_base + (uint32_t)(RT + jc), t1);
+        tc::tmem_ld16(lane_base + (uint32_t)(2 * RT + jc), t2);
+      } else {
 #pragma unroll
-    for (int c = 0; c < NB; ++c) acc[c] = 0.f;
-  }
-  if (m < rows) {
-    float* dst = out + (int64_t)blockIdx.y * rows * r + m * r;
+        for (int i = 0; i < 16; ++i) { t0[i] = 0.f; t1[i] = 0.f; t2[i] = 0.f; }
+      }
+      if (m < rows) {
 #pragma unroll
-    for (int j = 0; j < RT; ++j)
-      if (j < r) dst[j] = (acc[j] + acc[RT + j]) + acc[2 * RT + j];
+        for (int i = 0; i < 16; ++i)
+          if (jc + i < r) dst[jc + i] = (t0[i] + t1[i]) + t2[i];
+      }
+    }
   }
   tc::tc_fence_before();
   __syncthreads();
@@ -171,54 +197,64 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ 
   }
 }
 
-__global__ void splitk_sum_kernel(const float* __restrict__ part, float* __restrict__ P, int64_t n, int splits) {
+// P[t, j0 + j] = sum over splits of part[split][t][j] (split order), j < rg; P rows have stride ldp.
+__global__ void splitk_sum_kernel(const float* __restrict__ part, float* __restrict__ P, int64_t n, int splits, int rg,
+                                  int ldp, int j0) {
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
     float s = 0.f;
     for (int k = 0; k < splits; ++k) s += part[(int64_t)k * n + i];
-    P[i] = s;
+    const int64_t t = i / rg;
+    P[t * ldp + j0 + (i - t * rg)] = s;
   }
 }
 
 template <int NB, int RT, int AB>
-int launch_one(Ctx* ctx, const CUtensorMap& mx, const CUtensorMap& mu, float* out, int64_t rows, int r, int kbps,
-               int num_kb, dim3 grid) {
+int launch_one(Ctx* ctx, const CUtensorMap& mx, const CUtensorMap& mu, float* out, int64_t rows, int r, int ld_out,
+               int kbps, int num_kb, dim3 grid) {
   auto kern = proj_tc_kernel<NB, RT, AB>;
   ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p_smem_bytes<NB>()));
-  kern<<<grid, 128, p_smem_bytes<NB>(), ctx->stream>>>(mx, mu, out, rows, r, kbps, num_kb, ctx->d_status);
+  kern<<<grid, 128, p_smem_bytes<NB>(), ctx->stream>>>(mx, mu, out, rows, r, ld_out, kbps, num_kb, ctx->d_status);
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
 }
 
 template <int AB>
-int dispatch(Ctx* ctx, int rt, const CUtensorMap& mx, const CUtensorMap& mu, float* out, int64_t rows, int r, int kbps,
-             int num_kb, dim3 grid) {
+int dispatch(Ctx* ctx, int rt, const CUtensorMap& mx, const CUtensorMap& mu, float* out, int64_t rows, int r,
+             int ld_out, int kbps, int num_kb, dim3 grid) {
   switch (rt) {
-    case 4: return launch_one<16, 4, AB>(ctx, mx, mu, out, rows, r, kbps, num_kb, grid);
-    case 8: return launch_one<32, 8, AB>(ctx, mx, mu, out, rows, r, kbps, num_kb, grid);
-    case 16: return launch_one<48, 16, AB>(ctx, mx, mu, out, rows, r, kbps, num_kb, grid);
-    default: return launch_one<96, 32, AB>(ctx, mx, mu, out, rows, r, kbps, num_kb, grid);
+    case 4: return launch_one<16, 4, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid);
+    case 8: return launch_one<32, 8, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid);
+    case 16: return launch_one<48, 16, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid);
+    case 32: return launch_one<96, 32, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid);
+    default: return launch_one<192, 64, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid);
   }
 }
+
+// ranks per group of the split basis (one group up to 32 ranks, groups of 64 above) and rows per group
+int proj_rt(int r) { return r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : r <= 32 ? 32 : 64; }
+int proj_nb(int rt) { return rt == 4 ? 16 : rt == 8 ? 32 : rt == 16 ? 48 : rt == 32 ? 96 : 192; }
 
 }  // namespace
 
 int basis_tc_rows(int r) {
-  const int rt = r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32;
-  return 3 * rt <= 16 ? 16 : (3 * rt <= 32 ? 32 : (3 * rt <= 48 ? 48 : 96));
+  const int rt = proj_rt(r);
+  return proj_nb(rt) * ((r + rt - 1) / rt);
 }
 
 int launch_basis_prepare(Ctx* ctx, const float* U, int d_in, int r, int xdtype, void* Ut) {
-  const int rt = r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32;
-  const int nb = basis_tc_rows(r);
-  const int64_t n = (int64_t)nb * d_in;
+  const int rt = proj_rt(r);
+  const int nb = proj_nb(rt);
+  const int groups = (r + rt - 1) / rt;
+  const int64_t n = (int64_t)groups * nb * d_in;
   int64_t blocks = (n + 255) / 256;
   if (blocks > 8LL * ctx->sm_count) blocks = 8LL * ctx->sm_count;
   if (xdtype == ZOACT_DT_BF16)
     split_u_kernel<__nv_bfloat16><<<(unsigned)blocks, 256, 0, ctx->stream>>>(U, static_cast<__nv_bfloat16*>(Ut), d_in,
-                                                                             r, rt, nb);
+                                                                             r, rt, nb, groups);
   else
-    split_u_kernel<__half><<<(unsigned)blocks, 256, 0, ctx->stream>>>(U, static_cast<__half*>(Ut), d_in, r, rt, nb);
+    split_u_kernel<__half><<<(unsigned)blocks, 256, 0, ctx->stream>>>(U, static_cast<__half*>(Ut), d_in, r, rt, nb,
+                                                                      groups);
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
@@ -238,12 +274,11 @@ int launch_lowrank_proj_tc(Ctx* ctx, const void* X, int xdtype, int64_t rows, in
 int launch_lowrank_proj_tc_prepared(Ctx* ctx, const void* X, int xdtype, int64_t rows, int d_in, const void* Ut,
                                     int r, float* P) {
   if (rows <= 0) return ZOACT_OK;
-  const int rt = r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32;
-  const int nb = basis_tc_rows(r);
-  CUtensorMap mx, mu;
+  const int rt = proj_rt(r);
+  const int nb = proj_nb(rt);
+  const int groups = (r + rt - 1) / rt;
+  CUtensorMap mx;
   int st = encode_tmap_2d_16bit(&mx, X, xdtype, rows, d_in, PBM);
-  if (st) return st;
-  st = encode_tmap_2d_16bit(&mu, Ut, xdtype, nb, d_in, nb);
   if (st) return st;
   const int num_kb = (d_in + PBK - 1) / PBK;
   const int64_t row_blocks = (rows + PBM - 1) / PBM;
@@ -253,22 +288,31 @@ int launch_lowrank_proj_tc_prepared(Ctx* ctx, const void* X, int xdtype, int64_t
   if (splits < 1) splits = 1;
   const int kbps = (num_kb + splits - 1) / splits;
   splits = (num_kb + kbps - 1) / kbps;
-  float* out = P;
-  if (splits > 1) {
-    out = static_cast<float*>(scratch(ctx, SLOT_SPLITK, (size_t)splits * rows * r * sizeof(float)));
-    if (!out) return ZOACT_ERR_NOMEM;
-  }
-  const dim3 grid((unsigned)row_blocks, (unsigned)splits);
-  st = xdtype == ZOACT_DT_BF16 ? dispatch<1>(ctx, rt, mx, mu, out, rows, r, kbps, num_kb, grid)
-                               : dispatch<0>(ctx, rt, mx, mu, out, rows, r, kbps, num_kb, grid);
-  if (st) return st;
-  if (splits > 1) {
-    const int64_t n = rows * r;
-    int64_t blocks = (n + 255) / 256;
-    if (blocks > 4LL * ctx->sm_count) blocks = 4LL * ctx->sm_count;
-    splitk_sum_kernel<<<(unsigned)blocks, 256, 0, ctx->stream>>>(out, P, n, splits);
-    ++ctx->n_launch;
-    ZOACT_CHECK_LAUNCH();
+  // one launch per group of ranks (X is re-read per group; a single group up to r = 32)
+  for (int g = 0; g < groups; ++g) {
+    const int j0 = g * rt, rg = r - j0 < rt ? r - j0 : rt;
+    CUtensorMap mu;
+    st = encode_tmap_2d_16bit(&mu, static_cast<const uint8_t*>(Ut) + (size_t)g * nb * d_in * 2, xdtype, nb, d_in, nb);
+    if (st) return st;
+    float* out = P + j0;
+    int ld_out = r;
+    if (splits > 1) {
+      out = static_cast<float*>(scratch(ctx, SLOT_SPLITK, (size_t)splits * rows * rg * sizeof(float)));
+      if (!out) return ZOACT_ERR_NOMEM;
+      ld_out = rg;
+    }
+    const dim3 grid((unsigned)row_blocks, (unsigned)splits);
+    st = xdtype == ZOACT_DT_BF16 ? dispatch<1>(ctx, rt, mx, mu, out, rows, rg, ld_out, kbps, num_kb, grid)
+                                 : dispatch<0>(ctx, rt, mx, mu, out, rows, rg, ld_out, kbps, num_kb, grid);
+    if (st) return st;
+    if (splits > 1) {
+      const int64_t n = rows * rg;
+      int64_t blocks = (n + 255) / 256;
+      if (blocks > 4LL * ctx->sm_count) blocks = 4LL * ctx->sm_count;
+      splitk_sum_kernel<<<(unsigned)blocks, 256, 0, ctx->stream>>>(out, P, n, splits, rg, r, j0);
+      ++ctx->n_launch;
+      ZOACT_CHECK_LAUNCH();
+    }
   }
   return ZOACT_OK;
 }

@@ -107,7 +107,7 @@ struct Params {
   int aug_mode;      // LowrankMode
   int aug_kb;        // extra K-blocks per tile from A_aug / B_aug (0 with LOWRANK_EPILOGUE)
   int aug_kb_slot;   // K-blocks of one slot (B_aug row width / 64)
-  int aug_slots;     // LOWRANK_ALL_ON_TC: 1, or 2 when tiles straddle two evaluation blocks
+  int aug_slots;     // LOWRANK_ALL_ON_TC: 1, or S when a tile spans up to S evaluation blocks (slot = block mod S)
   int64_t aug_block_rows;   // rows of one block's table in B_aug (LOWRANK_ALL_ON_TC)
   // LOWRANK_C_ON_TC: Z of each distinct query, transposed [q][r][d_out] (gate / up), and the table of each block
   const float* Zt;
@@ -139,7 +139,8 @@ static_assert(sizeof(SharedState) <= 256, "barrier block outgrew its shared-memo
 
 // TMA coordinates of low-rank K-block `ka` (0 .. aug_kb) of a tile whose rows start at tile_row0:
 // x in A_aug (slots side by side), x in B_aug (one slot wide), and the first B_aug row of the table the
-// slot meets -- the tile's block (one slot), or the tile's block of the slot's parity (two slots).
+// slot meets -- the tile's block (one slot), or the tile's block congruent to the slot mod S (S slots;
+// a slot no block of the tile maps to has zero A columns and reads any table).
 __device__ __forceinline__ void aug_coords(const Params& prm, int64_t tile_row0, int tile_rows, int ka, int& kx_a,
                                            int& kx_b, int& y_b) {
   const int slot = ka / prm.aug_kb_slot;
@@ -149,7 +150,9 @@ __device__ __forceinline__ void aug_coords(const Params& prm, int64_t tile_row0,
   if (prm.aug_mode == LOWRANK_ALL_ON_TC) {
     const int b_lo = (int)(tile_row0 / prm.T);
     const int b_hi = (int)((min(tile_row0 + tile_rows, prm.rows) - 1) / prm.T);
-    const int blk = prm.aug_slots == 1 ? b_lo : (((b_lo & 1) == slot) ? b_lo : min(b_lo + 1, b_hi));
+    const int S = prm.aug_slots;
+    int blk = b_lo + ((slot - b_lo % S) % S + S) % S;
+    if (blk > b_hi) blk = b_lo;
     y_b = (int)(blk * prm.aug_block_rows);
   }
 }

@@ -101,7 +101,7 @@ class ZOStep:
             return
         for l in self.linears:
             key = l.U.data_ptr()
-            if key in self._utc or l.r > 32:
+            if key in self._utc:
                 continue
             t = torch.empty(Z.zoact_basis_prepared_bytes(l.d_in, l.r), dtype=torch.uint8, device=self.device)
             Z.zoact_basis_prepare(self.ctx, l.U, Z.TORCH_DT[self.dtype], t)
