@@ -297,7 +297,7 @@ int zoact_sgd_step_multi(zoact_ctx* ctx, float* C, int64_t n_total, const zoact_
  * (element i*k + j), Q0 = orth(Omega), Q <- orth(G Q) n_iter times, then
  * Rayleigh-Ritz.  Columns in descending eigenvalue order, each flipped so its
  * largest-magnitude entry is positive.  Optional evals_out [k] fp32 (device)
- * receives the Ritz values.  Requires k <= 64 and k <= d_in; uses d_in^2 * 4
+ * receives the Ritz values.  Requires k <= 512 and k <= d_in; uses d_in^2 * 4
  * bytes of context scratch.                                                    */
 int zoact_basis_init(zoact_ctx* ctx, const void* X_cal, int xdtype, int64_t n_tok, int32_t d_in,
                      int32_t r, int32_t oversample, int32_t n_iter, uint64_t seed, float* U_out,

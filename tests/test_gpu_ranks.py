@@ -132,3 +132,29 @@ def test_adam_rank_256(ctx):
     f32 = lambda x: float(np.float32(x))
     Cr, _, _ = optim.adam_step(C0, 0, 0, g, f32(1e-3), f32(0.9), f32(0.999), f32(1e-8), 1)
     np.testing.assert_allclose(np64(C), Cr, rtol=1e-4, atol=1e-9)
+
+
+@pytest.mark.parametrize("r,p", [(128, 16), (256, 16), (40, 24)])
+def test_basis_large_rank(ctx, r, p):
+    # a planted spectrum with a clear gap after r: the device iteration (k = r + p, parallel Jacobi for
+    # k > 64) reaches the exact top-r eigenspace of X^T X and its Ritz values
+    from oracle import basis
+    rng = np.random.default_rng(r)
+    n, d = 3072, 1024
+    A = rng.standard_normal((n, 300))
+    s = np.concatenate([np.linspace(10.0, 6.0, r), 0.3 * np.ones(300 - r)])
+    B = np.linalg.qr(rng.standard_normal((d, 300)))[0].T
+    Xn = (A * s) @ B + 1e-3 * rng.standard_normal((n, d))
+    X = torch.tensor(Xn, dtype=torch.float32, device=DEV).to(torch.bfloat16)
+    Xb = np64(X)
+    U = torch.empty(d, r, device=DEV)
+    ev = torch.empty(r + p, device=DEV)
+    zo.zoact_basis_init(ctx, X, r, U, oversample=p, n_iter=8, seed=2, evals_out=ev)
+    torch.cuda.synchronize()
+    assert ctx.device_status() == 0
+    Ug = np64(U)
+    np.testing.assert_allclose(Ug.T @ Ug, np.eye(r), atol=2e-4)
+    lam, V = np.linalg.eigh(Xb.T @ Xb)
+    order = np.argsort(lam)[::-1]
+    assert basis.subspace_overlap(Ug, V[:, order[:r]]) >= 1 - 1e-5
+    np.testing.assert_allclose(np64(ev)[:r], lam[order[:r]], rtol=1e-4)
