@@ -116,7 +116,7 @@ def dist_setup():
     return world, rank, local
 
 
-def build(ctx, dev, rank, name, tokens=None, n_queries=None):
+def build(ctx, dev, rank, name, tokens=None, n_queries=None, r=None):
     """Weights, bases (Algorithm 1 on the device) and the ZOStep of a workload.
 
     Returns (step, x, target, basis_seconds, workload).  Weights are the same on every
@@ -126,7 +126,12 @@ def build(ctx, dev, rank, name, tokens=None, n_queries=None):
     import paper_2607_01125_gb300 as zo
     from paper_2607_01125_gb300.model import AdaptedLinear, ZOStep, coefficient_offsets, calibrate_bases
     from synth import workload, normal, lowrank_activations, quantize_int4_g128, tensor_seed
-    w = workload(name) if tokens is None else workload(name, T=tokens)
+    over = {}
+    if tokens is not None:
+        over["T"] = tokens
+    if r is not None:
+        over["r"] = r
+    w = workload(name, **over)
     dt = {"bf16": torch.bfloat16, "fp16": torch.float16}[w.act_dtype]
     specs = w.linears()
     offs = coefficient_offsets(specs, w.r)
@@ -210,7 +215,7 @@ def run_ours(args):
     dev = f"cuda:{local}"
     torch.cuda.set_device(local)
     ctx = zo.Context(local)
-    step, x, target, basis_s, w = build(ctx, dev, rank, args.workload, args.tokens, args.queries)
+    step, x, target, basis_s, w = build(ctx, dev, rank, args.workload, args.tokens, args.queries, args.rank)
     seed = 1234
 
     def barrier():
@@ -300,7 +305,7 @@ def run_ours(args):
                      "kernel": "pair_tc2_kernel / pair_tc_kernel (every pair-forward launch of the step)",
                      "algorithmic_flops_per_step": gemm_flops / args.steps,
                      "traffic": (PAIR_TRAFFIC_BYTES.get(w.name)
-                                 if args.tokens is None and args.queries is None else None),
+                                 if args.tokens is None and args.queries is None and args.rank is None else None),
                      "traffic_unit": "bytes per step (both pair launches)"},
         "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": 8 * step.loss_out.numel()},
@@ -310,7 +315,8 @@ def run_ours(args):
     }
     if args.diag:
         line["diag"] = time_diagnostics(ctx, step, dev)
-    if world == 1 and not args.no_cpu_baseline and args.workload == DEFAULT_WORKLOAD and args.queries is None:
+    if (world == 1 and not args.no_cpu_baseline and args.workload == DEFAULT_WORKLOAD and args.queries is None
+            and args.rank is None):
         line["cpu_baseline"] = cpu_baseline(step, budget_s=args.cpu_budget)
     print(json.dumps(line))
 
@@ -401,6 +407,7 @@ def main():
     ap.add_argument("--tokens", type=int, default=None, help="tokens per perturbation (default: the workload's)")
     ap.add_argument("--queries", type=int, default=None,
                     help="one-sided estimator with this many queries (Algorithm 2); default: two-sided pair")
+    ap.add_argument("--rank", type=int, default=None, help="basis rank r (default: the workload's; 1..256)")
     ap.add_argument("--diag", action="store_true", help="also time the Section 5.3 subspace diagnostics")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--soak", type=float, default=2.0,

@@ -131,9 +131,8 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   if (w4 ? a.xdtype != ZOACT_DT_BF16 : a.wtype != a.xdtype) return ZOACT_ERR_UNSUPPORTED;
   if (a.ydtype != a.xdtype && a.ydtype != ZOACT_DT_FP32) return ZOACT_ERR_UNSUPPORTED;
   const bool gated = a.W2 != nullptr;
-  // epilogue-table rank template; above 32 ranks (whole term on the tensor cores) the tables are unused
-  const int rt = big_r ? (gated ? 16 : 32) : rank_template(a.r);
-  if (gated && rt > 16) return ZOACT_ERR_UNSUPPORTED;
+  // epilogue-table rank template (set below: the smallest one when the tables go unused)
+  int rt = rank_template(a.r);
   if (a.rows <= 0) return ZOACT_OK;
   TmaSet tm;
   int st = encode_tmap_2d_16bit(&tm.a, a.X, a.xdtype, a.rows, a.d_in, BM);
@@ -177,6 +176,7 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     }
   }
   if (big_r && lmode != LOWRANK_ALL_ON_TC) return ZOACT_ERR_UNSUPPORTED;
+  if (lmode == LOWRANK_ALL_ON_TC) rt = 4;   // whole term on the tensor cores: no epilogue tables
   const int ka = aug_cols(a.r);
   const int ka_tot = distinct ? 2 * ka : ka;
   tm.aa = tm.a; tm.ba = tm.b; tm.ba2 = tm.b2;

@@ -22,6 +22,7 @@ static int by_rank_two(Ctx* ctx, int mode, int rt, const TmaSet& tm, const Param
       case 4: return launch_two<TO, 4, MODE_GATED>(ctx, tm, p);
       case 8: return launch_two<TO, 8, MODE_GATED>(ctx, tm, p);
       case 16: return launch_two<TO, 16, MODE_GATED>(ctx, tm, p);
+      case 32: return launch_two<TO, 32, MODE_GATED>(ctx, tm, p);
       default: return ZOACT_ERR_UNSUPPORTED;
     }
   }

@@ -21,6 +21,7 @@ static int by_rank(Ctx* ctx, int mode, int rt, const TmaSet& tm, const Params& p
       case 4: return launch_one<TO, 4, MODE_GATED>(ctx, tm, p);
       case 8: return launch_one<TO, 8, MODE_GATED>(ctx, tm, p);
       case 16: return launch_one<TO, 16, MODE_GATED>(ctx, tm, p);
+      case 32: return launch_one<TO, 32, MODE_GATED>(ctx, tm, p);
       default: return ZOACT_ERR_UNSUPPORTED;
     }
   }

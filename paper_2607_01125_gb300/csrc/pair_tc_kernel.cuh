@@ -69,6 +69,10 @@ constexpr int TPAD = 4;
 __host__ __device__ constexpr int pair_slots(int rt) {
   return (2 * rt * (BN + TPAD) <= TBL_FLOATS) ? BN : (2 * rt * (BN / 2 + TPAD) <= TBL_FLOATS ? BN / 2 : BN / 4);
 }
+// gated tiles: four tables (gate and up, two blocks) over at most BN / 2 columns
+__host__ __device__ constexpr int gated_slots(int rt) {
+  return (4 * rt * (BN / 2 + TPAD) <= TBL_FLOATS) ? BN / 2 : (4 * rt * (BN / 4 + TPAD) <= TBL_FLOATS ? BN / 4 : BN / 8);
+}
 constexpr int EPI_WARPS = 8;
 constexpr int EPI_THREADS = 32 * EPI_WARPS;
 constexpr int DQ_THREADS = 128;                     // INT4 dequantisation warps
@@ -436,7 +440,7 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
                                               int64_t row0, int64_t m, bool row_ok, int n_blk, int bn, int buf,
                                               uint32_t acc_phase, uint32_t t_row, volatile int* abort_flag) {
   constexpr bool GATED = MODE == MODE_GATED;
-  constexpr int SLOTS = GATED ? BN / 2 : pair_slots(RT);   // table columns per chunk
+  constexpr int SLOTS = GATED ? gated_slots(RT) : pair_slots(RT);   // table columns per chunk
   constexpr int STRIDE = SLOTS + TPAD;
   constexpr int TSZ = RT * STRIDE;                         // floats per table
   static_assert((GATED ? 4 : 2) * TSZ <= TBL_FLOATS, "epilogue tables exceed their shared-memory region");

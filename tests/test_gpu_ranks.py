@@ -65,9 +65,11 @@ def test_pair_forward_large_rank(ctx, r, T, shared):
     assert err.max() <= 1e-4 * np.abs(ref).max()
 
 
-@pytest.mark.parametrize("T,shared,nb", [(256, True, 2), (130, False, 5)])
-def test_gated_and_multi_large_rank(ctx, T, shared, nb):
-    d_in, d_out, r, seed, mu = 512, 400, 128, 8, 0.25
+@pytest.mark.parametrize("T,shared,nb,r", [(256, True, 2, 128), (130, False, 5, 128), (200, True, 2, 32),
+                                          (96, True, 5, 24), (150, False, 2, 32)])
+def test_gated_and_multi_large_rank(ctx, T, shared, nb, r):
+    # r = 17..32 gated on a shared input keeps its +-Z p tables in narrower column chunks
+    d_in, d_out, seed, mu = 512, 400, 8, 0.25
     X = normal(((T if shared else nb * T), d_in), 31, DEV, dtype=torch.bfloat16)
     Wg = normal((d_out, d_in), 32, DEV, std=d_in ** -0.5, dtype=torch.bfloat16)
     Wu = normal((d_out, d_in), 33, DEV, std=d_in ** -0.5, dtype=torch.bfloat16)
