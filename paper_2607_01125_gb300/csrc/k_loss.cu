@@ -5,9 +5,9 @@
 // One pass over the stacked outputs (HBM-bound).  Each thread reads 16-byte
 // vectors of y+, y- and t (kept as raw words until used; 64 registers, four
 // 256-thread blocks per SM), sums a round of two vectors' terms (16 per
-// accumulator) in fp32 and adds the round's sum to fp64 accumulators (fp64 adds
-// are scarce on this part: one per 16 terms keeps them off the critical path);
-// warps reduce by shuffles, blocks write fp64 partials to scratch, and the last
+// accumulator) in fp32 and adds the round's sum to a compensated fp32 running
+// sum (fp64 units are scarce on this part); each block adds its threads' sums
+// in fp64 in a fixed order, writes the block partials to scratch, and the last
 // block to finish (an atomic ticket) adds the partials in block order, so the
 // result is deterministic.  The ticket is reset by that
 // block, leaving the scratch ready for the next call.
@@ -81,6 +81,35 @@ __device__ __forceinline__ double warp_sum(double v) {
   return v;
 }
 
+// A running sum in fp32 with Neumaier compensation: s + c carries the sum of the
+// added values to about twice fp32 precision, without the scarce fp64 units.
+struct CSum {
+  float s = 0.f, c = 0.f;
+  __device__ __forceinline__ void add(float x) {
+    const float t = s + x;
+    c += fabsf(s) >= fabsf(x) ? (s - t) + x : (x - t) + s;
+    s = t;
+  }
+  __device__ __forceinline__ double value() const { return (double)s + (double)c; }
+};
+
+// Sum v over the block's threads in fp64 (one conversion per thread; warp 0 adds the
+// per-thread values in a fixed order).  Result valid in thread 0.
+template <int NV>
+__device__ __forceinline__ void block_sum(const double (&v)[NV], double (&out)[NV], double (*sm)[LOSS_THREADS]) {
+#pragma unroll
+  for (int i = 0; i < NV; ++i) sm[i][threadIdx.x] = v[i];
+  __syncthreads();
+  if (threadIdx.x < 32) {
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+      double a = 0.0;
+      for (int t = threadIdx.x; t < LOSS_THREADS; t += 32) a += sm[i][t];
+      out[i] = warp_sum(a);
+    }
+  }
+}
+
 template <typename TY>
 __global__ void __launch_bounds__(LOSS_THREADS, 4)
 loss_pair_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t count, int vec_ok, float eps,
@@ -88,7 +117,7 @@ loss_pair_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t c
                  int* __restrict__ status) {
   const TY* yp = Y;
   const TY* ym = Y + count;
-  double ap = 0.0, am = 0.0, ad = 0.0;
+  CSum ap, am, ad;
   // 16-byte vectors need y+, y- and t 16-byte aligned (host checks the bases;
   // y- = y+ + count is aligned when count % 8 == 0)
   const int64_t n_vec = vec_ok ? count / 8 : 0;
@@ -124,7 +153,7 @@ loss_pair_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t c
         sd = fmaf(p[i] - m[i], dp + dm, sd);
       }
     }
-    ap += sp; am += sm; ad += sd;
+    ap.add(sp); am.add(sm); ad.add(sd);
   }
   for (; v < n_vec; v += stride) {
     float p[8], m[8], t[8];
@@ -144,24 +173,21 @@ loss_pair_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t c
       sm = fmaf(dm, dm, sm);
       sd = fmaf(p[i] - m[i], dp + dm, sd);
     }
-    ap += sp; am += sm; ad += sd;
+    ap.add(sp); am.add(sm); ad.add(sd);
   }
   // scalar remainder (everything when the vector path is off)
   for (int64_t i = 8 * n_vec + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < count; i += stride) {
     const float tv = tgt ? to_f32<TY>(tgt[i]) : 0.f;
     const float dp = to_f32<TY>(yp[i]) - tv, dm = to_f32<TY>(ym[i]) - tv;
-    ap += (double)(dp * dp); am += (double)(dm * dm);
-    ad += (double)((to_f32<TY>(yp[i]) - to_f32<TY>(ym[i])) * (dp + dm));
+    ap.add(dp * dp); am.add(dm * dm);
+    ad.add((to_f32<TY>(yp[i]) - to_f32<TY>(ym[i])) * (dp + dm));
   }
-  __shared__ double red[3][LOSS_THREADS / 32];
+  __shared__ double tree[3][LOSS_THREADS];
   __shared__ bool is_last;
-  ap = warp_sum(ap); am = warp_sum(am); ad = warp_sum(ad);
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (lane == 0) { red[0][warp] = ap; red[1][warp] = am; red[2][warp] = ad; }
-  __syncthreads();
+  double bs[3];
+  block_sum<3>({ap.value(), am.value(), ad.value()}, bs, tree);
   if (threadIdx.x == 0) {
-    double s0 = 0.0, s1 = 0.0, s2 = 0.0;
-    for (int w = 0; w < LOSS_THREADS / 32; ++w) { s0 += red[0][w]; s1 += red[1][w]; s2 += red[2][w]; }
+    const double s0 = bs[0], s1 = bs[1], s2 = bs[2];
     partials[3 * blockIdx.x + 0] = s0;
     partials[3 * blockIdx.x + 1] = s1;
     partials[3 * blockIdx.x + 2] = s2;
@@ -180,7 +206,7 @@ loss_pair_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t c
     s1 += __ldcg(partials + 3 * b + 1);
     s2 += __ldcg(partials + 3 * b + 2);
   }
-  __shared__ double tree[3][LOSS_THREADS];
+  __syncthreads();                 // the block sum's readers of `tree` are done
   tree[0][threadIdx.x] = s0; tree[1][threadIdx.x] = s1; tree[2][threadIdx.x] = s2;
   __syncthreads();
   for (int h = LOSS_THREADS / 2; h > 0; h >>= 1) {
@@ -228,11 +254,11 @@ loss_multi_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t 
   const int b = blockIdx.y;
   const TY* yb = Y + (int64_t)b * count;
   const TY* y0 = Y;
-  double as = 0.0, ad = 0.0;
+  CSum as, ad;
   const int64_t n_vec = vec_ok ? count / 8 : 0;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int64_t first = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  // rounds of two vectors, all loads issued first; one fp64 add per accumulator per round
+  // rounds of two vectors, all loads issued first; one compensated add per accumulator per round
   int64_t v = first;
   constexpr int R = sizeof(TY) == 4 ? 1 : 2;   // vectors per round (fp32 words take twice the registers)
   for (; v + (R - 1) * stride < n_vec; v += R * stride) {
@@ -262,7 +288,7 @@ loss_multi_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t 
         if (b > 0) sd = fmaf(y[i] - z[i], dy + (z[i] - t[i]), sd);
       }
     }
-    as += ss; ad += sd;
+    as.add(ss); ad.add(sd);
   }
   for (; v < n_vec; v += stride) {
     float y[8], z[8], t[8];
@@ -281,27 +307,24 @@ loss_multi_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t 
       ss = fmaf(dy, dy, ss);
       if (b > 0) sd = fmaf(y[i] - z[i], dy + (z[i] - t[i]), sd);
     }
-    as += ss; ad += sd;
+    as.add(ss); ad.add(sd);
   }
   for (int64_t i = 8 * n_vec + first; i < count; i += stride) {
     const float tv = tgt ? to_f32<TY>(tgt[i]) : 0.f;
     const float yv = to_f32<TY>(yb[i]);
     const float dy = yv - tv;
-    as += (double)(dy * dy);
+    as.add(dy * dy);
     if (b > 0) {
       const float zv = to_f32<TY>(y0[i]);
-      ad += (double)((yv - zv) * (dy + (zv - tv)));
+      ad.add((yv - zv) * (dy + (zv - tv)));
     }
   }
-  __shared__ double red[2][LOSS_THREADS / 32];
+  __shared__ double red[2][LOSS_THREADS];
   __shared__ bool is_last;
-  as = warp_sum(as); ad = warp_sum(ad);
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (lane == 0) { red[0][warp] = as; red[1][warp] = ad; }
-  __syncthreads();
+  double bs[2];
+  block_sum<2>({as.value(), ad.value()}, bs, red);
   if (threadIdx.x == 0) {
-    double s0 = 0.0, s1 = 0.0;
-    for (int w = 0; w < LOSS_THREADS / 32; ++w) { s0 += red[0][w]; s1 += red[1][w]; }
+    const double s0 = bs[0], s1 = bs[1];
     double* pb = partials + 2 * ((int64_t)b * gridDim.x + blockIdx.x);
     pb[0] = s0;
     pb[1] = s1;

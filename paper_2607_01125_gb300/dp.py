@@ -1,9 +1,10 @@
 """Data-parallel exchange of one ZO step: ranks split the tokens, share everything else.
 
 Every rank holds the same W, U, C, m, v and seed, runs the pair forward and the
-loss pair on its own token shard, and the ranks then average the four loss
-scalars [L+, L-, D, a] (each a mean over the rank's T * n elements, so with
-equal shards their average is the global value; a = D / (2 eps) is linear in D).
+loss pair on its own token shard, and the ranks then average the loss vector --
+[L+, L-, D, a], or [L_0 .. L_q, a_1 .. a_q] for the one-sided q-query estimator
+(each entry a mean over the rank's T * n elements, so with equal shards their
+average is the global value; every a is linear in the losses).
 Each rank then applies the same Adam update with the same regenerated Z, so C
 stays identical on every rank without a gradient all-reduce.
 """
@@ -11,7 +12,7 @@ import torch.distributed as dist
 
 
 def allreduce_loss(loss_out, group=None):
-    """Average the device (or CPU, for gloo) tensor [L+, L-, D, a] over the ranks, in place."""
+    """Average the device (or CPU, for gloo) loss vector over the ranks, in place."""
     world = dist.get_world_size(group)
     if world == 1:
         return loss_out

@@ -82,3 +82,52 @@ def test_two_rank_scalar_exchange_matches_single_process():
         np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-15)
         for g in gathered:                           # every rank holds the same C, equal to the reference
             np.testing.assert_allclose(g, Cref.reshape(-1), rtol=0, atol=1e-15)
+
+
+def _multi_rank(rank, T, W, U, C, X, tgt, q, mu=1e-3, seed=9):
+    Zs = [philox.perturbation(seed, 3, 100 + j, *C.shape) for j in range(q)]
+    xs, ts = X[rank * T:(rank + 1) * T], tgt[rank * T:(rank + 1) * T]
+    Y = layers.multi_forward(W, U, C, [None] + Zs, [0.0] + [mu] * q, xs, T, True)
+    L, a = oloss.loss_queries(Y, T, q + 1, ts, mu)
+    return torch.tensor(L + a, dtype=torch.float64), Zs
+
+
+def _worker_multi(rank, world, port, q, n_queries):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    from paper_2607_01125_gb300.dp import allreduce_loss
+    W, U, C, X, tgt, T = _problem()
+    out, Zs = _multi_rank(rank, T, W, U, C, X, tgt, n_queries)
+    allreduce_loss(out)
+    a = out.numpy()[n_queries + 1:]
+    Cn, _, _ = optim.adam_step(C, 0, 0, optim.zo_gradient_queries(a, Zs), 1e-3, 0.9, 0.999, 1e-8, 1)
+    q.put((rank, out.numpy().tolist(), Cn.reshape(-1)))
+    dist.destroy_process_group()
+
+
+def test_two_rank_exchange_of_the_q_query_losses():
+    # Algorithm 2's one-sided estimator: the averaged vector [L_0..L_q, a_1..a_q] is that of the whole batch,
+    # so both ranks apply the single-process update
+    nq = 4
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker_multi, args=(r, 2, port, q, nq)) for r in range(2)]
+    for p in procs:
+        p.start()
+    results = [q.get(timeout=120) for _ in procs]
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    W, U, C, X, tgt, T = _problem()
+    Zs = [philox.perturbation(9, 3, 100 + j, *C.shape) for j in range(nq)]
+    blocks = [layers.multi_forward(W, U, C, [None] + Zs, [0.0] + [1e-3] * nq, X[i * T:(i + 1) * T], T, True)
+              for i in range(2)]
+    # the whole batch: block b holds both shards' rows of evaluation point b
+    Yfull = np.concatenate([np.concatenate([blk[b * T:(b + 1) * T] for blk in blocks]) for b in range(nq + 1)])
+    L, a = oloss.loss_queries(Yfull, 2 * T, nq + 1, tgt, 1e-3)
+    Cref, _, _ = optim.adam_step(C, 0, 0, optim.zo_gradient_queries(a, Zs), 1e-3, 0.9, 0.999, 1e-8, 1)
+    for rank, vec, Cn in results:
+        np.testing.assert_allclose(vec, L + a, rtol=1e-10, atol=1e-12)
+        np.testing.assert_allclose(Cn, Cref.reshape(-1), rtol=1e-10, atol=1e-14)
