@@ -121,6 +121,15 @@ int zoact_device_sm_count(zoact_ctx* ctx, int* sm_count);
  * counter, incremented at every launch; no synchronisation).                   */
 int zoact_get_launch_count(zoact_ctx* ctx, int64_t* count);
 
+/* Kernel timing: with enable != 0 the context records CUDA events on its stream
+ * around every tensor-core pair-forward kernel (the MMA kernel alone, without
+ * the preparation kernels of the same call; up to 4096 launches between reads).
+ * zoact_kernel_timing(ctx, 0/1) switches it and forgets recorded launches;
+ * zoact_kernel_time synchronises the stream and returns the summed duration (ms)
+ * and the number of timed launches since the last read, then forgets them.      */
+int zoact_kernel_timing(zoact_ctx* ctx, int enable);
+int zoact_kernel_time(zoact_ctx* ctx, double* ms_total, int64_t* launches);
+
 /* ---- Z: the perturbation generator (Section 3, Z ~ N(0, I)) ----
  * Writes the first n elements of the (seed, layer_id, query) stream:
  * z_out[e] (fp32 normal) and, if words_out != NULL, the raw Philox word of

@@ -36,7 +36,8 @@ EXPORTS = [
     "zoact_pair_forward_noalloc", "zoact_pair_forward_gated", "zoact_loss_pair", "zoact_adam_step", "zoact_sgd_step", "zoact_basis_init",
     "zoact_rms_norm", "zoact_mix_rms", "zoact_multi_forward", "zoact_multi_forward_gated", "zoact_loss_multi",
     "zoact_adam_step_multi", "zoact_sgd_step_multi", "zoact_basis_prepared_bytes", "zoact_basis_prepare",
-    "zoact_lowrank_proj_prepared", "zoact_subspace_overlap", "zoact_gradient_energy",
+    "zoact_lowrank_proj_prepared", "zoact_subspace_overlap", "zoact_gradient_energy", "zoact_kernel_timing",
+    "zoact_kernel_time",
 ]
 
 
@@ -113,6 +114,8 @@ def load():
         "zoact_mix_rms": [P, P, P, P, I32, I64, I32, I32, I32, F32, P],
         "zoact_basis_prepare": [P, P, I32, I32, I32, P],
         "zoact_lowrank_proj_prepared": [P, P, I32, I64, I32, P, I32, P],
+        "zoact_kernel_timing": [P, I32],
+        "zoact_kernel_time": [P, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int64)],
         "zoact_subspace_overlap": [P, P, P, I32, I32, I32, P],
         "zoact_gradient_energy": [P, P, I32, I32, P, I32, I64, P],
         "zoact_multi_forward": [P, ctypes.POINTER(zoact_layer), P, I32, I64, I32, P, ctypes.POINTER(zoact_eval_blocks),
@@ -186,6 +189,16 @@ class Context:
         v = ctypes.c_int64()
         _check("zoact_get_launch_count", load().zoact_get_launch_count(self.handle, ctypes.byref(v)))
         return v.value
+
+    def kernel_timing(self, enable=True):
+        """Record events around every tensor-core pair-forward kernel (see zoact_kernel_timing)."""
+        _check("zoact_kernel_timing", load().zoact_kernel_timing(self.handle, int(enable)))
+
+    def kernel_time(self):
+        """(summed milliseconds, launches) of the timed pair-forward kernels since the last read; syncs."""
+        ms, n = ctypes.c_double(), ctypes.c_int64()
+        _check("zoact_kernel_time", load().zoact_kernel_time(self.handle, ctypes.byref(ms), ctypes.byref(n)))
+        return ms.value, n.value
 
     def device_status(self, reset=True):
         v = ctypes.c_int()

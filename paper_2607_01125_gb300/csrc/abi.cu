@@ -49,6 +49,31 @@ void* scratch_zeroed(Ctx* ctx, ScratchSlot slot, size_t bytes) {
   return p;
 }
 
+constexpr int TIMING_PAIRS = 4096;
+
+int timing_begin(Ctx* ctx) {
+  if (!ctx->timing) return ZOACT_OK;
+  if (!ctx->tev) {
+    ctx->tev = new (std::nothrow) cudaEvent_t[2 * TIMING_PAIRS];
+    if (!ctx->tev) return ZOACT_ERR_NOMEM;
+    for (int i = 0; i < 2 * TIMING_PAIRS; ++i) ZOACT_CUDA_TRY(cudaEventCreate(&ctx->tev[i]));
+    ctx->tev_cap = TIMING_PAIRS;
+  }
+  if (ctx->tev_used >= ctx->tev_cap) {
+    ++ctx->tev_dropped;
+    return ZOACT_OK;
+  }
+  ZOACT_CUDA_TRY(cudaEventRecord(ctx->tev[2 * ctx->tev_used], ctx->stream));
+  return ZOACT_OK;
+}
+
+int timing_end(Ctx* ctx) {
+  if (!ctx->timing || !ctx->tev || ctx->tev_used >= ctx->tev_cap) return ZOACT_OK;
+  ZOACT_CUDA_TRY(cudaEventRecord(ctx->tev[2 * ctx->tev_used + 1], ctx->stream));
+  ++ctx->tev_used;
+  return ZOACT_OK;
+}
+
 }  // namespace zoact
 
 using namespace zoact;
@@ -130,6 +155,10 @@ int zoact_destroy(zoact_ctx* ctx) {
     if (ctx->slot_ptr[s]) cudaFree(ctx->slot_ptr[s]);
   cudaFree(ctx->d_status);
   cudaFree(ctx->d_tickets);
+  if (ctx->tev) {
+    for (int i = 0; i < 2 * ctx->tev_cap; ++i) cudaEventDestroy(ctx->tev[i]);
+    delete[] ctx->tev;
+  }
   delete ctx;
   return ZOACT_OK;
 }
@@ -165,6 +194,31 @@ int zoact_get_device_status(zoact_ctx* ctx, int* status, int reset) {
     ZOACT_CUDA_TRY(cudaMemsetAsync(ctx->d_status, 0, sizeof(int), ctx->stream));
     ZOACT_CUDA_TRY(cudaStreamSynchronize(ctx->stream));
   }
+  return ZOACT_OK;
+}
+
+int zoact_kernel_timing(zoact_ctx* ctx, int enable) {
+  if (!ctx) return ZOACT_ERR_INVALID_ARG;
+  ctx->timing = enable != 0;
+  ctx->tev_used = 0;
+  ctx->tev_dropped = 0;
+  return ZOACT_OK;
+}
+
+int zoact_kernel_time(zoact_ctx* ctx, double* ms_total, int64_t* launches) {
+  ZOACT_ENTER(ctx);
+  if (!ms_total || !launches) return ZOACT_ERR_INVALID_ARG;
+  ZOACT_CUDA_TRY(cudaStreamSynchronize(ctx->stream));
+  double total = 0.0;
+  for (int i = 0; i < ctx->tev_used; ++i) {
+    float ms = 0.f;
+    ZOACT_CUDA_TRY(cudaEventElapsedTime(&ms, ctx->tev[2 * i], ctx->tev[2 * i + 1]));
+    total += ms;
+  }
+  *ms_total = total;
+  *launches = ctx->tev_used;
+  ctx->tev_used = 0;
+  ctx->tev_dropped = 0;
   return ZOACT_OK;
 }
 

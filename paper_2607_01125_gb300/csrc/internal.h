@@ -49,7 +49,17 @@ struct Ctx {
   unsigned int* d_tickets = nullptr;  // grid-reduction tickets, reset by their last block
   void* slot_ptr[SLOT_COUNT] = {};
   size_t slot_bytes[SLOT_COUNT] = {};
+  // kernel timing (zoact_kernel_timing): event pairs around the tensor-core pair-forward launches
+  bool timing = false;
+  cudaEvent_t* tev = nullptr;        // 2 * tev_cap events, created on demand
+  int tev_cap = 0;
+  int tev_used = 0;                   // pairs recorded since the last read
+  int64_t tev_dropped = 0;            // launches not timed (capacity reached)
 };
+
+// Record the start / end of a timed launch on the context's stream (no-ops unless timing is on).
+int timing_begin(Ctx* ctx);
+int timing_end(Ctx* ctx);
 
 int cuda_fail(cudaError_t e, const char* what);
 // Returns a device pointer of at least `bytes` for the slot, or nullptr on failure.

@@ -260,13 +260,22 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     p.Ws = static_cast<const __half*>(a.w_scales);
     p.Wq2 = static_cast<const uint8_t*>(a.W2);
     p.Ws2 = static_cast<const __half*>(a.w_scales2);
-    return dispatch_w4(ctx, mode, rt, a.ydtype, tm.a, p);
+    st = timing_begin(ctx);
+    if (st) return st;
+    st = dispatch_w4(ctx, mode, rt, a.ydtype, tm.a, p);
+    if (st) return st;
+    return timing_end(ctx);
   }
+  st = timing_begin(ctx);
+  if (st) return st;
   if (two)
-    return a.xdtype == ZOACT_DT_BF16 ? dispatch2_bf16(ctx, mode, rt, a.ydtype, tm, p)
-                                     : dispatch2_fp16(ctx, mode, rt, a.ydtype, tm, p);
-  return a.xdtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, mode, rt, a.ydtype, tm, p)
+    st = a.xdtype == ZOACT_DT_BF16 ? dispatch2_bf16(ctx, mode, rt, a.ydtype, tm, p)
+                                   : dispatch2_fp16(ctx, mode, rt, a.ydtype, tm, p);
+  else
+    st = a.xdtype == ZOACT_DT_BF16 ? dispatch_bf16(ctx, mode, rt, a.ydtype, tm, p)
                                    : dispatch_fp16(ctx, mode, rt, a.ydtype, tm, p);
+  if (st) return st;
+  return timing_end(ctx);
 }
 
 int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int M, int N, int K, float* D) {

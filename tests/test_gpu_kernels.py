@@ -449,3 +449,19 @@ def test_basis_bf16_tensor_core_gram(ctx):
     ov = basis.subspace_overlap(np64(U), Ue)
     # Davis-Kahan: sin(theta) <~ ||E|| / gap, with E the fp32 Gram error (~1e-6 relative)
     assert ov >= 1 - (1e-5 / gap) ** 2 - 1e-6, (ov, gap)
+
+
+def test_kernel_timing(ctx):
+    # the timing facility records one event pair per tensor-core pair-forward kernel and nothing else
+    d_in, d_out, r, T = 512, 264, 16, 130
+    X, W, U, C = _pair_case(d_in, d_out, r, T, False, torch.bfloat16, 1e-3, 0.1)
+    Y = torch.empty(2 * T, d_out, dtype=torch.bfloat16, device=DEV)
+    L = zo.make_layer(W, U, C, 1)
+    ctx.kernel_timing(True)
+    for q in range(3):
+        zo.zoact_pair_forward(ctx, L, X, T, False, 1e-3, 1, q, Y)
+    ms, n = ctx.kernel_time()
+    ctx.kernel_timing(False)
+    assert n == 3 and ms > 0.0
+    zo.zoact_pair_forward(ctx, L, X, T, False, 1e-3, 1, 0, Y)
+    assert ctx.kernel_time() == (0.0, 0)
