@@ -133,12 +133,22 @@ aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const
       const int mat = (int)(rest / blk.nzq);
       float* dst = (mat ? Zt2 : Zt) + (int64_t)qi * r * d_out;
       const uint32_t layer = mat ? lid2 : lid;
+      if ((r & 3) == 0) {
+        // the four ranks are one Philox group
+        const float4 z = z_normals4(seed, layer, blk.zq[qi], (uint64_t)(((int64_t)n * r + 4 * jg) >> 2));
+        dst[(int64_t)(4 * jg) * d_out + n] = z.x;
+        dst[(int64_t)(4 * jg + 1) * d_out + n] = z.y;
+        dst[(int64_t)(4 * jg + 2) * d_out + n] = z.z;
+        dst[(int64_t)(4 * jg + 3) * d_out + n] = z.w;
+      } else {
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int j = 4 * jg + i;
-        if (j < r) {
-          const int64_t e = (int64_t)n * r + j;
-          dst[(int64_t)j * d_out + n] = z_select(z_normals4(seed, layer, blk.zq[qi], (uint64_t)(e >> 2)), (int)(e & 3));
+        for (int i = 0; i < 4; ++i) {
+          const int j = 4 * jg + i;
+          if (j < r) {
+            const int64_t e = (int64_t)n * r + j;
+            dst[(int64_t)j * d_out + n] =
+                z_select(z_normals4(seed, layer, blk.zq[qi], (uint64_t)(e >> 2)), (int)(e & 3));
+          }
         }
       }
     }

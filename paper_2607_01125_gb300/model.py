@@ -262,6 +262,41 @@ class ZOStep:
         return self.loss_out
 
 
+def run_from_host(batches, step_fn, out_host):
+    """Run one ZO step per batch of PINNED host tensors, overlapping each batch's host-to-device copy
+    (on a side stream, into one of two device buffer sets) with the previous step's compute.
+
+    batches: list of tuples of pinned host tensors (e.g. (x, target) or (x,)); step_fn(device_tensors, i)
+    issues step i on torch's current stream and returns its device loss vector, which is copied back
+    into out_host[i] (pinned).  Returns after issuing all work (no synchronisation).
+    """
+    if not batches:
+        return
+    main = torch.cuda.current_stream()
+    side = torch.cuda.Stream()
+    bufs = [[torch.empty(h.shape, dtype=h.dtype, device=main.device) for h in batches[0]] for _ in range(2)]
+    copied = [torch.cuda.Event(), torch.cuda.Event()]
+    free = [torch.cuda.Event(), torch.cuda.Event()]
+
+    def fetch(i):
+        b = i % 2
+        side.wait_stream(main) if i < 2 else side.wait_event(free[b])   # buffer b no longer read
+        with torch.cuda.stream(side):
+            for d, h in zip(bufs[b], batches[i]):
+                d.copy_(h, non_blocking=True)
+            copied[b].record(side)
+
+    fetch(0)
+    for i in range(len(batches)):
+        if i + 1 < len(batches):
+            fetch(i + 1)
+        b = i % 2
+        main.wait_event(copied[b])
+        out = step_fn(bufs[b], i)
+        free[b].record(main)
+        out_host[i].copy_(out, non_blocking=True)
+
+
 def coefficient_offsets(specs, r):
     """Offsets (multiples of 4) of each layer's [d_out, r] block in the flat arena."""
     offs, cur = [], 0
