@@ -40,7 +40,7 @@ LR = 1e-4
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one step's pair launches, from one ncu
 # capture of the current kernels at the default sizes; workloads without such a capture report null.
-PAIR_TRAFFIC_BYTES = {"llama_mlp_bf16": 900.9e6}
+PAIR_TRAFFIC_BYTES = {"llama_mlp_bf16": 902.8e6}
 
 
 def _peaks():
@@ -233,10 +233,8 @@ def run_ours(args):
         run_step(step, x, target, t, seed, world); t += 1
         torch.cuda.synchronize()
 
-    # ---- timed region: exactly args.steps steps ----
+    # ---- timed region: exactly args.steps steps, no per-kernel instrumentation ----
     n0 = ctx.launch_count()
-    step.timer = []
-    ctx.kernel_timing(True)              # events around each tensor-core pair-forward kernel
     barrier(); torch.cuda.synchronize()
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.nvtx.range_push("timed")          # profilers select the timed steps by this range
@@ -248,9 +246,22 @@ def run_ours(args):
     torch.cuda.synchronize(); barrier()
     launches = ctx.launch_count() - n0
     ms = start.elapsed_time(end) / args.steps
-    gemm_ms = sum(a.elapsed_time(b) for a, b, _ in step.timer)
-    gemm_flops = sum(f for _, _, f in step.timer)
-    step.timer = None
+
+    # ---- kernel timing: the same number of steps again, with the library recording CUDA events on its
+    # stream around every tensor-core pair-forward kernel (the events themselves lengthen a step by a few
+    # per cent, so the throughput above is taken without them) ----
+    step.flops = []
+    ctx.kernel_timing(True)
+    barrier(); torch.cuda.synchronize()
+    i_s, i_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    i_s.record()
+    for _ in range(args.steps):
+        run_step(step, x, target, t, seed, world); t += 1
+    i_e.record()
+    torch.cuda.synchronize(); barrier()
+    instr_ms = i_s.elapsed_time(i_e) / args.steps
+    gemm_flops = sum(step.flops)
+    step.flops = None
     kern_ms, kern_launches = ctx.kernel_time()
     ctx.kernel_timing(False)
 
@@ -303,15 +314,16 @@ def run_ours(args):
                    "parallelism": f"dp{world}" if world > 1 else "single"},
         "evaluated_tokens_per_s": world * step.nb * T / (ms * 1e-3),
         "zo_steps_per_s": 1e3 / ms,
-        "pair_forward_ms_per_step": gemm_ms / args.steps,
         "pair_kernel_ms_per_step": kern_ms / args.steps,
+        "instrumented_ms_per_step": instr_ms,
         "pair_kernel_launches": kern_launches,
         "basis_init_s": basis_s,
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak,
                      "peak_kind": f"bf16 dense {'sustained' if long_step else 'burst'}, {peak_kind}",
                      "kernel": "pair_tc2_kernel / pair_tc_kernel (every pair-forward launch of the step, "
-                               "timed alone by events on the library's stream)",
+                               "timed alone by events on the library's stream over a second run of the same "
+                               "number of steps)",
                      "algorithmic_flops_per_step": gemm_flops / args.steps,
                      "traffic": (PAIR_TRAFFIC_BYTES.get(w.name)
                                  if args.tokens is None and args.queries is None and args.rank is None else None),

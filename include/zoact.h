@@ -124,6 +124,8 @@ int zoact_get_launch_count(zoact_ctx* ctx, int64_t* count);
 /* Kernel timing: with enable != 0 the context records CUDA events on its stream
  * around every tensor-core pair-forward kernel (the MMA kernel alone, without
  * the preparation kernels of the same call; up to 4096 launches between reads).
+ * Switching it on creates the event pool (ZOACT_ERR_CUDA if that fails).  The
+ * events themselves lengthen a step: measure throughput with timing off.
  * zoact_kernel_timing(ctx, 0/1) switches it and forgets recorded launches;
  * zoact_kernel_time synchronises the stream and returns the summed duration (ms)
  * and the number of timed launches since the last read, then forgets them.      */

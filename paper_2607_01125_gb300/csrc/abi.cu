@@ -51,14 +51,25 @@ void* scratch_zeroed(Ctx* ctx, ScratchSlot slot, size_t bytes) {
 
 constexpr int TIMING_PAIRS = 4096;
 
-int timing_begin(Ctx* ctx) {
-  if (!ctx->timing) return ZOACT_OK;
-  if (!ctx->tev) {
-    ctx->tev = new (std::nothrow) cudaEvent_t[2 * TIMING_PAIRS];
-    if (!ctx->tev) return ZOACT_ERR_NOMEM;
-    for (int i = 0; i < 2 * TIMING_PAIRS; ++i) ZOACT_CUDA_TRY(cudaEventCreate(&ctx->tev[i]));
-    ctx->tev_cap = TIMING_PAIRS;
+// The event pool is created when timing is switched on, so that no launch pays for it.
+int timing_pool(Ctx* ctx) {
+  if (ctx->tev) return ZOACT_OK;
+  ctx->tev = new (std::nothrow) cudaEvent_t[2 * TIMING_PAIRS];
+  if (!ctx->tev) return ZOACT_ERR_NOMEM;
+  for (int i = 0; i < 2 * TIMING_PAIRS; ++i) {
+    if (cudaEventCreate(&ctx->tev[i]) != cudaSuccess) {
+      for (int j = 0; j < i; ++j) cudaEventDestroy(ctx->tev[j]);
+      delete[] ctx->tev;
+      ctx->tev = nullptr;
+      return ZOACT_ERR_CUDA;
+    }
   }
+  ctx->tev_cap = TIMING_PAIRS;
+  return ZOACT_OK;
+}
+
+int timing_begin(Ctx* ctx) {
+  if (!ctx->timing || !ctx->tev) return ZOACT_OK;
   if (ctx->tev_used >= ctx->tev_cap) {
     ++ctx->tev_dropped;
     return ZOACT_OK;
@@ -198,7 +209,11 @@ int zoact_get_device_status(zoact_ctx* ctx, int* status, int reset) {
 }
 
 int zoact_kernel_timing(zoact_ctx* ctx, int enable) {
-  if (!ctx) return ZOACT_ERR_INVALID_ARG;
+  ZOACT_ENTER(ctx);
+  if (enable) {
+    const int st = timing_pool(ctx);
+    if (st != ZOACT_OK) return st;
+  }
   ctx->timing = enable != 0;
   ctx->tev_used = 0;
   ctx->tev_dropped = 0;

@@ -44,78 +44,126 @@ __device__ __forceinline__ uint32_t pack_bf16x2(__nv_bfloat16 a, __nv_bfloat16 b
   return (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(b) << 16);
 }
 
-// One warp per output row: rows [0, nA) of A_aug, then the nB rows of B_aug
-// (block b, column n), then those of B_aug2.  The warp stages the row's r source
-// values (and those of the second projection, distinct gated A rows only) in its
-// slice of shared memory, then writes the row as bf16 pairs, each lane splitting
-// its K columns' source values into hi/lo.  r <= 256.
+// The split parts of four consecutive ranks j0..j0+3 of one source row: hi
+// (want_lo false) or lo, packed as bf16 pairs.
+__device__ __forceinline__ uint2 split_quad(float4 v, bool want_lo) {
+  __nv_bfloat16 h[4], l[4];
+  split16(v.x, h[0], l[0]);
+  split16(v.y, h[1], l[1]);
+  split16(v.z, h[2], l[2]);
+  split16(v.w, h[3], l[3]);
+  const __nv_bfloat16* o = want_lo ? l : h;
+  return make_uint2(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]));
+}
+
+// One thread per 16-byte chunk (8 K columns) of an output row: rows [0, nA)
+// of A_aug, then the nB rows of B_aug (block b, column n), then those of
+// B_aug2.  Each column k of a row maps to (slot, half, part, rank j); the chunk
+// is built from the source values it needs (P or P2 for A rows, T = C + c_b Z_b
+// for B rows; source rows are re-read from L1/L2 by the row's chunks).  With
+// QUAD (r a multiple of 4 and 16-byte aligned sources) every 4 columns are one
+// part of one slot: one float4 load and one Philox call per 4 columns.
+template <bool QUAD>
 __global__ void __launch_bounds__(256)
 aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const float* __restrict__ C,
                 const float* __restrict__ C2, __nv_bfloat16* __restrict__ A, __nv_bfloat16* __restrict__ B,
                 __nv_bfloat16* __restrict__ B2, int64_t rows, int d_out, int r, int ka, int distinct, int full,
                 int nb, const __grid_constant__ AugBlocks blk, uint64_t seed, uint32_t lid, uint32_t lid2,
                 float* __restrict__ Zt, float* __restrict__ Zt2, int slots, int64_t T) {
-  __shared__ float stage[8][2][256];
-  const int lane = threadIdx.x & 31;
-  float* s0 = stage[threadIdx.x >> 5][0];
-  float* s1 = stage[threadIdx.x >> 5][1];
-  const int ka_row = distinct ? 2 * ka : ka;          // columns of one slot
-  const int ka_tot_a = slots * ka_row;                // A_aug row width
-  const int ka_tot = ka_row;                          // B_aug row width
+  const int ka_row = distinct ? 2 * ka : ka;          // columns of one slot (= B_aug row width)
+  const int cA = slots * ka_row / 8, cB = ka_row / 8; // 16-byte chunks per A / B row
   const int nbB = full ? nb : 1;
-  const int64_t nA = rows;
   const int64_t nB = (int64_t)nbB * d_out;
-  const int64_t total = nA + (B2 ? 2 * nB : nB);
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; w < total; w += nwarps) {
-    const bool is_a = w < nA;
+  const int64_t itA = rows * cA;
+  const int64_t items = itA + (B2 ? 2 : 1) * nB * cB;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < items; it += stride) {
+    const bool is_a = it < itA;
     bool up = false;
     int64_t orow;
-    __syncwarp();                                    // the previous row's readers are done with the stage
+    int c;
     if (is_a) {
-      orow = w;
-      for (int j = lane; j < r; j += 32) {
-        s0[j] = P[w * r + j];
-        if (distinct) s1[j] = P2[w * r + j];
-      }
+      orow = it / cA;
+      c = (int)(it - orow * cA);
     } else {
-      const int64_t ib = w - nA;
-      up = ib >= nB;
-      orow = up ? ib - nB : ib;                      // b * d_out + n
-      const int b = (int)(orow / d_out), n = (int)(orow - (int64_t)b * d_out);
-      const float cb = full ? blk.coef[b] : 0.f;
-      for (int j = lane; j < r; j += 32) {
-        const int64_t e = (int64_t)n * r + j;
-        float v = (up ? C2 : C)[e];
-        if (cb != 0.f)
-          v = fmaf(cb, z_select(z_normals4(seed, up ? lid2 : lid, blk.qry[b], (uint64_t)(e >> 2)), (int)(e & 3)), v);
-        s0[j] = v;
-      }
+      const int64_t ib = it - itA;
+      const int64_t rb = ib / cB;
+      c = (int)(ib - rb * cB);
+      up = rb >= nB;
+      orow = up ? rb - nB : rb;                      // b * d_out + n
     }
-    __syncwarp();
-    __nv_bfloat16* dst = is_a ? A : (up ? B2 : B);
-    const int row_w = is_a ? ka_tot_a : ka_tot;
-    const int my_slot = (is_a && slots > 1) ? (int)((orow / T) % slots) : 0;
-    uint32_t* drow = reinterpret_cast<uint32_t*>(dst + orow * row_w);
-    for (int wd = lane; wd < row_w / 2; wd += 32) {
-      __nv_bfloat16 o[2];
+    int my_slot = 0, n = 0;
+    float cb = 0.f;
+    uint64_t q = 0;
+    if (is_a) {
+      if (slots > 1) my_slot = (int)((orow / T) % slots);
+    } else {
+      const int b = (int)(orow / d_out);
+      n = (int)(orow - (int64_t)b * d_out);
+      if (full) { cb = blk.coef[b]; q = blk.qry[b]; }
+    }
+    const uint32_t layer = up ? lid2 : lid;
+    uint32_t w[4];
 #pragma unroll
-      for (int e2 = 0; e2 < 2; ++e2) {
-        const int slot = (2 * wd + e2) / ka_row;
-        const int k = 2 * wd + e2 - slot * ka_row;
-        const int half = k >= ka ? 1 : 0, kk = k - half * ka;
-        const int part = kk / r, j = kk - part * r;
-        // A: [hi | hi | lo], B: [hi | lo | hi]
-        const bool want_lo = is_a ? part == 2 : part == 1;
-        const bool second = is_a && half == 1;       // distinct A: the up projection's parts
+    for (int h4 = 0; h4 < 2; ++h4) {
+      if (QUAD) {
+        const int k0 = 8 * c + 4 * h4;
+        const int slot = k0 / ka_row;
+        const int kk = k0 - slot * ka_row;
+        const int half = kk >= ka ? 1 : 0, kq = kk - half * ka;
+        const int part = kq / r, j0 = kq - part * r;
+        // A: [hi | hi | lo], B: [hi | lo | hi]; distinct gated A: [gate parts | up parts];
         // distinct gated B: gate rows fill the first half, up rows the second
         const bool live = part < 3 && slot == my_slot && (is_a || !distinct || half == (up ? 1 : 0));
-        __nv_bfloat16 hi = __float2bfloat16_rn(0.f), lo = hi;
-        if (live) split16(second ? s1[j] : s0[j], hi, lo);
-        o[e2] = live ? (want_lo ? lo : hi) : __float2bfloat16_rn(0.f);
+        uint2 o = make_uint2(0u, 0u);
+        if (live) {
+          float4 v;
+          if (is_a) {
+            v = *reinterpret_cast<const float4*>((distinct && half ? P2 : P) + orow * r + j0);
+          } else {
+            const int64_t e = (int64_t)n * r + j0;
+            v = *reinterpret_cast<const float4*>((up ? C2 : C) + e);
+            if (cb != 0.f) {
+              const float4 z = z_normals4(seed, layer, q, (uint64_t)(e >> 2));
+              v.x = fmaf(cb, z.x, v.x); v.y = fmaf(cb, z.y, v.y);
+              v.z = fmaf(cb, z.z, v.z); v.w = fmaf(cb, z.w, v.w);
+            }
+          }
+          o = split_quad(v, is_a ? part == 2 : part == 1);
+        }
+        w[2 * h4] = o.x;
+        w[2 * h4 + 1] = o.y;
+      } else {
+        __nv_bfloat16 e4[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int k = 8 * c + 4 * h4 + i;
+          const int slot = k / ka_row;
+          const int kk = k - slot * ka_row;
+          const int half = kk >= ka ? 1 : 0, kq = kk - half * ka;
+          const int part = kq / r, j = kq - part * r;
+          const bool live = part < 3 && slot == my_slot && (is_a || !distinct || half == (up ? 1 : 0));
+          __nv_bfloat16 hi = __float2bfloat16_rn(0.f), lo = hi;
+          if (live) {
+            float v;
+            if (is_a) {
+              v = (distinct && half ? P2 : P)[orow * r + j];
+            } else {
+              const int64_t e = (int64_t)n * r + j;
+              v = (up ? C2 : C)[e];
+              if (cb != 0.f) v = fmaf(cb, z_select(z_normals4(seed, layer, q, (uint64_t)(e >> 2)), (int)(e & 3)), v);
+            }
+            split16(v, hi, lo);
+          }
+          e4[i] = live ? ((is_a ? part == 2 : part == 1) ? lo : hi) : __float2bfloat16_rn(0.f);
+        }
+        w[2 * h4] = pack_bf16x2(e4[0], e4[1]);
+        w[2 * h4 + 1] = pack_bf16x2(e4[2], e4[3]);
       }
-      drow[wd] = pack_bf16x2(o[0], o[1]);
     }
+    __nv_bfloat16* dst = is_a ? A : (up ? B2 : B);
+    const int64_t row_w = 8 * (int64_t)(is_a ? cA : cB);
+    *reinterpret_cast<uint4*>(dst + orow * row_w + 8 * c) = make_uint4(w[0], w[1], w[2], w[3]);
   }
   // transposed Z tables: Zt[q][j][n] for each distinct query (gate, then up); one thread per
   // (matrix, query, group of 4 ranks, column n), columns fastest so that the stores coalesce
@@ -155,6 +203,8 @@ aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const
   }
 }
 
+bool aligned16_or_null(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
 }  // namespace
 
 int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct, int slots, void* A_aug,
@@ -164,15 +214,20 @@ int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct,
   for (int i = 0; i < nzq; ++i) blk.zq[i] = zq[i];
   blk.nzq = Zt ? nzq : 0;
   const int full = mode == LOWRANK_ALL_ON_TC;
-  const int ka_tot = distinct ? 2 * ka : ka;
-  (void)ka_tot;
+  const int ka_row = distinct ? 2 * ka : ka;
   const int64_t nbB = full ? a.nb : 1;
-  const int64_t total_rows = a.rows + (B_aug2 ? 2 : 1) * nbB * a.d_out;   // one warp per row, 8 per block
-  int64_t grid = (total_rows + 7) / 8;
-  const int64_t cap = (int64_t)ctx->sm_count * 16;
+  const int64_t items = a.rows * (slots * ka_row / 8) + (B_aug2 ? 2 : 1) * nbB * a.d_out * (ka_row / 8);
+  const int64_t z_items = Zt ? (int64_t)(Zt2 ? 2 : 1) * blk.nzq * ((a.r + 3) / 4) * a.d_out : 0;
+  const int64_t work = items > z_items ? items : z_items;
+  int64_t grid = (work + 255) / 256;
+  const int64_t cap = (int64_t)ctx->sm_count * 32;
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
-  aug_prep_kernel<<<(unsigned)grid, 256, 0, ctx->stream>>>(
+  // float4 source loads need 16-byte aligned rows: r a multiple of 4 and aligned bases (null: unused)
+  const bool quad = a.r % 4 == 0 && aligned16_or_null(a.P) && aligned16_or_null(distinct ? a.P2 : nullptr) &&
+                    aligned16_or_null(a.C) && aligned16_or_null(a.C2);
+  auto kern = quad ? aug_prep_kernel<true> : aug_prep_kernel<false>;
+  kern<<<(unsigned)grid, 256, 0, ctx->stream>>>(
       a.P, distinct ? a.P2 : nullptr, a.C, a.C2, static_cast<__nv_bfloat16*>(A_aug),
       static_cast<__nv_bfloat16*>(B_aug), static_cast<__nv_bfloat16*>(B_aug2), a.rows, a.d_out, a.r, ka, distinct,
       full, a.nb, blk, a.seed, a.layer_id, a.layer_id2, Zt, Zt2, slots, a.T);

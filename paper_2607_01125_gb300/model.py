@@ -29,8 +29,8 @@ Graph wiring (names follow synth.Workload):
 
 Hooks: `capture(name, X)` is called with each linear's input (the + half)
 before its pair forward -- Algorithm 1's calibration pass uses it to take the
-bases; `timer`, when a list, receives (start event, end event, flops) around
-every tensor-core pair-forward launch.
+bases; `flops`, when a list, receives the algorithmic FLOP count (2 rows d_in
+d_out, gated x2) of every pair-forward call, with no events or synchronisation.
 """
 import torch
 
@@ -89,7 +89,7 @@ class ZOStep:
         self._pcache = {}
         self.device = dev
         self.capture = None
-        self.timer = None
+        self.flops = None
         self._utc = {}
         self.prepare_bases()
 
@@ -139,15 +139,10 @@ class ZOStep:
         self._pcache[slot] = (key, P)
         return P
 
-    def _timed(self, fn, flops):
-        if self.timer is None:
-            fn()
-            return
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
+    def _counted(self, fn, flops):
         fn()
-        e1.record()
-        self.timer.append((e0, e1, flops))
+        if self.flops is not None:
+            self.flops.append(flops)
 
     def query_ids(self, query):
         """The q Philox query ids of one one-sided step."""
@@ -169,7 +164,7 @@ class ZOStep:
         else:
             fn = lambda: Z.zoact_multi_forward(self.ctx, l.layer, X, self.T, shared, self.points(query), seed, Y,
                                                P=P, act=act)
-        self._timed(fn, flops)
+        self._counted(fn, flops)
         self._wrote(Y)
         return Y
 
@@ -188,7 +183,7 @@ class ZOStep:
         else:
             fn = lambda: Z.zoact_multi_forward_gated(self.ctx, g.layer, u.layer, X, self.T, shared,
                                                      self.points(query), seed, H, P_gate=Pg, P_up=Pu)
-        self._timed(fn, flops)
+        self._counted(fn, flops)
         self._wrote(H)
         return H
 
