@@ -138,6 +138,11 @@ int zoact_create(zoact_ctx** out, int device, void* stream) {
   if (!ctx) return ZOACT_ERR_NOMEM;
   ctx->device = device;
   ctx->stream = static_cast<cudaStream_t>(stream);
+  {
+    // programmatic dependent launch of the step's kernels: on unless ZOACT_PDL=0
+    const char* pdl = std::getenv("ZOACT_PDL");
+    ctx->pdl = !(pdl && pdl[0] == '0');
+  }
   int st = set_device(ctx);
   if (st) { delete ctx; return st; }
   if (cudaDeviceGetAttribute(&ctx->sm_count, cudaDevAttrMultiProcessorCount, device) != cudaSuccess) {

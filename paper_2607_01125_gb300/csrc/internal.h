@@ -45,6 +45,7 @@ struct Ctx {
   int sm_count = 0;
   int64_t n_launch = 0;              // kernels launched through this context (host counter)
   bool may_allocate = true;          // false: no scratch may be allocated (kernels that need none only)
+  bool pdl = false;                   // step-path kernels launched with programmatic dependent launch
   int* d_status = nullptr;            // device status word (first error wins)
   unsigned int* d_tickets = nullptr;  // grid-reduction tickets, reset by their last block
   void* slot_ptr[SLOT_COUNT] = {};
@@ -66,6 +67,35 @@ int cuda_fail(cudaError_t e, const char* what);
 void* scratch(Ctx* ctx, ScratchSlot slot, size_t bytes);
 // As scratch(), and a newly allocated buffer is zero-filled (on the context's stream).
 void* scratch_zeroed(Ctx* ctx, ScratchSlot slot, size_t bytes);
+
+// ---- programmatic dependent launch ----
+// launch_pdl puts a kernel on the context's stream; with ctx->pdl the launch
+// allows its blocks to be scheduled while the previous kernel on the stream
+// drains (from the moment every block of that kernel has called pdl_trigger()
+// or exited).  Every kernel launched this way calls pdl_wait() before its first
+// global memory access, read or write: it returns once the previous kernel has
+// completed and its writes are visible, so stream order holds for memory and
+// only the launch latency and the block prologue overlap the previous kernel.
+// A kernel calls pdl_trigger() only after its own pdl_wait(), which keeps the
+// chain transitive (kernel i+2 cannot start before kernel i has completed).
+// Both are no-ops in a kernel launched without the attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(Ctx* ctx, void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = ctx->stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = ctx->pdl ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<Args&&>(args)...);
+}
 
 // Device-side error recording: keeps the first non-zero code.
 __device__ __forceinline__ void record_error(int* status, int code) {

@@ -49,6 +49,8 @@ zo_update_kernel(float* __restrict__ C, float* __restrict__ m, float* __restrict
                  int64_t g_begin, int64_t g_end, const double* __restrict__ a_dev, int nq,
                  const __grid_constant__ QueryList qs, float lr, float b1, float b2, float adam_eps, float step_size,
                  float inv_sqrt_bc2, uint64_t seed, int* __restrict__ status) {
+  pdl_wait();                              // a (the loss kernel's output) is visible
+  pdl_trigger();
   bool finite = true;
   for (int j = 0; j < nq; ++j) finite = finite && isfinite(a_dev[j]);
   if (!finite) {
@@ -149,17 +151,10 @@ int launch_adam(Ctx* ctx, float* C, float* m, float* v, const zoact_coeff_block*
     int64_t nb = (g_end - g_begin + 255) / 256;
     const int64_t cap = (int64_t)ctx->sm_count * 8;
     if (nb > cap) nb = cap;
-    if (sgd) {
-      zo_update_kernel<true><<<(unsigned)nb, 256, 0, ctx->stream>>>(C, m, v, tab, g_begin, g_end, a, q, qs, lr, b1,
-                                                                    b2, adam_eps, step_size, inv_sqrt_bc2, seed,
-                                                                    ctx->d_status);
-    } else {
-      zo_update_kernel<false><<<(unsigned)nb, 256, 0, ctx->stream>>>(C, m, v, tab, g_begin, g_end, a, q, qs, lr, b1,
-                                                                     b2, adam_eps, step_size, inv_sqrt_bc2, seed,
-                                                                     ctx->d_status);
-    }
+    ZOACT_CUDA_TRY(launch_pdl(ctx, sgd ? zo_update_kernel<true> : zo_update_kernel<false>, dim3((unsigned)nb),
+                              dim3(256), 0, C, m, v, tab, g_begin, g_end, a, q, qs, lr, b1, b2, adam_eps, step_size,
+                              inv_sqrt_bc2, seed, ctx->d_status));
     ++ctx->n_launch;
-    ZOACT_CHECK_LAUNCH();
   }
   return ZOACT_OK;
 }

@@ -70,6 +70,8 @@ aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const
                 __nv_bfloat16* __restrict__ B2, int64_t rows, int d_out, int r, int ka, int distinct, int full,
                 int nb, const __grid_constant__ AugBlocks blk, uint64_t seed, uint32_t lid, uint32_t lid2,
                 float* __restrict__ Zt, float* __restrict__ Zt2, int slots, int64_t T) {
+  pdl_wait();                                         // P and C written by the previous kernels
+  pdl_trigger();
   const int ka_row = distinct ? 2 * ka : ka;          // columns of one slot (= B_aug row width)
   const int cA = slots * ka_row / 8, cB = ka_row / 8; // 16-byte chunks per A / B row
   const int nbB = full ? nb : 1;
@@ -227,10 +229,10 @@ int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct,
   const bool quad = a.r % 4 == 0 && aligned16_or_null(a.P) && aligned16_or_null(distinct ? a.P2 : nullptr) &&
                     aligned16_or_null(a.C) && aligned16_or_null(a.C2);
   auto kern = quad ? aug_prep_kernel<true> : aug_prep_kernel<false>;
-  kern<<<(unsigned)grid, 256, 0, ctx->stream>>>(
-      a.P, distinct ? a.P2 : nullptr, a.C, a.C2, static_cast<__nv_bfloat16*>(A_aug),
-      static_cast<__nv_bfloat16*>(B_aug), static_cast<__nv_bfloat16*>(B_aug2), a.rows, a.d_out, a.r, ka, distinct,
-      full, a.nb, blk, a.seed, a.layer_id, a.layer_id2, Zt, Zt2, slots, a.T);
+  ZOACT_CUDA_TRY(launch_pdl(ctx, kern, dim3((unsigned)grid), dim3(256), 0, a.P, distinct ? a.P2 : nullptr, a.C,
+                            a.C2, static_cast<__nv_bfloat16*>(A_aug), static_cast<__nv_bfloat16*>(B_aug),
+                            static_cast<__nv_bfloat16*>(B_aug2), a.rows, a.d_out, a.r, ka, distinct, full, a.nb, blk,
+                            a.seed, a.layer_id, a.layer_id2, Zt, Zt2, slots, a.T));
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;

@@ -13,6 +13,8 @@ namespace {
 
 __global__ void dequant_int4_kernel(const uint8_t* __restrict__ Wq, const __half* __restrict__ Ws,
                                     __nv_bfloat16* __restrict__ Wb, int64_t d_out, int d_in) {
+  pdl_wait();                              // the previous kernel may still read the scratch copy Wb
+  pdl_trigger();
   const int words_per_row = d_in / 8;                  // 8 nibbles per 32-bit word
   const int64_t n_words = d_out * words_per_row;
   const uint32_t* src = reinterpret_cast<const uint32_t*>(Wq);
@@ -41,10 +43,10 @@ int launch_dequant_int4(Ctx* ctx, const void* Wq, const void* Ws, void* Wb, int6
   const int64_t n_words = d_out * (d_in / 8);
   int64_t blocks = (n_words + 255) / 256;
   if (blocks > 16LL * ctx->sm_count) blocks = 16LL * ctx->sm_count;
-  dequant_int4_kernel<<<(unsigned)blocks, 256, 0, ctx->stream>>>(
-      static_cast<const uint8_t*>(Wq), static_cast<const __half*>(Ws), static_cast<__nv_bfloat16*>(Wb), d_out, d_in);
+  ZOACT_CUDA_TRY(launch_pdl(ctx, dequant_int4_kernel, dim3((unsigned)blocks), dim3(256), 0,
+                            static_cast<const uint8_t*>(Wq), static_cast<const __half*>(Ws),
+                            static_cast<__nv_bfloat16*>(Wb), d_out, d_in));
   ++ctx->n_launch;
-  ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
 }
 

@@ -25,6 +25,8 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 template <typename T>
 __global__ void __launch_bounds__(GLUE_THREADS)
 rms_norm_kernel(const T* __restrict__ X, T* __restrict__ Y, int n, float eps) {
+  pdl_wait();                              // the input rows written by the previous kernel
+  pdl_trigger();
   __shared__ float red[GLUE_THREADS / 32];
   const int64_t row = blockIdx.x;
   const T* x = X + row * n;
@@ -48,6 +50,8 @@ template <typename T>
 __global__ void __launch_bounds__(GLUE_THREADS)
 mix_rms_kernel(const T* __restrict__ Q, const T* __restrict__ K, const T* __restrict__ V, T* __restrict__ Y, int n,
                int n_rep, int head_dim, float eps) {
+  pdl_wait();                              // the input rows written by the previous kernel
+  pdl_trigger();
   __shared__ float red[GLUE_THREADS / 32];
   const int64_t row = blockIdx.x;
   const int nk = n / n_rep;
@@ -89,6 +93,8 @@ __device__ __forceinline__ uint4 f32_to_vec(const float* f) {
 template <typename T, int VPT>
 __global__ void __launch_bounds__(GLUE_THREADS)
 rms_norm_reg_kernel(const T* __restrict__ X, T* __restrict__ Y, int n, float eps) {
+  pdl_wait();                              // the input rows written by the previous kernel
+  pdl_trigger();
   constexpr int E = Vec<T>::N;
   __shared__ float red[GLUE_THREADS / 32];
   const int64_t row = blockIdx.x;
@@ -122,6 +128,8 @@ template <typename T, int VPT>
 __global__ void __launch_bounds__(GLUE_THREADS)
 mix_rms_reg_kernel(const T* __restrict__ Q, const T* __restrict__ K, const T* __restrict__ V, T* __restrict__ Y,
                    int n, int n_rep, int head_dim, float eps) {
+  pdl_wait();                              // the input rows written by the previous kernel
+  pdl_trigger();
   constexpr int E = Vec<T>::N;
   __shared__ float red[GLUE_THREADS / 32];
   const int64_t row = blockIdx.x;
@@ -181,15 +189,16 @@ int reg_vpt(int n) {
 template <typename T>
 int rms_dispatch(Ctx* ctx, const T* X, T* Y, int64_t rows, int n, float eps) {
   const int vpt = (aligned16(X) && aligned16(Y)) ? reg_vpt<T>(n) : 0;
+  void (*kern)(const T*, T*, int, float) = rms_norm_kernel<T>;
   switch (vpt) {
-    case 2: rms_norm_reg_kernel<T, 2><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(X, Y, n, eps); break;
-    case 4: rms_norm_reg_kernel<T, 4><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(X, Y, n, eps); break;
-    case 8: rms_norm_reg_kernel<T, 8><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(X, Y, n, eps); break;
-    case 12: rms_norm_reg_kernel<T, 12><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(X, Y, n, eps); break;
-    default: rms_norm_kernel<T><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(X, Y, n, eps); break;
+    case 2: kern = rms_norm_reg_kernel<T, 2>; break;
+    case 4: kern = rms_norm_reg_kernel<T, 4>; break;
+    case 8: kern = rms_norm_reg_kernel<T, 8>; break;
+    case 12: kern = rms_norm_reg_kernel<T, 12>; break;
+    default: break;
   }
+  ZOACT_CUDA_TRY(launch_pdl(ctx, kern, dim3((unsigned)rows), dim3(GLUE_THREADS), 0, X, Y, n, eps));
   ++ctx->n_launch;
-  ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
 }
 
@@ -200,15 +209,17 @@ int mix_dispatch(Ctx* ctx, const T* q, const T* k, const T* v, T* Y, int64_t row
   const bool ok = aligned16(q) && aligned16(k) && aligned16(v) && aligned16(Y) && head_dim % E == 0 &&
                   (n / n_rep) % E == 0;
   const int vpt = ok ? reg_vpt<T>(n) : 0;
+  void (*kern)(const T*, const T*, const T*, T*, int, int, int, float) = mix_rms_kernel<T>;
   switch (vpt) {
-    case 2: mix_rms_reg_kernel<T, 2><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(q, k, v, Y, n, n_rep, head_dim, eps); break;
-    case 4: mix_rms_reg_kernel<T, 4><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(q, k, v, Y, n, n_rep, head_dim, eps); break;
-    case 8: mix_rms_reg_kernel<T, 8><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(q, k, v, Y, n, n_rep, head_dim, eps); break;
-    case 12: mix_rms_reg_kernel<T, 12><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(q, k, v, Y, n, n_rep, head_dim, eps); break;
-    default: mix_rms_kernel<T><<<(unsigned)rows, GLUE_THREADS, 0, ctx->stream>>>(q, k, v, Y, n, n_rep, head_dim, eps); break;
+    case 2: kern = mix_rms_reg_kernel<T, 2>; break;
+    case 4: kern = mix_rms_reg_kernel<T, 4>; break;
+    case 8: kern = mix_rms_reg_kernel<T, 8>; break;
+    case 12: kern = mix_rms_reg_kernel<T, 12>; break;
+    default: break;
   }
+  ZOACT_CUDA_TRY(launch_pdl(ctx, kern, dim3((unsigned)rows), dim3(GLUE_THREADS), 0, q, k, v, Y, n, n_rep, head_dim,
+                            eps));
   ++ctx->n_launch;
-  ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
 }
 

@@ -115,6 +115,8 @@ __global__ void __launch_bounds__(LOSS_THREADS, 4)
 loss_pair_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t count, int vec_ok, float eps,
                  double* __restrict__ out, double* __restrict__ partials, unsigned int* __restrict__ ticket,
                  int* __restrict__ status) {
+  pdl_wait();                              // Y written by the previous kernel
+  pdl_trigger();
   const TY* yp = Y;
   const TY* ym = Y + count;
   CSum ap, am, ad;
@@ -234,9 +236,9 @@ int loss_dispatch(Ctx* ctx, const TY* Y, const TY* tgt, int64_t count, float eps
   int64_t blocks = ((vec_ok ? count / 8 : count) + LOSS_THREADS - 1) / LOSS_THREADS;
   if (blocks < 1) blocks = 1;
   if (blocks > max_blocks) blocks = max_blocks;
-  loss_pair_kernel<TY><<<(unsigned)blocks, LOSS_THREADS, 0, ctx->stream>>>(Y, tgt, count, vec_ok, eps, out,
-                                                                           partials, ticket, ctx->d_status); ++ctx->n_launch;
-  ZOACT_CHECK_LAUNCH();
+  ZOACT_CUDA_TRY(launch_pdl(ctx, loss_pair_kernel<TY>, dim3((unsigned)blocks), dim3(LOSS_THREADS), 0, Y, tgt, count,
+                            vec_ok, eps, out, partials, ticket, ctx->d_status));
+  ++ctx->n_launch;
   return ZOACT_OK;
 }
 
@@ -251,6 +253,8 @@ __global__ void __launch_bounds__(LOSS_THREADS, 4)
 loss_multi_kernel(const TY* __restrict__ Y, const TY* __restrict__ tgt, int64_t count, int vec_ok, int nb, float mu,
                   double* __restrict__ out, double* __restrict__ partials, unsigned int* __restrict__ ticket,
                   int* __restrict__ status) {
+  pdl_wait();
+  pdl_trigger();
   const int b = blockIdx.y;
   const TY* yb = Y + (int64_t)b * count;
   const TY* y0 = Y;
@@ -382,10 +386,9 @@ int loss_multi_dispatch(Ctx* ctx, const TY* Y, const TY* tgt, int64_t count, int
   if (cap < 1) cap = 1;
   if (bx > cap) bx = cap;
   dim3 grid((unsigned)bx, (unsigned)nb);
-  loss_multi_kernel<TY><<<grid, LOSS_THREADS, 0, ctx->stream>>>(Y, tgt, count, vec_ok, nb, mu, out, partials, ticket,
-                                                               ctx->d_status);
+  ZOACT_CUDA_TRY(launch_pdl(ctx, loss_multi_kernel<TY>, grid, dim3(LOSS_THREADS), 0, Y, tgt, count, vec_ok, nb, mu,
+                            out, partials, ticket, ctx->d_status));
   ++ctx->n_launch;
-  ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
 }
 

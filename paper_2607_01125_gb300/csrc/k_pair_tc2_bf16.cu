@@ -9,7 +9,7 @@ static int launch_two(Ctx* ctx, const TmaSet& tm, const Params& p) {
   auto kern = pair_tc2_kernel<TO, RT, MODE, 1>;
   ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES));
   const int clusters = p.num_tiles < ctx->sm_count / 2 ? p.num_tiles : ctx->sm_count / 2;
-  kern<<<2 * clusters, num_threads(false), SMEM2_BYTES, ctx->stream>>>(tm, p);
+  ZOACT_CUDA_TRY(launch_pdl(ctx, kern, dim3(2 * clusters), dim3(num_threads(false)), SMEM2_BYTES, tm, p));
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;

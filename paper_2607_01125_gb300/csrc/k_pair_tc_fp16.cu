@@ -9,7 +9,7 @@ static int launch_one(Ctx* ctx, const TmaSet& tm, const Params& p) {
   auto kern = pair_tc_kernel<TO, RT, MODE, 0, false>;
   ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
   const int grid = p.num_tiles < ctx->sm_count ? p.num_tiles : ctx->sm_count;
-  kern<<<grid, num_threads(false), SMEM_BYTES, ctx->stream>>>(tm, p); ++ctx->n_launch;
+  ZOACT_CUDA_TRY(launch_pdl(ctx, kern, dim3(grid), dim3(num_threads(false)), SMEM_BYTES, tm, p)); ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
 }

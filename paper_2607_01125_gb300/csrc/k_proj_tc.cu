@@ -96,6 +96,8 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ 
   __syncthreads();
   tc::tc_fence_after();
   const uint32_t tmem = ss->tmem_base;
+  pdl_wait();                             // X (the previous kernel's output) is visible
+  pdl_trigger();
 
   if (warp == 0 && lane == 0) {
     // ---- TMA producer ----
@@ -200,6 +202,8 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ 
 // P[t, j0 + j] = sum over splits of part[split][t][j] (split order), j < rg; P rows have stride ldp.
 __global__ void splitk_sum_kernel(const float* __restrict__ part, float* __restrict__ P, int64_t n, int splits, int rg,
                                   int ldp, int j0) {
+  pdl_wait();
+  pdl_trigger();
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
     float s = 0.f;
     for (int k = 0; k < splits; ++k) s += part[(int64_t)k * n + i];
@@ -213,7 +217,8 @@ int launch_one(Ctx* ctx, const CUtensorMap& mx, const CUtensorMap& mu, float* ou
                int kbps, int num_kb, dim3 grid) {
   auto kern = proj_tc_kernel<NB, RT, AB>;
   ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p_smem_bytes<NB>()));
-  kern<<<grid, 128, p_smem_bytes<NB>(), ctx->stream>>>(mx, mu, out, rows, r, ld_out, kbps, num_kb, ctx->d_status);
+  ZOACT_CUDA_TRY(launch_pdl(ctx, kern, grid, dim3(128), p_smem_bytes<NB>(), mx, mu, out, rows, r, ld_out, kbps,
+                            num_kb, ctx->d_status));
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
@@ -309,7 +314,8 @@ int launch_lowrank_proj_tc_prepared(Ctx* ctx, const void* X, int xdtype, int64_t
       const int64_t n = rows * rg;
       int64_t blocks = (n + 255) / 256;
       if (blocks > 4LL * ctx->sm_count) blocks = 4LL * ctx->sm_count;
-      splitk_sum_kernel<<<(unsigned)blocks, 256, 0, ctx->stream>>>(out, P, n, splits, rg, r, j0);
+      ZOACT_CUDA_TRY(launch_pdl(ctx, splitk_sum_kernel, dim3((unsigned)blocks), dim3(256), 0, out, P, n, splits, rg,
+                                r, j0));
       ++ctx->n_launch;
       ZOACT_CHECK_LAUNCH();
     }

@@ -153,6 +153,8 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
   tc2::cluster_sync();                    // both CTAs' barriers exist before any remote arrival
   tc::tc_fence_after();
   const uint32_t tmem_base = ss->tmem_base;
+  pdl_wait();                             // the previous kernel's outputs (X, P, operand tables) are visible
+  pdl_trigger();
 
   const int num_m = prm.num_m, num_n = prm.num_n, num_k = prm.num_k;
   const int total_k = num_k + prm.aug_kb;   // main K-blocks, then the low-rank ones

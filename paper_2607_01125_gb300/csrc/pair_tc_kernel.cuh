@@ -669,6 +669,8 @@ pair_tc_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
   __syncthreads();
   tc::tc_fence_after();
   const uint32_t tmem_base = ss->tmem_base;
+  pdl_wait();                             // the previous kernel's outputs (X, P, operand tables) are visible
+  pdl_trigger();
 
   const int num_m = prm.num_m, num_n = prm.num_n, num_k = prm.num_k;
   const int total_k = num_k + (W4 ? 0 : prm.aug_kb);   // main K-blocks, then the low-rank ones

@@ -186,3 +186,35 @@ def test_basis_full_width():
             assert basis.subspace_overlap(Ug, V[:, :r]) >= 1 - 1e-4
             np.testing.assert_allclose(n64(ev)[:r], lam[:r], rtol=1e-4)
     ctx.close()
+
+
+@pytest.mark.parametrize("name,n_dec,T", [("llama_stack_bf16", 2, 300), ("llama_stack_int4", 1, 64),
+                                          ("llama_mlp_bf16", 1, 256)])
+def test_dependent_launch_bit_identical(name, n_dec, T, monkeypatch):
+    # programmatic dependent launch only lets a kernel's blocks start early and wait in the kernel for the
+    # previous one: three whole steps (forward, loss, Adam) must match the fully serialised stream bit for bit
+    w = workload(name, T=T, n_decoder=n_dec)
+    step, _ = _build(w)
+    dt = torch.bfloat16 if w.act_dtype == "bf16" else torch.float16
+    x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=dt)
+    tgt = normal((w.T, w.d_model), tensor_seed(w, "t"), DEV, dtype=dt) if w.kind == "llama_mlp" else None
+    C0 = step.C.clone()
+    monkeypatch.setenv("ZOACT_PDL", "0")
+    serial = zo.Context(0)
+    runs = []
+    for ctx in (step.ctx, serial):
+        step.ctx = ctx
+        step.C.copy_(C0); step.m.zero_(); step.v.zero_()
+        outs = []
+        for t in range(1, 4):
+            Y = step.forward(x, 5, t)
+            outs.append((Y.clone(), step.loss(Y, tgt).clone()))
+            step.update(t, 5, t)
+        torch.cuda.synchronize()
+        assert ctx.device_status() == 0
+        runs.append((outs, step.C.clone(), step.m.clone(), step.v.clone()))
+    (o1, C1, m1, v1), (o2, C2, m2, v2) = runs
+    for (Ya, la), (Yb, lb) in zip(o1, o2):
+        assert torch.equal(Ya, Yb) and torch.equal(la, lb)
+    assert torch.equal(C1, C2) and torch.equal(m1, m2) and torch.equal(v1, v2)
+    serial.close()
