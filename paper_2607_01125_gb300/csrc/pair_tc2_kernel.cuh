@@ -20,15 +20,20 @@
 namespace zoact {
 namespace pairtc {
 
-constexpr int STAGES2 = 6;
+constexpr int STAGES2 = 6;        // ring depth beside the epilogue tables
+constexpr int STAGES2_NOTBL = 7;  // ring depth when the whole low-rank term is on the MMA (no tables)
 constexpr int B_HALF_BYTES = (BN / 2) * BK * 2;
 constexpr int STAGE2_BYTES = A_BYTES + B_HALF_BYTES;
-constexpr int SMEM2_BYTES = 1024 + STAGES2 * STAGE2_BYTES + TBL_FLOATS * 4 + 256;
+// Dynamic shared memory of a launch with ring depth nst: the table region exists only at the default depth.
+constexpr int smem2_bytes(int nst) {
+  return 1024 + nst * STAGE2_BYTES + (nst == STAGES2 ? TBL_FLOATS * 4 : 0) + 256;
+}
+constexpr int SMEM2_BYTES = smem2_bytes(STAGES2);
 constexpr int BM2 = 2 * BM;
 
 struct SharedState2 {
-  uint64_t full[STAGES2];
-  uint64_t empty[STAGES2];
+  uint64_t full[STAGES2_NOTBL];
+  uint64_t empty[STAGES2_NOTBL];
   uint64_t tmem_full[2];
   uint64_t tmem_empty[2];
   uint64_t drain;
@@ -37,7 +42,8 @@ struct SharedState2 {
   int epi_ok;
 };
 static_assert(sizeof(SharedState2) <= 256, "barrier block outgrew its shared-memory slot");
-static_assert(SMEM2_BYTES <= 232448, "dynamic shared memory above the 227 KB a CTA may use");
+static_assert(SMEM2_BYTES <= 232448 && smem2_bytes(STAGES2_NOTBL) <= 232448,
+              "dynamic shared memory above the 227 KB a CTA may use");
 
 namespace tc2 {
 
@@ -108,14 +114,25 @@ __device__ __forceinline__ void commit2_own(uint32_t bar) {
 
 }  // namespace tc2
 
-template <typename TO, int RT, int MODE, int AB_BF16>
+// NST: ring depth.  At STAGES2_NOTBL the epilogue-table region holds a seventh
+// stage instead, and the kernel serves only launches whose whole low-rank term
+// is on the MMA (aug_mode LOWRANK_ALL_ON_TC; any other launch records
+// ZOACT_ERR_INVALID_ARG and exits before touching shared memory).
+template <typename TO, int RT, int MODE, int AB_BF16, int NST = STAGES2>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(num_threads(false), 1)
 pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
   constexpr int CW = MODE == MODE_GATED ? 8 : 16;   // epilogue chunk width (gated: two accumulators)
+  constexpr bool NOTBL = NST != STAGES2;
+  static_assert(NST == STAGES2 || NST == STAGES2_NOTBL, "ring depth");
+  if (NOTBL && prm.aug_mode != LOWRANK_ALL_ON_TC) {   // uniform over the grid: both CTAs of a pair leave
+    pdl_wait();
+    if (threadIdx.x == 0 && blockIdx.x == 0) record_error(prm.status, ZOACT_ERR_INVALID_ARG);
+    return;
+  }
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  float* tbl = reinterpret_cast<float*>(smem + STAGES2 * STAGE2_BYTES);
-  SharedState2* ss = reinterpret_cast<SharedState2*>(tbl + TBL_FLOATS);
+  float* tbl = reinterpret_cast<float*>(smem + NST * STAGE2_BYTES);
+  SharedState2* ss = reinterpret_cast<SharedState2*>(tbl + (NOTBL ? 0 : TBL_FLOATS));
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -124,7 +141,7 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
   volatile int* abort_flag = &ss->abort_flag;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES2; ++s) {
+    for (int s = 0; s < NST; ++s) {
       tc::mbar_init(tc::smem_u32(&ss->full[s]), 2);     // one producer arrival from each CTA (leader's copy is used)
       tc::mbar_init(tc::smem_u32(&ss->empty[s]), 1);
     }
@@ -187,7 +204,7 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
                                   yb + n_blk * (BN / 2), full_leader);
           else
             tc2::tma_load_2d_pair(sb, aug ? &tm.ba : &tm.b, kxb, yb + n_blk * bn + (int)rank * bh, full_leader);
-          if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
+          if (++stage == NST) { stage = 0; phase ^= 1u; }
         }
       }
       if (!ok) {
@@ -225,7 +242,7 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
                           (kb | k) != 0 ? 1u : 0u);
           tc2::commit2_both(tc::smem_u32(&ss->empty[stage]));    // frees the stage in both CTAs
           issued_any = true;
-          if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
+          if (++stage == NST) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
         tc2::commit2_both(tc::smem_u32(&ss->tmem_full[buf]));   // accumulator ready in both CTAs
@@ -252,7 +269,7 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       const int64_t m = (int64_t)m_blk * BM2 + (int64_t)rank * BM + row_in_tile;
       const bool row_ok = m < prm.rows;
       const uint32_t t_row = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * BN);
-      const bool ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, tbl, etid, half,
+      const bool ok = epi_pair_tile<TO, RT, MODE, CW, NOTBL>(prm, ss, tbl, etid, half,
                                                       (int64_t)m_blk * BM2 + (int64_t)rank * BM, m, row_ok,
                                                       n_blk, bn, buf,
                                                       acc_phase, t_row, abort_flag);

@@ -435,7 +435,8 @@ __device__ __forceinline__ void load_p(float* p, const float* __restrict__ P, in
 // over the two signs of one query (coefficients +c, -c) builds one Z table and
 // forms acc +- c Z p.  With the whole term on the tensor cores it only converts
 // and stores.  Returns false when the wait gave up.
-template <typename TO, int RT, int MODE, int CW, typename SS>
+// ALL_ONLY: the launch has the whole low-rank term on the MMA (no tables exist).
+template <typename TO, int RT, int MODE, int CW, bool ALL_ONLY = false, typename SS>
 __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* tbl, int etid, int half,
                                               int64_t row0, int64_t m, bool row_ok, int n_blk, int bn, int buf,
                                               uint32_t acc_phase, uint32_t t_row, volatile int* abort_flag) {
@@ -448,7 +449,7 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
   const int64_t T = prm.T;
   TO* Y = static_cast<TO*>(prm.Y);
   const int ncol_tile = GATED ? BN / 2 : bn;               // output columns of this tile
-  if (prm.aug_mode == LOWRANK_ALL_ON_TC) {
+  if (ALL_ONLY || prm.aug_mode == LOWRANK_ALL_ON_TC) {
     // stacked rows, the whole low-rank term in the accumulator
     if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
     const int cbeg = half * (ncol_tile / 2);
@@ -473,6 +474,9 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
     }
     return true;
   }
+  if constexpr (ALL_ONLY) {
+    return true;
+  } else {
   const bool c_in_acc = prm.aug_mode == LOWRANK_C_ON_TC;
   float p[RT], p2[RT];
   const bool vec = prm.vec_ok != 0;
@@ -622,6 +626,7 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
     }
   }
   return true;
+  }  // !ALL_ONLY
 }
 
 template <typename TO, int RT, int MODE, int AB_BF16, bool W4>
