@@ -309,7 +309,9 @@ int zoact_sgd_step_multi(zoact_ctx* ctx, float* C, int64_t n_total, const zoact_
  * Rayleigh-Ritz.  Columns in descending eigenvalue order, each flipped so its
  * largest-magnitude entry is positive.  Optional evals_out [k] fp32 (device)
  * receives the Ritz values.  Requires k <= 512 and k <= d_in; uses d_in^2 * 4
- * bytes of context scratch.                                                    */
+ * bytes of context scratch.  Non-finite calibration data gives a non-finite
+ * basis and sets the device status word to ZOACT_ERR_NONFINITE (a column with
+ * no finite entry is left unflipped).                                          */
 int zoact_basis_init(zoact_ctx* ctx, const void* X_cal, int xdtype, int64_t n_tok, int32_t d_in,
                      int32_t r, int32_t oversample, int32_t n_iter, uint64_t seed, float* U_out,
                      float* evals_out);

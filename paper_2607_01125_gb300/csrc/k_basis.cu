@@ -490,7 +490,9 @@ __global__ void ritz_kernel(const float* __restrict__ Q, const double* __restric
 }
 
 // ---- flip column j so its largest-|.| entry (first index on ties) is positive ----
-__global__ void sign_fix_kernel(float* __restrict__ U, int d, int r) {
+// A column without a finite entry (non-finite calibration data) is left as it is and
+// the status word records ZOACT_ERR_NONFINITE.
+__global__ void sign_fix_kernel(float* __restrict__ U, int d, int r, int* __restrict__ status) {
   const int j = blockIdx.x;
   __shared__ float bv[256];
   __shared__ int bi[256];
@@ -514,7 +516,12 @@ __global__ void sign_fix_kernel(float* __restrict__ U, int d, int r) {
     }
     __syncthreads();
   }
-  const bool flip = U[(int64_t)bi[0] * r + j] < 0.f;
+  const int top = bi[0];
+  if (top < 0 || top >= d) {                 // no finite |U| in this column
+    if (threadIdx.x == 0) record_error(status, ZOACT_ERR_NONFINITE);
+    return;
+  }
+  const bool flip = U[(int64_t)top * r + j] < 0.f;
   __syncthreads();
   if (flip)
     for (int i = threadIdx.x; i < d; i += blockDim.x) U[(int64_t)i * r + j] = -U[(int64_t)i * r + j];
@@ -634,7 +641,7 @@ int run_basis_init(Ctx* ctx, const void* X, int xdtype, int64_t n_tok, int d, in
   }
   ++ctx->n_launch;
   ritz_kernel<<<(unsigned)(((int64_t)d * r + 255) / 256), 256, 0, ctx->stream>>>(w.Q, w.V, U_out, d, k, r); ++ctx->n_launch;
-  sign_fix_kernel<<<r, 256, 0, ctx->stream>>>(U_out, d, r); ++ctx->n_launch;
+  sign_fix_kernel<<<r, 256, 0, ctx->stream>>>(U_out, d, r, ctx->d_status); ++ctx->n_launch;
   if (evals_out) {
     f64_to_f32_kernel<<<1, 256, 0, ctx->stream>>>(w.ev, evals_out, k);
     ++ctx->n_launch;

@@ -75,6 +75,24 @@ int encode_tmap_2d_16bit(CUtensorMap* map, const void* base, int dtype, int64_t 
   return res == CUDA_SUCCESS ? ZOACT_OK : ZOACT_ERR_INVALID_ARG;
 }
 
+int encode_tmap_store(CUtensorMap* map, void* base, int ydtype, int64_t rows, int64_t cols, int box_cols,
+                      int box_rows, bool swizzle128) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return ZOACT_ERR_CUDA;
+  const size_t es = dtype_size(ydtype);
+  const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)cols * es};
+  const cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
+  const cuuint32_t estr[2] = {1u, 1u};
+  const CUtensorMapDataType dt = ydtype == ZOACT_DT_FP32   ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32
+                                 : ydtype == ZOACT_DT_FP16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
+                                                           : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  const CUresult res = fn(map, dt, 2, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                          CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return res == CUDA_SUCCESS ? ZOACT_OK : ZOACT_ERR_INVALID_ARG;
+}
+
 int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   using namespace pairtc;
   // ranks above 32 have no epilogue tables: the low-rank term must ride the MMA, which needs stacked rows
@@ -243,6 +261,17 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   p.num_tiles = p.num_m * p.num_n;
   p.ldy = a.d_out;
   p.aug_mode = lmode;
+  // CTA pairs with the whole term on the MMA write Y through staged bulk stores
+  tm.y = tm.y16 = tm.a;
+  p.y_staged = 0;
+  if (two && lmode == LOWRANK_ALL_ON_TC && rt == 4) {
+    const int es = (int)dtype_size(a.ydtype);
+    st = encode_tmap_store(&tm.y, a.Y, a.ydtype, a.rows, a.d_out, 128 / es, BM, true);
+    if (st) return st;
+    st = encode_tmap_store(&tm.y16, a.Y, a.ydtype, a.rows, a.d_out, 16, BM, false);
+    if (st) return st;
+    p.y_staged = 1;
+  }
   p.aug_kb = lmode == LOWRANK_EPILOGUE ? 0 : slots * ka_tot / BK;
   p.aug_kb_slot = ka_tot / BK;
   p.aug_slots = slots;
@@ -287,7 +316,7 @@ int launch_gemm_tc_f32out(Ctx* ctx, const void* A, const void* B, int dtype, int
   if (st) return st;
   st = encode_tmap_2d_16bit(&tm.b, B, dtype, N, K, bn);
   if (st) return st;
-  tm.b2 = tm.ba = tm.ba2 = tm.b;
+  tm.b2 = tm.ba = tm.ba2 = tm.y = tm.y16 = tm.b;
   tm.aa = tm.a;
   Params p{};
   p.Y = D;

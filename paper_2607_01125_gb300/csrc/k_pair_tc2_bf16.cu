@@ -4,13 +4,12 @@
 namespace zoact {
 namespace pairtc {
 
-template <typename TO, int RT, int MODE, int NST = STAGES2>
+template <typename TO, int RT, int MODE, bool STAGED = false>
 static int launch_two(Ctx* ctx, const TmaSet& tm, const Params& p) {
-  auto kern = pair_tc2_kernel<TO, RT, MODE, 1, NST>;
-  constexpr int smem = smem2_bytes(NST);
-  ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+  auto kern = pair_tc2_kernel<TO, RT, MODE, 1, STAGED>;
+  ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES));
   const int clusters = p.num_tiles < ctx->sm_count / 2 ? p.num_tiles : ctx->sm_count / 2;
-  ZOACT_CUDA_TRY(launch_pdl(ctx, kern, dim3(2 * clusters), dim3(num_threads(false)), smem, tm, p));
+  ZOACT_CUDA_TRY(launch_pdl(ctx, kern, dim3(2 * clusters), dim3(num_threads(false)), SMEM2_BYTES, tm, p));
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
@@ -18,10 +17,10 @@ static int launch_two(Ctx* ctx, const TmaSet& tm, const Params& p) {
 
 template <typename TO>
 static int by_rank_two(Ctx* ctx, int mode, int rt, const TmaSet& tm, const Params& p) {
-  // the whole low-rank term on the MMA (rank tile 4, no epilogue tables): a seven-stage ring
-  if (p.aug_mode == LOWRANK_ALL_ON_TC && rt == 4)
-    return mode == MODE_GATED ? launch_two<TO, 4, MODE_GATED, STAGES2_NOTBL>(ctx, tm, p)
-                              : launch_two<TO, 4, MODE_PAIR, STAGES2_NOTBL>(ctx, tm, p);
+  // the whole low-rank term on the MMA (rank tile 4, no epilogue tables): output staged for bulk stores
+  if (p.y_staged && p.aug_mode == LOWRANK_ALL_ON_TC && rt == 4)
+    return mode == MODE_GATED ? launch_two<TO, 4, MODE_GATED, true>(ctx, tm, p)
+                              : launch_two<TO, 4, MODE_PAIR, true>(ctx, tm, p);
   if (mode == MODE_GATED) {
     switch (rt) {
       case 4: return launch_two<TO, 4, MODE_GATED>(ctx, tm, p);

@@ -10,7 +10,7 @@ static int launch_one(Ctx* ctx, const CUtensorMap& a, const Params& p) {
   ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
   const int grid = p.num_tiles < ctx->sm_count ? p.num_tiles : ctx->sm_count;
   TmaSet tm;
-  tm.a = tm.b = tm.b2 = tm.aa = tm.ba = tm.ba2 = a;   // only X comes by TMA
+  tm.a = tm.b = tm.b2 = tm.aa = tm.ba = tm.ba2 = tm.y = tm.y16 = a;   // only X comes by TMA
   ZOACT_CUDA_TRY(launch_pdl(ctx, kern, dim3(grid), dim3(num_threads(true)), SMEM_BYTES, tm, p));
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();

@@ -20,20 +20,19 @@
 namespace zoact {
 namespace pairtc {
 
-constexpr int STAGES2 = 6;        // ring depth beside the epilogue tables
-constexpr int STAGES2_NOTBL = 7;  // ring depth when the whole low-rank term is on the MMA (no tables)
+constexpr int STAGES2 = 6;
 constexpr int B_HALF_BYTES = (BN / 2) * BK * 2;
 constexpr int STAGE2_BYTES = A_BYTES + B_HALF_BYTES;
-// Dynamic shared memory of a launch with ring depth nst: the table region exists only at the default depth.
-constexpr int smem2_bytes(int nst) {
-  return 1024 + nst * STAGE2_BYTES + (nst == STAGES2 ? TBL_FLOATS * 4 : 0) + 256;
-}
-constexpr int SMEM2_BYTES = smem2_bytes(STAGES2);
+constexpr int SMEM2_BYTES = 1024 + STAGES2 * STAGE2_BYTES + TBL_FLOATS * 4 + 256;
 constexpr int BM2 = 2 * BM;
+// Staged output (whole low-rank term on the MMA: no tables): each epilogue
+// warpgroup owns one 16 KB buffer in the table region for 128 rows x 128 bytes.
+constexpr int STG_BYTES = 16384;
+static_assert(2 * STG_BYTES <= TBL_FLOATS * 4, "staging buffers exceed the table region");
 
 struct SharedState2 {
-  uint64_t full[STAGES2_NOTBL];
-  uint64_t empty[STAGES2_NOTBL];
+  uint64_t full[STAGES2];
+  uint64_t empty[STAGES2];
   uint64_t tmem_full[2];
   uint64_t tmem_empty[2];
   uint64_t drain;
@@ -42,8 +41,7 @@ struct SharedState2 {
   int epi_ok;
 };
 static_assert(sizeof(SharedState2) <= 256, "barrier block outgrew its shared-memory slot");
-static_assert(SMEM2_BYTES <= 232448 && smem2_bytes(STAGES2_NOTBL) <= 232448,
-              "dynamic shared memory above the 227 KB a CTA may use");
+static_assert(SMEM2_BYTES <= 232448, "dynamic shared memory above the 227 KB a CTA may use");
 
 namespace tc2 {
 
@@ -114,25 +112,128 @@ __device__ __forceinline__ void commit2_own(uint32_t bar) {
 
 }  // namespace tc2
 
-// NST: ring depth.  At STAGES2_NOTBL the epilogue-table region holds a seventh
-// stage instead, and the kernel serves only launches whose whole low-rank term
-// is on the MMA (aug_mode LOWRANK_ALL_ON_TC; any other launch records
+// Byte offset of 16-byte granule g of row r in a 128-byte-swizzled staging box
+// (the layout a SWIZZLE_128B tensor map reads: granule index XOR row mod 8).
+__device__ __forceinline__ uint32_t sw128_off(int r, int g) {
+  return (uint32_t)(r * 128 + ((g ^ (r & 7)) << 4));
+}
+
+template <typename TO>
+__device__ __forceinline__ uint4 pack8_16(const float* v) {
+  return make_uint4(pack2(v[0], v[1], (TO*)nullptr), pack2(v[2], v[3], (TO*)nullptr), pack2(v[4], v[5], (TO*)nullptr),
+                    pack2(v[6], v[7], (TO*)nullptr));
+}
+
+// Write PW values of staging row rl, starting at column p of the chunk, as
+// 16-byte granules: 128-byte swizzled rows (full chunks) or unswizzled rows of
+// 16 columns (narrow chunks).
+template <typename TO, int PW>
+__device__ __forceinline__ void stage_granules(uint32_t sbuf, int rl, int p, const float* v, bool full) {
+  constexpr int EB = (int)sizeof(TO);
+  constexpr int GE = 16 / EB;       // values per granule
+#pragma unroll
+  for (int q = 0; q < PW / GE; ++q) {
+    const int gi = p / GE + q;
+    const uint32_t off = full ? sw128_off(rl, gi) : (uint32_t)(rl * 16 * EB + gi * 16);
+    if constexpr (EB == 2)
+      tc::st_shared_v4(sbuf + off, pack8_16<TO>(v + 8 * q));
+    else
+      tc::st_shared_v4(sbuf + off, make_uint4(__float_as_uint(v[4 * q]), __float_as_uint(v[4 * q + 1]),
+                                              __float_as_uint(v[4 * q + 2]), __float_as_uint(v[4 * q + 3])));
+  }
+}
+
+// Epilogue of one accumulator tile whose whole low-rank term is in the
+// accumulator, written through shared memory: this warpgroup's columns go in
+// chunks of 128 bytes per row (then 16-column chunks for the remainder) into
+// its staging buffer, and one thread stores each chunk with a bulk tensor store
+// of 128 rows (rows and columns outside Y are dropped by the store).  Returns
+// false when the accumulator wait gave up.  `pending`: the issuing thread has
+// bulk stores in flight.
+template <typename TO, int MODE>
+__device__ __forceinline__ bool epi_all_staged(const Params& prm, const TmaSet& tm, SharedState2* ss, uint8_t* stg,
+                                               int etid, int half, int rl, int64_t row0, int n_blk, int bn, int buf,
+                                               uint32_t acc_phase, uint32_t t_row, volatile int* abort_flag,
+                                               bool& pending) {
+  constexpr bool GATED = MODE == MODE_GATED;
+  constexpr int EB = (int)sizeof(TO);
+  constexpr int CC = 128 / EB;      // columns of a full chunk (one swizzled 128-byte row each)
+  constexpr int NC = 16;            // columns of a narrow chunk (unswizzled rows of 16 * EB bytes)
+  if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
+  const int ncol_tile = GATED ? BN / 2 : bn;
+  const int wcols = ncol_tile / 2;  // this warpgroup's columns, a multiple of 16
+  const int cb = half * wcols;
+  const bool issuer = (etid & 127) == 0;
+  const uint32_t sbuf = tc::smem_u32(stg + half * STG_BYTES);
+  for (int c = 0; c < wcols;) {
+    const int n = n_blk * ncol_tile + cb + c;
+    if (n >= prm.d_out) break;                      // uniform over the warpgroup
+    const bool full = wcols - c >= CC;
+    const int cw = full ? CC : NC;
+    if (issuer && pending) tc::bulk_wait_read0();   // the buffer's previous store has read it
+    tc::named_bar_sync(4 + half, 128);
+    if (full) {
+      // 32 columns per TMEM load: few tcgen05.ld / wait pairs beside the MMAs
+#pragma unroll 1
+      for (int p = 0; p < CC; p += 32) {
+        float v[32];
+        if (GATED) {
+          float u[32];
+          tc::tmem_ld32(t_row + (uint32_t)(cb + c + p), v);
+          tc::tmem_ld32(t_row + (uint32_t)(BN / 2 + cb + c + p), u);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = silu_fast(v[i]) * u[i];
+        } else {
+          tc::tmem_ld32(t_row + (uint32_t)(cb + c + p), v);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = apply_act(v[i], prm.act);
+        }
+        stage_granules<TO, 32>(sbuf, rl, p, v, true);
+      }
+    } else {
+      float v[16];
+      if (GATED) {
+        float u[16];
+        tc::tmem_ld16(t_row + (uint32_t)(cb + c), v);
+        tc::tmem_ld16(t_row + (uint32_t)(BN / 2 + cb + c), u);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = silu_fast(v[i]) * u[i];
+      } else {
+        tc::tmem_ld16(t_row + (uint32_t)(cb + c), v);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = apply_act(v[i], prm.act);
+      }
+      stage_granules<TO, 16>(sbuf, rl, 0, v, false);
+    }
+    tc::fence_proxy_async_smem();                   // the staging writes, before the bulk store reads them
+    tc::named_bar_sync(4 + half, 128);
+    if (issuer) {
+      tc::tma_store_2d(full ? &tm.y : &tm.y16, n, (int)row0, sbuf);
+      tc::bulk_commit();
+      pending = true;
+    }
+    c += cw;
+  }
+  return true;
+}
+
+// STAGED: the launch has the whole low-rank term on the MMA (aug_mode
+// LOWRANK_ALL_ON_TC) and Y's store maps in tm.y / tm.y16; the table region then
+// holds the output staging buffers (any other launch records
 // ZOACT_ERR_INVALID_ARG and exits before touching shared memory).
-template <typename TO, int RT, int MODE, int AB_BF16, int NST = STAGES2>
+template <typename TO, int RT, int MODE, int AB_BF16, bool STAGED = false>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(num_threads(false), 1)
 pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
   constexpr int CW = MODE == MODE_GATED ? 8 : 16;   // epilogue chunk width (gated: two accumulators)
-  constexpr bool NOTBL = NST != STAGES2;
-  static_assert(NST == STAGES2 || NST == STAGES2_NOTBL, "ring depth");
-  if (NOTBL && prm.aug_mode != LOWRANK_ALL_ON_TC) {   // uniform over the grid: both CTAs of a pair leave
+  if (STAGED && (prm.aug_mode != LOWRANK_ALL_ON_TC || !prm.y_staged)) {   // uniform: both CTAs of a pair leave
     pdl_wait();
     if (threadIdx.x == 0 && blockIdx.x == 0) record_error(prm.status, ZOACT_ERR_INVALID_ARG);
     return;
   }
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-  float* tbl = reinterpret_cast<float*>(smem + NST * STAGE2_BYTES);
-  SharedState2* ss = reinterpret_cast<SharedState2*>(tbl + (NOTBL ? 0 : TBL_FLOATS));
+  float* tbl = reinterpret_cast<float*>(smem + STAGES2 * STAGE2_BYTES);
+  SharedState2* ss = reinterpret_cast<SharedState2*>(tbl + TBL_FLOATS);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -141,7 +242,7 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
   volatile int* abort_flag = &ss->abort_flag;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < NST; ++s) {
+    for (int s = 0; s < STAGES2; ++s) {
       tc::mbar_init(tc::smem_u32(&ss->full[s]), 2);     // one producer arrival from each CTA (leader's copy is used)
       tc::mbar_init(tc::smem_u32(&ss->empty[s]), 1);
     }
@@ -204,7 +305,7 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
                                   yb + n_blk * (BN / 2), full_leader);
           else
             tc2::tma_load_2d_pair(sb, aug ? &tm.ba : &tm.b, kxb, yb + n_blk * bn + (int)rank * bh, full_leader);
-          if (++stage == NST) { stage = 0; phase ^= 1u; }
+          if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
         }
       }
       if (!ok) {
@@ -242,7 +343,7 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
                           (kb | k) != 0 ? 1u : 0u);
           tc2::commit2_both(tc::smem_u32(&ss->empty[stage]));    // frees the stage in both CTAs
           issued_any = true;
-          if (++stage == NST) { stage = 0; phase ^= 1u; }
+          if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
         tc2::commit2_both(tc::smem_u32(&ss->tmem_full[buf]));   // accumulator ready in both CTAs
@@ -261,23 +362,29 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
     const uint32_t tmem_empty_leader0 = tc2::map_to(tc::smem_u32(&ss->tmem_empty[0]), 0);
     const uint32_t tmem_empty_leader1 = tc2::map_to(tc::smem_u32(&ss->tmem_empty[1]), 0);
     int local = 0;
+    bool pending = false;                   // staged output: this thread has bulk stores in flight
     for (int tile = cluster_id; tile < prm.num_tiles; tile += n_clusters, ++local) {
       int m_blk, n_blk;
       tile_coords(tile, num_m, num_n, m_blk, n_blk);
       const int buf = local & 1;
       const uint32_t acc_phase = (local >> 1) & 1;
-      const int64_t m = (int64_t)m_blk * BM2 + (int64_t)rank * BM + row_in_tile;
+      const int64_t row0 = (int64_t)m_blk * BM2 + (int64_t)rank * BM;
+      const int64_t m = row0 + row_in_tile;
       const bool row_ok = m < prm.rows;
       const uint32_t t_row = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * BN);
-      const bool ok = epi_pair_tile<TO, RT, MODE, CW, NOTBL>(prm, ss, tbl, etid, half,
-                                                      (int64_t)m_blk * BM2 + (int64_t)rank * BM, m, row_ok,
-                                                      n_blk, bn, buf,
-                                                      acc_phase, t_row, abort_flag);
+      bool ok;
+      if constexpr (STAGED)
+        ok = epi_all_staged<TO, MODE>(prm, tm, ss, reinterpret_cast<uint8_t*>(tbl), etid, half, row_in_tile, row0,
+                                      n_blk, bn, buf, acc_phase, t_row, abort_flag, pending);
+      else
+        ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, tbl, etid, half, row0, m, row_ok, n_blk, bn, buf, acc_phase,
+                                             t_row, abort_flag);
       if (!ok) break;
       tc::tc_fence_before();
       tc::named_bar_sync(3, EPI_THREADS);        // every epilogue thread of this CTA has read the tile
       if (etid == 0) tc2::arrive_cluster(buf ? tmem_empty_leader1 : tmem_empty_leader0);
     }
+    if (pending) tc::bulk_wait0();           // the stores have read the staging buffers and completed
   }
 
   tc::tc_fence_before();

@@ -89,6 +89,7 @@ enum Mode { MODE_PAIR = 0, MODE_GATED = 1, MODE_PLAIN = 2 };
 // A_aug, B_aug, B_aug up (unused ones are copies of a valid map).
 struct TmaSet {
   CUtensorMap a, b, b2, aa, ba, ba2;
+  CUtensorMap y, y16;   // output Y for staged bulk stores: 128-byte swizzled rows, and 16-column boxes
 };
 
 struct Params {
@@ -109,6 +110,7 @@ struct Params {
   uint32_t layer_id, layer_id2;
   int num_m, num_n, num_k, num_tiles;
   int aug_mode;      // LowrankMode
+  int y_staged;      // tm.y / tm.y16 hold Y's store maps (CTA-pair kernel, whole term on the MMA)
   int aug_kb;        // extra K-blocks per tile from A_aug / B_aug (0 with LOWRANK_EPILOGUE)
   int aug_kb_slot;   // K-blocks of one slot (B_aug row width / 64)
   int aug_slots;     // LOWRANK_ALL_ON_TC: 1, or S when a tile spans up to S evaluation blocks (slot = block mod S)
@@ -435,8 +437,7 @@ __device__ __forceinline__ void load_p(float* p, const float* __restrict__ P, in
 // over the two signs of one query (coefficients +c, -c) builds one Z table and
 // forms acc +- c Z p.  With the whole term on the tensor cores it only converts
 // and stores.  Returns false when the wait gave up.
-// ALL_ONLY: the launch has the whole low-rank term on the MMA (no tables exist).
-template <typename TO, int RT, int MODE, int CW, bool ALL_ONLY = false, typename SS>
+template <typename TO, int RT, int MODE, int CW, typename SS>
 __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* tbl, int etid, int half,
                                               int64_t row0, int64_t m, bool row_ok, int n_blk, int bn, int buf,
                                               uint32_t acc_phase, uint32_t t_row, volatile int* abort_flag) {
@@ -449,7 +450,7 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
   const int64_t T = prm.T;
   TO* Y = static_cast<TO*>(prm.Y);
   const int ncol_tile = GATED ? BN / 2 : bn;               // output columns of this tile
-  if (ALL_ONLY || prm.aug_mode == LOWRANK_ALL_ON_TC) {
+  if (prm.aug_mode == LOWRANK_ALL_ON_TC) {
     // stacked rows, the whole low-rank term in the accumulator
     if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
     const int cbeg = half * (ncol_tile / 2);
@@ -474,9 +475,6 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
     }
     return true;
   }
-  if constexpr (ALL_ONLY) {
-    return true;
-  } else {
   const bool c_in_acc = prm.aug_mode == LOWRANK_C_ON_TC;
   float p[RT], p2[RT];
   const bool vec = prm.vec_ok != 0;
@@ -626,7 +624,6 @@ __device__ __forceinline__ bool epi_pair_tile(const Params& prm, SS* ss, float* 
     }
   }
   return true;
-  }  // !ALL_ONLY
 }
 
 template <typename TO, int RT, int MODE, int AB_BF16, bool W4>

@@ -151,6 +151,21 @@ def test_nonfinite_outputs_are_flagged(ctx):
     assert ctx.device_status() == 0               # read and reset
 
 
+def test_basis_init_nonfinite_calibration_is_flagged(ctx):
+    # one NaN in the calibration activations makes G, and so every basis column, non-finite: the
+    # sign fix finds no finite entry to orient a column by and the status word says so
+    X = normal((300, 256), 31, DEV)
+    X[7, 11] = float("nan")
+    U = torch.empty(256, 8, device=DEV)
+    zo.zoact_basis_init(ctx, X, 8, U)
+    torch.cuda.synchronize()
+    assert ctx.device_status() == -4
+    X[7, 11] = 0.0
+    zo.zoact_basis_init(ctx, X, 8, U)            # the context stays usable
+    torch.cuda.synchronize()
+    assert ctx.device_status() == 0 and torch.isfinite(U).all()
+
+
 def test_maximum_size_sampled(ctx):
     # 65536 tokens per perturbation through a 4096 -> 4096 layer (131072 stacked rows, 1 GiB per side):
     # every M tile of the CTA-pair kernel, sampled rows against the oracle
