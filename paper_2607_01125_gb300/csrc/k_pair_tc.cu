@@ -261,16 +261,25 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   p.num_tiles = p.num_m * p.num_n;
   p.ldy = a.d_out;
   p.aug_mode = lmode;
-  // CTA pairs with the whole term on the MMA write Y through staged bulk stores
+  // CTA pairs write Y through staged bulk stores when the whole term is on the MMA, and for the two signs
+  // of one query on a shared input with 16-bit outputs (one store map per sign: rows [0, T) and [T, 2T))
   tm.y = tm.y16 = tm.a;
-  p.y_staged = 0;
+  p.y_staged = STAGE_NONE;
+  const int es = (int)dtype_size(a.ydtype);
   if (two && lmode == LOWRANK_ALL_ON_TC && rt == 4) {
-    const int es = (int)dtype_size(a.ydtype);
     st = encode_tmap_store(&tm.y, a.Y, a.ydtype, a.rows, a.d_out, 128 / es, BM, true);
     if (st) return st;
     st = encode_tmap_store(&tm.y16, a.Y, a.ydtype, a.rows, a.d_out, 16, BM, false);
     if (st) return st;
-    p.y_staged = 1;
+    p.y_staged = STAGE_ALL;
+  } else if (two && lmode == LOWRANK_C_ON_TC && a.shared && a.nb == 2 && es == 2 && a.qry[0] == a.qry[1] &&
+             a.coef[1] == -a.coef[0] && a.coef[0] != 0.f) {
+    uint8_t* y0 = static_cast<uint8_t*>(a.Y);
+    st = encode_tmap_store(&tm.y, y0, a.ydtype, a.T, a.d_out, 16, BM, false);
+    if (st) return st;
+    st = encode_tmap_store(&tm.y16, y0 + (size_t)a.T * a.d_out * es, a.ydtype, a.T, a.d_out, 16, BM, false);
+    if (st) return st;
+    p.y_staged = STAGE_MIRROR;
   }
   p.aug_kb = lmode == LOWRANK_EPILOGUE ? 0 : slots * ka_tot / BK;
   p.aug_kb_slot = ka_tot / BK;

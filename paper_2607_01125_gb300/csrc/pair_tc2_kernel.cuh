@@ -29,6 +29,14 @@ constexpr int BM2 = 2 * BM;
 // warpgroup owns one 16 KB buffer in the table region for 128 rows x 128 bytes.
 constexpr int STG_BYTES = 16384;
 static_assert(2 * STG_BYTES <= TBL_FLOATS * 4, "staging buffers exceed the table region");
+// Staged output of the two signs on a shared input: the Z tables (gate, up) fill the
+// region's first MIRROR_STG_OFF bytes and each warpgroup stages 16 columns of both
+// signs (2 x 128 rows x 32 bytes) above them.
+constexpr int MIRROR_STG_OFF = 17408;
+constexpr int MIRROR_STG_BYTES = 8192;
+static_assert(MIRROR_STG_OFF % 1024 == 0 && MIRROR_STG_OFF + 2 * MIRROR_STG_BYTES <= TBL_FLOATS * 4,
+              "mirror staging buffers exceed the table region");
+
 
 struct SharedState2 {
   uint64_t full[STAGES2];
@@ -217,15 +225,111 @@ __device__ __forceinline__ bool epi_all_staged(const Params& prm, const TmaSet& 
   return true;
 }
 
-// STAGED: the launch has the whole low-rank term on the MMA (aug_mode
-// LOWRANK_ALL_ON_TC) and Y's store maps in tm.y / tm.y16; the table region then
-// holds the output staging buffers (any other launch records
-// ZOACT_ERR_INVALID_ARG and exits before touching shared memory).
-template <typename TO, int RT, int MODE, int AB_BF16, bool STAGED = false>
+// Epilogue of the two signs of one query on a shared input (C p in the
+// accumulator, c_1 = -c_0, 16-bit outputs), staged: per column pass the Z
+// tables of gate (and up) are built at tbl (and tbl + TSZ), then each warpgroup
+// forms acc +- c_0 Z p for 16 columns of its 128 rows, writes both signs into
+// its staging buffer and one thread stores them with bulk tensor stores through
+// tm.y (rows [0, T) of Y) and tm.y16 (rows [T, 2T)), which drop rows past T and
+// columns past d_out.  Returns false when the accumulator wait gave up.
+template <typename TO, int RT, int MODE>
+__device__ __forceinline__ bool epi_mirror_staged(const Params& prm, const TmaSet& tm, SharedState2* ss, float* tbl,
+                                                  int etid, int half, int rl, int64_t row0, int64_t m, bool row_ok,
+                                                  int n_blk, int bn, int buf, uint32_t acc_phase, uint32_t t_row,
+                                                  volatile int* abort_flag, bool& pending) {
+  constexpr bool GATED = MODE == MODE_GATED;
+  constexpr int SLOTS = GATED ? gated_slots(RT) : pair_slots(RT);
+  constexpr int STRIDE = SLOTS + TPAD;
+  constexpr int TSZ = RT * STRIDE;
+  static_assert((GATED ? 2 : 1) * TSZ * 4 <= MIRROR_STG_OFF, "mirror tables overlap the staging buffers");
+  static_assert(sizeof(TO) == 2, "staged mirror output is 16-bit");
+  const int r = prm.r;
+  float p[RT], p2[RT];
+  const bool vec = prm.vec_ok != 0;
+  load_p<RT>(p, prm.P, m, r, row_ok, vec);
+  if (GATED) load_p<RT>(p2, prm.P2, m, r, row_ok, vec);
+  const int ncol_tile = GATED ? BN / 2 : bn;
+  const float cz = prm.coef[0];
+  const int zq = prm.zq[0];
+  const bool issuer = (etid & 127) == 0;
+  const uint32_t sp = tc::smem_u32(tbl) + MIRROR_STG_OFF + half * MIRROR_STG_BYTES;   // + sign; - sign at +4096
+  bool waited = false;
+  for (int s0 = 0; s0 < ncol_tile; s0 += SLOTS) {
+    const int cwid = min(SLOTS, ncol_tile - s0);            // a multiple of 32
+    const int col0 = n_blk * ncol_tile + s0;
+    tc::named_bar_sync(1, EPI_THREADS);                     // previous pass's readers are done
+    build_tables_z<RT>(tbl, nullptr, STRIDE, prm.Zt + zq * prm.zt_qstride, prm.Zt + zq * prm.zt_qstride, 1.f, 0.f,
+                       col0, cwid, prm.d_out, r, etid);
+    if (GATED)
+      build_tables_z<RT>(tbl + TSZ, nullptr, STRIDE, prm.Zt2 + zq * prm.zt_qstride, prm.Zt2 + zq * prm.zt_qstride,
+                         1.f, 0.f, col0, cwid, prm.d_out, r, etid);
+    tc::named_bar_sync(1, EPI_THREADS);
+    if (!waited) {
+      if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
+      waited = true;
+    }
+    const int cbeg = s0 + half * (cwid / 2);
+    for (int c0 = cbeg; c0 < cbeg + cwid / 2; c0 += 16) {
+      const int n = n_blk * ncol_tile + c0;
+      if (n >= prm.d_out) break;                            // uniform over the warpgroup
+      if (issuer && pending) tc::bulk_wait_read0();         // the buffers' previous stores have read them
+      tc::named_bar_sync(4 + half, 128);
+#pragma unroll
+      for (int k8 = 0; k8 < 16; k8 += 8) {
+        float hp[8], hm[8];
+        if (GATED) {
+          float g[8], u[8], sg[8], su[8];
+          tc::tmem_ld8(t_row + (uint32_t)(c0 + k8), g);
+          tc::tmem_ld8(t_row + (uint32_t)(BN / 2 + c0 + k8), u);
+          lowrank_t<RT, 8>(tbl, STRIDE, c0 + k8 - s0, p, sg);
+          lowrank_t<RT, 8>(tbl + TSZ, STRIDE, c0 + k8 - s0, p2, su);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            hp[i] = silu_fast(fmaf(cz, sg[i], g[i])) * fmaf(cz, su[i], u[i]);
+            hm[i] = silu_fast(fmaf(-cz, sg[i], g[i])) * fmaf(-cz, su[i], u[i]);
+          }
+        } else {
+          float a[8], sl[8];
+          tc::tmem_ld8(t_row + (uint32_t)(c0 + k8), a);
+          lowrank_t<RT, 8>(tbl, STRIDE, c0 + k8 - s0, p, sl);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            hp[i] = apply_act(fmaf(cz, sl[i], a[i]), prm.act);
+            hm[i] = apply_act(fmaf(-cz, sl[i], a[i]), prm.act);
+          }
+        }
+        tc::st_shared_v4(sp + (uint32_t)(rl * 32 + (k8 >> 3) * 16), pack8_16<TO>(hp));
+        tc::st_shared_v4(sp + 4096u + (uint32_t)(rl * 32 + (k8 >> 3) * 16), pack8_16<TO>(hm));
+      }
+      tc::fence_proxy_async_smem();
+      tc::named_bar_sync(4 + half, 128);
+      if (issuer) {
+        tc::tma_store_2d(&tm.y, n, (int)row0, sp);
+        tc::tma_store_2d(&tm.y16, n, (int)row0, sp + 4096u);
+        tc::bulk_commit();
+        pending = true;
+      }
+    }
+  }
+  return true;
+}
+
+// SMODE (StageMode): STAGE_ALL -- the launch has the whole low-rank term on the
+// MMA (aug_mode LOWRANK_ALL_ON_TC) and Y's store maps in tm.y / tm.y16, the
+// table region holds the output staging buffers; STAGE_MIRROR -- the two signs
+// of one query on a shared input (aug_mode LOWRANK_C_ON_TC, two blocks), the
+// region holds the Z tables and two smaller buffers.  A launch that does not
+// match its SMODE records ZOACT_ERR_INVALID_ARG and exits before touching
+// shared memory.
+template <typename TO, int RT, int MODE, int AB_BF16, int SMODE = STAGE_NONE>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(num_threads(false), 1)
 pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
   constexpr int CW = MODE == MODE_GATED ? 8 : 16;   // epilogue chunk width (gated: two accumulators)
-  if (STAGED && (prm.aug_mode != LOWRANK_ALL_ON_TC || !prm.y_staged)) {   // uniform: both CTAs of a pair leave
+  const bool mismatch =
+      (SMODE == STAGE_ALL && (prm.aug_mode != LOWRANK_ALL_ON_TC || prm.y_staged != STAGE_ALL)) ||
+      (SMODE == STAGE_MIRROR && (prm.aug_mode != LOWRANK_C_ON_TC || prm.y_staged != STAGE_MIRROR || !prm.shared ||
+                                 prm.nb != 2));
+  if (mismatch) {                                   // uniform: both CTAs of a pair leave
     pdl_wait();
     if (threadIdx.x == 0 && blockIdx.x == 0) record_error(prm.status, ZOACT_ERR_INVALID_ARG);
     return;
@@ -373,9 +477,12 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       const bool row_ok = m < prm.rows;
       const uint32_t t_row = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * BN);
       bool ok;
-      if constexpr (STAGED)
+      if constexpr (SMODE == STAGE_ALL)
         ok = epi_all_staged<TO, MODE>(prm, tm, ss, reinterpret_cast<uint8_t*>(tbl), etid, half, row_in_tile, row0,
                                       n_blk, bn, buf, acc_phase, t_row, abort_flag, pending);
+      else if constexpr (SMODE == STAGE_MIRROR)
+        ok = epi_mirror_staged<TO, RT, MODE>(prm, tm, ss, tbl, etid, half, row_in_tile, row0, m, row_ok, n_blk, bn,
+                                             buf, acc_phase, t_row, abort_flag, pending);
       else
         ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, tbl, etid, half, row0, m, row_ok, n_blk, bn, buf, acc_phase,
                                              t_row, abort_flag);

@@ -87,6 +87,10 @@ enum Mode { MODE_PAIR = 0, MODE_GATED = 1, MODE_PLAIN = 2 };
 
 // Tensor maps of one launch: X, W (gate), W up, and the low-rank K columns
 // A_aug, B_aug, B_aug up (unused ones are copies of a valid map).
+// Output staging of a CTA-pair launch (Params::y_staged, the kernel's SMODE): none, the whole
+// low-rank term on the MMA, or the two signs of one query on a shared input.
+enum StageMode { STAGE_NONE = 0, STAGE_ALL = 1, STAGE_MIRROR = 2 };
+
 struct TmaSet {
   CUtensorMap a, b, b2, aa, ba, ba2;
   CUtensorMap y, y16;   // output Y for staged bulk stores: 128-byte swizzled rows, and 16-column boxes
@@ -110,7 +114,7 @@ struct Params {
   uint32_t layer_id, layer_id2;
   int num_m, num_n, num_k, num_tiles;
   int aug_mode;      // LowrankMode
-  int y_staged;      // tm.y / tm.y16 hold Y's store maps (CTA-pair kernel, whole term on the MMA)
+  int y_staged;      // StageMode: tm.y / tm.y16 hold Y's store maps for the CTA-pair kernel's staged epilogue
   int aug_kb;        // extra K-blocks per tile from A_aug / B_aug (0 with LOWRANK_EPILOGUE)
   int aug_kb_slot;   // K-blocks of one slot (B_aug row width / 64)
   int aug_slots;     // LOWRANK_ALL_ON_TC: 1, or S when a tile spans up to S evaluation blocks (slot = block mod S)

@@ -465,3 +465,35 @@ def test_kernel_timing(ctx):
     assert n == 3 and ms > 0.0
     zo.zoact_pair_forward(ctx, L, X, T, False, 1e-3, 1, 0, Y)
     assert ctx.kernel_time() == (0.0, 0)
+
+
+@pytest.mark.parametrize("gated", [False, True])
+@pytest.mark.parametrize("T,d_out,r,dt", [(300, 264, 16, torch.bfloat16), (640, 392, 32, torch.float16),
+                                          (257, 136, 4, torch.bfloat16), (512, 520, 8, torch.bfloat16)])
+def test_shared_pair_16bit_staged(ctx, gated, T, d_out, r, dt):
+    # the two signs on a shared input with 16-bit outputs (CTA pairs): both signs go through shared-memory
+    # staging and bulk stores -- rows past T (a partial second M tile) and columns past d_out (a partial last
+    # 16-column chunk) must be dropped, the other sign's rows untouched
+    d_in, eps, seed, query = 512, 0.5, 23, 7
+    X, W, U, C = _pair_case(d_in, d_out, r, T, True, dt, eps, 0.3, seed=90)
+    Y = torch.full((2 * T + 8, d_out), 7.0, dtype=dt, device=DEV)         # 8 guard rows after the output
+    Yv = Y[:2 * T]
+    if gated:
+        W2 = normal((d_out, d_in), 95, DEV, std=d_in ** -0.5, dtype=dt)
+        U2 = normal((d_in, r), 96, DEV) / np.sqrt(d_in)
+        C2 = normal((d_out * r,), 97, DEV, std=0.3)
+        zo.zoact_pair_forward_gated(ctx, zo.make_layer(W, U, C, 3), zo.make_layer(W2, U2, C2, 4), X, T, True,
+                                    eps, seed, query, Yv)
+        torch.cuda.synchronize()
+        g, _, _ = _oracle_pair(X, W, U, C, eps, T, True, seed, 3, query, d_out, r)
+        u, _, _ = _oracle_pair(X, W2, U2, C2, eps, T, True, seed, 4, query, d_out, r)
+        ref = layers.silu(g) * u
+    else:
+        zo.zoact_pair_forward(ctx, zo.make_layer(W, U, C, 3), X, T, True, eps, seed, query, Yv)
+        torch.cuda.synchronize()
+        ref, _, _ = _oracle_pair(X, W, U, C, eps, T, True, seed, 3, query, d_out, r)
+    assert ctx.device_status() == 0
+    rel = {torch.bfloat16: 2.0 ** -8, torch.float16: 2.0 ** -11}[dt]
+    err = np.abs(np64(Yv) - ref)
+    assert np.all(err <= rel * np.abs(ref) + 2e-3 * np.abs(ref).max()), err.max()
+    assert torch.all(Y[2 * T:] == 7.0)                                   # nothing written past the output
