@@ -279,7 +279,8 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     if (st) return st;
     st = encode_tmap_store(&tm.y16, y0 + (size_t)a.T * a.d_out * es, a.ydtype, a.T, a.d_out, 16, BM, false);
     if (st) return st;
-    p.y_staged = STAGE_MIRROR;
+    // four rows per thread where the projections fit in registers (rank tile <= 16, one P for gate and up)
+    p.y_staged = (rt <= 16 && (!gated || a.P2 == a.P)) ? STAGE_MIRROR4 : STAGE_MIRROR;
   }
   p.aug_kb = lmode == LOWRANK_EPILOGUE ? 0 : slots * ka_tot / BK;
   p.aug_kb_slot = ka_tot / BK;

@@ -314,6 +314,142 @@ __device__ __forceinline__ bool epi_mirror_staged(const Params& prm, const TmaSe
   return true;
 }
 
+// Column order of a 16-column table chunk for four-row epilogue threads: thread t
+// (q = t % 4) uses chunk columns 2q, 2q+1, 8+2q, 9+2q, stored contiguously at 4q.
+__device__ __forceinline__ int perm16(int c) { return 4 * ((c & 7) >> 1) + ((c >> 3) << 1) + (c & 1); }
+
+// Z table of one query over columns [col0, col0 + ncols) in 16-column chunks
+// permuted by perm16: tb[j * stride + (s & ~15) + perm16(s & 15)] = Z[j][col0 + s],
+// zero where col0 + s >= d_out or j >= r.  One thread per 4 consecutive columns.
+template <int RT>
+__device__ __forceinline__ void build_tables_z16(float* tb, int stride, const float* __restrict__ Zq, int col0,
+                                                 int ncols, int d_out, int r, int tid) {
+  const int per_row = ncols / 4;
+  for (int it = tid; it < RT * per_row; it += EPI_THREADS) {
+    const int j = it / per_row, s = 4 * (it - j * per_row);
+    const int col = col0 + s;
+    float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (j < r && col < d_out) z = *reinterpret_cast<const float4*>(Zq + (int64_t)j * d_out + col);
+    float* row = tb + j * stride + (s & ~15);
+    const int c = s & 15;                       // columns c, c+1 and c+2, c+3 land as two pairs
+    *reinterpret_cast<float2*>(row + perm16(c)) = make_float2(z.x, z.y);
+    *reinterpret_cast<float2*>(row + perm16(c + 2)) = make_float2(z.z, z.w);
+  }
+}
+
+// The staged two-sign epilogue with four rows per thread (rank tile <= 16; a gated
+// launch whose gate and up share one projection P).  TMEM is read with 16x256b
+// loads, so each thread holds rows t/4 + 8k (k = 0..3) of its warp's 32 and four
+// columns of each 16-column chunk; one 16-byte shared read of the permuted Z table
+// then feeds 16 FMAs (4 rows x 4 columns) instead of 4, a quarter of the table
+// reads of the row-per-thread form.  Outputs are staged as in epi_mirror_staged.
+template <typename TO, int RT, int MODE>
+__device__ __forceinline__ bool epi_mirror4_staged(const Params& prm, const TmaSet& tm, SharedState2* ss, float* tbl,
+                                                   int etid, int half, int quad, int lane, int64_t row0, int n_blk,
+                                                   int bn, int buf, uint32_t acc_phase, uint32_t t_q,
+                                                   volatile int* abort_flag, bool& pending) {
+  constexpr bool GATED = MODE == MODE_GATED;
+  constexpr int SLOTS = GATED ? gated_slots(RT) : pair_slots(RT);
+  constexpr int STRIDE = SLOTS + TPAD;
+  constexpr int TSZ = RT * STRIDE;
+  static_assert(RT <= 16, "four rows of projections per thread");
+  static_assert((GATED ? 2 : 1) * TSZ * 4 <= MIRROR_STG_OFF, "mirror tables overlap the staging buffers");
+  static_assert(SLOTS % 32 == 0 && STRIDE % 4 == 0, "16-column chunks of 16-byte aligned table rows");
+  static_assert(sizeof(TO) == 2, "staged mirror output is 16-bit");
+  const int r = prm.r;
+  const int q = lane & 3, rq = lane >> 2;
+  const bool vec = prm.vec_ok != 0;
+  float p[4][RT];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int64_t m = row0 + quad * 32 + rq + 8 * k;
+    load_p<RT>(p[k], prm.P, m, r, m < prm.rows, vec);
+  }
+  const int ncol_tile = GATED ? BN / 2 : bn;
+  const float cz = prm.coef[0];
+  const int zq = prm.zq[0];
+  const bool issuer = (etid & 127) == 0;
+  const uint32_t sp = tc::smem_u32(tbl) + MIRROR_STG_OFF + half * MIRROR_STG_BYTES;   // + sign; - sign at +4096
+  bool waited = false;
+  for (int s0 = 0; s0 < ncol_tile; s0 += SLOTS) {
+    const int cwid = min(SLOTS, ncol_tile - s0);            // a multiple of 32
+    const int col0 = n_blk * ncol_tile + s0;
+    tc::named_bar_sync(1, EPI_THREADS);                     // previous pass's readers are done
+    build_tables_z16<RT>(tbl, STRIDE, prm.Zt + zq * prm.zt_qstride, col0, cwid, prm.d_out, r, etid);
+    if (GATED) build_tables_z16<RT>(tbl + TSZ, STRIDE, prm.Zt2 + zq * prm.zt_qstride, col0, cwid, prm.d_out, r, etid);
+    tc::named_bar_sync(1, EPI_THREADS);
+    if (!waited) {
+      if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
+      waited = true;
+    }
+    const int cbeg = s0 + half * (cwid / 2);
+    for (int c0 = cbeg; c0 < cbeg + cwid / 2; c0 += 16) {
+      const int n = n_blk * ncol_tile + c0;
+      if (n >= prm.d_out) break;                            // uniform over the warpgroup
+      float g[16], u[16];
+      tc::tmem_ld_rows4(t_q + (uint32_t)c0, g);
+      if (GATED) tc::tmem_ld_rows4(t_q + (uint32_t)(BN / 2 + c0), u);
+      float2 zg[4][2], zu[4][2];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        zg[k][0] = zg[k][1] = zu[k][0] = zu[k][1] = make_float2(0.f, 0.f);
+      }
+      const float* tg = tbl + (c0 - s0) + 4 * q;
+#pragma unroll
+      for (int j = 0; j < RT; ++j) {
+        const float4 a = *reinterpret_cast<const float4*>(tg + j * STRIDE);
+        float4 b = a;
+        if (GATED) b = *reinterpret_cast<const float4*>(tg + TSZ + j * STRIDE);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float2 pj = make_float2(p[k][j], p[k][j]);
+          zg[k][0] = ffma2(make_float2(a.x, a.y), pj, zg[k][0]);
+          zg[k][1] = ffma2(make_float2(a.z, a.w), pj, zg[k][1]);
+          if (GATED) {
+            zu[k][0] = ffma2(make_float2(b.x, b.y), pj, zu[k][0]);
+            zu[k][1] = ffma2(make_float2(b.z, b.w), pj, zu[k][1]);
+          }
+        }
+      }
+      if (issuer && pending) tc::bulk_wait_read0();         // the buffers' previous stores have read them
+      tc::named_bar_sync(4 + half, 128);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float zgk[4] = {zg[k][0].x, zg[k][0].y, zg[k][1].x, zg[k][1].y};
+        const float zuk[4] = {zu[k][0].x, zu[k][0].y, zu[k][1].x, zu[k][1].y};
+        float hp[4], hm[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float gv = g[4 * k + i];
+          if (GATED) {
+            const float uv = u[4 * k + i];
+            hp[i] = silu_fast(fmaf(cz, zgk[i], gv)) * fmaf(cz, zuk[i], uv);
+            hm[i] = silu_fast(fmaf(-cz, zgk[i], gv)) * fmaf(-cz, zuk[i], uv);
+          } else {
+            hp[i] = apply_act(fmaf(cz, zgk[i], gv), prm.act);
+            hm[i] = apply_act(fmaf(-cz, zgk[i], gv), prm.act);
+          }
+        }
+        // row quad*32 + rq + 8k of the staging rows (32 bytes each): columns 2q, 2q+1 and 8+2q, 9+2q
+        const uint32_t ro = (uint32_t)((quad * 32 + rq + 8 * k) * 32 + 4 * q);
+        tc::st_shared_b32(sp + ro, pack2(hp[0], hp[1], (TO*)nullptr));
+        tc::st_shared_b32(sp + ro + 16u, pack2(hp[2], hp[3], (TO*)nullptr));
+        tc::st_shared_b32(sp + 4096u + ro, pack2(hm[0], hm[1], (TO*)nullptr));
+        tc::st_shared_b32(sp + 4096u + ro + 16u, pack2(hm[2], hm[3], (TO*)nullptr));
+      }
+      tc::fence_proxy_async_smem();
+      tc::named_bar_sync(4 + half, 128);
+      if (issuer) {
+        tc::tma_store_2d(&tm.y, n, (int)row0, sp);
+        tc::tma_store_2d(&tm.y16, n, (int)row0, sp + 4096u);
+        tc::bulk_commit();
+        pending = true;
+      }
+    }
+  }
+  return true;
+}
+
 // SMODE (StageMode): STAGE_ALL -- the launch has the whole low-rank term on the
 // MMA (aug_mode LOWRANK_ALL_ON_TC) and Y's store maps in tm.y / tm.y16, the
 // table region holds the output staging buffers; STAGE_MIRROR -- the two signs
@@ -327,8 +463,9 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
   constexpr int CW = MODE == MODE_GATED ? 8 : 16;   // epilogue chunk width (gated: two accumulators)
   const bool mismatch =
       (SMODE == STAGE_ALL && (prm.aug_mode != LOWRANK_ALL_ON_TC || prm.y_staged != STAGE_ALL)) ||
-      (SMODE == STAGE_MIRROR && (prm.aug_mode != LOWRANK_C_ON_TC || prm.y_staged != STAGE_MIRROR || !prm.shared ||
-                                 prm.nb != 2));
+      ((SMODE == STAGE_MIRROR || SMODE == STAGE_MIRROR4) &&
+       (prm.aug_mode != LOWRANK_C_ON_TC || prm.y_staged != SMODE || !prm.shared || prm.nb != 2)) ||
+      (SMODE == STAGE_MIRROR4 && MODE == MODE_GATED && prm.P2 != prm.P);
   if (mismatch) {                                   // uniform: both CTAs of a pair leave
     pdl_wait();
     if (threadIdx.x == 0 && blockIdx.x == 0) record_error(prm.status, ZOACT_ERR_INVALID_ARG);
@@ -483,6 +620,9 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       else if constexpr (SMODE == STAGE_MIRROR)
         ok = epi_mirror_staged<TO, RT, MODE>(prm, tm, ss, tbl, etid, half, row_in_tile, row0, m, row_ok, n_blk, bn,
                                              buf, acc_phase, t_row, abort_flag, pending);
+      else if constexpr (SMODE == STAGE_MIRROR4)
+        ok = epi_mirror4_staged<TO, RT, MODE>(prm, tm, ss, tbl, etid, half, quad, lane, row0, n_blk, bn, buf,
+                                              acc_phase, t_row, abort_flag, pending);
       else
         ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, tbl, etid, half, row0, m, row_ok, n_blk, bn, buf, acc_phase,
                                              t_row, abort_flag);

@@ -159,6 +159,38 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// Four rows x four columns per thread from 32 TMEM lanes (two 16x256b.x2 loads at lanes +0
+// and +16 of taddr, one wait): thread t holds rows t/4 + 8k (k = 0..3) and columns
+// (2(t%4), 2(t%4)+1, 8+2(t%4), 9+2(t%4)) of the 16 at taddr, as v[4k + i].
+__device__ __forceinline__ void tmem_ld_rows4(uint32_t taddr, float* v) {
+  uint32_t a[8], b[8];
+  asm volatile("tcgen05.ld.sync.aligned.16x256b.x2.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3]), "=r"(a[4]), "=r"(a[5]), "=r"(a[6]), "=r"(a[7])
+               : "r"(taddr)
+               : "memory");
+  asm volatile("tcgen05.ld.sync.aligned.16x256b.x2.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(b[0]), "=r"(b[1]), "=r"(b[2]), "=r"(b[3]), "=r"(b[4]), "=r"(b[5]), "=r"(b[6]), "=r"(b[7])
+               : "r"(taddr + (16u << 16))
+               : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+  // registers of one load: {0,1,4,5} = first row's columns, {2,3,6,7} = the row 8 lanes down
+  const uint32_t* src[2] = {a, b};
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      v[8 * h + 4 * k + 0] = __uint_as_float(src[h][2 * k + 0]);
+      v[8 * h + 4 * k + 1] = __uint_as_float(src[h][2 * k + 1]);
+      v[8 * h + 4 * k + 2] = __uint_as_float(src[h][2 * k + 4]);
+      v[8 * h + 4 * k + 3] = __uint_as_float(src[h][2 * k + 5]);
+    }
+  }
+}
+
+__device__ __forceinline__ void st_shared_b32(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared.b32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
 __device__ __forceinline__ void tmem_ld8(uint32_t taddr, float* v) {
   uint32_t r[8];
   asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
