@@ -243,7 +243,8 @@ int zoact_multi_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoa
  * H = silu(y_gate) * y_up for both signs, with y_gate, y_up the pair forwards of
  * `gate` and `up` on the same X (same d_in, d_out, r and wtype).  H [2T, d_out]
  * of ydtype.  Gate and up keep their own U, C and layer_id (P_gate / P_up may be
- * the same pointer when the bases are equal; NULL computes them).               */
+ * the same pointer when the bases are equal; NULL computes them, once when gate
+ * and up point at the same U).                                                 */
 int zoact_pair_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up,
                              const void* X, int xdtype, int64_t T, int input_shared,
                              const float* P_gate, const float* P_up, float eps, uint64_t seed,

@@ -344,6 +344,7 @@ static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* 
     if (st) return st;
     P = p;
   }
+  if (L2 && !P2 && L2->U == L->U && L2->r == L->r && L2->d_in == L->d_in) P2 = P;   // one basis: one projection
   if (L2 && !P2) {
     float* p = static_cast<float*>(scratch(ctx, SLOT_P1, (size_t)rows * L2->r * sizeof(float)));
     if (!p) return ZOACT_ERR_NOMEM;

@@ -93,6 +93,23 @@ int encode_tmap_store(CUtensorMap* map, void* base, int ydtype, int64_t rows, in
   return res == CUDA_SUCCESS ? ZOACT_OK : ZOACT_ERR_INVALID_ARG;
 }
 
+int encode_tmap_store3(CUtensorMap* map, void* base, int ydtype, int64_t nb, int64_t rows, int64_t cols,
+                       int box_cols, int box_rows) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return ZOACT_ERR_CUDA;
+  const size_t es = dtype_size(ydtype);
+  const cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)rows, (cuuint64_t)nb};
+  const cuuint64_t strides[2] = {(cuuint64_t)cols * es, (cuuint64_t)rows * cols * es};
+  const cuuint32_t box[3] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows, 1u};
+  const cuuint32_t estr[3] = {1u, 1u, 1u};
+  const CUtensorMapDataType dt = ydtype == ZOACT_DT_FP32   ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32
+                                 : ydtype == ZOACT_DT_FP16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
+                                                           : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  const CUresult res = fn(map, dt, 3, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return res == CUDA_SUCCESS ? ZOACT_OK : ZOACT_ERR_INVALID_ARG;
+}
+
 int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   using namespace pairtc;
   // ranks above 32 have no epilogue tables: the low-rank term must ride the MMA, which needs stacked rows
@@ -281,6 +298,13 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     if (st) return st;
     // four rows per thread where the projections fit in registers (rank tile <= 16, one P for gate and up)
     p.y_staged = (rt <= 16 && (!gated || a.P2 == a.P)) ? STAGE_MIRROR4 : STAGE_MIRROR;
+  } else if (two && lmode == LOWRANK_C_ON_TC && a.shared && a.nb >= 2 && es == 2 && rt <= 16 &&
+             (!gated || a.P2 == a.P)) {
+    // other evaluation blocks on a shared input (the one-sided q-query estimator): one 3-D store map
+    st = encode_tmap_store3(&tm.y, a.Y, a.ydtype, a.nb, a.T, a.d_out, 16, BM);
+    if (st) return st;
+    tm.y16 = tm.y;
+    p.y_staged = STAGE_MULTI4;
   }
   p.aug_kb = lmode == LOWRANK_EPILOGUE ? 0 : slots * ka_tot / BK;
   p.aug_kb_slot = ka_tot / BK;

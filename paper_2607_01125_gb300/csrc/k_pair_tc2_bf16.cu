@@ -23,6 +23,17 @@ static int by_rank_two(Ctx* ctx, int mode, int rt, const TmaSet& tm, const Param
                               : launch_two<TO, 4, MODE_PAIR, STAGE_ALL>(ctx, tm, p);
   // the two signs on a shared input with 16-bit outputs: both signs staged for bulk stores
   if constexpr (sizeof(TO) == 2) {
+    if (p.y_staged == STAGE_MULTI4) {
+      switch (rt) {
+        case 4: return mode == MODE_GATED ? launch_two<TO, 4, MODE_GATED, STAGE_MULTI4>(ctx, tm, p)
+                                          : launch_two<TO, 4, MODE_PAIR, STAGE_MULTI4>(ctx, tm, p);
+        case 8: return mode == MODE_GATED ? launch_two<TO, 8, MODE_GATED, STAGE_MULTI4>(ctx, tm, p)
+                                          : launch_two<TO, 8, MODE_PAIR, STAGE_MULTI4>(ctx, tm, p);
+        case 16: return mode == MODE_GATED ? launch_two<TO, 16, MODE_GATED, STAGE_MULTI4>(ctx, tm, p)
+                                           : launch_two<TO, 16, MODE_PAIR, STAGE_MULTI4>(ctx, tm, p);
+        default: return ZOACT_ERR_UNSUPPORTED;
+      }
+    }
     if (p.y_staged == STAGE_MIRROR4) {
       switch (rt) {
         case 4: return mode == MODE_GATED ? launch_two<TO, 4, MODE_GATED, STAGE_MIRROR4>(ctx, tm, p)

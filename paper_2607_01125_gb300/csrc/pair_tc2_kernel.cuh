@@ -319,10 +319,10 @@ __device__ __forceinline__ bool epi_mirror_staged(const Params& prm, const TmaSe
 __device__ __forceinline__ int perm16(int c) { return 4 * ((c & 7) >> 1) + ((c >> 3) << 1) + (c & 1); }
 
 // Z table of one query over columns [col0, col0 + ncols) in 16-column chunks
-// permuted by perm16: tb[j * stride + (s & ~15) + perm16(s & 15)] = Z[j][col0 + s],
+// permuted by perm16: tb[j * stride + (s & ~15) + perm16(s & 15)] = c Z[j][col0 + s],
 // zero where col0 + s >= d_out or j >= r.  One thread per 4 consecutive columns.
 template <int RT>
-__device__ __forceinline__ void build_tables_z16(float* tb, int stride, const float* __restrict__ Zq, int col0,
+__device__ __forceinline__ void build_tables_z16(float* tb, int stride, const float* __restrict__ Zq, float c, int col0,
                                                  int ncols, int d_out, int r, int tid) {
   const int per_row = ncols / 4;
   for (int it = tid; it < RT * per_row; it += EPI_THREADS) {
@@ -331,9 +331,9 @@ __device__ __forceinline__ void build_tables_z16(float* tb, int stride, const fl
     float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
     if (j < r && col < d_out) z = *reinterpret_cast<const float4*>(Zq + (int64_t)j * d_out + col);
     float* row = tb + j * stride + (s & ~15);
-    const int c = s & 15;                       // columns c, c+1 and c+2, c+3 land as two pairs
-    *reinterpret_cast<float2*>(row + perm16(c)) = make_float2(z.x, z.y);
-    *reinterpret_cast<float2*>(row + perm16(c + 2)) = make_float2(z.z, z.w);
+    const int cc = s & 15;                      // columns cc, cc+1 and cc+2, cc+3 land as two pairs
+    *reinterpret_cast<float2*>(row + perm16(cc)) = make_float2(c * z.x, c * z.y);
+    *reinterpret_cast<float2*>(row + perm16(cc + 2)) = make_float2(c * z.z, c * z.w);
   }
 }
 
@@ -375,8 +375,9 @@ __device__ __forceinline__ bool epi_mirror4_staged(const Params& prm, const TmaS
     const int cwid = min(SLOTS, ncol_tile - s0);            // a multiple of 32
     const int col0 = n_blk * ncol_tile + s0;
     tc::named_bar_sync(1, EPI_THREADS);                     // previous pass's readers are done
-    build_tables_z16<RT>(tbl, STRIDE, prm.Zt + zq * prm.zt_qstride, col0, cwid, prm.d_out, r, etid);
-    if (GATED) build_tables_z16<RT>(tbl + TSZ, STRIDE, prm.Zt2 + zq * prm.zt_qstride, col0, cwid, prm.d_out, r, etid);
+    build_tables_z16<RT>(tbl, STRIDE, prm.Zt + zq * prm.zt_qstride, 1.f, col0, cwid, prm.d_out, r, etid);
+    if (GATED)
+      build_tables_z16<RT>(tbl + TSZ, STRIDE, prm.Zt2 + zq * prm.zt_qstride, 1.f, col0, cwid, prm.d_out, r, etid);
     tc::named_bar_sync(1, EPI_THREADS);
     if (!waited) {
       if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
@@ -450,6 +451,128 @@ __device__ __forceinline__ bool epi_mirror4_staged(const Params& prm, const TmaS
   return true;
 }
 
+// Column width of one table pass of the staged q-query epilogue: four permuted tables
+// (two blocks x gate, up) of RT x (MULTI4_SLOTS + TPAD) floats below the staging buffers.
+constexpr int MULTI4_SLOTS = 64;
+
+// The staged epilogue of several evaluation blocks on a shared input (C p in the
+// accumulator; the one-sided q-query estimator, or any blocks that are not the two
+// signs of one query), four rows per thread as in epi_mirror4_staged.  Blocks go in
+// pairs: per column pass the permuted tables c_b Z_b of both (gate at tbl + t TSZ,
+// up at tbl + (2 + t) TSZ; none for c_b = 0) are built, then each warpgroup forms
+// acc + c_b Z_b p for 16 columns of its 128 rows, one block after the other, stages
+// both blocks' outputs and one thread stores them through tm.y, a 3-D map over
+// the blocks' [T, d_out] slabs that drops rows past T and columns past d_out.
+template <typename TO, int RT, int MODE>
+__device__ __forceinline__ bool epi_multi4_staged(const Params& prm, const TmaSet& tm, SharedState2* ss, float* tbl,
+                                                  int etid, int half, int quad, int lane, int64_t row0, int n_blk,
+                                                  int bn, int buf, uint32_t acc_phase, uint32_t t_q,
+                                                  volatile int* abort_flag, bool& pending) {
+  constexpr bool GATED = MODE == MODE_GATED;
+  constexpr int SLOTS = MULTI4_SLOTS;
+  constexpr int STRIDE = SLOTS + TPAD;
+  constexpr int TSZ = RT * STRIDE;
+  static_assert(RT <= 16, "four rows of projections per thread");
+  static_assert((GATED ? 4 : 2) * TSZ * 4 <= MIRROR_STG_OFF, "q-query tables overlap the staging buffers");
+  static_assert(sizeof(TO) == 2, "staged q-query output is 16-bit");
+  const int r = prm.r;
+  const int q = lane & 3, rq = lane >> 2;
+  const bool vec = prm.vec_ok != 0;
+  float p[4][RT];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int64_t m = row0 + quad * 32 + rq + 8 * k;
+    load_p<RT>(p[k], prm.P, m, r, m < prm.rows, vec);
+  }
+  const int ncol_tile = GATED ? BN / 2 : bn;
+  const bool issuer = (etid & 127) == 0;
+  const uint32_t sp = tc::smem_u32(tbl) + MIRROR_STG_OFF + half * MIRROR_STG_BYTES;   // block slot t at +4096 t
+  bool waited = false;
+  for (int s0 = 0; s0 < ncol_tile; s0 += SLOTS) {
+    const int cwid = min(SLOTS, ncol_tile - s0);            // a multiple of 32
+    const int col0 = n_blk * ncol_tile + s0;
+    for (int bp = 0; bp < prm.nb; bp += 2) {
+      const int nblk = min(2, prm.nb - bp);
+      tc::named_bar_sync(1, EPI_THREADS);                   // previous pass's readers are done
+      for (int t = 0; t < nblk; ++t) {
+        const int b = bp + t;
+        if (prm.coef[b] == 0.f) continue;                   // its term is already in the accumulator
+        build_tables_z16<RT>(tbl + t * TSZ, STRIDE, prm.Zt + prm.zq[b] * prm.zt_qstride, prm.coef[b], col0, cwid,
+                             prm.d_out, r, etid);
+        if (GATED)
+          build_tables_z16<RT>(tbl + (2 + t) * TSZ, STRIDE, prm.Zt2 + prm.zq[b] * prm.zt_qstride, prm.coef[b], col0,
+                               cwid, prm.d_out, r, etid);
+      }
+      tc::named_bar_sync(1, EPI_THREADS);
+      if (!waited) {
+        if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
+        waited = true;
+      }
+      const int cbeg = s0 + half * (cwid / 2);
+      for (int c0 = cbeg; c0 < cbeg + cwid / 2; c0 += 16) {
+        const int n = n_blk * ncol_tile + c0;
+        if (n >= prm.d_out) break;                          // uniform over the warpgroup
+        float g[16], u[16];
+        tc::tmem_ld_rows4(t_q + (uint32_t)c0, g);
+        if (GATED) tc::tmem_ld_rows4(t_q + (uint32_t)(BN / 2 + c0), u);
+        if (issuer && pending) tc::bulk_wait_read0();       // the buffers' previous stores have read them
+        tc::named_bar_sync(4 + half, 128);
+#pragma unroll 1
+        for (int t = 0; t < nblk; ++t) {
+          float2 zg[4][2], zu[4][2];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) zg[k][0] = zg[k][1] = zu[k][0] = zu[k][1] = make_float2(0.f, 0.f);
+          if (prm.coef[bp + t] != 0.f) {
+            const float* tg = tbl + t * TSZ + (c0 - s0) + 4 * q;
+            const float* tu = tbl + (2 + t) * TSZ + (c0 - s0) + 4 * q;
+#pragma unroll
+            for (int j = 0; j < RT; ++j) {
+              const float4 a = *reinterpret_cast<const float4*>(tg + j * STRIDE);
+              float4 bv = a;
+              if (GATED) bv = *reinterpret_cast<const float4*>(tu + j * STRIDE);
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const float2 pj = make_float2(p[k][j], p[k][j]);
+                zg[k][0] = ffma2(make_float2(a.x, a.y), pj, zg[k][0]);
+                zg[k][1] = ffma2(make_float2(a.z, a.w), pj, zg[k][1]);
+                if (GATED) {
+                  zu[k][0] = ffma2(make_float2(bv.x, bv.y), pj, zu[k][0]);
+                  zu[k][1] = ffma2(make_float2(bv.z, bv.w), pj, zu[k][1]);
+                }
+              }
+            }
+          }
+          const uint32_t sb = sp + 4096u * (uint32_t)t;
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const float zgk[4] = {zg[k][0].x, zg[k][0].y, zg[k][1].x, zg[k][1].y};
+            const float zuk[4] = {zu[k][0].x, zu[k][0].y, zu[k][1].x, zu[k][1].y};
+            float h[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              if (GATED)
+                h[i] = silu_fast(g[4 * k + i] + zgk[i]) * (u[4 * k + i] + zuk[i]);
+              else
+                h[i] = apply_act(g[4 * k + i] + zgk[i], prm.act);
+            }
+            const uint32_t ro = (uint32_t)((quad * 32 + rq + 8 * k) * 32 + 4 * q);
+            tc::st_shared_b32(sb + ro, pack2(h[0], h[1], (TO*)nullptr));
+            tc::st_shared_b32(sb + ro + 16u, pack2(h[2], h[3], (TO*)nullptr));
+          }
+        }
+        tc::fence_proxy_async_smem();
+        tc::named_bar_sync(4 + half, 128);
+        if (issuer) {
+          for (int t = 0; t < nblk; ++t) tc::tma_store_3d(&tm.y, n, (int)row0, bp + t, sp + 4096u * (uint32_t)t);
+          tc::bulk_commit();
+          pending = true;
+        }
+      }
+    }
+  }
+  return true;
+}
+
 // SMODE (StageMode): STAGE_ALL -- the launch has the whole low-rank term on the
 // MMA (aug_mode LOWRANK_ALL_ON_TC) and Y's store maps in tm.y / tm.y16, the
 // table region holds the output staging buffers; STAGE_MIRROR -- the two signs
@@ -465,7 +588,9 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       (SMODE == STAGE_ALL && (prm.aug_mode != LOWRANK_ALL_ON_TC || prm.y_staged != STAGE_ALL)) ||
       ((SMODE == STAGE_MIRROR || SMODE == STAGE_MIRROR4) &&
        (prm.aug_mode != LOWRANK_C_ON_TC || prm.y_staged != SMODE || !prm.shared || prm.nb != 2)) ||
-      (SMODE == STAGE_MIRROR4 && MODE == MODE_GATED && prm.P2 != prm.P);
+      (SMODE == STAGE_MULTI4 && (prm.aug_mode != LOWRANK_C_ON_TC || prm.y_staged != SMODE || !prm.shared ||
+                                 prm.nb < 2)) ||
+      ((SMODE == STAGE_MIRROR4 || SMODE == STAGE_MULTI4) && MODE == MODE_GATED && prm.P2 != prm.P);
   if (mismatch) {                                   // uniform: both CTAs of a pair leave
     pdl_wait();
     if (threadIdx.x == 0 && blockIdx.x == 0) record_error(prm.status, ZOACT_ERR_INVALID_ARG);
@@ -623,6 +748,9 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       else if constexpr (SMODE == STAGE_MIRROR4)
         ok = epi_mirror4_staged<TO, RT, MODE>(prm, tm, ss, tbl, etid, half, quad, lane, row0, n_blk, bn, buf,
                                               acc_phase, t_row, abort_flag, pending);
+      else if constexpr (SMODE == STAGE_MULTI4)
+        ok = epi_multi4_staged<TO, RT, MODE>(prm, tm, ss, tbl, etid, half, quad, lane, row0, n_blk, bn, buf,
+                                             acc_phase, t_row, abort_flag, pending);
       else
         ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, tbl, etid, half, row0, m, row_ok, n_blk, bn, buf, acc_phase,
                                              t_row, abort_flag);

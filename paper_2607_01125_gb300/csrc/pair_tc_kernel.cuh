@@ -88,9 +88,10 @@ enum Mode { MODE_PAIR = 0, MODE_GATED = 1, MODE_PLAIN = 2 };
 // Tensor maps of one launch: X, W (gate), W up, and the low-rank K columns
 // A_aug, B_aug, B_aug up (unused ones are copies of a valid map).
 // Output staging of a CTA-pair launch (Params::y_staged, the kernel's SMODE): none, the whole
-// low-rank term on the MMA, or the two signs of one query on a shared input (row per thread, or
-// four rows per thread when the rank tile is <= 16 and a gated pair shares one projection).
-enum StageMode { STAGE_NONE = 0, STAGE_ALL = 1, STAGE_MIRROR = 2, STAGE_MIRROR4 = 3 };
+// low-rank term on the MMA, the two signs of one query on a shared input (row per thread, or
+// four rows per thread when the rank tile is <= 16 and a gated pair shares one projection), or
+// other evaluation blocks on a shared input (four rows per thread, same conditions).
+enum StageMode { STAGE_NONE = 0, STAGE_ALL = 1, STAGE_MIRROR = 2, STAGE_MIRROR4 = 3, STAGE_MULTI4 = 4 };
 
 struct TmaSet {
   CUtensorMap a, b, b2, aa, ba, ba2;

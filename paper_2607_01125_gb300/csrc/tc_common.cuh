@@ -238,6 +238,12 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int32_t x, 
                "r"(y), "r"(src)
                : "memory");
 }
+// The same for a 3-D tensor (x, y, z): z selects a slab, so a box is clipped at each slab's edge.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, int32_t x, int32_t y, int32_t z, uint32_t src) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(map), "r"(x),
+               "r"(y), "r"(z), "r"(src)
+               : "memory");
+}
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 // This thread's committed bulk stores have finished reading shared memory.
 __device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
@@ -263,5 +269,9 @@ int encode_tmap_2d_16bit(CUtensorMap* map, const void* base, int dtype, int64_t 
 // swizzle128 (box_cols * element size must then be 128) else none.
 int encode_tmap_store(CUtensorMap* map, void* base, int ydtype, int64_t rows, int64_t cols, int box_cols,
                       int box_rows, bool swizzle128);
+// Host: a 3-D output map over nb slabs of [rows, cols] (slab b at base + b rows cols), box =
+// 1 x box_rows x box_cols, no swizzle: a store is clipped at its slab's last row.
+int encode_tmap_store3(CUtensorMap* map, void* base, int ydtype, int64_t nb, int64_t rows, int64_t cols,
+                       int box_cols, int box_rows);
 
 }  // namespace zoact

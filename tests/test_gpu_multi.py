@@ -314,3 +314,38 @@ def test_bf16_one_sided_step(name, n_dec, T, q):
     assert np.mean(np.abs(Yg - Yo)) <= 1e-2 * np.mean(np.abs(Yo))
     np.testing.assert_allclose(out.cpu().numpy()[:q + 1], L, rtol=2e-2)
     step.ctx.close()
+
+
+@pytest.mark.parametrize("gated", [False, True])
+@pytest.mark.parametrize("T,nb,d_out,r,dt", [(300, 9, 264, 16, torch.bfloat16), (257, 3, 136, 8, torch.float16),
+                                             (512, 5, 520, 4, torch.bfloat16), (300, 2, 264, 16, torch.bfloat16)])
+def test_multi_shared_16bit_staged(ctx, gated, T, nb, d_out, r, dt):
+    # evaluation blocks on a shared input with 16-bit outputs (CTA pairs, one basis for gate and up): four rows
+    # per thread, outputs staged and written per block through a 3-D store map that drops rows past T (the
+    # partial last M tile) and columns past d_out -- no block may spill into the next, nothing past the output
+    d_in, seed, mu = 512, 8, 0.25
+    pts = _points(nb, mu) if nb > 2 else [(mu, 3), (mu, 4)]          # nb = 2: two queries, not a +/- pair
+    X = normal((T, d_in), 41, DEV, dtype=dt)
+    Wg = normal((d_out, d_in), 42, DEV, std=d_in ** -0.5, dtype=dt)
+    U = normal((d_in, r), 44, DEV) / np.sqrt(d_in)
+    Cg = normal((d_out * r,), 46, DEV, std=0.2)
+    Y = torch.full((nb * T + 8, d_out), 7.0, dtype=dt, device=DEV)
+    Yv = Y[:nb * T]
+    if gated:
+        Wu = normal((d_out, d_in), 43, DEV, std=d_in ** -0.5, dtype=dt)
+        Cu = normal((d_out * r,), 47, DEV, std=0.2)
+        zo.zoact_multi_forward_gated(ctx, zo.make_layer(Wg, U, Cg, 0), zo.make_layer(Wu, U, Cu, 1), X, T, True,
+                                     pts, seed, Yv)
+        torch.cuda.synchronize()
+        g, _, _ = _oracle(np64(Wg), np64(U), np64(Cg).reshape(d_out, r), np64(X), pts, T, True, seed, 0)
+        u, _, _ = _oracle(np64(Wu), np64(U), np64(Cu).reshape(d_out, r), np64(X), pts, T, True, seed, 1)
+        ref = layers.silu(g) * u
+    else:
+        zo.zoact_multi_forward(ctx, zo.make_layer(Wg, U, Cg, 0), X, T, True, pts, seed, Yv)
+        torch.cuda.synchronize()
+        ref, _, _ = _oracle(np64(Wg), np64(U), np64(Cg).reshape(d_out, r), np64(X), pts, T, True, seed, 0)
+    assert ctx.device_status() == 0
+    rel = {torch.bfloat16: 2.0 ** -8, torch.float16: 2.0 ** -11}[dt]
+    err = np.abs(np64(Yv) - ref)
+    assert np.all(err <= rel * np.abs(ref) + 2e-3 * np.abs(ref).max()), err.max()
+    assert torch.all(Y[nb * T:] == 7.0)
