@@ -84,7 +84,11 @@ class ZOStep:
         self.blocks = [(l.offset, l.d_out, l.r, l.layer_id) for l in linears]
         self.n_queries = n_queries                  # None: two-sided pair; q: one-sided with q queries
         self.nb = 2 if n_queries is None else int(n_queries) + 1
-        self.loss_out = torch.zeros(4 if n_queries is None else 2 * self.nb - 1, dtype=torch.float64, device=dev)
+        # two loss vectors, alternated by loss(): a step's result can be read back (on another stream) while
+        # the next step writes the other one
+        n_loss = 4 if n_queries is None else 2 * self.nb - 1
+        self._loss_bufs = [torch.zeros(n_loss, dtype=torch.float64, device=dev) for _ in range(2)]
+        self._loss_i = 0
         self._bufs = {}
         self._pcache = {}
         self.device = dev
@@ -232,8 +236,15 @@ class ZOStep:
         return h
 
     # ---- loss and update ----
+    @property
+    def loss_out(self):
+        """The device loss vector of the latest loss() call (update() reads it)."""
+        return self._loss_bufs[self._loss_i]
+
     def loss(self, Y, target):
-        """Two-sided: [L+, L-, D, a].  One-sided: [L_0 .. L_q, a_1 .. a_q]."""
+        """Two-sided: [L+, L-, D, a].  One-sided: [L_0 .. L_q, a_1 .. a_q].  Each call writes the loss vector
+        the previous call did not, so the previous step's vector stays valid until the call after next."""
+        self._loss_i ^= 1
         if self.n_queries is None:
             Z.zoact_loss_pair(self.ctx, Y, self.T, self.eps, self.loss_out, target=target)
         else:
@@ -262,8 +273,11 @@ def run_from_host(batches, step_fn, out_host):
     (on a side stream, into one of two device buffer sets) with the previous step's compute.
 
     batches: list of tuples of pinned host tensors (e.g. (x, target) or (x,)); step_fn(device_tensors, i)
-    issues step i on torch's current stream and returns its device loss vector, which is copied back
-    into out_host[i] (pinned).  Returns after issuing all work (no synchronisation).
+    issues step i on torch's current stream and returns its device loss vector, which is copied into
+    out_host[i] (pinned) on the side stream once step i has finished, so no copy sits between two steps'
+    kernels.  That needs consecutive steps to return different loss vectors (ZOStep.loss alternates two;
+    step i + 2 rewrites step i's only after its read-back): a step function that returns the same vector
+    twice in a row raises ValueError.  Returns after issuing all work (no synchronisation).
     """
     if not batches:
         return
@@ -272,6 +286,8 @@ def run_from_host(batches, step_fn, out_host):
     bufs = [[torch.empty(h.shape, dtype=h.dtype, device=main.device) for h in batches[0]] for _ in range(2)]
     copied = [torch.cuda.Event(), torch.cuda.Event()]
     free = [torch.cuda.Event(), torch.cuda.Event()]
+    read = [torch.cuda.Event(), torch.cuda.Event()]      # loss vector of step i read back (parity i % 2)
+    prev_ptr = None
 
     def fetch(i):
         b = i % 2
@@ -287,9 +303,17 @@ def run_from_host(batches, step_fn, out_host):
             fetch(i + 1)
         b = i % 2
         main.wait_event(copied[b])
+        if i >= 2:
+            main.wait_event(read[b])                     # step i - 2's loss vector, which step i rewrites, is read
         out = step_fn(bufs[b], i)
+        if out.data_ptr() == prev_ptr:
+            raise ValueError("run_from_host: consecutive steps must return different loss vectors")
+        prev_ptr = out.data_ptr()
         free[b].record(main)
-        out_host[i].copy_(out, non_blocking=True)
+        side.wait_event(free[b])
+        with torch.cuda.stream(side):
+            out_host[i].copy_(out, non_blocking=True)
+            read[b].record(side)
 
 
 def coefficient_offsets(specs, r):

@@ -218,3 +218,43 @@ def test_dependent_launch_bit_identical(name, n_dec, T, monkeypatch):
         assert torch.equal(Ya, Yb) and torch.equal(la, lb)
     assert torch.equal(C1, C2) and torch.equal(m1, m2) and torch.equal(v1, v2)
     serial.close()
+
+
+def test_run_from_host_matches_device_steps():
+    # the end-to-end path (pinned host inputs copied on a side stream, loss vectors read back there) runs the
+    # same steps as device-resident inputs: losses and coefficients bit for bit
+    from paper_2607_01125_gb300.model import run_from_host
+    w = workload("llama_mlp_bf16", T=256)
+    step, _ = _build(w)
+    n = 4
+    xs = [lowrank_activations(w.T, 4096, 64, 0.05, tensor_seed(w, "x", i), DEV)[0] for i in range(n)]
+    tgts = [normal((w.T, 4096), tensor_seed(w, "t", i), DEV, dtype=torch.bfloat16) for i in range(n)]
+    C0 = step.C.clone()
+    ref = []
+    for i in range(n):
+        Y = step.forward(xs[i], 5, i + 1)
+        ref.append(step.loss(Y, tgts[i]).clone())
+        step.update(i + 1, 5, i + 1)
+    torch.cuda.synchronize()
+    C_ref = step.C.clone()
+    step.C.copy_(C0); step.m.zero_(); step.v.zero_()
+    batches = [(xs[i].cpu().pin_memory(), tgts[i].cpu().pin_memory()) for i in range(n)]
+    outs = [torch.empty(ref[0].numel(), dtype=torch.float64).pin_memory() for _ in range(n)]
+
+    def sf(dev, i):
+        Y = step.forward(dev[0], 5, i + 1)
+        out = step.loss(Y, dev[1])
+        step.update(i + 1, 5, i + 1)
+        return out
+
+    run_from_host(batches, sf, outs)
+    torch.cuda.synchronize()
+    for i in range(n):
+        assert torch.equal(outs[i], ref[i].cpu()), i
+    assert torch.equal(step.C, C_ref)
+    assert step.ctx.device_status() == 0
+    fixed = torch.zeros(ref[0].numel(), dtype=torch.float64, device=DEV)
+    with pytest.raises(ValueError):
+        run_from_host(batches, lambda dev, i: fixed, outs)
+    torch.cuda.synchronize()
+    step.ctx.close()
