@@ -196,8 +196,7 @@ def time_diagnostics(ctx, step, dev, reps=20):
 
 
 def run_step(step, x, target, t, seed, world):
-    Y = step.forward(x, seed, t)
-    step.loss(Y, target)
+    step.forward_loss(x, target, seed, t)            # the pair forwards, then the loss pair
     if world > 1:
         from paper_2607_01125_gb300.dp import allreduce_loss
         allreduce_loss(step.loss_out)            # losses and a's are means over equal token counts

@@ -250,6 +250,24 @@ int zoact_pair_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoac
                              const float* P_gate, const float* P_up, float eps, uint64_t seed,
                              uint64_t query, void* H, int ydtype);
 
+/* ---- the last pair forward fused with its loss pair (Section 3; Algorithm 2) ----
+ * The losses zoact_loss_pair would return for Y = zoact_pair_forward(layer, X,
+ * stacked rows, eps, seed, query, act) rounded to ydtype, computed inside the
+ * pair forward's epilogue without writing Y.  X [2T, d_in] stacked (+ rows then
+ * - rows), target [T, d_out] of ydtype (16-byte aligned) or NULL for the mean
+ * square loss, out[4] = {L+, L-, D, a} fp64 in DEVICE memory, D = L+ - L- (the
+ * difference of the two sums, each over T * d_out rounded outputs; fp64 partials
+ * of compensated fp32 sums), a = D / (2 eps).  Qualifies: two-sided stacked rows,
+ * T a multiple of 256, 16-bit ydtype, the CTA-pair tensor-core path with the whole
+ * low-rank term on the MMA; otherwise ZOACT_ERR_UNSUPPORTED is returned before
+ * any launch of the pair forward itself (a projection U^T x, when P is NULL, may
+ * already have run) and the caller uses zoact_pair_forward + zoact_loss_pair.
+ * T = 0 writes nothing.  A non-finite result sets ZOACT_ERR_NONFINITE; a launch
+ * that timed out (ZOACT_ERR_TIMEOUT) writes no loss.                            */
+int zoact_pair_forward_loss(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype, int64_t T,
+                            const float* P, float eps, uint64_t seed, uint64_t query, int act, int ydtype,
+                            const void* target, double* out);
+
 /* ---- the loss pair (Section 3 estimator, two-sided; Algorithm 2) ----
  * Y [2T, n] stacked outputs of ydtype; target [T, n] of ydtype, or NULL for the
  * mean square loss.  Writes out[0] = L+ = mean((y+ - t)^2), out[1] = L-,

@@ -37,7 +37,7 @@ EXPORTS = [
     "zoact_rms_norm", "zoact_mix_rms", "zoact_multi_forward", "zoact_multi_forward_gated", "zoact_loss_multi",
     "zoact_adam_step_multi", "zoact_sgd_step_multi", "zoact_basis_prepared_bytes", "zoact_basis_prepare",
     "zoact_lowrank_proj_prepared", "zoact_subspace_overlap", "zoact_gradient_energy", "zoact_kernel_timing",
-    "zoact_kernel_time",
+    "zoact_kernel_time", "zoact_pair_forward_loss",
 ]
 
 
@@ -105,6 +105,7 @@ def load():
         "zoact_pair_forward_noalloc": [ctypes.POINTER(zoact_layer), P, I32, I64, I32, F32, U64, U64, I32, P, I32, P],
         "zoact_pair_forward_gated": [P, ctypes.POINTER(zoact_layer), ctypes.POINTER(zoact_layer), P, I32, I64, I32,
                                      P, P, F32, U64, U64, P, I32],
+        "zoact_pair_forward_loss": [P, ctypes.POINTER(zoact_layer), P, I32, I64, P, F32, U64, U64, I32, I32, P, P],
         "zoact_loss_pair": [P, P, I32, P, I64, I64, F32, P],
         "zoact_adam_step": [P, P, P, P, I64, ctypes.POINTER(zoact_coeff_block), I32, P, F32, F32, F32, F32, I64,
                             U64, U64],
@@ -268,6 +269,15 @@ def zoact_pair_forward_gated(ctx, gate, up, X, T, input_shared, eps, seed, query
     _check("zoact_pair_forward_gated", load().zoact_pair_forward_gated(
         ctx.handle, ctypes.byref(gate), ctypes.byref(up), _ptr(X), _dt(X), int(T), int(input_shared), _ptr(P_gate),
         _ptr(P_up), float(eps), int(seed), int(query), _ptr(H), _dt(H)))
+
+
+def zoact_pair_forward_loss(ctx, layer, X, T, eps, seed, query, ydtype, out, target=None, P=None, act=ACT_NONE):
+    """The pair forward of `layer` on stacked X [2T, d_in] fused with its loss pair: out[4] = {L+, L-, D, a} of
+    the outputs rounded to ydtype (DT_BF16 / DT_FP16), Y not written.  Raises ZoactError with status
+    ZOACT_ERR_UNSUPPORTED when the launch does not qualify (see include/zoact.h)."""
+    _check("zoact_pair_forward_loss", load().zoact_pair_forward_loss(
+        ctx.handle, ctypes.byref(layer), _ptr(X), _dt(X), int(T), _ptr(P), float(eps), int(seed), int(query),
+        int(act), int(ydtype), _ptr(target), _ptr(out)))
 
 
 def zoact_loss_pair(ctx, Y, T, eps, out, target=None):

@@ -314,9 +314,16 @@ int zoact_lowrank_proj_prepared(zoact_ctx* ctx, const void* X, int xdtype, int64
   return launch_lowrank_proj_tc_prepared(ctx, X, xdtype, rows, d_in, U_tc, r, P);
 }
 
+// The loss pair fused into the last pair forward (zoact_pair_forward_loss).
+struct FusedLoss {
+  const void* target;
+  double* out;
+  float eps;
+};
+
 static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* L2, const void* X, int xdtype,
                        int64_t T, int input_shared, const float* P, const float* P2, const zoact_eval_blocks* blk,
-                       uint64_t seed, int act, void* Y, int ydtype) {
+                       uint64_t seed, int act, void* Y, int ydtype, const FusedLoss* fl = nullptr) {
   if (check_eval_blocks(blk)) return ZOACT_ERR_INVALID_ARG;
   int st = check_layer(L);
   if (st) return st;
@@ -328,10 +335,17 @@ static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* 
   }
   if (T < 0 || !valid_act_dtype(xdtype) || !valid_act_dtype(ydtype)) return ZOACT_ERR_INVALID_ARG;
   if (act < ZOACT_ACT_NONE || act > ZOACT_ACT_GELU) return ZOACT_ERR_INVALID_ARG;
+  if (fl) {
+    if (!fl->out || !(fl->eps > 0.0f) || (fl->target && !aligned16(fl->target))) return ZOACT_ERR_INVALID_ARG;
+    if (input_shared || blk->n_blocks != 2 || T % 256 != 0 || xdtype == ZOACT_DT_FP32 ||
+        (ydtype != ZOACT_DT_BF16 && ydtype != ZOACT_DT_FP16))
+      return ZOACT_ERR_UNSUPPORTED;
+  }
   if (T == 0) return ZOACT_OK;
-  if (!X || !Y) return ZOACT_ERR_INVALID_ARG;
+  if (!X || (!Y && !fl)) return ZOACT_ERR_INVALID_ARG;
   if (L->wtype == ZOACT_DT_INT4_G128 ? xdtype != ZOACT_DT_BF16 : xdtype != L->wtype) return ZOACT_ERR_INVALID_ARG;
-  if (!aligned16(X) || !aligned16(Y) || !aligned16(L->W) || (L2 && !aligned16(L2->W))) return ZOACT_ERR_INVALID_ARG;
+  if (!aligned16(X) || (Y && !aligned16(Y)) || !aligned16(L->W) || (L2 && !aligned16(L2->W)))
+    return ZOACT_ERR_INVALID_ARG;
   if (L->d_in % (xdtype == ZOACT_DT_FP32 ? 4 : 8) != 0) return ZOACT_ERR_INVALID_ARG;
   if (L->d_out % 8 != 0) return ZOACT_ERR_INVALID_ARG;
   if (T > ((int64_t)1 << 40) / blk->n_blocks) return ZOACT_ERR_INVALID_ARG;
@@ -361,8 +375,18 @@ static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* 
   for (int b = 0; b < blk->n_blocks; ++b) { a.coef[b] = blk->coef[b]; a.qry[b] = blk->query[b]; }
   a.seed = seed; a.layer_id = L->layer_id;
   if (L2) { a.W2 = L2->W; a.w_scales2 = L2->w_scales; a.P2 = P2; a.C2 = L2->C; a.layer_id2 = L2->layer_id; }
+  if (fl) { a.fuse_loss = 1; a.target = fl->target; a.loss_out = fl->out; a.loss_eps = fl->eps; }
   if (xdtype == ZOACT_DT_FP32) return launch_pair_simt(ctx, a);
   return launch_pair_tc(ctx, a);
+}
+
+int zoact_pair_forward_loss(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype, int64_t T,
+                            const float* P, float eps, uint64_t seed, uint64_t query, int act, int ydtype,
+                            const void* target, double* out) {
+  ZOACT_ENTER(ctx);
+  const zoact_eval_blocks b = pair_blocks(eps, query);
+  const FusedLoss fl{target, out, eps};
+  return pair_common(ctx, layer, nullptr, X, xdtype, T, 0, P, nullptr, &b, seed, act, nullptr, ydtype, &fl);
 }
 
 int zoact_pair_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype, int64_t T,

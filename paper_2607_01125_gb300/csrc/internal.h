@@ -168,6 +168,11 @@ struct PairArgs {
   const float* P2;
   const float* C2;
   uint32_t layer_id2;
+  // fused loss pair (zoact_pair_forward_loss): Y is not written; the losses of the rounded outputs
+  int fuse_loss;
+  const void* target;   // [T, d_out] of ydtype, or nullptr (mean of squares)
+  double* loss_out;     // [4] = {L+, L-, D, a}
+  float loss_eps;
 };
 // The two-sided pair as evaluation blocks: {+eps, -eps} with the same query.
 inline void set_pair_blocks(PairArgs& a, float eps, uint64_t query) {

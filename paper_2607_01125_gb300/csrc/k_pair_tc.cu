@@ -212,6 +212,10 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   }
   if (big_r && lmode != LOWRANK_ALL_ON_TC) return ZOACT_ERR_UNSUPPORTED;
   if (lmode == LOWRANK_ALL_ON_TC) rt = 4;   // whole term on the tensor cores: no epilogue tables
+  // the fused loss needs CTA pairs whose 128-row halves each lie in one sign block, whole term on the MMA
+  if (a.fuse_loss && !(two && !gated && lmode == LOWRANK_ALL_ON_TC && a.nb == 2 && !a.shared &&
+                       a.T % (2 * BM) == 0 && dtype_size(a.ydtype) == 2))
+    return ZOACT_ERR_UNSUPPORTED;
   const int ka = aug_cols(a.r);
   const int ka_tot = distinct ? 2 * ka : ka;
   tm.aa = tm.a; tm.ba = tm.b; tm.ba2 = tm.b2;
@@ -283,7 +287,23 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   tm.y = tm.y16 = tm.a;
   p.y_staged = STAGE_NONE;
   const int es = (int)dtype_size(a.ydtype);
-  if (two && lmode == LOWRANK_ALL_ON_TC && rt == 4) {
+  if (a.fuse_loss) {
+    // no output: the target comes through tm.y / tm.y16 into the staging buffers
+    p.y_staged = STAGE_LOSS;
+    p.has_target = a.target ? 1 : 0;
+    p.loss_eps = a.loss_eps;
+    p.loss_out = a.loss_out;
+    p.loss_ticket = ctx->d_tickets + 4;
+    p.loss_part = static_cast<double*>(scratch(ctx, SLOT_PARTIALS, (size_t)ctx->sm_count * 2 * sizeof(double)));
+    if (!p.loss_part) return ZOACT_ERR_NOMEM;
+    if (a.target) {
+      void* t0 = const_cast<void*>(a.target);
+      st = encode_tmap_store(&tm.y, t0, a.ydtype, a.T, a.d_out, 128 / es, BM, true);
+      if (st) return st;
+      st = encode_tmap_store(&tm.y16, t0, a.ydtype, a.T, a.d_out, 16, BM, false);
+      if (st) return st;
+    }
+  } else if (two && lmode == LOWRANK_ALL_ON_TC && rt == 4) {
     st = encode_tmap_store(&tm.y, a.Y, a.ydtype, a.rows, a.d_out, 128 / es, BM, true);
     if (st) return st;
     st = encode_tmap_store(&tm.y16, a.Y, a.ydtype, a.rows, a.d_out, 16, BM, false);

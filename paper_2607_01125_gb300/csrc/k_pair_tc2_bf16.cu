@@ -23,6 +23,8 @@ static int by_rank_two(Ctx* ctx, int mode, int rt, const TmaSet& tm, const Param
                               : launch_two<TO, 4, MODE_PAIR, STAGE_ALL>(ctx, tm, p);
   // the two signs on a shared input with 16-bit outputs: both signs staged for bulk stores
   if constexpr (sizeof(TO) == 2) {
+    if (p.y_staged == STAGE_LOSS)
+      return mode == MODE_PAIR && rt == 4 ? launch_two<TO, 4, MODE_PAIR, STAGE_LOSS>(ctx, tm, p) : ZOACT_ERR_UNSUPPORTED;
     if (p.y_staged == STAGE_MULTI4) {
       switch (rt) {
         case 4: return mode == MODE_GATED ? launch_two<TO, 4, MODE_GATED, STAGE_MULTI4>(ctx, tm, p)

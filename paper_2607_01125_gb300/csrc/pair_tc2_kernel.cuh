@@ -44,6 +44,7 @@ struct SharedState2 {
   uint64_t tmem_full[2];
   uint64_t tmem_empty[2];
   uint64_t drain;
+  uint64_t tload[2];      // fused loss: target chunk landed in a warpgroup's staging buffer
   uint32_t tmem_base;
   int abort_flag;
   int epi_ok;
@@ -573,6 +574,157 @@ __device__ __forceinline__ bool epi_multi4_staged(const Params& prm, const TmaSe
   return true;
 }
 
+// Compensated fp32 sum of squares: d^2 = p + e exactly (p = fp32(d d), e = fma(d, d, -p));
+// the p go into a Neumaier sum (the rounding error of every add carried in c) and the
+// tiny e into a plain sum, so S = s + c + e keeps about twice fp32 precision without
+// fp64 adds -- enough that the difference of the two signs' sums is still accurate.
+struct CompSum {
+  float s = 0.f, c = 0.f, e = 0.f;
+  __device__ __forceinline__ void add_sq(float d) {
+    const float p = d * d;
+    e += fmaf(d, d, -p);
+    const float t = s + p;
+    c += fabsf(s) >= p ? (s - t) + p : (p - t) + s;
+    s = t;
+  }
+  __device__ __forceinline__ double value() const { return (double)s + (double)c + (double)e; }
+};
+
+// 8 16-bit values of a 16-byte granule.
+template <typename TO>
+__device__ __forceinline__ void unpack8_16(uint4 g, float* v) {
+  const uint32_t w[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    TO lo, hi;
+    const uint16_t a = (uint16_t)(w[i] & 0xFFFFu), b = (uint16_t)(w[i] >> 16);
+    memcpy(&lo, &a, 2);
+    memcpy(&hi, &b, 2);
+    v[2 * i] = to_f32<TO>(lo);
+    v[2 * i + 1] = to_f32<TO>(hi);
+  }
+}
+
+// Loss-pair epilogue of one accumulator tile (STAGE_LOSS: stacked rows, the whole
+// low-rank term in the accumulator, T a multiple of 256 so that this CTA's 128 rows
+// all belong to one sign).  Y is not written: for each 128-byte chunk of this
+// warpgroup's columns one thread loads the target's matching [128 x chunk] box into
+// the warpgroup's staging buffer (tm.y, 128-byte swizzled; tm.y16 for 16-column
+// remainders), and every thread adds (round(y) - t)^2 of its row -- y rounded to
+// Y's 16-bit type as zoact_loss_pair would read it -- to the compensated sum of
+// squares of the row's sign.  Columns past d_out are skipped (their accumulator columns hold the
+// other block's low-rank term).  Returns false when the accumulator wait gave up.
+template <typename TO>
+__device__ __forceinline__ bool epi_loss_staged(const Params& prm, const TmaSet& tm, SharedState2* ss, uint8_t* stg,
+                                                int etid, int half, int rl, int64_t row0, int n_blk, int bn, int buf,
+                                                uint32_t acc_phase, uint32_t t_row, volatile int* abort_flag,
+                                                uint32_t& tphase, CompSum* acc) {
+  constexpr int EB = (int)sizeof(TO);
+  constexpr int CC = 128 / EB;      // columns of a full chunk
+  constexpr int NC = 16;            // columns of a narrow chunk
+  static_assert(EB == 2, "fused loss of 16-bit outputs");
+  if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
+  const int wcols = bn / 2;
+  const int cb = half * wcols;
+  const int sgn = row0 >= prm.T ? 1 : 0;
+  const int64_t trow0 = row0 - (sgn ? prm.T : 0);
+  const bool issuer = (etid & 127) == 0;
+  const uint32_t sbuf = tc::smem_u32(stg + half * STG_BYTES);
+  const uint32_t tbar = tc::smem_u32(&ss->tload[half]);
+  CompSum& S = acc[sgn];
+  for (int c = 0; c < wcols;) {
+    const int n = n_blk * bn + cb + c;
+    if (n >= prm.d_out) break;                      // uniform over the warpgroup
+    const bool full = wcols - c >= CC;
+    const int cw = full ? CC : NC;
+    if (prm.has_target) {
+      tc::named_bar_sync(4 + half, 128);            // the previous chunk's readers of the buffer are done
+      if (issuer) {
+        tc::mbar_arrive_expect_tx(tbar, (uint32_t)(BM * cw * EB));
+        tc::tma_load_2d(sbuf, full ? &tm.y : &tm.y16, n, (int)trow0, tbar);
+        // bounded: on expiry the abort flag is set and the launch writes no loss, but the warpgroup stays
+        // on one path (no thread leaves a named barrier short)
+        tc::mbar_wait(tbar, tphase, abort_flag, prm.status);
+      }
+      tphase ^= 1u;
+      tc::named_bar_sync(4 + half, 128);            // the chunk has landed
+    }
+    for (int p = 0; p < cw; p += 16) {
+      float v[16];
+      tc::tmem_ld16(t_row + (uint32_t)(cb + c + p), v);
+#pragma unroll
+      for (int g = 0; g < 2; ++g) {
+        float t8[8];
+        if (prm.has_target) {
+          const int gi = (p >> 3) + g;
+          unpack8_16<TO>(tc::ld_shared_v4(sbuf + (full ? sw128_off(rl, gi) : (uint32_t)(rl * NC * EB + gi * 16))),
+                         t8);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) t8[i] = 0.f;
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float y = to_f32<TO>(from_f32<TO>(apply_act(v[8 * g + i], prm.act)));
+          if (n + p + 8 * g + i < prm.d_out) S.add_sq(y - t8[i]);   // y - t is exact in fp32
+        }
+      }
+    }
+    c += cw;
+  }
+  return true;
+}
+
+// The end of a fused-loss launch: the epilogue threads' sums (two signs) are added
+// in a fixed order into this CTA's partial; the last CTA to finish (atomic ticket)
+// adds all partials in CTA order and writes {L+, L-, D, a}, D = L+ - L- and
+// a = D / (2 eps), then resets the ticket.  red: 2 x EPI_THREADS doubles of shared memory.
+__device__ __forceinline__ void loss_finish(const Params& prm, const CompSum* acc, double* red, int etid) {
+  red[2 * etid] = acc[0].value();
+  red[2 * etid + 1] = acc[1].value();
+  tc::named_bar_sync(3, EPI_THREADS);
+  if (etid >= 32) return;
+  // warp 0 of the epilogue: lane l adds threads l, l + 32, ...; then a fixed butterfly
+  double s0 = 0.0, s1 = 0.0;
+  for (int i = etid; i < EPI_THREADS; i += 32) { s0 += red[2 * i]; s1 += red[2 * i + 1]; }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    s0 += __shfl_xor_sync(0xffffffffu, s0, o);
+    s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+  }
+  unsigned int last = 0;
+  if (etid == 0) {
+    prm.loss_part[2 * blockIdx.x] = s0;
+    prm.loss_part[2 * blockIdx.x + 1] = s1;
+    __threadfence();
+    last = atomicAdd(prm.loss_ticket, 1u) == gridDim.x - 1 ? 1u : 0u;
+  }
+  last = __shfl_sync(0xffffffffu, last, 0);
+  if (!last) return;
+  __threadfence();
+  double a0 = 0.0, a1 = 0.0;
+  for (unsigned int b = etid; b < gridDim.x; b += 32) {
+    a0 += __ldcg(prm.loss_part + 2 * b);
+    a1 += __ldcg(prm.loss_part + 2 * b + 1);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    a0 += __shfl_xor_sync(0xffffffffu, a0, o);
+    a1 += __shfl_xor_sync(0xffffffffu, a1, o);
+  }
+  if (etid == 0) {
+    const double inv = 1.0 / ((double)prm.T * (double)prm.d_out);
+    const double Lp = a0 * inv, Lm = a1 * inv, D = (a0 - a1) * inv;
+    const double a = D / (2.0 * (double)prm.loss_eps);
+    prm.loss_out[0] = Lp;
+    prm.loss_out[1] = Lm;
+    prm.loss_out[2] = D;
+    prm.loss_out[3] = a;
+    if (!isfinite(Lp) || !isfinite(Lm) || !isfinite(a)) record_error(prm.status, ZOACT_ERR_NONFINITE);
+    *prm.loss_ticket = 0u;
+  }
+}
+
 // SMODE (StageMode): STAGE_ALL -- the launch has the whole low-rank term on the
 // MMA (aug_mode LOWRANK_ALL_ON_TC) and Y's store maps in tm.y / tm.y16, the
 // table region holds the output staging buffers; STAGE_MIRROR -- the two signs
@@ -590,7 +742,9 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
        (prm.aug_mode != LOWRANK_C_ON_TC || prm.y_staged != SMODE || !prm.shared || prm.nb != 2)) ||
       (SMODE == STAGE_MULTI4 && (prm.aug_mode != LOWRANK_C_ON_TC || prm.y_staged != SMODE || !prm.shared ||
                                  prm.nb < 2)) ||
-      ((SMODE == STAGE_MIRROR4 || SMODE == STAGE_MULTI4) && MODE == MODE_GATED && prm.P2 != prm.P);
+      ((SMODE == STAGE_MIRROR4 || SMODE == STAGE_MULTI4) && MODE == MODE_GATED && prm.P2 != prm.P) ||
+      (SMODE == STAGE_LOSS && (MODE != MODE_PAIR || prm.aug_mode != LOWRANK_ALL_ON_TC || prm.y_staged != SMODE ||
+                               prm.shared || prm.nb != 2 || prm.T % BM2 != 0));
   if (mismatch) {                                   // uniform: both CTAs of a pair leave
     pdl_wait();
     if (threadIdx.x == 0 && blockIdx.x == 0) record_error(prm.status, ZOACT_ERR_INVALID_ARG);
@@ -617,6 +771,8 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       tc::mbar_init(tc::smem_u32(&ss->tmem_empty[b]), 2);   // one arrival per CTA (leader's copy is used)
     }
     tc::mbar_init(tc::smem_u32(&ss->drain), 1);
+    tc::mbar_init(tc::smem_u32(&ss->tload[0]), 1);
+    tc::mbar_init(tc::smem_u32(&ss->tload[1]), 1);
     ss->abort_flag = 0;
     tc::fence_mbar_init();
     tc::prefetch_tmap(&tm.a);
@@ -729,6 +885,9 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
     const uint32_t tmem_empty_leader1 = tc2::map_to(tc::smem_u32(&ss->tmem_empty[1]), 0);
     int local = 0;
     bool pending = false;                   // staged output: this thread has bulk stores in flight
+    uint32_t tphase = 0;                    // fused loss: parity of this warpgroup's next target load
+    CompSum lacc[2];                        // fused loss: running sums of the + and - rows
+    bool aborted = false;
     for (int tile = cluster_id; tile < prm.num_tiles; tile += n_clusters, ++local) {
       int m_blk, n_blk;
       tile_coords(tile, num_m, num_n, m_blk, n_blk);
@@ -751,15 +910,32 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       else if constexpr (SMODE == STAGE_MULTI4)
         ok = epi_multi4_staged<TO, RT, MODE>(prm, tm, ss, tbl, etid, half, quad, lane, row0, n_blk, bn, buf,
                                              acc_phase, t_row, abort_flag, pending);
+      else if constexpr (SMODE == STAGE_LOSS)
+        ok = epi_loss_staged<TO>(prm, tm, ss, reinterpret_cast<uint8_t*>(tbl), etid, half, row_in_tile, row0, n_blk,
+                                 bn, buf, acc_phase, t_row, abort_flag, tphase, lacc);
       else
         ok = epi_pair_tile<TO, RT, MODE, CW>(prm, ss, tbl, etid, half, row0, m, row_ok, n_blk, bn, buf, acc_phase,
                                              t_row, abort_flag);
-      if (!ok) break;
+      if (!ok) { aborted = true; break; }
       tc::tc_fence_before();
       tc::named_bar_sync(3, EPI_THREADS);        // every epilogue thread of this CTA has read the tile
       if (etid == 0) tc2::arrive_cluster(buf ? tmem_empty_leader1 : tmem_empty_leader0);
     }
     if (pending) tc::bulk_wait0();           // the stores have read the staging buffers and completed
+    if constexpr (SMODE == STAGE_LOSS) {
+      // every epilogue thread gets here (the accumulator wait gives up uniformly); an aborted CTA adds no
+      // partial, so the ticket stays short and the launch reports ZOACT_ERR_TIMEOUT with no loss written
+      tc::named_bar_sync(3, EPI_THREADS);
+      if (etid == 0) ss->epi_ok = (*abort_flag || aborted) ? 0 : 1;   // one reading, shared by all
+      tc::named_bar_sync(3, EPI_THREADS);
+      if (*reinterpret_cast<volatile int*>(&ss->epi_ok) != 0) {
+        loss_finish(prm, lacc, reinterpret_cast<double*>(tbl), etid);
+      } else if ((etid & 127) == 0) {               // give a target load still in flight time to land
+        const uint64_t t0 = tc::global_timer_ns();
+        while (tc::global_timer_ns() - t0 < 2000000ull) {
+        }
+      }
+    }
   }
 
   tc::tc_fence_before();

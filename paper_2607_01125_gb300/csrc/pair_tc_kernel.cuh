@@ -90,8 +90,10 @@ enum Mode { MODE_PAIR = 0, MODE_GATED = 1, MODE_PLAIN = 2 };
 // Output staging of a CTA-pair launch (Params::y_staged, the kernel's SMODE): none, the whole
 // low-rank term on the MMA, the two signs of one query on a shared input (row per thread, or
 // four rows per thread when the rank tile is <= 16 and a gated pair shares one projection), or
-// other evaluation blocks on a shared input (four rows per thread, same conditions).
-enum StageMode { STAGE_NONE = 0, STAGE_ALL = 1, STAGE_MIRROR = 2, STAGE_MIRROR4 = 3, STAGE_MULTI4 = 4 };
+// other evaluation blocks on a shared input (four rows per thread, same conditions), or no output at
+// all: the loss pair of the rounded outputs, fused (zoact_pair_forward_loss).
+enum StageMode { STAGE_NONE = 0, STAGE_ALL = 1, STAGE_MIRROR = 2, STAGE_MIRROR4 = 3, STAGE_MULTI4 = 4,
+                 STAGE_LOSS = 5 };
 
 struct TmaSet {
   CUtensorMap a, b, b2, aa, ba, ba2;
@@ -135,6 +137,13 @@ struct Params {
   const uint8_t* Wq2;
   const __half* Ws2;
   int* status;
+  // fused loss pair (STAGE_LOSS): target [T, d_out] of Y's type through tm.y / tm.y16 (or none: mean of
+  // squares), per-CTA partial sums, the ticket of the last CTA, and out[4] = {L+, L-, D, a}
+  int has_target;
+  float loss_eps;
+  double* loss_part;
+  unsigned int* loss_ticket;
+  double* loss_out;
 };
 
 struct SharedState {

@@ -94,6 +94,9 @@ class ZOStep:
         self.device = dev
         self.capture = None
         self.flops = None
+        # forward_loss fuses the loss pair into the last linear when set; off by default: the fused epilogue
+        # lengthens the Llama-3-8B down launch by more than the separate loss launch takes
+        self.fuse_loss = False
         self._utc = {}
         self.prepare_bases()
 
@@ -155,13 +158,25 @@ class ZOStep:
     def points(self, query):
         return Z.one_sided_blocks(self.eps, self.query_ids(query))
 
-    def pair(self, name, X, shared, seed, query, out_key, act=Z.ACT_NONE):
+    def pair(self, name, X, shared, seed, query, out_key, act=Z.ACT_NONE, fused=None):
+        """fused = (target, out): the last linear with the loss pair fused (zoact_pair_forward_loss); returns None
+        when that ran, else (the launch does not qualify) the output as without it."""
         l = self.by_name[name]
         if self.capture is not None:
             self.capture(name, X[:self.T])
         P = self._proj(l, X, 0)
-        Y = self.buf(out_key, self.nb * self.T, l.d_out)
         flops = 2.0 * X.shape[0] * l.d_in * l.d_out
+        if fused is not None and self.n_queries is None and not shared:
+            target, out = fused
+            try:
+                self._counted(lambda: Z.zoact_pair_forward_loss(self.ctx, l.layer, X, self.T, self.eps, seed, query,
+                                                                Z.TORCH_DT[self.dtype], out, target=target, P=P,
+                                                                act=act), flops)
+                return None
+            except Z.ZoactError as e:
+                if e.status != Z.ZOACT_ERR_UNSUPPORTED:
+                    raise
+        Y = self.buf(out_key, self.nb * self.T, l.d_out)
         if self.n_queries is None:
             fn = lambda: Z.zoact_pair_forward(self.ctx, l.layer, X, self.T, shared, self.eps, seed, query, Y, P=P,
                                               act=act)
@@ -198,17 +213,32 @@ class ZOStep:
         return Y
 
     # ---- forward graphs ----
-    def forward(self, x, seed, query):
+    def forward(self, x, seed, query, fused=None):
+        """The graph's output; with fused = (target, out) the last linear writes the loss pair into out instead
+        where it can (then None is returned)."""
         self._pcache = {}
         if self.kind == "toy":
             h = self.pair("l1", x, True, seed, query, "h", act=Z.ACT_GELU)
-            return self.pair("l2", h, False, seed, query, "y")
+            return self.pair("l2", h, False, seed, query, "y", fused=fused)
         if self.kind == "llama_mlp":
             H = self.gated("gate", "up", x, True, seed, query, "h")
-            return self.pair("down", H, False, seed, query, "y")
-        return self._stack(x, seed, query)
+            return self.pair("down", H, False, seed, query, "y", fused=fused)
+        return self._stack(x, seed, query, fused)
 
-    def _stack(self, x, seed, query):
+    def forward_loss(self, x, target, seed, query):
+        """forward() and then loss(); with fuse_loss set, the last linear's pair forward and the loss pair run
+        as one launch (zoact_pair_forward_loss, two-sided only) when it qualifies.  Returns the device loss
+        vector."""
+        if self.n_queries is not None or not self.fuse_loss:
+            return self.loss(self.forward(x, seed, query), target)
+        self._loss_i ^= 1
+        Y = self.forward(x, seed, query, fused=(target, self.loss_out))
+        if Y is not None:                  # not fused: the separate loss pair (which takes the same vector)
+            self._loss_i ^= 1
+            self.loss(Y, target)
+        return self.loss_out
+
+    def _stack(self, x, seed, query, fused=None):
         T = self.T
         n_dec = len(self.linears) // (7 if self.kind == "llama" else 6)
         h = x
@@ -228,11 +258,13 @@ class ZOStep:
             if self.kind == "llama":
                 H = self.gated(f"{L}.gate", f"{L}.up", b, False, seed, query, "hmlp")
                 Hn = self._glue_rms(H, "hmlp_n")
-                h = self.pair(f"{L}.down", Hn, False, seed, query, "h" if L % 2 == 0 else "h2")
+                h = self.pair(f"{L}.down", Hn, False, seed, query, "h" if L % 2 == 0 else "h2",
+                              fused=fused if L == n_dec - 1 else None)
             else:
                 f = self.pair(f"{L}.fc1", b, False, seed, query, "f", act=Z.ACT_RELU)
                 fn = self._glue_rms(f, "f_n")
-                h = self.pair(f"{L}.fc2", fn, False, seed, query, "h" if L % 2 == 0 else "h2")
+                h = self.pair(f"{L}.fc2", fn, False, seed, query, "h" if L % 2 == 0 else "h2",
+                              fused=fused if L == n_dec - 1 else None)
         return h
 
     # ---- loss and update ----

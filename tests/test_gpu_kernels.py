@@ -497,3 +497,62 @@ def test_shared_pair_16bit_staged(ctx, gated, T, d_out, r, dt):
     err = np.abs(np64(Yv) - ref)
     assert np.all(err <= rel * np.abs(ref) + 2e-3 * np.abs(ref).max()), err.max()
     assert torch.all(Y[2 * T:] == 7.0)                                   # nothing written past the output
+
+
+@pytest.mark.parametrize("d_in,d_out,T,r,dt,act,with_target", [
+    (1024, 520, 256, 16, torch.bfloat16, zo.ACT_NONE, True),     # ragged last 16-column chunk of d_out
+    (2048, 1024, 512, 16, torch.bfloat16, zo.ACT_NONE, False),   # mean of squares
+    (1024, 264, 256, 8, torch.float16, zo.ACT_GELU, True),
+    (512, 768, 768, 4, torch.bfloat16, zo.ACT_RELU, True),
+])
+def test_pair_forward_loss_fused(ctx, d_in, d_out, T, r, dt, act, with_target):
+    # the loss pair fused into the pair forward equals the pair forward (rounded output) followed by the loss
+    # kernel, and the oracle's loss of the oracle's rounded output
+    eps, seed, query, lid = 1e-3, 13, 4, 6
+    X, W, U, C = _pair_case(d_in, d_out, r, T, False, dt, eps, 0.05, seed=110)
+    tgt = normal((T, d_out), 120, DEV, dtype=dt) if with_target else None
+    L = zo.make_layer(W, U, C, lid)
+    out = torch.zeros(4, dtype=torch.float64, device=DEV)
+    zo.zoact_pair_forward_loss(ctx, L, X, T, eps, seed, query, zo.TORCH_DT[dt], out, target=tgt, act=act)
+    Y = torch.empty(2 * T, d_out, dtype=dt, device=DEV)
+    zo.zoact_pair_forward(ctx, L, X, T, False, eps, seed, query, Y, act=act)
+    ref = torch.zeros(4, dtype=torch.float64, device=DEV)
+    zo.zoact_loss_pair(ctx, Y, T, eps, ref, target=tgt)
+    torch.cuda.synchronize()
+    assert ctx.device_status() == 0
+    o, rf = out.cpu().numpy(), ref.cpu().numpy()
+    # the exact (fp64) losses of the same rounded outputs Y. A compensated fp32 sum of n terms per thread
+    # is off by about n u^2 S (u = 2^-24: ~1e-11 for the few hundred to thousand terms a thread adds here),
+    # so even D = L+ - L- as a difference of the two sums is accurate; the loss kernel forms D directly
+    Yd = Y.double()
+    td = tgt.double() if with_target else torch.zeros(T, d_out, dtype=torch.float64, device=DEV)
+    Lp_x = ((Yd[:T] - td) ** 2).mean().item()
+    Lm_x = ((Yd[T:] - td) ** 2).mean().item()
+    D_x = ((Yd[:T] - Yd[T:]) * (Yd[:T] + Yd[T:] - 2 * td)).mean().item()
+    assert abs(o[0] - Lp_x) <= 1e-10 * Lp_x and abs(o[1] - Lm_x) <= 1e-10 * Lm_x, (o, Lp_x, Lm_x)
+    assert abs(o[2] - D_x) <= 1e-10 * max(Lp_x, Lm_x), (o[2], D_x)
+    eps32 = float(np.float32(eps))                   # eps crosses the ABI as a float
+    assert abs(o[3] - D_x / (2 * eps32)) <= 1e-10 * max(Lp_x, Lm_x) / (2 * eps32)
+    assert np.allclose(o[:2], rf[:2], rtol=1e-7, atol=0), (o, rf)
+    assert abs(rf[2] - D_x) <= 1e-7 * max(Lp_x, Lm_x), (rf[2], D_x)
+    # the oracle: its own output, rounded to the output type, then its loss pair
+    yo, _, _ = _oracle_pair(X, W, U, C, eps, T, False, seed, lid, query, d_out, r)
+    yo = {zo.ACT_NONE: lambda y: y, zo.ACT_RELU: layers.relu, zo.ACT_GELU: layers.gelu_erf}[act](yo)
+    yo = torch.from_numpy(yo).to(dt).double().numpy()
+    Lp, Lm, D, a = oloss.loss_pair(yo, T, np64(tgt) if with_target else None, eps)
+    assert abs(o[0] - Lp) <= 1e-3 * Lp and abs(o[1] - Lm) <= 1e-3 * Lm
+
+
+def test_pair_forward_loss_refusals(ctx):
+    # launches that cannot fuse are refused before any pair-forward launch (the caller falls back)
+    d_in, d_out, r, eps = 512, 256, 8, 1e-3
+    X, W, U, C = _pair_case(d_in, d_out, r, 300, False, torch.bfloat16, eps, 0.05)
+    L = zo.make_layer(W, U, C, 1)
+    P = torch.zeros(600, r, device=DEV)
+    out = torch.zeros(4, dtype=torch.float64, device=DEV)
+    n0 = ctx.launch_count()
+    for T, ydt in [(300, zo.DT_BF16), (256, zo.DT_FP32)]:
+        with pytest.raises(zo.ZoactError) as e:
+            zo.zoact_pair_forward_loss(ctx, L, X[:2 * T], T, eps, 1, 1, ydt, out, P=P[:2 * T])
+        assert e.value.status == -2
+    assert ctx.launch_count() == n0

@@ -258,3 +258,41 @@ def test_run_from_host_matches_device_steps():
         run_from_host(batches, lambda dev, i: fixed, outs)
     torch.cuda.synchronize()
     step.ctx.close()
+
+
+@pytest.mark.parametrize("name,n_dec,T", [("llama_mlp_bf16", 1, 256), ("llama_stack_bf16", 1, 256)])
+def test_forward_loss_matches_forward_then_loss(name, n_dec, T):
+    # ZOStep.forward_loss (last linear and loss pair fused) against forward() then loss(): the same losses
+    # up to summation order, and the same Adam update of C up to that
+    w = workload(name, T=T, n_decoder=n_dec)
+    step, _ = _build(w)
+    step.fuse_loss = True
+    dt = torch.bfloat16
+    x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=dt)
+    tgt = normal((w.T, w.d_model), tensor_seed(w, "t"), DEV, dtype=dt) if w.kind == "llama_mlp" else None
+    C0 = step.C.clone()
+    n0 = step.ctx.launch_count()
+    fused = step.forward_loss(x, tgt, 3, 1).clone()
+    n_fused = step.ctx.launch_count() - n0
+    step.update(1, 3, 1)
+    C1 = step.C.clone()
+    step.C.copy_(C0); step.m.zero_(); step.v.zero_()
+    n0 = step.ctx.launch_count()
+    Y = step.forward(x, 3, 1)
+    ref = step.loss(Y, tgt).clone()
+    n_ref = step.ctx.launch_count() - n0
+    step.update(1, 3, 1)
+    torch.cuda.synchronize()
+    assert step.ctx.device_status() == 0
+    assert n_fused == n_ref - 1                      # the loss kernel is gone
+    f, r = fused.cpu().numpy(), ref.cpu().numpy()
+    # both against the exact (fp64) losses of the same rounded output
+    Yd = Y.double()
+    td = tgt.double() if tgt is not None else torch.zeros_like(Yd[:w.T])
+    Lp_x, Lm_x = ((Yd[:w.T] - td) ** 2).mean().item(), ((Yd[w.T:] - td) ** 2).mean().item()
+    D_x = ((Yd[:w.T] - Yd[w.T:]) * (Yd[:w.T] + Yd[w.T:] - 2 * td)).mean().item()
+    assert abs(f[0] - Lp_x) <= 1e-10 * Lp_x and abs(f[1] - Lm_x) <= 1e-10 * Lm_x
+    assert abs(f[2] - D_x) <= 1e-10 * max(Lp_x, Lm_x)
+    assert np.allclose(r[:2], [Lp_x, Lm_x], rtol=1e-7) and abs(r[2] - D_x) <= 1e-7 * max(Lp_x, Lm_x)
+    assert torch.allclose(step.C, C1, rtol=1e-4, atol=1e-9)
+    step.ctx.close()
