@@ -37,10 +37,11 @@ EncodeTiledFn get_encode_fn() {
 
 int rank_template(int r) { return r <= 4 ? 4 : r <= 8 ? 8 : r <= 16 ? 16 : 32; }
 
-// N-tile width for a rows x n output on sm_count persistent CTAs: the width whose
-// tiles fill the last wave best (useful outputs / (waves * SMs * tile size)); ties
-// go to the wider tile, which reuses each A tile for more columns.  Widths below
-// 192 measured slower per FLOP than the wave model predicts, so they are not tried.
+// N-tile width of the one-CTA kernel for a rows x n output on sm_count persistent
+// CTAs: the width whose tiles fill the last wave best (useful outputs / (waves *
+// SMs * tile size)); ties go to the wider tile, which reuses each A tile for more
+// columns.  Widths below 192 measured slower per FLOP than this model predicts, so
+// they are not tried.  (CTA pairs always take 256: see launch_pair_tc.)
 int choose_bn(int64_t rows, int64_t n, int sm_count, int bm = pairtc::BM) {
   static const int cand[] = {256, 224, 192};
   const int64_t num_m = (rows + bm - 1) / bm;
@@ -175,9 +176,10 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   // CTA pairs (256-row tiles) once there are enough rows to fill them; INT4 in-kernel dequant stays on one CTA
   const char* sel = std::getenv("ZOACT_PAIR_KERNEL");
   const bool two = !w4 && a.rows >= 2 * BM && !(sel && std::strcmp(sel, "1cta") == 0);
-  const int bn = (gated || w4) ? BN
-                               : (two ? choose_bn(a.rows, a.d_out, ctx->sm_count / 2, 2 * BM)
-                                      : choose_bn(a.rows, a.d_out, ctx->sm_count));
+  // CTA pairs: always 256-wide tiles.  A 256 x bn x 16 MMA measured the same time for bn = 192, 224 and 256, so
+  // a tile costs the same at any of these widths and the widest needs the fewest waves (the Llama-3-8B MLP step:
+  // 0.645 ms at 256 and at 224, 0.709 at 192; the OPT stack: 145.7 ms at 256, 149.1 at 224).
+  const int bn = (gated || w4 || two) ? BN : choose_bn(a.rows, a.d_out, ctx->sm_count);
   const int b_box = gated ? BN / 2 : (two ? bn / 2 : bn);
   if (w4) {
     tm.b = tm.b2 = tm.a;                 // W arrives through the dequantising warps, not TMA
