@@ -36,6 +36,8 @@ enum ScratchSlot {
   SLOT_PROJ_TICKETS, // split-K tickets of the tensor-core projection (zero between calls)
   SLOT_DIAG,         // partial products of the subspace diagnostics
   SLOT_STACKED_X,    // a shared input and its projection copied once per evaluation block (ranks above 32)
+  SLOT_SK_PART,      // partial accumulators of the CTA-pair kernel's split tail
+  SLOT_SK_TICKETS,   // its per-tile tickets (zero between launches)
   SLOT_COUNT
 };
 

@@ -338,6 +338,26 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   for (int b = 0; b < ZOACT_MAX_EVAL_BLOCKS; ++b) p.zq[b] = b < a.nb ? zq_of[b] : -1;
   auto al16 = [](const void* q) { return q == nullptr || ((uintptr_t)q & 15u) == 0; };
   p.vec_ok = al16(a.C) && al16(a.C2) && al16(a.P) && al16(a.P2);
+  // Split tail: when the last wave of whole tiles would leave at least half of the pairs idle, each of its tiles
+  // is cut into S = pairs / tail-tiles (<= 4) equal K ranges, one per pair, and the last piece of a tile to finish
+  // adds the partials; the tail then takes 1/S of a tile's time.  ZOACT_SPLIT_TAIL=0 keeps whole tiles.
+  const char* sksel = std::getenv("ZOACT_SPLIT_TAIL");
+  if (two && ctx->may_allocate && !(sksel && sksel[0] == '0')) {
+    const int pairs = ctx->sm_count / 2;
+    const int rem = p.num_tiles % pairs;
+    const int total_k = p.num_k + p.aug_kb;
+    int split = rem > 0 ? pairs / rem : 0;
+    if (split > 4) split = 4;
+    if (split >= 2 && total_k / split >= 4) {
+      p.sk_first = p.num_tiles - rem;
+      p.sk_tiles = rem;
+      p.sk_split = split;
+      p.sk_part = static_cast<float*>(scratch(ctx, SLOT_SK_PART, (size_t)pairs * 2 * BM * BN * sizeof(float)));
+      p.sk_ticket =
+          static_cast<unsigned int*>(scratch_zeroed(ctx, SLOT_SK_TICKETS, (size_t)pairs * 2 * sizeof(unsigned)));
+      if (!p.sk_part || !p.sk_ticket) return ZOACT_ERR_NOMEM;
+    }
+  }
   p.status = ctx->d_status;
   const int mode = gated ? MODE_GATED : MODE_PAIR;
   if (w4) {

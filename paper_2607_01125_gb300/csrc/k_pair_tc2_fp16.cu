@@ -8,7 +8,8 @@ template <typename TO, int RT, int MODE, int SMODE = STAGE_NONE>
 static int launch_two(Ctx* ctx, const TmaSet& tm, const Params& p) {
   auto kern = pair_tc2_kernel<TO, RT, MODE, 0, SMODE>;
   ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES));
-  const int clusters = p.num_tiles < ctx->sm_count / 2 ? p.num_tiles : ctx->sm_count / 2;
+  // every pair when the tail is split (its pieces are laid out over all of them)
+  const int clusters = p.sk_tiles > 0 || p.num_tiles >= ctx->sm_count / 2 ? ctx->sm_count / 2 : p.num_tiles;
   ZOACT_CUDA_TRY(launch_pdl(ctx, kern, dim3(2 * clusters), dim3(num_threads(false)), SMEM2_BYTES, tm, p));
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();

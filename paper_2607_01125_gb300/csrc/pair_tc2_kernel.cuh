@@ -48,6 +48,7 @@ struct SharedState2 {
   uint32_t tmem_base;
   int abort_flag;
   int epi_ok;
+  int sk_last;            // split tail: this CTA's piece was the tile's last to finish
 };
 static_assert(sizeof(SharedState2) <= 256, "barrier block outgrew its shared-memory slot");
 static_assert(SMEM2_BYTES <= 232448, "dynamic shared memory above the 227 KB a CTA may use");
@@ -732,6 +733,103 @@ __device__ __forceinline__ void loss_finish(const Params& prm, const CompSum* ac
 // region holds the Z tables and two smaller buffers.  A launch that does not
 // match its SMODE records ZOACT_ERR_INVALID_ARG and exits before touching
 // shared memory.
+// One unit of a pair's work: K-blocks [kb0, kb1) of a tile.  Whole tiles have
+// npieces = 1; a piece of a split tail tile is piece `piece` (in K order) of
+// `npieces` and keeps its partial accumulator in slot `slot`.
+struct WorkUnit {
+  int tile, kb0, kb1, piece, npieces, slot;
+};
+
+// The i-th unit of cluster c: whole tiles c, c + n, ... below sk_first (all tiles
+// without a split tail), then at most one tail piece: pair c = j * sk_tiles + t
+// takes K range j of tail tile t, so the pieces running side by side cover the
+// same K range of neighbouring tiles and share operand panels in L2 as a wave of
+// whole tiles does.  False past the last unit.  The producer, the MMA issuer and
+// the epilogue walk the same sequence.
+__device__ __forceinline__ bool next_unit(const Params& prm, int c, int n, int K, int i, WorkUnit& u) {
+  const int lim = prm.sk_tiles > 0 ? prm.sk_first : prm.num_tiles;
+  const int whole = c < lim ? (lim - c + n - 1) / n : 0;
+  if (i < whole) {
+    u.tile = c + i * n; u.kb0 = 0; u.kb1 = K; u.piece = 0; u.npieces = 1; u.slot = -1;
+    return true;
+  }
+  if (prm.sk_tiles == 0 || i != whole || c >= prm.sk_tiles * prm.sk_split) return false;
+  const int j = c / prm.sk_tiles, t = c - j * prm.sk_tiles;
+  u.tile = prm.sk_first + t;
+  u.kb0 = (int)((int64_t)j * K / prm.sk_split);
+  u.kb1 = (int)((int64_t)(j + 1) * K / prm.sk_split);
+  u.piece = j; u.npieces = prm.sk_split; u.slot = c;
+  return true;
+}
+
+// A tail piece: the accumulator holds only this piece's K-blocks.  Every piece
+// stores its fp32 partial (this CTA's 128 rows x bn columns) in its slot and
+// takes a ticket of the tile; the piece that arrives last adds all pieces'
+// partials in K order -- its own from TMEM -- and writes the sum back to TMEM,
+// where the epilogue finds the whole accumulator.  No CTA waits for another, and
+// the fixed order makes the sum independent of which piece ends last.  Returns
+// whether this piece was the last.  Slot layout: element (row, col) at float4
+// (col / 4) * BM + row, so a warp's 32 rows are 512 contiguous bytes.
+__device__ __forceinline__ bool sk_fixup(const Params& prm, SharedState2* ss, const WorkUnit& u, int etid, int half,
+                                         int row, uint32_t t_row, int bn, uint32_t rank) {
+  constexpr size_t SLOT_F4 = (size_t)BM * BN / 4;
+  const int wcols = bn / 2, cb = half * wcols;
+  float4* own = reinterpret_cast<float4*>(prm.sk_part) + (size_t)(2 * u.slot + (int)rank) * SLOT_F4;
+  for (int p = 0; p < wcols; p += 16) {
+    float v[16];
+    tc::tmem_ld16(t_row + (uint32_t)(cb + p), v);
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      __stcg(own + (size_t)((cb + p) / 4 + q) * BM + row,
+             make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
+  }
+  __threadfence();
+  tc::named_bar_sync(3, EPI_THREADS);
+  const int t = u.tile - prm.sk_first;
+  if (etid == 0) {
+    unsigned int* tk = prm.sk_ticket + 2 * t + (int)rank;
+    const bool last = atomicAdd(tk, 1u) == (unsigned int)(u.npieces - 1);
+    if (last) atomicExch(tk, 0u);                   // every piece has arrived: zero for the next launch
+    ss->sk_last = last ? 1 : 0;
+  }
+  tc::named_bar_sync(3, EPI_THREADS);
+  const bool last = *reinterpret_cast<volatile int*>(&ss->sk_last) != 0;
+  if (!last) return false;
+  __threadfence();
+  // piece j of tail tile t is pair j * sk_tiles + t's; each 16-column chunk adds the pieces in K order, the
+  // four loads of one piece in flight together (few registers beside the epilogue's)
+  const float4* base = reinterpret_cast<const float4*>(prm.sk_part) + (size_t)rank * SLOT_F4;
+  for (int p = 0; p < wcols; p += 16) {
+    float sum[16];
+    tc::tmem_ld16(t_row + (uint32_t)(cb + p), sum);     // this piece's own partial, used at its place below
+    float mine[16];
+#pragma unroll
+    for (int e = 0; e < 16; ++e) mine[e] = sum[e];
+#pragma unroll 1
+    for (int j = 0; j < u.npieces; ++j) {
+      float v[16];
+      if (j == u.piece) {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) v[e] = mine[e];
+      } else {
+        const float4* src = base + (size_t)(2 * (j * prm.sk_tiles + t)) * SLOT_F4 + (size_t)((cb + p) / 4) * BM + row;
+        float4 x[4];
+#pragma unroll
+        for (int qq = 0; qq < 4; ++qq) x[qq] = __ldcg(src + (size_t)qq * BM);
+#pragma unroll
+        for (int qq = 0; qq < 4; ++qq) {
+          v[4 * qq] = x[qq].x; v[4 * qq + 1] = x[qq].y; v[4 * qq + 2] = x[qq].z; v[4 * qq + 3] = x[qq].w;
+        }
+      }
+#pragma unroll
+      for (int e = 0; e < 16; ++e) sum[e] = j == 0 ? v[e] : sum[e] + v[e];
+    }
+    tc::tmem_st16(t_row + (uint32_t)(cb + p), sum);
+  }
+  tc::tmem_wait_st();
+  return true;
+}
+
 template <typename TO, int RT, int MODE, int AB_BF16, int SMODE = STAGE_NONE>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(num_threads(false), 1)
 pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
@@ -809,10 +907,11 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
-      for (int tile = cluster_id; tile < prm.num_tiles && ok; tile += n_clusters) {
+      WorkUnit u;
+      for (int i = 0; ok && next_unit(prm, cluster_id, n_clusters, total_k, i, u); ++i) {
         int m_blk, n_blk;
-        tile_coords(tile, num_m, num_n, m_blk, n_blk);
-        for (int kb = 0; kb < total_k; ++kb) {
+        tile_coords(u.tile, num_m, num_n, m_blk, n_blk);
+        for (int kb = u.kb0; kb < u.kb1; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
           const uint32_t full_leader = tc2::map_to(tc::smem_u32(&ss->full[stage]), 0);
           tc2::arrive_expect_tx_cluster(full_leader, stage_tx);
@@ -847,13 +946,14 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       bool ok = true;
       int local = 0;
       bool issued_any = false;
-      for (int tile = cluster_id; tile < prm.num_tiles && ok; tile += n_clusters, ++local) {
+      WorkUnit u;
+      for (int i = 0; ok && next_unit(prm, cluster_id, n_clusters, total_k, i, u); ++i, ++local) {
         const int buf = local & 1;
         const uint32_t acc_phase = (local >> 1) & 1;
         if (!tc::mbar_wait(tc::smem_u32(&ss->tmem_empty[buf]), acc_phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
         tc::tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
-        for (int kb = 0; kb < total_k; ++kb) {
+        for (int kb = u.kb0; kb < u.kb1; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->full[stage]), phase, abort_flag, prm.status)) { ok = false; break; }
           tc::tc_fence_after();
           const uint32_t sa = tc::smem_u32(smem + stage * STAGE2_BYTES);
@@ -862,7 +962,7 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             tc2::mma2_f16(d_tmem, tc::sdesc_k_sw128(sa + k * 32), tc::sdesc_k_sw128(sb + k * 32), idesc,
-                          (kb | k) != 0 ? 1u : 0u);
+                          (kb != u.kb0 || k != 0) ? 1u : 0u);
           tc2::commit2_both(tc::smem_u32(&ss->empty[stage]));    // frees the stage in both CTAs
           issued_any = true;
           if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
@@ -888,17 +988,30 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
     uint32_t tphase = 0;                    // fused loss: parity of this warpgroup's next target load
     CompSum lacc[2];                        // fused loss: running sums of the + and - rows
     bool aborted = false;
-    for (int tile = cluster_id; tile < prm.num_tiles; tile += n_clusters, ++local) {
+    WorkUnit u;
+    for (int i = 0; next_unit(prm, cluster_id, n_clusters, total_k, i, u); ++i, ++local) {
       int m_blk, n_blk;
-      tile_coords(tile, num_m, num_n, m_blk, n_blk);
+      tile_coords(u.tile, num_m, num_n, m_blk, n_blk);
       const int buf = local & 1;
       const uint32_t acc_phase = (local >> 1) & 1;
       const int64_t row0 = (int64_t)m_blk * BM2 + (int64_t)rank * BM;
       const int64_t m = row0 + row_in_tile;
       const bool row_ok = m < prm.rows;
       const uint32_t t_row = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(buf * BN);
-      bool ok;
-      if constexpr (SMODE == STAGE_ALL)
+      bool ok = true;
+      bool epi = true;
+      if (u.npieces > 1) {
+        // a tail piece: only the last one to finish runs the epilogue, on the summed accumulator
+        ok = epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid);
+        if (ok) {
+          epi = sk_fixup(prm, ss, u, etid, half, row_in_tile, t_row, bn, rank);
+          tc::tc_fence_before();
+          tc::named_bar_sync(3, EPI_THREADS);       // the summed accumulator is in TMEM for every warp
+          tc::tc_fence_after();
+        }
+      }
+      if (!ok || !epi) {
+      } else if constexpr (SMODE == STAGE_ALL)
         ok = epi_all_staged<TO, MODE>(prm, tm, ss, reinterpret_cast<uint8_t*>(tbl), etid, half, row_in_tile, row0,
                                       n_blk, bn, buf, acc_phase, t_row, abort_flag, pending);
       else if constexpr (SMODE == STAGE_MIRROR)

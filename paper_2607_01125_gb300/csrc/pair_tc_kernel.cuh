@@ -144,6 +144,12 @@ struct Params {
   double* loss_part;
   unsigned int* loss_ticket;
   double* loss_out;
+  // split tail (CTA-pair kernel): tiles [sk_first, sk_first + sk_tiles) are each cut into sk_split equal
+  // K ranges, one per pair (sk_tiles = 0: every tile whole); sk_part holds one 128 x BN fp32 partial
+  // accumulator per pair and CTA, sk_ticket one counter per tail tile and CTA (zero between launches)
+  int sk_first, sk_tiles, sk_split;
+  float* sk_part;
+  unsigned int* sk_ticket;
 };
 
 struct SharedState {

@@ -260,6 +260,59 @@ def test_pair_forward_gated(ctx, T, shared, dt):
     assert np.abs(np64(H) - ref).max() <= 1e-4 * np.abs(ref).max()
 
 
+
+# ---------------- split tail of the CTA-pair kernel ----------------
+# With 152 SMs (76 CTA pairs), when the last wave of whole tiles leaves half of the pairs or more idle, its tiles
+# are each cut into S = 76 / tail-tiles (<= 4) equal K ranges and the last piece of each adds the partials.
+# Cases:
+# - 600 stacked rows x 520 outputs: 9 tiles, S = 4;
+# - 512 x 256: two tiles, S = 4;
+# - a gated launch on a shared input with 16-bit staged outputs (the MLP block's gate/up form): 10 tiles, S = 4;
+# - 4096 stacked rows x 4096 (the MLP block's down form, K = 1024): three waves of 76 whole tiles, then 28 tail
+#   tiles in two pieces.
+@pytest.mark.parametrize("d_in,d_out,r,T,shared,gated,ydt", [
+    (1024, 520, 16, 300, False, False, torch.float32),
+    (1024, 256, 8, 256, False, False, torch.float32),
+    (1024, 520, 16, 300, True, True, torch.bfloat16),
+    (1024, 4096, 16, 2048, False, False, torch.float32),
+])
+def test_pair_forward_split_tail(ctx, monkeypatch, d_in, d_out, r, T, shared, gated, ydt):
+    eps, seed, query = 0.5, 13, 2
+    X, W, U, C = _pair_case(d_in, d_out, r, T, shared, torch.bfloat16, eps, 0.3, seed=40)
+    L = zo.make_layer(W, U, C, 3)
+    if gated:
+        W2 = normal((d_out, d_in), 51, DEV, std=d_in ** -0.5, dtype=torch.bfloat16)
+        C2 = normal((d_out * r,), 52, DEV, std=0.3)
+        L2 = zo.make_layer(W2, U, C2, 4)           # one basis for gate and up, as the MLP block's
+    def run():
+        Y = torch.empty(2 * T, d_out, dtype=ydt, device=DEV)
+        if gated:
+            zo.zoact_pair_forward_gated(ctx, L, L2, X, T, shared, eps, seed, query, Y)
+        else:
+            zo.zoact_pair_forward(ctx, L, X, T, shared, eps, seed, query, Y)
+        torch.cuda.synchronize()
+        assert ctx.device_status() == 0
+        return Y
+    Y1, Y2 = run(), run()
+    assert torch.equal(Y1, Y2)                     # the fixed piece order makes the sum reproducible
+    monkeypatch.setenv("ZOACT_SPLIT_TAIL", "0")
+    Yw = run()                                     # whole tiles: the same sums in another order
+    monkeypatch.delenv("ZOACT_SPLIT_TAIL")
+    assert torch.equal(run(), Y1)                  # the tickets were left at zero
+    if gated:
+        g, _, _ = _oracle_pair(X, W, U, C, eps, T, shared, seed, 3, query, d_out, r)
+        u, _, _ = _oracle_pair(X, W2, U, C2, eps, T, shared, seed, 4, query, d_out, r)
+        ref = layers.silu(g) * u
+        tol = 2.0 ** -7 * np.abs(ref) + 1e-3 * np.abs(ref).max()
+        assert np.all(np.abs(np64(Y1) - ref) <= tol)
+        # one bf16 step, or the fp32 summation-order difference where SiLU(g) u is near zero
+        assert np.all(np.abs(np64(Y1) - np64(Yw)) <= 2.0 ** -7 * np.abs(np64(Yw)) + 1e-4 * np.abs(ref).max())
+    else:
+        ref, absb, lrabs = _oracle_pair(X, W, U, C, eps, T, shared, seed, 3, query, d_out, r)
+        assert np.all(np.abs(np64(Y1) - ref) <= _bound(d_in, absb, lrabs))
+        assert np.all(np.abs(np64(Y1) - np64(Yw)) <= 2 * 8 * np.sqrt(d_in) * 2.0 ** -24 * absb + 1e-6)
+
+
 # ---------------- INT4 weights ----------------
 def _int4_layer(d_in, d_out, r, seed, lid):
     Wf = normal((d_out, d_in), seed, DEV, std=0.02)
