@@ -62,7 +62,9 @@ class ClockSampler:
     def __init__(self, index):
         self.index = index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_gpu{index}.csv")
+        # the raw samples; BENCH_CLOCKS_DIR moves them (the JSON line carries their summary)
+        self.path = os.path.join(os.environ.get("BENCH_CLOCKS_DIR", os.path.join(ROOT, "bench_clocks")),
+                                 f"clocks_gpu{index}.csv")
 
     def start(self):
         os.makedirs(os.path.dirname(self.path), exist_ok=True)
