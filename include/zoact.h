@@ -111,8 +111,20 @@ int zoact_set_stream(zoact_ctx* ctx, void* stream);
 const char* zoact_status_string(int status);
 
 /* Synchronise the stream and read the device status word (ZOACT_OK or the
- * first device-side error recorded since the last reset).  reset != 0 clears it. */
+ * first device-side error recorded since the last reset).  reset != 0 clears it.
+ * On ZOACT_ERR_TIMEOUT the outputs of the launches since the last read are
+ * undefined; the context's grid-reduction tickets are zeroed here, so the
+ * context serves later calls normally.                                          */
 int zoact_get_device_status(zoact_ctx* ctx, int* status, int reset);
+
+/* Failure-detection test hook: one kernel that leaves every ticket of the
+ * context part-counted (as a launch that gave up can), then waits for a device
+ * flag that nothing sets, for at most wait_ns nanoseconds (0 < wait_ns <= 1e9),
+ * and records ZOACT_ERR_TIMEOUT in the device status word.  It shows that a
+ * bounded wait ends with a readable status and that zoact_get_device_status
+ * repairs the tickets; nothing faults or traps.  Returns ZOACT_ERR_INVALID_ARG
+ * for a wait_ns outside that range.                                              */
+int zoact_debug_timeout(zoact_ctx* ctx, int64_t wait_ns);
 
 /* Number of SMs of the context's device (host query, no launch).               */
 int zoact_device_sm_count(zoact_ctx* ctx, int* sm_count);

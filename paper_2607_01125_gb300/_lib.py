@@ -37,7 +37,7 @@ EXPORTS = [
     "zoact_rms_norm", "zoact_mix_rms", "zoact_multi_forward", "zoact_multi_forward_gated", "zoact_loss_multi",
     "zoact_adam_step_multi", "zoact_sgd_step_multi", "zoact_basis_prepared_bytes", "zoact_basis_prepare",
     "zoact_lowrank_proj_prepared", "zoact_subspace_overlap", "zoact_gradient_energy", "zoact_kernel_timing",
-    "zoact_kernel_time", "zoact_pair_forward_loss",
+    "zoact_kernel_time", "zoact_pair_forward_loss", "zoact_debug_timeout",
 ]
 
 
@@ -99,6 +99,7 @@ def load():
         "zoact_get_device_status": [P, ctypes.POINTER(ctypes.c_int), I32],
         "zoact_device_sm_count": [P, ctypes.POINTER(ctypes.c_int)],
         "zoact_get_launch_count": [P, ctypes.POINTER(ctypes.c_int64)],
+        "zoact_debug_timeout": [P, I64],
         "zoact_philox_normals": [P, U64, U32, U64, I64, P, P],
         "zoact_lowrank_proj": [P, P, I32, I64, I32, P, I32, P],
         "zoact_pair_forward": [P, ctypes.POINTER(zoact_layer), P, I32, I64, I32, P, F32, U64, U64, I32, P, I32],
@@ -200,6 +201,10 @@ class Context:
         ms, n = ctypes.c_double(), ctypes.c_int64()
         _check("zoact_kernel_time", load().zoact_kernel_time(self.handle, ctypes.byref(ms), ctypes.byref(n)))
         return ms.value, n.value
+
+    def debug_timeout(self, wait_ns):
+        """Failure-detection test hook (see zoact_debug_timeout): a bounded wait that runs out."""
+        _check("zoact_debug_timeout", load().zoact_debug_timeout(self.handle, int(wait_ns)))
 
     def device_status(self, reset=True):
         v = ctypes.c_int()

@@ -188,3 +188,32 @@ def test_maximum_size_sampled(ctx):
     assert np.all(np.abs(got - ref) <= 2.0 ** -7 * np.abs(ref) + 2e-3 * np.abs(ref).max())
     del X, Y
     torch.cuda.empty_cache()
+
+
+def test_bounded_wait_timeout_is_reported_and_the_context_recovers(ctx):
+    # a bounded wait that runs out (a flag that nothing sets, 1 ms) ends with ZOACT_ERR_TIMEOUT in the status
+    # word, not a hang or a trap; the hook also leaves the context's tickets part-counted, as a launch that gave up
+    # can, and reading the status repairs them: a split-tail pair forward (600 stacked rows x 520 outputs: 9 tiles
+    # in 4 pieces) and a loss pair give the same bits before and after
+    d_in, d_out, r, T = 1024, 520, 16, 300
+    X, W, U, C = _pair_case(d_in, d_out, r, T, False, torch.bfloat16, 0.5, 0.3, seed=60)
+    L = zo.make_layer(W, U, C, 2)
+
+    def run():
+        Y = torch.empty(2 * T, d_out, dtype=torch.bfloat16, device=DEV)
+        zo.zoact_pair_forward(ctx, L, X, T, False, 0.5, 3, 1, Y)
+        out = torch.zeros(4, dtype=torch.float64, device=DEV)
+        zo.zoact_loss_pair(ctx, Y, T, 0.5, out)
+        torch.cuda.synchronize()
+        return Y, out
+
+    Y0, l0 = run()
+    assert ctx.device_status() == 0
+    with pytest.raises(zo.ZoactError):
+        ctx.debug_timeout(0)                     # outside (0, 1e9]: refused on the host
+    ctx.debug_timeout(1_000_000)
+    assert ctx.device_status() == -5             # ZOACT_ERR_TIMEOUT, read and reset; tickets zeroed
+    assert ctx.device_status() == 0
+    Y1, l1 = run()
+    assert ctx.device_status() == 0
+    assert torch.equal(Y0, Y1) and torch.equal(l0, l1)
