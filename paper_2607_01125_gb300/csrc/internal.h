@@ -33,7 +33,6 @@ enum ScratchSlot {
   SLOT_AUG_A,        // 16-bit split of the projection P (extra K columns of the tensor-core pair forward)
   SLOT_AUG_B,        // 16-bit split of C (+ c_b Z_b) for those K columns (gate and up)
   SLOT_AUG_Z,        // Z of each query, transposed, for the epilogue (C on the tensor cores)
-  SLOT_PROJ_TICKETS, // split-K tickets of the tensor-core projection (zero between calls)
   SLOT_DIAG,         // partial products of the subspace diagnostics
   SLOT_STACKED_X,    // a shared input and its projection copied once per evaluation block (ranks above 32)
   SLOT_SK_PART,      // partial accumulators of the CTA-pair kernel's split tail
