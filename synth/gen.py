@@ -59,10 +59,11 @@ def lowrank_activations(n_tok, d, rank, noise, seed, device="cpu", dtype=torch.b
 
 
 def decaying_spectrum_activations(n_tok, d, rank, noise, seed, device="cpu", dtype=torch.float16):
-    """Tokens whose top `rank` singular values decay as i^-1, plus isotropic noise.
+    """Tokens with a rank-`rank` signal whose singular values decay as i^-1, plus isotropic noise.
 
     x = A diag(1/i) B + noise * N(0,1), A ~ N(0,1)^{n_tok x rank},
-    B = orthonormal rows (QR of a Gaussian), then unit RMS per token.
+    B = orthonormal rows (QR of a Gaussian), then unit RMS per token (which
+    flattens the 1/i decay somewhat: tokens led by the first direction shrink most).
     """
     g = _gen(seed, device)
     B = torch.linalg.qr(torch.randn(d, rank, generator=g, device=device))[0].T.contiguous()  # [rank, d]
