@@ -268,10 +268,12 @@ int zoact_pair_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoac
  * pair forward's epilogue without writing Y.  X [2T, d_in] stacked (+ rows then
  * - rows), target [T, d_out] of ydtype (16-byte aligned) or NULL for the mean
  * square loss, out[4] = {L+, L-, D, a} fp64 in DEVICE memory, D = L+ - L- (the
- * difference of the two sums, each over T * d_out rounded outputs; fp64 partials
- * of compensated fp32 sums), a = D / (2 eps).  Qualifies: two-sided stacked rows,
- * T a multiple of 256, 16-bit ydtype, the CTA-pair tensor-core path with the whole
- * low-rank term on the MMA; otherwise ZOACT_ERR_UNSUPPORTED is returned before
+ * difference of the two sums, each over T * d_out rounded outputs; every square
+ * split exactly into two fp32 terms, compensated fp32 sums, fp64 partials: L+ and
+ * L- within ~1e-11 relative of their exact values), a = D / (2 eps).  Qualifies:
+ * two-sided stacked rows, T a multiple of 256, 16-bit ydtype, the CTA-pair
+ * tensor-core path with the whole low-rank term on the MMA; otherwise
+ * ZOACT_ERR_UNSUPPORTED is returned before
  * any launch of the pair forward itself (a projection U^T x, when P is NULL, may
  * already have run) and the caller uses zoact_pair_forward + zoact_loss_pair.
  * T = 0 writes nothing.  A non-finite result sets ZOACT_ERR_NONFINITE; a launch
