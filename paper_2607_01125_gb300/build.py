@@ -2,9 +2,12 @@
 
 Every .cu under csrc/ is compiled in parallel into _build/ and linked into
 paper_2607_01125_gb300/libzoact.so.  A rebuild happens only when a source or
-header is newer than the library.  Usage: ``python -m paper_2607_01125_gb300.build``.
+header is newer than the library.  Processes that build at the same time (the
+ranks of one torchrun job) take turns on a file lock, and each re-checks the
+library once it holds the lock.  Usage: ``python -m paper_2607_01125_gb300.build``.
 """
 import concurrent.futures as cf
+import fcntl
 import glob
 import os
 import shutil
@@ -48,8 +51,19 @@ def build(force=False, verbose=False, jobs=None):
     """Compile and link libzoact.so; returns its path."""
     if not force and up_to_date():
         return LIB
-    nvcc = _nvcc()
     os.makedirs(BUILD, exist_ok=True)
+    with open(os.path.join(BUILD, ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        try:
+            if not force and up_to_date():        # another process built it while this one waited
+                return LIB
+            return _build_locked(verbose, jobs)
+        finally:
+            fcntl.flock(lock, fcntl.LOCK_UN)
+
+
+def _build_locked(verbose, jobs):
+    nvcc = _nvcc()
     srcs = _sources()
 
     def compile_one(src):
@@ -65,7 +79,7 @@ def build(force=False, verbose=False, jobs=None):
     jobs = jobs or max(1, min(len(srcs), os.cpu_count() or 4))
     with cf.ThreadPoolExecutor(max_workers=jobs) as ex:
         objs = list(ex.map(compile_one, srcs))
-    tmp = LIB + ".tmp"
+    tmp = f"{LIB}.{os.getpid()}.tmp"
     cmd = [nvcc, "-shared", "-Xcompiler", "-fPIC"] + ARCH + objs + ["-o", tmp]
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
