@@ -121,8 +121,9 @@ def dist_setup():
 def build(ctx, dev, rank, name, tokens=None, n_queries=None, r=None):
     """Weights, bases (Algorithm 1 on the device) and the ZOStep of a workload.
 
-    Returns (step, x, target, basis_seconds, workload).  Weights are the same on every
-    rank; the calibration and training tokens and the targets are drawn per rank.
+    Returns (step, x, target, basis_seconds, workload).  Weights and calibration tokens, hence the bases,
+    are the same on every rank; the training tokens (in the calibration set's signal subspace) and the
+    targets are drawn per rank.
     """
     import torch
     import paper_2607_01125_gb300 as zo
@@ -150,9 +151,8 @@ def build(ctx, dev, rank, name, tokens=None, n_queries=None, r=None):
             W = normal((s.d_out, s.d_in), tensor_seed(w, "W", s.name), dev, std=w.weight_std, dtype=dt)
             lins.append(AdaptedLinear(s.name, W, U, s.layer_id, off, w.r))
     n_cal = N_CAL[name]
-    x_all, _ = lowrank_activations(n_cal + w.T, w.d_model, 64, 0.05, tensor_seed(w, "x", rank), dev, dtype=dt)
-    x_cal, x = x_all[:n_cal].contiguous(), x_all[n_cal:].contiguous()
-    del x_all
+    x_cal, B = lowrank_activations(n_cal, w.d_model, 64, 0.05, tensor_seed(w, "x"), dev, dtype=dt)
+    x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x", rank), dev, dtype=dt, basis=B)
     target = normal((w.T, w.d_model), tensor_seed(w, "target", rank), dev, dtype=dt) if w.kind == "llama_mlp" else None
     # Algorithm 1: calibration forward pass of the base model, one basis per layer input
     step_cal = ZOStep(ctx, w.kind, lins, n_cal, w.act_dtype, eps=w.eps)
