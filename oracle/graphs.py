@@ -69,15 +69,21 @@ def llama_mlp_forward(layers, x, eps, seed, query, store="bf16", blocks=None):
 
 
 def stack_forward(decoder_layers, x, eps, seed, query, kind, store="bf16",
-                  n_heads=32, n_kv_heads=8, head_dim=128, blocks=None):
+                  n_heads=32, n_kv_heads=8, head_dim=128, blocks=None, first=True):
     """Linear stack of the llama / opt kind.  decoder_layers: list of dicts of layers.
 
     llama dict keys: q k v o gate up down;  opt dict keys: q k v o fc1 fc2.
+
+    first=True: x [T, d] is the graph input, the same for every evaluation
+    point.  first=False continues a stack from a later decoder: x is the stacked
+    output [n_points * T, d] of the decoders before it (so a deep stack can be
+    run one decoder at a time, with one decoder's weights in memory).
     """
     rnd = STORE_ROUNDING[store]
-    T = x.shape[0]
+    n_points = 2 if blocks is None else len(blocks)
+    T = x.shape[0] if first else x.shape[0] // n_points
     h = np.asarray(x, np.float64)
-    shared = True
+    shared = first
     for dl in decoder_layers:
         a = rnd(rms_norm(h))
         q = rnd(layer_forward(dl["q"], a, eps, seed, query, T, shared, blocks))

@@ -20,6 +20,7 @@ rows [T, 2T) hold sigma = -1.
 All arithmetic is fp64 on values read exactly from their stored precision.
 """
 import numpy as np
+import torch
 from scipy.special import erf
 
 
@@ -89,17 +90,18 @@ def dequant_int4_g128(packed, scales, d_in):
     even k and high nibble for odd k, each nibble a 4-bit two's complement
     integer q in [-8, 7]; scales [d_out, d_in/128] (fp16 values); w = q * s.
     """
-    packed = np.asarray(packed, dtype=np.uint8)
-    d_out = packed.shape[0]
-    lo = (packed & 0x0F).astype(np.int64)
-    hi = (packed >> 4).astype(np.int64)
-    q = np.empty((d_out, d_in), dtype=np.int64)
-    q[:, 0::2] = lo[:, : (d_in + 1) // 2]
-    q[:, 1::2] = hi[:, : d_in // 2]
-    q = np.where(q >= 8, q - 16, q)                       # two's complement nibble
-    s = np.asarray(scales, dtype=np.float64)
-    s_full = np.repeat(s, 128, axis=1)[:, :d_in]
-    return q.astype(np.float64) * s_full
+    # plain torch CPU element-wise ops (multi-threaded): a full Llama-3-8B stack has 7e9 weights
+    pk = torch.from_numpy(np.ascontiguousarray(packed, dtype=np.uint8))
+    d_out = pk.shape[0]
+    # byte k/2 -> (low nibble, high nibble) = elements (k, k + 1)
+    q = torch.stack([pk & 0x0F, pk >> 4], dim=-1).reshape(d_out, -1)[:, :d_in].to(torch.int8)
+    q = torch.where(q >= 8, q - 16, q)                    # two's complement nibble
+    n_groups = (d_in + 127) // 128
+    w = torch.zeros(d_out, n_groups * 128, dtype=torch.float64)
+    w[:, :d_in] = q
+    s = torch.from_numpy(np.asarray(scales, dtype=np.float64))[:, :n_groups]
+    w.view(d_out, n_groups, 128).mul_(s[:, :, None])      # every element of group g times s[g]
+    return w[:, :d_in].numpy()
 
 
 # ---- glue ops of the synthetic graphs (exact definitions, fp64) ----

@@ -99,3 +99,23 @@ def test_stack_graph(kind):
                                                n_heads=4, n_kv_heads=2, head_dim=4)
     # ReLU is not smooth: keep eps small enough that no pre-activation changes sign
     _check_rate(fwd, tl, lays, x, None, eps_list=(2e-2, 1e-2, 5e-3) if kind == "llama" else (2e-3, 1e-3, 5e-4))
+
+
+@pytest.mark.parametrize("kind,blocks", [("llama", None), ("opt", None), ("llama", [(0.0, 0), (0.3, 1), (0.3, 2)])])
+def test_stack_one_decoder_at_a_time(kind, blocks):
+    # a deep stack run decoder by decoder (first=False after the first) gives the same array as one call
+    rng = np.random.default_rng(2)
+    d, f, r, T, nl = 16, 24, 2, 5, 3
+    kvd = 8 if kind == "llama" else d
+    names = ["q", "k", "v", "o", "gate", "up", "down"] if kind == "llama" else ["q", "k", "v", "o", "fc1", "fc2"]
+    dims = {"q": (d, d), "k": (d, kvd), "v": (d, kvd), "o": (d, d), "gate": (d, f), "up": (d, f),
+            "down": (f, d), "fc1": (d, f), "fc2": (f, d)}
+    dls = [{nm: _layer(rng, *dims[nm], r, L * len(names) + i) for i, nm in enumerate(names)} for L in range(nl)]
+    x = rng.standard_normal((T, d))
+    kw = dict(store="bf16", n_heads=4, n_kv_heads=2, head_dim=4, blocks=blocks)
+    whole = graphs.stack_forward(dls, x, 0.1, 3, 4, kind, **kw)
+    h = graphs.stack_forward(dls[:1], x, 0.1, 3, 4, kind, **kw)
+    for dl in dls[1:]:
+        h = graphs.stack_forward([dl], h, 0.1, 3, 4, kind, first=False, **kw)
+    np.testing.assert_array_equal(h, whole)
+    assert whole.shape == ((2 if blocks is None else len(blocks)) * T, d)

@@ -78,11 +78,12 @@ def test_perturbation_identity_section3():
     np.testing.assert_allclose(proj, dY, atol=1e-9 * np.abs(dY).max())
 
 
-def test_int4_dequant_brute_force():
+@pytest.mark.parametrize("d_in", [256, 200, 131])
+def test_int4_dequant_brute_force(d_in):
     rng = np.random.default_rng(5)
-    d_out, d_in = 3, 256
-    packed = rng.integers(0, 256, size=(d_out, d_in // 2), dtype=np.uint8)
-    scales = rng.standard_normal((d_out, 2)).astype(np.float16)
+    d_out = 3
+    packed = rng.integers(0, 256, size=(d_out, (d_in + 1) // 2), dtype=np.uint8)
+    scales = rng.standard_normal((d_out, (d_in + 127) // 128)).astype(np.float16)
     W = layers.dequant_int4_g128(packed, scales, d_in)
     for i in range(d_out):
         for k in range(d_in):
