@@ -29,8 +29,11 @@ Graph wiring (names follow synth.Workload):
 
 Hooks: `capture(name, X)` is called with each linear's input (the + half)
 before its pair forward -- Algorithm 1's calibration pass uses it to take the
-bases; `flops`, when a list, receives the algorithmic FLOP count (2 rows d_in
-d_out, gated x2) of every pair-forward call, with no events or synchronisation.
+bases; `on_decoder(L, h)` with the input of decoder L of a stack ([T, d] for
+the first, the stacked [n_blocks T, d] after it; the buffer is reused later,
+so a hook that keeps it clones it); `flops`, when a list, receives the
+algorithmic FLOP count (2 rows d_in d_out, gated x2) of every pair-forward
+call, with no events or synchronisation.
 """
 import torch
 
@@ -93,6 +96,7 @@ class ZOStep:
         self._pcache = {}
         self.device = dev
         self.capture = None
+        self.on_decoder = None
         self.flops = None
         # forward_loss fuses the loss pair into the last linear when set; off by default: the fused epilogue
         # lengthens the Llama-3-8B down launch by more than the separate loss launch takes
@@ -244,6 +248,8 @@ class ZOStep:
         h = x
         shared = True
         for L in range(n_dec):
+            if self.on_decoder is not None:
+                self.on_decoder(L, h)
             rows = T if shared else self.nb * T
             a = self._glue_rms(h, f"a{rows}")
             q = self.pair(f"{L}.q", a, shared, seed, query, "q")
@@ -300,52 +306,75 @@ class ZOStep:
         return self.loss_out
 
 
-def run_from_host(batches, step_fn, out_host):
-    """Run one ZO step per batch of PINNED host tensors, overlapping each batch's host-to-device copy
-    (on a side stream, into one of two device buffer sets) with the previous step's compute.
+class HostFeeder:
+    """Runs ZO steps on batches of PINNED host tensors, overlapping each batch's host-to-device copy (on a
+    side stream, into one of two device buffer sets) with the previous step's compute.
 
-    batches: list of tuples of pinned host tensors (e.g. (x, target) or (x,)); step_fn(device_tensors, i)
-    issues step i on torch's current stream and returns its device loss vector, which is copied into
-    out_host[i] (pinned) on the side stream once step i has finished, so no copy sits between two steps'
-    kernels.  That needs consecutive steps to return different loss vectors (ZOStep.loss alternates two;
-    step i + 2 rewrites step i's only after its read-back): a step function that returns the same vector
-    twice in a row raises ValueError.  Returns after issuing all work (no synchronisation).
+    The device buffers, the side stream and the events are made once, here, for batches shaped like
+    `example` (a tuple of host tensors, e.g. (x, target) or (x,)); run() then only issues copies, waits and
+    steps, so a timed region around run() holds no allocation or stream creation.
     """
+
+    def __init__(self, example, device=None):
+        self.main = torch.cuda.current_stream(device)
+        self.side = torch.cuda.Stream(device=self.main.device)
+        self.shapes = [(h.shape, h.dtype) for h in example]
+        self.bufs = [[torch.empty(sh, dtype=dt, device=self.main.device) for sh, dt in self.shapes]
+                     for _ in range(2)]
+        self.copied = [torch.cuda.Event(), torch.cuda.Event()]
+        self.free = [torch.cuda.Event(), torch.cuda.Event()]
+        self.read = [torch.cuda.Event(), torch.cuda.Event()]   # loss vector of step i read back (parity i % 2)
+
+    def run(self, batches, step_fn, out_host):
+        """One ZO step per batch.  step_fn(device_tensors, i) issues step i on the feeder's main stream (torch's
+        current stream when the feeder was made) and returns its device loss vector, which is copied into
+        out_host[i] (pinned) on the side stream once step i has finished, so no copy sits between two steps'
+        kernels.  That needs consecutive steps to return different loss vectors (ZOStep.loss alternates two;
+        step i + 2 rewrites step i's only after its read-back): a step function that returns the same vector
+        twice in a row raises ValueError.  Returns after issuing all work (no synchronisation)."""
+        if not batches:
+            return
+        for b in batches:
+            if [(h.shape, h.dtype) for h in b] != self.shapes:
+                raise ValueError("HostFeeder.run: every batch must match the feeder's shapes and dtypes")
+        main, side, bufs = self.main, self.side, self.bufs
+        copied, free, read = self.copied, self.free, self.read
+        prev_ptr = None
+
+        def fetch(i):
+            b = i % 2
+            side.wait_stream(main) if i < 2 else side.wait_event(free[b])   # buffer b no longer read
+            with torch.cuda.stream(side):
+                for d, h in zip(bufs[b], batches[i]):
+                    d.copy_(h, non_blocking=True)
+                copied[b].record(side)
+
+        fetch(0)
+        for i in range(len(batches)):
+            if i + 1 < len(batches):
+                fetch(i + 1)
+            b = i % 2
+            main.wait_event(copied[b])
+            if i >= 2:
+                main.wait_event(read[b])                 # step i - 2's loss vector, which step i rewrites, is read
+            with torch.cuda.stream(main):
+                out = step_fn(bufs[b], i)
+            if out.data_ptr() == prev_ptr:
+                raise ValueError("run_from_host: consecutive steps must return different loss vectors")
+            prev_ptr = out.data_ptr()
+            free[b].record(main)
+            side.wait_event(free[b])
+            with torch.cuda.stream(side):
+                out_host[i].copy_(out, non_blocking=True)
+                read[b].record(side)
+
+
+def run_from_host(batches, step_fn, out_host):
+    """HostFeeder(batches[0]).run(batches, step_fn, out_host): the feeder's buffers are made on every call;
+    keep a HostFeeder to reuse them."""
     if not batches:
         return
-    main = torch.cuda.current_stream()
-    side = torch.cuda.Stream()
-    bufs = [[torch.empty(h.shape, dtype=h.dtype, device=main.device) for h in batches[0]] for _ in range(2)]
-    copied = [torch.cuda.Event(), torch.cuda.Event()]
-    free = [torch.cuda.Event(), torch.cuda.Event()]
-    read = [torch.cuda.Event(), torch.cuda.Event()]      # loss vector of step i read back (parity i % 2)
-    prev_ptr = None
-
-    def fetch(i):
-        b = i % 2
-        side.wait_stream(main) if i < 2 else side.wait_event(free[b])   # buffer b no longer read
-        with torch.cuda.stream(side):
-            for d, h in zip(bufs[b], batches[i]):
-                d.copy_(h, non_blocking=True)
-            copied[b].record(side)
-
-    fetch(0)
-    for i in range(len(batches)):
-        if i + 1 < len(batches):
-            fetch(i + 1)
-        b = i % 2
-        main.wait_event(copied[b])
-        if i >= 2:
-            main.wait_event(read[b])                     # step i - 2's loss vector, which step i rewrites, is read
-        out = step_fn(bufs[b], i)
-        if out.data_ptr() == prev_ptr:
-            raise ValueError("run_from_host: consecutive steps must return different loss vectors")
-        prev_ptr = out.data_ptr()
-        free[b].record(main)
-        side.wait_event(free[b])
-        with torch.cuda.stream(side):
-            out_host[i].copy_(out, non_blocking=True)
-            read[b].record(side)
+    HostFeeder(batches[0]).run(batches, step_fn, out_host)
 
 
 def coefficient_offsets(specs, r):

@@ -6,13 +6,19 @@ oracle (with bf16/fp16 rounding mirrored where activations are stored).  Bases
 are inputs here (random orthonormal U from synth) so the step is tested on its
 own; the device basis is tested in test_gpu_kernels.py and below at full width.
 
-Tolerances (the benchmark spec): 16-bit outputs and L+- within 2e-2 relative; the sign
-of a must agree whenever |L+ - L-| exceeds 2e-2 max(L+, L-).  Below that bound
-a is not comparable between two implementations of a 16-bit graph: with
-eps = 1e-3 the +/- difference of every stored activation is below bf16
-resolution, so each side's a carries its own rounding noise.  When the signs
-agree, C after Adam (step 1: C - lr g / (|g| + eps)) must match within
-2e-2 * lr.  The fp32 toy graph checks outputs to 1e-4 and a to 1e-3 over two steps.
+Tolerances (the benchmark spec): 16-bit outputs and L+- within 2e-2 relative; the
+estimator scalar a within 2e-2 relative (its sign agreeing) whenever
+|L+ - L-| exceeds 2e-2 max(L+, L-).  The 16-bit step tests are built so that
+it does: the coefficients are drawn as C = 0.3 Z(seed, layer, query) plus
+noise and eps = 0.05, which moves every layer's output along its own
+perturbation at first order (on the last linear D = L+ - L- ~ 4 eps 0.3
+mean((Z p)^2), about a tenth of L), and each test asserts that bound before
+comparing a.  (With eps = 1e-3 and C independent of Z, L+ - L- sits below the
+bf16 resolution of the outputs and a is each side's rounding noise.)  Adam
+step 1 is then checked on all three arenas: m = (1 - beta1) a Z and
+v = (1 - beta2) (a Z)^2 carry |a| (2e-2 and 4e-2 relative), C - lr g/(|g| + eps)
+its sign (2e-2 lr).  The fp32 toy graph checks outputs to 1e-4 and a to 1e-3
+over two steps.
 """
 import numpy as np
 import pytest
@@ -27,40 +33,74 @@ from oracle import layers as olayers
 pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
 f32 = lambda v: float(np.float32(v))
+C_ALIGN = 0.3
 
 
 def n64(t):
-    return t.detach().double().cpu().numpy()
+    return t.detach().cpu().double().numpy()
 
 
-def _build(w, c_std=0.01):
-    """Weights, bases, coefficients of workload w on the device, and their fp64 copies."""
+def _build(w, c_std=0.01, align=None):
+    """Weights and bases of workload w on the device, its ZOStep, and a function that gives the oracle's
+    fp64 copy of one layer (W, U, C, layer_id) on demand, so that deep stacks never hold every layer's
+    fp64 weights at once.
+
+    The coefficients are drawn on the host: N(0, c_std^2), plus C_ALIGN Z(seed, layer, query) from the
+    oracle's generator when align = (seed, query).
+    """
     dt = {"bf16": torch.bfloat16, "fp16": torch.float16, "fp32": torch.float32}[w.act_dtype]
     specs = w.linears()
     offs = coefficient_offsets(specs, w.r)
-    lins, ora = [], {}
-    Wfp64 = {}
+    lins = []
     for s, off in zip(specs, offs):
         U = random_orthonormal(s.d_in, w.r, tensor_seed(w, "U", s.name), DEV)
         if w.wtype == "int4_g128":
             Wf = normal((s.d_out, s.d_in), tensor_seed(w, "W", s.name), DEV, std=w.weight_std)
             packed, scales = quantize_int4_g128(Wf)
+            del Wf
             lins.append(AdaptedLinear(s.name, packed, U, s.layer_id, off, w.r, w_scales=scales,
                                       wtype=zo.DT_INT4_G128, d_in=s.d_in))
-            Wfp64[s.name] = olayers.dequant_int4_g128(packed.cpu().numpy(), scales.float().cpu().numpy(), s.d_in)
         else:
             W = normal((s.d_out, s.d_in), tensor_seed(w, "W", s.name), DEV, std=w.weight_std, dtype=dt)
             lins.append(AdaptedLinear(s.name, W, U, s.layer_id, off, w.r))
     step = ZOStep(zo.Context(0), w.kind, lins, w.T, w.act_dtype, eps=w.eps, lr=w.lr)
-    step.C.copy_(normal(tuple(step.C.shape), tensor_seed(w, "C0"), DEV, std=c_std))
-    for l in lins:
-        C = n64(step.C[l.offset:l.offset + l.d_out * w.r]).reshape(l.d_out, w.r)
-        Wo = Wfp64[l.name] if l.name in Wfp64 else n64(l.W)
-        ora[l.name] = dict(W=Wo, U=n64(l.U), C=C, layer_id=l.layer_id)
-    return step, ora
+    C = normal(tuple(step.C.shape), tensor_seed(w, "C0"), "cpu", std=c_std).double().numpy()
+    if align is not None:
+        for l in lins:
+            C[l.offset:l.offset + l.d_out * w.r] += C_ALIGN * philox.perturbation(
+                align[0], l.layer_id, align[1], l.d_out, w.r).reshape(-1)
+    step.C.copy_(torch.from_numpy(C.astype(np.float32)))
+    C_stored = n64(step.C)
+
+    def oracle_layer(name, weights=True):
+        l = step.by_name[name]
+        d = dict(C=C_stored[l.offset:l.offset + l.d_out * w.r].reshape(l.d_out, w.r), layer_id=l.layer_id)
+        if weights:
+            d["U"] = n64(l.U)
+            if w.wtype == "int4_g128":
+                d["W"] = olayers.dequant_int4_g128(l.W.cpu().numpy(), l.w_scales.float().cpu().numpy(), l.d_in)
+            else:
+                d["W"] = n64(l.W)
+        return d
+
+    return step, oracle_layer
 
 
-def _check_step(step, ora_layers, Y, out, Yo, tgt_o, w, seed, query):
+def _stack_names(kind):
+    return ["q", "k", "v", "o", "gate", "up", "down"] if kind == "llama" else ["q", "k", "v", "o", "fc1", "fc2"]
+
+
+def _oracle_stack(w, oracle_layer, x, seed, query):
+    """The oracle's stack, one decoder at a time (one decoder's fp64 weights in memory)."""
+    h = n64(x)
+    for L in range(w.n_decoder):
+        dl = {nm: oracle_layer(f"{L}.{nm}") for nm in _stack_names(w.kind)}
+        h = graphs.stack_forward([dl], h, w.eps, seed, query, w.kind, store=w.act_dtype, first=(L == 0))
+    return h
+
+
+def _check_step(step, oracle_layer, Y, out, Yo, tgt_o, w, seed, query):
+    """Outputs, losses, a, and Adam step 1 (from m = v = 0) of every layer against the oracle."""
     Lp, Lm, D, a = oloss.loss_pair(Yo, w.T, tgt_o, w.eps)
     Yg = n64(Y)
     err_max = float(np.abs(Yg - Yo).max() / np.abs(Yo).max())
@@ -71,62 +111,117 @@ def _check_step(step, ora_layers, Y, out, Yo, tgt_o, w, seed, query):
     assert err_mean <= 1e-2, ("mean |dY| / mean |Y|", err_mean)
     o = out.cpu().numpy()
     assert abs(o[0] - Lp) <= 2e-2 * Lp and abs(o[1] - Lm) <= 2e-2 * Lm, (o[:2], Lp, Lm)
-    if abs(Lp - Lm) > 2e-2 * max(Lp, Lm):
-        assert np.sign(o[3]) == np.sign(a), (o[3], a)
-    if np.sign(o[3]) != np.sign(a):
-        return
-    # Adam step 1 from m = v = 0 with the oracle's own a: C - lr g / (|g| + adam_eps).  Where |g| is
-    # within ~1e3 adam_eps the update depends on |a| itself, which the two sides do not share.
-    for name, l in ora_layers.items():
-        lin = step.by_name[name]
-        g = optim.zo_gradient(a, philox.perturbation(seed, l["layer_id"], query, *l["C"].shape))
-        Cn, _, _ = optim.adam_step(l["C"], 0, 0, g, f32(w.lr), f32(w.beta1), f32(w.beta2), f32(w.adam_eps), 1)
-        Cg = n64(step.C[lin.offset:lin.offset + lin.d_out * w.r]).reshape(l["C"].shape)
-        big = np.abs(g) > 1e3 * w.adam_eps
-        err = float(np.abs(Cg - Cn)[big].max())
-        assert err <= 2e-2 * w.lr, (name, err, o[3], a)
+    # the inputs are built so that the benchmark spec's bound applies: a is compared, never skipped
+    assert abs(Lp - Lm) > 2e-2 * max(Lp, Lm), ("the test's inputs must make L+ - L- resolvable", Lp, Lm)
+    assert np.sign(o[3]) == np.sign(a), (o[3], a)
+    assert abs(o[3] - a) <= 2e-2 * abs(a), (o[3], a)
+    assert abs(o[2] - D) <= 2e-2 * abs(D), (o[2], D)
+    b1, b2, lr, ae = f32(w.beta1), f32(w.beta2), f32(w.lr), f32(w.adam_eps)
+    n_checked = 0
+    for lin in step.linears:
+        l = oracle_layer(lin.name, weights=False)
+        sl = slice(lin.offset, lin.offset + lin.d_out * w.r)
+        Zl = philox.perturbation(seed, l["layer_id"], query, *l["C"].shape)
+        g = optim.zo_gradient(a, Zl)
+        Cn, mn, vn = optim.adam_step(l["C"], 0, 0, g, lr, b1, b2, ae, 1)
+        Cg, mg, vg = (n64(t[sl]).reshape(l["C"].shape) for t in (step.C, step.m, step.v))
+        # a within 2e-2, and the device's normals within 1e-6 (1 + |z|) of the oracle's (fp32 Box-Muller)
+        dz = 1e-6 * (1.0 + np.abs(Zl))
+        bad = np.abs(mg - mn) > 2e-2 * np.abs(mn) + (1 - b1) * 1.02 * abs(a) * dz
+        assert not bad.any(), (lin.name, mg[bad][:4], mn[bad][:4], Zl[bad][:4], o[3], a)
+        assert np.all(np.abs(vg - vn) <= 4.1e-2 * np.abs(vn) + (1 - b2) * 1.05 * a * a * (2 * np.abs(Zl) + dz) * dz), \
+            lin.name
+        # where |g| is within ~1e3 adam_eps the step-1 update depends on |a| itself, and where |z| < 1e-4 the
+        # normals' absolute tolerance may flip its sign: those elements are bounded through m, v above
+        big = (np.abs(g) > 1e3 * w.adam_eps) & (np.abs(Zl) > 1e-4)
+        assert np.abs(Cg - Cn)[big].max() <= 2e-2 * w.lr, (lin.name, o[3], a)
+        n_checked += 1
+    assert n_checked == len(step.linears)
 
 
-def test_llama_mlp_step_full_width():
-    w = workload("llama_mlp_bf16", T=256)
-    step, ora = _build(w)
-    x, _ = lowrank_activations(w.T, 4096, 64, 0.05, tensor_seed(w, "x"), DEV)
-    tgt = normal((w.T, 4096), tensor_seed(w, "t"), DEV, dtype=torch.bfloat16)
-    seed, query = 17, 1
+def _run_step(step, x, tgt, seed, query):
     Y = step.forward(x, seed, query).clone()
     out = step.loss(Y, tgt).clone()
     step.update(1, seed, query)
     torch.cuda.synchronize()
     assert step.ctx.device_status() == 0
-    lay = [ora["gate"], ora["up"], ora["down"]]
+    return Y, out
+
+
+def test_llama_mlp_step_full_width():
+    # gate/up on the shared input (CTA-pair kernel, epilogue Z tables), down on 512 stacked rows
+    seed, query = 17, 1
+    w = workload("llama_mlp_bf16", T=256, eps=0.05)
+    step, ol = _build(w, align=(seed, query))
+    x, _ = lowrank_activations(w.T, 4096, 64, 0.05, tensor_seed(w, "x"), DEV)
+    tgt = normal((w.T, 4096), tensor_seed(w, "t"), DEV, dtype=torch.bfloat16)
+    Y, out = _run_step(step, x, tgt, seed, query)
+    lay = [ol("gate"), ol("up"), ol("down")]
     Yo = graphs.llama_mlp_forward(lay, n64(x), w.eps, seed, query, store="bf16")
-    _check_step(step, ora, Y, out, Yo, n64(tgt), w, seed, query)
+    _check_step(step, ol, Y, out, Yo, n64(tgt), w, seed, query)
     step.ctx.close()
 
 
-@pytest.mark.parametrize("name,n_dec,T", [("llama_stack_bf16", 2, 64), ("opt_stack_fp16", 2, 48),
-                                          ("llama_stack_int4", 1, 64)])
+@pytest.mark.parametrize("name,n_dec,T", [
+    ("llama_stack_bf16", 2, 64), ("opt_stack_fp16", 2, 48), ("llama_stack_int4", 1, 64),   # one-CTA kernel
+    # 512 stacked rows: the CTA-pair kernel (whole low-rank term on the MMA, split last wave) in the graph
+    ("llama_stack_bf16", 2, 256), ("opt_stack_fp16", 2, 256),
+    # 1024 stacked rows: INT4 weights expanded once per call, then the bf16 CTA-pair kernel
+    ("llama_stack_int4", 1, 512)])
 def test_stack_step(name, n_dec, T):
-    w = workload(name, T=T, n_decoder=n_dec)
-    step, ora = _build(w)
+    seed, query = 23, 2
+    w = workload(name, T=T, n_decoder=n_dec, eps=0.05)
+    step, ol = _build(w, align=(seed, query))
     dt = torch.bfloat16 if w.act_dtype == "bf16" else torch.float16
     x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=dt)
-    seed, query = 23, 2
-    Y = step.forward(x, seed, query).clone()
-    out = step.loss(Y, None).clone()
-    step.update(1, seed, query)
-    torch.cuda.synchronize()
-    assert step.ctx.device_status() == 0
-    names = ["q", "k", "v", "o", "gate", "up", "down"] if w.kind == "llama" else ["q", "k", "v", "o", "fc1", "fc2"]
-    dls = [{nm: ora[f"{L}.{nm}"] for nm in names} for L in range(n_dec)]
-    Yo = graphs.stack_forward(dls, n64(x), w.eps, seed, query, w.kind, store=w.act_dtype)
-    _check_step(step, ora, Y, out, Yo, None, w, seed, query)
+    Y, out = _run_step(step, x, None, seed, query)
+    Yo = _oracle_stack(w, ol, x, seed, query)
+    _check_step(step, ol, Y, out, Yo, None, w, seed, query)
+    step.ctx.close()
+
+
+def _check_outputs(Yg, Yo, what):
+    err_max = float(np.abs(Yg - Yo).max() / np.abs(Yo).max())
+    err_mean = float(np.mean(np.abs(Yg - Yo)) / np.mean(np.abs(Yo)))
+    assert err_max <= 2e-2 and err_mean <= 1e-2, (what, err_max, err_mean)
+
+
+@pytest.mark.parametrize("name", ["llama_stack_bf16", "opt_stack_fp16", "llama_stack_int4"])
+def test_stack_step_full_depth(name):
+    # Every decoder of the configuration (32 or 40) at full width on 16 tokens per perturbation: layer ids, the
+    # shared-input rule of the first decoder and the buffer rotation over the whole chain.
+    # The synthetic stack is chaotic: a relative difference of 1e-3 in a decoder's input grows about 1.45x per
+    # decoder (measured on the oracle alone, with C = 0 as with C = 0.3 Z), so two correct implementations
+    # that round a stored activation differently decorrelate after ~20 decoders and their final outputs are
+    # not comparable element by element.  Each decoder is therefore checked on identical inputs: the oracle
+    # is fed the GPU's stored input to that decoder, and its output is compared with the GPU's input to the
+    # next decoder (the step's output after the last).  L+-, D, a and Adam step 1 of all layers are then
+    # checked against the oracle's last decoder on the GPU's input to it.
+    seed, query = 29, 3
+    w = workload(name, T=16, eps=0.05)
+    assert w.n_decoder in (32, 40)
+    step, ol = _build(w, align=(seed, query))
+    dt = torch.bfloat16 if w.act_dtype == "bf16" else torch.float16
+    x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=dt)
+    ins = []
+    step.on_decoder = lambda L, h: ins.append(h.clone())
+    Y, out = _run_step(step, x, None, seed, query)
+    assert len(ins) == w.n_decoder and ins[0].shape == (w.T, w.d_model)
+    outs = ins[1:] + [Y]
+    for L in range(w.n_decoder):
+        dl = {nm: ol(f"{L}.{nm}") for nm in _stack_names(w.kind)}
+        assert outs[L].shape == (2 * w.T, w.d_model)
+        Yo = graphs.stack_forward([dl], n64(ins[L]), w.eps, seed, query, w.kind, store=w.act_dtype,
+                                  first=(L == 0))
+        _check_outputs(n64(outs[L]), Yo, f"decoder {L}")
+    _check_step(step, ol, Y, out, Yo, None, w, seed, query)
     step.ctx.close()
 
 
 def test_toy_two_steps():
     w = workload("toy_fp32")
-    step, ora = _build(w, c_std=0.05)
+    step, ol = _build(w, c_std=0.05)
+    ora = {nm: ol(nm) for nm in ("l1", "l2")}
     x, _ = lowrank_activations(w.T, 256, 16, 0.1, tensor_seed(w, "x"), DEV, dtype=torch.float32, unit_rms=False,
                                noise_is_energy=False)
     tgt = normal((w.T, 256), tensor_seed(w, "t"), DEV)
