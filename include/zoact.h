@@ -135,7 +135,9 @@ int zoact_get_launch_count(zoact_ctx* ctx, int64_t* count);
 
 /* Kernel timing: with enable != 0 the context records CUDA events on its stream
  * around every tensor-core pair-forward kernel (the MMA kernel alone, without
- * the preparation kernels of the same call; up to 4096 launches between reads).
+ * the preparation kernels of the same call -- except that INT4 weights expanded
+ * to bf16 first are timed with that expansion; up to 4096 launches between
+ * reads, later ones are not timed and not counted).
  * Switching it on creates the event pool (ZOACT_ERR_CUDA if that fails).  The
  * events themselves lengthen a step: measure throughput with timing off.
  * zoact_kernel_timing(ctx, 0/1) switches it and forgets recorded launches;
@@ -196,20 +198,28 @@ int zoact_pair_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X, 
  * The paper has no counterpart: this entry point exists for callers that must
  * not allocate device memory (a framework whose allocator owns all device
  * memory, a real-time loop that cannot afford a synchronising cudaMalloc, a
- * process under a hard memory budget).  It computes exactly what
- * zoact_pair_forward computes with P == NULL, on `stream` (a cudaStream_t),
- * without a context and without calling cudaMalloc, cudaFree or any allocating
- * library routine.  Its only scratch is one file-scope device array of
+ * process under a hard memory budget).  It computes the pair forward of
+ * zoact_pair_forward with P == NULL, on `stream` (a cudaStream_t), without a
+ * context and without calling cudaMalloc, cudaFree or any allocating library
+ * routine.  It adds the low-rank term from fp32 epilogue tables, so its
+ * outputs agree with zoact_pair_forward within the pair forward's tolerance
+ * (1e-4 of the output scale for fp32 outputs), not bit for bit.  Limits beyond
+ * zoact_pair_forward's: r <= 32, and weights of type FP32, BF16 or FP16 (INT4
+ * returns ZOACT_ERR_UNSUPPORTED).  Its only scratch is one file-scope device array of
  * ZOACT_NOALLOC_MAX_PROJ_FLOATS floats (4 MiB) plus a status slot, which every
  * GPU that loads the library holds until the process exits; it holds the
  * projection U^T x of the rows(X) x r inputs, so rows(X) * r above
  * ZOACT_NOALLOC_MAX_PROJ_FLOATS returns ZOACT_ERR_TOO_LARGE and launches nothing.
  * The first call on each device looks up the array's device address (with that
- * device current); make that first call before any stream capture.  All calls
+ * device current); make that first call before any stream capture.  The address
+ * belongs to the CUDA context it was looked up in: after cudaDeviceReset (or
+ * with another context current) the next call looks it up again, so that call
+ * too should come before any stream capture.  All calls
  * share the array: calls that overlap on the GPU (other streams or threads)
  * race and must be ordered by the caller.  Device-side errors are not
  * reported back (there is no context); the returned status covers argument
- * and launch errors.  Other requirements as for zoact_pair_forward.            */
+ * and launch errors.  Other requirements (alignment, d_in and d_out multiples)
+ * as for zoact_pair_forward.                                                    */
 #define ZOACT_NOALLOC_MAX_PROJ_FLOATS (1 << 20)
 int zoact_pair_forward_noalloc(const zoact_layer* layer, const void* X, int xdtype, int64_t T,
                                int input_shared, float eps, uint64_t seed, uint64_t query, int act,
@@ -372,6 +382,31 @@ int zoact_rms_norm(zoact_ctx* ctx, const void* X, int dtype, int64_t rows, int32
  * consecutive query heads (n_rep = 1: plain sum).                              */
 int zoact_mix_rms(zoact_ctx* ctx, const void* q, const void* k, const void* v, int dtype,
                   int64_t rows, int32_t n, int32_t n_rep, int32_t head_dim, float eps, void* Y);
+
+/* ---- data-parallel replicas ----
+ * A data-parallel ZO step shares everything but the tokens: every rank holds
+ * the same W, U, C, m, v and seed, runs its token shard, and the ranks
+ * all-reduce the loss vector once (MeZO's property, which Section 3 keeps: Z
+ * is regenerated from the seed, so C stays identical on every rank without a
+ * gradient exchange).
+ * zoact_mean_over_ranks: v[i] = v[i] / world for the n doubles of the
+ *   all-reduced (summed) loss vector v (DEVICE): every entry is a mean over a
+ *   rank's equal token share and a is linear in the losses, so the result is
+ *   the whole batch's vector.  1 <= world; n >= 0.
+ * zoact_arena_hash: a 64-bit fingerprint of n_words 32-bit words at `data`
+ *   (DEVICE, 4-byte aligned; 16-byte aligned for full speed), written to
+ *   *hash_out (DEVICE uint64):
+ *       h = sum_i mix64(((i << 32) | w_i) + 0x9E3779B97F4A7C15)  mod 2^64
+ *   with mix64 the output function of SplitMix64 (Steele, Lea, Flood, OOPSLA
+ *   2014): z ^= z >> 30; z *= 0xBF58476D1CE4E5B9; z ^= z >> 27;
+ *   z *= 0x94D049BB133111EB; z ^= z >> 31.  The same on every GPU and launch
+ *   configuration (integer sums).  Replicas compare their fingerprints of C
+ *   (and m, v) to detect one that diverged; ZOACT_ERR_REPLICA_MISMATCH is the
+ *   status the Python layer reports then.  0 <= n_words < 2^32.
+ * The paper has no counterpart of either call (it runs on one device).        */
+#define ZOACT_ERR_REPLICA_MISMATCH (-8)  /* data-parallel replicas hold different coefficients */
+int zoact_mean_over_ranks(zoact_ctx* ctx, double* v, int64_t n, int32_t world);
+int zoact_arena_hash(zoact_ctx* ctx, const void* data, int64_t n_words, uint64_t* hash_out);
 
 #ifdef __cplusplus
 }

@@ -14,6 +14,6 @@ from ._lib import (  # noqa: F401
     zoact_multi_forward, zoact_multi_forward_gated, zoact_loss_multi, zoact_adam_step_multi, zoact_sgd_step_multi,
     eval_blocks, one_sided_blocks, MAX_EVAL_BLOCKS,
     zoact_basis_prepared_bytes, zoact_basis_prepare, zoact_lowrank_proj_prepared,
-    zoact_subspace_overlap, zoact_gradient_energy,
+    zoact_subspace_overlap, zoact_gradient_energy, zoact_mean_over_ranks, zoact_arena_hash,
     DT_FP32, DT_BF16, DT_FP16, DT_INT4_G128, ACT_NONE, ACT_RELU, ACT_GELU, EXPORTS, LIB_PATH, TORCH_DT,
 )

@@ -21,6 +21,7 @@ ZOACT_ERR_NONFINITE = -4
 ZOACT_ERR_TIMEOUT = -5
 ZOACT_ERR_NOMEM = -6
 ZOACT_ERR_TOO_LARGE = -7
+ZOACT_ERR_REPLICA_MISMATCH = -8
 NOALLOC_MAX_PROJ_FLOATS = 1 << 20
 MAX_EVAL_BLOCKS = 17
 
@@ -37,7 +38,8 @@ EXPORTS = [
     "zoact_rms_norm", "zoact_mix_rms", "zoact_multi_forward", "zoact_multi_forward_gated", "zoact_loss_multi",
     "zoact_adam_step_multi", "zoact_sgd_step_multi", "zoact_basis_prepared_bytes", "zoact_basis_prepare",
     "zoact_lowrank_proj_prepared", "zoact_subspace_overlap", "zoact_gradient_energy", "zoact_kernel_timing",
-    "zoact_kernel_time", "zoact_pair_forward_loss", "zoact_debug_timeout",
+    "zoact_kernel_time", "zoact_pair_forward_loss", "zoact_debug_timeout", "zoact_mean_over_ranks",
+    "zoact_arena_hash",
 ]
 
 
@@ -129,6 +131,8 @@ def load():
                                   ctypes.POINTER(ctypes.c_uint64), F32, F32, F32, F32, I64, U64],
         "zoact_sgd_step_multi": [P, P, I64, ctypes.POINTER(zoact_coeff_block), I32, P, I32,
                                  ctypes.POINTER(ctypes.c_uint64), F32, U64],
+        "zoact_mean_over_ranks": [P, P, I64, I32],
+        "zoact_arena_hash": [P, P, I64, P],
     }
     for name, argtypes in sig.items():
         fn = getattr(lib, name)
@@ -403,3 +407,17 @@ def zoact_gradient_energy(ctx, U, G, out):
     d_in, r = U.shape
     _check("zoact_gradient_energy", load().zoact_gradient_energy(ctx.handle, _ptr(U), d_in, r, _ptr(G), _dt(G),
                                                                   G.shape[1], _ptr(out)))
+
+
+def zoact_mean_over_ranks(ctx, v, world):
+    """v (device fp64) /= world in place: the all-reduced sum of the ranks' loss vectors -> their mean."""
+    _check("zoact_mean_over_ranks", load().zoact_mean_over_ranks(ctx.handle, _ptr(v), v.numel(), int(world)))
+
+
+def zoact_arena_hash(ctx, t, out):
+    """The 64-bit fingerprint of t's bytes (a device tensor whose size is a multiple of 4 bytes) written to
+    out (a device int64 tensor of one element holding the uint64's bits)."""
+    nbytes = t.numel() * t.element_size()
+    if nbytes % 4 or out.dtype != torch.int64 or out.numel() != 1:
+        raise ValueError("zoact_arena_hash: a tensor of whole 32-bit words and a one-element int64 output")
+    _check("zoact_arena_hash", load().zoact_arena_hash(ctx.handle, _ptr(t), nbytes // 4, _ptr(out)))

@@ -68,8 +68,10 @@ int timing_pool(Ctx* ctx) {
   return ZOACT_OK;
 }
 
+// Nested begin / end pairs (a launch that runs another launcher inside it) time the outermost pair only.
 int timing_begin(Ctx* ctx) {
   if (!ctx->timing || !ctx->tev) return ZOACT_OK;
+  if (ctx->tev_depth++ > 0) return ZOACT_OK;
   if (ctx->tev_used >= ctx->tev_cap) {
     ++ctx->tev_dropped;
     return ZOACT_OK;
@@ -79,7 +81,9 @@ int timing_begin(Ctx* ctx) {
 }
 
 int timing_end(Ctx* ctx) {
-  if (!ctx->timing || !ctx->tev || ctx->tev_used >= ctx->tev_cap) return ZOACT_OK;
+  if (!ctx->timing || !ctx->tev) return ZOACT_OK;
+  if (ctx->tev_depth > 0 && --ctx->tev_depth > 0) return ZOACT_OK;
+  if (ctx->tev_used >= ctx->tev_cap) return ZOACT_OK;
   ZOACT_CUDA_TRY(cudaEventRecord(ctx->tev[2 * ctx->tev_used + 1], ctx->stream));
   ++ctx->tev_used;
   return ZOACT_OK;
@@ -195,6 +199,7 @@ const char* zoact_status_string(int status) {
     case ZOACT_ERR_TIMEOUT: return "bounded device wait timed out";
     case ZOACT_ERR_NOMEM: return "out of device memory";
     case ZOACT_ERR_TOO_LARGE: return "request exceeds the fixed scratch of the no-allocation entry point";
+    case ZOACT_ERR_REPLICA_MISMATCH: return "data-parallel replicas hold different coefficients";
     default: return "unknown status";
   }
 }
@@ -267,6 +272,7 @@ int zoact_kernel_timing(zoact_ctx* ctx, int enable) {
   ctx->timing = enable != 0;
   ctx->tev_used = 0;
   ctx->tev_dropped = 0;
+  ctx->tev_depth = 0;
   return ZOACT_OK;
 }
 
@@ -284,6 +290,7 @@ int zoact_kernel_time(zoact_ctx* ctx, double* ms_total, int64_t* launches) {
   *launches = ctx->tev_used;
   ctx->tev_used = 0;
   ctx->tev_dropped = 0;
+  ctx->tev_depth = 0;
   return ZOACT_OK;
 }
 
@@ -599,3 +606,18 @@ int zoact_mix_rms(zoact_ctx* ctx, const void* q, const void* k, const void* v, i
 }
 
 }  // extern "C"
+
+int zoact_mean_over_ranks(zoact_ctx* ctx, double* v, int64_t n, int32_t world) {
+  ZOACT_ENTER(ctx);
+  if (n < 0 || world < 1 || (n > 0 && !v)) return ZOACT_ERR_INVALID_ARG;
+  return launch_mean_over_ranks(ctx, v, n, world);
+}
+
+int zoact_arena_hash(zoact_ctx* ctx, const void* data, int64_t n_words, uint64_t* hash_out) {
+  ZOACT_ENTER(ctx);
+  if (!hash_out || n_words < 0 || n_words >= ((int64_t)1 << 32) || (n_words > 0 && !data)) return ZOACT_ERR_INVALID_ARG;
+  if (((uintptr_t)hash_out & 7u) != 0) return ZOACT_ERR_INVALID_ARG;
+  if (n_words >= 4 && ((uintptr_t)data & 15u) != 0) return ZOACT_ERR_INVALID_ARG;
+  if (((uintptr_t)data & 3u) != 0) return ZOACT_ERR_INVALID_ARG;
+  return launch_arena_hash(ctx, data, n_words, hash_out);
+}

@@ -57,6 +57,7 @@ struct Ctx {
   int tev_cap = 0;
   int tev_used = 0;                   // pairs recorded since the last read
   int64_t tev_dropped = 0;            // launches not timed (capacity reached)
+  int tev_depth = 0;                  // nesting of timing_begin / timing_end (the outermost pair records)
 };
 
 // Record the start / end of a timed launch on the context's stream (no-ops unless timing is on).
@@ -228,6 +229,10 @@ int launch_mix_rms(Ctx* ctx, const void* q, const void* k, const void* v, int dt
 int launch_subspace_overlap(Ctx* ctx, const float* Ua, const float* Ub, int d, int ra, int rb, double* out);
 int launch_gradient_energy(Ctx* ctx, const float* U, int d_in, int r, const void* G, int gdtype, int64_t n,
                            double* out);
+
+// Data-parallel replicas (k_replica.cu): the SplitMix64-tagged sum of an arena's words; v /= world.
+int launch_arena_hash(Ctx* ctx, const void* data, int64_t n_words, uint64_t* out);
+int launch_mean_over_ranks(Ctx* ctx, double* v, int64_t n, int world);
 
 int run_basis_init(Ctx* ctx, const void* X, int xdtype, int64_t n_tok, int d_in, int r, int oversample,
                    int n_iter, uint64_t seed, float* U_out, float* evals_out);

@@ -142,11 +142,13 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     return launch_pair_tc(ctx, b);
   }
   if (a.wtype == ZOACT_DT_INT4_G128 && (a.rows >= INT4_STAGED_MIN_ROWS || big_r)) {
-    // staged INT4: expand W (and W2) to bf16 in context scratch, then the bf16 kernel
+    // staged INT4: expand W (and W2) to bf16 in context scratch, then the bf16 kernel (timed together)
     const size_t bytes = (size_t)a.d_out * a.d_in * 2;
     void* wb = scratch(ctx, SLOT_WDQ0, bytes);
     if (!wb) return ZOACT_ERR_NOMEM;
-    int st = launch_dequant_int4(ctx, a.W, a.w_scales, wb, a.d_out, a.d_in);
+    int st = timing_begin(ctx);
+    if (st) return st;
+    st = launch_dequant_int4(ctx, a.W, a.w_scales, wb, a.d_out, a.d_in);
     if (st) return st;
     PairArgs b = a;
     b.W = wb;
@@ -160,7 +162,9 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
       b.W2 = wb2;
       b.w_scales2 = nullptr;
     }
-    return launch_pair_tc(ctx, b);
+    st = launch_pair_tc(ctx, b);
+    if (st) return st;
+    return timing_end(ctx);
   }
   if (a.xdtype != ZOACT_DT_BF16 && a.xdtype != ZOACT_DT_FP16) return ZOACT_ERR_UNSUPPORTED;
   const bool w4 = a.wtype == ZOACT_DT_INT4_G128;

@@ -11,6 +11,11 @@
 //
 // Its only scratch is the file-scope device array below (4 MiB plus a status
 // slot), which every GPU that loads libzoact holds until the process exits.
+// Limits beyond the regular entry point's: ranks up to 32 and 16-bit or fp32
+// weights (INT4 is refused with ZOACT_ERR_UNSUPPORTED); the low-rank term is
+// added from fp32 epilogue tables (the regular entry point can put it on the
+// tensor cores), so the outputs agree with zoact_pair_forward within the pair
+// forward's tolerance, not bit for bit.
 // It stores P = X U ([rows, r] fp32) and, when room is left, the split-K
 // partials of that projection.  A request with rows * r above
 // ZOACT_NOALLOC_MAX_PROJ_FLOATS is rejected with ZOACT_ERR_TOO_LARGE before
@@ -18,6 +23,8 @@
 // call's contents: the status slot is cleared at every call, and P and the
 // partials are fully rewritten before they are read.  Calls that overlap on
 // the GPU (other streams, other host threads) race on the array.
+#include <cuda.h>
+
 #include <mutex>
 
 #include "internal.h"
@@ -34,14 +41,47 @@ static __device__ __align__(256) float g_noalloc_scratch[NOALLOC_FLOATS + 64];
 std::mutex g_mu;
 float* g_addr[NOALLOC_MAX_DEVICES] = {};
 int g_sm_count[NOALLOC_MAX_DEVICES] = {};
+unsigned long long g_ctx_id[NOALLOC_MAX_DEVICES] = {};
 
-// Device address of the array on the current device, looked up once per device.
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+
+// The process-unique id of the current CUDA context (driver API, CUDA >= 12.0); 0 when there is none yet or
+// the query is not available.  A device reset destroys the context, and the array lives in a module loaded
+// into it: its address is only valid for the context it was looked up in.
+unsigned long long current_context_id() {
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS)
+    return 0;
+  return id;
+}
+
+// Device address of the array in the current context of device `dev`.  Looked up (with the device current)
+// on the first call on the device, and again whenever the current context is not the one of the last lookup
+// (after cudaDeviceReset, or when the caller binds another context), so a cached address is never used in a
+// context it does not belong to.  Where the context id cannot be read, every call looks the address up.
 int scratch_address(int dev, float** out, int* sm_count) {
   if (dev < 0 || dev >= NOALLOC_MAX_DEVICES) return ZOACT_ERR_UNSUPPORTED;
   std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_addr[dev]) {
+  const unsigned long long id = current_context_id();
+  if (!g_addr[dev] || id == 0 || id != g_ctx_id[dev]) {
     void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);   // creates the context if needed
     if (e != cudaSuccess || !p) {
       cudaGetLastError();
       return ZOACT_ERR_CUDA;
@@ -50,6 +90,7 @@ int scratch_address(int dev, float** out, int* sm_count) {
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return ZOACT_ERR_CUDA;
     g_addr[dev] = static_cast<float*>(p);
     g_sm_count[dev] = sms;
+    g_ctx_id[dev] = current_context_id();      // the context the lookup ran in (0: look up again next call)
   }
   *out = g_addr[dev];
   *sm_count = g_sm_count[dev];
