@@ -1,15 +1,18 @@
 #!/usr/bin/env python
 """ZO-step throughput of the ZO-Act hot path on GB300.
 
-Default workload: the Llama-3-8B MLP block in bf16 -- gate/up 4096 -> 14336 on
-a shared input, SiLU gate, down 14336 -> 4096 -- r = 16, T = 2048 tokens per
-perturbation (4096 stacked rows for the +/- pair), MSE to N(0,1) targets,
-eps = 1e-3, Adam on all coefficients.  Other workloads (--workload):
-llama_stack_bf16 (224 linears, T = 16 x 256), llama_stack_int4 (same, INT4 g128
-weights), opt_stack_fp16 (240 linears, r = 32).  Synthetic data: rank-64
-Gaussian signal plus 5% noise, unit RMS per token; W ~ N(0, 0.02).  The bases
-come from Algorithm 1 on the device before timing: one calibration forward pass
-of the base model, then zoact_basis_init on every layer's input.
+Default workload: the full Llama-3-8B linear stack in bf16 -- 32 decoder layers
+x {q 4096->4096, k/v 4096->1024, o 4096->4096, gate/up 4096->14336, down
+14336->4096} = 224 adapted linears, r = 16, T = 16 x 256 = 4096 tokens per
+perturbation (8192 stacked rows for the +/- pair), each layer's input the
+RMS-normalised output before it, loss = mean squared output, eps = 1e-3, Adam
+on all 22.0 M coefficients.  Other workloads (--workload): llama_mlp_bf16 (the
+MLP block: gate/up 4096 -> 14336 on a shared input, down 14336 -> 4096, MSE to
+N(0,1) targets, T = 2048), llama_stack_int4 (the stack with INT4 g128 weights),
+opt_stack_fp16 (240 linears, r = 32).  Synthetic data: rank-64 Gaussian signal
+plus 5% noise, unit RMS per token; W ~ N(0, 0.02).  The bases come from
+Algorithm 1 on the device before timing: one calibration forward pass of the
+base model, then zoact_basis_init on every layer's input.
 
 One step = per adapted linear zoact_lowrank_proj + zoact_pair_forward (gate/up:
 zoact_pair_forward_gated) with the glue ops, then zoact_loss_pair and
@@ -19,6 +22,8 @@ value = training tokens/s = world_size * T / step time (CUDA events around
 exactly --steps steps, max over ranks).  The frozen weights are larger than L2
 (129 MB), so every step reads them from HBM.  `--impl reference` times the CPU
 oracle (numpy fp64) on a bounded sample of the default workload instead.
+`--measure-peak fp16` measures the dense fp16 tensor peak the OPT-13B workload
+is graded against.
 """
 import argparse
 import json
@@ -33,9 +38,10 @@ sys.path.insert(0, ROOT)
 
 METRIC = "ZO-step tokens/s per adapted-linear stack; % of HBM or tensor-pipe roofline"
 UNIT = "tokens/s"
-DEFAULT_WORKLOAD = "llama_mlp_bf16"
+DEFAULT_WORKLOAD = "llama_stack_bf16"
 N_CAL = {"llama_mlp_bf16": 2048, "llama_stack_bf16": 512, "llama_stack_int4": 512, "opt_stack_fp16": 4096}
 LR = 1e-4
+TIMING_PAIRS = 4096          # event pairs in the library's kernel-timing pool (launches timed per read)
 
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one step's pair launches, from one ncu
@@ -43,13 +49,65 @@ LR = 1e-4
 PAIR_TRAFFIC_BYTES = {"llama_mlp_bf16": 938.5e6}
 
 
-def _peaks():
+# Dense fp16 tensor peak of the GB300s (TFLOP/s), measured like the bf16 peaks of MEASURED_PEAKS.json
+# with `python bench.py --measure-peak fp16`: torch.matmul fp16 8192^3, best of 10 (burst) and back to back
+# for 4 s (sustained, under the power cap).  The same command for bf16 gave 1924.6 / 1735.2 on that box
+# (MEASURED_PEAKS.json: 1910.6 / 1699.8).
+FP16_PEAKS = {"burst": 1819.3, "sustained": 1640.4}
+
+
+def _peaks(dtype="bf16"):
+    """(HBM GB/s, dense burst TFLOP/s, dense sustained TFLOP/s, provenance) for the compute dtype."""
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             p = json.load(f)
-        return p["hbm_gbs"], p["bf16_tflops"], p["bf16_tflops_sustained"], "measured"
+        hbm, burst, sust, kind = p["hbm_gbs"], p["bf16_tflops"], p["bf16_tflops_sustained"], "measured"
     except Exception:
-        return 6800.0, 1900.0, 1700.0, "fallback"
+        hbm, burst, sust, kind = 6800.0, 1900.0, 1700.0, "fallback"
+    if dtype == "fp16":
+        if FP16_PEAKS is not None:
+            return hbm, FP16_PEAKS["burst"], FP16_PEAKS["sustained"], "measured fp16"
+        return hbm, burst, sust, kind + " (bf16 peak: fp16 not measured)"
+    return hbm, burst, sust, kind
+
+
+def measure_peak(dtype, seconds=4.0):
+    """Dense tensor peak of one GPU: torch.matmul of 8192^3 in dtype, best of 10 (burst), and back-to-back
+    matmuls for `seconds` (sustained), CUDA events; clocks sampled meanwhile."""
+    import torch
+    dt = {"fp16": torch.float16, "bf16": torch.bfloat16}[dtype]
+    n = 8192
+    g = torch.Generator(device="cuda").manual_seed(0)
+    a = torch.randn(n, n, device="cuda", dtype=dt, generator=g)
+    b = torch.randn(n, n, device="cuda", dtype=dt, generator=g)
+    c = torch.empty(n, n, device="cuda", dtype=dt)
+    flop = 2.0 * n ** 3
+    for _ in range(5):
+        torch.matmul(a, b, out=c)
+    torch.cuda.synchronize()
+    sampler = ClockSampler(torch.cuda.current_device())
+    sampler.start()
+    best = float("inf")
+    for _ in range(10):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(); torch.matmul(a, b, out=c); e1.record()
+        torch.cuda.synchronize()
+        best = min(best, e0.elapsed_time(e1))
+    reps, t_end = 0, time.time() + seconds
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    while time.time() < t_end:
+        for _ in range(20):
+            torch.matmul(a, b, out=c)
+        reps += 20
+        torch.cuda.synchronize()
+    e1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    print(json.dumps({"peak": f"{dtype} dense", "shape": [n, n, n], "burst_tflops": flop / (best * 1e-3) / 1e12,
+                      "sustained_tflops": flop * reps / (e0.elapsed_time(e1) * 1e-3) / 1e12,
+                      "sustained_s": e0.elapsed_time(e1) * 1e-3, "matmuls": reps, "clocks": clocks,
+                      "gpu": torch.cuda.get_device_name(), "torch": torch.__version__}))
 
 
 class ClockSampler:
@@ -201,7 +259,7 @@ def run_step(step, x, target, t, seed, world):
     step.forward_loss(x, target, seed, t)            # the pair forwards, then the loss pair
     if world > 1:
         from paper_2607_01125_gb300.dp import allreduce_loss
-        allreduce_loss(step.loss_out)            # losses and a's are means over equal token counts
+        allreduce_loss(step.loss_out, ctx=step.ctx)   # losses and a's are means over equal token counts
     step.update(t, seed, t)
     return step.loss_out
 
@@ -248,31 +306,39 @@ def run_ours(args):
     launches = ctx.launch_count() - n0
     ms = start.elapsed_time(end) / args.steps
 
-    # ---- kernel timing: the same number of steps again, with the library recording CUDA events on its
-    # stream around every tensor-core pair-forward kernel (the events themselves lengthen a step by a few
-    # per cent, so the throughput above is taken without them) ----
+    # ---- kernel timing: the steps again (as many as the library's pool of event pairs covers whole), with
+    # the library recording CUDA events on its stream around every tensor-core pair-forward kernel (the
+    # events themselves lengthen a step by a few per cent, so the throughput above is taken without them) ----
+    step.flops = []
+    run_step(step, x, target, t, seed, world); t += 1          # one untimed step counts the launches per step
+    per_step = max(1, len(step.flops))
+    instr_steps = max(1, min(args.steps, TIMING_PAIRS // per_step))
     step.flops = []
     ctx.kernel_timing(True)
     barrier(); torch.cuda.synchronize()
     i_s, i_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     i_s.record()
-    for _ in range(args.steps):
+    for _ in range(instr_steps):
         run_step(step, x, target, t, seed, world); t += 1
     i_e.record()
     torch.cuda.synchronize(); barrier()
-    instr_ms = i_s.elapsed_time(i_e) / args.steps
-    gemm_flops = sum(step.flops)
-    step.flops = None
+    instr_ms = i_s.elapsed_time(i_e) / instr_steps
     kern_ms, kern_launches = ctx.kernel_time()
     ctx.kernel_timing(False)
+    if kern_launches != len(step.flops):
+        raise RuntimeError(f"timed {kern_launches} pair launches of {len(step.flops)}: the timing is incomplete")
+    gemm_flops = sum(step.flops)
+    step.flops = None
 
     # ---- end to end through the public API with host buffers: every step's inputs are copied from pinned
-    # host memory (overlapped with the previous step on a side stream) and its loss vector read back ----
-    from paper_2607_01125_gb300.model import run_from_host
+    # host memory (overlapped with the previous step on a side stream) and its loss vector read back.  The
+    # feeder's device buffers, side stream and events are made before the timed region ----
+    from paper_2607_01125_gb300.model import HostFeeder
     x_h = x.cpu().pin_memory()
     t_h = target.cpu().pin_memory() if target is not None else None
     outs_h = [torch.empty(step.loss_out.numel(), dtype=torch.float64).pin_memory() for _ in range(args.steps)]
     batches = [(x_h, t_h) if t_h is not None else (x_h,) for _ in range(args.steps)]
+    feeder = HostFeeder(batches[0])
     t_e2e = t
 
     def e2e_step(dev, i):
@@ -281,13 +347,18 @@ def run_ours(args):
     barrier(); torch.cuda.synchronize()
     e_s, e_e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e_s.record()
-    run_from_host(batches, e2e_step, outs_h)
+    feeder.run(batches, e2e_step, outs_h)
     e_e.record()
     t += args.steps
     torch.cuda.synchronize(); barrier()
     clocks = sampler.stop()
     e2e_ms = e_s.elapsed_time(e_e) / args.steps
     status = ctx.device_status()
+    replicas = None
+    if world > 1:                               # every rank must still hold the same coefficients and moments
+        from paper_2607_01125_gb300.dp import check_replicas
+        st, bad = check_replicas([step.C, step.m, step.v], ctx=ctx)
+        replicas = {"status": st, "ranks_differing_from_rank0": bad}
 
     if world > 1:
         tt = torch.tensor([ms, e2e_ms], device=dev)
@@ -295,7 +366,7 @@ def run_ours(args):
         ms, e2e_ms = float(tt[0]), float(tt[1])
     if rank != 0:
         return
-    hbm, tf_burst, tf_sust, peak_kind = _peaks()
+    hbm, tf_burst, tf_sust, peak_kind = _peaks(w.act_dtype)
     # a step of about a millisecond times its kernels as bursts; the stacks' ~100 ms steps use the sustained peak
     long_step = ms > 20.0
     peak = tf_sust if long_step else tf_burst
@@ -315,31 +386,33 @@ def run_ours(args):
                    "parallelism": f"dp{world}" if world > 1 else "single"},
         "evaluated_tokens_per_s": world * step.nb * T / (ms * 1e-3),
         "zo_steps_per_s": 1e3 / ms,
-        "pair_kernel_ms_per_step": kern_ms / args.steps,
+        "pair_kernel_ms_per_step": kern_ms / instr_steps,
         "instrumented_ms_per_step": instr_ms,
         "pair_kernel_launches": kern_launches,
+        "instrumented_steps": instr_steps,
         "basis_init_s": basis_s,
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak,
-                     "peak_kind": f"bf16 dense {'sustained' if long_step else 'burst'}, {peak_kind}",
+                     "peak_kind": f"{w.act_dtype} dense {'sustained' if long_step else 'burst'}, {peak_kind}",
                      "kernel": "pair_tc2_kernel / pair_tc_kernel (every pair-forward launch of the step, "
                                "timed alone by events on the library's stream over a second run of the same "
                                "number of steps)",
-                     "algorithmic_flops_per_step": gemm_flops / args.steps,
+                     "algorithmic_flops_per_step": gemm_flops / instr_steps,
                      "traffic": (PAIR_TRAFFIC_BYTES.get(w.name)
                                  if args.tokens is None and args.queries is None and args.rank is None else None),
-                     "traffic_unit": "bytes per step (both pair launches)"},
+                     "traffic_unit": "bytes per step (all pair launches of the step)"},
         "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": 8 * step.loss_out.numel()},
         "gpu_launches": launches,
         "clocks": clocks,
         "device_status": status,
     }
+    if replicas is not None:
+        line["replicas"] = replicas
     if args.diag:
         line["diag"] = time_diagnostics(ctx, step, dev)
-    if (world == 1 and not args.no_cpu_baseline and args.workload == DEFAULT_WORKLOAD and args.queries is None
-            and args.rank is None):
-        line["cpu_baseline"] = cpu_baseline(step, budget_s=args.cpu_budget)
+    if world == 1 and not args.no_cpu_baseline and args.queries is None and args.rank is None:
+        line["cpu_baseline"] = cpu_baseline(step, w, budget_s=args.cpu_budget)
     print(json.dumps(line))
 
 
@@ -367,25 +440,110 @@ def _oracle_mlp(weights, n_tok):
     return lay, x.double().numpy(), tgt.double().numpy()
 
 
-def cpu_baseline(step, budget_s=20.0, n_tok=256):
-    """The oracle (as it stands) on the host cores: ZO steps of the same block on a token sample."""
-    n64 = lambda t: t.detach().double().cpu().numpy()
-    lay, x, tgt = _oracle_mlp([n64(step.by_name[n].W) for n in ("gate", "up", "down")], n_tok)
+def _blas_threads():
+    """Threads of numpy's BLAS (the oracle's matrix products): threadpoolctl's count where it is installed,
+    else the host's cores (OpenBLAS's default)."""
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i["num_threads"] for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return max(n)
+    except Exception:
+        pass
+    return os.cpu_count()
+
+
+def _stack_names(kind):
+    return ["q", "k", "v", "o", "gate", "up", "down"] if kind == "llama" else ["q", "k", "v", "o", "fc1", "fc2"]
+
+
+def _oracle_decoder(w, weights, n_tok):
+    """The oracle's inputs for one full-width decoder layer of a stack (a later decoder: its input holds
+    both signs' activations, [2 n_tok, d]), outside any timing.  weights: name -> fp64 W."""
+    import numpy as np
+    from synth import lowrank_activations, random_orthonormal
+    dl = {nm: dict(W=W, U=random_orthonormal(W.shape[1], w.r, 90 + i).double().numpy(),
+                   C=np.zeros((W.shape[0], w.r)), layer_id=7 + i) for i, (nm, W) in enumerate(weights.items())}
+    x, _ = lowrank_activations(2 * n_tok, w.d_model, 64, 0.05, 77, "cpu")
+    return dl, x.double().numpy()
+
+
+def _oracle_decoder_step(w, dl, x, seed, query, t):
+    """One decoder's share of a ZO step: its pair forwards with the glue, then its layers' Adam updates with
+    the estimator scalar of the loss pair on its output.  Returns seconds of (decoder, loss)."""
+    import numpy as np
+    from oracle import graphs, loss as oloss, optim, philox
     t0 = time.time()
-    _oracle_step(lay, x, tgt, 5, 0, 1)
+    Y = graphs.stack_forward([dl], x, w.eps, seed, query, w.kind, store=w.act_dtype, first=False)
+    t1 = time.time()
+    _, _, _, a = oloss.loss_pair(Y, x.shape[0] // 2, None, w.eps)
+    t2 = time.time()
+    for l in dl.values():
+        gz = optim.zo_gradient(a, philox.perturbation(seed, l["layer_id"], query, *l["C"].shape))
+        l.setdefault("m", np.zeros_like(l["C"]))
+        l.setdefault("v", np.zeros_like(l["C"]))
+        l["C"], l["m"], l["v"] = optim.adam_step(l["C"], l["m"], l["v"], gz, LR, 0.9, 0.999, 1e-8, t)
+    t3 = time.time()
+    return (t1 - t0) + (t3 - t2), t2 - t1
+
+
+def _time_decoders(w, dl, x, n_steps, t0_step=1):
+    """Extrapolated seconds per full ZO step from n_steps timed decoder steps: n_decoder decoders plus one
+    loss pair."""
+    dec, loss = [], []
+    for i in range(n_steps):
+        d, l = _oracle_decoder_step(w, dl, x, 5, i + t0_step, i + t0_step)
+        dec.append(d)
+        loss.append(l)
+    return w.n_decoder * statistics.mean(dec) + statistics.mean(loss)
+
+
+def cpu_baseline(step, w, budget_s=20.0):
+    """The oracle (as it stands) on the host cores.  MLP block: whole ZO steps on a 256-token sample.  Stacks:
+    one full-width decoder layer (its linears, glue and Adam updates) on a 256-token sample, timed and scaled
+    to the workload's decoder count (extrapolated)."""
+    import torch
+    n64 = lambda t: t.detach().cpu().double().numpy()
+    n_tok = 256
+    if w.kind == "llama_mlp":
+        lay, x, tgt = _oracle_mlp([n64(step.by_name[n].W) for n in ("gate", "up", "down")], n_tok)
+        t0 = time.time()
+        _oracle_step(lay, x, tgt, 5, 0, 1)
+        one = time.time() - t0
+        reps = max(1, min(20, int(budget_s / max(one, 1e-3)) - 1))
+        t0 = time.time()
+        for i in range(reps):
+            _oracle_step(lay, x, tgt, 5, i + 1, i + 2)
+        dt = (time.time() - t0) / reps
+        return {"value": n_tok / dt, "unit": UNIT, "cores": _blas_threads(), "kind": "oracle",
+                "sample": f"{reps} ZO steps of the full-width Llama MLP block on {n_tok} tokens "
+                          f"(numpy fp64, default BLAS threads); {dt:.3f} s per step"}
+    from oracle import layers as olayers
+    weights = {}
+    for nm in _stack_names(w.kind):
+        lin = step.by_name[f"1.{nm}"]                  # a decoder past the first (input not shared)
+        if lin.w_scales is not None:
+            weights[nm] = olayers.dequant_int4_g128(lin.W.cpu().numpy(), lin.w_scales.float().cpu().numpy(),
+                                                    lin.d_in)
+        else:
+            weights[nm] = n64(lin.W)
+    dl, x = _oracle_decoder(w, weights, n_tok)
+    t0 = time.time()
+    _oracle_decoder_step(w, dl, x, 5, 0, 1)
     one = time.time() - t0
-    reps = max(1, min(20, int(budget_s / max(one, 1e-3)) - 1))
-    t0 = time.time()
-    for i in range(reps):
-        _oracle_step(lay, x, tgt, 5, i + 1, i + 2)
-    dt = (time.time() - t0) / reps
-    return {"value": n_tok / dt, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{reps} ZO steps of the full-width Llama MLP block on {n_tok} tokens "
-                      f"(numpy fp64, default BLAS threads); {dt:.3f} s per step"}
+    reps = max(1, min(10, int(budget_s / max(one, 1e-3)) - 1))
+    dt = _time_decoders(w, dl, x, reps, 2)
+    return {"value": n_tok / dt, "unit": UNIT, "cores": _blas_threads(), "kind": "oracle",
+            "extrapolated": True,
+            "sample": f"{reps} timed ZO-step shares of one full-width decoder layer ({len(dl)} linears, glue, "
+                      f"Adam) of {w.name} on {n_tok} tokens per perturbation (numpy fp64, default BLAS "
+                      f"threads), scaled to {w.n_decoder} decoders plus one loss pair (extrapolated): "
+                      f"{dt:.2f} s per full step"}
 
 
 def run_reference(args):
-    """The CPU oracle as the reference arm: --steps timed ZO steps on a bounded token sample."""
+    """The CPU oracle as the reference arm: --steps timed steps, each one full-width decoder layer's share of
+    a ZO step of the default workload on a bounded token sample, reported as the extrapolated full step."""
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     if rank != 0:
@@ -394,26 +552,26 @@ def run_reference(args):
     from synth import workload, normal, tensor_seed
     w = workload(DEFAULT_WORKLOAD)
     n_tok = args.ref_tokens
+    dims = {s.name.split(".")[1]: (s.d_out, s.d_in) for s in w.linears() if s.name.startswith("1.")}
     # the weights drawn on the CPU with the same shapes (the reference arm never touches the GPU)
-    weights = [normal((do, di), tensor_seed(w, "W", nm), "cpu", std=w.weight_std,
-                      dtype=torch.bfloat16).double().numpy()
-               for nm, do, di in (("gate", 14336, 4096), ("up", 14336, 4096), ("down", 4096, 14336))]
-    lay, x, tgt = _oracle_mlp(weights, n_tok)
-    t = 1
-    for _ in range(args.warmup):
-        _oracle_step(lay, x, tgt, 5, t, t); t += 1
-    t0 = time.time()
-    for _ in range(args.steps):
-        _oracle_step(lay, x, tgt, 5, t, t); t += 1
-    dt = (time.time() - t0) / args.steps
+    weights = {nm: normal(dims[nm], tensor_seed(w, "W", f"1.{nm}"), "cpu", std=w.weight_std,
+                          dtype=torch.bfloat16).double().numpy() for nm in _stack_names(w.kind)}
+    dl, x = _oracle_decoder(w, weights, n_tok)
+    for i in range(args.warmup):
+        _oracle_decoder_step(w, dl, x, 5, i + 1, i + 1)
+    dt = _time_decoders(w, dl, x, args.steps, args.warmup + 1)
     v = n_tok / dt
-    sample = f"{args.steps} ZO steps of the full-width Llama MLP block on {n_tok} tokens (numpy fp64)"
+    sample = (f"{args.steps} timed ZO-step shares of one full-width decoder layer of {w.name} on {n_tok} tokens "
+              f"per perturbation (numpy fp64), scaled to {w.n_decoder} decoders plus one loss pair "
+              f"(extrapolated)")
     print(json.dumps({
         "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f64", "data": "synthetic", "impl": "reference",
-        "config": {"workload": DEFAULT_WORKLOAD, "tokens_per_perturbation": n_tok, "r": 16, "eps": 1e-3},
-        "cpu_baseline": {"value": v, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample},
+        "config": {"workload": DEFAULT_WORKLOAD, "tokens_per_perturbation": n_tok, "r": w.r, "eps": w.eps,
+                   "adapted_linears": len(w.linears())},
+        "cpu_baseline": {"value": v, "unit": UNIT, "cores": _blas_threads(), "kind": "oracle",
+                         "sample": sample, "extrapolated": True},
         "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
 
@@ -436,10 +594,14 @@ def main():
                     help="seconds of untimed steps before the timed region (clocks reach their loaded state)")
     ap.add_argument("--cpu-budget", type=float, default=20.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--ref-tokens", type=int, default=64, help="tokens per oracle step in the reference arm")
+    ap.add_argument("--measure-peak", choices=["fp16", "bf16"], default=None,
+                    help="only measure the dense tensor peak of this dtype (torch.matmul 8192^3) and exit")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
-    if args.impl == "reference":
+    if args.measure_peak:
+        measure_peak(args.measure_peak)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)

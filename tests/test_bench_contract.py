@@ -28,14 +28,15 @@ def test_reference_arm_prints_one_contract_line():
         assert k in d, k
     assert d["impl"] == "reference" and d["n_gpus"] == 1 and d["steps"] == 1 and d["warmup"] == 3
     assert d["value"] > 0 and d["higher_is_better"] is True and d["vs_baseline"] is None
-    assert d["config"]["workload"] == "llama_mlp_bf16"
+    assert d["config"]["workload"] == "llama_stack_bf16" and d["config"]["adapted_linears"] == 224
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["unit"] == d["unit"] and cb["cores"] >= 1
-    assert cb["sample"]
+    assert cb["sample"] and cb["extrapolated"] is True and "32 decoders" in cb["sample"]
     e = d["e2e"]
     assert e["value"] == d["value"] and e["unit"] == d["unit"]
     assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
-    # tokens/s from the step time: two perturbations of 8 tokens are one ZO step's evaluated tokens, 8 its tokens
+    # tokens/s from the (extrapolated) step time: two perturbations of 8 tokens are one ZO step's evaluated
+    # tokens, 8 its tokens
     assert d["value"] == pytest.approx(8 / (d["ms_per_step"] * 1e-3), rel=1e-6)
 
 
