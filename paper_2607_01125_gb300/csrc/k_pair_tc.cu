@@ -14,6 +14,7 @@ int dispatch_fp16(Ctx* ctx, int mode, int rt, int ydtype, const TmaSet& tm, cons
 int dispatch_w4(Ctx* ctx, int mode, int rt, int ydtype, const CUtensorMap& a, const Params& p);
 int dispatch2_bf16(Ctx* ctx, int mode, int rt, int ydtype, const TmaSet& tm, const Params& p);
 int dispatch2_fp16(Ctx* ctx, int mode, int rt, int ydtype, const TmaSet& tm, const Params& p);
+int dispatch2_w4(Ctx* ctx, int mode, int ydtype, const TmaSet& tm, const Params& p);
 }  // namespace pairtc
 
 namespace {
@@ -72,6 +73,22 @@ int encode_tmap_2d_16bit(CUtensorMap* map, const void* base, int dtype, int64_t 
       dtype == ZOACT_DT_FP16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
   const CUresult res = fn(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                           CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return res == CUDA_SUCCESS ? ZOACT_OK : ZOACT_ERR_INVALID_ARG;
+}
+
+// Unswizzled boxes of 8- or 16-bit integers (INT4 packed weights, fp16 scales read as raw bits).
+int encode_tmap_2d_int(CUtensorMap* map, const void* base, int elem_bytes, int64_t rows, int64_t cols, int box_cols,
+                       int box_rows) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return ZOACT_ERR_CUDA;
+  const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)cols * elem_bytes};
+  const cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
+  const cuuint32_t estr[2] = {1u, 1u};
+  const CUtensorMapDataType dt = elem_bytes == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16;
+  const CUresult res = fn(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return res == CUDA_SUCCESS ? ZOACT_OK : ZOACT_ERR_INVALID_ARG;
 }
@@ -141,7 +158,26 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     b.rows = (int64_t)a.nb * a.T;
     return launch_pair_tc(ctx, b);
   }
-  if (a.wtype == ZOACT_DT_INT4_G128 && (a.rows >= INT4_STAGED_MIN_ROWS || big_r)) {
+  // INT4 weights.  Below 1024 rows the one-CTA kernel dequantises in the kernel; from 1024 rows W is expanded
+  // to bf16 once per call and the bf16 kernel runs (the default: measured faster, see pair_tc2_kernel.cuh).
+  // ZOACT_INT4=kernel runs stacked rows from 256 on the CTA-pair kernel with its own dequantising warps
+  // (bf16 or fp32 output, d_in a multiple of 1024); ZOACT_INT4=staged expands W at every row count.
+  const char* sel = std::getenv("ZOACT_PAIR_KERNEL");
+  const bool one_cta = sel && std::strcmp(sel, "1cta") == 0;
+  const char* lsel = std::getenv("ZOACT_LOWRANK");
+  const bool lr_epi = lsel && std::strcmp(lsel, "epilogue") == 0;
+  const char* isel = std::getenv("ZOACT_INT4");
+  const bool int4_staged = isel && std::strcmp(isel, "staged") == 0;   // expansion at any row count
+  const bool int4_kernel = isel && std::strcmp(isel, "kernel") == 0;   // CTA-pair in-kernel dequantisation
+  // (the scales' tensor map wants rows of a multiple of 16 bytes: d_in a multiple of 1024)
+  auto al16 = [](const void* q) { return q == nullptr || ((uintptr_t)q & 15u) == 0; };
+  const bool w4_two = a.wtype == ZOACT_DT_INT4_G128 && !big_r && ctx->may_allocate && !a.shared && !a.fuse_loss &&
+                      a.rows >= 2 * BM && a.xdtype == ZOACT_DT_BF16 && a.d_in % 1024 == 0 &&
+                      al16(a.w_scales) && al16(a.w_scales2) &&
+                      (a.ydtype == ZOACT_DT_BF16 || a.ydtype == ZOACT_DT_FP32) && !one_cta && !lr_epi &&
+                      int4_kernel;
+  if (a.wtype == ZOACT_DT_INT4_G128 && !w4_two &&
+      (a.rows >= INT4_STAGED_MIN_ROWS || big_r || (int4_staged && ctx->may_allocate))) {
     // staged INT4: expand W (and W2) to bf16 in context scratch, then the bf16 kernel (timed together)
     const size_t bytes = (size_t)a.d_out * a.d_in * 2;
     void* wb = scratch(ctx, SLOT_WDQ0, bytes);
@@ -177,15 +213,29 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   TmaSet tm;
   int st = encode_tmap_2d_16bit(&tm.a, a.X, a.xdtype, a.rows, a.d_in, BM);
   if (st) return st;
-  // CTA pairs (256-row tiles) once there are enough rows to fill them; INT4 in-kernel dequant stays on one CTA
-  const char* sel = std::getenv("ZOACT_PAIR_KERNEL");
-  const bool two = !w4 && a.rows >= 2 * BM && !(sel && std::strcmp(sel, "1cta") == 0);
+  // CTA pairs (256-row tiles) once there are enough rows to fill them (INT4: where w4_two allows)
+  const bool two = (w4 ? w4_two : a.rows >= 2 * BM && !one_cta);
   // CTA pairs: always 256-wide tiles.  A 256 x bn x 16 MMA measured the same time for bn = 192, 224 and 256, so
   // a tile costs the same at any of these widths and the widest needs the fewest waves (the Llama-3-8B MLP step:
   // 0.645 ms at 256 and at 224, 0.709 at 192; the OPT stack: 145.7 ms at 256, 149.1 at 224).
   const int bn = (gated || w4 || two) ? BN : choose_bn(a.rows, a.d_out, ctx->sm_count);
   const int b_box = gated ? BN / 2 : (two ? bn / 2 : bn);
-  if (w4) {
+  tm.s = tm.s2 = tm.a;
+  if (w4 && two) {
+    // packed rows and their scales by TMA, dequantised in shared memory by the kernel's own warps
+    st = encode_tmap_2d_int(&tm.b, a.W, 1, a.d_out, a.d_in / 2, BK / 2, BM);
+    if (st) return st;
+    st = encode_tmap_2d_int(&tm.s, a.w_scales, 2, a.d_out, a.d_in / 128, 8, BM);
+    if (st) return st;
+    tm.b2 = tm.b;
+    tm.s2 = tm.s;
+    if (gated) {
+      st = encode_tmap_2d_int(&tm.b2, a.W2, 1, a.d_out, a.d_in / 2, BK / 2, BM);
+      if (st) return st;
+      st = encode_tmap_2d_int(&tm.s2, a.w_scales2, 2, a.d_out, a.d_in / 128, 8, BM);
+      if (st) return st;
+    }
+  } else if (w4) {
     tm.b = tm.b2 = tm.a;                 // W arrives through the dequantising warps, not TMA
   } else {
     st = encode_tmap_2d_16bit(&tm.b, a.W, a.wtype, a.d_out, a.d_in, b_box);
@@ -197,12 +247,11 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
       tm.b2 = tm.b;
     }
   }
-  // low-rank term: on the tensor cores where the context may hold the split operands
-  const char* lsel = std::getenv("ZOACT_LOWRANK");
+  // low-rank term: on the tensor cores where the context may hold the split operands (INT4: on CTA pairs)
   int lmode = LOWRANK_EPILOGUE;
   const bool distinct = gated && a.P2 != a.P;
   int slots = 1;
-  if (!w4 && ctx->may_allocate && (big_r || !(lsel && std::strcmp(lsel, "epilogue") == 0))) {
+  if ((!w4 || two) && ctx->may_allocate && (big_r || !lr_epi)) {
     // stacked rows: the whole term on the tensor cores -- one K slot when every tile lies in one evaluation
     // block, else S slots (block index mod S) with S the most blocks a tile can span; shared inputs keep
     // +-Z p in the epilogue (C p on the tensor cores)
@@ -340,7 +389,7 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   p.Zt2 = zt2;
   p.zt_qstride = (int64_t)a.r * a.d_out;
   for (int b = 0; b < ZOACT_MAX_EVAL_BLOCKS; ++b) p.zq[b] = b < a.nb ? zq_of[b] : -1;
-  auto al16 = [](const void* q) { return q == nullptr || ((uintptr_t)q & 15u) == 0; };
+  // (al16: 16-byte alignment, defined above)
   p.vec_ok = al16(a.C) && al16(a.C2) && al16(a.P) && al16(a.P2);
   // Split tail: when the last wave of whole tiles would leave at least half of the pairs idle, each of its tiles
   // is cut into S = pairs / tail-tiles (<= 4) equal K ranges, one per pair, and the last piece of a tile to finish
@@ -371,7 +420,7 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     p.Ws2 = static_cast<const __half*>(a.w_scales2);
     st = timing_begin(ctx);
     if (st) return st;
-    st = dispatch_w4(ctx, mode, rt, a.ydtype, tm.a, p);
+    st = two ? dispatch2_w4(ctx, mode, a.ydtype, tm, p) : dispatch_w4(ctx, mode, rt, a.ydtype, tm.a, p);
     if (st) return st;
     return timing_end(ctx);
   }

@@ -14,6 +14,27 @@
 // accumulator-free barrier once all of its threads have read the tile.
 // Gated mode: the leader's half of B is W_gate, the peer's W_up, so the
 // accumulator columns are [gate | up] as in the one-CTA kernel.
+//
+// INT4 weights (W4, stacked rows with the whole low-rank term on the MMA; opt-in,
+// ZOACT_INT4=kernel): W comes as packed nibbles and never as bf16 in HBM.  Per
+// K-block each CTA's producer brings its 128 rows of packed bytes (4 KB) and
+// their fp16 scales (a box of 8 groups, 2 KB) by TMA into the stage's B slot,
+// completing on a CTA-local barrier (raw).  Eight more warps per CTA (576
+// threads) dequantise in batches of DQ_BATCH stages: they read every packed
+// half-row, synchronise, overwrite the slots with the 128-byte-swizzled bf16 B
+// half -- every weight q * s formed in fp32 (exact) and rounded once to bf16,
+// the value an expansion of W to bf16 holds -- fence the async proxy, and one
+// thread arrives on the leader's stage barriers: the batch's first with
+// cluster-scope release, the others relaxed (the MMA issuer, which waits with
+// cluster-scope acquire, takes the stages in order).  The leader's stage
+// barrier counts two dequantising arrivals besides the two producers' (whose
+// TMA on it brings only X).
+// Measured on the Llama-3-8B gate/up shapes (8192 stacked rows): one release per
+// stage made a gated call 3.3x slower than expanding W first (a cluster-scope
+// release took ~0.5 us); batches of three and eight warps bring it to 1.8x
+// (2.09 vs 1.14 ms), now bound by the pipeline: a packed block can only be
+// fetched once its B slot is free, and that TMA's latency plus the release
+// exceed one batch's MMA time.  The expansion therefore stays the default.
 #pragma once
 #include "pair_tc_kernel.cuh"
 
@@ -49,6 +70,8 @@ struct SharedState2 {
   int abort_flag;
   int epi_ok;
   int sk_last;            // split tail: this CTA's piece was the tile's last to finish
+  int dq_ok;              // INT4: the dequantising group's stage waits succeeded
+  uint64_t raw[STAGES2];  // INT4: the stage's packed weights and scales landed (CTA-local TMA)
 };
 static_assert(sizeof(SharedState2) <= 256, "barrier block outgrew its shared-memory slot");
 static_assert(SMEM2_BYTES <= 232448, "dynamic shared memory above the 227 KB a CTA may use");
@@ -78,6 +101,16 @@ __device__ __forceinline__ void arrive_expect_tx_cluster(uint32_t bar_cluster, u
 }
 __device__ __forceinline__ void arrive_cluster(uint32_t bar_cluster) {
   asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+// An arrival with cluster-scope release: shared-memory writes this CTA made before it (and fenced for the
+// async proxy) are visible to a cluster-scope acquire of the completed phase in the other CTA.
+__device__ __forceinline__ void arrive_release_cluster(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+// An arrival without ordering: only for a phase whose data an earlier release arrival (to a barrier the
+// consumer acquires first) already covers.
+__device__ __forceinline__ void arrive_relaxed_cluster(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
 // TMA tile load into this CTA's shared memory whose completion is signalled on
 // a barrier of the leader CTA of the pair.
@@ -830,9 +863,51 @@ __device__ __forceinline__ bool sk_fixup(const Params& prm, SharedState2* ss, co
   return true;
 }
 
-template <typename TO, int RT, int MODE, int AB_BF16, int SMODE = STAGE_NONE>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(num_threads(false), 1)
+// ---- INT4 dequantisation on CTA pairs ----
+constexpr int DQ_BAR = 7;                   // named barrier of the dequantising group
+constexpr int DQ2_THREADS = 256;            // dequantising warps of an INT4 CTA-pair launch (half a row each)
+constexpr int DQ_BATCH = 3;                 // stages per cluster-scope release (STAGES2 is a multiple)
+static_assert(STAGES2 % DQ_BATCH == 0, "release batches must tile the ring");
+__host__ __device__ constexpr int num_threads2(bool w4) { return 64 + EPI_THREADS + (w4 ? DQ2_THREADS : 0); }
+__host__ __device__ constexpr int epi_base2(bool w4) { return 64 + (w4 ? DQ2_THREADS : 0); }
+constexpr uint32_t W4_PACKED_BYTES = 4096;  // 128 rows x 32 packed bytes (64 weights) of one K-block
+constexpr uint32_t W4_SCALE_BYTES = 2048;   // 128 rows x 8 fp16 scale groups (the box holding this K-block's)
+
+// Eight INT4 elements of one word (element j in bits 4j..4j+3, 4-bit two's complement) times the scale s,
+// in K order as 8 bf16 (one 16-byte granule).  With v = q + 8 (the nibble XOR 8), a byte permute puts the
+// byte of elements (2b, 2b+1) into bits 8..15 under the exponent of 2^15; masking leaves the fp32 values
+// 32768 + v_lo and 32768 + 16 v_hi exactly.  One packed FMA then gives (32768 + v_lo) s - 32776 s = q_lo s
+// and (32768 + 16 v_hi)(s / 16) - 2056 s = q_hi s exactly -- every product and offset has at most 24
+// significant bits -- and the conversion rounds both to bf16 once.
+__device__ __forceinline__ uint4 dequant8_exact(uint32_t w, float s, float off_lo, float s16, float off_hi) {
+  const uint32_t x = w ^ 0x88888888u;
+  uint32_t out[4];
+#pragma unroll
+  for (int b = 0; b < 4; ++b) {
+    const uint32_t r = __byte_perm(x, 0x47000000u, 0x7504u | ((uint32_t)b << 4));   // 0x47 00 byte_b 00
+    const float2 q = ffma2(make_float2(__uint_as_float(r & 0xFF000F00u), __uint_as_float(r & 0xFF00F000u)),
+                           make_float2(s, s16), make_float2(off_lo, off_hi));
+    const __nv_bfloat162 h = __floats2bfloat162_rn(q.x, q.y);
+    out[b] = *reinterpret_cast<const uint32_t*>(&h);
+  }
+  return make_uint4(out[0], out[1], out[2], out[3]);
+}
+
+// Half `hf` (granules 4 hf .. 4 hf + 3) of row `row` of the stage's 128-byte-swizzled B half, from 16
+// packed bytes and the row's scale.
+__device__ __forceinline__ void dq2_store_half(uint32_t btile, int row, int hf, uint4 q, float s) {
+  const float off_lo = -32776.0f * s, s16 = 0.0625f * s, off_hi = -2056.0f * s;
+  const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+  for (int c = 0; c < 4; ++c)
+    tc::st_shared_v4(btile + sw128_off(row, 4 * hf + c), dequant8_exact(w[c], s, off_lo, s16, off_hi));
+}
+
+template <typename TO, int RT, int MODE, int AB_BF16, int SMODE = STAGE_NONE, bool W4 = false>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(num_threads2(W4), 1)
 pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
+  static_assert(!W4 || (SMODE == STAGE_ALL && AB_BF16 == 1 && MODE != MODE_PLAIN),
+                "INT4 CTA pairs: stacked rows with the whole low-rank term on the MMA, bf16 operands");
   constexpr int CW = MODE == MODE_GATED ? 8 : 16;   // epilogue chunk width (gated: two accumulators)
   const bool mismatch =
       (SMODE == STAGE_ALL && (prm.aug_mode != LOWRANK_ALL_ON_TC || prm.y_staged != STAGE_ALL)) ||
@@ -861,13 +936,17 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES2; ++s) {
-      tc::mbar_init(tc::smem_u32(&ss->full[s]), 2);     // one producer arrival from each CTA (leader's copy is used)
+      // one producer arrival from each CTA (leader's copy is used), and with INT4 one from each CTA's
+      // dequantising group
+      tc::mbar_init(tc::smem_u32(&ss->full[s]), W4 ? 4 : 2);
       tc::mbar_init(tc::smem_u32(&ss->empty[s]), 1);
     }
     for (int b = 0; b < 2; ++b) {
       tc::mbar_init(tc::smem_u32(&ss->tmem_full[b]), 1);
       tc::mbar_init(tc::smem_u32(&ss->tmem_empty[b]), 2);   // one arrival per CTA (leader's copy is used)
     }
+    if (W4)
+      for (int st = 0; st < STAGES2; ++st) tc::mbar_init(tc::smem_u32(&ss->raw[st]), 1);
     tc::mbar_init(tc::smem_u32(&ss->drain), 1);
     tc::mbar_init(tc::smem_u32(&ss->tload[0]), 1);
     tc::mbar_init(tc::smem_u32(&ss->tload[1]), 1);
@@ -876,6 +955,10 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
     tc::prefetch_tmap(&tm.a);
     tc::prefetch_tmap(&tm.b);
     if (MODE == MODE_GATED) tc::prefetch_tmap(&tm.b2);
+    if (W4) {
+      tc::prefetch_tmap(&tm.s);
+      if (MODE == MODE_GATED) tc::prefetch_tmap(&tm.s2);
+    }
     if (prm.aug_kb > 0) {
       tc::prefetch_tmap(&tm.aa);
       tc::prefetch_tmap(&tm.ba);
@@ -914,14 +997,23 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
         for (int kb = u.kb0; kb < u.kb1; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
           const uint32_t full_leader = tc2::map_to(tc::smem_u32(&ss->full[stage]), 0);
-          tc2::arrive_expect_tx_cluster(full_leader, stage_tx);
+          const bool aug = kb >= num_k;
+          // INT4: W's K-blocks come from the dequantising warps, only X (and the low-rank blocks) by TMA
+          tc2::arrive_expect_tx_cluster(full_leader, (W4 && !aug) ? (uint32_t)A_BYTES : stage_tx);
           const uint32_t sa = tc::smem_u32(smem + stage * STAGE2_BYTES);
           const uint32_t sb = sa + A_BYTES;
-          const bool aug = kb >= num_k;
           int kx = kb * BK, kxb = kb * BK, yb = 0;
           if (aug) aug_coords(prm, (int64_t)m_blk * BM2, BM2, kb - num_k, kx, kxb, yb);
           tc2::tma_load_2d_pair(sa, aug ? &tm.aa : &tm.a, kx, m_blk * BM2 + (int)rank * BM, full_leader);
-          if (MODE == MODE_GATED)
+          if (W4 && !aug) {
+            // this CTA's packed rows and their scales into the B slot, for the dequantising warps
+            const uint32_t raw = tc::smem_u32(&ss->raw[stage]);
+            const bool up = MODE == MODE_GATED && !leader;
+            const int y0 = MODE == MODE_GATED ? n_blk * (BN / 2) : n_blk * bn + (int)rank * bh;
+            tc::mbar_arrive_expect_tx(raw, W4_PACKED_BYTES + W4_SCALE_BYTES);
+            tc::tma_load_2d(sb, up ? &tm.b2 : &tm.b, kb * (BK / 2), y0, raw);
+            tc::tma_load_2d(sb + W4_PACKED_BYTES, up ? &tm.s2 : &tm.s, ((kb * BK) / 128) & ~7, y0, raw);
+          } else if (MODE == MODE_GATED)
             tc2::tma_load_2d_pair(sb, aug ? (leader ? &tm.ba : &tm.ba2) : (leader ? &tm.b : &tm.b2), kxb,
                                   yb + n_blk * (BN / 2), full_leader);
           else
@@ -954,7 +1046,10 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
         tc::tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
         for (int kb = u.kb0; kb < u.kb1; ++kb) {
-          if (!tc::mbar_wait(tc::smem_u32(&ss->full[stage]), phase, abort_flag, prm.status)) { ok = false; break; }
+          // INT4: the stage also carries the dequantising groups' cluster-scope release arrivals
+          const bool got = W4 ? tc::mbar_wait_cl(tc::smem_u32(&ss->full[stage]), phase, abort_flag, prm.status)
+                              : tc::mbar_wait(tc::smem_u32(&ss->full[stage]), phase, abort_flag, prm.status);
+          if (!got) { ok = false; break; }
           tc::tc_fence_after();
           const uint32_t sa = tc::smem_u32(smem + stage * STAGE2_BYTES);
           const uint32_t sb = sa + A_BYTES;
@@ -975,9 +1070,80 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
         tc::mbar_wait_drain(tc::smem_u32(&ss->drain), 0, 100000000ull);
       }
     }
+  } else if (W4 && warp < 2 + DQ2_THREADS / 32) {
+    // ---------------- INT4 dequantisation (warps 2..9, both CTAs) ----------------
+    // Batches of DQ_BATCH stages: one thread waits for all of them (packed block landed, or the stage free
+    // for a low-rank block the producer loads itself), the group reads every packed half-row, then
+    // overwrites the slots with bf16, fences the async proxy, and one thread arrives on the leader's
+    // stage barriers: the first with cluster-scope release (it orders the whole batch's writes), the
+    // others relaxed -- the MMA issuer acquires the first before it looks at the others.
+    const int dt = threadIdx.x - 64;
+    const int row = dt >> 1, hf = dt & 1;           // this thread's half of one of the CTA's 128 W rows
+    int stage = 0;
+    uint32_t phase = 0;
+    uint32_t raw_par = 0;                           // per stage: parity of its next raw phase (W blocks only)
+    int i = 0, kb = 0;
+    WorkUnit u;
+    bool live = next_unit(prm, cluster_id, n_clusters, total_k, 0, u);
+    if (live) kb = u.kb0;
+    while (live) {
+      int bst[DQ_BATCH], bkb[DQ_BATCH];
+      bool bmain[DQ_BATCH];
+      uint32_t bpar[DQ_BATCH], bphase[DQ_BATCH];
+      int nb = 0;
+#pragma unroll
+      for (int b = 0; b < DQ_BATCH; ++b) {
+        if (live) {
+          bst[b] = stage; bkb[b] = kb; bmain[b] = kb < num_k;
+          bpar[b] = (raw_par >> stage) & 1u; bphase[b] = phase;
+          if (bmain[b]) raw_par ^= 1u << stage;
+          if (++stage == STAGES2) { stage = 0; phase ^= 1u; }
+          if (++kb >= u.kb1) {
+            ++i;
+            live = next_unit(prm, cluster_id, n_clusters, total_k, i, u);
+            if (live) kb = u.kb0;
+          }
+          nb = b + 1;
+        }
+      }
+      if (dt == 0) {
+        bool ok = true;
+        for (int b = 0; b < nb && ok; ++b)
+          ok = bmain[b] ? tc::mbar_wait(tc::smem_u32(&ss->raw[bst[b]]), bpar[b], abort_flag, prm.status)
+                        : tc::mbar_wait(tc::smem_u32(&ss->empty[bst[b]]), bphase[b] ^ 1u, abort_flag, prm.status);
+        ss->dq_ok = ok ? 1 : 0;
+      }
+      tc::named_bar_sync(DQ_BAR, DQ2_THREADS);
+      if (*reinterpret_cast<volatile int*>(&ss->dq_ok) == 0) break;
+      uint4 q[DQ_BATCH];
+      float sc[DQ_BATCH];
+#pragma unroll
+      for (int b = 0; b < DQ_BATCH; ++b) {
+        if (b < nb && bmain[b]) {
+          const uint32_t sb = tc::smem_u32(smem + bst[b] * STAGE2_BYTES + A_BYTES);
+          q[b] = tc::ld_shared_v4(sb + (uint32_t)row * 32u + (uint32_t)hf * 16u);
+          const int g = (bkb[b] * BK) / 128;                      // the scale group of this K-block
+          const uint32_t sw = tc::ld_shared_b32(sb + W4_PACKED_BYTES + (uint32_t)row * 16u + (uint32_t)(g & 6) * 2u);
+          const uint16_t sh = (uint16_t)((g & 1) ? (sw >> 16) : (sw & 0xFFFFu));
+          __half hs;
+          memcpy(&hs, &sh, 2);
+          sc[b] = __half2float(hs);
+        }
+      }
+      tc::named_bar_sync(DQ_BAR, DQ2_THREADS);     // every packed row is read: overwrite the slots
+#pragma unroll
+      for (int b = 0; b < DQ_BATCH; ++b)
+        if (b < nb && bmain[b]) dq2_store_half(tc::smem_u32(smem + bst[b] * STAGE2_BYTES + A_BYTES), row, hf, q[b], sc[b]);
+      tc::fence_proxy_async_smem();                 // generic writes -> the tensor cores' reads
+      tc::named_bar_sync(DQ_BAR, DQ2_THREADS);     // the batch's half-tiles are written
+      if (dt == 0) {
+        tc2::arrive_release_cluster(tc2::map_to(tc::smem_u32(&ss->full[bst[0]]), 0));
+        for (int b = 1; b < nb; ++b) tc2::arrive_relaxed_cluster(tc2::map_to(tc::smem_u32(&ss->full[bst[b]]), 0));
+      }
+    }
   } else {
-    // ---------------- epilogue (warps 2..9, both CTAs) ----------------
-    const int etid = threadIdx.x - epi_base(false);
+    // ---------------- epilogue (warps 2..9, both CTAs; INT4: warps 10..17) ----------------
+    const int etid = threadIdx.x - epi_base2(W4);
     const int half = etid >> 7;
     const int quad = warp & 3;
     const int row_in_tile = quad * 32 + lane;

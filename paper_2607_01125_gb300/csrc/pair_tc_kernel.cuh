@@ -98,6 +98,9 @@ enum StageMode { STAGE_NONE = 0, STAGE_ALL = 1, STAGE_MIRROR = 2, STAGE_MIRROR4 
 struct TmaSet {
   CUtensorMap a, b, b2, aa, ba, ba2;
   CUtensorMap y, y16;   // output Y for staged bulk stores: 128-byte swizzled rows, and 16-column boxes
+  // INT4 on CTA pairs: b / b2 map the packed weights ([d_out, d_in/2] bytes, 32 x 128 boxes), s / s2 their
+  // fp16 scales ([d_out, d_in/128], 8 x 128 boxes)
+  CUtensorMap s, s2;
 };
 
 struct Params {

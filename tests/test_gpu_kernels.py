@@ -346,9 +346,59 @@ def test_pair_forward_int4(ctx, d_in, d_out, r, T, shared):
 
 
 @pytest.mark.parametrize("d_in,d_out,r,T,shared", [(1024, 520, 16, 600, False), (4096, 768, 8, 1100, True)])
-def test_pair_forward_int4_staged(ctx, d_in, d_out, r, T, shared):
-    # >= 1024 token rows: W is first expanded to bf16 (fp32 product q * s, one rounding), then the bf16 kernel
+def test_pair_forward_int4_staged(ctx, monkeypatch, d_in, d_out, r, T, shared):
+    # W first expanded to bf16 (fp32 product q * s, one rounding), then the bf16 kernel: a shared input from
+    # 1024 rows, and stacked rows when ZOACT_INT4=staged asks for it
+    monkeypatch.setenv("ZOACT_INT4", "staged")
     test_pair_forward_int4(ctx, d_in, d_out, r, T, shared)
+
+
+@pytest.mark.parametrize("d_in,d_out,r,T,gated,ydt", [
+    (1024, 520, 16, 200, False, torch.float32),     # 400 rows: tiles across the sign boundary (two K slots)
+    (4096, 1024, 16, 256, False, torch.bfloat16),   # 512 rows: tiles inside one sign, split last wave
+    (2048, 776, 32, 600, False, torch.float32),     # ragged N, rank 32
+    (1024, 384, 16, 300, True, torch.bfloat16),     # gated (gate rows on the leader, up rows on the peer)
+    (4096, 1024, 8, 1024, True, torch.float32),
+])
+def test_pair_forward_int4_cta_pairs(ctx, monkeypatch, d_in, d_out, r, T, gated, ydt):
+    # ZOACT_INT4=kernel, stacked rows from 256: INT4 dequantised by the CTA-pair kernel's own warps, every weight
+    # q * s rounded once to bf16 -- the values the expansion to bf16 holds, so the output is bit-identical to the
+    # staged path (same MMAs in the same order) and within the rounding of the weights of the fp64 oracle
+    eps, seed, query = 0.5, 17, 4
+    L, Wd, U, C = _int4_layer(d_in, d_out, r, 70, 3)
+    X = normal((2 * T, d_in), 71, DEV, dtype=torch.bfloat16)
+    outs = []
+    Lu = None
+    if gated:
+        Lu, Wu, Uu, Cu = _int4_layer(d_in, d_out, r, 80, 4)
+    for mode in ("kernel", "staged"):
+        monkeypatch.setenv("ZOACT_INT4", mode)
+        Y = torch.full((2 * T, d_out), float("nan"), dtype=ydt, device=DEV)
+        if gated:
+            zo.zoact_pair_forward_gated(ctx, L, Lu, X, T, False, eps, seed, query, Y)
+        else:
+            zo.zoact_pair_forward(ctx, L, X, T, False, eps, seed, query, Y)
+        torch.cuda.synchronize()
+        assert ctx.device_status() == 0
+        outs.append(Y)
+    monkeypatch.delenv("ZOACT_INT4")
+    assert torch.equal(outs[0], outs[1])
+    Xn = np64(X)
+    Zm = philox.perturbation(seed, 3, query, d_out, r)
+    ref = layers.pair_forward(Wd, np64(U), np64(C).reshape(d_out, r), Zm, Xn, eps, T, False)
+    absw = np.abs(Xn) @ np.abs(Wd).T
+    absl = np.abs(Xn @ np64(U)) @ (np.abs(np64(C).reshape(d_out, r)) + eps * np.abs(Zm)).T
+    if gated:
+        u = layers.pair_forward(Wu, np64(Uu), np64(Cu).reshape(d_out, r), philox.perturbation(seed, 4, query, d_out, r),
+                                Xn, eps, T, False)
+        ref = layers.silu(ref) * u
+        assert np.abs(np64(outs[0]) - ref).max() <= 2e-2 * np.abs(ref).max()
+        assert np.mean(np.abs(np64(outs[0]) - ref)) <= 5e-3 * np.mean(np.abs(ref))
+        return
+    # weights rounded to bf16 (2^-9 relative) plus fp32 accumulation, plus the output's own rounding
+    out_r = 2.0 ** -8 if ydt == torch.bfloat16 else 0.0
+    err = np.abs(np64(outs[0]) - ref)
+    assert np.all(err <= 2.0 ** -9 * absw + _bound(d_in, absw + absl, absl) + out_r * np.abs(ref)), err.max()
 
 
 def test_pair_forward_gated_int4(ctx):
