@@ -194,6 +194,45 @@ int zoact_pair_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X, 
                        int64_t T, int input_shared, const float* P, float eps, uint64_t seed,
                        uint64_t query, int act, void* Y, int ydtype);
 
+/* ---- RMS-normalised inputs without a normalisation pass ----
+ * The synthetic stacks normalise a linear's input, rms(x) = x / sqrt(mean(x^2)
+ * + eps) per row (zoact_rms_norm), before the next adapted linear.  That is a
+ * per-row scale 1/s, and the pair forward is linear in its input:
+ *     W (x/s) + (C +- eps Z) U^T (x/s) = (W x + (C +- eps Z) U^T x) / s,
+ * so a pair forward can take x itself (and its projection U^T x) and scale its
+ * accumulator rows.  zoact_rowscale, passed by HOST pointer, read during the call:
+ *   in_scale  [rows(X)] fp32 (DEVICE, or NULL): output row t (both the W x and
+ *             the low-rank terms) is multiplied by in_scale[t] before the
+ *             activation / SiLU gate.
+ *   out_sumsq [ceil(d_out / 64), rows(Y)] fp32 (DEVICE, or NULL): element
+ *             [p][t] receives the sum of squares of Y's stored values (after
+ *             rounding to ydtype) in columns [64 p, 64 p + 64) of row t, ready
+ *             for zoact_rms_scale.
+ * zoact_pair_forward_rs / zoact_pair_forward_gated_rs are zoact_pair_forward /
+ * _gated with row scales.  They apply them on the CTA-pair kernel's stacked-row
+ * path only: input_shared == 0, rows(X) >= 256, 16-bit X, and INT4 weights from
+ * 1024 rows; any other request returns ZOACT_ERR_UNSUPPORTED before anything is
+ * launched (callers then normalise explicitly).  rs == NULL or both pointers
+ * NULL is the plain call.  Relative to normalising the stored input first, the
+ * outputs skip one rounding of the normalised input to the activation dtype.
+ * zoact_rms_scale: inv_scale[t] = 1 / sqrt(sum_p sumsq[p][t] / n + eps) over the
+ * ceil(n / 64) parts of a [ceil(n / 64), rows] array, in part order (n = the
+ * producer's d_out).  The paper has no counterpart: this is how the device
+ * runs the synthetic graphs' normalisations.                                    */
+typedef struct zoact_rowscale {
+  const float* in_scale;
+  float* out_sumsq;
+} zoact_rowscale;
+int zoact_pair_forward_rs(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype,
+                          int64_t T, int input_shared, const float* P, float eps, uint64_t seed,
+                          uint64_t query, int act, void* Y, int ydtype, const zoact_rowscale* rs);
+int zoact_pair_forward_gated_rs(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up,
+                                const void* X, int xdtype, int64_t T, int input_shared,
+                                const float* P_gate, const float* P_up, float eps, uint64_t seed,
+                                uint64_t query, void* H, int ydtype, const zoact_rowscale* rs);
+int zoact_rms_scale(zoact_ctx* ctx, const float* sumsq, int64_t rows, int32_t n, float eps,
+                    float* inv_scale);
+
 /* ---- the pair forward without any allocation ----
  * The paper has no counterpart: this entry point exists for callers that must
  * not allocate device memory (a framework whose allocator owns all device

@@ -39,7 +39,7 @@ EXPORTS = [
     "zoact_adam_step_multi", "zoact_sgd_step_multi", "zoact_basis_prepared_bytes", "zoact_basis_prepare",
     "zoact_lowrank_proj_prepared", "zoact_subspace_overlap", "zoact_gradient_energy", "zoact_kernel_timing",
     "zoact_kernel_time", "zoact_pair_forward_loss", "zoact_debug_timeout", "zoact_mean_over_ranks",
-    "zoact_arena_hash",
+    "zoact_arena_hash", "zoact_pair_forward_rs", "zoact_pair_forward_gated_rs", "zoact_rms_scale",
 ]
 
 
@@ -58,6 +58,10 @@ class zoact_layer(ctypes.Structure):
 class zoact_coeff_block(ctypes.Structure):
     _fields_ = [("offset", ctypes.c_int64), ("d_out", ctypes.c_int32), ("r", ctypes.c_int32),
                 ("layer_id", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+
+
+class zoact_rowscale(ctypes.Structure):
+    _fields_ = [("in_scale", ctypes.c_void_p), ("out_sumsq", ctypes.c_void_p)]
 
 
 class zoact_eval_blocks(ctypes.Structure):
@@ -132,6 +136,11 @@ def load():
         "zoact_sgd_step_multi": [P, P, I64, ctypes.POINTER(zoact_coeff_block), I32, P, I32,
                                  ctypes.POINTER(ctypes.c_uint64), F32, U64],
         "zoact_mean_over_ranks": [P, P, I64, I32],
+        "zoact_pair_forward_rs": [P, ctypes.POINTER(zoact_layer), P, I32, I64, I32, P, F32, U64, U64, I32, P, I32,
+                                  ctypes.POINTER(zoact_rowscale)],
+        "zoact_pair_forward_gated_rs": [P, ctypes.POINTER(zoact_layer), ctypes.POINTER(zoact_layer), P, I32, I64, I32,
+                                        P, P, F32, U64, U64, P, I32, ctypes.POINTER(zoact_rowscale)],
+        "zoact_rms_scale": [P, P, I64, I32, F32, P],
         "zoact_arena_hash": [P, P, I64, P],
     }
     for name, argtypes in sig.items():
@@ -421,3 +430,38 @@ def zoact_arena_hash(ctx, t, out):
     if nbytes % 4 or out.dtype != torch.int64 or out.numel() != 1:
         raise ValueError("zoact_arena_hash: a tensor of whole 32-bit words and a one-element int64 output")
     _check("zoact_arena_hash", load().zoact_arena_hash(ctx.handle, _ptr(t), nbytes // 4, _ptr(out)))
+
+
+def rowscale_parts(d_out):
+    """Rows of the out_sumsq array a pair forward with row scales writes for d_out output columns."""
+    return (int(d_out) + 63) // 64
+
+
+def _rowscale(in_scale, out_sumsq):
+    return zoact_rowscale(in_scale=None if in_scale is None else _ptr(in_scale).value,
+                          out_sumsq=None if out_sumsq is None else _ptr(out_sumsq).value)
+
+
+def zoact_pair_forward_rs(ctx, layer, X, T, input_shared, eps, seed, query, Y, P=None, act=ACT_NONE, in_scale=None,
+                          out_sumsq=None):
+    """zoact_pair_forward with row scales (see include/zoact.h); raises ZoactError with ZOACT_ERR_UNSUPPORTED
+    where the launch cannot apply them."""
+    rs = _rowscale(in_scale, out_sumsq)
+    _check("zoact_pair_forward_rs", load().zoact_pair_forward_rs(
+        ctx.handle, ctypes.byref(layer), _ptr(X), _dt(X), int(T), int(input_shared), _ptr(P), float(eps), int(seed),
+        int(query), int(act), _ptr(Y), _dt(Y), ctypes.byref(rs)))
+
+
+def zoact_pair_forward_gated_rs(ctx, gate, up, X, T, input_shared, eps, seed, query, H, P_gate=None, P_up=None,
+                                in_scale=None, out_sumsq=None):
+    rs = _rowscale(in_scale, out_sumsq)
+    _check("zoact_pair_forward_gated_rs", load().zoact_pair_forward_gated_rs(
+        ctx.handle, ctypes.byref(gate), ctypes.byref(up), _ptr(X), _dt(X), int(T), int(input_shared), _ptr(P_gate),
+        _ptr(P_up), float(eps), int(seed), int(query), _ptr(H), _dt(H), ctypes.byref(rs)))
+
+
+def zoact_rms_scale(ctx, sumsq, n, inv_scale, eps=1e-5):
+    """inv_scale [rows] = 1 / sqrt(sum_p sumsq[p] / n + eps) for sumsq [rowscale_parts(n), rows]."""
+    rows = sumsq.shape[-1]
+    _check("zoact_rms_scale", load().zoact_rms_scale(ctx.handle, _ptr(sumsq), int(rows), int(n), float(eps),
+                                                      _ptr(inv_scale)))

@@ -375,7 +375,8 @@ struct FusedLoss {
 
 static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* L2, const void* X, int xdtype,
                        int64_t T, int input_shared, const float* P, const float* P2, const zoact_eval_blocks* blk,
-                       uint64_t seed, int act, void* Y, int ydtype, const FusedLoss* fl = nullptr) {
+                       uint64_t seed, int act, void* Y, int ydtype, const FusedLoss* fl = nullptr,
+                       const zoact_rowscale* rs = nullptr) {
   if (check_eval_blocks(blk)) return ZOACT_ERR_INVALID_ARG;
   int st = check_layer(L);
   if (st) return st;
@@ -402,6 +403,14 @@ static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* 
   if (L->d_out % 8 != 0) return ZOACT_ERR_INVALID_ARG;
   if (T > ((int64_t)1 << 40) / blk->n_blocks) return ZOACT_ERR_INVALID_ARG;
   const int64_t rows = input_shared ? T : blk->n_blocks * T;
+  const bool rowscale = rs && (rs->in_scale || rs->out_sumsq);
+  if (rowscale) {
+    auto al4 = [](const void* q) { return ((uintptr_t)q & 3u) == 0; };
+    if ((rs->in_scale && !al4(rs->in_scale)) || (rs->out_sumsq && !al4(rs->out_sumsq))) return ZOACT_ERR_INVALID_ARG;
+    // before anything is launched: the kernels that apply row scales serve stacked rows from 256 on CTA pairs
+    if (fl || !pair_rowscale_supported(ctx, rows, input_shared, xdtype, L->wtype, blk->n_blocks))
+      return ZOACT_ERR_UNSUPPORTED;
+  }
   // projection(s) U^T x, unless the caller passed them
   if (!P) {
     float* p = static_cast<float*>(scratch(ctx, SLOT_P0, (size_t)rows * L->r * sizeof(float)));
@@ -428,6 +437,7 @@ static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* 
   a.seed = seed; a.layer_id = L->layer_id;
   if (L2) { a.W2 = L2->W; a.w_scales2 = L2->w_scales; a.P2 = P2; a.C2 = L2->C; a.layer_id2 = L2->layer_id; }
   if (fl) { a.fuse_loss = 1; a.target = fl->target; a.loss_out = fl->out; a.loss_eps = fl->eps; }
+  if (rowscale) { a.in_scale = rs->in_scale; a.out_sumsq = rs->out_sumsq; }
   if (xdtype == ZOACT_DT_FP32) return launch_pair_simt(ctx, a);
   return launch_pair_tc(ctx, a);
 }
@@ -464,6 +474,35 @@ int zoact_multi_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoa
   if (xdtype == ZOACT_DT_FP32) return ZOACT_ERR_UNSUPPORTED;
   return pair_common(ctx, gate, up, X, xdtype, T, input_shared, P_gate, P_up, blocks, seed, ZOACT_ACT_NONE, H,
                      ydtype);
+}
+
+int zoact_pair_forward_rs(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype, int64_t T,
+                          int input_shared, const float* P, float eps, uint64_t seed, uint64_t query, int act, void* Y,
+                          int ydtype, const zoact_rowscale* rs) {
+  ZOACT_ENTER(ctx);
+  const zoact_eval_blocks b = pair_blocks(eps, query);
+  return pair_common(ctx, layer, nullptr, X, xdtype, T, input_shared, P, nullptr, &b, seed, act, Y, ydtype, nullptr,
+                     rs);
+}
+
+int zoact_pair_forward_gated_rs(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up, const void* X,
+                                int xdtype, int64_t T, int input_shared, const float* P_gate, const float* P_up,
+                                float eps, uint64_t seed, uint64_t query, void* H, int ydtype,
+                                const zoact_rowscale* rs) {
+  ZOACT_ENTER(ctx);
+  if (!gate || !up) return ZOACT_ERR_INVALID_ARG;
+  if (xdtype == ZOACT_DT_FP32) return ZOACT_ERR_UNSUPPORTED;
+  const zoact_eval_blocks b = pair_blocks(eps, query);
+  return pair_common(ctx, gate, up, X, xdtype, T, input_shared, P_gate, P_up, &b, seed, ZOACT_ACT_NONE, H, ydtype,
+                     nullptr, rs);
+}
+
+int zoact_rms_scale(zoact_ctx* ctx, const float* sumsq, int64_t rows, int32_t n, float eps, float* inv_scale) {
+  ZOACT_ENTER(ctx);
+  if (rows < 0 || n <= 0 || !(eps >= 0.0f)) return ZOACT_ERR_INVALID_ARG;
+  if (rows == 0) return ZOACT_OK;
+  if (!sumsq || !inv_scale || ((uintptr_t)sumsq & 3u) || ((uintptr_t)inv_scale & 3u)) return ZOACT_ERR_INVALID_ARG;
+  return launch_rms_scale(ctx, sumsq, rows, n, eps, inv_scale);
 }
 
 int zoact_pair_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up, const void* X,

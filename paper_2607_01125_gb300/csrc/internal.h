@@ -175,7 +175,16 @@ struct PairArgs {
   const void* target;   // [T, d_out] of ydtype, or nullptr (mean of squares)
   double* loss_out;     // [4] = {L+, L-, D, a}
   float loss_eps;
+  // row scales (zoact_pair_forward_rs): in_scale [rows] multiplies each output row before the activation;
+  // out_sumsq [ceil(d_out / 64), nb T] receives per-64-column-part sums of squares of the stored outputs
+  const float* in_scale;
+  float* out_sumsq;
 };
+// Whether a launch with row scales runs on a kernel that applies them (CTA pairs, stacked rows, the whole
+// low-rank term on the MMA, staged output) -- decided before anything is launched.
+bool pair_rowscale_supported(const Ctx* ctx, int64_t rows, int shared, int xdtype, int wtype, int nb);
+// inv[t] = 1 / sqrt(sum_p parts[p][t] / n + eps) over the ceil(n / 64) parts, in part order.
+int launch_rms_scale(Ctx* ctx, const float* parts, int64_t rows, int n, float eps, float* inv);
 // The two-sided pair as evaluation blocks: {+eps, -eps} with the same query.
 inline void set_pair_blocks(PairArgs& a, float eps, uint64_t query) {
   a.nb = 2;

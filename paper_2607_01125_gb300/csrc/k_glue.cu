@@ -223,7 +223,43 @@ int mix_dispatch(Ctx* ctx, const T* q, const T* k, const T* v, T* Y, int64_t row
   return ZOACT_OK;
 }
 
+// 1/s per row from the per-part sums of squares a pair forward's epilogue wrote: 32 rows per block (one per
+// lane), the parts split over the 8 warps (warp w takes parts w, w + 8, ...), the 8 warp sums added in warp
+// order -- a fixed order, so the result is bit-reproducible.
+constexpr int RS_WARPS = 8;
+__global__ void __launch_bounds__(32 * RS_WARPS)
+rms_scale_kernel(const float* __restrict__ parts, int64_t rows, int n_parts, int n, float eps, float* __restrict__ inv) {
+  pdl_wait();                              // the partial sums written by the previous kernel
+  pdl_trigger();
+  __shared__ float red[RS_WARPS][32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t t = (int64_t)blockIdx.x * 32 + lane;
+  float s = 0.f;
+  if (t < rows) {
+#pragma unroll 4
+    for (int p = warp; p < n_parts; p += RS_WARPS) s += __ldg(parts + (int64_t)p * rows + t);
+  }
+  red[warp][lane] = s;
+  __syncthreads();
+  if (warp == 0 && t < rows) {
+    float tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < RS_WARPS; ++w) tot += red[w][lane];
+    inv[t] = rsqrtf(tot / (float)n + eps);
+  }
+}
+
 }  // namespace
+
+int launch_rms_scale(Ctx* ctx, const float* parts, int64_t rows, int n, float eps, float* inv) {
+  if (rows <= 0) return ZOACT_OK;
+  const int64_t blocks = (rows + 31) / 32;
+  if (blocks > 0x7fffffff) return ZOACT_ERR_UNSUPPORTED;
+  ZOACT_CUDA_TRY(launch_pdl(ctx, rms_scale_kernel, dim3((unsigned)blocks), dim3(32 * RS_WARPS), 0, parts, rows,
+                            (n + 63) / 64, n, eps, inv));
+  ++ctx->n_launch;
+  return ZOACT_OK;
+}
 
 int launch_rms_norm(Ctx* ctx, const void* X, int dtype, int64_t rows, int n, float eps, void* Y) {
   if (rows <= 0) return ZOACT_OK;

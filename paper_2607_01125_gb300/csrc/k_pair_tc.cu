@@ -128,6 +128,22 @@ int encode_tmap_store3(CUtensorMap* map, void* base, int ydtype, int64_t nb, int
   return res == CUDA_SUCCESS ? ZOACT_OK : ZOACT_ERR_INVALID_ARG;
 }
 
+bool pair_rowscale_supported(const Ctx* ctx, int64_t rows, int shared, int xdtype, int wtype, int nb) {
+  using namespace pairtc;
+  if (!ctx->may_allocate || shared || rows < 2 * BM || nb < 1) return false;
+  if (xdtype != ZOACT_DT_BF16 && xdtype != ZOACT_DT_FP16) return false;
+  const char* sel = std::getenv("ZOACT_PAIR_KERNEL");
+  const char* lsel = std::getenv("ZOACT_LOWRANK");
+  if ((sel && std::strcmp(sel, "1cta") == 0) || (lsel && std::strcmp(lsel, "epilogue") == 0)) return false;
+  if (wtype == ZOACT_DT_INT4_G128) {
+    // INT4 reaches the CTA-pair kernel expanded to bf16 (from 1024 rows, or ZOACT_INT4=staged) or with
+    // ZOACT_INT4=kernel; below 1024 rows the one-CTA kernel dequantises it
+    const char* isel = std::getenv("ZOACT_INT4");
+    return rows >= INT4_STAGED_MIN_ROWS || (isel && (std::strcmp(isel, "staged") == 0 || std::strcmp(isel, "kernel") == 0));
+  }
+  return true;
+}
+
 int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   using namespace pairtc;
   // ranks above 32 have no epilogue tables: the low-rank term must ride the MMA, which needs stacked rows
@@ -381,6 +397,10 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     tm.y16 = tm.y;
     p.y_staged = STAGE_MULTI4;
   }
+  // row scales ride the staged epilogue of stacked rows only (pair_rowscale_supported screens the rest first)
+  if ((a.in_scale || a.out_sumsq) && p.y_staged != STAGE_ALL) return ZOACT_ERR_UNSUPPORTED;
+  p.in_scale = a.in_scale;
+  p.out_sumsq = a.out_sumsq;
   p.aug_kb = lmode == LOWRANK_EPILOGUE ? 0 : slots * ka_tot / BK;
   p.aug_kb_slot = ka_tot / BK;
   p.aug_slots = slots;

@@ -204,15 +204,29 @@ __device__ __forceinline__ bool epi_all_staged(const Params& prm, const TmaSet& 
   constexpr int NC = 16;            // columns of a narrow chunk (unswizzled rows of 16 * EB bytes)
   if (!epi_wait_full(ss, buf, acc_phase, abort_flag, prm.status, etid)) return false;
   const int ncol_tile = GATED ? BN / 2 : bn;
-  const int wcols = ncol_tile / 2;  // this warpgroup's columns, a multiple of 16
+  const int wcols = ncol_tile / 2;  // this warpgroup's columns, a multiple of 16 (of 64 with row scales)
   const int cb = half * wcols;
   const bool issuer = (etid & 127) == 0;
   const uint32_t sbuf = tc::smem_u32(stg + half * STG_BYTES);
+  const int64_t row = row0 + rl;
+  const bool row_ok = row < prm.rows;
+  // row scales: the input row's 1/s (uniform test), and this row's running sum of squares of the stored
+  // outputs of the current 64-column part
+  const bool scaled = prm.in_scale != nullptr;
+  const float rs = scaled && row_ok ? __ldg(prm.in_scale + row) : 1.f;
+  const bool sums = prm.out_sumsq != nullptr;
+  float ssq = 0.f;
+  int part = -1;
   for (int c = 0; c < wcols;) {
     const int n = n_blk * ncol_tile + cb + c;
     if (n >= prm.d_out) break;                      // uniform over the warpgroup
     const bool full = wcols - c >= CC;
     const int cw = full ? CC : NC;
+    if (sums && (n >> 6) != part) {                 // a new 64-column part (parts never straddle chunks)
+      if (part >= 0 && row_ok) prm.out_sumsq[(int64_t)part * prm.rows + row] = ssq;
+      part = n >> 6;
+      ssq = 0.f;
+    }
     if (issuer && pending) tc::bulk_wait_read0();   // the buffer's previous store has read it
     tc::named_bar_sync(4 + half, 128);
     if (full) {
@@ -224,12 +238,27 @@ __device__ __forceinline__ bool epi_all_staged(const Params& prm, const TmaSet& 
           float u[32];
           tc::tmem_ld32(t_row + (uint32_t)(cb + c + p), v);
           tc::tmem_ld32(t_row + (uint32_t)(BN / 2 + cb + c + p), u);
+          if (scaled) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) { v[i] *= rs; u[i] *= rs; }
+          }
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = silu_fast(v[i]) * u[i];
         } else {
           tc::tmem_ld32(t_row + (uint32_t)(cb + c + p), v);
+          if (scaled) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] *= rs;
+          }
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = apply_act(v[i], prm.act);
+        }
+        if (sums) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float y = to_f32<TO>(from_f32<TO>(v[i]));   // the value Y stores
+            if (n + p + i < prm.d_out) ssq = fmaf(y, y, ssq);
+          }
         }
         stage_granules<TO, 32>(sbuf, rl, p, v, true);
       }
@@ -239,12 +268,27 @@ __device__ __forceinline__ bool epi_all_staged(const Params& prm, const TmaSet& 
         float u[16];
         tc::tmem_ld16(t_row + (uint32_t)(cb + c), v);
         tc::tmem_ld16(t_row + (uint32_t)(BN / 2 + cb + c), u);
+        if (scaled) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) { v[i] *= rs; u[i] *= rs; }
+        }
 #pragma unroll
         for (int i = 0; i < 16; ++i) v[i] = silu_fast(v[i]) * u[i];
       } else {
         tc::tmem_ld16(t_row + (uint32_t)(cb + c), v);
+        if (scaled) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) v[i] *= rs;
+        }
 #pragma unroll
         for (int i = 0; i < 16; ++i) v[i] = apply_act(v[i], prm.act);
+      }
+      if (sums) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float y = to_f32<TO>(from_f32<TO>(v[i]));
+          if (n + i < prm.d_out) ssq = fmaf(y, y, ssq);
+        }
       }
       stage_granules<TO, 16>(sbuf, rl, 0, v, false);
     }
@@ -257,6 +301,7 @@ __device__ __forceinline__ bool epi_all_staged(const Params& prm, const TmaSet& 
     }
     c += cw;
   }
+  if (sums && part >= 0 && row_ok) prm.out_sumsq[(int64_t)part * prm.rows + row] = ssq;
   return true;
 }
 

@@ -150,6 +150,11 @@ struct Params {
   // split tail (CTA-pair kernel): tiles [sk_first, sk_first + sk_tiles) are each cut into sk_split equal
   // K ranges, one per pair (sk_tiles = 0: every tile whole); sk_part holds one 128 x BN fp32 partial
   // accumulator per pair and CTA, sk_ticket one counter per tail tile and CTA (zero between launches)
+  // row scales (CTA-pair staged epilogue of stacked rows only): in_scale [rows] multiplies every accumulator row
+  // before the activation (an RMS-normalised input given unnormalised); out_sumsq [ceil(d_out / 64), rows]
+  // receives, per 64-column part, the row's sum of squares of the stored (rounded) outputs
+  const float* in_scale;
+  float* out_sumsq;
   int sk_first, sk_tiles, sk_split;
   float* sk_part;
   unsigned int* sk_ticket;

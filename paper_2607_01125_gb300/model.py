@@ -101,6 +101,8 @@ class ZOStep:
         # forward_loss fuses the loss pair into the last linear when set; off by default: the fused epilogue
         # lengthens the Llama-3-8B down launch by more than the separate loss launch takes
         self.fuse_loss = False
+        # stacks: RMS normalisations as row scales of the pair forwards where the library applies them
+        self.row_scales = True
         self._utc = {}
         self.prepare_bases()
 
@@ -162,14 +164,40 @@ class ZOStep:
     def points(self, query):
         return Z.one_sided_blocks(self.eps, self.query_ids(query))
 
-    def pair(self, name, X, shared, seed, query, out_key, act=Z.ACT_NONE, fused=None):
+    def _sums(self, key, d_out, rows):
+        """The out_sumsq array of a pair forward with row scales, and the 1/rms vector made from it."""
+        return (self.buf(f"ss_{key}", Z.rowscale_parts(d_out), rows, torch.float32),
+                self.buf(f"inv_{key}", 1, rows, torch.float32).view(rows))
+
+    def pair(self, name, X, shared, seed, query, out_key, act=Z.ACT_NONE, fused=None, in_scale=None, sums=False):
         """fused = (target, out): the last linear with the loss pair fused (zoact_pair_forward_loss); returns None
-        when that ran, else (the launch does not qualify) the output as without it."""
+        when that ran, else (the launch does not qualify) the output as without it.
+
+        Row scales (two-sided stacked rows): in_scale [rows] is 1/rms of X's rows, applied to the output rows
+        (X is the unnormalised input).  sums=True returns (Y, 1/rms of Y's rows) from the partial sums of squares
+        the launch writes, or (Y, None) where the launch cannot write them (the caller then normalises Y)."""
         l = self.by_name[name]
         if self.capture is not None:
             self.capture(name, X[:self.T])
         P = self._proj(l, X, 0)
         flops = 2.0 * X.shape[0] * l.d_in * l.d_out
+        if in_scale is not None or sums:
+            Y = self.buf(out_key, self.nb * self.T, l.d_out)
+            ss, inv = self._sums(out_key, l.d_out, Y.shape[0]) if sums else (None, None)
+            try:
+                self._counted(lambda: Z.zoact_pair_forward_rs(self.ctx, l.layer, X, self.T, shared, self.eps, seed,
+                                                              query, Y, P=P, act=act, in_scale=in_scale,
+                                                              out_sumsq=ss), flops)
+            except Z.ZoactError as e:
+                if e.status != Z.ZOACT_ERR_UNSUPPORTED or in_scale is not None:
+                    raise
+                Y = self.pair(name, X, shared, seed, query, out_key, act)
+                return (Y, None) if sums else Y
+            self._wrote(Y)
+            if sums:
+                Z.zoact_rms_scale(self.ctx, ss, l.d_out, inv)
+                return Y, inv
+            return Y
         if fused is not None and self.n_queries is None and not shared:
             target, out = fused
             try:
@@ -191,7 +219,8 @@ class ZOStep:
         self._wrote(Y)
         return Y
 
-    def gated(self, gname, uname, X, shared, seed, query, out_key):
+    def gated(self, gname, uname, X, shared, seed, query, out_key, in_scale=None, sums=False):
+        """silu(gate X) * up X; row scales as in pair()."""
         g, u = self.by_name[gname], self.by_name[uname]
         if self.capture is not None:
             self.capture(gname, X[:self.T])
@@ -200,6 +229,22 @@ class ZOStep:
         Pu = self._proj(u, X, 1)
         H = self.buf(out_key, self.nb * self.T, g.d_out)
         flops = 2.0 * X.shape[0] * g.d_in * g.d_out * 2
+        if in_scale is not None or sums:
+            ss, inv = self._sums(out_key, g.d_out, H.shape[0]) if sums else (None, None)
+            try:
+                self._counted(lambda: Z.zoact_pair_forward_gated_rs(self.ctx, g.layer, u.layer, X, self.T, shared,
+                                                                    self.eps, seed, query, H, P_gate=Pg, P_up=Pu,
+                                                                    in_scale=in_scale, out_sumsq=ss), flops)
+            except Z.ZoactError as e:
+                if e.status != Z.ZOACT_ERR_UNSUPPORTED or in_scale is not None:
+                    raise
+                H = self.gated(gname, uname, X, shared, seed, query, out_key)
+                return (H, None) if sums else H
+            self._wrote(H)
+            if sums:
+                Z.zoact_rms_scale(self.ctx, ss, g.d_out, inv)
+                return H, inv
+            return H
         if self.n_queries is None:
             fn = lambda: Z.zoact_pair_forward_gated(self.ctx, g.layer, u.layer, X, self.T, shared, self.eps, seed,
                                                     query, H, P_gate=Pg, P_up=Pu)
@@ -243,34 +288,68 @@ class ZOStep:
         return self.loss_out
 
     def _stack(self, x, seed, query, fused=None):
+        """The stack's decoders.  With row scales (two-sided steps outside calibration, where the library applies
+        them) the RMS normalisations of o, of the MLP hidden and of each decoder's output are not separate passes:
+        the producing pair forward writes per-row sums of squares, zoact_rms_scale turns them into 1/rms, and the
+        consuming pair forward scales its rows (include/zoact.h, row scales).  Otherwise, and wherever a launch
+        cannot apply them, the normalised tensor is written by zoact_rms_norm first."""
         T = self.T
         n_dec = len(self.linears) // (7 if self.kind == "llama" else 6)
-        h = x
+        rs = self.row_scales and self.capture is None and self.n_queries is None
+        h, inv_h = x, None
         shared = True
         for L in range(n_dec):
             if self.on_decoder is not None:
                 self.on_decoder(L, h)
+            last = L == n_dec - 1
             rows = T if shared else self.nb * T
-            a = self._glue_rms(h, f"a{rows}")
-            q = self.pair(f"{L}.q", a, shared, seed, query, "q")
-            k = self.pair(f"{L}.k", a, shared, seed, query, "k")
-            v = self.pair(f"{L}.v", a, shared, seed, query, "v")
+            if inv_h is None:
+                a = self._glue_rms(h, f"a{rows}")
+                q = self.pair(f"{L}.q", a, shared, seed, query, "q")
+                k = self.pair(f"{L}.k", a, shared, seed, query, "k")
+                v = self.pair(f"{L}.v", a, shared, seed, query, "v")
+            else:
+                q = self.pair(f"{L}.q", h, False, seed, query, "q", in_scale=inv_h)
+                k = self.pair(f"{L}.k", h, False, seed, query, "k", in_scale=inv_h)
+                v = self.pair(f"{L}.v", h, False, seed, query, "v", in_scale=inv_h)
             shared = False
             mix = self.buf("mix", self.nb * T, q.shape[1])
             Z.zoact_mix_rms(self.ctx, q, k, v, mix, self.n_rep if self.kind == "llama" else 1, self.head_dim)
             self._wrote(mix)
-            o = self.pair(f"{L}.o", mix, False, seed, query, "o")
-            b = self._glue_rms(o, "b")
-            if self.kind == "llama":
-                H = self.gated(f"{L}.gate", f"{L}.up", b, False, seed, query, "hmlp")
-                Hn = self._glue_rms(H, "hmlp_n")
-                h = self.pair(f"{L}.down", Hn, False, seed, query, "h" if L % 2 == 0 else "h2",
-                              fused=fused if L == n_dec - 1 else None)
+            inv_o = None
+            if rs:
+                o, inv_o = self.pair(f"{L}.o", mix, False, seed, query, "o", sums=True)
             else:
-                f = self.pair(f"{L}.fc1", b, False, seed, query, "f", act=Z.ACT_RELU)
-                fn = self._glue_rms(f, "f_n")
-                h = self.pair(f"{L}.fc2", fn, False, seed, query, "h" if L % 2 == 0 else "h2",
-                              fused=fused if L == n_dec - 1 else None)
+                o = self.pair(f"{L}.o", mix, False, seed, query, "o")
+            b, sb = (o, inv_o) if inv_o is not None else (self._glue_rms(o, "b"), None)
+            out_key = "h" if L % 2 == 0 else "h2"
+            if self.kind == "llama":
+                inv_m = None
+                if sb is not None:
+                    H, inv_m = self.gated(f"{L}.gate", f"{L}.up", b, False, seed, query, "hmlp", in_scale=sb, sums=True)
+                else:
+                    H = self.gated(f"{L}.gate", f"{L}.up", b, False, seed, query, "hmlp")
+                m, sm, lname = (H, inv_m, f"{L}.down") if inv_m is not None else (self._glue_rms(H, "hmlp_n"), None,
+                                                                                  f"{L}.down")
+            else:
+                inv_f = None
+                if sb is not None:
+                    f, inv_f = self.pair(f"{L}.fc1", b, False, seed, query, "f", act=Z.ACT_RELU, in_scale=sb, sums=True)
+                else:
+                    f = self.pair(f"{L}.fc1", b, False, seed, query, "f", act=Z.ACT_RELU)
+                m, sm, lname = (f, inv_f, f"{L}.fc2") if inv_f is not None else (self._glue_rms(f, "f_n"), None,
+                                                                                 f"{L}.fc2")
+            inv_h = None
+            if sm is not None and last and fused is not None:
+                # the fused loss pair takes a normalised input: normalise it explicitly for that launch
+                m, sm = self._glue_rms(m, "hmlp_n" if self.kind == "llama" else "f_n"), None
+            if sm is not None:
+                if last:
+                    h = self.pair(lname, m, False, seed, query, out_key, in_scale=sm)
+                else:
+                    h, inv_h = self.pair(lname, m, False, seed, query, out_key, in_scale=sm, sums=True)
+            else:
+                h = self.pair(lname, m, False, seed, query, out_key, fused=fused if last else None)
         return h
 
     # ---- loss and update ----

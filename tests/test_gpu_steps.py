@@ -362,6 +362,9 @@ def test_forward_loss_matches_forward_then_loss(name, n_dec, T):
     w = workload(name, T=T, n_decoder=n_dec)
     step, _ = _build(w)
     step.fuse_loss = True
+    # the fused loss pair takes a normalised input; the stack's row scales would feed the reference's last linear
+    # an unnormalised one (one rounding apart), so both runs here normalise explicitly
+    step.row_scales = False
     dt = torch.bfloat16
     x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=dt)
     tgt = normal((w.T, w.d_model), tensor_seed(w, "t"), DEV, dtype=dt) if w.kind == "llama_mlp" else None
