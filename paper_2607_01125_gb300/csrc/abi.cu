@@ -215,8 +215,8 @@ int zoact_get_device_status(zoact_ctx* ctx, int* status, int reset) {
     // a launch that gave up may have left a grid-reduction or split-tail ticket part-counted: zero them all so
     // that the context's next launches count from zero again (the stream is idle here)
     ZOACT_CUDA_TRY(cudaMemsetAsync(ctx->d_tickets, 0, 256, ctx->stream));
-    for (ScratchSlot t : {SLOT_SK_TICKETS, SLOT_PROJ_TICKETS})
-      if (ctx->slot_ptr[t]) ZOACT_CUDA_TRY(cudaMemsetAsync(ctx->slot_ptr[t], 0, ctx->slot_bytes[t], ctx->stream));
+    if (ctx->slot_ptr[SLOT_SK_TICKETS])
+      ZOACT_CUDA_TRY(cudaMemsetAsync(ctx->slot_ptr[SLOT_SK_TICKETS], 0, ctx->slot_bytes[SLOT_SK_TICKETS], ctx->stream));
     ZOACT_CUDA_TRY(cudaStreamSynchronize(ctx->stream));
   }
   if (reset) {
@@ -232,10 +232,9 @@ namespace {
 // at most wait_ns of %globaltimer, and record ZOACT_ERR_TIMEOUT as the library's
 // bounded waits do.  One block; nothing traps or faults.
 __global__ void timeout_probe_kernel(const volatile int* flag, int64_t wait_ns, int* status, unsigned int* t0,
-                                     int n0, unsigned int* t1, int n1, unsigned int* t2, int n2) {
+                                     int n0, unsigned int* t1, int n1) {
   for (int i = threadIdx.x; i < n0; i += blockDim.x) t0[i] = 1u;
   for (int i = threadIdx.x; i < n1; i += blockDim.x) t1[i] = 1u;
-  for (int i = threadIdx.x; i < n2; i += blockDim.x) t2[i] = 1u;
   if (threadIdx.x != 0) return;
   uint64_t start, now;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(start));
@@ -256,13 +255,9 @@ int zoact_debug_timeout(zoact_ctx* ctx, int64_t wait_ns) {
   const int* flag = ctx->d_status + 16;
   const int sk_words =
       ctx->slot_ptr[SLOT_SK_TICKETS] ? (int)(ctx->slot_bytes[SLOT_SK_TICKETS] / sizeof(unsigned)) : 0;
-  const int pj_words =
-      ctx->slot_ptr[SLOT_PROJ_TICKETS] ? (int)(ctx->slot_bytes[SLOT_PROJ_TICKETS] / sizeof(unsigned)) : 0;
   timeout_probe_kernel<<<1, 128, 0, ctx->stream>>>(flag, wait_ns, ctx->d_status, ctx->d_tickets,
                                                    256 / (int)sizeof(unsigned),
-                                                   static_cast<unsigned int*>(ctx->slot_ptr[SLOT_SK_TICKETS]), sk_words,
-                                                   static_cast<unsigned int*>(ctx->slot_ptr[SLOT_PROJ_TICKETS]),
-                                                   pj_words);
+                                                   static_cast<unsigned int*>(ctx->slot_ptr[SLOT_SK_TICKETS]), sk_words);
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;

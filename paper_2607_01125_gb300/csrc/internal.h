@@ -37,7 +37,6 @@ enum ScratchSlot {
   SLOT_STACKED_X,    // a shared input and its projection copied once per evaluation block (ranks above 32)
   SLOT_SK_PART,      // partial accumulators of the CTA-pair kernel's split tail
   SLOT_SK_TICKETS,   // its per-tile tickets (zero between launches)
-  SLOT_PROJ_TICKETS, // the tensor-core projection's per-row-block split-K tickets (zero between launches)
   SLOT_COUNT
 };
 

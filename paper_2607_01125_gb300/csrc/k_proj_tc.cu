@@ -36,15 +36,6 @@ struct ProjShared {
   uint32_t tmem_base;
   int abort_flag;
   int ok;
-  int last;           // split-K: this CTA was the row block's last to finish
-};
-
-// Split-K finish of one row block, run by the block's last CTA: P[m][j0 + j] = sum over splits, in split order.
-struct SplitSum {
-  float* P;           // [rows, ldp]
-  int ldp, j0;
-  int splits;         // 1: no split (the kernel writes P directly)
-  unsigned int* tickets;   // one per row block, zero between launches
 };
 
 // Ut: groups of RT ranks (one group for r <= 32; groups of 64 above), each NB rows:
@@ -74,7 +65,7 @@ __global__ void split_u_kernel(const float* __restrict__ U, T16* __restrict__ Ut
 template <int NB, int RT, int AB_BF16>
 __global__ void __launch_bounds__(128, 1)
 proj_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmU, float* __restrict__ out,
-               int64_t rows, int r, int ld_out, int kb_per_split, int num_kb, int* status, SplitSum fin) {
+               int64_t rows, int r, int ld_out, int kb_per_split, int num_kb, int* status) {
   constexpr int STAGE = p_stage_bytes<NB>();
   constexpr uint32_t TCOLS = NB <= 32 ? 32 : (NB <= 64 ? 64 : (NB <= 128 ? 128 : 256));
   extern __shared__ uint8_t smem_raw[];
@@ -206,36 +197,28 @@ proj_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ 
     tc::tc_fence_after();
     tc::tmem_dealloc(tmem, TCOLS);
   }
-  if (fin.splits > 1) {
-    // every split of this row block takes a ticket (also after an abort: the count stays whole); the last adds
-    // the partials in split order -- the order of a separate split-K sum -- and rezeroes the ticket
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0)
-      ss->last = atomicAdd(fin.tickets + blockIdx.x, 1u) == (unsigned int)(fin.splits - 1) ? 1 : 0;
-    __syncthreads();
-    if (*reinterpret_cast<volatile int*>(&ss->last) != 0) {
-      __threadfence();
-      if (m < rows) {
-        const float* src = out + m * ld_out;          // split 0's row m; split k at + k rows ld_out
-        for (int j = 0; j < r; ++j) {
-          float acc = 0.f;
-          for (int k = 0; k < fin.splits; ++k) acc += __ldcg(src + (int64_t)k * rows * ld_out + j);
-          fin.P[m * fin.ldp + fin.j0 + j] = acc;
-        }
-      }
-      if (threadIdx.x == 0) fin.tickets[blockIdx.x] = 0u;
-    }
+}
+
+// P[t, j0 + j] = sum over splits of part[split][t][j] (split order), j < rg; P rows have stride ldp.
+__global__ void splitk_sum_kernel(const float* __restrict__ part, float* __restrict__ P, int64_t n, int splits, int rg,
+                                  int ldp, int j0) {
+  pdl_wait();
+  pdl_trigger();
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    float s = 0.f;
+    for (int k = 0; k < splits; ++k) s += part[(int64_t)k * n + i];
+    const int64_t t = i / rg;
+    P[t * ldp + j0 + (i - t * rg)] = s;
   }
 }
 
 template <int NB, int RT, int AB>
 int launch_one(Ctx* ctx, const CUtensorMap& mx, const CUtensorMap& mu, float* out, int64_t rows, int r, int ld_out,
-               int kbps, int num_kb, dim3 grid, const SplitSum& fin) {
+               int kbps, int num_kb, dim3 grid) {
   auto kern = proj_tc_kernel<NB, RT, AB>;
   ZOACT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, p_smem_bytes<NB>()));
   ZOACT_CUDA_TRY(launch_pdl(ctx, kern, grid, dim3(128), p_smem_bytes<NB>(), mx, mu, out, rows, r, ld_out, kbps,
-                            num_kb, ctx->d_status, fin));
+                            num_kb, ctx->d_status));
   ++ctx->n_launch;
   ZOACT_CHECK_LAUNCH();
   return ZOACT_OK;
@@ -243,13 +226,13 @@ int launch_one(Ctx* ctx, const CUtensorMap& mx, const CUtensorMap& mu, float* ou
 
 template <int AB>
 int dispatch(Ctx* ctx, int rt, const CUtensorMap& mx, const CUtensorMap& mu, float* out, int64_t rows, int r,
-             int ld_out, int kbps, int num_kb, dim3 grid, const SplitSum& fin) {
+             int ld_out, int kbps, int num_kb, dim3 grid) {
   switch (rt) {
-    case 4: return launch_one<16, 4, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid, fin);
-    case 8: return launch_one<32, 8, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid, fin);
-    case 16: return launch_one<48, 16, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid, fin);
-    case 32: return launch_one<96, 32, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid, fin);
-    default: return launch_one<192, 64, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid, fin);
+    case 4: return launch_one<16, 4, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid);
+    case 8: return launch_one<32, 8, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid);
+    case 16: return launch_one<48, 16, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid);
+    case 32: return launch_one<96, 32, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid);
+    default: return launch_one<192, 64, AB>(ctx, mx, mu, out, rows, r, ld_out, kbps, num_kb, grid);
   }
 }
 
@@ -318,20 +301,24 @@ int launch_lowrank_proj_tc_prepared(Ctx* ctx, const void* X, int xdtype, int64_t
     if (st) return st;
     float* out = P + j0;
     int ld_out = r;
-    SplitSum fin{P, r, j0, 1, nullptr};
     if (splits > 1) {
       out = static_cast<float*>(scratch(ctx, SLOT_SPLITK, (size_t)splits * rows * rg * sizeof(float)));
       if (!out) return ZOACT_ERR_NOMEM;
       ld_out = rg;
-      // the splits are added by each row block's last CTA (tickets zero between launches)
-      fin.splits = splits;
-      fin.tickets = static_cast<unsigned int*>(scratch_zeroed(ctx, SLOT_PROJ_TICKETS, (size_t)row_blocks * sizeof(unsigned)));
-      if (!fin.tickets) return ZOACT_ERR_NOMEM;
     }
     const dim3 grid((unsigned)row_blocks, (unsigned)splits);
-    st = xdtype == ZOACT_DT_BF16 ? dispatch<1>(ctx, rt, mx, mu, out, rows, rg, ld_out, kbps, num_kb, grid, fin)
-                                 : dispatch<0>(ctx, rt, mx, mu, out, rows, rg, ld_out, kbps, num_kb, grid, fin);
+    st = xdtype == ZOACT_DT_BF16 ? dispatch<1>(ctx, rt, mx, mu, out, rows, rg, ld_out, kbps, num_kb, grid)
+                                 : dispatch<0>(ctx, rt, mx, mu, out, rows, rg, ld_out, kbps, num_kb, grid);
     if (st) return st;
+    if (splits > 1) {
+      const int64_t n = rows * rg;
+      int64_t blocks = (n + 255) / 256;
+      if (blocks > 4LL * ctx->sm_count) blocks = 4LL * ctx->sm_count;
+      ZOACT_CUDA_TRY(launch_pdl(ctx, splitk_sum_kernel, dim3((unsigned)blocks), dim3(256), 0, out, P, n, splits, rg,
+                                r, j0));
+      ++ctx->n_launch;
+      ZOACT_CHECK_LAUNCH();
+    }
   }
   return ZOACT_OK;
 }
