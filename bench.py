@@ -44,9 +44,10 @@ LR = 1e-4
 TIMING_PAIRS = 4096          # event pairs in the library's kernel-timing pool (launches timed per read)
 
 
-# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one step's pair launches, from one ncu
-# capture of the current kernels at the default sizes; workloads without such a capture report null.
-PAIR_TRAFFIC_BYTES = {"llama_mlp_bf16": 938.5e6}
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one step's pair launches, from ncu captures of
+# the current kernels; workloads without such a capture report null.  The Llama stack's is scaled from a
+# 2-decoder capture (`--decoders 2`): decoder 0 plus 31 times decoder 1 (the later decoders have its shapes).
+PAIR_TRAFFIC_BYTES = {"llama_stack_bf16": 81.92e9}
 
 
 # Dense fp16 tensor peak of the GB300s (TFLOP/s), measured like the bf16 peaks of MEASURED_PEAKS.json
@@ -176,7 +177,7 @@ def dist_setup():
     return world, rank, local
 
 
-def build(ctx, dev, rank, name, tokens=None, n_queries=None, r=None):
+def build(ctx, dev, rank, name, tokens=None, n_queries=None, r=None, n_decoder=None):
     """Weights, bases (Algorithm 1 on the device) and the ZOStep of a workload.
 
     Returns (step, x, target, basis_seconds, workload).  Weights and calibration tokens, hence the bases,
@@ -192,6 +193,8 @@ def build(ctx, dev, rank, name, tokens=None, n_queries=None, r=None):
         over["T"] = tokens
     if r is not None:
         over["r"] = r
+    if n_decoder is not None:
+        over["n_decoder"] = n_decoder
     w = workload(name, **over)
     dt = {"bf16": torch.bfloat16, "fp16": torch.float16}[w.act_dtype]
     specs = w.linears()
@@ -274,7 +277,8 @@ def run_ours(args):
     dev = f"cuda:{local}"
     torch.cuda.set_device(local)
     ctx = zo.Context(local)
-    step, x, target, basis_s, w = build(ctx, dev, rank, args.workload, args.tokens, args.queries, args.rank)
+    step, x, target, basis_s, w = build(ctx, dev, rank, args.workload, args.tokens, args.queries, args.rank,
+                                        args.decoders)
     seed = 1234
 
     def barrier():
@@ -379,7 +383,8 @@ def run_ours(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int4-bf16" if w.wtype == "int4_g128" else w.act_dtype,
         "data": "synthetic",
-        "config": {"workload": w.name, "tokens_per_perturbation": T, "stacked_rows": step.nb * T, "r": w.r,
+        "config": {"workload": w.name if args.decoders is None else f"{w.name} ({w.n_decoder} decoders)",
+                   "tokens_per_perturbation": T, "stacked_rows": step.nb * T, "r": w.r,
                    "eps": w.eps, "adapted_linears": len(w.linears()),
                    "estimator": "two-sided, q=1" if args.queries is None else f"one-sided, q={args.queries}",
                    "l2": "inputs larger than L2 (frozen weights streamed from HBM every step)",
@@ -399,7 +404,8 @@ def run_ours(args):
                                "number of steps)",
                      "algorithmic_flops_per_step": gemm_flops / instr_steps,
                      "traffic": (PAIR_TRAFFIC_BYTES.get(w.name)
-                                 if args.tokens is None and args.queries is None and args.rank is None else None),
+                                 if args.tokens is None and args.queries is None and args.rank is None
+                                 and args.decoders is None else None),
                      "traffic_unit": "bytes per step (all pair launches of the step)"},
         "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": 8 * step.loss_out.numel()},
@@ -520,8 +526,9 @@ def cpu_baseline(step, w, budget_s=20.0):
                           f"(numpy fp64, default BLAS threads); {dt:.3f} s per step"}
     from oracle import layers as olayers
     weights = {}
+    later = 1 if w.n_decoder > 1 else 0              # a decoder past the first (input not shared) where there is one
     for nm in _stack_names(w.kind):
-        lin = step.by_name[f"1.{nm}"]                  # a decoder past the first (input not shared)
+        lin = step.by_name[f"{later}.{nm}"]
         if lin.w_scales is not None:
             weights[nm] = olayers.dequant_int4_g128(lin.W.cpu().numpy(), lin.w_scales.float().cpu().numpy(),
                                                     lin.d_in)
@@ -588,6 +595,8 @@ def main():
     ap.add_argument("--queries", type=int, default=None,
                     help="one-sided estimator with this many queries (Algorithm 2); default: two-sided pair")
     ap.add_argument("--rank", type=int, default=None, help="basis rank r (default: the workload's; 1..256)")
+    ap.add_argument("--decoders", type=int, default=None,
+                    help="stacks only: fewer decoder layers (profiling captures of a few GB; not a bench workload)")
     ap.add_argument("--diag", action="store_true", help="also time the Section 5.3 subspace diagnostics")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--soak", type=float, default=2.0,

@@ -353,6 +353,16 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
   p.num_tiles = p.num_m * p.num_n;
   p.ldy = a.d_out;
   p.aug_mode = lmode;
+  if (two) {
+    // CTA pairs: M-groups as large as keep the group's X rows within ~48 MB of L2 (at least GROUP_M): each W
+    // panel is then read once per group -- with d_in = 4096 and 32 M-tiles, twice instead of four times
+    const double x_group = 2.0 * BM * (double)a.d_in * (double)dtype_size(a.xdtype);
+    int gm = GROUP_M;
+    while (2 * gm <= p.num_m && 2 * gm * x_group <= 48e6) gm *= 2;
+    const char* gsel = std::getenv("ZOACT_GROUP_M");   // comparisons
+    if (gsel && std::atoi(gsel) > 0) gm = std::atoi(gsel);
+    p.group_m = gm;
+  }
   // CTA pairs write Y through staged bulk stores when the whole term is on the MMA, and for the two signs
   // of one query on a shared input with 16-bit outputs (one store map per sign: rows [0, T) and [T, 2T))
   tm.y = tm.y16 = tm.a;

@@ -1038,7 +1038,7 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
       WorkUnit u;
       for (int i = 0; ok && next_unit(prm, cluster_id, n_clusters, total_k, i, u); ++i) {
         int m_blk, n_blk;
-        tile_coords(u.tile, num_m, num_n, m_blk, n_blk);
+        tile_coords(u.tile, num_m, num_n, m_blk, n_blk, prm.group_m);
         for (int kb = u.kb0; kb < u.kb1; ++kb) {
           if (!tc::mbar_wait(tc::smem_u32(&ss->empty[stage]), phase ^ 1u, abort_flag, prm.status)) { ok = false; break; }
           const uint32_t full_leader = tc2::map_to(tc::smem_u32(&ss->full[stage]), 0);
@@ -1202,7 +1202,7 @@ pair_tc2_kernel(const __grid_constant__ TmaSet tm, const Params prm) {
     WorkUnit u;
     for (int i = 0; next_unit(prm, cluster_id, n_clusters, total_k, i, u); ++i, ++local) {
       int m_blk, n_blk;
-      tile_coords(u.tile, num_m, num_n, m_blk, n_blk);
+      tile_coords(u.tile, num_m, num_n, m_blk, n_blk, prm.group_m);
       const int buf = local & 1;
       const uint32_t acc_phase = (local >> 1) & 1;
       const int64_t row0 = (int64_t)m_blk * BM2 + (int64_t)rank * BM;

@@ -155,6 +155,7 @@ struct Params {
   // receives, per 64-column part, the row's sum of squares of the stored (rounded) outputs
   const float* in_scale;
   float* out_sumsq;
+  int group_m;       // M-tiles per group of the tile order (0: GROUP_M)
   int sk_first, sk_tiles, sk_split;
   float* sk_part;
   unsigned int* sk_ticket;
@@ -192,11 +193,15 @@ __device__ __forceinline__ void aug_coords(const Params& prm, int64_t tile_row0,
   }
 }
 
-__device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& m_blk, int& n_blk) {
-  const int per_group = GROUP_M * num_n;
+// Grouped tile order: groups of group_m M-tiles (0: GROUP_M), every N-tile of a group before the next group,
+// the M-tiles of one N-tile consecutive -- a wave reads each W panel once per group while the group's X rows
+// stay in L2.
+__device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& m_blk, int& n_blk, int group_m = 0) {
+  const int G = group_m > 0 ? group_m : GROUP_M;
+  const int per_group = G * num_n;
   const int group = tile / per_group;
-  const int first_m = group * GROUP_M;
-  const int gm = min(GROUP_M, num_m - first_m);
+  const int first_m = group * G;
+  const int gm = min(G, num_m - first_m);
   const int in_group = tile - group * per_group;
   m_blk = first_m + in_group % gm;
   n_blk = in_group / gm;
