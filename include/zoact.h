@@ -208,8 +208,10 @@ int zoact_pair_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X, 
  *             [p][t] receives the sum of squares of Y's stored values (after
  *             rounding to ydtype) in columns [64 p, 64 p + 64) of row t, ready
  *             for zoact_rms_scale.
- * zoact_pair_forward_rs / zoact_pair_forward_gated_rs are zoact_pair_forward /
- * _gated with row scales.  They apply them on the CTA-pair kernel's stacked-row
+ * zoact_pair_forward_rs / zoact_pair_forward_gated_rs / zoact_multi_forward_rs /
+ * zoact_multi_forward_gated_rs are zoact_pair_forward / _gated and
+ * zoact_multi_forward / _gated (declared below) with row scales; out_sumsq then
+ * has n_blocks T rows.  They apply them on the CTA-pair kernel's stacked-row
  * path only: input_shared == 0, rows(X) >= 256, 16-bit X, and INT4 weights from
  * 1024 rows; any other request returns ZOACT_ERR_UNSUPPORTED before anything is
  * launched (callers then normalise explicitly).  rs == NULL or both pointers
@@ -232,6 +234,16 @@ int zoact_pair_forward_gated_rs(zoact_ctx* ctx, const zoact_layer* gate, const z
                                 uint64_t query, void* H, int ydtype, const zoact_rowscale* rs);
 int zoact_rms_scale(zoact_ctx* ctx, const float* sumsq, int64_t rows, int32_t n, float eps,
                     float* inv_scale);
+struct zoact_eval_blocks;
+int zoact_multi_forward_rs(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype,
+                           int64_t T, int input_shared, const float* P,
+                           const struct zoact_eval_blocks* blocks, uint64_t seed, int act, void* Y,
+                           int ydtype, const zoact_rowscale* rs);
+int zoact_multi_forward_gated_rs(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up,
+                                 const void* X, int xdtype, int64_t T, int input_shared,
+                                 const float* P_gate, const float* P_up,
+                                 const struct zoact_eval_blocks* blocks, uint64_t seed, void* H,
+                                 int ydtype, const zoact_rowscale* rs);
 
 /* ---- the pair forward without any allocation ----
  * The paper has no counterpart: this entry point exists for callers that must

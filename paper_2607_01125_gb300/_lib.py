@@ -40,6 +40,7 @@ EXPORTS = [
     "zoact_lowrank_proj_prepared", "zoact_subspace_overlap", "zoact_gradient_energy", "zoact_kernel_timing",
     "zoact_kernel_time", "zoact_pair_forward_loss", "zoact_debug_timeout", "zoact_mean_over_ranks",
     "zoact_arena_hash", "zoact_pair_forward_rs", "zoact_pair_forward_gated_rs", "zoact_rms_scale",
+    "zoact_multi_forward_rs", "zoact_multi_forward_gated_rs",
 ]
 
 
@@ -141,6 +142,11 @@ def load():
         "zoact_pair_forward_gated_rs": [P, ctypes.POINTER(zoact_layer), ctypes.POINTER(zoact_layer), P, I32, I64, I32,
                                         P, P, F32, U64, U64, P, I32, ctypes.POINTER(zoact_rowscale)],
         "zoact_rms_scale": [P, P, I64, I32, F32, P],
+        "zoact_multi_forward_rs": [P, ctypes.POINTER(zoact_layer), P, I32, I64, I32, P,
+                                   ctypes.POINTER(zoact_eval_blocks), U64, I32, P, I32, ctypes.POINTER(zoact_rowscale)],
+        "zoact_multi_forward_gated_rs": [P, ctypes.POINTER(zoact_layer), ctypes.POINTER(zoact_layer), P, I32, I64, I32,
+                                         P, P, ctypes.POINTER(zoact_eval_blocks), U64, P, I32,
+                                         ctypes.POINTER(zoact_rowscale)],
         "zoact_arena_hash": [P, P, I64, P],
     }
     for name, argtypes in sig.items():
@@ -465,3 +471,22 @@ def zoact_rms_scale(ctx, sumsq, n, inv_scale, eps=1e-5):
     rows = sumsq.shape[-1]
     _check("zoact_rms_scale", load().zoact_rms_scale(ctx.handle, _ptr(sumsq), int(rows), int(n), float(eps),
                                                       _ptr(inv_scale)))
+
+
+def zoact_multi_forward_rs(ctx, layer, X, T, input_shared, points, seed, Y, P=None, act=ACT_NONE, in_scale=None,
+                           out_sumsq=None):
+    """zoact_multi_forward with row scales (see include/zoact.h)."""
+    b = eval_blocks(points)
+    rs = _rowscale(in_scale, out_sumsq)
+    _check("zoact_multi_forward_rs", load().zoact_multi_forward_rs(
+        ctx.handle, ctypes.byref(layer), _ptr(X), _dt(X), int(T), int(input_shared), _ptr(P), ctypes.byref(b),
+        int(seed), int(act), _ptr(Y), _dt(Y), ctypes.byref(rs)))
+
+
+def zoact_multi_forward_gated_rs(ctx, gate, up, X, T, input_shared, points, seed, H, P_gate=None, P_up=None,
+                                 in_scale=None, out_sumsq=None):
+    b = eval_blocks(points)
+    rs = _rowscale(in_scale, out_sumsq)
+    _check("zoact_multi_forward_gated_rs", load().zoact_multi_forward_gated_rs(
+        ctx.handle, ctypes.byref(gate), ctypes.byref(up), _ptr(X), _dt(X), int(T), int(input_shared), _ptr(P_gate),
+        _ptr(P_up), ctypes.byref(b), int(seed), _ptr(H), _dt(H), ctypes.byref(rs)))

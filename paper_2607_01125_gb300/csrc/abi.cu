@@ -466,6 +466,23 @@ int zoact_multi_forward(zoact_ctx* ctx, const zoact_layer* layer, const void* X,
   return pair_common(ctx, layer, nullptr, X, xdtype, T, input_shared, P, nullptr, blocks, seed, act, Y, ydtype);
 }
 
+int zoact_multi_forward_rs(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype, int64_t T,
+                           int input_shared, const float* P, const zoact_eval_blocks* blocks, uint64_t seed, int act,
+                           void* Y, int ydtype, const zoact_rowscale* rs) {
+  ZOACT_ENTER(ctx);
+  return pair_common(ctx, layer, nullptr, X, xdtype, T, input_shared, P, nullptr, blocks, seed, act, Y, ydtype,
+                     nullptr, rs);
+}
+int zoact_multi_forward_gated_rs(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up, const void* X,
+                                 int xdtype, int64_t T, int input_shared, const float* P_gate, const float* P_up,
+                                 const zoact_eval_blocks* blocks, uint64_t seed, void* H, int ydtype,
+                                 const zoact_rowscale* rs) {
+  ZOACT_ENTER(ctx);
+  if (!gate || !up) return ZOACT_ERR_INVALID_ARG;
+  if (xdtype == ZOACT_DT_FP32) return ZOACT_ERR_UNSUPPORTED;
+  return pair_common(ctx, gate, up, X, xdtype, T, input_shared, P_gate, P_up, blocks, seed, ZOACT_ACT_NONE, H,
+                     ydtype, nullptr, rs);
+}
 int zoact_multi_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoact_layer* up, const void* X,
                               int xdtype, int64_t T, int input_shared, const float* P_gate, const float* P_up,
                               const zoact_eval_blocks* blocks, uint64_t seed, void* H, int ydtype) {

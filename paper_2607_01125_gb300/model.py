@@ -173,7 +173,7 @@ class ZOStep:
         """fused = (target, out): the last linear with the loss pair fused (zoact_pair_forward_loss); returns None
         when that ran, else (the launch does not qualify) the output as without it.
 
-        Row scales (two-sided stacked rows): in_scale [rows] is 1/rms of X's rows, applied to the output rows
+        Row scales (stacked rows): in_scale [rows] is 1/rms of X's rows, applied to the output rows
         (X is the unnormalised input).  sums=True returns (Y, 1/rms of Y's rows) from the partial sums of squares
         the launch writes, or (Y, None) where the launch cannot write them (the caller then normalises Y)."""
         l = self.by_name[name]
@@ -184,10 +184,14 @@ class ZOStep:
         if in_scale is not None or sums:
             Y = self.buf(out_key, self.nb * self.T, l.d_out)
             ss, inv = self._sums(out_key, l.d_out, Y.shape[0]) if sums else (None, None)
+            if self.n_queries is None:
+                fn = lambda: Z.zoact_pair_forward_rs(self.ctx, l.layer, X, self.T, shared, self.eps, seed, query, Y,
+                                                     P=P, act=act, in_scale=in_scale, out_sumsq=ss)
+            else:
+                fn = lambda: Z.zoact_multi_forward_rs(self.ctx, l.layer, X, self.T, shared, self.points(query), seed,
+                                                      Y, P=P, act=act, in_scale=in_scale, out_sumsq=ss)
             try:
-                self._counted(lambda: Z.zoact_pair_forward_rs(self.ctx, l.layer, X, self.T, shared, self.eps, seed,
-                                                              query, Y, P=P, act=act, in_scale=in_scale,
-                                                              out_sumsq=ss), flops)
+                self._counted(fn, flops)
             except Z.ZoactError as e:
                 if e.status != Z.ZOACT_ERR_UNSUPPORTED or in_scale is not None:
                     raise
@@ -231,10 +235,16 @@ class ZOStep:
         flops = 2.0 * X.shape[0] * g.d_in * g.d_out * 2
         if in_scale is not None or sums:
             ss, inv = self._sums(out_key, g.d_out, H.shape[0]) if sums else (None, None)
+            if self.n_queries is None:
+                fn = lambda: Z.zoact_pair_forward_gated_rs(self.ctx, g.layer, u.layer, X, self.T, shared, self.eps,
+                                                           seed, query, H, P_gate=Pg, P_up=Pu, in_scale=in_scale,
+                                                           out_sumsq=ss)
+            else:
+                fn = lambda: Z.zoact_multi_forward_gated_rs(self.ctx, g.layer, u.layer, X, self.T, shared,
+                                                            self.points(query), seed, H, P_gate=Pg, P_up=Pu,
+                                                            in_scale=in_scale, out_sumsq=ss)
             try:
-                self._counted(lambda: Z.zoact_pair_forward_gated_rs(self.ctx, g.layer, u.layer, X, self.T, shared,
-                                                                    self.eps, seed, query, H, P_gate=Pg, P_up=Pu,
-                                                                    in_scale=in_scale, out_sumsq=ss), flops)
+                self._counted(fn, flops)
             except Z.ZoactError as e:
                 if e.status != Z.ZOACT_ERR_UNSUPPORTED or in_scale is not None:
                     raise
@@ -288,14 +298,13 @@ class ZOStep:
         return self.loss_out
 
     def _stack(self, x, seed, query, fused=None):
-        """The stack's decoders.  With row scales (two-sided steps outside calibration, where the library applies
-        them) the RMS normalisations of o, of the MLP hidden and of each decoder's output are not separate passes:
+        """The stack's decoders.  With row scales (outside calibration, where the library applies them) the RMS normalisations of o, of the MLP hidden and of each decoder's output are not separate passes:
         the producing pair forward writes per-row sums of squares, zoact_rms_scale turns them into 1/rms, and the
         consuming pair forward scales its rows (include/zoact.h, row scales).  Otherwise, and wherever a launch
         cannot apply them, the normalised tensor is written by zoact_rms_norm first."""
         T = self.T
         n_dec = len(self.linears) // (7 if self.kind == "llama" else 6)
-        rs = self.row_scales and self.capture is None and self.n_queries is None
+        rs = self.row_scales and self.capture is None
         h, inv_h = x, None
         shared = True
         for L in range(n_dec):

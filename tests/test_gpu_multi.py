@@ -287,10 +287,12 @@ def test_toy_one_sided_steps():
     step.ctx.close()
 
 
-@pytest.mark.parametrize("name,n_dec,T,q", [("llama_mlp_bf16", None, 256, 8), ("llama_stack_bf16", 1, 64, 4)])
+@pytest.mark.parametrize("name,n_dec,T,q", [("llama_mlp_bf16", None, 256, 8), ("llama_stack_bf16", 1, 64, 4),
+                                            ("llama_stack_bf16", 2, 64, 4)])
 def test_bf16_one_sided_step(name, n_dec, T, q):
     # 16-bit graphs: every block's output and every L_b within 2e-2 (the a_j of a bf16 graph at mu = 1e-3 are
-    # below the outputs' rounding and are not compared)
+    # below the outputs' rounding and are not compared).  The stacks' 5 x 64 stacked rows run the RMS
+    # normalisations as row scales (the second decoder's q, k, v take its unnormalised input)
     w = workload(name, T=T) if n_dec is None else workload(name, T=T, n_decoder=n_dec)
     step, ora = _build(w, q, c_std=0.01)
     x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV)
@@ -306,8 +308,8 @@ def test_bf16_one_sided_step(name, n_dec, T, q):
                                       blocks=blocks)
     else:
         names = ["q", "k", "v", "o", "gate", "up", "down"]
-        Yo = graphs.stack_forward([{nm: ora[f"0.{nm}"] for nm in names}], np64(x), 0.0, seed, 0, "llama",
-                                  store="bf16", blocks=blocks)
+        Yo = graphs.stack_forward([{nm: ora[f"{L}.{nm}"] for nm in names} for L in range(w.n_decoder)], np64(x), 0.0,
+                                  seed, 0, "llama", store="bf16", blocks=blocks)
     L, _ = oloss.loss_queries(Yo, w.T, q + 1, None if tgt is None else np64(tgt), w.eps)
     Yg = np64(Y)
     assert np.abs(Yg - Yo).max() <= 2e-2 * np.abs(Yo).max()
