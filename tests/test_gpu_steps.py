@@ -6,7 +6,7 @@ oracle (with bf16/fp16 rounding mirrored where activations are stored).  Bases
 are inputs here (random orthonormal U from synth) so the step is tested on its
 own; the device basis is tested in test_gpu_kernels.py and below at full width.
 
-Tolerances (the benchmark spec): 16-bit outputs and L+- within 2e-2 relative; the
+Tolerances (the parity bar): 16-bit outputs and L+- within 2e-2 relative; the
 estimator scalar a within 2e-2 relative (its sign agreeing) whenever
 |L+ - L-| exceeds 2e-2 max(L+, L-).  The 16-bit step tests are built so that
 it does: the coefficients are drawn as C = 0.3 Z(seed, layer, query) plus
@@ -111,7 +111,7 @@ def _check_step(step, oracle_layer, Y, out, Yo, tgt_o, w, seed, query):
     assert err_mean <= 1e-2, ("mean |dY| / mean |Y|", err_mean)
     o = out.cpu().numpy()
     assert abs(o[0] - Lp) <= 2e-2 * Lp and abs(o[1] - Lm) <= 2e-2 * Lm, (o[:2], Lp, Lm)
-    # the inputs are built so that the benchmark spec's bound applies: a is compared, never skipped
+    # the inputs are built so that the bound applies: a is compared, never skipped
     assert abs(Lp - Lm) > 2e-2 * max(Lp, Lm), ("the test's inputs must make L+ - L- resolvable", Lp, Lm)
     assert np.sign(o[3]) == np.sign(a), (o[3], a)
     assert abs(o[3] - a) <= 2e-2 * abs(a), (o[3], a)
