@@ -218,6 +218,34 @@ def test_stack_step_full_depth(name):
     step.ctx.close()
 
 
+@pytest.mark.parametrize("name", ["llama_stack_bf16", "opt_stack_fp16"])
+def test_stack_full_size_sampled(name):
+    # the bench's launches of a stack at full size (T = 4096, 8192 stacked rows: row-scaled normalisations, L2-sized
+    # M-groups, split tails, eps = 1e-3) on two decoders.  Every op of a decoder acts on each token row on its own,
+    # so the oracle runs each decoder on 24 sampled rows of the GPU's stored input to it (the same rows of both
+    # signs) and checks the same rows of the decoder's output
+    w = workload(name, n_decoder=2)
+    assert w.T == 4096
+    step, ol = _build(w)
+    dt = torch.bfloat16 if w.act_dtype == "bf16" else torch.float16
+    x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=dt)
+    ins = []
+    step.on_decoder = lambda L, h: ins.append(h.clone())
+    seed, query = 31, 4
+    Y = step.forward(x, seed, query)
+    torch.cuda.synchronize()
+    assert step.ctx.device_status() == 0
+    tok = np.sort(np.random.default_rng(3).choice(w.T, 24, replace=False))
+    both = np.concatenate([tok, w.T + tok])
+    outs = [ins[1], Y]
+    for L in range(2):
+        dl = {nm: ol(f"{L}.{nm}") for nm in _stack_names(w.kind)}
+        h_in = n64(ins[L])[tok if L == 0 else both]
+        Yo = graphs.stack_forward([dl], h_in, w.eps, seed, query, w.kind, store=w.act_dtype, first=(L == 0))
+        _check_outputs(n64(outs[L])[both], Yo, f"decoder {L}")
+    step.ctx.close()
+
+
 def test_toy_two_steps():
     w = workload("toy_fp32")
     step, ol = _build(w, c_std=0.05)
