@@ -32,9 +32,10 @@
 // Measured on the Llama-3-8B gate/up shapes (8192 stacked rows): one release per
 // stage made a gated call 3.3x slower than expanding W first (a cluster-scope
 // release took ~0.5 us); batches of three and eight warps bring it to 1.8x
-// (2.09 vs 1.14 ms), now bound by the pipeline: a packed block can only be
-// fetched once its B slot is free, and that TMA's latency plus the release
-// exceed one batch's MMA time.  The expansion therefore stays the default.
+// (2.09 vs 1.14 ms).  A separate ring that fetched the packed blocks ahead of
+// their stages, with two groups taking alternate batches, measured 2.17 ms;
+// with no dequantisation at all (only its waits, barriers and arrivals) that
+// structure still took 1.47 ms.  The expansion therefore stays the default.
 #pragma once
 #include "pair_tc_kernel.cuh"
 
