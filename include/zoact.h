@@ -323,6 +323,42 @@ int zoact_pair_forward_gated(zoact_ctx* ctx, const zoact_layer* gate, const zoac
                              const float* P_gate, const float* P_up, float eps, uint64_t seed,
                              uint64_t query, void* H, int ydtype);
 
+/* ---- adapted linears that read one input, as one launch (Section 3 perturbed
+ * forward of each; Algorithm 2) ----
+ * Linears with the same input have, by Algorithm 1, the same basis U, hence one
+ * projection P = X U: attention's q, k and v.  Run one by one, the narrow ones
+ * (k and v of a grouped-query model) leave pairs of SMs idle in their last wave;
+ * run as one pair forward over their concatenated weights they do not.
+ * layers[0 .. n_layers), 1 <= n_layers <= ZOACT_MAX_GROUP: the same d_in, r,
+ * wtype and U (pointer), and W rows that follow one another in memory: layers[i].W
+ * is layers[0].W advanced by d_out_0 + ... + d_out_{i-1} rows (INT4: the packed
+ * rows and the scale rows both).  Each layer keeps its own C and layer_id, so
+ * every output element is the one its layer's own pair forward computes: the
+ * same Z and the same K order (a tile of a last wave whose K range is split sums
+ * its pieces in fixed order, and the split can fall on other tiles than in the
+ * per-layer calls: equal within rounding there).
+ * X: stacked [n_blocks T, d_in] (a shared input has no grouped form).  Y
+ * [n_blocks T, sum d_out] of ydtype holds the layers' outputs side by side:
+ * layer i in columns [d_out_0 + ... + d_out_{i-1}, that + d_out_i).  P: optional
+ * [n_blocks T, r] fp32 projection (NULL: computed once into context scratch).
+ * rs: row scales as for zoact_pair_forward_rs over the sum d_out columns (NULL:
+ * none).  zoact_pair_forward_group_rs evaluates the two-sided pair ({+eps, -eps},
+ * one query), zoact_multi_forward_group_rs the blocks of `blocks`.
+ * One launch serves the request where the kernel takes the whole low-rank term
+ * from the tensor-core operand tables: stacked rows from 256 on CTA pairs, 16-bit
+ * X (INT4 from 1024 rows); any other request returns ZOACT_ERR_UNSUPPORTED before
+ * anything is launched, and the caller runs the layers one by one.  Layers that
+ * differ in d_in, r, wtype or U, or whose W (or scales) do not follow one
+ * another: ZOACT_ERR_INVALID_ARG.  n_layers == 1 is zoact_pair_forward_rs /
+ * zoact_multi_forward_rs on stacked rows.                                       */
+#define ZOACT_MAX_GROUP 4
+int zoact_pair_forward_group_rs(zoact_ctx* ctx, const zoact_layer* layers, int32_t n_layers, const void* X,
+                                int xdtype, int64_t T, const float* P, float eps, uint64_t seed,
+                                uint64_t query, int act, void* Y, int ydtype, const zoact_rowscale* rs);
+int zoact_multi_forward_group_rs(zoact_ctx* ctx, const zoact_layer* layers, int32_t n_layers, const void* X,
+                                 int xdtype, int64_t T, const float* P, const zoact_eval_blocks* blocks,
+                                 uint64_t seed, int act, void* Y, int ydtype, const zoact_rowscale* rs);
+
 /* ---- the last pair forward fused with its loss pair (Section 3; Algorithm 2) ----
  * The losses zoact_loss_pair would return for Y = zoact_pair_forward(layer, X,
  * stacked rows, eps, seed, query, act) rounded to ydtype, computed inside the
@@ -433,6 +469,13 @@ int zoact_rms_norm(zoact_ctx* ctx, const void* X, int dtype, int64_t rows, int32
  * consecutive query heads (n_rep = 1: plain sum).                              */
 int zoact_mix_rms(zoact_ctx* ctx, const void* q, const void* k, const void* v, int dtype,
                   int64_t rows, int32_t n, int32_t n_rep, int32_t head_dim, float eps, void* Y);
+/* zoact_mix_rms_strided: the same with row strides in elements: row t of q at
+ * q + t ld_q (ld_q >= n), of k and v at k + t ld_kv, v + t ld_kv (ld_kv >=
+ * n / n_rep), e.g. column views of a zoact_pair_forward_group_rs output; Y is
+ * [rows, n] contiguous.                                                        */
+int zoact_mix_rms_strided(zoact_ctx* ctx, const void* q, const void* k, const void* v, int dtype,
+                          int64_t rows, int32_t n, int32_t n_rep, int32_t head_dim, int64_t ld_q,
+                          int64_t ld_kv, float eps, void* Y);
 
 /* ---- data-parallel replicas ----
  * A data-parallel ZO step shares everything but the tokens: every rank holds

@@ -16,6 +16,7 @@ from ._lib import (  # noqa: F401
     zoact_basis_prepared_bytes, zoact_basis_prepare, zoact_lowrank_proj_prepared,
     zoact_subspace_overlap, zoact_gradient_energy, zoact_mean_over_ranks, zoact_arena_hash,
     zoact_pair_forward_rs, zoact_pair_forward_gated_rs, zoact_rms_scale, rowscale_parts,
-    zoact_multi_forward_rs, zoact_multi_forward_gated_rs,
+    zoact_multi_forward_rs, zoact_multi_forward_gated_rs, zoact_pair_forward_group_rs, zoact_multi_forward_group_rs,
+    MAX_GROUP,
     DT_FP32, DT_BF16, DT_FP16, DT_INT4_G128, ACT_NONE, ACT_RELU, ACT_GELU, EXPORTS, LIB_PATH, TORCH_DT,
 )

@@ -24,6 +24,7 @@ ZOACT_ERR_TOO_LARGE = -7
 ZOACT_ERR_REPLICA_MISMATCH = -8
 NOALLOC_MAX_PROJ_FLOATS = 1 << 20
 MAX_EVAL_BLOCKS = 17
+MAX_GROUP = 4
 
 DT_FP32, DT_BF16, DT_FP16, DT_INT4_G128 = 0, 1, 2, 3
 ACT_NONE, ACT_RELU, ACT_GELU = 0, 1, 2
@@ -40,7 +41,8 @@ EXPORTS = [
     "zoact_lowrank_proj_prepared", "zoact_subspace_overlap", "zoact_gradient_energy", "zoact_kernel_timing",
     "zoact_kernel_time", "zoact_pair_forward_loss", "zoact_debug_timeout", "zoact_mean_over_ranks",
     "zoact_arena_hash", "zoact_pair_forward_rs", "zoact_pair_forward_gated_rs", "zoact_rms_scale",
-    "zoact_multi_forward_rs", "zoact_multi_forward_gated_rs",
+    "zoact_multi_forward_rs", "zoact_multi_forward_gated_rs", "zoact_pair_forward_group_rs",
+    "zoact_multi_forward_group_rs", "zoact_mix_rms_strided",
 ]
 
 
@@ -148,6 +150,12 @@ def load():
                                          P, P, ctypes.POINTER(zoact_eval_blocks), U64, P, I32,
                                          ctypes.POINTER(zoact_rowscale)],
         "zoact_arena_hash": [P, P, I64, P],
+        "zoact_pair_forward_group_rs": [P, ctypes.POINTER(zoact_layer), I32, P, I32, I64, P, F32, U64, U64, I32, P,
+                                        I32, ctypes.POINTER(zoact_rowscale)],
+        "zoact_multi_forward_group_rs": [P, ctypes.POINTER(zoact_layer), I32, P, I32, I64, P,
+                                         ctypes.POINTER(zoact_eval_blocks), U64, I32, P, I32,
+                                         ctypes.POINTER(zoact_rowscale)],
+        "zoact_mix_rms_strided": [P, P, P, P, I32, I64, I32, I32, I32, I64, I64, F32, P],
     }
     for name, argtypes in sig.items():
         fn = getattr(lib, name)
@@ -345,9 +353,18 @@ def zoact_rms_norm(ctx, X, Y, eps=1e-5):
 
 
 def zoact_mix_rms(ctx, q, k, v, Y, n_rep, head_dim, eps=1e-5):
+    """Y = rms(q + rep(k) + rep(v)).  q, k and v may be column views (unit column stride) of wider row-major
+    tensors -- the layers' columns of a zoact_pair_forward_group_rs output -- which go to zoact_mix_rms_strided."""
     rows, n = q.shape
-    _check("zoact_mix_rms", load().zoact_mix_rms(ctx.handle, _ptr(q), _ptr(k), _ptr(v), _dt(q), rows, n,
-                                                  int(n_rep), int(head_dim), float(eps), _ptr(Y)))
+    if q.is_contiguous() and k.is_contiguous() and v.is_contiguous():
+        _check("zoact_mix_rms", load().zoact_mix_rms(ctx.handle, _ptr(q), _ptr(k), _ptr(v), _dt(q), rows, n,
+                                                      int(n_rep), int(head_dim), float(eps), _ptr(Y)))
+        return
+    if q.stride(1) != 1 or k.stride(1) != 1 or v.stride(1) != 1 or k.stride(0) != v.stride(0):
+        raise ValueError("libzoact takes rows with unit column stride (k and v with one row stride)")
+    _check("zoact_mix_rms_strided", load().zoact_mix_rms_strided(
+        ctx.handle, ctypes.c_void_p(q.data_ptr()), ctypes.c_void_p(k.data_ptr()), ctypes.c_void_p(v.data_ptr()),
+        _dt(q), rows, n, int(n_rep), int(head_dim), int(q.stride(0)), int(k.stride(0)), float(eps), _ptr(Y)))
 
 
 def zoact_multi_forward(ctx, layer, X, T, input_shared, points, seed, Y, P=None, act=ACT_NONE):
@@ -481,6 +498,38 @@ def zoact_multi_forward_rs(ctx, layer, X, T, input_shared, points, seed, Y, P=No
     _check("zoact_multi_forward_rs", load().zoact_multi_forward_rs(
         ctx.handle, ctypes.byref(layer), _ptr(X), _dt(X), int(T), int(input_shared), _ptr(P), ctypes.byref(b),
         int(seed), int(act), _ptr(Y), _dt(Y), ctypes.byref(rs)))
+
+
+def _layer_array(layers):
+    if not 1 <= len(layers) <= MAX_GROUP:
+        raise ValueError(f"1 .. {MAX_GROUP} layers per group")
+    arr = (zoact_layer * len(layers))()
+    for i, l in enumerate(layers):
+        ctypes.memmove(ctypes.byref(arr[i]), ctypes.byref(l), ctypes.sizeof(zoact_layer))
+    return arr
+
+
+def zoact_pair_forward_group_rs(ctx, layers, X, T, eps, seed, query, Y, P=None, act=ACT_NONE, in_scale=None,
+                                out_sumsq=None):
+    """Layers that read X (stacked rows), with contiguous weights and one basis, as one pair forward: Y
+    [2T, sum d_out] holds their outputs side by side (include/zoact.h).  Raises ZoactError with
+    ZOACT_ERR_UNSUPPORTED, before anything is launched, where one launch cannot serve them."""
+    arr = _layer_array(layers)
+    rs = _rowscale(in_scale, out_sumsq)
+    _check("zoact_pair_forward_group_rs", load().zoact_pair_forward_group_rs(
+        ctx.handle, arr, len(layers), _ptr(X), _dt(X), int(T), _ptr(P), float(eps), int(seed), int(query), int(act),
+        _ptr(Y), _dt(Y), ctypes.byref(rs)))
+
+
+def zoact_multi_forward_group_rs(ctx, layers, X, T, points, seed, Y, P=None, act=ACT_NONE, in_scale=None,
+                                 out_sumsq=None):
+    """zoact_pair_forward_group_rs over the evaluation blocks `points` (list of (coef, query))."""
+    arr = _layer_array(layers)
+    b = eval_blocks(points)
+    rs = _rowscale(in_scale, out_sumsq)
+    _check("zoact_multi_forward_group_rs", load().zoact_multi_forward_group_rs(
+        ctx.handle, arr, len(layers), _ptr(X), _dt(X), int(T), _ptr(P), ctypes.byref(b), int(seed), int(act),
+        _ptr(Y), _dt(Y), ctypes.byref(rs)))
 
 
 def zoact_multi_forward_gated_rs(ctx, gate, up, X, T, input_shared, points, seed, H, P_gate=None, P_up=None,

@@ -373,10 +373,19 @@ struct FusedLoss {
   float eps;
 };
 
+// Adapted linears run as one launch (zoact_pair_forward_group_rs): the columns, coefficients and Philox
+// stream of each.
+struct PairSegs {
+  int n;
+  int off[ZOACT_MAX_GROUP + 1];
+  const float* C[ZOACT_MAX_GROUP];
+  uint32_t lid[ZOACT_MAX_GROUP];
+};
+
 static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* L2, const void* X, int xdtype,
                        int64_t T, int input_shared, const float* P, const float* P2, const zoact_eval_blocks* blk,
                        uint64_t seed, int act, void* Y, int ydtype, const FusedLoss* fl = nullptr,
-                       const zoact_rowscale* rs = nullptr) {
+                       const zoact_rowscale* rs = nullptr, const PairSegs* segs = nullptr) {
   if (check_eval_blocks(blk)) return ZOACT_ERR_INVALID_ARG;
   int st = check_layer(L);
   if (st) return st;
@@ -438,8 +447,58 @@ static int pair_common(zoact_ctx* ctx, const zoact_layer* L, const zoact_layer* 
   if (L2) { a.W2 = L2->W; a.w_scales2 = L2->w_scales; a.P2 = P2; a.C2 = L2->C; a.layer_id2 = L2->layer_id; }
   if (fl) { a.fuse_loss = 1; a.target = fl->target; a.loss_out = fl->out; a.loss_eps = fl->eps; }
   if (rowscale) { a.in_scale = rs->in_scale; a.out_sumsq = rs->out_sumsq; }
+  if (segs && segs->n > 1) {
+    a.nseg = segs->n;
+    for (int g = 0; g <= segs->n; ++g) a.seg_off[g] = segs->off[g];
+    for (int g = 0; g < segs->n; ++g) { a.seg_C[g] = segs->C[g]; a.seg_lid[g] = segs->lid[g]; }
+  }
   if (xdtype == ZOACT_DT_FP32) return launch_pair_simt(ctx, a);
   return launch_pair_tc(ctx, a);
+}
+
+// Layers that read one input as one pair forward over their concatenated weights (include/zoact.h).
+static int group_common(zoact_ctx* ctx, const zoact_layer* layers, int32_t n_layers, const void* X, int xdtype,
+                        int64_t T, const float* P, const zoact_eval_blocks* blk, uint64_t seed, int act, void* Y,
+                        int ydtype, const zoact_rowscale* rs) {
+  if (!layers || n_layers < 1 || n_layers > ZOACT_MAX_GROUP) return ZOACT_ERR_INVALID_ARG;
+  if (check_eval_blocks(blk)) return ZOACT_ERR_INVALID_ARG;
+  const zoact_layer& L0 = layers[0];
+  int st = check_layer(&L0);
+  if (st) return st;
+  const bool int4 = L0.wtype == ZOACT_DT_INT4_G128;
+  const int64_t w_row = int4 ? L0.d_in / 2 : (int64_t)L0.d_in * (int64_t)dtype_size(L0.wtype);
+  const int64_t s_row = int4 ? (int64_t)(L0.d_in / 128) * 2 : 0;
+  PairSegs sg{};
+  sg.n = n_layers;
+  int64_t off = 0;
+  for (int i = 0; i < n_layers; ++i) {
+    const zoact_layer& Li = layers[i];
+    st = check_layer(&Li);
+    if (st) return st;
+    if (Li.d_in != L0.d_in || Li.r != L0.r || Li.wtype != L0.wtype || Li.U != L0.U) return ZOACT_ERR_INVALID_ARG;
+    // W rows (and INT4 scale rows) of layer i follow those of the layers before it
+    if (static_cast<const char*>(Li.W) != static_cast<const char*>(L0.W) + off * w_row) return ZOACT_ERR_INVALID_ARG;
+    if (int4 && static_cast<const char*>(Li.w_scales) != static_cast<const char*>(L0.w_scales) + off * s_row)
+      return ZOACT_ERR_INVALID_ARG;
+    sg.off[i] = (int)off;
+    sg.C[i] = Li.C;
+    sg.lid[i] = Li.layer_id;
+    off += Li.d_out;
+    if (off > 0x7fffffff) return ZOACT_ERR_INVALID_ARG;
+  }
+  sg.off[n_layers] = (int)off;
+  zoact_layer Lc = L0;
+  Lc.d_out = (int32_t)off;
+  st = check_layer(&Lc);
+  if (st) return st;
+  if (T < 0 || T > ((int64_t)1 << 40) / blk->n_blocks) return ZOACT_ERR_INVALID_ARG;
+  // one launch only where the kernel takes the whole low-rank term from the operand tables: decided before
+  // anything (the projection included) is launched
+  if (n_layers > 1 && T > 0 &&
+      !pair_rowscale_supported(ctx, (int64_t)blk->n_blocks * T, 0, xdtype, L0.wtype, blk->n_blocks))
+    return ZOACT_ERR_UNSUPPORTED;
+  return pair_common(ctx, &Lc, nullptr, X, xdtype, T, 0, P, nullptr, blk, seed, act, Y, ydtype, nullptr, rs,
+                     n_layers > 1 ? &sg : nullptr);
 }
 
 int zoact_pair_forward_loss(zoact_ctx* ctx, const zoact_layer* layer, const void* X, int xdtype, int64_t T,
@@ -512,6 +571,21 @@ int zoact_pair_forward_gated_rs(zoact_ctx* ctx, const zoact_layer* gate, const z
   const zoact_eval_blocks b = pair_blocks(eps, query);
   return pair_common(ctx, gate, up, X, xdtype, T, input_shared, P_gate, P_up, &b, seed, ZOACT_ACT_NONE, H, ydtype,
                      nullptr, rs);
+}
+
+int zoact_pair_forward_group_rs(zoact_ctx* ctx, const zoact_layer* layers, int32_t n_layers, const void* X,
+                                int xdtype, int64_t T, const float* P, float eps, uint64_t seed, uint64_t query,
+                                int act, void* Y, int ydtype, const zoact_rowscale* rs) {
+  ZOACT_ENTER(ctx);
+  const zoact_eval_blocks b = pair_blocks(eps, query);
+  return group_common(ctx, layers, n_layers, X, xdtype, T, P, &b, seed, act, Y, ydtype, rs);
+}
+
+int zoact_multi_forward_group_rs(zoact_ctx* ctx, const zoact_layer* layers, int32_t n_layers, const void* X,
+                                 int xdtype, int64_t T, const float* P, const zoact_eval_blocks* blocks,
+                                 uint64_t seed, int act, void* Y, int ydtype, const zoact_rowscale* rs) {
+  ZOACT_ENTER(ctx);
+  return group_common(ctx, layers, n_layers, X, xdtype, T, P, blocks, seed, act, Y, ydtype, rs);
 }
 
 int zoact_rms_scale(zoact_ctx* ctx, const float* sumsq, int64_t rows, int32_t n, float eps, float* inv_scale) {
@@ -658,7 +732,18 @@ int zoact_mix_rms(zoact_ctx* ctx, const void* q, const void* k, const void* v, i
   if (n % (n_rep * head_dim) != 0) return ZOACT_ERR_INVALID_ARG;
   if (rows > 0 && (!q || !k || !v || !Y)) return ZOACT_ERR_INVALID_ARG;
   if (rows > 0x7fffffff) return ZOACT_ERR_UNSUPPORTED;
-  return launch_mix_rms(ctx, q, k, v, dtype, rows, n, n_rep, head_dim, eps, Y);
+  return launch_mix_rms(ctx, q, k, v, dtype, rows, n, n_rep, head_dim, eps, Y, n, n / n_rep);
+}
+
+int zoact_mix_rms_strided(zoact_ctx* ctx, const void* q, const void* k, const void* v, int dtype, int64_t rows,
+                          int32_t n, int32_t n_rep, int32_t head_dim, int64_t ld_q, int64_t ld_kv, float eps,
+                          void* Y) {
+  ZOACT_ENTER(ctx);
+  if (rows < 0 || n <= 0 || n_rep <= 0 || head_dim <= 0 || !valid_act_dtype(dtype)) return ZOACT_ERR_INVALID_ARG;
+  if (n % (n_rep * head_dim) != 0 || ld_q < n || ld_kv < n / n_rep) return ZOACT_ERR_INVALID_ARG;
+  if (rows > 0 && (!q || !k || !v || !Y)) return ZOACT_ERR_INVALID_ARG;
+  if (rows > 0x7fffffff) return ZOACT_ERR_UNSUPPORTED;
+  return launch_mix_rms(ctx, q, k, v, dtype, rows, n, n_rep, head_dim, eps, Y, ld_q, ld_kv);
 }
 
 }  // extern "C"

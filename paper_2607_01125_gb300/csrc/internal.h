@@ -179,6 +179,13 @@ struct PairArgs {
   // out_sumsq [ceil(d_out / 64), nb T] receives per-64-column-part sums of squares of the stored outputs
   const float* in_scale;
   float* out_sumsq;
+  // adapted linears that read one input, run as one (zoact_pair_forward_group_rs): output columns
+  // [seg_off[s], seg_off[s + 1]) are layer s's, with coefficients seg_C[s] and Philox stream seg_lid[s]
+  // (d_out is the sum, W the first layer's rows followed by the others'); nseg <= 1: one layer
+  int nseg;
+  int seg_off[ZOACT_MAX_GROUP + 1];
+  const float* seg_C[ZOACT_MAX_GROUP];
+  uint32_t seg_lid[ZOACT_MAX_GROUP];
 };
 // Whether a launch with row scales runs on a kernel that applies them (CTA pairs, stacked rows, the whole
 // low-rank term on the MMA, staged output) -- decided before anything is launched.
@@ -231,7 +238,7 @@ int launch_adam(Ctx* ctx, float* C, float* m, float* v, const zoact_coeff_block*
 
 int launch_rms_norm(Ctx* ctx, const void* X, int dtype, int64_t rows, int n, float eps, void* Y);
 int launch_mix_rms(Ctx* ctx, const void* q, const void* k, const void* v, int dtype, int64_t rows,
-                   int n, int n_rep, int head_dim, float eps, void* Y);
+                   int n, int n_rep, int head_dim, float eps, void* Y, int64_t ld_q, int64_t ld_kv);
 
 // Section 5.3 diagnostics (k_diag.cu): out[0] = ||Ua^T Ub||_F^2, out[2] = out[0] / ra;
 // energy: out[0] = ||U^T G||_F^2, out[1] = ||G||_F^2, out[2] = their ratio.  out: device fp64 [3].

@@ -32,6 +32,12 @@ struct AugBlocks {
   uint64_t qry[ZOACT_MAX_EVAL_BLOCKS];
   uint64_t zq[ZOACT_MAX_EVAL_BLOCKS];   // distinct queries whose Z is written transposed
   int nzq;
+  // layers run as one (B rows only): row n of the table belongs to layer s with seg_off[s] <= n <
+  // seg_off[s + 1]; its T = C_s + c_b Z_b takes C_s and Z from that layer's own rows and Philox stream
+  int nseg;
+  int seg_off[ZOACT_MAX_GROUP + 1];
+  const float* seg_C[ZOACT_MAX_GROUP];
+  uint32_t seg_lid[ZOACT_MAX_GROUP];
 };
 
 // v = hi + lo (+ what bf16 cannot hold): hi = bf16(v), lo = bf16(v - hi); v - hi is exact in fp32.
@@ -97,14 +103,22 @@ aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const
     int my_slot = 0, n = 0;
     float cb = 0.f;
     uint64_t q = 0;
+    uint32_t layer = up ? lid2 : lid;
+    const float* Cs = up ? C2 : C;      // the coefficients row n indexes (a grouped layer's own)
     if (is_a) {
       if (slots > 1) my_slot = (int)((orow / T) % slots);
     } else {
       const int b = (int)(orow / d_out);
       n = (int)(orow - (int64_t)b * d_out);
       if (full) { cb = blk.coef[b]; q = blk.qry[b]; }
+      if (blk.nseg > 1) {
+        int sg = 0;
+        while (sg + 1 < blk.nseg && n >= blk.seg_off[sg + 1]) ++sg;
+        n -= blk.seg_off[sg];
+        Cs = blk.seg_C[sg];
+        layer = blk.seg_lid[sg];
+      }
     }
-    const uint32_t layer = up ? lid2 : lid;
     uint32_t w[4];
 #pragma unroll
     for (int h4 = 0; h4 < 2; ++h4) {
@@ -124,7 +138,7 @@ aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const
             v = *reinterpret_cast<const float4*>((distinct && half ? P2 : P) + orow * r + j0);
           } else {
             const int64_t e = (int64_t)n * r + j0;
-            v = *reinterpret_cast<const float4*>((up ? C2 : C) + e);
+            v = *reinterpret_cast<const float4*>(Cs + e);
             if (cb != 0.f) {
               const float4 z = z_normals4(seed, layer, q, (uint64_t)(e >> 2));
               v.x = fmaf(cb, z.x, v.x); v.y = fmaf(cb, z.y, v.y);
@@ -152,7 +166,7 @@ aug_prep_kernel(const float* __restrict__ P, const float* __restrict__ P2, const
               v = (distinct && half ? P2 : P)[orow * r + j];
             } else {
               const int64_t e = (int64_t)n * r + j;
-              v = (up ? C2 : C)[e];
+              v = Cs[e];
               if (cb != 0.f) v = fmaf(cb, z_select(z_normals4(seed, layer, q, (uint64_t)(e >> 2)), (int)(e & 3)), v);
             }
             split16(v, hi, lo);
@@ -213,6 +227,15 @@ int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct,
                     void* B_aug, void* B_aug2, float* Zt, float* Zt2, const uint64_t* zq, int nzq) {
   AugBlocks blk{};
   for (int b = 0; b < a.nb; ++b) { blk.coef[b] = a.coef[b]; blk.qry[b] = a.qry[b]; }
+  blk.nseg = a.nseg > 1 ? a.nseg : 0;
+  for (int g = 0; g < blk.nseg; ++g) {
+    blk.seg_off[g] = a.seg_off[g];
+    blk.seg_C[g] = a.seg_C[g];
+    blk.seg_lid[g] = a.seg_lid[g];
+  }
+  blk.seg_off[blk.nseg] = a.d_out;
+  // the operand rows of a grouped launch come from the layers' own coefficients (Z tables: one layer only)
+  if (blk.nseg > 1 && (Zt || B_aug2)) return ZOACT_ERR_UNSUPPORTED;
   for (int i = 0; i < nzq; ++i) blk.zq[i] = zq[i];
   blk.nzq = Zt ? nzq : 0;
   const int full = mode == LOWRANK_ALL_ON_TC;
@@ -226,8 +249,9 @@ int launch_aug_prep(Ctx* ctx, const PairArgs& a, int mode, int ka, int distinct,
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
   // float4 source loads need 16-byte aligned rows: r a multiple of 4 and aligned bases (null: unused)
-  const bool quad = a.r % 4 == 0 && aligned16_or_null(a.P) && aligned16_or_null(distinct ? a.P2 : nullptr) &&
-                    aligned16_or_null(a.C) && aligned16_or_null(a.C2);
+  bool quad = a.r % 4 == 0 && aligned16_or_null(a.P) && aligned16_or_null(distinct ? a.P2 : nullptr) &&
+              aligned16_or_null(a.C) && aligned16_or_null(a.C2);
+  for (int g = 0; g < blk.nseg; ++g) quad = quad && aligned16_or_null(a.seg_C[g]);
   auto kern = quad ? aug_prep_kernel<true> : aug_prep_kernel<false>;
   ZOACT_CUDA_TRY(launch_pdl(ctx, kern, dim3((unsigned)grid), dim3(256), 0, a.P, distinct ? a.P2 : nullptr, a.C,
                             a.C2, static_cast<__nv_bfloat16*>(A_aug), static_cast<__nv_bfloat16*>(B_aug),

@@ -49,15 +49,14 @@ __device__ __forceinline__ float mix_at(const T* q, const T* k, const T* v, int 
 template <typename T>
 __global__ void __launch_bounds__(GLUE_THREADS)
 mix_rms_kernel(const T* __restrict__ Q, const T* __restrict__ K, const T* __restrict__ V, T* __restrict__ Y, int n,
-               int n_rep, int head_dim, float eps) {
+               int n_rep, int head_dim, float eps, int64_t ld_q, int64_t ld_kv) {
   pdl_wait();                              // the input rows written by the previous kernel
   pdl_trigger();
   __shared__ float red[GLUE_THREADS / 32];
   const int64_t row = blockIdx.x;
-  const int nk = n / n_rep;
-  const T* q = Q + row * n;
-  const T* k = K + row * nk;
-  const T* v = V + row * nk;
+  const T* q = Q + row * ld_q;
+  const T* k = K + row * ld_kv;
+  const T* v = V + row * ld_kv;
   float ss = 0.f;
   for (int i = threadIdx.x; i < n; i += GLUE_THREADS) {
     const float f = mix_at(q, k, v, i, n_rep, head_dim);
@@ -127,16 +126,15 @@ rms_norm_reg_kernel(const T* __restrict__ X, T* __restrict__ Y, int n, float eps
 template <typename T, int VPT>
 __global__ void __launch_bounds__(GLUE_THREADS)
 mix_rms_reg_kernel(const T* __restrict__ Q, const T* __restrict__ K, const T* __restrict__ V, T* __restrict__ Y,
-                   int n, int n_rep, int head_dim, float eps) {
+                   int n, int n_rep, int head_dim, float eps, int64_t ld_q, int64_t ld_kv) {
   pdl_wait();                              // the input rows written by the previous kernel
   pdl_trigger();
   constexpr int E = Vec<T>::N;
   __shared__ float red[GLUE_THREADS / 32];
   const int64_t row = blockIdx.x;
-  const int nk = n / n_rep;
-  const uint4* q = reinterpret_cast<const uint4*>(Q + row * n);
-  const T* k = K + row * nk;
-  const T* v = V + row * nk;
+  const uint4* q = reinterpret_cast<const uint4*>(Q + row * ld_q);
+  const T* k = K + row * ld_kv;
+  const T* v = V + row * ld_kv;
   const int nv = n / E;
   float m[VPT][E];
   float ss = 0.f;
@@ -204,12 +202,13 @@ int rms_dispatch(Ctx* ctx, const T* X, T* Y, int64_t rows, int n, float eps) {
 
 template <typename T>
 int mix_dispatch(Ctx* ctx, const T* q, const T* k, const T* v, T* Y, int64_t rows, int n, int n_rep, int head_dim,
-                 float eps) {
+                 float eps, int64_t ld_q, int64_t ld_kv) {
   constexpr int E = Vec<T>::N;
+  // 16-byte vectors need every row of q, k and v to start on a 16-byte boundary
   const bool ok = aligned16(q) && aligned16(k) && aligned16(v) && aligned16(Y) && head_dim % E == 0 &&
-                  (n / n_rep) % E == 0;
+                  (n / n_rep) % E == 0 && ld_q % E == 0 && ld_kv % E == 0;
   const int vpt = ok ? reg_vpt<T>(n) : 0;
-  void (*kern)(const T*, const T*, const T*, T*, int, int, int, float) = mix_rms_kernel<T>;
+  void (*kern)(const T*, const T*, const T*, T*, int, int, int, float, int64_t, int64_t) = mix_rms_kernel<T>;
   switch (vpt) {
     case 2: kern = mix_rms_reg_kernel<T, 2>; break;
     case 4: kern = mix_rms_reg_kernel<T, 4>; break;
@@ -218,7 +217,7 @@ int mix_dispatch(Ctx* ctx, const T* q, const T* k, const T* v, T* Y, int64_t row
     default: break;
   }
   ZOACT_CUDA_TRY(launch_pdl(ctx, kern, dim3((unsigned)rows), dim3(GLUE_THREADS), 0, q, k, v, Y, n, n_rep, head_dim,
-                            eps));
+                            eps, ld_q, ld_kv));
   ++ctx->n_launch;
   return ZOACT_OK;
 }
@@ -276,19 +275,21 @@ int launch_rms_norm(Ctx* ctx, const void* X, int dtype, int64_t rows, int n, flo
 }
 
 int launch_mix_rms(Ctx* ctx, const void* q, const void* k, const void* v, int dtype, int64_t rows, int n, int n_rep,
-                   int head_dim, float eps, void* Y) {
+                   int head_dim, float eps, void* Y, int64_t ld_q, int64_t ld_kv) {
   if (rows <= 0) return ZOACT_OK;
   switch (dtype) {
     case ZOACT_DT_FP32:
       return mix_dispatch(ctx, static_cast<const float*>(q), static_cast<const float*>(k),
-                          static_cast<const float*>(v), static_cast<float*>(Y), rows, n, n_rep, head_dim, eps);
+                          static_cast<const float*>(v), static_cast<float*>(Y), rows, n, n_rep, head_dim, eps, ld_q,
+                          ld_kv);
     case ZOACT_DT_BF16:
       return mix_dispatch(ctx, static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k),
                           static_cast<const __nv_bfloat16*>(v), static_cast<__nv_bfloat16*>(Y), rows, n, n_rep,
-                          head_dim, eps);
+                          head_dim, eps, ld_q, ld_kv);
     case ZOACT_DT_FP16:
       return mix_dispatch(ctx, static_cast<const __half*>(q), static_cast<const __half*>(k),
-                          static_cast<const __half*>(v), static_cast<__half*>(Y), rows, n, n_rep, head_dim, eps);
+                          static_cast<const __half*>(v), static_cast<__half*>(Y), rows, n, n_rep, head_dim, eps, ld_q,
+                          ld_kv);
     default:
       return ZOACT_ERR_INVALID_ARG;
   }

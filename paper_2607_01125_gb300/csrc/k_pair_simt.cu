@@ -113,6 +113,7 @@ pair_simt_kernel(const float* __restrict__ X, const float* __restrict__ W, const
 }  // namespace
 
 int launch_pair_simt(Ctx* ctx, const PairArgs& a) {
+  if (a.nseg > 1) return ZOACT_ERR_UNSUPPORTED;     // layers run as one: 16-bit activations only
   if (a.xdtype != ZOACT_DT_FP32 || a.wtype != ZOACT_DT_FP32 || a.ydtype != ZOACT_DT_FP32)
     return ZOACT_ERR_UNSUPPORTED;
   if (a.W2) return ZOACT_ERR_UNSUPPORTED;

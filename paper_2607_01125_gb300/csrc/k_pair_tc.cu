@@ -282,6 +282,9 @@ int launch_pair_tc(Ctx* ctx, const PairArgs& a) {
     }
   }
   if (big_r && lmode != LOWRANK_ALL_ON_TC) return ZOACT_ERR_UNSUPPORTED;
+  // layers run as one: the kernel must read the low-rank term only from the operand tables, which take each
+  // layer's coefficients and Philox stream (callers check pair_rowscale_supported before launching anything)
+  if (a.nseg > 1 && (gated || a.fuse_loss || lmode != LOWRANK_ALL_ON_TC)) return ZOACT_ERR_UNSUPPORTED;
   if (lmode == LOWRANK_ALL_ON_TC) rt = 4;   // whole term on the tensor cores: no epilogue tables
   // the fused loss needs CTA pairs whose 128-row halves each lie in one sign block, whole term on the MMA
   if (a.fuse_loss && !(two && !gated && lmode == LOWRANK_ALL_ON_TC && a.nb == 2 && !a.shared &&

@@ -76,6 +76,12 @@ class ZOStep:
         self.head_dim = head_dim
         self.linears = linears                      # list of AdaptedLinear, forward order
         self.by_name = {l.name: l for l in linears}
+        # stacks: each decoder's q, k and v read one input; their weights share one buffer so that, on stacked
+        # rows, one launch can run all three (zoact_pair_forward_group_rs)
+        self.groups = ([[f"{L}.q", f"{L}.k", f"{L}.v"] for L in range(len(linears) // (7 if kind == "llama" else 6))]
+                       if kind in ("llama", "opt") else [])
+        self._nogroup = set()
+        colocate_weights([[self.by_name[n] for n in g] for g in self.groups])
         dev = linears[0].W.device
         n = max(l.offset + l.d_out * l.r for l in linears)
         n = (n + 3) // 4 * 4
@@ -265,6 +271,59 @@ class ZOStep:
         self._wrote(H)
         return H
 
+    def _groupable(self, ls):
+        """Whether the library may run these linears as one launch: one basis, one weight type and width, and
+        weight (and INT4 scale) rows that follow one another in memory."""
+        l0 = ls[0]
+        if self.dtype not in (torch.bfloat16, torch.float16):
+            return False
+        if any(l.U.data_ptr() != l0.U.data_ptr() or l.d_in != l0.d_in or l.r != l0.r or l.wtype != l0.wtype
+               for l in ls):
+            return False
+        rows = 0
+        for l in ls:
+            if l.W.data_ptr() != l0.W.data_ptr() + rows * l0.W.stride(0) * l0.W.element_size():
+                return False
+            if l.w_scales is not None and (l0.w_scales is None or l.w_scales.data_ptr() != l0.w_scales.data_ptr() +
+                                           rows * l0.w_scales.stride(0) * l0.w_scales.element_size()):
+                return False
+            rows += l.d_out
+        return True
+
+    def pair_group(self, names, X, seed, query, out_key, in_scale=None):
+        """Linears that read X (stacked rows) as one pair forward (zoact_pair_forward_group_rs /
+        zoact_multi_forward_group_rs).  Returns their outputs, column views of one [rows, sum d_out] buffer, or
+        None where the library cannot run them as one launch (it then launched nothing; the caller runs them one
+        by one)."""
+        key = tuple(names)
+        ls = [self.by_name[n] for n in names]
+        if key in self._nogroup or not self._groupable(ls):
+            self._nogroup.add(key)
+            return None
+        P = self._proj(ls[0], X, 0)
+        dsum = sum(l.d_out for l in ls)
+        Y = self.buf(out_key, self.nb * self.T, dsum)
+        layers = [l.layer for l in ls]
+        if self.n_queries is None:
+            fn = lambda: Z.zoact_pair_forward_group_rs(self.ctx, layers, X, self.T, self.eps, seed, query, Y, P=P,
+                                                       in_scale=in_scale)
+        else:
+            fn = lambda: Z.zoact_multi_forward_group_rs(self.ctx, layers, X, self.T, self.points(query), seed, Y, P=P,
+                                                        in_scale=in_scale)
+        try:
+            self._counted(fn, 2.0 * X.shape[0] * ls[0].d_in * dsum)
+        except Z.ZoactError as e:
+            if e.status != Z.ZOACT_ERR_UNSUPPORTED:
+                raise
+            self._nogroup.add(key)
+            return None
+        self._wrote(Y)
+        outs, c = [], 0
+        for l in ls:
+            outs.append(Y[:, c:c + l.d_out])
+            c += l.d_out
+        return outs
+
     def _glue_rms(self, X, key):
         Y = self.buf(key, X.shape[0], X.shape[1])
         Z.zoact_rms_norm(self.ctx, X, Y)
@@ -318,9 +377,13 @@ class ZOStep:
                 k = self.pair(f"{L}.k", a, shared, seed, query, "k")
                 v = self.pair(f"{L}.v", a, shared, seed, query, "v")
             else:
-                q = self.pair(f"{L}.q", h, False, seed, query, "q", in_scale=inv_h)
-                k = self.pair(f"{L}.k", h, False, seed, query, "k", in_scale=inv_h)
-                v = self.pair(f"{L}.v", h, False, seed, query, "v", in_scale=inv_h)
+                qkv = self.pair_group([f"{L}.q", f"{L}.k", f"{L}.v"], h, seed, query, "qkv", in_scale=inv_h)
+                if qkv is not None:
+                    q, k, v = qkv
+                else:
+                    q = self.pair(f"{L}.q", h, False, seed, query, "q", in_scale=inv_h)
+                    k = self.pair(f"{L}.k", h, False, seed, query, "k", in_scale=inv_h)
+                    v = self.pair(f"{L}.v", h, False, seed, query, "v", in_scale=inv_h)
             shared = False
             mix = self.buf("mix", self.nb * T, q.shape[1])
             Z.zoact_mix_rms(self.ctx, q, k, v, mix, self.n_rep if self.kind == "llama" else 1, self.head_dim)
@@ -472,6 +535,29 @@ def coefficient_offsets(specs, r):
         offs.append(cur)
         cur += (s.d_out * r + 3) // 4 * 4
     return offs
+
+
+def colocate_weights(groups):
+    """Put the weights of each group of AdaptedLinears (linears that read one input, e.g. a decoder's q, k and
+    v) in one buffer, rows in group order, so that the library can run the group as one launch; INT4 scales
+    likewise.  Values are unchanged; a group already laid out so is left alone.  Call before binding."""
+    for ls in groups:
+        if len(ls) < 2:
+            continue
+        rows, ok = 0, True
+        for l in ls:
+            ok = ok and l.W.data_ptr() == ls[0].W.data_ptr() + rows * ls[0].W.stride(0) * ls[0].W.element_size()
+            rows += l.d_out
+        if ok:
+            continue
+        W = torch.cat([l.W for l in ls])
+        S = torch.cat([l.w_scales for l in ls]) if ls[0].w_scales is not None else None
+        c = 0
+        for l in ls:
+            l.W = W[c:c + l.d_out]
+            if S is not None:
+                l.w_scales = S[c:c + l.d_out]
+            c += l.d_out
 
 
 def calibrate_bases(ctx, step_cal, x_cal, r, oversample=16, n_iter=8, seed=0):

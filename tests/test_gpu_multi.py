@@ -234,13 +234,24 @@ def test_multi_update_nonfinite_guard(ctx):
 
 
 # ---------------- whole one-sided steps ----------------
+def _basis(w, s, bases):
+    """A random orthonormal basis per layer input: a decoder's q, k and v read one input and share one basis (as
+    Algorithm 1 gives them), so the stack's pair forwards may run them as one launch."""
+    name = s.name
+    if name.endswith(".k") or name.endswith(".v"):
+        name = name[:-2] + ".q"
+    if name not in bases:
+        bases[name] = random_orthonormal(s.d_in, w.r, tensor_seed(w, "U", name), DEV)
+    return bases[name]
+
+
 def _build(w, n_queries, c_std=0.05):
     dt = {"bf16": torch.bfloat16, "fp16": torch.float16, "fp32": torch.float32}[w.act_dtype]
     specs = w.linears()
     offs = coefficient_offsets(specs, w.r)
-    lins, ora = [], {}
+    lins, ora, bases = [], {}, {}
     for s, off in zip(specs, offs):
-        U = random_orthonormal(s.d_in, w.r, tensor_seed(w, "U", s.name), DEV)
+        U = _basis(w, s, bases)
         W = normal((s.d_out, s.d_in), tensor_seed(w, "W", s.name), DEV, std=w.weight_std, dtype=dt)
         lins.append(AdaptedLinear(s.name, W, U, s.layer_id, off, w.r))
     step = ZOStep(zo.Context(0), w.kind, lins, w.T, w.act_dtype, eps=w.eps, lr=w.lr, n_queries=n_queries)

@@ -40,6 +40,17 @@ def n64(t):
     return t.detach().cpu().double().numpy()
 
 
+def _basis(w, s, bases):
+    """A random orthonormal basis per layer input: a decoder's q, k and v read one input and share one basis (as
+    Algorithm 1 gives them), so the stack's pair forwards may run them as one launch."""
+    name = s.name
+    if name.endswith(".k") or name.endswith(".v"):
+        name = name[:-2] + ".q"
+    if name not in bases:
+        bases[name] = random_orthonormal(s.d_in, w.r, tensor_seed(w, "U", name), DEV)
+    return bases[name]
+
+
 def _build(w, c_std=0.01, align=None):
     """Weights and bases of workload w on the device, its ZOStep, and a function that gives the oracle's
     fp64 copy of one layer (W, U, C, layer_id) on demand, so that deep stacks never hold every layer's
@@ -51,9 +62,9 @@ def _build(w, c_std=0.01, align=None):
     dt = {"bf16": torch.bfloat16, "fp16": torch.float16, "fp32": torch.float32}[w.act_dtype]
     specs = w.linears()
     offs = coefficient_offsets(specs, w.r)
-    lins = []
+    lins, bases = [], {}
     for s, off in zip(specs, offs):
-        U = random_orthonormal(s.d_in, w.r, tensor_seed(w, "U", s.name), DEV)
+        U = _basis(w, s, bases)
         if w.wtype == "int4_g128":
             Wf = normal((s.d_out, s.d_in), tensor_seed(w, "W", s.name), DEV, std=w.weight_std)
             packed, scales = quantize_int4_g128(Wf)
