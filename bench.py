@@ -47,7 +47,7 @@ TIMING_PAIRS = 4096          # event pairs in the library's kernel-timing pool (
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one step's pair launches, from ncu captures of
 # the current kernels; workloads without such a capture report null.  The Llama stack's is scaled from a
 # 2-decoder capture (`--decoders 2`): decoder 0 plus 31 times decoder 1 (the later decoders have its shapes).
-PAIR_TRAFFIC_BYTES = {"llama_stack_bf16": 81.92e9, "llama_mlp_bf16": 933.9e6}
+PAIR_TRAFFIC_BYTES = {"llama_stack_bf16": 82.95e9, "llama_mlp_bf16": 933.9e6}
 
 
 # Dense fp16 tensor peak of the GB300s (TFLOP/s), measured like the bf16 peaks of MEASURED_PEAKS.json
