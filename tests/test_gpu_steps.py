@@ -175,10 +175,12 @@ def test_llama_mlp_step_full_width():
 
 @pytest.mark.parametrize("name,n_dec,T", [
     ("llama_stack_bf16", 2, 64), ("opt_stack_fp16", 2, 48), ("llama_stack_int4", 1, 64),   # one-CTA kernel
-    # 512 stacked rows: the CTA-pair kernel (whole low-rank term on the MMA, split last wave) in the graph
+    # 512 stacked rows: the CTA-pair kernel (whole low-rank term on the MMA, split last wave) in the graph, the
+    # second decoder's q, k and v as one launch
     ("llama_stack_bf16", 2, 256), ("opt_stack_fp16", 2, 256),
-    # 1024 stacked rows: INT4 weights expanded once per call, then the bf16 CTA-pair kernel
-    ("llama_stack_int4", 1, 512)])
+    # 1024 stacked rows: INT4 weights expanded once per call (the second decoder's q, k, v as one array), then the
+    # bf16 CTA-pair kernel
+    ("llama_stack_int4", 2, 512)])
 def test_stack_step(name, n_dec, T):
     seed, query = 23, 2
     w = workload(name, T=T, n_decoder=n_dec, eps=0.05)
