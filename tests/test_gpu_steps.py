@@ -51,7 +51,7 @@ def _basis(w, s, bases):
     return bases[name]
 
 
-def _build(w, c_std=0.01, align=None):
+def _build(w, c_std=0.01, align=None, n_queries=None):
     """Weights and bases of workload w on the device, its ZOStep, and a function that gives the oracle's
     fp64 copy of one layer (W, U, C, layer_id) on demand, so that deep stacks never hold every layer's
     fp64 weights at once.
@@ -74,7 +74,7 @@ def _build(w, c_std=0.01, align=None):
         else:
             W = normal((s.d_out, s.d_in), tensor_seed(w, "W", s.name), DEV, std=w.weight_std, dtype=dt)
             lins.append(AdaptedLinear(s.name, W, U, s.layer_id, off, w.r))
-    step = ZOStep(zo.Context(0), w.kind, lins, w.T, w.act_dtype, eps=w.eps, lr=w.lr)
+    step = ZOStep(zo.Context(0), w.kind, lins, w.T, w.act_dtype, eps=w.eps, lr=w.lr, n_queries=n_queries)
     C = normal(tuple(step.C.shape), tensor_seed(w, "C0"), "cpu", std=c_std).double().numpy()
     if align is not None:
         for l in lins:
@@ -99,15 +99,6 @@ def _build(w, c_std=0.01, align=None):
 
 def _stack_names(kind):
     return ["q", "k", "v", "o", "gate", "up", "down"] if kind == "llama" else ["q", "k", "v", "o", "fc1", "fc2"]
-
-
-def _oracle_stack(w, oracle_layer, x, seed, query):
-    """The oracle's stack, one decoder at a time (one decoder's fp64 weights in memory)."""
-    h = n64(x)
-    for L in range(w.n_decoder):
-        dl = {nm: oracle_layer(f"{L}.{nm}") for nm in _stack_names(w.kind)}
-        h = graphs.stack_forward([dl], h, w.eps, seed, query, w.kind, store=w.act_dtype, first=(L == 0))
-    return h
 
 
 def _check_step(step, oracle_layer, Y, out, Yo, tgt_o, w, seed, query):
@@ -182,15 +173,8 @@ def test_llama_mlp_step_full_width():
     # bf16 CTA-pair kernel
     ("llama_stack_int4", 2, 512)])
 def test_stack_step(name, n_dec, T):
-    seed, query = 23, 2
     w = workload(name, T=T, n_decoder=n_dec, eps=0.05)
-    step, ol = _build(w, align=(seed, query))
-    dt = torch.bfloat16 if w.act_dtype == "bf16" else torch.float16
-    x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=dt)
-    Y, out = _run_step(step, x, None, seed, query)
-    Yo = _oracle_stack(w, ol, x, seed, query)
-    _check_step(step, ol, Y, out, Yo, None, w, seed, query)
-    step.ctx.close()
+    _stack_step_per_decoder(w, 23, 2)
 
 
 def _check_outputs(Yg, Yo, what):
@@ -199,20 +183,16 @@ def _check_outputs(Yg, Yo, what):
     assert err_max <= 2e-2 and err_mean <= 1e-2, (what, err_max, err_mean)
 
 
-@pytest.mark.parametrize("name", ["llama_stack_bf16", "opt_stack_fp16", "llama_stack_int4"])
-def test_stack_step_full_depth(name):
-    # Every decoder of the configuration (32 or 40) at full width on 16 tokens per perturbation: layer ids, the
-    # shared-input rule of the first decoder and the buffer rotation over the whole chain.
-    # The synthetic stack is chaotic: a relative difference of 1e-3 in a decoder's input grows about 1.45x per
-    # decoder (measured on the oracle alone, with C = 0 as with C = 0.3 Z), so two correct implementations
-    # that round a stored activation differently decorrelate after ~20 decoders and their final outputs are
-    # not comparable element by element.  Each decoder is therefore checked on identical inputs: the oracle
-    # is fed the GPU's stored input to that decoder, and its output is compared with the GPU's input to the
-    # next decoder (the step's output after the last).  L+-, D, a and Adam step 1 of all layers are then
-    # checked against the oracle's last decoder on the GPU's input to it.
-    seed, query = 29, 3
-    w = workload(name, T=16, eps=0.05)
-    assert w.n_decoder in (32, 40)
+def _stack_step_per_decoder(w, seed, query):
+    """One ZO step of stack w on the device, checked decoder by decoder.
+    The synthetic stack is chaotic: a relative difference of 1e-3 in a decoder's input grows about 1.45x per
+    decoder (measured on the oracle alone, with C = 0 as with C = 0.3 Z), so two correct implementations that
+    round a stored activation differently drift apart along the chain (two INT4 decoders at 1024 stacked rows:
+    0.74% and 0.77% mean error per decoder, 1.39% through both), and after ~20 decoders their final outputs are
+    not comparable element by element.  Each decoder is therefore checked on identical inputs: the oracle is fed
+    the GPU's stored input to that decoder, and its output is compared with the GPU's input to the next decoder
+    (the step's output after the last).  L+-, D, a and Adam step 1 of all layers are then checked against the
+    oracle's last decoder on the GPU's input to it."""
     step, ol = _build(w, align=(seed, query))
     dt = torch.bfloat16 if w.act_dtype == "bf16" else torch.float16
     x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=dt)
@@ -231,15 +211,27 @@ def test_stack_step_full_depth(name):
     step.ctx.close()
 
 
-@pytest.mark.parametrize("name", ["llama_stack_bf16", "opt_stack_fp16"])
-def test_stack_full_size_sampled(name):
-    # the bench's launches of a stack at full size (T = 4096, 8192 stacked rows: row-scaled normalisations, L2-sized
-    # M-groups, split tails, eps = 1e-3) on two decoders.  Every op of a decoder acts on each token row on its own,
-    # so the oracle runs each decoder on 24 sampled rows of the GPU's stored input to it (the same rows of both
-    # signs) and checks the same rows of the decoder's output
+@pytest.mark.parametrize("name", ["llama_stack_bf16", "opt_stack_fp16", "llama_stack_int4"])
+def test_stack_step_full_depth(name):
+    # Every decoder of the configuration (32 or 40) at full width on 16 tokens per perturbation: layer ids, the
+    # shared-input rule of the first decoder and the buffer rotation over the whole chain, each decoder checked
+    # on the GPU's stored input to it
+    w = workload(name, T=16, eps=0.05)
+    assert w.n_decoder in (32, 40)
+    _stack_step_per_decoder(w, 29, 3)
+
+
+@pytest.mark.parametrize("name,n_queries", [("llama_stack_bf16", None), ("opt_stack_fp16", None),
+                                            ("llama_stack_int4", None), ("llama_stack_bf16", 8)])
+def test_stack_full_size_sampled(name, n_queries):
+    # the bench's launches of a stack at full size (T = 4096: 8192 stacked rows for the two-sided pair, 9 x 4096
+    # for the one-sided estimator with q = 8; row-scaled normalisations, L2-sized M-groups, split tails, the second
+    # decoder's q, k and v as one launch, INT4 expanded per call, eps = 1e-3) on two decoders.  Every op of a
+    # decoder acts on each token row on its own, so the oracle runs each decoder on 24 sampled token rows of the
+    # GPU's stored input to it (the same rows of every evaluation block) and checks those rows of its output
     w = workload(name, n_decoder=2)
     assert w.T == 4096
-    step, ol = _build(w)
+    step, ol = _build(w, n_queries=n_queries)
     dt = torch.bfloat16 if w.act_dtype == "bf16" else torch.float16
     x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=dt)
     ins = []
@@ -248,14 +240,21 @@ def test_stack_full_size_sampled(name):
     Y = step.forward(x, seed, query)
     torch.cuda.synchronize()
     assert step.ctx.device_status() == 0
+    if n_queries is None:
+        blocks = None
+        nb = 2
+    else:
+        blocks = [(0.0, 0)] + [(w.eps, qq) for qq in step.query_ids(query)]
+        nb = len(blocks)
     tok = np.sort(np.random.default_rng(3).choice(w.T, 24, replace=False))
-    both = np.concatenate([tok, w.T + tok])
+    rows = np.concatenate([b * w.T + tok for b in range(nb)])
     outs = [ins[1], Y]
     for L in range(2):
         dl = {nm: ol(f"{L}.{nm}") for nm in _stack_names(w.kind)}
-        h_in = n64(ins[L])[tok if L == 0 else both]
-        Yo = graphs.stack_forward([dl], h_in, w.eps, seed, query, w.kind, store=w.act_dtype, first=(L == 0))
-        _check_outputs(n64(outs[L])[both], Yo, f"decoder {L}")
+        h_in = n64(ins[L])[tok if L == 0 else rows]
+        Yo = graphs.stack_forward([dl], h_in, w.eps, seed, query, w.kind, store=w.act_dtype, first=(L == 0),
+                                  blocks=blocks)
+        _check_outputs(n64(outs[L])[rows], Yo, f"decoder {L}")
     step.ctx.close()
 
 
