@@ -15,7 +15,8 @@ g = (1/q) sum_j a_j Z^(j).
 with no host synchronisation.  This module only allocates buffers and issues
 the calls; every arithmetic step runs in libzoact's kernels.  Layers that read
 the same input with the same basis (q/k/v, gate/up after a calibration pass)
-share one projection P = X U.
+share one projection P = X U; a stacked decoder's q, k and v, whose weights
+share one buffer, run as one pair forward (zoact_pair_forward_group_rs).
 
 Graph wiring (names follow synth.Workload):
   toy        h = GELU(l1 x) (shared input, GELU fused in the epilogue); y = l2 h
@@ -25,7 +26,8 @@ Graph wiring (names follow synth.Workload):
                o = O rms(q + rep(k) + rep(v));  b = rms(o)
                llama: h' = down rms(silu(gate b) * up b)
                opt:   h' = fc2 rms(relu(fc1 b))
-             the first layer's q, k, v see the same input for both signs.
+             the first layer's q, k, v see the same input for both signs;
+             after it, q, k, v are one launch and the mixer reads column views.
 
 Hooks: `capture(name, X)` is called with each linear's input (the + half)
 before its pair forward -- Algorithm 1's calibration pass uses it to take the
