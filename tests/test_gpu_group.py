@@ -176,6 +176,8 @@ def test_group_refusals_launch_nothing(ctx, monkeypatch):
     Y = torch.empty(2 * T, n, dtype=torch.bfloat16, device=DEV)
     n0 = ctx.launch_count()
     _expect(zo._lib.ZOACT_ERR_UNSUPPORTED, lambda: zo.zoact_pair_forward_group_rs(ctx, lay, X, T, 0.5, 1, 1, Y))
+    # no tokens: nothing to do, nothing launched
+    zo.zoact_pair_forward_group_rs(ctx, lay, X[:0], 0, 0.5, 1, 1, Y[:0])
     # the one-CTA kernel or the epilogue low-rank term: no operand tables
     T = 256
     X = normal((2 * T, d_in), 92, DEV, dtype=torch.bfloat16)
