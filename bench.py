@@ -45,9 +45,13 @@ TIMING_PAIRS = 4096          # event pairs in the library's kernel-timing pool (
 
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one step's pair launches, from ncu captures of
-# the current kernels; workloads without such a capture report null.  The Llama stack's is scaled from a
-# 2-decoder capture (`--decoders 2`): decoder 0 plus 31 times decoder 1 (the later decoders have its shapes).
-PAIR_TRAFFIC_BYTES = {"llama_stack_bf16": 82.95e9, "llama_mlp_bf16": 933.9e6}
+# the current kernels; workloads without such a capture report null.  The stacks' are scaled from 2-decoder
+# captures (`--decoders 2`): decoder 0 plus (decoders - 1) times decoder 1 (the later decoders have its shapes);
+# the INT4 stack's include the expansions of W timed with their pair launches.  A run with a kernel switch set
+# (other kernels than the captured ones) reports null.
+PAIR_TRAFFIC_BYTES = {"llama_stack_bf16": 82.95e9, "llama_mlp_bf16": 933.9e6, "opt_stack_fp16": 208.66e9,
+                      "llama_stack_int4": 91.08e9}
+KERNEL_SWITCHES = ("ZOACT_INT4", "ZOACT_PAIR_KERNEL", "ZOACT_LOWRANK", "ZOACT_GROUP_M", "ZOACT_SPLIT_TAIL")
 
 
 # Dense fp16 tensor peak of the GB300s (TFLOP/s), measured like the bf16 peaks of MEASURED_PEAKS.json
@@ -405,7 +409,8 @@ def run_ours(args):
                      "algorithmic_flops_per_step": gemm_flops / instr_steps,
                      "traffic": (PAIR_TRAFFIC_BYTES.get(w.name)
                                  if args.tokens is None and args.queries is None and args.rank is None
-                                 and args.decoders is None else None),
+                                 and args.decoders is None and not any(os.environ.get(k) for k in KERNEL_SWITCHES)
+                                 else None),
                      "traffic_unit": "bytes per step (all pair launches of the step)"},
         "e2e": {"value": world * T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": 8 * step.loss_out.numel()},
