@@ -115,6 +115,51 @@ def measure_peak(dtype, seconds=4.0):
                       "gpu": torch.cuda.get_device_name(), "torch": torch.__version__}))
 
 
+def measure_read():
+    """What one launch reading a given number of bytes reaches on this GPU.  zoact_loss_pair on the MLP block's
+    loss shape (y+, y- and t: 2 x 2048 x 4096 and 2048 x 4096 bf16, 50.3 MB) and on 2, 4 and 16 times as many
+    tokens, beside torch.sum over a bf16 buffer of the same bytes; best of 10 by CUDA events, each after writing
+    a 512 MB buffer (larger than L2).  An empty launch between the same events gives the events' own overhead
+    (host dispatch included)."""
+    import torch
+    import paper_2607_01125_gb300 as zo
+    ctx = zo.Context(torch.cuda.current_device())
+    n_col = 4096
+    base = 3 * 2048 * n_col                      # bf16 elements of the MLP block's loss pair
+    buf = torch.ones(16 * base, device="cuda", dtype=torch.bfloat16)
+    flush = torch.empty(512 << 20, device="cuda", dtype=torch.uint8)
+    tiny = torch.zeros(1, device="cuda")
+    loss_out = torch.zeros(4, device="cuda", dtype=torch.float64)
+    out = []
+
+    def best_us(fn):
+        best = float("inf")
+        for r in range(12):
+            flush.fill_(r)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(); fn(); e1.record()
+            torch.cuda.synchronize()
+            if r >= 2:
+                best = min(best, e0.elapsed_time(e1) * 1e3)
+        return best
+
+    for mult in (1, 2, 4, 16):
+        n = mult * base
+        T = mult * 2048
+        Y = buf[:2 * T * n_col].view(2 * T, n_col)
+        tgt = buf[2 * T * n_col:3 * T * n_col].view(T, n_col)
+        us_loss = best_us(lambda: zo.zoact_loss_pair(ctx, Y, T, 1e-3, loss_out, target=tgt))
+        us_sum = best_us(lambda: torch.sum(buf[:n]))
+        out.append({"mbytes": round(2 * n / 1e6, 1), "zoact_loss_pair_us": round(us_loss, 2),
+                    "zoact_loss_pair_tb_per_s": round(2 * n / us_loss / 1e6, 2), "torch_sum_us": round(us_sum, 2),
+                    "torch_sum_tb_per_s": round(2 * n / us_sum / 1e6, 2)})
+    print(json.dumps({"read": "one launch, L2 flushed, CUDA events", "sizes": out,
+                      "empty_launch_us": round(best_us(lambda: tiny.add_(0.0)), 2),
+                      "device_status": ctx.device_status(), "gpu": torch.cuda.get_device_name(),
+                      "torch": torch.__version__}))
+    ctx.close()
+
+
 class ClockSampler:
     """nvidia-smi clocks and throttle reasons sampled every 100 ms in a child process."""
 
@@ -610,11 +655,15 @@ def main():
     ap.add_argument("--ref-tokens", type=int, default=64, help="tokens per oracle step in the reference arm")
     ap.add_argument("--measure-peak", choices=["fp16", "bf16"], default=None,
                     help="only measure the dense tensor peak of this dtype (torch.matmul 8192^3) and exit")
+    ap.add_argument("--measure-read", action="store_true",
+                    help="only time one-launch reads of 50 MB to 805 MB (zoact_loss_pair, torch.sum) and exit")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.measure_peak:
         measure_peak(args.measure_peak)
+    elif args.measure_read:
+        measure_read()
     elif args.impl == "reference":
         run_reference(args)
     else:
