@@ -23,7 +23,8 @@ exactly --steps steps, max over ranks).  The frozen weights are larger than L2
 (129 MB), so every step reads them from HBM.  `--impl reference` times the CPU
 oracle (numpy fp64) on a bounded sample of the default workload instead.
 `--measure-peak fp16` measures the dense fp16 tensor peak the OPT-13B workload
-is graded against.
+is graded against; `--measure-read` times the loss launch (and torch.sum) on
+50 MB to 805 MB reads.
 """
 import argparse
 import json
