@@ -119,9 +119,10 @@ def measure_peak(dtype, seconds=4.0):
 def measure_read():
     """What one launch reading a given number of bytes reaches on this GPU.  zoact_loss_pair on the MLP block's
     loss shape (y+, y- and t: 2 x 2048 x 4096 and 2048 x 4096 bf16, 50.3 MB) and on 2, 4 and 16 times as many
-    tokens, beside torch.sum over a bf16 buffer of the same bytes; best of 10 by CUDA events, each after writing
-    a 512 MB buffer (larger than L2).  An empty launch between the same events gives the events' own overhead
-    (host dispatch included)."""
+    tokens, the projection (zoact_lowrank_proj_prepared, r = 16, split-K sum included) of an X of the same bytes,
+    and torch.sum over a bf16 buffer of the same bytes; best of 10 by CUDA events, each after writing a 512 MB
+    buffer (larger than L2).  An empty launch between the same events gives the events' own overhead (host
+    dispatch included)."""
     import torch
     import paper_2607_01125_gb300 as zo
     ctx = zo.Context(torch.cuda.current_device())
@@ -131,6 +132,11 @@ def measure_read():
     flush = torch.empty(512 << 20, device="cuda", dtype=torch.uint8)
     tiny = torch.zeros(1, device="cuda")
     loss_out = torch.zeros(4, device="cuda", dtype=torch.float64)
+    # the projection P = X U (r = 16, the prepared basis) over X of the same bytes: [6144 mult, 4096] bf16
+    U = torch.randn(n_col, 16, device="cuda") / n_col ** 0.5
+    utc = torch.empty(zo.zoact_basis_prepared_bytes(n_col, 16), dtype=torch.uint8, device="cuda")
+    zo.zoact_basis_prepare(ctx, U, zo.DT_BF16, utc)
+    P = torch.empty(16 * 6144, 16, device="cuda")
     out = []
 
     def best_us(fn):
@@ -150,9 +156,14 @@ def measure_read():
         Y = buf[:2 * T * n_col].view(2 * T, n_col)
         tgt = buf[2 * T * n_col:3 * T * n_col].view(T, n_col)
         us_loss = best_us(lambda: zo.zoact_loss_pair(ctx, Y, T, 1e-3, loss_out, target=tgt))
+        X = buf[:n].view(n // n_col, n_col)
+        Pm = P[:n // n_col]
+        us_proj = best_us(lambda: zo.zoact_lowrank_proj_prepared(ctx, X, utc, 16, Pm))
         us_sum = best_us(lambda: torch.sum(buf[:n]))
         out.append({"mbytes": round(2 * n / 1e6, 1), "zoact_loss_pair_us": round(us_loss, 2),
-                    "zoact_loss_pair_tb_per_s": round(2 * n / us_loss / 1e6, 2), "torch_sum_us": round(us_sum, 2),
+                    "zoact_loss_pair_tb_per_s": round(2 * n / us_loss / 1e6, 2),
+                    "zoact_lowrank_proj_us": round(us_proj, 2),
+                    "zoact_lowrank_proj_tb_per_s": round(2 * n / us_proj / 1e6, 2), "torch_sum_us": round(us_sum, 2),
                     "torch_sum_tb_per_s": round(2 * n / us_sum / 1e6, 2)})
     print(json.dumps({"read": "one launch, L2 flushed, CUDA events", "sizes": out,
                       "empty_launch_us": round(best_us(lambda: tiny.add_(0.0)), 2),
@@ -657,7 +668,7 @@ def main():
     ap.add_argument("--measure-peak", choices=["fp16", "bf16"], default=None,
                     help="only measure the dense tensor peak of this dtype (torch.matmul 8192^3) and exit")
     ap.add_argument("--measure-read", action="store_true",
-                    help="only time one-launch reads of 50 MB to 805 MB (zoact_loss_pair, torch.sum) and exit")
+                    help="only time reads of 50 MB to 805 MB (zoact_loss_pair, the projection, torch.sum) and exit")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
