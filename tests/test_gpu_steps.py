@@ -258,6 +258,31 @@ def test_stack_full_size_sampled(name, n_queries):
     step.ctx.close()
 
 
+def test_default_bench_step_every_decoder_sampled():
+    # the bench's default forward exactly as timed -- the Llama-3-8B stack, all 32 decoders, T = 4096 (8192
+    # stacked rows), eps = 1e-3, row scales, L2-sized M-groups, split tails, q/k/v as one launch -- with every
+    # decoder checked on 8 sampled token rows (both signs) of the GPU's stored input to it (every op of a decoder
+    # acts on each row on its own)
+    w = workload("llama_stack_bf16")
+    assert w.T == 4096 and w.n_decoder == 32
+    step, ol = _build(w)
+    x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=torch.bfloat16)
+    tok = np.sort(np.random.default_rng(5).choice(w.T, 8, replace=False))
+    rows = np.concatenate([tok, w.T + tok])
+    ins = []
+    step.on_decoder = lambda L, h: ins.append(n64(h[torch.from_numpy(tok if L == 0 else rows).to(DEV)]))
+    seed, query = 37, 6
+    Y = step.forward(x, seed, query)
+    torch.cuda.synchronize()
+    assert step.ctx.device_status() == 0 and len(ins) == w.n_decoder
+    outs = ins[1:] + [n64(Y[torch.from_numpy(rows).to(DEV)])]
+    for L in range(w.n_decoder):
+        dl = {nm: ol(f"{L}.{nm}") for nm in _stack_names(w.kind)}
+        Yo = graphs.stack_forward([dl], ins[L], w.eps, seed, query, w.kind, store=w.act_dtype, first=(L == 0))
+        _check_outputs(outs[L], Yo, f"decoder {L}")
+    step.ctx.close()
+
+
 def test_toy_two_steps():
     w = workload("toy_fp32")
     step, ol = _build(w, c_std=0.05)
