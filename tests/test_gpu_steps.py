@@ -258,15 +258,17 @@ def test_stack_full_size_sampled(name, n_queries):
     step.ctx.close()
 
 
-def test_default_bench_step_every_decoder_sampled():
-    # the bench's default forward exactly as timed -- the Llama-3-8B stack, all 32 decoders, T = 4096 (8192
-    # stacked rows), eps = 1e-3, row scales, L2-sized M-groups, split tails, q/k/v as one launch -- with every
-    # decoder checked on 8 sampled token rows (both signs) of the GPU's stored input to it (every op of a decoder
-    # acts on each row on its own)
-    w = workload("llama_stack_bf16")
-    assert w.T == 4096 and w.n_decoder == 32
+@pytest.mark.parametrize("name", ["llama_stack_bf16", "opt_stack_fp16", "llama_stack_int4"])
+def test_bench_step_every_decoder_sampled(name):
+    # the bench's forward of each stack exactly as timed -- all 32 (Llama, INT4) or 40 (OPT) decoders, T = 4096
+    # (8192 stacked rows), eps = 1e-3, row scales, L2-sized M-groups, split tails, q/k/v as one launch, INT4
+    # expanded per call -- with every decoder checked on 8 sampled token rows (both signs) of the GPU's stored
+    # input to it (every op of a decoder acts on each row on its own)
+    w = workload(name)
+    assert w.T == 4096 and w.n_decoder in (32, 40)
     step, ol = _build(w)
-    x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=torch.bfloat16)
+    dt = torch.bfloat16 if w.act_dtype == "bf16" else torch.float16
+    x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=dt)
     tok = np.sort(np.random.default_rng(5).choice(w.T, 8, replace=False))
     rows = np.concatenate([tok, w.T + tok])
     ins = []
