@@ -258,29 +258,37 @@ def test_stack_full_size_sampled(name, n_queries):
     step.ctx.close()
 
 
-@pytest.mark.parametrize("name", ["llama_stack_bf16", "opt_stack_fp16", "llama_stack_int4"])
-def test_bench_step_every_decoder_sampled(name):
+@pytest.mark.parametrize("name,n_queries", [("llama_stack_bf16", None), ("opt_stack_fp16", None),
+                                            ("llama_stack_int4", None), ("llama_stack_bf16", 8)])
+def test_bench_step_every_decoder_sampled(name, n_queries):
     # the bench's forward of each stack exactly as timed -- all 32 (Llama, INT4) or 40 (OPT) decoders, T = 4096
     # (8192 stacked rows), eps = 1e-3, row scales, L2-sized M-groups, split tails, q/k/v as one launch, INT4
     # expanded per call -- with every decoder checked on 8 sampled token rows (both signs) of the GPU's stored
-    # input to it (every op of a decoder acts on each row on its own)
+    # input to it (every op of a decoder acts on each row on its own); with n_queries the one-sided estimator's
+    # q + 1 evaluation blocks (9 x 4096 rows)
     w = workload(name)
     assert w.T == 4096 and w.n_decoder in (32, 40)
-    step, ol = _build(w)
+    step, ol = _build(w, n_queries=n_queries)
     dt = torch.bfloat16 if w.act_dtype == "bf16" else torch.float16
     x, _ = lowrank_activations(w.T, w.d_model, 64, 0.05, tensor_seed(w, "x"), DEV, dtype=dt)
     tok = np.sort(np.random.default_rng(5).choice(w.T, 8, replace=False))
-    rows = np.concatenate([tok, w.T + tok])
+    seed, query = 37, 6
+    if n_queries is None:
+        blocks, nb = None, 2
+    else:
+        blocks = [(0.0, 0)] + [(w.eps, qq) for qq in step.query_ids(query)]
+        nb = len(blocks)
+    rows = np.concatenate([b * w.T + tok for b in range(nb)])
     ins = []
     step.on_decoder = lambda L, h: ins.append(n64(h[torch.from_numpy(tok if L == 0 else rows).to(DEV)]))
-    seed, query = 37, 6
     Y = step.forward(x, seed, query)
     torch.cuda.synchronize()
     assert step.ctx.device_status() == 0 and len(ins) == w.n_decoder
     outs = ins[1:] + [n64(Y[torch.from_numpy(rows).to(DEV)])]
     for L in range(w.n_decoder):
         dl = {nm: ol(f"{L}.{nm}") for nm in _stack_names(w.kind)}
-        Yo = graphs.stack_forward([dl], ins[L], w.eps, seed, query, w.kind, store=w.act_dtype, first=(L == 0))
+        Yo = graphs.stack_forward([dl], ins[L], w.eps, seed, query, w.kind, store=w.act_dtype, first=(L == 0),
+                                  blocks=blocks)
         _check_outputs(outs[L], Yo, f"decoder {L}")
     step.ctx.close()
 
