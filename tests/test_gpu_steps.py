@@ -164,6 +164,32 @@ def test_llama_mlp_step_full_width():
     step.ctx.close()
 
 
+@pytest.mark.parametrize("n_queries", [None, 8])
+def test_bench_mlp_forward_sampled(n_queries):
+    # the bench's MLP-block forward exactly as timed (T = 2048, eps = 1e-3: gate/up on the shared input with the
+    # mirrored two-sign or nine-block epilogues, down on the stacked rows), checked on 16 sampled token rows of
+    # every evaluation block; every op acts on each row on its own
+    w = workload("llama_mlp_bf16")
+    assert w.T == 2048
+    step, ol = _build(w, n_queries=n_queries)
+    x, _ = lowrank_activations(w.T, 4096, 64, 0.05, tensor_seed(w, "x"), DEV)
+    seed, query = 41, 3
+    if n_queries is None:
+        blocks, nb = None, 2
+    else:
+        blocks = [(0.0, 0)] + [(w.eps, qq) for qq in step.query_ids(query)]
+        nb = len(blocks)
+    Y = step.forward(x, seed, query)
+    torch.cuda.synchronize()
+    assert step.ctx.device_status() == 0
+    tok = np.sort(np.random.default_rng(7).choice(w.T, 16, replace=False))
+    rows = np.concatenate([b * w.T + tok for b in range(nb)])
+    Yo = graphs.llama_mlp_forward([ol("gate"), ol("up"), ol("down")], n64(x)[tok], w.eps, seed, query, store="bf16",
+                                  blocks=blocks)
+    _check_outputs(n64(Y)[rows], Yo, "MLP block")
+    step.ctx.close()
+
+
 @pytest.mark.parametrize("name,n_dec,T", [
     ("llama_stack_bf16", 2, 64), ("opt_stack_fp16", 2, 48), ("llama_stack_int4", 1, 64),   # one-CTA kernel
     # 512 stacked rows: the CTA-pair kernel (whole low-rank term on the MMA, split last wave) in the graph, the
