@@ -284,15 +284,17 @@ def test_stack_full_size_sampled(name, n_queries):
     step.ctx.close()
 
 
-@pytest.mark.parametrize("name,n_queries", [("llama_stack_bf16", None), ("opt_stack_fp16", None),
-                                            ("llama_stack_int4", None), ("llama_stack_bf16", 8)])
-def test_bench_step_every_decoder_sampled(name, n_queries):
+@pytest.mark.parametrize("name,n_queries,r", [("llama_stack_bf16", None, None), ("opt_stack_fp16", None, None),
+                                              ("llama_stack_int4", None, None), ("llama_stack_bf16", 8, None),
+                                              ("llama_stack_int4", None, 32), ("llama_stack_bf16", None, 256)])
+def test_bench_step_every_decoder_sampled(name, n_queries, r):
     # the bench's forward of each stack exactly as timed -- all 32 (Llama, INT4) or 40 (OPT) decoders, T = 4096
     # (8192 stacked rows), eps = 1e-3, row scales, L2-sized M-groups, split tails, q/k/v as one launch, INT4
     # expanded per call -- with every decoder checked on 8 sampled token rows (both signs) of the GPU's stored
     # input to it (every op of a decoder acts on each row on its own); with n_queries the one-sided estimator's
-    # q + 1 evaluation blocks (9 x 4096 rows)
-    w = workload(name)
+    # q + 1 evaluation blocks (9 x 4096 rows); with r the rank ablation's bench lines (INT4 at the paper's r = 32,
+    # the stack at r = 256)
+    w = workload(name) if r is None else workload(name, r=r)
     assert w.T == 4096 and w.n_decoder in (32, 40)
     step, ol = _build(w, n_queries=n_queries)
     dt = torch.bfloat16 if w.act_dtype == "bf16" else torch.float16
